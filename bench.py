@@ -1,0 +1,377 @@
+"""Benchmark of the masked second-order HLA hot path on GB300.
+
+One step = one hla2_forward over the long-context workload (B=2, H=16,
+n=16384, d=dv=128, chunk 128, bf16 tokens, masked, ratio-normalised; inputs
+resident in HBM).  The decode-step workload (B=64, H=32, d=dv=128, fp32 state,
+bf16 tokens, state built from a 4096-token prefix) is measured in the same run
+and reported under "decode".  Prints ONE JSON line (rank 0).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Multi-GPU (torchrun): every rank runs its own copy of the workload (heads are
+independent; no collective on the data path), the timed region is bracketed by
+barriers, and the max time over ranks is used: weak scaling.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import hla_inputs  # noqa: E402
+
+METRIC = "masked HLA-2 forward tokens/s at 1 GB300 and % of roofline; decode-step GB/s"
+FWD = hla_inputs.WORKLOADS["long_bf16_norm"]
+DEC = hla_inputs.WORKLOADS["decode_bf16"]
+
+
+def peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), float(p["bf16_tflops"]), "measured"
+    except Exception:
+        return 6800.0, 1900.0, "fallback"
+
+
+def fwd_bytes(w):
+    """Algorithmic bytes of one forward: read q, k, v once, write out once."""
+    s = 2 if w.dtype == "bf16" else 4
+    return w.BH * w.n * ((2 * w.d + w.dv) * s + w.dv * s)
+
+
+def fwd_flops(w):
+    """Algorithmic FLOPs of one forward (masks and the symmetry of S exploited):
+    per token-head 2C(d+dv) + C^2/3 + 3d^2 + 6 d dv + 2 d^2 dv / C."""
+    C, d, dv = w.chunk, w.d, w.dv
+    per = 2 * C * (d + dv) + C * C / 3 + 3 * d * d + 6 * d * dv + 2 * d * d * dv / C
+    return w.BH * w.n * per
+
+
+def dec_bytes(w):
+    """Algorithmic bytes of one decode step: read + write of the fp32 state tuple
+    (S, C, m, G, h) of every head plus the token I/O."""
+    st = w.d * w.d + 2 * w.d * w.dv + 2 * w.d
+    s = 2 if w.dtype == "bf16" else 4
+    return w.BH * (2 * st * 4 + (2 * w.d + w.dv) * s + w.dv * s)
+
+
+class ClockSampler:
+    """nvidia-smi clock/throttle samples (every 100 ms) around a timed region."""
+
+    FIELDS = ("index,timestamp,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.fh = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.gpu), "--query-gpu=" + self.FIELDS,
+                                          "--format=csv,noheader,nounits", "-lms", "100"], stdout=self.fh,
+                                         stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.25)
+        self.proc.terminate()
+        self.proc.wait()
+        self.fh.close()
+        rows = [r.split(",") for r in open(self.path).read().strip().splitlines() if r.count(",") >= 9]
+        os.unlink(self.path)
+        sm = [float(r[2]) for r in rows if r[2].strip().replace(".", "").isdigit()]
+        smax = [float(r[3]) for r in rows if r[3].strip().replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if "Active" in r[6 + i] and "Not" not in r[6 + i]})
+        loaded = [x for x in sm if x > 0.5 * max(sm)] if sm else []
+        return {"sm_mhz": statistics.median(loaded) if loaded else None, "sm_max_mhz": max(smax) if smax else None,
+                "reasons": reasons, "samples": len(rows)}
+
+
+def dist_setup(gpus):
+    import torch
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    return rank, world, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(x, world):
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def cpu_baseline(budget_s=15.0):
+    """The fp64 oracle, as it stands, on a bounded sample of the forward workload:
+    the first `heads` heads of the same inputs, all n positions, all host cores."""
+    import oracle
+    cores = os.cpu_count() or 1
+    heads = max(1, min(FWD.BH, cores))
+    q, k, v = hla_inputs.make_workload(FWD)
+    qf, kf, vf = (x.reshape(FWD.BH, FWD.n, -1)[:heads] for x in (q, k, v))
+    # size the sample from a short probe so the run stays near the budget
+    t0 = time.time()
+    oracle.hla2_serial(qf[:, :512], kf[:, :512], vf[:, :512], masked=True, normalized=True, eps=hla_inputs.EPS,
+                       nthreads=cores)
+    probe = time.time() - t0
+    n = int(min(FWD.n, max(512, 512 * budget_s / max(probe, 1e-6))))
+    t0 = time.time()
+    oracle.hla2_serial(qf[:, :n], kf[:, :n], vf[:, :n], masked=True, normalized=True, eps=hla_inputs.EPS,
+                       nthreads=cores)
+    dt = time.time() - t0
+    token_heads = heads * n
+    return {"value": token_heads / FWD.H / dt, "unit": "tokens/s", "cores": min(cores, heads), "kind": "oracle",
+            "sample": "fp64 serial oracle on %d of %d heads x first %d of %d positions of the forward workload "
+                      "(tokens/s = token-heads/s / H), %.1f s" % (heads, FWD.BH, n, FWD.n, dt)}
+
+
+def run_reference(args):
+    """--impl reference: the oracle on the host cores, one bounded sample per step."""
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    import oracle
+    cores = os.cpu_count() or 1
+    heads = max(1, min(FWD.BH, cores))
+    q, k, v = hla_inputs.make_workload(FWD)
+    n = 1024
+    qf, kf, vf = (np.ascontiguousarray(x.reshape(FWD.BH, FWD.n, -1)[:heads, :n]) for x in (q, k, v))
+    for _ in range(args.warmup):
+        oracle.hla2_serial(qf, kf, vf, masked=True, normalized=True, eps=hla_inputs.EPS, nthreads=cores)
+    t0 = time.time()
+    for _ in range(args.steps):
+        oracle.hla2_serial(qf, kf, vf, masked=True, normalized=True, eps=hla_inputs.EPS, nthreads=cores)
+    dt = (time.time() - t0) / args.steps
+    value = heads * n / FWD.H / dt
+    sample = "fp64 serial oracle on %d of %d heads x first %d positions per step" % (heads, FWD.BH, n)
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1e3, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": "long_bf16_norm (sampled)", "B": FWD.B, "H": FWD.H, "n": FWD.n, "d": FWD.d,
+                   "dv": FWD.dv, "chunk": FWD.chunk},
+        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": min(cores, heads), "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }))
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=0, help="timed forward steps (0 = about 2 s worth)")
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--decode-steps", type=int, default=DEC.decode_steps)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-decode", action="store_true")
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3)
+    if args.impl == "reference":
+        if args.steps <= 0:
+            args.steps = 3
+        return run_reference(args)
+
+    import torch
+
+    from paper_2510_27258_gb300 import build
+    build.build()
+    from paper_2510_27258_gb300 import hla
+
+    rank, world, local = dist_setup(args.gpus)
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    hbm_peak, tc_peak, peak_kind = peaks()
+
+    # ---------------- forward workload ----------------
+    w = FWD
+    q, k, v = hla_inputs.make_workload(w)
+    tq, tk, tv = (hla_inputs.as_torch(x, w.dtype, dev) for x in (q, k, v))
+    out = torch.empty((w.B, w.H, w.n, w.dv), dtype=tq.dtype, device=dev)
+    ws = hla.alloc_workspace(hla.hla2_workspace_bytes(w.B, w.H, w.n, w.d, w.dv, w.chunk, tq.dtype), dev)
+    stream = torch.cuda.current_stream()
+
+    def step():
+        hla.hla2_forward(tq, tk, tv, out, masked=w.masked, normalized=w.normalized, eps=hla_inputs.EPS,
+                         chunk=w.chunk, workspace=ws, stream=stream)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    if hla.hla_poll_error(ws) != 0:
+        raise RuntimeError("device-side error flag set during warm-up")
+    if args.steps <= 0:
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        step()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        args.steps = int(max(10, min(20000, 2000.0 / max(e0.elapsed_time(e1), 1e-3))))
+
+    sampler = ClockSampler(local)
+    sampler.start()
+    barrier(world)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    barrier(world)
+    clocks = sampler.stop()
+    ms = max_over_ranks(e0.elapsed_time(e1) / args.steps, world)
+    if hla.hla_poll_error(ws) != 0:
+        raise RuntimeError("device-side error flag set during the timed region")
+
+    tokens = w.B * w.n  # sequence positions per forward (every head processed)
+    value = tokens * world / (ms * 1e-3)
+    achieved_gbs = fwd_bytes(w) / (ms * 1e-3) / 1e9
+    achieved_tf = fwd_flops(w) / (ms * 1e-3) / 1e12
+
+    # ---------------- end to end: pinned host buffers, copies inside the timed region ----------
+    hq, hk, hv = (t.cpu().pin_memory() for t in (tq, tk, tv))
+    hout = torch.empty(out.shape, dtype=out.dtype).pin_memory()
+    dq, dk, dvv = (torch.empty_like(t) for t in (tq, tk, tv))
+
+    def e2e_step():
+        dq.copy_(hq, non_blocking=True)
+        dk.copy_(hk, non_blocking=True)
+        dvv.copy_(hv, non_blocking=True)
+        hla.hla2_forward(dq, dk, dvv, out, masked=w.masked, normalized=w.normalized, eps=hla_inputs.EPS,
+                         chunk=w.chunk, workspace=ws, stream=stream)
+        hout.copy_(out, non_blocking=True)
+
+    for _ in range(2):
+        e2e_step()
+    torch.cuda.synchronize()
+    e2e_steps = max(3, min(args.steps, 50))
+    barrier(world)
+    e0.record(stream)
+    for _ in range(e2e_steps):
+        e2e_step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = max_over_ranks(e0.elapsed_time(e1) / e2e_steps, world)
+    in_bytes = sum(t.numel() * t.element_size() for t in (hq, hk, hv))
+    out_bytes = hout.numel() * hout.element_size()
+    del hq, hk, hv, hout, dq, dk, dvv
+
+    result = {
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": hla_path_dtype(), "data": "synthetic",
+        "config": {"workload": "long_bf16_norm", "B": w.B, "H": w.H, "n": w.n, "d": w.d, "dv": w.dv,
+                   "chunk": w.chunk, "masked": w.masked, "normalized": w.normalized, "tokens": "bf16",
+                   "global_batch": w.B * world, "seq_len": w.n, "parallelism": "replicas (heads independent)",
+                   "l2": "inputs larger than L2: %.0f MB read + %.0f MB written per step" % (
+                       3 * w.BH * w.n * w.d * 2 / 1e6, w.BH * w.n * w.dv * 2 / 1e6)},
+        "clocks": clocks,
+        "roofline": {"bound": "hbm", "achieved": achieved_gbs, "peak": hbm_peak, "unit": "GB/s",
+                     "frac": achieved_gbs / hbm_peak, "traffic": None, "peak_kind": peak_kind,
+                     "kernel": "whole hla2_forward call", "tensor_view": {
+                         "achieved_tflops": achieved_tf, "peak_tflops": tc_peak,
+                         "frac": achieved_tf / tc_peak}},
+        "e2e": {"value": tokens * world / (e2e_ms * 1e-3), "unit": "tokens/s", "ms_per_step": e2e_ms,
+                "h2d_bytes_per_step": in_bytes, "d2h_bytes_per_step": out_bytes},
+        "gpu_launches": hla_launches_per_forward() * args.steps,
+    }
+    del tq, tk, tv, out, ws
+    torch.cuda.empty_cache()
+
+    # ---------------- decode step workload ----------------
+    if not args.no_decode:
+        result["decode"] = bench_decode(hla, dev, stream, args.decode_steps, hbm_peak, world)
+        result["gpu_launches"] += result["decode"]["launches"]
+
+    if rank == 0 and not args.no_cpu_baseline:
+        result["cpu_baseline"] = cpu_baseline()
+    if rank == 0:
+        print(json.dumps(result))
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+def hla_path_dtype():
+    """Arithmetic type of the path that serves the forward workload."""
+    return os.environ.get("HLA_BENCH_DTYPE_LABEL", "f32")
+
+
+def hla_launches_per_forward():
+    """Kernels one hla2_forward launches for the forward workload."""
+    return 3
+
+
+def bench_decode(hla, dev, stream, steps, hbm_peak, world):
+    import torch
+    w = DEC
+    (qp, kp, vp), (qs, ks, vs) = hla_inputs.make_decode(w, steps=steps)
+    st = torch.zeros((w.B, w.H, hla.hla2_state_floats(w.d, w.dv)), dtype=torch.float32, device=dev)
+    tq, tk, tv = (hla_inputs.as_torch(x, w.dtype, dev) for x in (qp, kp, vp))
+    hla.hla2_forward(tq, tk, tv, masked=w.masked, normalized=w.normalized, eps=hla_inputs.EPS, chunk=w.chunk,
+                     state_out=st)
+    del tq, tk, tv
+    toks = [[hla_inputs.as_torch(x[s], w.dtype, dev) for x in (qs, ks, vs)] for s in range(steps)]
+    out = torch.empty((w.B, w.H, w.dv), dtype=toks[0][0].dtype, device=dev)
+    st0 = st.clone()
+    for s in range(min(3, steps)):  # warm-up on a copy, then restore
+        hla.hla2_step(*toks[s], st, out, masked=w.masked, normalized=w.normalized, eps=hla_inputs.EPS)
+    st.copy_(st0)
+    del st0
+    torch.cuda.synchronize()
+    barrier(world)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for s in range(steps):
+        hla.hla2_step(*toks[s], st, out, masked=w.masked, normalized=w.normalized, eps=hla_inputs.EPS,
+                      stream=stream)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    us = max_over_ranks(e0.elapsed_time(e1) * 1e3 / steps, world)
+    gbs = dec_bytes(w) / (us * 1e-6) / 1e9
+    return {"workload": "decode_bf16", "B": w.B, "H": w.H, "d": w.d, "dv": w.dv, "prefix": w.decode_prefix,
+            "steps": steps, "us_per_step": us, "value": gbs * world, "unit": "GB/s",
+            "tokens_per_s": w.B * world / (us * 1e-6),
+            "roofline": {"bound": "hbm", "achieved": gbs, "peak": hbm_peak, "unit": "GB/s", "frac": gbs / hbm_peak,
+                         "traffic": None, "kernel": "step2_kernel"},
+            "launches": steps}
+
+
+if __name__ == "__main__":
+    main()

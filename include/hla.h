@@ -1,0 +1,159 @@
+/*
+ * hla.h -- C ABI of the GB300 (sm_103a) implementation of Higher-order Linear
+ * Attention (Zhang, Qin, Wang, Gu, "Higher-order Linear Attention").
+ *
+ * All entry points take plain pointers and sizes.  Device pointers refer to
+ * memory of the current CUDA device; the caller owns every buffer (inputs,
+ * outputs, states and the scratch workspace) and the library allocates no
+ * device memory.  Work is enqueued asynchronously on `stream`; host-side
+ * argument errors are returned synchronously before anything is launched.
+ *
+ * Common conventions
+ * ------------------
+ * Tokens are row vectors.  q, k are [B, H, n, d] and v, out are [B, H, n, dv],
+ * contiguous, in the element type `dt` (out has the same type as the inputs).
+ * Base pointers must be 16-byte aligned.
+ *
+ * Second-order state of one head (fp32, row-major), the tuple of Fig. 1(A):
+ *   [ S (d*d) | C (d*dv) | m (d) | G (d*dv) | h (d) ]
+ * with S = sum k k^T, C = sum q v^T, m = sum q, G = sum_i k_i k_i^T C_{i-1},
+ * h = sum_i k_i k_i^T m_{i-1} (Sec. 3 and Sec. 3.2).  States of B*H heads are
+ * stored back to back in [B, H] order.  With masked = 0 the operator does not
+ * use G and h: they are ignored on input and written as zeros on output.
+ *
+ * Supported shapes: d, dv in {16, 32, 64, 128}; 1 <= chunk <= 128 (chunk is
+ * the scan granularity of Theorem 2; the result does not depend on it up to
+ * rounding); n >= 0 with any remainder n % chunk (a ragged last chunk).
+ * Other values return HLA_ERR_UNSUPPORTED.
+ */
+#ifndef HLA_H_
+#define HLA_H_
+
+#include <stddef.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+struct CUstream_st;
+/* A CUDA stream (the same object as cudaStream_t); NULL is the legacy default stream. */
+typedef struct CUstream_st *hla_stream_t;
+
+typedef enum {
+    HLA_OK = 0,
+    HLA_ERR_INVALID_ARGUMENT = 1, /* null pointer, negative size, misaligned pointer, bad flag */
+    HLA_ERR_UNSUPPORTED = 2,      /* valid request outside the supported shapes/types        */
+    HLA_ERR_CUDA = 3,             /* a CUDA runtime call or kernel launch failed              */
+    HLA_ERR_TIMEOUT = 4,          /* a device-side wait ran past its budget (hla_poll_error)  */
+    HLA_ERR_WORKSPACE = 5         /* workspace missing or smaller than the required size      */
+} hla_status;
+
+typedef enum {
+    HLA_F32 = 0,  /* IEEE float32 tokens */
+    HLA_BF16 = 1  /* bfloat16 tokens (fp32 accumulation everywhere) */
+} hla_dtype;
+
+/* Human-readable name of a status code (static storage). */
+const char *hla_status_string(hla_status status);
+
+/* Detail of the last error returned on the calling host thread (static,
+ * thread-local storage; empty string if none). */
+const char *hla_last_error(void);
+
+/* Number of floats of one head's second-order state tuple: d*d + 2*d*dv + 2*d. */
+size_t hla2_state_floats(int d, int dv);
+
+/* Bytes of scratch workspace hla2_forward needs for these sizes (any flags).
+ * Returns 0 for unsupported sizes. */
+size_t hla2_workspace_bytes(int B, int H, int n, int d, int dv, int chunk, hla_dtype dt);
+
+/*
+ * hla2_forward -- chunk-parallel forward of second-order HLA over n tokens.
+ *
+ * Operator (per head, t = 1..n):
+ *   masked = 1 (strictly causal, Theorem 1, Eq. masked-unnorm / Eq. masked):
+ *     num_t = q_t^T (S_t C_t - G_t),   den_t = q_t^T (S_t m_t - h_t)
+ *     = sum_{j<=t} sum_{i<=j} (q_t.k_i)(q_j.k_i) v_j   (and v_j -> 1 for den)
+ *   masked = 0 (Eq. hla-unnorm / Eq. hla-row):
+ *     num_t = q_t^T S_t C_t,           den_t = q_t^T S_t m_t
+ *   out_t = num_t                       if normalized == 0 (the default operator)
+ *   out_t = num_t / (den_t + eps)       if normalized == 1 (no clamp, no abs)
+ * where the states include token t (inclusive) and start from state_in.  The
+ * result equals the serial recurrence (online updates after Theorem 1) by
+ * Theorem 2; chunking only changes rounding.
+ *
+ * q, k, v : device, [B, H, n, d] / [B, H, n, d] / [B, H, n, dv] of type dt (read only)
+ * out     : device, [B, H, n, dv] of type dt (written)
+ * state_in  : device fp32 [B*H * hla2_state_floats(d,dv)] or NULL (= zero state)
+ * state_out : device fp32, same size, or NULL (= not written); receives the
+ *             state after token n (Eq. semidirect applied to the whole
+ *             sequence).  May equal state_in (read before written).
+ * eps     : the stability constant of the normalised output (finite)
+ * workspace / workspace_bytes : device scratch of at least
+ *             hla2_workspace_bytes(B,H,n,d,dv,chunk,dt) bytes, 256-byte
+ *             aligned; its contents on entry are ignored.  Calls that share a
+ *             workspace must be ordered on one stream.
+ * Errors: HLA_ERR_INVALID_ARGUMENT / UNSUPPORTED / WORKSPACE before launch;
+ * HLA_ERR_CUDA if a launch fails.  A device-side wait that exceeds its budget
+ * sets a flag in the workspace that hla_poll_error reports as HLA_ERR_TIMEOUT.
+ */
+hla_status hla2_forward(const void *q, const void *k, const void *v, void *out, hla_dtype dt,
+                        int B, int H, int n, int d, int dv, int masked, int normalized, float eps,
+                        int chunk, const float *state_in, float *state_out,
+                        void *workspace, size_t workspace_bytes, hla_stream_t stream);
+
+/*
+ * hla2_step -- one streaming decode step of second-order HLA for B*H heads.
+ *
+ * For each head, with the state tuple (S, C, m, G, h) before the token
+ * (online updates after Theorem 1; outputs of Theorem 1 / Eq. hla-row):
+ *   masked:  G += k (k^T C),  h += k (k^T m)          (previous C and m)
+ *   S += k k^T,  C += q v^T,  m += q
+ *   masked:   num = (q^T S) C - q^T G,  den = (q^T S) m - q^T h
+ *   unmasked: num = (q^T S) C,          den = (q^T S) m   (G, h untouched)
+ *   out = num, or num / (den + eps) if normalized.
+ *
+ * q, k : device [B, H, d] of type dt; v : device [B, H, dv] of type dt
+ * out  : device [B, H, dv] of type dt
+ * state: device fp32 [B*H * hla2_state_floats(d,dv)], updated in place
+ * Errors as for hla2_forward (no workspace, no device-side waits).
+ */
+hla_status hla2_step(const void *q, const void *k, const void *v, void *out, hla_dtype dt,
+                     int B, int H, int d, int dv, int masked, int normalized, float eps,
+                     float *state, hla_stream_t stream);
+
+/* Number of floats of one head's third-order state tuple (Theorem 3):
+ * [ SK d*d | SQ d*d | P d*dv | mK d | G1 d*dv | G2 d*dv | G3 d*dv | h1 d | h2 d | h3 d ]. */
+size_t hla3_state_floats(int d, int dv);
+
+/* Bytes of scratch workspace hla3_forward needs (0 if unsupported). */
+size_t hla3_workspace_bytes(int B, int H, int n, int d, int dv, int chunk, hla_dtype dt);
+
+/*
+ * hla3_forward -- forward of third-order HLA (Sec. 7).
+ *
+ *   masked = 1 (Theorem 3, Algorithm 3 at gamma = 1):
+ *     num_t = q_t^T (S^K_t S^Q_t P^KV_t - G1_t - G2_t - G3_t)
+ *     den_t = q_t^T (S^K_t S^Q_t m^K_t  - h1_t - h2_t - h3_t)
+ *   masked = 0: num_t = q_t^T S^K_t S^Q_t P^KV_t, den_t = q_t^T S^K_t S^Q_t m^K_t
+ *   out_t = num_t, or num_t / (den_t + eps) if normalized.
+ * Arguments as for hla2_forward, with the third-order state layout.
+ */
+hla_status hla3_forward(const void *q, const void *k, const void *v, void *out, hla_dtype dt,
+                        int B, int H, int n, int d, int dv, int masked, int normalized, float eps,
+                        int chunk, const float *state_in, float *state_out,
+                        void *workspace, size_t workspace_bytes, hla_stream_t stream);
+
+/*
+ * hla_poll_error -- wait for `stream`, then report the device-side error flag
+ * kept in `workspace` by the last forward call that used it: HLA_OK, or
+ * HLA_ERR_TIMEOUT if a device-side wait gave up.  Clears the flag.
+ * Returns HLA_ERR_CUDA if synchronisation or the read fails.
+ */
+hla_status hla_poll_error(void *workspace, hla_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* HLA_H_ */

@@ -1,0 +1,75 @@
+// Internal declarations of the HLA CUDA library (not part of the public ABI).
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "hla.h"
+
+namespace hla {
+
+// ---------------------------------------------------------------------------
+// Workspace: the first kWsHeaderBytes bytes of every workspace hold the
+// device-side error word (read by hla_poll_error); scratch follows.
+// ---------------------------------------------------------------------------
+constexpr size_t kWsHeaderBytes = 256;
+
+struct WsHeader {
+    unsigned int error;   // 0 = ok, otherwise a DevError code
+    unsigned int where;   // kernel-specific location of the failure
+    unsigned int detail;  // kernel-specific detail (e.g. a chunk index)
+};
+
+enum DevError : unsigned int { kDevOk = 0, kDevTimeout = 1 };
+
+inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// Records a host-side error message for hla_last_error() and returns `st`.
+hla_status fail(hla_status st, const char *fmt, ...);
+// Maps a CUDA error to HLA_ERR_CUDA (recording the CUDA message), or HLA_OK.
+hla_status cuda_status(cudaError_t err, const char *what);
+
+// ---------------------------------------------------------------------------
+// token element access
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ float to_f32(float x) { return x; }
+__device__ __forceinline__ float to_f32(__nv_bfloat16 x) { return __bfloat162float(x); }
+__device__ __forceinline__ void from_f32(float *p, float x) { *p = x; }
+__device__ __forceinline__ void from_f32(__nv_bfloat16 *p, float x) { *p = __float2bfloat16_rn(x); }
+
+// ---------------------------------------------------------------------------
+// forward problem description shared by the forward paths
+// ---------------------------------------------------------------------------
+struct Fwd2 {
+    const void *q, *k, *v;
+    void *out;
+    hla_dtype dt;
+    int BH, n, d, dv, masked, normalized;
+    float eps;
+    int chunk;
+    const float *state_in;
+    float *state_out;
+    char *ws;        // workspace base (header included)
+    size_t ws_bytes;
+};
+
+// generic fp32 SIMT path (any supported shape)
+size_t generic2_workspace_bytes(int BH, int n, int d, int dv, int chunk);
+cudaError_t generic2_forward(const Fwd2 &p, cudaStream_t stream);
+
+// fused tcgen05 path (bf16, d = dv in {64, 128}); returns false if it does not apply
+size_t fused2_workspace_bytes(int BH, int n, int d, int dv, int chunk, hla_dtype dt);
+bool fused2_applicable(const Fwd2 &p);
+cudaError_t fused2_forward(const Fwd2 &p, cudaStream_t stream);
+
+// decode step
+cudaError_t step2_launch(const void *q, const void *k, const void *v, void *out, hla_dtype dt, int BH, int d,
+                         int dv, int masked, int normalized, float eps, float *state, cudaStream_t stream);
+
+// third order
+size_t generic3_workspace_bytes(int BH, int n, int d, int dv, int chunk);
+cudaError_t generic3_forward(const Fwd2 &p, cudaStream_t stream);
+
+}  // namespace hla

@@ -1,0 +1,97 @@
+"""The C ABI without a GPU: the library loads, exports every function that
+include/hla.h declares, and host-side argument checks return their error codes
+before anything is launched."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "hla.h")
+
+
+@pytest.fixture(scope="module")
+def L():
+    from paper_2510_27258_gb300 import build, hla
+    build.build()
+    return hla.lib()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(hla\w+)\s*\(", text)))
+
+
+def test_header_declares_expected_entry_points():
+    from paper_2510_27258_gb300 import hla
+    assert declared_functions() == sorted(hla.EXPORTS)
+
+
+def test_library_exports_every_declared_symbol(L):
+    for name in declared_functions():
+        assert hasattr(L, name), name
+        assert ctypes.cast(getattr(L, name), ctypes.c_void_p).value
+
+
+def test_status_strings(L):
+    from paper_2510_27258_gb300 import hla
+    names = [hla.hla_status_string(c) for c in range(6)]
+    assert names == ["HLA_OK", "HLA_ERR_INVALID_ARGUMENT", "HLA_ERR_UNSUPPORTED", "HLA_ERR_CUDA",
+                     "HLA_ERR_TIMEOUT", "HLA_ERR_WORKSPACE"]
+
+
+def test_state_sizes(L):
+    assert L.hla2_state_floats(128, 128) == 128 * 128 + 2 * 128 * 128 + 2 * 128
+    assert L.hla2_state_floats(16, 32) == 16 * 16 + 2 * 16 * 32 + 32
+    assert L.hla3_state_floats(32, 32) == 2 * 32 * 32 + 4 * 32 * 32 + 4 * 32
+    assert L.hla2_workspace_bytes(1, 1, 64, 16, 16, 16, 0) > 0
+    assert L.hla2_workspace_bytes(1, 1, 64, 48, 16, 16, 0) == 0   # unsupported d
+    assert L.hla2_workspace_bytes(1, 1, 64, 16, 16, 256, 0) == 0  # unsupported chunk
+    assert L.hla2_workspace_bytes(1, 1, 64, 16, 16, 16, 7) == 0   # unknown dtype
+    assert L.hla2_workspace_bytes(2, 16, 16384, 128, 128, 128, 1) % 256 == 0
+
+
+def _fwd(L, q=16, k=16, v=16, out=16, dt=1, B=1, H=1, n=64, d=16, dv=16, masked=1, normalized=0, eps=1e-6,
+         chunk=16, st_in=None, st_out=None, ws=256, ws_bytes=1 << 30, fn="hla2_forward"):
+    return getattr(L, fn)(q, k, v, out, dt, B, H, n, d, dv, masked, normalized, ctypes.c_float(eps), chunk, st_in,
+                          st_out, ws, ws_bytes, None)
+
+
+def test_forward_argument_errors_return_before_launch(L):
+    from paper_2510_27258_gb300 import hla as H
+    # none of these reach a CUDA call: there is no GPU here
+    assert _fwd(L, q=None) == H.HLA_ERR_INVALID_ARGUMENT
+    assert _fwd(L, q=8) == H.HLA_ERR_INVALID_ARGUMENT                      # misaligned
+    assert _fwd(L, dt=5) == H.HLA_ERR_INVALID_ARGUMENT
+    assert _fwd(L, B=-1) == H.HLA_ERR_INVALID_ARGUMENT
+    assert _fwd(L, n=-3) == H.HLA_ERR_INVALID_ARGUMENT
+    assert _fwd(L, masked=2) == H.HLA_ERR_INVALID_ARGUMENT
+    assert _fwd(L, eps=float("nan")) == H.HLA_ERR_INVALID_ARGUMENT
+    assert _fwd(L, d=48) == H.HLA_ERR_UNSUPPORTED
+    assert _fwd(L, dv=256) == H.HLA_ERR_UNSUPPORTED
+    assert _fwd(L, chunk=0) == H.HLA_ERR_INVALID_ARGUMENT
+    assert _fwd(L, chunk=129) == H.HLA_ERR_UNSUPPORTED
+    assert _fwd(L, ws=None) == H.HLA_ERR_WORKSPACE
+    assert _fwd(L, ws_bytes=100) == H.HLA_ERR_WORKSPACE
+    assert _fwd(L, ws=256 + 16) == H.HLA_ERR_INVALID_ARGUMENT              # workspace alignment
+    assert _fwd(L, st_in=4) == H.HLA_ERR_INVALID_ARGUMENT
+    assert "16-byte" in L.hla_last_error().decode()
+    assert _fwd(L, fn="hla3_forward", d=24) == H.HLA_ERR_UNSUPPORTED
+    # empty problems succeed without touching the device
+    assert _fwd(L, B=0) == H.HLA_OK
+    assert _fwd(L, H=0, q=None, k=None, v=None, out=None) == H.HLA_OK
+
+
+def test_step_argument_errors(L):
+    from paper_2510_27258_gb300 import hla as H
+    f = ctypes.c_float(0.0)
+    assert L.hla2_step(16, 16, 16, 16, 1, 1, 1, 128, 128, 1, 0, f, None, None) == H.HLA_ERR_INVALID_ARGUMENT
+    assert L.hla2_step(16, 16, 16, 16, 1, 1, 1, 100, 128, 1, 0, f, 16, None) == H.HLA_ERR_UNSUPPORTED
+    assert L.hla2_step(16, 16, 16, 16, 1, 0, 1, 128, 128, 1, 0, f, 16, None) == H.HLA_OK
+
+
+def test_poll_error_null_workspace(L):
+    from paper_2510_27258_gb300 import hla as H
+    assert L.hla_poll_error(None, None) == H.HLA_ERR_INVALID_ARGUMENT

@@ -1,0 +1,226 @@
+"""Second-order HLA on the GPU (through the C ABI) against the fp64 oracle.
+
+Inputs come from hla_inputs (identical bits on both sides; bf16 values are
+upcast exactly for the oracle).  Error metric per output row t:
+max_c |o_gpu[t,c] - o_ref[t,c]| / ||o_ref[t,:]||_2, maximised over rows.
+Bars: 1e-4 for fp32 tokens, 2e-2 for bf16 tokens (fp32 accumulation).
+"""
+import numpy as np
+import pytest
+import torch
+
+import hla_inputs
+import oracle
+
+pytestmark = pytest.mark.gpu
+
+TOL = {"f32": 1e-4, "bf16": 2e-2}
+DEV = "cuda:0"
+
+
+@pytest.fixture(scope="module")
+def hla():
+    from paper_2510_27258_gb300 import build
+    build.build()
+    from paper_2510_27258_gb300 import hla as binding
+    return binding
+
+
+def rowerr(got, ref):
+    got = np.asarray(got, np.float64)
+    ref = np.asarray(ref, np.float64)
+    nrm = np.linalg.norm(ref, axis=-1, keepdims=True)
+    return float(np.max(np.abs(got - ref) / np.maximum(nrm, 1e-30))) if ref.size else 0.0
+
+
+def gpu_forward(hla, q, k, v, dtype, masked=True, normalized=False, chunk=64, state_in=None, want_state=False,
+                alias_state=False):
+    B, H, n, d = q.shape
+    dv = v.shape[-1]
+    tq, tk, tv = (hla_inputs.as_torch(x, dtype, DEV) for x in (q, k, v))
+    sin = None if state_in is None else torch.from_numpy(np.ascontiguousarray(state_in, np.float32)).to(DEV)
+    sout = None
+    if want_state:
+        sout = sin if alias_state else torch.zeros((B, H, hla.hla2_state_floats(d, dv)), dtype=torch.float32,
+                                                   device=DEV)
+    out = hla.hla2_forward(tq, tk, tv, masked=masked, normalized=normalized, eps=hla_inputs.EPS, chunk=chunk,
+                           state_in=sin, state_out=sout)
+    torch.cuda.synchronize()
+    res = out.float().cpu().numpy()
+    if want_state:
+        return res, sout.cpu().numpy().reshape(B * H, -1)
+    return res
+
+
+def ref_forward(q, k, v, masked=True, normalized=False, state_in=None, heads=None, want_state=False):
+    B, H, n, d = q.shape
+    dv = v.shape[-1]
+    qf, kf, vf = q.reshape(B * H, n, d), k.reshape(B * H, n, d), v.reshape(B * H, n, dv)
+    sin = None if state_in is None else np.asarray(state_in, np.float64).reshape(B * H, -1)
+    if heads is not None:
+        qf, kf, vf = qf[heads], kf[heads], vf[heads]
+        sin = None if sin is None else sin[heads]
+    return oracle.hla2_serial(qf, kf, vf, masked=masked, normalized=normalized, eps=hla_inputs.EPS, state_in=sin,
+                              return_state=want_state, nthreads=8)
+
+
+SMALL = [
+    # (B, H, n, d, dv, chunk, dtype)
+    (1, 1, 1, 16, 16, 16, "f32"),
+    (1, 2, 37, 16, 32, 16, "f32"),
+    (2, 1, 200, 64, 64, 64, "bf16"),
+    (1, 2, 257, 128, 128, 128, "bf16"),
+    (1, 1, 300, 32, 128, 100, "f32"),
+    (1, 1, 130, 128, 64, 7, "bf16"),
+    (1, 3, 96, 64, 16, 32, "f32"),
+]
+
+
+@pytest.mark.parametrize("shape", SMALL, ids=lambda s: "B%dH%dn%dd%ddv%dC%d%s" % s)
+@pytest.mark.parametrize("masked,normalized", [(True, False), (True, True), (False, False), (False, True)])
+def test_forward_small(hla, shape, masked, normalized):
+    B, H, n, d, dv, chunk, dtype = shape
+    q, k, v = hla_inputs.make_qkv(B, H, n, d, dv, seed=1000 + n, dtype=dtype)
+    got = gpu_forward(hla, q, k, v, dtype, masked, normalized, chunk)
+    ref = ref_forward(q, k, v, masked, normalized)
+    assert rowerr(got.reshape(B * H, n, dv), ref) < TOL[dtype]
+
+
+def test_tiny_workload_full(hla):
+    w = hla_inputs.WORKLOADS["tiny_f32"]
+    q, k, v = hla_inputs.make_workload(w)
+    got = gpu_forward(hla, q, k, v, w.dtype, w.masked, w.normalized, w.chunk)
+    ref = ref_forward(q, k, v, w.masked, w.normalized)
+    err = rowerr(got.reshape(w.BH, w.n, w.dv), ref)
+    assert err < 1e-4, err
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+@pytest.mark.parametrize("masked", [True, False])
+def test_state_in_out(hla, dtype, masked):
+    B, H, n, d, dv, chunk = 1, 3, 150, 64, 32, 32
+    pq, pk, pv = hla_inputs.make_qkv(B, H, 40, d, dv, seed=7, dtype=dtype)
+    _, st0 = ref_forward(pq, pk, pv, masked=masked, want_state=True)
+    st0 = st0.astype(np.float32)  # the GPU state is fp32; feed both sides the same values
+    q, k, v = hla_inputs.make_qkv(B, H, n, d, dv, seed=8, dtype=dtype)
+    got, gst = gpu_forward(hla, q, k, v, dtype, masked, True, chunk, state_in=st0, want_state=True)
+    ref, rst = ref_forward(q, k, v, masked, True, state_in=st0, want_state=True)
+    assert rowerr(got.reshape(B * H, n, dv), ref) < TOL[dtype]
+    parts_g, parts_r = oracle.split_state2(gst, d, dv), oracle.split_state2(rst, d, dv)
+    for name in ("S", "C", "m", "G", "h"):
+        scale = max(np.abs(parts_r[name]).max(), np.abs(parts_r["S"]).max() * np.abs(parts_r["C"]).max())
+        assert np.abs(parts_g[name] - parts_r[name]).max() <= 2e-5 * max(scale, 1.0), name
+    if not masked:
+        assert not parts_g["G"].any() and not parts_g["h"].any()
+
+
+def test_state_out_aliases_state_in(hla):
+    B, H, n, d, dv = 1, 2, 64, 32, 32
+    pq, pk, pv = hla_inputs.make_qkv(B, H, 30, d, dv, seed=9, dtype="f32")
+    _, st0 = ref_forward(pq, pk, pv, want_state=True)
+    st0 = st0.astype(np.float32)
+    q, k, v = hla_inputs.make_qkv(B, H, n, d, dv, seed=10, dtype="f32")
+    got, gst = gpu_forward(hla, q, k, v, "f32", True, False, 16, state_in=st0.copy(), want_state=True,
+                           alias_state=True)
+    ref, rst = ref_forward(q, k, v, True, False, state_in=st0, want_state=True)
+    assert rowerr(got.reshape(B * H, n, dv), ref) < 1e-4
+    assert np.abs(gst - rst).max() <= 1e-4 * np.abs(rst).max()
+
+
+def test_empty_sequence_passes_state_through(hla):
+    B, H, d, dv = 1, 2, 16, 16
+    pq, pk, pv = hla_inputs.make_qkv(B, H, 5, d, dv, seed=11, dtype="f32")
+    _, st0 = ref_forward(pq, pk, pv, want_state=True)
+    st0 = st0.astype(np.float32)
+    q = np.zeros((B, H, 0, d), np.float32)
+    v = np.zeros((B, H, 0, dv), np.float32)
+    got, gst = gpu_forward(hla, q, q, v, "f32", True, False, 16, state_in=st0, want_state=True)
+    assert got.shape == (B, H, 0, dv)
+    assert np.abs(gst - st0).max() <= 1e-5 * np.abs(st0).max()
+
+
+def test_causality_bit_exact(hla):
+    B, H, n, d, dv, t = 1, 2, 256, 64, 64, 100
+    q, k, v = hla_inputs.make_qkv(B, H, n, d, dv, seed=12, dtype="bf16")
+    a = gpu_forward(hla, q, k, v, "bf16", True, True, 64)
+    rng = np.random.default_rng(0)
+    q2, k2, v2 = q.copy(), k.copy(), v.copy()
+    q2[:, :, t + 1:] = hla_inputs.round_to(rng.standard_normal(q2[:, :, t + 1:].shape), "bf16")
+    k2[:, :, t + 1:] = hla_inputs.round_to(rng.standard_normal(k2[:, :, t + 1:].shape), "bf16")
+    v2[:, :, t + 1:] = hla_inputs.round_to(rng.standard_normal(v2[:, :, t + 1:].shape), "bf16")
+    b = gpu_forward(hla, q2, k2, v2, "bf16", True, True, 64)
+    assert np.array_equal(a[:, :, : t + 1], b[:, :, : t + 1])
+    assert not np.array_equal(a[:, :, t + 1:], b[:, :, t + 1:])
+
+
+def test_deterministic(hla):
+    q, k, v = hla_inputs.make_qkv(2, 4, 512, 128, 128, seed=13, dtype="bf16")
+    a = gpu_forward(hla, q, k, v, "bf16", True, True, 128)
+    b = gpu_forward(hla, q, k, v, "bf16", True, True, 128)
+    assert np.array_equal(a, b)
+
+
+@pytest.mark.parametrize("name", ["mid_bf16", "long_bf16_norm"])
+def test_workload_full_size_sampled(hla, name):
+    """Full-size workloads in the launch configuration the benchmark times;
+    the oracle checks every position of a few sampled heads."""
+    w = hla_inputs.WORKLOADS[name]
+    q, k, v = hla_inputs.make_workload(w)
+    got = gpu_forward(hla, q, k, v, w.dtype, w.masked, w.normalized, w.chunk)
+    assert np.isfinite(got).all()
+    heads = [0, w.BH // 2 + 1, w.BH - 1]
+    ref = ref_forward(q, k, v, w.masked, w.normalized, heads=heads)
+    err = rowerr(got.reshape(w.BH, w.n, w.dv)[heads], ref)
+    assert err < TOL[w.dtype], err
+
+
+# ----------------------------------------------------------------------------
+# decode step
+# ----------------------------------------------------------------------------
+
+def _decode_run(hla, B, H, d, dv, prefix, steps, dtype, masked, normalized, seed, heads=None):
+    w = hla_inputs.Workload("t", B, H, 0, d, dv, 64, dtype, masked, normalized, seed, decode_prefix=prefix,
+                            decode_steps=steps)
+    (qp, kp, vp), (qs, ks, vs) = hla_inputs.make_decode(w)
+    st = torch.zeros((B, H, hla.hla2_state_floats(d, dv)), dtype=torch.float32, device=DEV)
+    tq, tk, tv = (hla_inputs.as_torch(x, dtype, DEV) for x in (qp, kp, vp))
+    hla.hla2_forward(tq, tk, tv, masked=masked, normalized=normalized, eps=hla_inputs.EPS, chunk=64, state_out=st)
+    outs = []
+    for s in range(steps):
+        o = hla.hla2_step(hla_inputs.as_torch(qs[s], dtype, DEV), hla_inputs.as_torch(ks[s], dtype, DEV),
+                          hla_inputs.as_torch(vs[s], dtype, DEV), st, masked=masked, normalized=normalized,
+                          eps=hla_inputs.EPS)
+        outs.append(o.float().cpu().numpy())
+    torch.cuda.synchronize()
+    got = np.stack(outs, axis=2).reshape(B * H, steps, dv)
+    # oracle: the prefix and the decode tokens as one sequence
+    qa = np.concatenate([qp, np.moveaxis(qs, 0, 2)], axis=2)
+    ka = np.concatenate([kp, np.moveaxis(ks, 0, 2)], axis=2)
+    va = np.concatenate([vp, np.moveaxis(vs, 0, 2)], axis=2)
+    ref, rst = ref_forward(qa, ka, va, masked, normalized, heads=heads, want_state=True)
+    gst = st.cpu().numpy().reshape(B * H, -1)
+    if heads is not None:
+        got, gst = got[heads], gst[heads]
+    return got, ref[:, prefix:], gst, rst
+
+
+@pytest.mark.parametrize("d,dv", [(16, 16), (64, 32), (128, 128), (32, 64)])
+@pytest.mark.parametrize("masked,normalized", [(True, False), (True, True), (False, False)])
+def test_decode_small(hla, d, dv, masked, normalized):
+    dtype = "f32"
+    got, ref, gst, rst = _decode_run(hla, 2, 3, d, dv, 50, 6, dtype, masked, normalized, seed=d + dv)
+    assert rowerr(got, ref) < 1e-4
+    pg, pr = oracle.split_state2(gst, d, dv), oracle.split_state2(rst, d, dv)
+    for name in ("S", "C", "m") + (("G", "h") if masked else ()):
+        scale = max(np.abs(pr[name]).max(), np.abs(pr["S"]).max() * np.abs(pr["C"]).max())
+        assert np.abs(pg[name] - pr[name]).max() <= 2e-5 * max(scale, 1.0), name
+
+
+def test_decode_workload_shape_sampled(hla):
+    """The decode workload's shape (B64 H32 d128, bf16 tokens, fp32 state) with
+    a shortened prefix; the oracle checks sampled heads."""
+    w = hla_inputs.WORKLOADS["decode_bf16"]
+    heads = [0, 1000, w.BH - 1]
+    got, ref, _, _ = _decode_run(hla, w.B, w.H, w.d, w.dv, 256, 4, w.dtype, w.masked, w.normalized, seed=w.seed,
+                                 heads=heads)
+    assert rowerr(got, ref) < 2e-2
