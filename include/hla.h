@@ -122,6 +122,18 @@ hla_status hla2_step(const void *q, const void *k, const void *v, void *out, hla
                      int B, int H, int d, int dv, int masked, int normalized, float eps,
                      float *state, hla_stream_t stream);
 
+/*
+ * hla2_forward_path -- which CUDA path hla2_forward takes for these arguments
+ * on the current device, without launching anything:
+ *   0  generic path: fp32 CUDA-core kernels (every supported shape);
+ *   1  fused path: one persistent tcgen05/TMA kernel (bf16 tokens,
+ *      d = dv = 128, masked, chunk = 128, no state_out) on sm_103;
+ *  -1  the arguments are not supported.
+ * *launches (if not NULL) receives the number of kernels the call launches.
+ */
+int hla2_forward_path(int B, int H, int n, int d, int dv, int masked, int normalized, int chunk, hla_dtype dt,
+                      int has_state_in, int has_state_out, int *launches);
+
 /* Number of floats of one head's third-order state tuple (Theorem 3):
  * [ SK d*d | SQ d*d | P d*dv | mK d | G1 d*dv | G2 d*dv | G3 d*dv | h1 d | h2 d | h3 d ]. */
 size_t hla3_state_floats(int d, int dv);

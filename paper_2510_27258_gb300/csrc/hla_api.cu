@@ -128,6 +128,25 @@ hla_status hla2_forward(const void *q, const void *k, const void *v, void *out, 
     return cuda_status(generic2_forward(p, s), "generic forward");
 }
 
+int hla2_forward_path(int B, int H, int n, int d, int dv, int masked, int normalized, int chunk, hla_dtype dt,
+                      int has_state_in, int has_state_out, int *launches) {
+    const void *dummy = reinterpret_cast<const void *>(uintptr_t(256));
+    if (check_forward(dummy, dummy, dummy, const_cast<void *>(dummy), dt, B, H, n, d, dv, masked, normalized, 0.f,
+                      chunk, nullptr, nullptr) != HLA_OK)
+        return -1;
+    Fwd2 p{dummy, dummy, dummy, const_cast<void *>(dummy), dt, B * H, n, d, dv, masked, normalized, 0.f, chunk,
+           has_state_in ? static_cast<const float *>(dummy) : nullptr,
+           has_state_out ? static_cast<float *>(const_cast<void *>(dummy)) : nullptr, nullptr,
+           hla2_workspace_bytes(B, H, n, d, dv, chunk, dt)};
+    const bool fused = (long long)B * H > 0 && fused2_applicable(p);
+    if (launches) {
+        if ((long long)B * H == 0) *launches = 0;
+        else if (fused) *launches = 1 + (has_state_in ? 1 : 0);
+        else *launches = n > 0 ? 3 : 1;
+    }
+    return fused ? 1 : 0;
+}
+
 hla_status hla2_step(const void *q, const void *k, const void *v, void *out, hla_dtype dt, int B, int H, int d,
                      int dv, int masked, int normalized, float eps, float *state, hla_stream_t stream) {
     g_last_error[0] = 0;

@@ -21,7 +21,8 @@ HLA_F32, HLA_BF16 = 0, 1
 
 # every symbol include/hla.h declares
 EXPORTS = ("hla_status_string", "hla_last_error", "hla2_state_floats", "hla2_workspace_bytes", "hla2_forward",
-           "hla2_step", "hla3_state_floats", "hla3_workspace_bytes", "hla3_forward", "hla_poll_error")
+           "hla2_forward_path", "hla2_step", "hla3_state_floats", "hla3_workspace_bytes", "hla3_forward",
+           "hla_poll_error")
 
 _lib = None
 
@@ -55,6 +56,8 @@ def lib():
         for name in ("hla2_forward", "hla3_forward"):
             getattr(L, name).argtypes = [vp, vp, vp, vp, i, i, i, i, i, i, i, i, f, i, vp, vp, vp, sz, vp]
             getattr(L, name).restype = i
+        L.hla2_forward_path.argtypes = [i, i, i, i, i, i, i, i, i, i, i, ctypes.POINTER(i)]
+        L.hla2_forward_path.restype = i
         L.hla2_step.argtypes = [vp, vp, vp, vp, i, i, i, i, i, i, i, f, vp, vp]
         L.hla2_step.restype = i
         L.hla_poll_error.argtypes = [vp, vp]
@@ -147,6 +150,16 @@ def hla3_forward(q, k, v, out=None, *, masked=True, normalized=False, eps=1e-6, 
     """Third-order HLA forward (include/hla.h: hla3_forward). Returns ``out``."""
     return _forward("hla3_forward", hla3_workspace_bytes, q, k, v, out, masked, normalized, eps, chunk, state_in,
                     state_out, workspace, stream)
+
+
+def hla2_forward_path(B, H, n, d, dv, *, masked=True, normalized=False, chunk=128, dtype=torch.bfloat16,
+                      has_state_in=False, has_state_out=False):
+    """(path, launches) that hla2_forward takes: path 1 = fused tcgen05 kernel, 0 = generic, -1 = unsupported."""
+    code = dtype if isinstance(dtype, int) else (HLA_BF16 if dtype == torch.bfloat16 else HLA_F32)
+    n_launch = ctypes.c_int(0)
+    path = lib().hla2_forward_path(B, H, n, d, dv, int(masked), int(normalized), int(chunk), code,
+                                   int(has_state_in), int(has_state_out), ctypes.byref(n_launch))
+    return int(path), int(n_launch.value)
 
 
 def hla2_step(q, k, v, state, out=None, *, masked=True, normalized=False, eps=1e-6, stream=None):

@@ -1,0 +1,127 @@
+"""The fused tcgen05 forward (bf16, d = dv = 128, masked, chunk 128) against the
+fp64 oracle, including its cross-SM chained scans (forced short segments),
+ragged tails, an initial state, and the device-side timeout path."""
+import numpy as np
+import pytest
+import torch
+
+import hla_inputs
+import oracle
+from parity import check_normalized, rowerr
+
+pytestmark = pytest.mark.gpu
+DEV = "cuda:0"
+
+
+@pytest.fixture(scope="module")
+def hla():
+    from paper_2510_27258_gb300 import build
+    build.build()
+    from paper_2510_27258_gb300 import hla as binding
+    return binding
+
+
+def run(hla, q, k, v, normalized, state_in=None):
+    tq, tk, tv = (hla_inputs.as_torch(x, "bf16", DEV) for x in (q, k, v))
+    sin = None if state_in is None else torch.from_numpy(np.ascontiguousarray(state_in, np.float32)).to(DEV)
+    ws = hla.alloc_workspace(hla.hla2_workspace_bytes(*q.shape, v.shape[-1], 128, torch.bfloat16), DEV)
+    out = hla.hla2_forward(tq, tk, tv, masked=True, normalized=normalized, eps=hla_inputs.EPS, chunk=128,
+                           state_in=sin, workspace=ws)
+    torch.cuda.synchronize()
+    assert hla.hla_poll_error(ws) == 0
+    B, H, n, _ = q.shape
+    return out.float().cpu().numpy().reshape(B * H, n, -1)
+
+
+def check(hla, q, k, v, normalized, state_in=None):
+    B, H, n, d = q.shape
+    assert hla.hla2_forward_path(B, H, n, d, d, normalized=normalized, has_state_in=state_in is not None)[0] == 1
+    sin = None if state_in is None else np.asarray(state_in, np.float64).reshape(B * H, -1)
+    num_ref, den_ref = oracle.hla2_serial(q.reshape(B * H, n, d), k.reshape(B * H, n, d), v.reshape(B * H, n, d),
+                                          masked=True, normalized=False, state_in=sin, return_den=True, nthreads=8)
+    num = run(hla, q, k, v, False, state_in)
+    if not normalized:
+        err = rowerr(num, num_ref)
+        assert err < 2e-2, err
+        return err
+    o = run(hla, q, k, v, True, state_in)
+    return check_normalized(o, num, num_ref, den_ref, hla_inputs.EPS, 2e-2)
+
+
+def test_fused_path_selected(hla):
+    assert hla.hla2_forward_path(2, 16, 16384, 128, 128, normalized=True) == (1, 1)
+    assert hla.hla2_forward_path(2, 16, 16384, 128, 128, normalized=True, has_state_out=True)[0] == 0
+    assert hla.hla2_forward_path(2, 16, 16384, 128, 128, masked=False)[0] == 0
+    assert hla.hla2_forward_path(2, 16, 16384, 64, 64)[0] == 0
+
+
+@pytest.mark.parametrize("B,H,n", [(1, 1, 1), (1, 2, 127), (1, 2, 128), (1, 3, 129), (2, 2, 600), (1, 1, 2000)])
+@pytest.mark.parametrize("seg", ["1", "2", "3", "default"])
+@pytest.mark.parametrize("normalized", [False, True])
+def test_fused_matches_oracle(hla, monkeypatch, B, H, n, seg, normalized):
+    if seg != "default":
+        monkeypatch.setenv("HLA_FUSED_SEGMENT_TILES", seg)
+    q, k, v = hla_inputs.make_qkv(B, H, n, 128, 128, seed=n + 17 * H, dtype="bf16")
+    check(hla, q, k, v, normalized)
+
+
+@pytest.mark.parametrize("seg", ["1", "default"])
+def test_fused_initial_state(hla, monkeypatch, seg):
+    if seg != "default":
+        monkeypatch.setenv("HLA_FUSED_SEGMENT_TILES", seg)
+    B, H, d = 1, 2, 128
+    pq, pk, pv = hla_inputs.make_qkv(B, H, 300, d, d, seed=5, dtype="bf16")
+    _, st0 = oracle.hla2_serial(pq.reshape(B * H, 300, d), pk.reshape(B * H, 300, d), pv.reshape(B * H, 300, d),
+                                masked=True, return_state=True)
+    st0 = st0.astype(np.float32)
+    q, k, v = hla_inputs.make_qkv(B, H, 400, d, d, seed=6, dtype="bf16")
+    check(hla, q, k, v, True, state_in=st0)
+    check(hla, q, k, v, False, state_in=st0)
+
+
+def test_fused_deterministic(hla, monkeypatch):
+    monkeypatch.setenv("HLA_FUSED_SEGMENT_TILES", "2")
+    q, k, v = hla_inputs.make_qkv(2, 3, 1500, 128, 128, seed=21, dtype="bf16")
+    a = run(hla, q, k, v, True)
+    b = run(hla, q, k, v, True)
+    assert np.array_equal(a, b)
+
+
+def test_fused_equals_generic_closely(hla, monkeypatch):
+    """Both CUDA paths on the same inputs (the generic one in fp32 SIMT)."""
+    q, k, v = hla_inputs.make_qkv(1, 2, 700, 128, 128, seed=31, dtype="bf16")
+    a = run(hla, q, k, v, False)
+    monkeypatch.setenv("HLA_DISABLE_FUSED", "1")
+    b = run(hla, q, k, v, False)
+    assert rowerr(a, b) < 2e-2
+
+
+def test_fused_causality_bit_exact(hla):
+    B, H, n, t = 1, 2, 700, 300
+    q, k, v = hla_inputs.make_qkv(B, H, n, 128, 128, seed=40, dtype="bf16")
+    a = run(hla, q, k, v, True)
+    rng = np.random.default_rng(1)
+    q2, k2, v2 = q.copy(), k.copy(), v.copy()
+    for x in (q2, k2, v2):
+        x[:, :, t + 1:] = hla_inputs.round_to(rng.standard_normal(x[:, :, t + 1:].shape), "bf16")
+    b = run(hla, q2, k2, v2, True)
+    assert np.array_equal(a[:, : t + 1], b[:, : t + 1])
+
+
+def test_fused_wait_timeout_is_reported_not_hung(hla, monkeypatch):
+    """A segment that never publishes its S prefix (injected on the host side):
+    the next segment's bounded wait runs out, the kernel finishes, and
+    hla_poll_error reports HLA_ERR_TIMEOUT; the workspace then works again."""
+    monkeypatch.setenv("HLA_FUSED_SEGMENT_TILES", "1")
+    monkeypatch.setenv("HLA_TEST_WAIT_NS", "20000000")     # 20 ms budget
+    monkeypatch.setenv("HLA_TEST_SKIP_PUBLISH_ITEM", "0")  # (head 0, segment 0) skips its publish
+    q, k, v = hla_inputs.make_qkv(1, 1, 512, 128, 128, seed=50, dtype="bf16")
+    tq, tk, tv = (hla_inputs.as_torch(x, "bf16", DEV) for x in (q, k, v))
+    ws = hla.alloc_workspace(hla.hla2_workspace_bytes(1, 1, 512, 128, 128, 128, torch.bfloat16), DEV)
+    hla.hla2_forward(tq, tk, tv, masked=True, normalized=False, chunk=128, workspace=ws)
+    assert hla.hla_poll_error(ws) == hla.HLA_ERR_TIMEOUT
+    monkeypatch.delenv("HLA_TEST_SKIP_PUBLISH_ITEM")
+    out = hla.hla2_forward(tq, tk, tv, masked=True, normalized=False, chunk=128, workspace=ws)
+    assert hla.hla_poll_error(ws) == hla.HLA_OK
+    ref = oracle.hla2_serial(q.reshape(1, 512, 128), k.reshape(1, 512, 128), v.reshape(1, 512, 128), masked=True)
+    assert rowerr(out.float().cpu().numpy().reshape(1, 512, 128), ref) < 2e-2
