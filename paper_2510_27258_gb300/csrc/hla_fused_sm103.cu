@@ -7,7 +7,7 @@
 //   A = Q K^T,  W = L . A                        (L: lower triangle incl. diagonal)
 //   X = W K + Q S_p                              (rows x_t = S_t q_t)
 //   T = L . (Q X^T),  O = T V + Q D_p            (D = sum_j x_j v_j^T = S C - G)
-//   den_t = q_t . (e_p + sum_{j<=t} x_j)         (e = sum_j x_j = S m - h)
+//   den_t = sum_{j<=t} T_tj + q_t . e_p          (e = sum_j x_j = S m - h)
 //   S_p += K^T K,  D_p += X^T V,  e_p += X^T 1
 // The carries compose across tiles as the semidirect product of Eq. semidirect
 // does (D_AB = D_A + D_B + S_A C_B is the D-form of G_AB = G_A + G_B + S_B C_A).
@@ -26,12 +26,19 @@
 // The exclusive scan across segments is a chained scan; Theorem 2 guarantees
 // the result equals the serial recurrence.
 //
+// Roles: warp 8 issues TMA loads and MMAs (one thread); warps 0-7 are the
+// epilogue (TMEM -> registers -> shared memory): warp w reads TMEM lanes
+// 32 (w % 4) .. +31 (one row each) and columns 64 (w / 4) .. +63.
+//
 // Precision: tokens are bf16, every product accumulates in fp32 (TMEM).  The S
-// operand is split as S = c I + R (c = bf16(trace S / d)), R rounded to
-// bf16 hi (+ lo for the normalised output), and c q_t is added in fp32: x_t is
-// then accurate to ~2^-17 |R| although |S| grows like t/d.  X, T and D enter
-// later MMAs as bf16 (numerator only); the denominator is formed on CUDA cores
-// in fp32 from the fp32 X accumulator (prefix sums over the tile).
+// operand is split as S = c I + R (c = bf16(trace S / d)) with c q_t added in
+// fp32, so x_t is accurate although |S| grows like t/d.  X enters T = Q X^T as
+// bf16 hi + lo (with X rounded once, q_t . x_t = (q_t . k_t)^2 at t = 0 would
+// lose |q||k| / |q.k| times the bf16 rounding when q and k are nearly
+// orthogonal).  For the normalised output, whose denominator cancels heavily,
+// R and W are also split into hi + lo, so X and T are accurate to ~2^-16 of
+// each term; the denominator is the fp32 row sum of T plus q_t . e_p, with the
+// e carry summed in fp32 on CUDA cores.  T and D enter T V and Q D as bf16.
 #include "hla_internal.h"
 #include "sm103_prims.cuh"
 
@@ -42,17 +49,19 @@ using namespace sm103;
 
 constexpr int kD = 128;           // d = dv handled by this kernel
 constexpr int kTile = 128;        // tokens per tile (MMA M)
-constexpr int kEpiThreads = 128;  // 4 epilogue warps: warp w reads TMEM lanes 32w..32w+31
+constexpr int kEpiWarps = 8;      // 2 per TMEM lane quadrant
+constexpr int kEpiThreads = kEpiWarps * 32;
+constexpr int kIssuerWarp = kEpiWarps;
 constexpr int kThreads = kEpiThreads + 32;
 constexpr int kSlots = 7;
 constexpr uint32_t kSmemTiles = kSlots * kTileBytes;
-constexpr uint32_t kMiscBytes = 2048;
-constexpr uint32_t kSmemBytes = kSmemTiles + 1024 + kMiscBytes;  // + alignment slack
+constexpr uint32_t kMiscBytes = 3072;
+constexpr uint32_t kSmemBytes = kSmemTiles + kMiscBytes;  // = 227 KiB; base must be 1 KiB aligned
 
 // shared-memory slots (32 KiB each)
 enum Slot { kQ0 = 0, kQ1 = 1, kK = 2, kV = 3, kW = 4, kSX = 5, kSD = 6 };
 
-// TMEM columns
+// TMEM columns: S carry, D carry, A -> T, X -> O
 constexpr uint32_t kTS = 0, kTD = 128, kTA = 256, kTX = 384;
 
 // barrier indices
@@ -60,20 +69,22 @@ enum Bar {
     bLd0 = 0,  // + slot index for the four input slots (Q0, Q1, K, V)
     bPre = 4,  // pre-pass MMA done (per K tile)
     bEvP = 5, bEvA = 6, bEvX = 7, bEvT = 8, bEvO = 9, bEvF = 10,
-    bEpS = 11, bEpW = 12, bEpX = 13, bEpT = 14, bEpO = 15, bEpF = 16, bEpDF = 17,
-    kNumBars = 18
+    bEpW = 11, bEpX = 12, bEpT = 13, bEpF = 14, bEpDF = 15,
+    kNumBars = 16
 };
+constexpr int kFirstEpiBar = bEpW;
 
 struct Misc {
     uint64_t bar[kNumBars];
     uint32_t tmem_base;
     int item;        // current ticket
-    int abort_flag;  // a wait gave up: skip the rest of the work
-    float cshift[2]; // S shift of the next tiles
-    float red[4];
-    float eloc[kD];  // segment-local e carry
-    float den[kTile];
-    float tot[4][32];  // per-warp column totals of the prefix scan
+    int abort_flag;  // an mbarrier wait gave up
+    int pad;
+    float cshift[2]; // S shift of the current / next tile
+    float red[kEpiWarps];
+    float eloc[kD];      // segment-local e carry
+    float den[kTile];    // denominators of the current tile
+    float ebuf[2][kD];   // cross-quadrant partial column sums of X
 };
 static_assert(sizeof(Misc) <= kMiscBytes, "misc smem");
 
@@ -88,11 +99,13 @@ struct Params {
     unsigned *ticket;
     float *den_loc;         // [BH][n] provisional denominators (normalised, segments > 0)
     WsHeader *err;
-    unsigned long long wait_ns;      // budget of a cross-SM chain wait
-    int inject_skip_item;   // testing: this item does not publish its S prefix
+    unsigned long long wait_ns;  // budget of a cross-SM chain wait
+    int inject_skip_item;        // testing: this item does not publish its S prefix
 };
 
 constexpr int kRingFloats = kD * kD + kD * kD + kD;
+// floats of one head's state tuple [S | C | m | G | h] with d = dv = kD
+constexpr int kStateFloats = kD * kD + 2 * kD * kD + 2 * kD;
 // budget of an intra-CTA mbarrier wait (TMA or MMA completion, epilogue hand-off)
 constexpr unsigned long long kBarWaitNs = 2000000000ull;
 
@@ -105,7 +118,8 @@ __device__ __forceinline__ unsigned ld_acquire(const unsigned *p) {
     asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
     return v;
 }
-__device__ __forceinline__ void epi_sync() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
+// named barrier of the epilogue warps
+__device__ __forceinline__ void epi_sync() { asm volatile("bar.sync 1, 256;" ::: "memory"); }
 
 __device__ __forceinline__ void set_error(WsHeader *err, unsigned where, unsigned detail) {
     if (atomicCAS(&err->error, 0u, (unsigned)kDevTimeout) == 0u) {
@@ -139,7 +153,7 @@ __device__ __forceinline__ bool bar_wait(Misc *ms, int b, uint32_t parity, const
     return false;
 }
 
-// epilogue warps arrive (count 4): lane 0 after the warp's own fences
+// epilogue warps arrive (count kEpiWarps): lane 0 after the warp's own fences
 __device__ __forceinline__ void epi_arrive(Misc *ms, int b) {
     tc_fence_before();
     __syncwarp();
@@ -166,20 +180,42 @@ __device__ __forceinline__ void store_row8(uint8_t *tile, int r, int c, const fl
     *reinterpret_cast<uint4 *>(tile + tile_off(r, c)) = u;
 }
 
+__device__ __forceinline__ void store_zero32(uint8_t *tile, int r, int c0) {
+#pragma unroll
+    for (int j = 0; j < 32; j += 8) *reinterpret_cast<uint4 *>(tile + tile_off(r, c0 + j)) = make_uint4(0, 0, 0, 0);
+}
+
 __device__ __forceinline__ float bf16_round(float x) { return __bfloat162float(__float2bfloat16_rn(x)); }
 
-// S (row i of the carry, 128 fp32 in `s`) -> shift c, R_hi row -> tile SX, R_lo row -> tile SD (if lo)
-__device__ __forceinline__ void write_split_row(uint8_t *hi_tile, uint8_t *lo_tile, int i, const float *s, float c,
-                                                int c0, bool lo) {
-    float h[8], l[8];
+__device__ __forceinline__ void ld32(uint32_t addr, float (&f)[32]) {
+    uint32_t a[32];
+    tmem_ld32(addr, a);
+    tmem_ld_wait();
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
-        const float r = s[j] - ((c0 + j) == i ? c : 0.f);
-        h[j] = bf16_round(r);
-        l[j] = r - h[j];
+    for (int j = 0; j < 32; ++j) f[j] = __uint_as_float(a[j]);
+}
+
+// Column sums of v over the 32 lanes of a warp: returns, in lane l, the sum of
+// column l (31 shuffles: each step halves the columns a lane keeps).
+__device__ __forceinline__ float warp_colsum32(float (&v)[32]) {
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) {
+        const bool upper = (lane & o) != 0;
+#pragma unroll
+        for (int i = 0; i < o; ++i) {
+            const float send = upper ? v[i] : v[i + o];
+            const float keep = upper ? v[i + o] : v[i];
+            v[i] = keep + __shfl_xor_sync(0xffffffffu, send, o);
+        }
     }
-    store_row8(hi_tile, i, c0, h);
-    if (lo) store_row8(lo_tile, i, c0, l);
+    return v[0];
+}
+
+__device__ __forceinline__ float warp_sum(float x) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+    return x;
 }
 
 // ---------------------------------------------------------------------------
@@ -188,18 +224,20 @@ __device__ __forceinline__ void write_split_row(uint8_t *hi_tile, uint8_t *lo_ti
 __global__ void __launch_bounds__(kThreads, 1)
 hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                   const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_o, Params p) {
-    extern __shared__ uint8_t smem_raw[];
-    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    extern __shared__ __align__(1024) uint8_t smem[];
     Misc *ms = reinterpret_cast<Misc *>(smem + kSmemTiles);
     auto slot = [&](int s) { return smem + s * kTileBytes; };
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const bool issuer = (warp == 4);
+    const bool issuer = (warp == kIssuerWarp);
 
+    // the tile layout needs 1 KiB alignment of the dynamic shared memory
+    if (smem_u32(smem) & 1023u) {
+        if (tid == 0) set_error(p.err, 99, smem_u32(smem));
+        return;
+    }
     if (tid == 0) {
-        for (int b = 0; b < kNumBars; ++b) mbar_init(&ms->bar[b], 1);
-        // epilogue-arrival barriers complete when all four epilogue warps arrive
-        for (int b = bEpS; b <= bEpDF; ++b) mbar_init(&ms->bar[b], 4);
+        for (int b = 0; b < kNumBars; ++b) mbar_init(&ms->bar[b], b >= kFirstEpiBar ? kEpiWarps : 1);
         ms->abort_flag = 0;
         fence_mbar_init();
     }
@@ -235,12 +273,14 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
 
     while (true) {
         if (tid == 0) ms->item = (int)atomicAdd(p.ticket, 1u);
+        tc_fence_before();
         __syncthreads();
+        tc_fence_after();
         const int item = ms->item;
         if (item >= p.n_items || ms->abort_flag) break;
         const int sigma = item / p.BH, head = item % p.BH;
-        const int t0 = sigma * p.L;                       // first tile of the segment
-        const int nt = min(p.L, p.M - t0);                // tiles in this segment
+        const int t0 = sigma * p.L;           // first tile of the segment
+        const int nt = min(p.L, p.M - t0);    // tiles in this segment
         const int ip = n_items & 1;
 
         if (issuer) {
@@ -261,26 +301,28 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                     if (j + 2 < nt) load_tile(s, &tm_k, head, (t0 + j + 2) * kTile);
                 }
                 umma_commit(&ms->bar[bEvP]);
-                // first tile's inputs
+                // first tile's inputs and its A = Q K^T
                 load_tile(kQ0, &tm_q, head, t0 * kTile);
                 load_tile(kK, &tm_k, head, t0 * kTile);
                 load_tile(kV, &tm_v, head, t0 * kTile);
+                if (wait_ld(kQ0) && wait_ld(kK)) {
+                    tc_fence_after();
+                    for (int kk = 0; kk < 8; ++kk)
+                        umma_bf16(tb + kTA, desc_kmajor(tileQ[0], kk), desc_kmajor(sK, kk), idA, kk > 0);
+                    umma_commit(&ms->bar[bEvA]);
+                }
 
                 // ---- 2. sweep ----
                 for (int j = 0; j < nt && !ms->abort_flag; ++j) {
                     const uint32_t tp = n_tiles & 1;
-                    const int qs = (j & 1) ? kQ1 : kQ0;
-                    const uint32_t sQ = tileQ[j & 1];
-                    if (!wait_ld(qs) || !wait_ld(kK)) break;
+                    const uint32_t sQ = tileQ[j & 1], sQo = tileQ[(j + 1) & 1];
+                    if (!bar_wait(ms, bEpW, tp, p)) break;  // W (hi, lo), S split ready; TMEM X free
                     tc_fence_after();
-                    for (int kk = 0; kk < 8; ++kk)  // A = Q K^T
-                        umma_bf16(tb + kTA, desc_kmajor(sQ, kk), desc_kmajor(sK, kk), idA, kk > 0);
-                    umma_commit(&ms->bar[bEvA]);
-                    if (j + 1 < nt) load_tile((j & 1) ? kQ0 : kQ1, &tm_q, head, (t0 + j + 1) * kTile);
-                    if (!bar_wait(ms, bEpW, tp, p)) break;  // W, S split ready; TMEM X free
-                    tc_fence_after();
-                    for (int kk = 0; kk < 8; ++kk)  // X = W K
+                    for (int kk = 0; kk < 8; ++kk)  // X = W_hi K
                         umma_bf16(tb + kTX, desc_kmajor(sW, kk), desc_mnmajor(sK, kk), idKmn, kk > 0);
+                    if (p.normalized)
+                        for (int kk = 0; kk < 8; ++kk)  // X += W_lo K  (W_lo staged in the other Q slot)
+                            umma_bf16(tb + kTX, desc_kmajor(sQo, kk), desc_mnmajor(sK, kk), idKmn, 1u);
                     for (int kk = 0; kk < 8; ++kk)  // X += Q R_hi
                         umma_bf16(tb + kTX, desc_kmajor(sQ, kk), desc_kmajor(sSX, kk), idA, 1u);
                     if (p.normalized)
@@ -290,31 +332,42 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                         umma_bf16(tb + kTS, desc_mnmajor(sK, kk), desc_mnmajor(sK, kk), idMM, 1u);
                     umma_commit(&ms->bar[bEvX]);
                     if (!bar_wait(ms, bEvX, tp, p)) break;
-                    if (j + 1 < nt) load_tile(kK, &tm_k, head, (t0 + j + 1) * kTile);
-                    if (!bar_wait(ms, bEpX, tp, p)) break;  // X_hi and D_hi ready
+                    if (j + 1 < nt) {
+                        load_tile(kK, &tm_k, head, (t0 + j + 1) * kTile);
+                        load_tile((j & 1) ? kQ0 : kQ1, &tm_q, head, (t0 + j + 1) * kTile);
+                    }
+                    if (!bar_wait(ms, bEpX, tp, p)) break;  // X_hi, X_lo and D_hi ready
                     if (!wait_ld(kV)) break;
                     tc_fence_after();
-                    for (int kk = 0; kk < 8; ++kk)  // T = Q X^T
+                    for (int kk = 0; kk < 8; ++kk)  // T = Q X_hi^T
                         umma_bf16(tb + kTA, desc_kmajor(sQ, kk), desc_kmajor(sSX, kk), idA, kk > 0);
+                    for (int kk = 0; kk < 8; ++kk)  // T += Q X_lo^T  (X_lo staged in slot W)
+                        umma_bf16(tb + kTA, desc_kmajor(sQ, kk), desc_kmajor(sW, kk), idA, 1u);
                     for (int kk = 0; kk < 8; ++kk)  // D += X^T V
                         umma_bf16(tb + kTD, desc_mnmajor(sSX, kk), desc_mnmajor(sV, kk), idMM, 1u);
                     umma_commit(&ms->bar[bEvT]);
-                    if (!bar_wait(ms, bEpT, tp, p)) break;  // T ready
+                    if (!bar_wait(ms, bEpT, tp, p)) break;  // T ready; TMEM A free
                     tc_fence_after();
                     for (int kk = 0; kk < 8; ++kk)  // O = Q D_p
-                        umma_bf16(tb + kTA, desc_kmajor(sQ, kk), desc_mnmajor(sSD, kk), idKmn, kk > 0);
+                        umma_bf16(tb + kTX, desc_kmajor(sQ, kk), desc_mnmajor(sSD, kk), idKmn, kk > 0);
                     for (int kk = 0; kk < 8; ++kk)  // O += T V
-                        umma_bf16(tb + kTA, desc_kmajor(sW, kk), desc_mnmajor(sV, kk), idKmn, 1u);
+                        umma_bf16(tb + kTX, desc_kmajor(sW, kk), desc_mnmajor(sV, kk), idKmn, 1u);
                     umma_commit(&ms->bar[bEvO]);
+                    if (j + 1 < nt) {  // next tile's A = Q K^T overlaps this tile's output epilogue
+                        if (!wait_ld((j & 1) ? kQ0 : kQ1) || !wait_ld(kK)) break;
+                        tc_fence_after();
+                        for (int kk = 0; kk < 8; ++kk)
+                            umma_bf16(tb + kTA, desc_kmajor(sQo, kk), desc_kmajor(sK, kk), idA, kk > 0);
+                        umma_commit(&ms->bar[bEvA]);
+                    }
                     if (!bar_wait(ms, bEvO, tp, p)) break;
                     if (j + 1 < nt) load_tile(kV, &tm_v, head, (t0 + j + 1) * kTile);
-                    if (!bar_wait(ms, bEpO, tp, p)) break;  // O read, next S split ready
                     ++n_tiles;
                 }
 
                 // ---- 3. fix-up of segments > 0 ----
                 if (sigma > 0 && !ms->abort_flag) {
-                    if (bar_wait(ms, bEpDF, n_dfix & 1, p)) {  // D prefix (bf16) in SD
+                    if (bar_wait(ms, bEpDF, n_dfix & 1, p)) {  // D prefix (bf16) in SD; outputs written
                         load_tile(kQ0, &tm_q, head, t0 * kTile);
                         load_tile(kK, &tm_o, head, t0 * kTile);
                         for (int j = 0; j < nt; ++j) {
@@ -338,240 +391,252 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
             __syncwarp();
         } else {
             // ===================== epilogue warps =====================
-            const int r = tid;                 // TMEM lane = row handled by this thread
-            const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
-            float *ring_prev_S = p.ring + ((size_t)head * 2 + ((sigma + 1) & 1)) * kRingFloats;
+            const int et = tid;
+            const int qd = warp & 3, hf = warp >> 2;
+            const int r = 32 * qd + lane;        // TMEM lane = row handled by this thread
+            const int cb0 = 64 * hf;             // first of the 64 columns handled by this thread
+            const uint32_t lane_base = (uint32_t)(32 * qd) << 16;
+            const float *ring_prev = p.ring + ((size_t)head * 2 + ((sigma + 1) & 1)) * kRingFloats;
             float *ring_cur = p.ring + ((size_t)head * 2 + (sigma & 1)) * kRingFloats;
             unsigned *flagS = p.flags, *flagD = p.flags + 2 * p.BH;
 
-            // ---- 1. S chain ----
+            // ---- 1. S chain: carry-in S of the segment, publish the inclusive prefix ----
             bar_wait(ms, bEvP, ip, p);
             tc_fence_after();
-            if (sigma > 0 && r == 0) chain_wait(&flagS[head * 2 + ((sigma - 1) & 1)], (unsigned)sigma, p, 1, item);
+            if (sigma > 0 && et == 0) chain_wait(&flagS[head * 2 + ((sigma - 1) & 1)], (unsigned)sigma, p, 1, item);
             epi_sync();
             {
                 const float *sprev = nullptr;
-                if (sigma > 0) sprev = ring_prev_S + r * kD;
-                else if (p.state_in) sprev = p.state_in + (size_t)head * (2 * kD * kD + 2 * kD) + r * kD;
-                // diagonal element -> shift
-                const float diag = sprev ? __ldcg(sprev + r) : 0.f;
-                float s = diag;
-                for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+                if (sigma > 0) sprev = ring_prev + r * kD;
+                else if (p.state_in) sprev = p.state_in + (size_t)head * kStateFloats + r * kD;
+                float s = (sprev && (r >> 6) == hf) ? __ldcg(sprev + r) : 0.f;  // diagonal -> trace
+                s = warp_sum(s);
                 if (lane == 0) ms->red[warp] = s;
                 epi_sync();
-                const float c = bf16_round((ms->red[0] + ms->red[1] + ms->red[2] + ms->red[3]) / kD);
-                if (r == 0) ms->cshift[0] = c;
-                for (int c0 = 0; c0 < kD; c0 += 32) {
-                    uint32_t agg[32], sv[32];
-                    tmem_ld32(tb + lane_base + kTX + c0, agg);
-                    tmem_ld_wait();
-                    float sp[32];
+                float tr = 0.f;
+#pragma unroll
+                for (int w = 0; w < kEpiWarps; ++w) tr += ms->red[w];
+                const float c = bf16_round(tr / kD);
+                if (et == 0) ms->cshift[0] = c;
+                const float *d0 = (sigma == 0 && p.init_De) ? p.init_De + (size_t)head * (kD * kD + kD) : nullptr;
+#pragma unroll 1
+                for (int c0 = cb0; c0 < cb0 + 64; c0 += 32) {
+                    float agg[32], sp[32];
+                    ld32(tb + lane_base + kTX + c0, agg);
 #pragma unroll
                     for (int j = 0; j < 32; j += 4) {
-                        float4 v4 = sprev ? __ldcg(reinterpret_cast<const float4 *>(sprev + c0 + j))
-                                          : make_float4(0.f, 0.f, 0.f, 0.f);
+                        const float4 v4 = sprev ? __ldcg(reinterpret_cast<const float4 *>(sprev + c0 + j))
+                                                : make_float4(0.f, 0.f, 0.f, 0.f);
                         sp[j] = v4.x; sp[j + 1] = v4.y; sp[j + 2] = v4.z; sp[j + 3] = v4.w;
                     }
 #pragma unroll
-                    for (int j = 0; j < 32; j += 4) {
-                        float4 o4 = make_float4(sp[j] + __uint_as_float(agg[j]), sp[j + 1] + __uint_as_float(agg[j + 1]),
-                                                sp[j + 2] + __uint_as_float(agg[j + 2]),
-                                                sp[j + 3] + __uint_as_float(agg[j + 3]));
-                        __stcg(reinterpret_cast<float4 *>(ring_cur + r * kD + c0 + j), o4);
+                    for (int j = 0; j < 32; j += 4)
+                        __stcg(reinterpret_cast<float4 *>(ring_cur + r * kD + c0 + j),
+                               make_float4(sp[j] + agg[j], sp[j + 1] + agg[j + 1], sp[j + 2] + agg[j + 2],
+                                           sp[j + 3] + agg[j + 3]));
+                    uint32_t u[32];
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) u[j] = __float_as_uint(sp[j]);
+                    tmem_st32(tb + lane_base + kTS + c0, u);
+                    // split S_p = c I + R into R_hi (slot SX) and R_lo (slot SD)
+                    float hi[32], lo[32];
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) {
+                        const float rr = sp[j] - ((c0 + j) == r ? c : 0.f);
+                        hi[j] = bf16_round(rr);
+                        lo[j] = rr - hi[j];
                     }
 #pragma unroll
-                    for (int j = 0; j < 32; ++j) sv[j] = __float_as_uint(sp[j]);
-                    tmem_st32(tb + lane_base + kTS + c0, sv);
+                    for (int j = 0; j < 32; j += 8) {
+                        store_row8(slot(kSX), r, c0 + j, hi + j);
+                        if (p.normalized) store_row8(slot(kSD), r, c0 + j, lo + j);
+                    }
+                    // segment-local D carry: the initial state's D for the first segment
 #pragma unroll
-                    for (int j = 0; j < 32; j += 8) write_split_row(slot(kSX), slot(kSD), r, sp + j, c, c0 + j, p.normalized);
+                    for (int j = 0; j < 32; ++j) u[j] = __float_as_uint(d0 ? d0[r * kD + c0 + j] : 0.f);
+                    tmem_st32(tb + lane_base + kTD + c0, u);
                 }
-                // segment-local D carry (the initial state's D for the first segment), e carry
-                const float *d0 = (sigma == 0 && p.init_De) ? p.init_De + (size_t)head * (kD * kD + kD) : nullptr;
-                for (int c0 = 0; c0 < kD; c0 += 32) {
-                    uint32_t dv[32];
-#pragma unroll
-                    for (int j = 0; j < 32; ++j) dv[j] = __float_as_uint(d0 ? d0[r * kD + c0 + j] : 0.f);
-                    tmem_st32(tb + lane_base + kTD + c0, dv);
-                }
-                ms->eloc[r] = d0 ? d0[kD * kD + r] : 0.f;
+                if (hf == 0) ms->eloc[r] = d0 ? d0[kD * kD + r] : 0.f;
                 tmem_st_wait();
             }
+            fence_async_smem();
             epi_sync();
-            if (r == 0 && item != p.inject_skip_item) {
+            if (et == 0 && item != p.inject_skip_item) {
                 __threadfence();
                 st_release(&flagS[head * 2 + (sigma & 1)], (unsigned)(sigma + 1));
             }
-            fence_async_smem();
 
             // ---- 2. sweep ----
             for (int j = 0; j < nt; ++j) {
                 const uint32_t tp = n_tiles & 1;
                 const uint8_t *qt = slot((j & 1) ? kQ1 : kQ0);
+                uint8_t *wlo = slot((j & 1) ? kQ0 : kQ1);  // W_lo staging (the other Q slot)
                 const int tok0 = (t0 + j) * kTile;
-                const float cs = ms->cshift[j & 1];
-                // W = L . A
+
+                // W = L . A (hi, lo)
                 bar_wait(ms, bEvA, tp, p);
                 tc_fence_after();
-                if (r == 0) tma_store_wait_read();  // staging tile of the previous output
+                if (et == 0) tma_store_wait_read();  // the previous output tile has left slot W
                 epi_sync();
-                for (int c0 = 0; c0 < kTile; c0 += 32) {
-                    uint32_t a[32];
-                    tmem_ld32(tb + lane_base + kTA + c0, a);
-                    tmem_ld_wait();
-                    float f[32];
+#pragma unroll 1
+                for (int c0 = cb0; c0 < cb0 + 64; c0 += 32) {
+                    if ((c0 >> 5) > qd) {  // block entirely above the diagonal
+                        store_zero32(slot(kW), r, c0);
+                        if (p.normalized) store_zero32(wlo, r, c0);
+                        continue;
+                    }
+                    float f[32], g[32];
+                    ld32(tb + lane_base + kTA + c0, f);
 #pragma unroll
-                    for (int jj = 0; jj < 32; ++jj) f[jj] = (c0 + jj <= r) ? __uint_as_float(a[jj]) : 0.f;
+                    for (int jj = 0; jj < 32; ++jj) {
+                        if (c0 + jj > r) f[jj] = 0.f;
+                        g[jj] = f[jj] - bf16_round(f[jj]);
+                    }
 #pragma unroll
-                    for (int jj = 0; jj < 32; jj += 8) store_row8(slot(kW), r, c0 + jj, f + jj);
+                    for (int jj = 0; jj < 32; jj += 8) {
+                        store_row8(slot(kW), r, c0 + jj, f + jj);
+                        if (p.normalized) store_row8(wlo, r, c0 + jj, g + jj);
+                    }
                 }
                 fence_async_smem();
                 epi_arrive(ms, bEpW);
-                // X_hi (and D_p -> bf16)
+
+                // X -> X_hi (slot SX), X_lo (slot W); D_p -> bf16 (slot SD); e carry
                 bar_wait(ms, bEvX, tp, p);
                 tc_fence_after();
-                for (int c0 = 0; c0 < kD; c0 += 32) {
-                    uint32_t a[32];
-                    tmem_ld32(tb + lane_base + kTX + c0, a);
-                    tmem_ld_wait();
-                    float f[32];
+                const float cs = ms->cshift[j & 1];
+                float den_part = 0.f, ecol[2] = {0.f, 0.f};
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    const int c0 = cb0 + 32 * h;
+                    float x[32];
+                    ld32(tb + lane_base + kTX + c0, x);
 #pragma unroll
                     for (int jj = 0; jj < 32; jj += 8) {
-                        float q8[8];
+                        float q8[8], lo8[8];
                         tile_row8(qt, r, c0 + jj, q8);
 #pragma unroll
-                        for (int u = 0; u < 8; ++u) f[jj + u] = __uint_as_float(a[jj + u]) + cs * q8[u];
-                        store_row8(slot(kSX), r, c0 + jj, f + jj);
+                        for (int u = 0; u < 8; ++u) {
+                            x[jj + u] += cs * q8[u];
+                            lo8[u] = x[jj + u] - bf16_round(x[jj + u]);
+                            if (p.normalized) den_part += q8[u] * ms->eloc[c0 + jj + u];
+                        }
+                        store_row8(slot(kSX), r, c0 + jj, x + jj);
+                        store_row8(slot(kW), r, c0 + jj, lo8);
                     }
+                    if (p.normalized) ecol[h] = warp_colsum32(x);  // column c0 + lane over this warp's rows
                 }
-                for (int c0 = 0; c0 < kD; c0 += 32) {
-                    uint32_t a[32];
-                    tmem_ld32(tb + lane_base + kTD + c0, a);
-                    tmem_ld_wait();
+#pragma unroll 1
+                for (int c0 = cb0; c0 < cb0 + 64; c0 += 32) {
                     float f[32];
-#pragma unroll
-                    for (int jj = 0; jj < 32; ++jj) f[jj] = __uint_as_float(a[jj]);
+                    ld32(tb + lane_base + kTD + c0, f);
 #pragma unroll
                     for (int jj = 0; jj < 32; jj += 8) store_row8(slot(kSD), r, c0 + jj, f + jj);
                 }
                 fence_async_smem();
                 epi_arrive(ms, bEpX);
-                // denominator (normalised): den_t = q_t . (e_p + sum_{j<=t} x_j), and e_p update
-                if (p.normalized) {
-                    float den = 0.f;
-                    for (int c0 = 0; c0 < kD; c0 += 32) {
-                        uint32_t a[32];
-                        tmem_ld32(tb + lane_base + kTX + c0, a);
-                        tmem_ld_wait();
-                        float x[32];
-#pragma unroll
-                        for (int jj = 0; jj < 32; jj += 8) {
-                            float q8[8];
-                            tile_row8(qt, r, c0 + jj, q8);
-#pragma unroll
-                            for (int u = 0; u < 8; ++u) x[jj + u] = __uint_as_float(a[jj + u]) + cs * q8[u];
-                        }
-                        // inclusive prefix over the 32 lanes of this warp, per column
-#pragma unroll
-                        for (int off = 1; off < 32; off <<= 1) {
-#pragma unroll
-                            for (int jj = 0; jj < 32; ++jj) {
-                                const float y = __shfl_up_sync(0xffffffffu, x[jj], off);
-                                if (lane >= off) x[jj] += y;
-                            }
-                        }
-                        if (lane == 31)
-#pragma unroll
-                            for (int jj = 0; jj < 32; ++jj) ms->tot[warp][jj] = x[jj];
-                        epi_sync();
-#pragma unroll
-                        for (int jj = 0; jj < 32; jj += 8) {
-                            float q8[8];
-                            tile_row8(qt, r, c0 + jj, q8);
-#pragma unroll
-                            for (int u = 0; u < 8; ++u) {
-                                const int cc = jj + u;
-                                float before = ms->eloc[c0 + cc];
-                                for (int w2 = 0; w2 < warp; ++w2) before += ms->tot[w2][cc];
-                                den += q8[u] * (before + x[cc]);
-                            }
-                        }
-                        epi_sync();
-                        if (r < 32) {
-                            const int cc = r;
-                            ms->eloc[c0 + cc] += ms->tot[0][cc] + ms->tot[1][cc] + ms->tot[2][cc] + ms->tot[3][cc];
-                        }
-                        epi_sync();
-                    }
-                    ms->den[r] = den;
-                }
-                // T = L . (Q X^T); next S split (hi) from the updated S carry
+
+                // T = L . (Q X^T) -> bf16 (slot W); denominators; next S split (hi)
                 bar_wait(ms, bEvT, tp, p);
                 tc_fence_after();
-                for (int c0 = 0; c0 < kTile; c0 += 32) {
-                    uint32_t a[32];
-                    tmem_ld32(tb + lane_base + kTA + c0, a);
-                    tmem_ld_wait();
+#pragma unroll 1
+                for (int c0 = cb0; c0 < cb0 + 64; c0 += 32) {
+                    if ((c0 >> 5) > qd) {
+                        store_zero32(slot(kW), r, c0);
+                        continue;
+                    }
                     float f[32];
+                    ld32(tb + lane_base + kTA + c0, f);
 #pragma unroll
-                    for (int jj = 0; jj < 32; ++jj) f[jj] = (c0 + jj <= r) ? __uint_as_float(a[jj]) : 0.f;
+                    for (int jj = 0; jj < 32; ++jj) {
+                        if (c0 + jj > r) f[jj] = 0.f;
+                        den_part += f[jj];
+                    }
 #pragma unroll
                     for (int jj = 0; jj < 32; jj += 8) store_row8(slot(kW), r, c0 + jj, f + jj);
                 }
-                if (j + 1 < nt) {
-                    uint32_t a[32];
-                    tmem_ld32(tb + lane_base + kTS + r - (r & 31), a);  // diagonal block containing column r
-                    tmem_ld_wait();
-                    float s = __uint_as_float(a[r & 31]);
-                    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-                    if (lane == 0) ms->red[warp] = s;
+                if (p.normalized) {  // den_t = both halves' partial sums
+                    if (hf == 1) ms->den[r] = den_part;
                     epi_sync();
-                    const float c = bf16_round((ms->red[0] + ms->red[1] + ms->red[2] + ms->red[3]) / kD);
-                    if (r == 0) ms->cshift[(j + 1) & 1] = c;
-                    for (int c0 = 0; c0 < kD; c0 += 32) {
-                        tmem_ld32(tb + lane_base + kTS + c0, a);
-                        tmem_ld_wait();
+                    if (hf == 0) ms->den[r] += den_part;
+                }
+                if (j + 1 < nt) {
+                    // shift of the next tile from the trace of the updated S
+                    float dg = 0.f;
+                    if ((qd >> 1) == hf) {
                         float f[32];
+                        ld32(tb + lane_base + kTS + 32 * qd, f);  // block holding the diagonal of these rows
 #pragma unroll
-                        for (int jj = 0; jj < 32; ++jj) f[jj] = __uint_as_float(a[jj]);
+                        for (int jj = 0; jj < 32; ++jj)
+                            if (jj == lane) dg = f[jj];
+                    }
+                    dg = warp_sum(dg);
+                    if (lane == 0) ms->red[warp] = dg;
+                    epi_sync();
+                    float tr = 0.f;
 #pragma unroll
-                        for (int jj = 0; jj < 32; jj += 8) write_split_row(slot(kSX), nullptr, r, f + jj, c, c0 + jj, false);
+                    for (int w = 0; w < kEpiWarps; ++w) tr += ms->red[w];
+                    const float c = bf16_round(tr / kD);
+                    if (et == 0) ms->cshift[(j + 1) & 1] = c;
+#pragma unroll 1
+                    for (int c0 = cb0; c0 < cb0 + 64; c0 += 32) {
+                        float f[32];
+                        ld32(tb + lane_base + kTS + c0, f);
+#pragma unroll
+                        for (int jj = 0; jj < 32; ++jj) f[jj] -= ((c0 + jj) == r ? c : 0.f);
+#pragma unroll
+                        for (int jj = 0; jj < 32; jj += 8) store_row8(slot(kSX), r, c0 + jj, f + jj);
                     }
                 }
                 fence_async_smem();
+                epi_sync();
                 epi_arrive(ms, bEpT);
-                // O: provisional (segments > 0) or final output; staging in slot W
+
+                // e carry += column sums of X (fixed order ((q0 + q1) + (q2 + q3)))
+                if (p.normalized) {
+                    const int ca = cb0 + lane, cbx = cb0 + 32 + lane;
+                    if (qd & 1) { ms->ebuf[qd >> 1][ca] = ecol[0]; ms->ebuf[qd >> 1][cbx] = ecol[1]; }
+                    epi_sync();
+                    if (!(qd & 1)) { ecol[0] += ms->ebuf[qd >> 1][ca]; ecol[1] += ms->ebuf[qd >> 1][cbx]; }
+                    epi_sync();
+                    if (qd == 2) { ms->ebuf[0][ca] = ecol[0]; ms->ebuf[0][cbx] = ecol[1]; }
+                    epi_sync();
+                    if (qd == 0) {
+                        ms->eloc[ca] += ecol[0] + ms->ebuf[0][ca];
+                        ms->eloc[cbx] += ecol[1] + ms->ebuf[0][cbx];
+                    }
+                }
+
+                // O (provisional for segments > 0, final for the first) -> slot W, TMA store
                 bar_wait(ms, bEvO, tp, p);
                 tc_fence_after();
                 {
                     const bool final_out = (sigma == 0);
                     const float den = p.normalized ? ms->den[r] : 1.f;
-                    const float scale = (final_out && p.normalized) ? 1.f / (den + p.eps) : 1.f;
-                    for (int c0 = 0; c0 < kD; c0 += 32) {
-                        uint32_t a[32];
-                        tmem_ld32(tb + lane_base + kTA + c0, a);
-                        tmem_ld_wait();
+                    const bool divide = final_out && p.normalized;
+#pragma unroll 1
+                    for (int c0 = cb0; c0 < cb0 + 64; c0 += 32) {
                         float f[32];
+                        ld32(tb + lane_base + kTX + c0, f);
+                        if (divide) {
 #pragma unroll
-                        for (int jj = 0; jj < 32; ++jj) {
-                            const float num = __uint_as_float(a[jj]);
-                            f[jj] = (final_out && p.normalized) ? num / (den + p.eps) : num;
+                            for (int jj = 0; jj < 32; ++jj) f[jj] = f[jj] / (den + p.eps);
                         }
-                        (void)scale;
 #pragma unroll
                         for (int jj = 0; jj < 32; jj += 8) store_row8(slot(kW), r, c0 + jj, f + jj);
                     }
-                    if (!final_out && p.normalized && tok0 + r < p.n) p.den_loc[(size_t)head * p.n + tok0 + r] = den;
+                    if (!final_out && p.normalized && hf == 0 && tok0 + r < p.n)
+                        p.den_loc[(size_t)head * p.n + tok0 + r] = den;
                 }
                 if (j + 1 < nt && p.normalized) {  // next S split (lo): D_p (bf16) in SD is dead now
                     const float c = ms->cshift[(j + 1) & 1];
-                    for (int c0 = 0; c0 < kD; c0 += 32) {
-                        uint32_t a[32];
-                        tmem_ld32(tb + lane_base + kTS + c0, a);
-                        tmem_ld_wait();
+#pragma unroll 1
+                    for (int c0 = cb0; c0 < cb0 + 64; c0 += 32) {
                         float f[32];
+                        ld32(tb + lane_base + kTS + c0, f);
 #pragma unroll
                         for (int jj = 0; jj < 32; ++jj) {
-                            const float rr = __uint_as_float(a[jj]) - ((c0 + jj) == r ? c : 0.f);
+                            const float rr = f[jj] - ((c0 + jj) == r ? c : 0.f);
                             f[jj] = rr - bf16_round(rr);
                         }
 #pragma unroll
@@ -580,56 +645,53 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 }
                 fence_async_smem();
                 epi_sync();
-                if (r == 0) {
+                if (et == 0) {
                     tma_store_3d(&tm_o, slot(kW), 0, tok0, head);
                     tma_store_3d(&tm_o, slot(kW) + kBlockBytes, 64, tok0, head);
                     tma_store_commit();
                 }
-                epi_arrive(ms, bEpO);
                 ++n_tiles;
             }
 
             // ---- 3. D chain and fix-up ----
             {
-                // inclusive D prefix of the previous segment
-                float *ring_prev = p.ring + ((size_t)head * 2 + ((sigma + 1) & 1)) * kRingFloats;
-                if (sigma > 0 && r == 0) chain_wait(&flagD[head * 2 + ((sigma - 1) & 1)], (unsigned)sigma, p, 2, item);
+                if (sigma > 0 && et == 0) chain_wait(&flagD[head * 2 + ((sigma - 1) & 1)], (unsigned)sigma, p, 2, item);
                 epi_sync();
                 const float *dprev = sigma > 0 ? ring_prev + kD * kD + r * kD : nullptr;
-                for (int c0 = 0; c0 < kD; c0 += 32) {
-                    uint32_t a[32];
-                    tmem_ld32(tb + lane_base + kTD + c0, a);
-                    tmem_ld_wait();
-                    float dp[32];
+#pragma unroll 1
+                for (int c0 = cb0; c0 < cb0 + 64; c0 += 32) {
+                    float f[32], dp[32];
+                    ld32(tb + lane_base + kTD + c0, f);
 #pragma unroll
                     for (int jj = 0; jj < 32; jj += 4) {
-                        float4 v4 = dprev ? __ldcg(reinterpret_cast<const float4 *>(dprev + c0 + jj))
-                                          : make_float4(0.f, 0.f, 0.f, 0.f);
+                        const float4 v4 = dprev ? __ldcg(reinterpret_cast<const float4 *>(dprev + c0 + jj))
+                                                : make_float4(0.f, 0.f, 0.f, 0.f);
                         dp[jj] = v4.x; dp[jj + 1] = v4.y; dp[jj + 2] = v4.z; dp[jj + 3] = v4.w;
                     }
 #pragma unroll
-                    for (int jj = 0; jj < 32; jj += 4) {
-                        float4 o4 = make_float4(dp[jj] + __uint_as_float(a[jj]), dp[jj + 1] + __uint_as_float(a[jj + 1]),
-                                                dp[jj + 2] + __uint_as_float(a[jj + 2]),
-                                                dp[jj + 3] + __uint_as_float(a[jj + 3]));
-                        __stcg(reinterpret_cast<float4 *>(ring_cur + kD * kD + r * kD + c0 + jj), o4);
-                    }
+                    for (int jj = 0; jj < 32; jj += 4)
+                        __stcg(reinterpret_cast<float4 *>(ring_cur + kD * kD + r * kD + c0 + jj),
+                               make_float4(dp[jj] + f[jj], dp[jj + 1] + f[jj + 1], dp[jj + 2] + f[jj + 2],
+                                           dp[jj + 3] + f[jj + 3]));
                     if (sigma > 0) {
 #pragma unroll
                         for (int jj = 0; jj < 32; jj += 8) store_row8(slot(kSD), r, c0 + jj, dp + jj);
                     }
                 }
-                const float eprev = sigma > 0 ? __ldcg(ring_prev + 2 * kD * kD + r) : 0.f;
-                __stcg(ring_cur + 2 * kD * kD + r, eprev + ms->eloc[r]);
+                float eprev = 0.f;
+                if (hf == 0) {
+                    eprev = sigma > 0 ? __ldcg(ring_prev + 2 * kD * kD + r) : 0.f;
+                    __stcg(ring_cur + 2 * kD * kD + r, eprev + ms->eloc[r]);
+                }
                 tc_fence_before();
                 epi_sync();
-                if (r == 0) {
+                if (et == 0) {
                     __threadfence();
                     st_release(&flagD[head * 2 + (sigma & 1)], (unsigned)(sigma + 1));
                 }
                 if (sigma > 0) {
-                    ms->eloc[r] = eprev;  // now e of the prefix, for the fix-up denominators
-                    if (r == 0) tma_store_wait_all();  // provisional outputs written before they are re-read
+                    if (hf == 0) ms->eloc[r] = eprev;  // now e of the prefix, for the fix-up denominators
+                    if (et == 0) tma_store_wait_all();  // provisional outputs written before they are re-read
                     fence_async_smem();
                     epi_sync();
                     epi_arrive(ms, bEpDF);
@@ -640,29 +702,35 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                         tc_fence_after();
                         float den = 1.f;
                         if (p.normalized) {
+                            // den_t = provisional denominator + q_t . e_prefix (two column halves)
                             float qe = 0.f;
-                            for (int c0 = 0; c0 < kD; c0 += 8) {
+#pragma unroll
+                            for (int c0 = cb0; c0 < cb0 + 64; c0 += 8) {
                                 float q8[8];
                                 tile_row8(qt, r, c0, q8);
 #pragma unroll
                                 for (int u = 0; u < 8; ++u) qe += q8[u] * ms->eloc[c0 + u];
                             }
-                            den = (tok0 + r < p.n ? p.den_loc[(size_t)head * p.n + tok0 + r] : 0.f) + qe;
+                            if (hf == 1) ms->den[r] = qe;
+                            epi_sync();
+                            if (hf == 0)
+                                ms->den[r] += qe + (tok0 + r < p.n ? p.den_loc[(size_t)head * p.n + tok0 + r] : 0.f);
+                            epi_sync();
+                            den = ms->den[r];
                         }
-                        if (r == 0) tma_store_wait_read();
+                        if (et == 0) tma_store_wait_read();
                         epi_sync();
-                        for (int c0 = 0; c0 < kD; c0 += 32) {
-                            uint32_t a[32];
-                            tmem_ld32(tb + lane_base + kTA + c0, a);
-                            tmem_ld_wait();
+#pragma unroll 1
+                        for (int c0 = cb0; c0 < cb0 + 64; c0 += 32) {
                             float f[32];
+                            ld32(tb + lane_base + kTA + c0, f);
 #pragma unroll
                             for (int jj = 0; jj < 32; jj += 8) {
                                 float o8[8];
                                 tile_row8(ot, r, c0 + jj, o8);
 #pragma unroll
                                 for (int u = 0; u < 8; ++u) {
-                                    const float num = o8[u] + __uint_as_float(a[jj + u]);
+                                    const float num = o8[u] + f[jj + u];
                                     f[jj + u] = p.normalized ? num / (den + p.eps) : num;
                                 }
                             }
@@ -671,7 +739,7 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                         }
                         fence_async_smem();
                         epi_sync();
-                        if (r == 0) {
+                        if (et == 0) {
                             tma_store_3d(&tm_o, slot(kW), 0, tok0, head);
                             tma_store_3d(&tm_o, slot(kW) + kBlockBytes, 64, tok0, head);
                             tma_store_commit();
@@ -684,9 +752,8 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
         }
         ++n_items;
         if (sigma > 0) ++n_dfix;
-        // every role has finished this item (stores of the outputs may still be in flight)
+        // every role has finished this item (output stores may still be in flight)
         if (!issuer && tid == 0) tma_store_wait_all();
-        __syncthreads();
     }
 
     tc_fence_before();
@@ -700,7 +767,7 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
 // initial-state carries D_0 = S_0 C_0 - G_0 and e_0 = S_0 m_0 - h_0 of each head (fp32)
 __global__ void __launch_bounds__(256) init_carry_kernel(const float *__restrict__ st, float *__restrict__ out) {
     const int hd = blockIdx.x;
-    const size_t L = 2 * (size_t)kD * kD + 2 * kD;
+    const size_t L = kStateFloats;
     const float *S = st + hd * L, *C = S + kD * kD, *m = C + kD * kD, *G = m + kD, *h = G + kD * kD;
     float *D = out + (size_t)hd * (kD * kD + kD), *e = D + kD * kD;
     for (int idx = threadIdx.x; idx < kD * kD + kD; idx += blockDim.x) {
