@@ -157,6 +157,37 @@ hla_status hla3_forward(const void *q, const void *k, const void *v, void *out, 
                         void *workspace, size_t workspace_bytes, hla_stream_t stream);
 
 /*
+ * hla2_forward_noalloc -- hla2_forward for callers that cannot allocate device
+ * memory (no counterpart in the paper: it only changes where scratch lives).
+ *
+ * Some callers cannot call cudaMalloc or hand over a workspace: code that runs
+ * under an allocator it does not own (a framework's caching pool, a memory
+ * budget that forbids extra reservations), or host code that links this
+ * library without any device-memory management of its own.  This entry point
+ * computes exactly what hla2_forward computes (same arguments, minus the
+ * workspace and state_out) and allocates nothing: its scratch is a 16 MiB
+ * array in device memory that belongs to the library.  Every GPU on which the
+ * library is used holds that array until the process exits.
+ *
+ * Scope: the fused path only (bf16 tokens, d = dv = 128, masked = 1,
+ * chunk = 128, no state_out, an sm_103 device); other arguments return
+ * HLA_ERR_UNSUPPORTED.  Sizes whose scratch exceeds 16 MiB (it grows with
+ * B*H, about 263 KiB per head, and with B*H*n*4 bytes when normalized) return
+ * HLA_ERR_WORKSPACE before anything is launched.
+ * Set-up: the first call on a device looks up the array's device address
+ * (cudaGetSymbolAddress) with that device current; make that first call before
+ * any stream capture.
+ * Sharing: all calls use the same array and it keeps the last call's contents
+ * (each call clears what must start at zero).  Calls whose kernels overlap on
+ * the GPU (different streams, or several host threads) race on it: order them
+ * on one stream.  Device-side wait timeouts are not reported for this entry
+ * point (hla_poll_error needs a workspace).
+ */
+hla_status hla2_forward_noalloc(const void *q, const void *k, const void *v, void *out, hla_dtype dt,
+                                int B, int H, int n, int d, int dv, int masked, int normalized, float eps,
+                                int chunk, const float *state_in, hla_stream_t stream);
+
+/*
  * hla_poll_error -- wait for `stream`, then report the device-side error flag
  * kept in `workspace` by the last forward call that used it: HLA_OK, or
  * HLA_ERR_TIMEOUT if a device-side wait gave up.  Clears the flag.

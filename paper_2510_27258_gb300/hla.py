@@ -22,7 +22,7 @@ HLA_F32, HLA_BF16 = 0, 1
 # every symbol include/hla.h declares
 EXPORTS = ("hla_status_string", "hla_last_error", "hla2_state_floats", "hla2_workspace_bytes", "hla2_forward",
            "hla2_forward_path", "hla2_step", "hla3_state_floats", "hla3_workspace_bytes", "hla3_forward",
-           "hla_poll_error")
+           "hla2_forward_noalloc", "hla_poll_error")
 
 _lib = None
 
@@ -56,6 +56,8 @@ def lib():
         for name in ("hla2_forward", "hla3_forward"):
             getattr(L, name).argtypes = [vp, vp, vp, vp, i, i, i, i, i, i, i, i, f, i, vp, vp, vp, sz, vp]
             getattr(L, name).restype = i
+        L.hla2_forward_noalloc.argtypes = [vp, vp, vp, vp, i, i, i, i, i, i, i, i, f, i, vp, vp]
+        L.hla2_forward_noalloc.restype = i
         L.hla2_forward_path.argtypes = [i, i, i, i, i, i, i, i, i, i, i, ctypes.POINTER(i)]
         L.hla2_forward_path.restype = i
         L.hla2_step.argtypes = [vp, vp, vp, vp, i, i, i, i, i, i, i, f, vp, vp]
@@ -150,6 +152,22 @@ def hla3_forward(q, k, v, out=None, *, masked=True, normalized=False, eps=1e-6, 
     """Third-order HLA forward (include/hla.h: hla3_forward). Returns ``out``."""
     return _forward("hla3_forward", hla3_workspace_bytes, q, k, v, out, masked, normalized, eps, chunk, state_in,
                     state_out, workspace, stream)
+
+
+def hla2_forward_noalloc(q, k, v, out=None, *, masked=True, normalized=False, eps=1e-6, chunk=128, state_in=None,
+                         stream=None):
+    """hla2_forward without a workspace, for callers that cannot allocate device
+    memory; the library's own 16 MiB device array serves as scratch (include/hla.h:
+    hla2_forward_noalloc).  Returns ``out``."""
+    B, H, n, d = q.shape
+    dv = v.shape[-1]
+    if out is None:
+        out = torch.empty((B, H, n, dv), dtype=q.dtype, device=q.device)
+    code = lib().hla2_forward_noalloc(_ptr(q), _ptr(k), _ptr(v), _ptr(out), _dtype_code(q), B, H, n, d, dv,
+                                      int(masked), int(normalized), float(eps), int(chunk), _ptr(state_in),
+                                      _stream(stream))
+    _check(code, "hla2_forward_noalloc")
+    return out
 
 
 def hla2_forward_path(B, H, n, d, dv, *, masked=True, normalized=False, chunk=128, dtype=torch.bfloat16,
