@@ -86,7 +86,11 @@ class ClockSampler:
             self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.gpu), "--query-gpu=" + self.FIELDS,
                                           "--format=csv,noheader,nounits", "-lms", "100"], stdout=self.fh,
                                          stderr=subprocess.DEVNULL)
-            time.sleep(0.3)
+            # nvidia-smi can take seconds to start; a timed region must not include that
+            t_end = time.time() + 20.0
+            while time.time() < t_end and os.path.getsize(self.path) == 0 and self.proc.poll() is None:
+                time.sleep(0.05)
+            time.sleep(0.2)
         except Exception:
             self.proc = None
 

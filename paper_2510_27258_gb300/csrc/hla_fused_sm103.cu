@@ -26,9 +26,11 @@
 // The exclusive scan across segments is a chained scan; Theorem 2 guarantees
 // the result equals the serial recurrence.
 //
-// Roles: warp 8 issues TMA loads and MMAs (one thread); warps 0-7 are the
-// epilogue (TMEM -> registers -> shared memory): warp w reads TMEM lanes
-// 32 (w % 4) .. +31 (one row each) and columns 64 (w / 4) .. +63.
+// Roles: warp 8 issues TMA loads and MMAs (one thread); warp 9 releases the
+// cross-SM prefix flags once the epilogue has written a prefix (the GPU-scope
+// fence this takes stays off the epilogue's path); warps 0-7 are the epilogue
+// (TMEM -> registers -> shared memory): warp w reads TMEM lanes 32 (w % 4) ..
+// +31 (one row each) and columns 64 (w / 4) .. +63.
 //
 // Precision: tokens are bf16, every product accumulates in fp32 (TMEM).  The S
 // operand is split as S = c I + R (c = bf16(trace S / d)) with c q_t added in
@@ -52,7 +54,8 @@ constexpr int kTile = 128;        // tokens per tile (MMA M)
 constexpr int kEpiWarps = 8;      // 2 per TMEM lane quadrant
 constexpr int kEpiThreads = kEpiWarps * 32;
 constexpr int kIssuerWarp = kEpiWarps;
-constexpr int kThreads = kEpiThreads + 32;
+constexpr int kPubWarp = kEpiWarps + 1;  // releases the cross-SM prefix flags
+constexpr int kThreads = kEpiThreads + 64;
 constexpr int kSlots = 7;
 constexpr uint32_t kSmemTiles = kSlots * kTileBytes;
 constexpr uint32_t kMiscBytes = 3072;
@@ -66,11 +69,14 @@ constexpr uint32_t kTS = 0, kTD = 128, kTA = 256, kTX = 384;
 
 // barrier indices
 enum Bar {
-    bLd0 = 0,  // + slot index for the four input slots (Q0, Q1, K, V)
-    bPre = 4,  // pre-pass MMA done (per K tile)
-    bEvP = 5, bEvA = 6, bEvX = 7, bEvT = 8, bEvO = 9, bEvF = 10,
-    bEpW = 11, bEpX = 12, bEpT = 13, bEpF = 14, bEpDF = 15,
-    kNumBars = 16
+    bLd0 = 0,  // + slot index for the TMA-loaded slots (Q0, Q1, K, V, W)
+    bPre = 5,  // pre-pass MMA done (per K tile)
+    bEvP = 6, bEvA = 7, bEvX = 8, bEvS = 9, bEvT = 10, bEvO = 11, bEvD = 12,
+    bEvF = 13,  // + TMEM region of the fix-up tile (0: A, 1: X)
+    bEpW = 15, bEpX = 16, bEpT = 17,
+    bEpF = 18,  // + TMEM region of the fix-up tile
+    bEpDF = 20,
+    kNumBars = 21
 };
 constexpr int kFirstEpiBar = bEpW;
 
@@ -94,7 +100,7 @@ struct Params {
     float eps;
     const float *state_in;  // S_0 of each head (paper tuple), or null
     const float *init_De;   // D_0 (d*dv) and e_0 (d) of each head, or null
-    float *ring;            // [BH][2][d*d + d*dv + d]
+    float *ring;            // [BH][2][d*d + d*dv + d]; S and D parts thread-major (see ring4)
     unsigned *flags;        // [2][BH][2]: S flags then D flags
     unsigned *ticket;
     float *den_loc;         // [BH][n] provisional denominators (normalised, segments > 0)
@@ -104,6 +110,12 @@ struct Params {
 };
 
 constexpr int kRingFloats = kD * kD + kD * kD + kD;
+
+// The S and D prefixes in the ring are stored in the order the epilogue holds
+// them: float4 c (columns cb0 + 4c .. +3 of row r) of epilogue thread et at
+// float4 index c * 256 + et, so that every warp access is 512 contiguous bytes.
+// Writer and reader (the next segment of the head) use the same thread mapping.
+__device__ __forceinline__ int ring4(int c, int et) { return c * kEpiThreads + et; }
 // floats of one head's state tuple [S | C | m | G | h] with d = dv = kD
 constexpr int kStateFloats = kD * kD + 2 * kD * kD + 2 * kD;
 // budget of an intra-CTA mbarrier wait (TMA or MMA completion, epilogue hand-off)
@@ -120,6 +132,16 @@ __device__ __forceinline__ unsigned ld_acquire(const unsigned *p) {
 }
 // named barrier of the epilogue warps
 __device__ __forceinline__ void epi_sync() { asm volatile("bar.sync 1, 256;" ::: "memory"); }
+// Hand-offs epilogue -> publisher warp (named barriers 2 and 3, 288 threads): the
+// epilogue arrives after writing a prefix to the ring and goes on; the publisher
+// waits, then makes the ring writes visible GPU-wide and releases the flag.
+constexpr int kBarPubS = 2, kBarPubD = 3;
+__device__ __forceinline__ void pub_arrive(int id) {
+    asm volatile("bar.arrive %0, %1;" ::"r"(id), "r"(kEpiThreads + 32) : "memory");
+}
+__device__ __forceinline__ void pub_wait(int id) {
+    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(kEpiThreads + 32) : "memory");
+}
 
 __device__ __forceinline__ void set_error(WsHeader *err, unsigned where, unsigned detail) {
     if (atomicCAS(&err->error, 0u, (unsigned)kDevTimeout) == 0u) {
@@ -187,12 +209,56 @@ __device__ __forceinline__ void store_zero32(uint8_t *tile, int r, int c0) {
 
 __device__ __forceinline__ float bf16_round(float x) { return __bfloat162float(__float2bfloat16_rn(x)); }
 
+// row r, columns c0..c0+31 of L . A -> W_hi (tile w) and, if lo, W_lo (tile wl)
+__device__ __forceinline__ void emit_w(uint8_t *w, uint8_t *wl, int r, int c0, float (&f)[32], bool lo) {
+#pragma unroll
+    for (int jj = 0; jj < 32; jj += 8) {
+        float h8[8], l8[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+            h8[u] = (c0 + jj + u > r) ? 0.f : f[jj + u];
+            l8[u] = h8[u] - bf16_round(h8[u]);
+        }
+        store_row8(w, r, c0 + jj, h8);
+        if (lo) store_row8(wl, r, c0 + jj, l8);
+    }
+}
+
+// row r, columns c0..c0+31 of L . T -> bf16 tile; returns the row sum of the masked values
+__device__ __forceinline__ float emit_t(uint8_t *t, int r, int c0, float (&f)[32]) {
+    float sum = 0.f;
+#pragma unroll
+    for (int jj = 0; jj < 32; jj += 8) {
+        float h8[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+            h8[u] = (c0 + jj + u > r) ? 0.f : f[jj + u];
+            sum += h8[u];
+        }
+        store_row8(t, r, c0 + jj, h8);
+    }
+    return sum;
+}
+
 __device__ __forceinline__ void ld32(uint32_t addr, float (&f)[32]) {
     uint32_t a[32];
     tmem_ld32(addr, a);
     tmem_ld_wait();
 #pragma unroll
     for (int j = 0; j < 32; ++j) f[j] = __uint_as_float(a[j]);
+}
+
+// two 32-column TMEM loads with one wait
+__device__ __forceinline__ void ld64(uint32_t addr, float (&f0)[32], float (&f1)[32]) {
+    uint32_t a[32], b[32];
+    tmem_ld32(addr, a);
+    tmem_ld32(addr + 32, b);
+    tmem_ld_wait();
+#pragma unroll
+    for (int j = 0; j < 32; ++j) {
+        f0[j] = __uint_as_float(a[j]);
+        f1[j] = __uint_as_float(b[j]);
+    }
 }
 
 // Column sums of v over the 32 lanes of a warp: returns, in lane l, the sum of
@@ -218,6 +284,30 @@ __device__ __forceinline__ float warp_sum(float x) {
     return x;
 }
 
+// High word of every shared-memory descriptor used here: stride between 8-row
+// groups 1024 B, tcgen05 descriptor version, 128-byte swizzle.
+constexpr uint32_t kDescHi = (1024u >> 4) | (1u << 14) | (2u << 29);
+// low-word leading-byte-offset fields of K-major (unused, 16 B) and MN-major
+// (stride between 64-element blocks) operands
+constexpr uint32_t kLboK = 1u << 16, kLboMN = (kBlockBytes >> 4) << 16;
+
+// One 128 x 128 x 128 product D (+)= A B as eight K = 16 steps, from the low
+// descriptor words of the two operand tiles (address >> 4 | LBO field).  The
+// step offsets are compile-time constants, so each MMA costs one add per operand.
+template <bool A_MN, bool B_MN>
+__device__ __forceinline__ void mma128(uint32_t d_tmem, uint32_t a_lo, uint32_t b_lo, uint32_t accumulate) {
+    constexpr uint32_t id = idesc_bf16(128, 128, A_MN, B_MN);
+#pragma unroll
+    for (int kk = 0; kk < 8; ++kk) {
+        // K-major: the second 64-element column block is 16 KiB on, 32 B per K step within a block;
+        // MN-major: 8 K rows of 128 B (2 KiB with the swizzle atom) per K step
+        const uint32_t ka = A_MN ? kk * 128u : (kk >> 2) * (kBlockBytes >> 4) + (kk & 3) * 2u;
+        const uint32_t kb = B_MN ? kk * 128u : (kk >> 2) * (kBlockBytes >> 4) + (kk & 3) * 2u;
+        umma_bf16(d_tmem, (static_cast<uint64_t>(kDescHi) << 32) | (a_lo + ka),
+                  (static_cast<uint64_t>(kDescHi) << 32) | (b_lo + kb), id, kk > 0 ? 1u : accumulate);
+    }
+}
+
 // ---------------------------------------------------------------------------
 // the kernel
 // ---------------------------------------------------------------------------
@@ -229,7 +319,7 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
     auto slot = [&](int s) { return smem + s * kTileBytes; };
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const bool issuer = (warp == kIssuerWarp);
+    const bool issuer = (warp == kIssuerWarp), publisher = (warp == kPubWarp);
 
     // the tile layout needs 1 KiB alignment of the dynamic shared memory
     if (smem_u32(smem) & 1023u) {
@@ -254,22 +344,25 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
     const uint32_t tb = ms->tmem_base;
 
     // per-CTA event counters (identical sequences on both sides)
-    uint32_t n_tiles = 0, n_items = 0, n_fix = 0, n_pre = 0, n_dfix = 0;
-    uint32_t ld_cnt[4] = {0, 0, 0, 0};
+    uint32_t n_tiles = 0, n_items = 0, n_pre = 0, n_dfix = 0;
+    uint32_t ld_par = 0;  // bit s: parity of the next load completion of slot s
+    uint32_t fx_par = 0;  // bit g: parity of the next fix-up hand-off in TMEM region g
 
-    constexpr uint32_t idA = idesc_bf16(128, 128, 0, 0);   // Q K^T, Q R, Q X^T: both K-major
-    constexpr uint32_t idKmn = idesc_bf16(128, 128, 0, 1); // W K, T V, Q D: B MN-major
-    constexpr uint32_t idMM = idesc_bf16(128, 128, 1, 1);  // K^T K, X^T V: both MN-major
-    const uint32_t tileQ[2] = {smem_u32(slot(kQ0)), smem_u32(slot(kQ1))};
-    const uint32_t sK = smem_u32(slot(kK)), sV = smem_u32(slot(kV)), sW = smem_u32(slot(kW));
-    const uint32_t sSX = smem_u32(slot(kSX)), sSD = smem_u32(slot(kSD));
+    // descriptor low words of the slots, as K-major (lk) and MN-major (lm) operands
+    const uint32_t sb4 = smem_u32(smem) >> 4;
+    auto lk = [&](int s) { return sb4 + (uint32_t)s * (kTileBytes >> 4) + kLboK; };
+    auto lm = [&](int s) { return sb4 + (uint32_t)s * (kTileBytes >> 4) + kLboMN; };
 
     auto load_tile = [&](int s, const CUtensorMap *map, int head, int tok0) {
         mbar_arrive_expect_tx(&ms->bar[bLd0 + s], kTileBytes);
         tma_load_3d(slot(s), map, &ms->bar[bLd0 + s], 0, tok0, head);
         tma_load_3d(slot(s) + kBlockBytes, map, &ms->bar[bLd0 + s], 64, tok0, head);
     };
-    auto wait_ld = [&](int s) { return bar_wait(ms, bLd0 + s, (ld_cnt[s]++) & 1, p); };
+    auto wait_ld = [&](int s) {
+        const uint32_t par = (ld_par >> s) & 1u;
+        ld_par ^= 1u << s;
+        return bar_wait(ms, bLd0 + s, par, p);
+    };
 
     while (true) {
         if (tid == 0) ms->item = (int)atomicAdd(p.ticket, 1u);
@@ -286,81 +379,71 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
         if (issuer) {
             if (lane == 0) {
                 // ---- 1. pre-pass: S aggregate of the segment into TMEM cols kTX ----
-                const int ps[2] = {kK, kV};
-                load_tile(ps[0], &tm_k, head, (t0 + 0) * kTile);
-                if (nt > 1) load_tile(ps[1], &tm_k, head, (t0 + 1) * kTile);
+                // K tiles go to four idle slots (K, V, W, Q1); tile 0 stays in K for the sweep
+                const int ps[4] = {kK, kV, kW, kQ1};
+                load_tile(kQ0, &tm_q, head, t0 * kTile);
+                for (int j = 0; j < nt && j < 4; ++j) load_tile(ps[j], &tm_k, head, (t0 + j) * kTile);
                 for (int j = 0; j < nt; ++j) {
-                    const int s = ps[j & 1];
+                    const int s = ps[j & 3];
                     if (!wait_ld(s)) break;
                     tc_fence_after();
-                    for (int kk = 0; kk < 8; ++kk)
-                        umma_bf16(tb + kTX, desc_mnmajor(smem_u32(slot(s)), kk), desc_mnmajor(smem_u32(slot(s)), kk),
-                                  idMM, (j > 0 || kk > 0) ? 1u : 0u);
-                    umma_commit(&ms->bar[bPre]);
-                    if (!bar_wait(ms, bPre, (n_pre++) & 1, p)) break;
-                    if (j + 2 < nt) load_tile(s, &tm_k, head, (t0 + j + 2) * kTile);
+                    mma128<true, true>(tb + kTX, lm(s), lm(s), j > 0 ? 1u : 0u);  // S_agg += K^T K
+                    if (j + 4 < nt) {  // long segment: reuse this slot once its MMA is done
+                        umma_commit(&ms->bar[bPre]);
+                        if (!bar_wait(ms, bPre, (n_pre++) & 1, p)) break;
+                        load_tile(s, &tm_k, head, (t0 + j + 4) * kTile);
+                    }
                 }
                 umma_commit(&ms->bar[bEvP]);
-                // first tile's inputs and its A = Q K^T
-                load_tile(kQ0, &tm_q, head, t0 * kTile);
-                load_tile(kK, &tm_k, head, t0 * kTile);
+                if (!bar_wait(ms, bEvP, ip, p)) break;  // the pre-pass slots are free again
+                // first tile's inputs (K tile 0 is still in slot K unless the segment is long)
+                if (nt > 4) load_tile(kK, &tm_k, head, t0 * kTile);
                 load_tile(kV, &tm_v, head, t0 * kTile);
-                if (wait_ld(kQ0) && wait_ld(kK)) {
+                if (wait_ld(kQ0) && (nt <= 4 || wait_ld(kK))) {
                     tc_fence_after();
-                    for (int kk = 0; kk < 8; ++kk)
-                        umma_bf16(tb + kTA, desc_kmajor(tileQ[0], kk), desc_kmajor(sK, kk), idA, kk > 0);
+                    mma128<false, false>(tb + kTA, lk(kQ0), lk(kK), 0u);  // A = Q K^T
                     umma_commit(&ms->bar[bEvA]);
                 }
 
                 // ---- 2. sweep ----
                 for (int j = 0; j < nt && !ms->abort_flag; ++j) {
                     const uint32_t tp = n_tiles & 1;
-                    const uint32_t sQ = tileQ[j & 1], sQo = tileQ[(j + 1) & 1];
+                    const int qs = (j & 1) ? kQ1 : kQ0, qo = (j & 1) ? kQ0 : kQ1;
                     if (!bar_wait(ms, bEpW, tp, p)) break;  // W (hi, lo), S split ready; TMEM X free
                     tc_fence_after();
-                    for (int kk = 0; kk < 8; ++kk)  // X = W_hi K
-                        umma_bf16(tb + kTX, desc_kmajor(sW, kk), desc_mnmajor(sK, kk), idKmn, kk > 0);
-                    if (p.normalized)
-                        for (int kk = 0; kk < 8; ++kk)  // X += W_lo K  (W_lo staged in the other Q slot)
-                            umma_bf16(tb + kTX, desc_kmajor(sQo, kk), desc_mnmajor(sK, kk), idKmn, 1u);
-                    for (int kk = 0; kk < 8; ++kk)  // X += Q R_hi
-                        umma_bf16(tb + kTX, desc_kmajor(sQ, kk), desc_kmajor(sSX, kk), idA, 1u);
-                    if (p.normalized)
-                        for (int kk = 0; kk < 8; ++kk)  // X += Q R_lo
-                            umma_bf16(tb + kTX, desc_kmajor(sQ, kk), desc_kmajor(sSD, kk), idA, 1u);
-                    for (int kk = 0; kk < 8; ++kk)  // S += K^T K
-                        umma_bf16(tb + kTS, desc_mnmajor(sK, kk), desc_mnmajor(sK, kk), idMM, 1u);
+                    mma128<false, true>(tb + kTX, lk(kW), lm(kK), 0u);        // X = W_hi K
+                    if (p.normalized) mma128<false, true>(tb + kTX, lk(qo), lm(kK), 1u);  // += W_lo K
+                    mma128<false, false>(tb + kTX, lk(qs), lk(kSX), 1u);      // += Q R_hi
+                    if (p.normalized) mma128<false, false>(tb + kTX, lk(qs), lk(kSD), 1u);  // += Q R_lo
                     umma_commit(&ms->bar[bEvX]);
-                    if (!bar_wait(ms, bEvX, tp, p)) break;
+                    mma128<true, true>(tb + kTS, lm(kK), lm(kK), 1u);         // S += K^T K
+                    umma_commit(&ms->bar[bEvS]);
+                    if (!bar_wait(ms, bEvS, tp, p)) break;  // X and S MMAs done: K and W_lo slots free
                     if (j + 1 < nt) {
                         load_tile(kK, &tm_k, head, (t0 + j + 1) * kTile);
-                        load_tile((j & 1) ? kQ0 : kQ1, &tm_q, head, (t0 + j + 1) * kTile);
+                        load_tile(qo, &tm_q, head, (t0 + j + 1) * kTile);
                     }
                     if (!bar_wait(ms, bEpX, tp, p)) break;  // X_hi, X_lo and D_hi ready
                     if (!wait_ld(kV)) break;
                     tc_fence_after();
-                    for (int kk = 0; kk < 8; ++kk)  // T = Q X_hi^T
-                        umma_bf16(tb + kTA, desc_kmajor(sQ, kk), desc_kmajor(sSX, kk), idA, kk > 0);
-                    for (int kk = 0; kk < 8; ++kk)  // T += Q X_lo^T  (X_lo staged in slot W)
-                        umma_bf16(tb + kTA, desc_kmajor(sQ, kk), desc_kmajor(sW, kk), idA, 1u);
-                    for (int kk = 0; kk < 8; ++kk)  // D += X^T V
-                        umma_bf16(tb + kTD, desc_mnmajor(sSX, kk), desc_mnmajor(sV, kk), idMM, 1u);
+                    mma128<false, false>(tb + kTA, lk(qs), lk(kSX), 0u);      // T = Q X_hi^T
+                    mma128<false, false>(tb + kTA, lk(qs), lk(kW), 1u);       // += Q X_lo^T (X_lo in W)
                     umma_commit(&ms->bar[bEvT]);
-                    if (!bar_wait(ms, bEpT, tp, p)) break;  // T ready; TMEM A free
+                    // T (bf16) in W and D_p (bf16) in SD; TMEM A free; the epilogue has read D_p from TMEM
+                    if (!bar_wait(ms, bEpT, tp, p)) break;
                     tc_fence_after();
-                    for (int kk = 0; kk < 8; ++kk)  // O = Q D_p
-                        umma_bf16(tb + kTX, desc_kmajor(sQ, kk), desc_mnmajor(sSD, kk), idKmn, kk > 0);
-                    for (int kk = 0; kk < 8; ++kk)  // O += T V
-                        umma_bf16(tb + kTX, desc_kmajor(sW, kk), desc_mnmajor(sV, kk), idKmn, 1u);
+                    mma128<false, true>(tb + kTX, lk(qs), lm(kSD), 0u);       // O = Q D_p
+                    mma128<false, true>(tb + kTX, lk(kW), lm(kV), 1u);        // += T V
                     umma_commit(&ms->bar[bEvO]);
+                    mma128<true, true>(tb + kTD, lm(kSX), lm(kV), 1u);        // D += X^T V
+                    umma_commit(&ms->bar[bEvD]);
                     if (j + 1 < nt) {  // next tile's A = Q K^T overlaps this tile's output epilogue
-                        if (!wait_ld((j & 1) ? kQ0 : kQ1) || !wait_ld(kK)) break;
+                        if (!wait_ld(qo) || !wait_ld(kK)) break;
                         tc_fence_after();
-                        for (int kk = 0; kk < 8; ++kk)
-                            umma_bf16(tb + kTA, desc_kmajor(sQo, kk), desc_kmajor(sK, kk), idA, kk > 0);
+                        mma128<false, false>(tb + kTA, lk(qo), lk(kK), 0u);
                         umma_commit(&ms->bar[bEvA]);
                     }
-                    if (!bar_wait(ms, bEvO, tp, p)) break;
+                    if (!bar_wait(ms, bEvD, tp, p)) break;  // D += X^T V (the last reader of V) done
                     if (j + 1 < nt) load_tile(kV, &tm_v, head, (t0 + j + 1) * kTile);
                     ++n_tiles;
                 }
@@ -368,25 +451,48 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 // ---- 3. fix-up of segments > 0 ----
                 if (sigma > 0 && !ms->abort_flag) {
                     if (bar_wait(ms, bEpDF, n_dfix & 1, p)) {  // D prefix (bf16) in SD; outputs written
-                        load_tile(kQ0, &tm_q, head, t0 * kTile);
-                        load_tile(kK, &tm_o, head, t0 * kTile);
+                        // tile j: Q in slot Q(j&1), provisional output in slot K/V (j&1), F in TMEM A/X (j&1)
+                        auto load_fix = [&](int j) {
+                            load_tile((j & 1) ? kQ1 : kQ0, &tm_q, head, (t0 + j) * kTile);
+                            load_tile((j & 1) ? kV : kK, &tm_o, head, (t0 + j) * kTile);
+                        };
+                        load_fix(0);
+                        if (nt > 1) load_fix(1);
                         for (int j = 0; j < nt; ++j) {
-                            const int qs = (j & 1) ? kQ1 : kQ0, os = (j & 1) ? kV : kK;
-                            if (!wait_ld(qs) || !wait_ld(os)) break;
+                            if (!wait_ld((j & 1) ? kQ1 : kQ0) || !wait_ld((j & 1) ? kV : kK)) break;
                             tc_fence_after();
-                            for (int kk = 0; kk < 8; ++kk)  // F = Q D_prefix
-                                umma_bf16(tb + kTA, desc_kmajor(tileQ[j & 1], kk), desc_mnmajor(sSD, kk), idKmn,
-                                          kk > 0);
-                            umma_commit(&ms->bar[bEvF]);
-                            if (j + 1 < nt) {
-                                // the other pair of slots was released by the previous fix-up epilogue
-                                load_tile((j & 1) ? kQ0 : kQ1, &tm_q, head, (t0 + j + 1) * kTile);
-                                load_tile((j & 1) ? kK : kV, &tm_o, head, (t0 + j + 1) * kTile);
+                            mma128<false, true>(tb + ((j & 1) ? kTX : kTA), lk((j & 1) ? kQ1 : kQ0), lm(kSD),
+                                                0u);  // F = Q D_prefix
+                            umma_commit(&ms->bar[bEvF + (j & 1)]);
+                            if (j >= 1) {  // tile j-1 done: its slots and TMEM region take tile j+1
+                                const int g = (j - 1) & 1;
+                                const bool ok = bar_wait(ms, bEpF + g, (fx_par >> g) & 1u, p);
+                                fx_par ^= 1u << g;
+                                if (!ok) break;
+                                if (j + 1 < nt) load_fix(j + 1);
                             }
-                            if (!bar_wait(ms, bEpF, (n_fix++) & 1, p)) break;
+                        }
+                        {  // the last tile
+                            const int g = (nt - 1) & 1;
+                            bar_wait(ms, bEpF + g, (fx_par >> g) & 1u, p);
+                            fx_par ^= 1u << g;
                         }
                     }
                 }
+            }
+            __syncwarp();
+        } else if (publisher) {
+            // one S prefix and one D prefix per item (the epilogue arrives once at each, on every path)
+            unsigned *flagS = p.flags, *flagD = p.flags + 2 * p.BH;
+            pub_wait(kBarPubS);
+            if (lane == 0 && item != p.inject_skip_item) {
+                __threadfence();
+                st_release(&flagS[head * 2 + (sigma & 1)], (unsigned)(sigma + 1));
+            }
+            pub_wait(kBarPubD);
+            if (lane == 0) {
+                __threadfence();
+                st_release(&flagD[head * 2 + (sigma & 1)], (unsigned)(sigma + 1));
             }
             __syncwarp();
         } else {
@@ -398,7 +504,7 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
             const uint32_t lane_base = (uint32_t)(32 * qd) << 16;
             const float *ring_prev = p.ring + ((size_t)head * 2 + ((sigma + 1) & 1)) * kRingFloats;
             float *ring_cur = p.ring + ((size_t)head * 2 + (sigma & 1)) * kRingFloats;
-            unsigned *flagS = p.flags, *flagD = p.flags + 2 * p.BH;
+            const unsigned *flagS = p.flags, *flagD = p.flags + 2 * p.BH;
 
             // ---- 1. S chain: carry-in S of the segment, publish the inclusive prefix ----
             bar_wait(ms, bEvP, ip, p);
@@ -406,10 +512,23 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
             if (sigma > 0 && et == 0) chain_wait(&flagS[head * 2 + ((sigma - 1) & 1)], (unsigned)sigma, p, 1, item);
             epi_sync();
             {
-                const float *sprev = nullptr;
-                if (sigma > 0) sprev = ring_prev + r * kD;
-                else if (p.state_in) sprev = p.state_in + (size_t)head * kStateFloats + r * kD;
-                float s = (sprev && (r >> 6) == hf) ? __ldcg(sprev + r) : 0.f;  // diagonal -> trace
+                // carry-in S: the previous segment's prefix (ring) or the initial state (row-major)
+                const float4 *ringS = sigma > 0 ? reinterpret_cast<const float4 *>(ring_prev) : nullptr;
+                const float4 *st_row = (sigma == 0 && p.state_in)
+                    ? reinterpret_cast<const float4 *>(p.state_in + (size_t)head * kStateFloats + r * kD + cb0)
+                    : nullptr;
+                auto s_in = [&](int c) {  // float4 c of this thread's 64 columns
+                    if (ringS) return __ldcg(ringS + ring4(c, et));
+                    if (st_row) return __ldcg(st_row + c);
+                    return make_float4(0.f, 0.f, 0.f, 0.f);
+                };
+                // diagonal element (from the thread whose columns contain r) -> trace -> shift
+                float s = 0.f;
+                if ((r >> 6) == hf) {
+                    const float4 v4 = s_in((r - cb0) >> 2);
+                    const int cc = r & 3;
+                    s = cc == 0 ? v4.x : cc == 1 ? v4.y : cc == 2 ? v4.z : v4.w;
+                }
                 s = warp_sum(s);
                 if (lane == 0) ms->red[warp] = s;
                 epi_sync();
@@ -420,51 +539,54 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 if (et == 0) ms->cshift[0] = c;
                 const float *d0 = (sigma == 0 && p.init_De) ? p.init_De + (size_t)head * (kD * kD + kD) : nullptr;
 #pragma unroll 1
-                for (int c0 = cb0; c0 < cb0 + 64; c0 += 32) {
-                    float agg[32], sp[32];
-                    ld32(tb + lane_base + kTX + c0, agg);
+                for (int h = 0; h < 2; ++h) {
+                    const int c0 = cb0 + 32 * h;
+                    float sp[32], agg[32];
 #pragma unroll
                     for (int j = 0; j < 32; j += 4) {
-                        const float4 v4 = sprev ? __ldcg(reinterpret_cast<const float4 *>(sprev + c0 + j))
-                                                : make_float4(0.f, 0.f, 0.f, 0.f);
+                        const float4 v4 = s_in(8 * h + j / 4);
                         sp[j] = v4.x; sp[j + 1] = v4.y; sp[j + 2] = v4.z; sp[j + 3] = v4.w;
                     }
+                    ld32(tb + lane_base + kTX + c0, agg);
+                    // inclusive S prefix of this segment -> ring
 #pragma unroll
                     for (int j = 0; j < 32; j += 4)
-                        __stcg(reinterpret_cast<float4 *>(ring_cur + r * kD + c0 + j),
+                        __stcg(reinterpret_cast<float4 *>(ring_cur) + ring4(8 * h + j / 4, et),
                                make_float4(sp[j] + agg[j], sp[j + 1] + agg[j + 1], sp[j + 2] + agg[j + 2],
                                            sp[j + 3] + agg[j + 3]));
+                    // S carry in TMEM
                     uint32_t u[32];
 #pragma unroll
                     for (int j = 0; j < 32; ++j) u[j] = __float_as_uint(sp[j]);
                     tmem_st32(tb + lane_base + kTS + c0, u);
                     // split S_p = c I + R into R_hi (slot SX) and R_lo (slot SD)
-                    float hi[32], lo[32];
-#pragma unroll
-                    for (int j = 0; j < 32; ++j) {
-                        const float rr = sp[j] - ((c0 + j) == r ? c : 0.f);
-                        hi[j] = bf16_round(rr);
-                        lo[j] = rr - hi[j];
-                    }
 #pragma unroll
                     for (int j = 0; j < 32; j += 8) {
-                        store_row8(slot(kSX), r, c0 + j, hi + j);
-                        if (p.normalized) store_row8(slot(kSD), r, c0 + j, lo + j);
+                        float hi[8], lo[8];
+#pragma unroll
+                        for (int t = 0; t < 8; ++t) {
+                            const float rr = sp[j + t] - ((c0 + j + t) == r ? c : 0.f);
+                            hi[t] = bf16_round(rr);
+                            lo[t] = rr - hi[t];
+                        }
+                        store_row8(slot(kSX), r, c0 + j, hi);
+                        if (p.normalized) store_row8(slot(kSD), r, c0 + j, lo);
                     }
                     // segment-local D carry: the initial state's D for the first segment
 #pragma unroll
-                    for (int j = 0; j < 32; ++j) u[j] = __float_as_uint(d0 ? d0[r * kD + c0 + j] : 0.f);
+                    for (int j = 0; j < 32; j += 4) {
+                        const float4 v4 = d0 ? __ldcg(reinterpret_cast<const float4 *>(d0 + r * kD + c0 + j))
+                                             : make_float4(0.f, 0.f, 0.f, 0.f);
+                        u[j] = __float_as_uint(v4.x); u[j + 1] = __float_as_uint(v4.y);
+                        u[j + 2] = __float_as_uint(v4.z); u[j + 3] = __float_as_uint(v4.w);
+                    }
                     tmem_st32(tb + lane_base + kTD + c0, u);
                 }
                 if (hf == 0) ms->eloc[r] = d0 ? d0[kD * kD + r] : 0.f;
                 tmem_st_wait();
             }
             fence_async_smem();
-            epi_sync();
-            if (et == 0 && item != p.inject_skip_item) {
-                __threadfence();
-                st_release(&flagS[head * 2 + (sigma & 1)], (unsigned)(sigma + 1));
-            }
+            pub_arrive(kBarPubS);  // S prefix in the ring
 
             // ---- 2. sweep ----
             for (int j = 0; j < nt; ++j) {
@@ -478,39 +600,43 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 tc_fence_after();
                 if (et == 0) tma_store_wait_read();  // the previous output tile has left slot W
                 epi_sync();
-#pragma unroll 1
-                for (int c0 = cb0; c0 < cb0 + 64; c0 += 32) {
-                    if ((c0 >> 5) > qd) {  // block entirely above the diagonal
-                        store_zero32(slot(kW), r, c0);
-                        if (p.normalized) store_zero32(wlo, r, c0);
-                        continue;
-                    }
-                    float f[32], g[32];
-                    ld32(tb + lane_base + kTA + c0, f);
-#pragma unroll
-                    for (int jj = 0; jj < 32; ++jj) {
-                        if (c0 + jj > r) f[jj] = 0.f;
-                        g[jj] = f[jj] - bf16_round(f[jj]);
-                    }
-#pragma unroll
-                    for (int jj = 0; jj < 32; jj += 8) {
-                        store_row8(slot(kW), r, c0 + jj, f + jj);
-                        if (p.normalized) store_row8(wlo, r, c0 + jj, g + jj);
-                    }
+                {
+                    // blocks of 32 columns above the diagonal block of these rows are zero
+                    const int nblk = min(2, max(0, qd - 2 * hf + 1));  // blocks of this thread to load
+                    float f0[32], f1[32];
+                    if (nblk == 2) ld64(tb + lane_base + kTA + cb0, f0, f1);
+                    else if (nblk == 1) ld32(tb + lane_base + kTA + cb0, f0);
+                    if (nblk >= 1) emit_w(slot(kW), wlo, r, cb0, f0, p.normalized);
+                    else { store_zero32(slot(kW), r, cb0); if (p.normalized) store_zero32(wlo, r, cb0); }
+                    if (nblk == 2) emit_w(slot(kW), wlo, r, cb0 + 32, f1, p.normalized);
+                    else { store_zero32(slot(kW), r, cb0 + 32); if (p.normalized) store_zero32(wlo, r, cb0 + 32); }
                 }
                 fence_async_smem();
                 epi_arrive(ms, bEpW);
 
-                // X -> X_hi (slot SX), X_lo (slot W); D_p -> bf16 (slot SD); e carry
+                // while X = W K + Q S_p runs: q_t . e_p, the carried part of the denominator
+                float den_part = 0.f;
+                if (p.normalized) {
+#pragma unroll
+                    for (int c0 = cb0; c0 < cb0 + 64; c0 += 8) {
+                        float q8[8];
+                        tile_row8(qt, r, c0, q8);
+#pragma unroll
+                        for (int u = 0; u < 8; ++u) den_part += q8[u] * ms->eloc[c0 + u];
+                    }
+                }
+
+                // X -> X_hi (slot SX), X_lo (slot W)
                 bar_wait(ms, bEvX, tp, p);
                 tc_fence_after();
                 const float cs = ms->cshift[j & 1];
-                float den_part = 0.f, ecol[2] = {0.f, 0.f};
+                float ecol[2] = {0.f, 0.f};
+                float xs[2][32];
+                ld64(tb + lane_base + kTX + cb0, xs[0], xs[1]);
 #pragma unroll
                 for (int h = 0; h < 2; ++h) {
                     const int c0 = cb0 + 32 * h;
-                    float x[32];
-                    ld32(tb + lane_base + kTX + c0, x);
+                    float (&x)[32] = xs[h];
 #pragma unroll
                     for (int jj = 0; jj < 32; jj += 8) {
                         float q8[8], lo8[8];
@@ -519,78 +645,50 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                         for (int u = 0; u < 8; ++u) {
                             x[jj + u] += cs * q8[u];
                             lo8[u] = x[jj + u] - bf16_round(x[jj + u]);
-                            if (p.normalized) den_part += q8[u] * ms->eloc[c0 + jj + u];
                         }
                         store_row8(slot(kSX), r, c0 + jj, x + jj);
                         store_row8(slot(kW), r, c0 + jj, lo8);
                     }
-                    if (p.normalized) ecol[h] = warp_colsum32(x);  // column c0 + lane over this warp's rows
-                }
-#pragma unroll 1
-                for (int c0 = cb0; c0 < cb0 + 64; c0 += 32) {
-                    float f[32];
-                    ld32(tb + lane_base + kTD + c0, f);
-#pragma unroll
-                    for (int jj = 0; jj < 32; jj += 8) store_row8(slot(kSD), r, c0 + jj, f + jj);
                 }
                 fence_async_smem();
                 epi_arrive(ms, bEpX);
 
-                // T = L . (Q X^T) -> bf16 (slot W); denominators; next S split (hi)
+                // while T = Q X^T runs: column sums of X (e carry) and D_p -> bf16 (slot SD; R_lo
+                // there is dead once X is done; D += X^T V is issued after this tile's T hand-off)
+                if (p.normalized) {
+                    ecol[0] = warp_colsum32(xs[0]);  // column cb0 + lane over this warp's rows
+                    ecol[1] = warp_colsum32(xs[1]);
+                }
+                {
+                    float f0[32], f1[32];
+                    ld64(tb + lane_base + kTD + cb0, f0, f1);
+#pragma unroll
+                    for (int jj = 0; jj < 32; jj += 8) {
+                        store_row8(slot(kSD), r, cb0 + jj, f0 + jj);
+                        store_row8(slot(kSD), r, cb0 + 32 + jj, f1 + jj);
+                    }
+                }
+
+                // T = L . (Q X^T) -> bf16 (slot W); denominators
                 bar_wait(ms, bEvT, tp, p);
                 tc_fence_after();
-#pragma unroll 1
-                for (int c0 = cb0; c0 < cb0 + 64; c0 += 32) {
-                    if ((c0 >> 5) > qd) {
-                        store_zero32(slot(kW), r, c0);
-                        continue;
-                    }
-                    float f[32];
-                    ld32(tb + lane_base + kTA + c0, f);
-#pragma unroll
-                    for (int jj = 0; jj < 32; ++jj) {
-                        if (c0 + jj > r) f[jj] = 0.f;
-                        den_part += f[jj];
-                    }
-#pragma unroll
-                    for (int jj = 0; jj < 32; jj += 8) store_row8(slot(kW), r, c0 + jj, f + jj);
+                {
+                    const int nblk = min(2, max(0, qd - 2 * hf + 1));
+                    float f0[32], f1[32];
+                    if (nblk == 2) ld64(tb + lane_base + kTA + cb0, f0, f1);
+                    else if (nblk == 1) ld32(tb + lane_base + kTA + cb0, f0);
+                    if (nblk >= 1) den_part += emit_t(slot(kW), r, cb0, f0);
+                    else store_zero32(slot(kW), r, cb0);
+                    if (nblk == 2) den_part += emit_t(slot(kW), r, cb0 + 32, f1);
+                    else store_zero32(slot(kW), r, cb0 + 32);
                 }
+                fence_async_smem();
+                epi_arrive(ms, bEpT);
                 if (p.normalized) {  // den_t = both halves' partial sums
                     if (hf == 1) ms->den[r] = den_part;
                     epi_sync();
                     if (hf == 0) ms->den[r] += den_part;
                 }
-                if (j + 1 < nt) {
-                    // shift of the next tile from the trace of the updated S
-                    float dg = 0.f;
-                    if ((qd >> 1) == hf) {
-                        float f[32];
-                        ld32(tb + lane_base + kTS + 32 * qd, f);  // block holding the diagonal of these rows
-#pragma unroll
-                        for (int jj = 0; jj < 32; ++jj)
-                            if (jj == lane) dg = f[jj];
-                    }
-                    dg = warp_sum(dg);
-                    if (lane == 0) ms->red[warp] = dg;
-                    epi_sync();
-                    float tr = 0.f;
-#pragma unroll
-                    for (int w = 0; w < kEpiWarps; ++w) tr += ms->red[w];
-                    const float c = bf16_round(tr / kD);
-                    if (et == 0) ms->cshift[(j + 1) & 1] = c;
-#pragma unroll 1
-                    for (int c0 = cb0; c0 < cb0 + 64; c0 += 32) {
-                        float f[32];
-                        ld32(tb + lane_base + kTS + c0, f);
-#pragma unroll
-                        for (int jj = 0; jj < 32; ++jj) f[jj] -= ((c0 + jj) == r ? c : 0.f);
-#pragma unroll
-                        for (int jj = 0; jj < 32; jj += 8) store_row8(slot(kSX), r, c0 + jj, f + jj);
-                    }
-                }
-                fence_async_smem();
-                epi_sync();
-                epi_arrive(ms, bEpT);
 
                 // e carry += column sums of X (fixed order ((q0 + q1) + (q2 + q3)))
                 if (p.normalized) {
@@ -614,33 +712,62 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                     const bool final_out = (sigma == 0);
                     const float den = p.normalized ? ms->den[r] : 1.f;
                     const bool divide = final_out && p.normalized;
-#pragma unroll 1
-                    for (int c0 = cb0; c0 < cb0 + 64; c0 += 32) {
-                        float f[32];
-                        ld32(tb + lane_base + kTX + c0, f);
-                        if (divide) {
+                    float f0[32], f1[32];
+                    ld64(tb + lane_base + kTX + cb0, f0, f1);
+                    if (divide) {
+                        const float inv = 1.f / (den + p.eps);
 #pragma unroll
-                            for (int jj = 0; jj < 32; ++jj) f[jj] = f[jj] / (den + p.eps);
+                        for (int jj = 0; jj < 32; ++jj) {
+                            f0[jj] *= inv;
+                            f1[jj] *= inv;
                         }
+                    }
 #pragma unroll
-                        for (int jj = 0; jj < 32; jj += 8) store_row8(slot(kW), r, c0 + jj, f + jj);
+                    for (int jj = 0; jj < 32; jj += 8) {
+                        store_row8(slot(kW), r, cb0 + jj, f0 + jj);
+                        store_row8(slot(kW), r, cb0 + 32 + jj, f1 + jj);
                     }
                     if (!final_out && p.normalized && hf == 0 && tok0 + r < p.n)
                         p.den_loc[(size_t)head * p.n + tok0 + r] = den;
                 }
-                if (j + 1 < nt && p.normalized) {  // next S split (lo): D_p (bf16) in SD is dead now
-                    const float c = ms->cshift[(j + 1) & 1];
+                // D += X^T V done: X_hi in SX and D_p (bf16) in SD are dead, the D carry is current
+                bar_wait(ms, bEvD, tp, p);
+                tc_fence_after();
+                if (j + 1 < nt) {
+                    // split of the updated S for the next tile
+                    float dg = 0.f;
+                    if ((qd >> 1) == hf) {
+                        float f[32];
+                        ld32(tb + lane_base + kTS + 32 * qd, f);  // block holding the diagonal of these rows
+#pragma unroll
+                        for (int jj = 0; jj < 32; ++jj)
+                            if (jj == lane) dg = f[jj];
+                    }
+                    dg = warp_sum(dg);
+                    if (lane == 0) ms->red[warp] = dg;
+                    epi_sync();
+                    float tr = 0.f;
+#pragma unroll
+                    for (int w = 0; w < kEpiWarps; ++w) tr += ms->red[w];
+                    const float c = bf16_round(tr / kD);
+                    if (et == 0) ms->cshift[(j + 1) & 1] = c;
 #pragma unroll 1
-                    for (int c0 = cb0; c0 < cb0 + 64; c0 += 32) {
+                    for (int h = 0; h < 2; ++h) {
+                        const int c0 = cb0 + 32 * h;
                         float f[32];
                         ld32(tb + lane_base + kTS + c0, f);
 #pragma unroll
-                        for (int jj = 0; jj < 32; ++jj) {
-                            const float rr = f[jj] - ((c0 + jj) == r ? c : 0.f);
-                            f[jj] = rr - bf16_round(rr);
-                        }
+                        for (int jj = 0; jj < 32; jj += 8) {
+                            float hi[8], lo[8];
 #pragma unroll
-                        for (int jj = 0; jj < 32; jj += 8) store_row8(slot(kSD), r, c0 + jj, f + jj);
+                            for (int u = 0; u < 8; ++u) {
+                                const float rr = f[jj + u] - ((c0 + jj + u) == r ? c : 0.f);
+                                hi[u] = bf16_round(rr);
+                                lo[u] = rr - hi[u];
+                            }
+                            store_row8(slot(kSX), r, c0 + jj, hi);
+                            if (p.normalized) store_row8(slot(kSD), r, c0 + jj, lo);
+                        }
                     }
                 }
                 fence_async_smem();
@@ -657,20 +784,22 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
             {
                 if (sigma > 0 && et == 0) chain_wait(&flagD[head * 2 + ((sigma - 1) & 1)], (unsigned)sigma, p, 2, item);
                 epi_sync();
-                const float *dprev = sigma > 0 ? ring_prev + kD * kD + r * kD : nullptr;
+                const float4 *dprev = sigma > 0 ? reinterpret_cast<const float4 *>(ring_prev + kD * kD) : nullptr;
+                float4 *dcur = reinterpret_cast<float4 *>(ring_cur + kD * kD);
 #pragma unroll 1
-                for (int c0 = cb0; c0 < cb0 + 64; c0 += 32) {
+                for (int h = 0; h < 2; ++h) {
+                    const int c0 = cb0 + 32 * h;
                     float f[32], dp[32];
                     ld32(tb + lane_base + kTD + c0, f);
 #pragma unroll
                     for (int jj = 0; jj < 32; jj += 4) {
-                        const float4 v4 = dprev ? __ldcg(reinterpret_cast<const float4 *>(dprev + c0 + jj))
+                        const float4 v4 = dprev ? __ldcg(dprev + ring4(8 * h + jj / 4, et))
                                                 : make_float4(0.f, 0.f, 0.f, 0.f);
                         dp[jj] = v4.x; dp[jj + 1] = v4.y; dp[jj + 2] = v4.z; dp[jj + 3] = v4.w;
                     }
 #pragma unroll
                     for (int jj = 0; jj < 32; jj += 4)
-                        __stcg(reinterpret_cast<float4 *>(ring_cur + kD * kD + r * kD + c0 + jj),
+                        __stcg(dcur + ring4(8 * h + jj / 4, et),
                                make_float4(dp[jj] + f[jj], dp[jj + 1] + f[jj + 1], dp[jj + 2] + f[jj + 2],
                                            dp[jj + 3] + f[jj + 3]));
                     if (sigma > 0) {
@@ -683,12 +812,7 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                     eprev = sigma > 0 ? __ldcg(ring_prev + 2 * kD * kD + r) : 0.f;
                     __stcg(ring_cur + 2 * kD * kD + r, eprev + ms->eloc[r]);
                 }
-                tc_fence_before();
-                epi_sync();
-                if (et == 0) {
-                    __threadfence();
-                    st_release(&flagD[head * 2 + (sigma & 1)], (unsigned)(sigma + 1));
-                }
+                pub_arrive(kBarPubD);  // D and e prefixes in the ring
                 if (sigma > 0) {
                     if (hf == 0) ms->eloc[r] = eprev;  // now e of the prefix, for the fix-up denominators
                     if (et == 0) tma_store_wait_all();  // provisional outputs written before they are re-read
@@ -697,8 +821,12 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                     epi_arrive(ms, bEpDF);
                     for (int j = 0; j < nt; ++j) {
                         const uint8_t *qt = slot((j & 1) ? kQ1 : kQ0), *ot = slot((j & 1) ? kV : kK);
+                        uint8_t *stg = slot((j & 1) ? kSX : kW);  // output staging alternates W / SX
                         const int tok0 = (t0 + j) * kTile;
-                        bar_wait(ms, bEvF, n_fix & 1, p);
+                        const float dl = (p.normalized && hf == 0 && tok0 + r < p.n)
+                                             ? __ldcg(p.den_loc + (size_t)head * p.n + tok0 + r) : 0.f;
+                        const int g = j & 1;
+                        bar_wait(ms, bEvF + g, (fx_par >> g) & 1u, p);
                         tc_fence_after();
                         float den = 1.f;
                         if (p.normalized) {
@@ -713,39 +841,37 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                             }
                             if (hf == 1) ms->den[r] = qe;
                             epi_sync();
-                            if (hf == 0)
-                                ms->den[r] += qe + (tok0 + r < p.n ? p.den_loc[(size_t)head * p.n + tok0 + r] : 0.f);
-                            epi_sync();
-                            den = ms->den[r];
+                            if (hf == 0) ms->den[r] += qe + dl;
                         }
-                        if (et == 0) tma_store_wait_read();
+                        if (et == 0) tma_store_wait_read1();  // the store that used stg two tiles ago is done
                         epi_sync();
-#pragma unroll 1
-                        for (int c0 = cb0; c0 < cb0 + 64; c0 += 32) {
-                            float f[32];
-                            ld32(tb + lane_base + kTA + c0, f);
+                        if (p.normalized) den = ms->den[r];
+                        {
+                            float f0[32], f1[32];
+                            ld64(tb + lane_base + ((j & 1) ? kTX : kTA) + cb0, f0, f1);
+                            const float inv = p.normalized ? 1.f / (den + p.eps) : 1.f;
 #pragma unroll
                             for (int jj = 0; jj < 32; jj += 8) {
-                                float o8[8];
-                                tile_row8(ot, r, c0 + jj, o8);
+                                float o8[8], w8[8];
+                                tile_row8(ot, r, cb0 + jj, o8);
 #pragma unroll
-                                for (int u = 0; u < 8; ++u) {
-                                    const float num = o8[u] + f[jj + u];
-                                    f[jj + u] = p.normalized ? num / (den + p.eps) : num;
-                                }
+                                for (int u = 0; u < 8; ++u) w8[u] = (o8[u] + f0[jj + u]) * inv;
+                                store_row8(stg, r, cb0 + jj, w8);
+                                tile_row8(ot, r, cb0 + 32 + jj, o8);
+#pragma unroll
+                                for (int u = 0; u < 8; ++u) w8[u] = (o8[u] + f1[jj + u]) * inv;
+                                store_row8(stg, r, cb0 + 32 + jj, w8);
                             }
-#pragma unroll
-                            for (int jj = 0; jj < 32; jj += 8) store_row8(slot(kW), r, c0 + jj, f + jj);
                         }
                         fence_async_smem();
                         epi_sync();
                         if (et == 0) {
-                            tma_store_3d(&tm_o, slot(kW), 0, tok0, head);
-                            tma_store_3d(&tm_o, slot(kW) + kBlockBytes, 64, tok0, head);
+                            tma_store_3d(&tm_o, stg, 0, tok0, head);
+                            tma_store_3d(&tm_o, stg + kBlockBytes, 64, tok0, head);
                             tma_store_commit();
                         }
-                        epi_arrive(ms, bEpF);
-                        ++n_fix;
+                        epi_arrive(ms, bEpF + g);
+                        fx_par ^= 1u << g;
                     }
                 }
             }

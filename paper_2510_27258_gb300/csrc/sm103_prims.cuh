@@ -89,6 +89,9 @@ __device__ __forceinline__ void tma_store_commit() { asm volatile("cp.async.bulk
 // waits until all committed bulk stores of this thread have finished reading shared memory
 __device__ __forceinline__ void tma_store_wait_read() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
 
+// waits until at most the most recent committed bulk store group may still be reading shared memory
+__device__ __forceinline__ void tma_store_wait_read1() { asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory"); }
+
 // waits until all committed bulk stores of this thread are complete (globally visible)
 __device__ __forceinline__ void tma_store_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 
