@@ -26,11 +26,11 @@
 // The exclusive scan across segments is a chained scan; Theorem 2 guarantees
 // the result equals the serial recurrence.
 //
-// Roles: warp 8 issues TMA loads and MMAs (one thread); warp 9 releases the
+// Roles: warp 16 issues TMA loads and MMAs (one thread); warp 17 releases the
 // cross-SM prefix flags once the epilogue has written a prefix (the GPU-scope
-// fence this takes stays off the epilogue's path); warps 0-7 are the epilogue
+// fence this takes stays off the epilogue's path); warps 0-15 are the epilogue
 // (TMEM -> registers -> shared memory): warp w reads TMEM lanes 32 (w % 4) ..
-// +31 (one row each) and columns 64 (w / 4) .. +63.
+// +31 (one row each) and columns 32 (w / 4) .. +31.
 //
 // Precision: tokens are bf16, every product accumulates in fp32 (TMEM).  The S
 // operand is split as S = c I + R (c = bf16(trace S / d)) with c q_t added in
@@ -51,7 +51,7 @@ using namespace sm103;
 
 constexpr int kD = 128;           // d = dv handled by this kernel
 constexpr int kTile = 128;        // tokens per tile (MMA M)
-constexpr int kEpiWarps = 8;      // 2 per TMEM lane quadrant
+constexpr int kEpiWarps = 16;     // 4 per TMEM lane quadrant
 constexpr int kEpiThreads = kEpiWarps * 32;
 constexpr int kIssuerWarp = kEpiWarps;
 constexpr int kPubWarp = kEpiWarps + 1;  // releases the cross-SM prefix flags
@@ -90,7 +90,7 @@ struct Misc {
     float red[kEpiWarps];
     float eloc[kD];      // segment-local e carry
     float den[kTile];    // denominators of the current tile
-    float ebuf[2][kD];   // cross-quadrant partial column sums of X
+    float part[3][kD];   // partial sums of the other three column quarters / lane quadrants
 };
 static_assert(sizeof(Misc) <= kMiscBytes, "misc smem");
 
@@ -112,8 +112,9 @@ struct Params {
 constexpr int kRingFloats = kD * kD + kD * kD + kD;
 
 // The S and D prefixes in the ring are stored in the order the epilogue holds
-// them: float4 c (columns cb0 + 4c .. +3 of row r) of epilogue thread et at
-// float4 index c * 256 + et, so that every warp access is 512 contiguous bytes.
+// them: float4 c (columns c0 + 4c .. +3 of row r) of epilogue thread et at
+// float4 index c * kEpiThreads + et, so that every warp access is 512
+// contiguous bytes.
 // Writer and reader (the next segment of the head) use the same thread mapping.
 __device__ __forceinline__ int ring4(int c, int et) { return c * kEpiThreads + et; }
 // floats of one head's state tuple [S | C | m | G | h] with d = dv = kD
@@ -131,7 +132,7 @@ __device__ __forceinline__ unsigned ld_acquire(const unsigned *p) {
     return v;
 }
 // named barrier of the epilogue warps
-__device__ __forceinline__ void epi_sync() { asm volatile("bar.sync 1, 256;" ::: "memory"); }
+__device__ __forceinline__ void epi_sync() { asm volatile("bar.sync 1, %0;" ::"n"(kEpiThreads) : "memory"); }
 // Hand-offs epilogue -> publisher warp (named barriers 2 and 3, 288 threads): the
 // epilogue arrives after writing a prefix to the ring and goes on; the publisher
 // waits, then makes the ring writes visible GPU-wide and releases the flag.
@@ -246,19 +247,6 @@ __device__ __forceinline__ void ld32(uint32_t addr, float (&f)[32]) {
     tmem_ld_wait();
 #pragma unroll
     for (int j = 0; j < 32; ++j) f[j] = __uint_as_float(a[j]);
-}
-
-// two 32-column TMEM loads with one wait
-__device__ __forceinline__ void ld64(uint32_t addr, float (&f0)[32], float (&f1)[32]) {
-    uint32_t a[32], b[32];
-    tmem_ld32(addr, a);
-    tmem_ld32(addr + 32, b);
-    tmem_ld_wait();
-#pragma unroll
-    for (int j = 0; j < 32; ++j) {
-        f0[j] = __uint_as_float(a[j]);
-        f1[j] = __uint_as_float(b[j]);
-    }
 }
 
 // Column sums of v over the 32 lanes of a warp: returns, in lane l, the sum of
@@ -498,10 +486,12 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
         } else {
             // ===================== epilogue warps =====================
             const int et = tid;
-            const int qd = warp & 3, hf = warp >> 2;
+            const int qd = warp & 3, cq = warp >> 2;
             const int r = 32 * qd + lane;        // TMEM lane = row handled by this thread
-            const int cb0 = 64 * hf;             // first of the 64 columns handled by this thread
+            const int c0 = 32 * cq;              // first of the 32 columns handled by this thread
             const uint32_t lane_base = (uint32_t)(32 * qd) << 16;
+            // this thread's 32-column block of L . A and L . T lies above the diagonal (zero), on it, or below
+            const bool blk_zero = cq > qd;
             const float *ring_prev = p.ring + ((size_t)head * 2 + ((sigma + 1) & 1)) * kRingFloats;
             float *ring_cur = p.ring + ((size_t)head * 2 + (sigma & 1)) * kRingFloats;
             const unsigned *flagS = p.flags, *flagD = p.flags + 2 * p.BH;
@@ -515,19 +505,21 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 // carry-in S: the previous segment's prefix (ring) or the initial state (row-major)
                 const float4 *ringS = sigma > 0 ? reinterpret_cast<const float4 *>(ring_prev) : nullptr;
                 const float4 *st_row = (sigma == 0 && p.state_in)
-                    ? reinterpret_cast<const float4 *>(p.state_in + (size_t)head * kStateFloats + r * kD + cb0)
+                    ? reinterpret_cast<const float4 *>(p.state_in + (size_t)head * kStateFloats + r * kD + c0)
                     : nullptr;
-                auto s_in = [&](int c) {  // float4 c of this thread's 64 columns
-                    if (ringS) return __ldcg(ringS + ring4(c, et));
-                    if (st_row) return __ldcg(st_row + c);
-                    return make_float4(0.f, 0.f, 0.f, 0.f);
-                };
-                // diagonal element (from the thread whose columns contain r) -> trace -> shift
+                float sp[32];
+#pragma unroll
+                for (int c = 0; c < 8; ++c) {
+                    const float4 v4 = ringS ? __ldcg(ringS + ring4(c, et))
+                                            : st_row ? __ldcg(st_row + c) : make_float4(0.f, 0.f, 0.f, 0.f);
+                    sp[4 * c] = v4.x; sp[4 * c + 1] = v4.y; sp[4 * c + 2] = v4.z; sp[4 * c + 3] = v4.w;
+                }
+                // trace -> shift (the diagonal element of row r lies in column block qd)
                 float s = 0.f;
-                if ((r >> 6) == hf) {
-                    const float4 v4 = s_in((r - cb0) >> 2);
-                    const int cc = r & 3;
-                    s = cc == 0 ? v4.x : cc == 1 ? v4.y : cc == 2 ? v4.z : v4.w;
+                if (cq == qd) {
+#pragma unroll
+                    for (int jj = 0; jj < 32; ++jj)
+                        if (jj == lane) s = sp[jj];
                 }
                 s = warp_sum(s);
                 if (lane == 0) ms->red[warp] = s;
@@ -537,52 +529,45 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 for (int w = 0; w < kEpiWarps; ++w) tr += ms->red[w];
                 const float c = bf16_round(tr / kD);
                 if (et == 0) ms->cshift[0] = c;
-                const float *d0 = (sigma == 0 && p.init_De) ? p.init_De + (size_t)head * (kD * kD + kD) : nullptr;
-#pragma unroll 1
-                for (int h = 0; h < 2; ++h) {
-                    const int c0 = cb0 + 32 * h;
-                    float sp[32], agg[32];
-#pragma unroll
-                    for (int j = 0; j < 32; j += 4) {
-                        const float4 v4 = s_in(8 * h + j / 4);
-                        sp[j] = v4.x; sp[j + 1] = v4.y; sp[j + 2] = v4.z; sp[j + 3] = v4.w;
-                    }
-                    ld32(tb + lane_base + kTX + c0, agg);
+                {
                     // inclusive S prefix of this segment -> ring
+                    float agg[32];
+                    ld32(tb + lane_base + kTX + c0, agg);
+                    float4 *rc = reinterpret_cast<float4 *>(ring_cur);
 #pragma unroll
                     for (int j = 0; j < 32; j += 4)
-                        __stcg(reinterpret_cast<float4 *>(ring_cur) + ring4(8 * h + j / 4, et),
-                               make_float4(sp[j] + agg[j], sp[j + 1] + agg[j + 1], sp[j + 2] + agg[j + 2],
-                                           sp[j + 3] + agg[j + 3]));
-                    // S carry in TMEM
-                    uint32_t u[32];
-#pragma unroll
-                    for (int j = 0; j < 32; ++j) u[j] = __float_as_uint(sp[j]);
-                    tmem_st32(tb + lane_base + kTS + c0, u);
-                    // split S_p = c I + R into R_hi (slot SX) and R_lo (slot SD)
-#pragma unroll
-                    for (int j = 0; j < 32; j += 8) {
-                        float hi[8], lo[8];
-#pragma unroll
-                        for (int t = 0; t < 8; ++t) {
-                            const float rr = sp[j + t] - ((c0 + j + t) == r ? c : 0.f);
-                            hi[t] = bf16_round(rr);
-                            lo[t] = rr - hi[t];
-                        }
-                        store_row8(slot(kSX), r, c0 + j, hi);
-                        if (p.normalized) store_row8(slot(kSD), r, c0 + j, lo);
-                    }
-                    // segment-local D carry: the initial state's D for the first segment
-#pragma unroll
-                    for (int j = 0; j < 32; j += 4) {
-                        const float4 v4 = d0 ? __ldcg(reinterpret_cast<const float4 *>(d0 + r * kD + c0 + j))
-                                             : make_float4(0.f, 0.f, 0.f, 0.f);
-                        u[j] = __float_as_uint(v4.x); u[j + 1] = __float_as_uint(v4.y);
-                        u[j + 2] = __float_as_uint(v4.z); u[j + 3] = __float_as_uint(v4.w);
-                    }
-                    tmem_st32(tb + lane_base + kTD + c0, u);
+                        __stcg(rc + ring4(j / 4, et), make_float4(sp[j] + agg[j], sp[j + 1] + agg[j + 1],
+                                                                 sp[j + 2] + agg[j + 2], sp[j + 3] + agg[j + 3]));
                 }
-                if (hf == 0) ms->eloc[r] = d0 ? d0[kD * kD + r] : 0.f;
+                // S carry in TMEM
+                uint32_t u[32];
+#pragma unroll
+                for (int j = 0; j < 32; ++j) u[j] = __float_as_uint(sp[j]);
+                tmem_st32(tb + lane_base + kTS + c0, u);
+                // split S_p = c I + R into R_hi (slot SX) and R_lo (slot SD)
+#pragma unroll
+                for (int j = 0; j < 32; j += 8) {
+                    float hi[8], lo[8];
+#pragma unroll
+                    for (int t = 0; t < 8; ++t) {
+                        const float rr = sp[j + t] - ((c0 + j + t) == r ? c : 0.f);
+                        hi[t] = bf16_round(rr);
+                        lo[t] = rr - hi[t];
+                    }
+                    store_row8(slot(kSX), r, c0 + j, hi);
+                    if (p.normalized) store_row8(slot(kSD), r, c0 + j, lo);
+                }
+                // segment-local D carry: the initial state's D for the first segment
+                const float *d0 = (sigma == 0 && p.init_De) ? p.init_De + (size_t)head * (kD * kD + kD) : nullptr;
+#pragma unroll
+                for (int j = 0; j < 32; j += 4) {
+                    const float4 v4 = d0 ? __ldcg(reinterpret_cast<const float4 *>(d0 + r * kD + c0 + j))
+                                         : make_float4(0.f, 0.f, 0.f, 0.f);
+                    u[j] = __float_as_uint(v4.x); u[j + 1] = __float_as_uint(v4.y);
+                    u[j + 2] = __float_as_uint(v4.z); u[j + 3] = __float_as_uint(v4.w);
+                }
+                tmem_st32(tb + lane_base + kTD + c0, u);
+                if (cq == 0) ms->eloc[r] = d0 ? d0[kD * kD + r] : 0.f;
                 tmem_st_wait();
             }
             fence_async_smem();
@@ -600,16 +585,13 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 tc_fence_after();
                 if (et == 0) tma_store_wait_read();  // the previous output tile has left slot W
                 epi_sync();
-                {
-                    // blocks of 32 columns above the diagonal block of these rows are zero
-                    const int nblk = min(2, max(0, qd - 2 * hf + 1));  // blocks of this thread to load
-                    float f0[32], f1[32];
-                    if (nblk == 2) ld64(tb + lane_base + kTA + cb0, f0, f1);
-                    else if (nblk == 1) ld32(tb + lane_base + kTA + cb0, f0);
-                    if (nblk >= 1) emit_w(slot(kW), wlo, r, cb0, f0, p.normalized);
-                    else { store_zero32(slot(kW), r, cb0); if (p.normalized) store_zero32(wlo, r, cb0); }
-                    if (nblk == 2) emit_w(slot(kW), wlo, r, cb0 + 32, f1, p.normalized);
-                    else { store_zero32(slot(kW), r, cb0 + 32); if (p.normalized) store_zero32(wlo, r, cb0 + 32); }
+                if (blk_zero) {
+                    store_zero32(slot(kW), r, c0);
+                    if (p.normalized) store_zero32(wlo, r, c0);
+                } else {
+                    float f[32];
+                    ld32(tb + lane_base + kTA + c0, f);
+                    emit_w(slot(kW), wlo, r, c0, f, p.normalized);
                 }
                 fence_async_smem();
                 epi_arrive(ms, bEpW);
@@ -618,11 +600,11 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 float den_part = 0.f;
                 if (p.normalized) {
 #pragma unroll
-                    for (int c0 = cb0; c0 < cb0 + 64; c0 += 8) {
+                    for (int jj = 0; jj < 32; jj += 8) {
                         float q8[8];
-                        tile_row8(qt, r, c0, q8);
+                        tile_row8(qt, r, c0 + jj, q8);
 #pragma unroll
-                        for (int u = 0; u < 8; ++u) den_part += q8[u] * ms->eloc[c0 + u];
+                        for (int u = 0; u < 8; ++u) den_part += q8[u] * ms->eloc[c0 + jj + u];
                     }
                 }
 
@@ -630,79 +612,59 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 bar_wait(ms, bEvX, tp, p);
                 tc_fence_after();
                 const float cs = ms->cshift[j & 1];
-                float ecol[2] = {0.f, 0.f};
-                float xs[2][32];
-                ld64(tb + lane_base + kTX + cb0, xs[0], xs[1]);
+                float x[32];
+                ld32(tb + lane_base + kTX + c0, x);
 #pragma unroll
-                for (int h = 0; h < 2; ++h) {
-                    const int c0 = cb0 + 32 * h;
-                    float (&x)[32] = xs[h];
+                for (int jj = 0; jj < 32; jj += 8) {
+                    float q8[8], lo8[8];
+                    tile_row8(qt, r, c0 + jj, q8);
 #pragma unroll
-                    for (int jj = 0; jj < 32; jj += 8) {
-                        float q8[8], lo8[8];
-                        tile_row8(qt, r, c0 + jj, q8);
-#pragma unroll
-                        for (int u = 0; u < 8; ++u) {
-                            x[jj + u] += cs * q8[u];
-                            lo8[u] = x[jj + u] - bf16_round(x[jj + u]);
-                        }
-                        store_row8(slot(kSX), r, c0 + jj, x + jj);
-                        store_row8(slot(kW), r, c0 + jj, lo8);
+                    for (int u = 0; u < 8; ++u) {
+                        x[jj + u] += cs * q8[u];
+                        lo8[u] = x[jj + u] - bf16_round(x[jj + u]);
                     }
+                    store_row8(slot(kSX), r, c0 + jj, x + jj);
+                    store_row8(slot(kW), r, c0 + jj, lo8);
                 }
                 fence_async_smem();
                 epi_arrive(ms, bEpX);
 
                 // while T = Q X^T runs: column sums of X (e carry) and D_p -> bf16 (slot SD; R_lo
                 // there is dead once X is done; D += X^T V is issued after this tile's T hand-off)
-                if (p.normalized) {
-                    ecol[0] = warp_colsum32(xs[0]);  // column cb0 + lane over this warp's rows
-                    ecol[1] = warp_colsum32(xs[1]);
-                }
+                float ecol = 0.f;
+                if (p.normalized) ecol = warp_colsum32(x);  // column c0 + lane over this warp's rows
                 {
-                    float f0[32], f1[32];
-                    ld64(tb + lane_base + kTD + cb0, f0, f1);
+                    float f[32];
+                    ld32(tb + lane_base + kTD + c0, f);
 #pragma unroll
-                    for (int jj = 0; jj < 32; jj += 8) {
-                        store_row8(slot(kSD), r, cb0 + jj, f0 + jj);
-                        store_row8(slot(kSD), r, cb0 + 32 + jj, f1 + jj);
-                    }
+                    for (int jj = 0; jj < 32; jj += 8) store_row8(slot(kSD), r, c0 + jj, f + jj);
                 }
 
-                // T = L . (Q X^T) -> bf16 (slot W); denominators
+                // T = L . (Q X^T) -> bf16 (slot W); row sums
                 bar_wait(ms, bEvT, tp, p);
                 tc_fence_after();
-                {
-                    const int nblk = min(2, max(0, qd - 2 * hf + 1));
-                    float f0[32], f1[32];
-                    if (nblk == 2) ld64(tb + lane_base + kTA + cb0, f0, f1);
-                    else if (nblk == 1) ld32(tb + lane_base + kTA + cb0, f0);
-                    if (nblk >= 1) den_part += emit_t(slot(kW), r, cb0, f0);
-                    else store_zero32(slot(kW), r, cb0);
-                    if (nblk == 2) den_part += emit_t(slot(kW), r, cb0 + 32, f1);
-                    else store_zero32(slot(kW), r, cb0 + 32);
+                if (blk_zero) {
+                    store_zero32(slot(kW), r, c0);
+                } else {
+                    float f[32];
+                    ld32(tb + lane_base + kTA + c0, f);
+                    den_part += emit_t(slot(kW), r, c0, f);
                 }
                 fence_async_smem();
                 epi_arrive(ms, bEpT);
-                if (p.normalized) {  // den_t = both halves' partial sums
-                    if (hf == 1) ms->den[r] = den_part;
-                    epi_sync();
-                    if (hf == 0) ms->den[r] += den_part;
-                }
 
-                // e carry += column sums of X (fixed order ((q0 + q1) + (q2 + q3)))
+                // denominators (sum over the four column quarters) and e carry += column sums of X
+                // (sum over the four lane quadrants), both in a fixed order
                 if (p.normalized) {
-                    const int ca = cb0 + lane, cbx = cb0 + 32 + lane;
-                    if (qd & 1) { ms->ebuf[qd >> 1][ca] = ecol[0]; ms->ebuf[qd >> 1][cbx] = ecol[1]; }
+                    if (cq > 0) ms->part[cq - 1][r] = den_part;
                     epi_sync();
-                    if (!(qd & 1)) { ecol[0] += ms->ebuf[qd >> 1][ca]; ecol[1] += ms->ebuf[qd >> 1][cbx]; }
+                    if (cq == 0) ms->den[r] = ((den_part + ms->part[0][r]) + ms->part[1][r]) + ms->part[2][r];
                     epi_sync();
-                    if (qd == 2) { ms->ebuf[0][ca] = ecol[0]; ms->ebuf[0][cbx] = ecol[1]; }
+                    if (qd > 0) ms->part[qd - 1][c0 + lane] = ecol;
                     epi_sync();
-                    if (qd == 0) {
-                        ms->eloc[ca] += ecol[0] + ms->ebuf[0][ca];
-                        ms->eloc[cbx] += ecol[1] + ms->ebuf[0][cbx];
-                    }
+                    if (qd == 0)
+                        ms->eloc[c0 + lane] += (ecol + ms->part[0][c0 + lane]) +
+                                               (ms->part[1][c0 + lane] + ms->part[2][c0 + lane]);
                 }
 
                 // O (provisional for segments > 0, final for the first) -> slot W, TMA store
@@ -711,34 +673,27 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 {
                     const bool final_out = (sigma == 0);
                     const float den = p.normalized ? ms->den[r] : 1.f;
-                    const bool divide = final_out && p.normalized;
-                    float f0[32], f1[32];
-                    ld64(tb + lane_base + kTX + cb0, f0, f1);
-                    if (divide) {
+                    float f[32];
+                    ld32(tb + lane_base + kTX + c0, f);
+                    if (final_out && p.normalized) {
                         const float inv = 1.f / (den + p.eps);
 #pragma unroll
-                        for (int jj = 0; jj < 32; ++jj) {
-                            f0[jj] *= inv;
-                            f1[jj] *= inv;
-                        }
+                        for (int jj = 0; jj < 32; ++jj) f[jj] *= inv;
                     }
 #pragma unroll
-                    for (int jj = 0; jj < 32; jj += 8) {
-                        store_row8(slot(kW), r, cb0 + jj, f0 + jj);
-                        store_row8(slot(kW), r, cb0 + 32 + jj, f1 + jj);
-                    }
-                    if (!final_out && p.normalized && hf == 0 && tok0 + r < p.n)
+                    for (int jj = 0; jj < 32; jj += 8) store_row8(slot(kW), r, c0 + jj, f + jj);
+                    if (!final_out && p.normalized && cq == 0 && tok0 + r < p.n)
                         p.den_loc[(size_t)head * p.n + tok0 + r] = den;
                 }
                 // D += X^T V done: X_hi in SX and D_p (bf16) in SD are dead, the D carry is current
                 bar_wait(ms, bEvD, tp, p);
                 tc_fence_after();
                 if (j + 1 < nt) {
-                    // split of the updated S for the next tile
+                    // split of the updated S for the next tile, shifted by the mean of its diagonal
+                    float f[32];
+                    ld32(tb + lane_base + kTS + c0, f);
                     float dg = 0.f;
-                    if ((qd >> 1) == hf) {
-                        float f[32];
-                        ld32(tb + lane_base + kTS + 32 * qd, f);  // block holding the diagonal of these rows
+                    if (cq == qd) {
 #pragma unroll
                         for (int jj = 0; jj < 32; ++jj)
                             if (jj == lane) dg = f[jj];
@@ -751,23 +706,17 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                     for (int w = 0; w < kEpiWarps; ++w) tr += ms->red[w];
                     const float c = bf16_round(tr / kD);
                     if (et == 0) ms->cshift[(j + 1) & 1] = c;
-#pragma unroll 1
-                    for (int h = 0; h < 2; ++h) {
-                        const int c0 = cb0 + 32 * h;
-                        float f[32];
-                        ld32(tb + lane_base + kTS + c0, f);
 #pragma unroll
-                        for (int jj = 0; jj < 32; jj += 8) {
-                            float hi[8], lo[8];
+                    for (int jj = 0; jj < 32; jj += 8) {
+                        float hi[8], lo[8];
 #pragma unroll
-                            for (int u = 0; u < 8; ++u) {
-                                const float rr = f[jj + u] - ((c0 + jj + u) == r ? c : 0.f);
-                                hi[u] = bf16_round(rr);
-                                lo[u] = rr - hi[u];
-                            }
-                            store_row8(slot(kSX), r, c0 + jj, hi);
-                            if (p.normalized) store_row8(slot(kSD), r, c0 + jj, lo);
+                        for (int u = 0; u < 8; ++u) {
+                            const float rr = f[jj + u] - ((c0 + jj + u) == r ? c : 0.f);
+                            hi[u] = bf16_round(rr);
+                            lo[u] = rr - hi[u];
                         }
+                        store_row8(slot(kSX), r, c0 + jj, hi);
+                        if (p.normalized) store_row8(slot(kSD), r, c0 + jj, lo);
                     }
                 }
                 fence_async_smem();
@@ -786,35 +735,31 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 epi_sync();
                 const float4 *dprev = sigma > 0 ? reinterpret_cast<const float4 *>(ring_prev + kD * kD) : nullptr;
                 float4 *dcur = reinterpret_cast<float4 *>(ring_cur + kD * kD);
-#pragma unroll 1
-                for (int h = 0; h < 2; ++h) {
-                    const int c0 = cb0 + 32 * h;
+                {
                     float f[32], dp[32];
                     ld32(tb + lane_base + kTD + c0, f);
 #pragma unroll
                     for (int jj = 0; jj < 32; jj += 4) {
-                        const float4 v4 = dprev ? __ldcg(dprev + ring4(8 * h + jj / 4, et))
-                                                : make_float4(0.f, 0.f, 0.f, 0.f);
+                        const float4 v4 = dprev ? __ldcg(dprev + ring4(jj / 4, et)) : make_float4(0.f, 0.f, 0.f, 0.f);
                         dp[jj] = v4.x; dp[jj + 1] = v4.y; dp[jj + 2] = v4.z; dp[jj + 3] = v4.w;
                     }
 #pragma unroll
                     for (int jj = 0; jj < 32; jj += 4)
-                        __stcg(dcur + ring4(8 * h + jj / 4, et),
-                               make_float4(dp[jj] + f[jj], dp[jj + 1] + f[jj + 1], dp[jj + 2] + f[jj + 2],
-                                           dp[jj + 3] + f[jj + 3]));
-                    if (sigma > 0) {
+                        __stcg(dcur + ring4(jj / 4, et), make_float4(dp[jj] + f[jj], dp[jj + 1] + f[jj + 1],
+                                                                    dp[jj + 2] + f[jj + 2], dp[jj + 3] + f[jj + 3]));
+                    if (sigma > 0) {  // D prefix (bf16) for the fix-up
 #pragma unroll
                         for (int jj = 0; jj < 32; jj += 8) store_row8(slot(kSD), r, c0 + jj, dp + jj);
                     }
                 }
                 float eprev = 0.f;
-                if (hf == 0) {
+                if (cq == 0) {
                     eprev = sigma > 0 ? __ldcg(ring_prev + 2 * kD * kD + r) : 0.f;
                     __stcg(ring_cur + 2 * kD * kD + r, eprev + ms->eloc[r]);
                 }
                 pub_arrive(kBarPubD);  // D and e prefixes in the ring
                 if (sigma > 0) {
-                    if (hf == 0) ms->eloc[r] = eprev;  // now e of the prefix, for the fix-up denominators
+                    if (cq == 0) ms->eloc[r] = eprev;  // now e of the prefix, for the fix-up denominators
                     if (et == 0) tma_store_wait_all();  // provisional outputs written before they are re-read
                     fence_async_smem();
                     epi_sync();
@@ -823,45 +768,37 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                         const uint8_t *qt = slot((j & 1) ? kQ1 : kQ0), *ot = slot((j & 1) ? kV : kK);
                         uint8_t *stg = slot((j & 1) ? kSX : kW);  // output staging alternates W / SX
                         const int tok0 = (t0 + j) * kTile;
-                        const float dl = (p.normalized && hf == 0 && tok0 + r < p.n)
+                        const float dl = (p.normalized && cq == 0 && tok0 + r < p.n)
                                              ? __ldcg(p.den_loc + (size_t)head * p.n + tok0 + r) : 0.f;
                         const int g = j & 1;
                         bar_wait(ms, bEvF + g, (fx_par >> g) & 1u, p);
                         tc_fence_after();
-                        float den = 1.f;
                         if (p.normalized) {
-                            // den_t = provisional denominator + q_t . e_prefix (two column halves)
+                            // den_t = provisional denominator + q_t . e_prefix (four column quarters)
                             float qe = 0.f;
 #pragma unroll
-                            for (int c0 = cb0; c0 < cb0 + 64; c0 += 8) {
+                            for (int jj = 0; jj < 32; jj += 8) {
                                 float q8[8];
-                                tile_row8(qt, r, c0, q8);
+                                tile_row8(qt, r, c0 + jj, q8);
 #pragma unroll
-                                for (int u = 0; u < 8; ++u) qe += q8[u] * ms->eloc[c0 + u];
+                                for (int u = 0; u < 8; ++u) qe += q8[u] * ms->eloc[c0 + jj + u];
                             }
-                            if (hf == 1) ms->den[r] = qe;
+                            if (cq > 0) ms->part[cq - 1][r] = qe;
                             epi_sync();
-                            if (hf == 0) ms->den[r] += qe + dl;
+                            if (cq == 0) ms->den[r] = dl + (((qe + ms->part[0][r]) + ms->part[1][r]) + ms->part[2][r]);
                         }
                         if (et == 0) tma_store_wait_read1();  // the store that used stg two tiles ago is done
                         epi_sync();
-                        if (p.normalized) den = ms->den[r];
-                        {
-                            float f0[32], f1[32];
-                            ld64(tb + lane_base + ((j & 1) ? kTX : kTA) + cb0, f0, f1);
-                            const float inv = p.normalized ? 1.f / (den + p.eps) : 1.f;
+                        const float inv = p.normalized ? 1.f / (ms->den[r] + p.eps) : 1.f;
+                        float f[32];
+                        ld32(tb + lane_base + (g ? kTX : kTA) + c0, f);
 #pragma unroll
-                            for (int jj = 0; jj < 32; jj += 8) {
-                                float o8[8], w8[8];
-                                tile_row8(ot, r, cb0 + jj, o8);
+                        for (int jj = 0; jj < 32; jj += 8) {
+                            float o8[8], w8[8];
+                            tile_row8(ot, r, c0 + jj, o8);
 #pragma unroll
-                                for (int u = 0; u < 8; ++u) w8[u] = (o8[u] + f0[jj + u]) * inv;
-                                store_row8(stg, r, cb0 + jj, w8);
-                                tile_row8(ot, r, cb0 + 32 + jj, o8);
-#pragma unroll
-                                for (int u = 0; u < 8; ++u) w8[u] = (o8[u] + f1[jj + u]) * inv;
-                                store_row8(stg, r, cb0 + 32 + jj, w8);
-                            }
+                            for (int u = 0; u < 8; ++u) w8[u] = (o8[u] + f[jj + u]) * inv;
+                            store_row8(stg, r, c0 + jj, w8);
                         }
                         fence_async_smem();
                         epi_sync();
