@@ -74,9 +74,10 @@ enum Bar {
     bEvP = 6, bEvA = 7, bEvX = 8, bEvS = 9, bEvT = 10, bEvO = 11, bEvD = 12,
     bEvF = 13,  // + TMEM region of the fix-up tile (0: A, 1: X)
     bEpW = 15, bEpX = 16, bEpT = 17,
-    bEpF = 18,  // + TMEM region of the fix-up tile
-    bEpDF = 20,
-    kNumBars = 21
+    bEpR = 18,  // next tile's S split written, O read out of TMEM
+    bEpF = 19,  // + TMEM region of the fix-up tile
+    bEpDF = 21,
+    kNumBars = 22
 };
 constexpr int kFirstEpiBar = bEpW;
 
@@ -86,7 +87,6 @@ struct Misc {
     int item;        // current ticket
     int abort_flag;  // an mbarrier wait gave up
     int pad;
-    float cshift[2]; // S shift of the current / next tile
     float red[kEpiWarps];
     float eloc[kD];      // segment-local e carry
     float den[kTile];    // denominators of the current tile
@@ -210,33 +210,48 @@ __device__ __forceinline__ void store_zero32(uint8_t *tile, int r, int c0) {
 
 __device__ __forceinline__ float bf16_round(float x) { return __bfloat162float(__float2bfloat16_rn(x)); }
 
-// row r, columns c0..c0+31 of L . A -> W_hi (tile w) and, if lo, W_lo (tile wl)
-__device__ __forceinline__ void emit_w(uint8_t *w, uint8_t *wl, int r, int c0, float (&f)[32], bool lo) {
+// a, b -> bf16 pair hi (a in the low half) and the bf16 pair of the remainders a - hi_a, b - hi_b
+__device__ __forceinline__ void split2(float a, float b, uint32_t &hi, uint32_t &lo) {
+    hi = pack_bf16x2(a, b);
+    lo = pack_bf16x2(a - __uint_as_float(hi << 16), b - __uint_as_float(hi & 0xffff0000u));
+}
+
+// row r, columns c0..c0+31: v -> bf16 hi in tile th and, if lo, the bf16 remainder in tile tl
+__device__ __forceinline__ void store_split32(uint8_t *th, uint8_t *tl, int r, int c0, const float (&v)[32], bool lo) {
 #pragma unroll
     for (int jj = 0; jj < 32; jj += 8) {
-        float h8[8], l8[8];
+        uint32_t h[4], l[4];
 #pragma unroll
-        for (int u = 0; u < 8; ++u) {
-            h8[u] = (c0 + jj + u > r) ? 0.f : f[jj + u];
-            l8[u] = h8[u] - bf16_round(h8[u]);
-        }
-        store_row8(w, r, c0 + jj, h8);
-        if (lo) store_row8(wl, r, c0 + jj, l8);
+        for (int i = 0; i < 4; ++i) split2(v[jj + 2 * i], v[jj + 2 * i + 1], h[i], l[i]);
+        *reinterpret_cast<uint4 *>(th + tile_off(r, c0 + jj)) = make_uint4(h[0], h[1], h[2], h[3]);
+        if (lo) *reinterpret_cast<uint4 *>(tl + tile_off(r, c0 + jj)) = make_uint4(l[0], l[1], l[2], l[3]);
     }
 }
 
-// row r, columns c0..c0+31 of L . T -> bf16 tile; returns the row sum of the masked values
-__device__ __forceinline__ float emit_t(uint8_t *t, int r, int c0, float (&f)[32]) {
+// zero the entries of columns c0..c0+31 above the diagonal of row r (c > r); for the
+// 32 x 32 diagonal block of the tile, r - c0 = lane
+__device__ __forceinline__ void mask_upper32(float (&f)[32], int r, int c0) {
+#pragma unroll
+    for (int jj = 0; jj < 32; ++jj)
+        if (c0 + jj > r) f[jj] = 0.f;
+}
+
+// subtract c from the entry of column r (the diagonal), which this thread holds when
+// its block is the diagonal block
+__device__ __forceinline__ void shift_diag32(float (&f)[32], int lane, float c) {
+#pragma unroll
+    for (int jj = 0; jj < 32; ++jj)
+        if (jj == lane) f[jj] -= c;
+}
+
+// row r, columns c0..c0+31 -> bf16 tile; returns the fp32 sum of the values
+__device__ __forceinline__ float store_sum32(uint8_t *t, int r, int c0, const float (&f)[32]) {
     float sum = 0.f;
 #pragma unroll
     for (int jj = 0; jj < 32; jj += 8) {
-        float h8[8];
 #pragma unroll
-        for (int u = 0; u < 8; ++u) {
-            h8[u] = (c0 + jj + u > r) ? 0.f : f[jj + u];
-            sum += h8[u];
-        }
-        store_row8(t, r, c0 + jj, h8);
+        for (int u = 0; u < 8; ++u) sum += f[jj + u];
+        store_row8(t, r, c0 + jj, f + jj);
     }
     return sum;
 }
@@ -264,6 +279,19 @@ __device__ __forceinline__ float warp_colsum32(float (&v)[32]) {
         }
     }
     return v[0];
+}
+
+// sum of squares of row r, columns c0..c0+31 of a bf16 tile
+__device__ __forceinline__ float row_sumsq32(const uint8_t *tile, int r, int c0) {
+    float acc = 0.f;
+#pragma unroll
+    for (int jj = 0; jj < 32; jj += 8) {
+        float k8[8];
+        tile_row8(tile, r, c0 + jj, k8);
+#pragma unroll
+        for (int u = 0; u < 8; ++u) acc += k8[u] * k8[u];
+    }
+    return acc;
 }
 
 __device__ __forceinline__ float warp_sum(float x) {
@@ -335,6 +363,7 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
     uint32_t n_tiles = 0, n_items = 0, n_pre = 0, n_dfix = 0;
     uint32_t ld_par = 0;  // bit s: parity of the next load completion of slot s
     uint32_t fx_par = 0;  // bit g: parity of the next fix-up hand-off in TMEM region g
+    uint32_t n_r = 0;     // S-split hand-offs (one per tile that has a successor in its segment)
 
     // descriptor low words of the slots, as K-major (lk) and MN-major (lm) operands
     const uint32_t sb4 = smem_u32(smem) >> 4;
@@ -397,12 +426,18 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 for (int j = 0; j < nt && !ms->abort_flag; ++j) {
                     const uint32_t tp = n_tiles & 1;
                     const int qs = (j & 1) ? kQ1 : kQ0, qo = (j & 1) ? kQ0 : kQ1;
-                    if (!bar_wait(ms, bEpW, tp, p)) break;  // W (hi, lo), S split ready; TMEM X free
+                    // X = Q R_hi + Q R_lo + W_hi K + W_lo K; the Q R part runs while W is built.  The
+                    // split of S_p is ready (and O of the previous tile out of TMEM) at the R hand-off;
+                    // for the first tile of a segment it comes with W.
+                    if (j > 0 && !bar_wait(ms, bEpR, (n_r++) & 1, p)) break;
+                    if (j == 0 && !bar_wait(ms, bEpW, tp, p)) break;
                     tc_fence_after();
-                    mma128<false, true>(tb + kTX, lk(kW), lm(kK), 0u);        // X = W_hi K
-                    if (p.normalized) mma128<false, true>(tb + kTX, lk(qo), lm(kK), 1u);  // += W_lo K
-                    mma128<false, false>(tb + kTX, lk(qs), lk(kSX), 1u);      // += Q R_hi
+                    mma128<false, false>(tb + kTX, lk(qs), lk(kSX), 0u);      // X = Q R_hi
                     if (p.normalized) mma128<false, false>(tb + kTX, lk(qs), lk(kSD), 1u);  // += Q R_lo
+                    if (j > 0 && !bar_wait(ms, bEpW, tp, p)) break;  // W (hi, lo) ready
+                    tc_fence_after();
+                    mma128<false, true>(tb + kTX, lk(kW), lm(kK), 1u);        // += W_hi K
+                    if (p.normalized) mma128<false, true>(tb + kTX, lk(qo), lm(kK), 1u);  // += W_lo K
                     umma_commit(&ms->bar[bEvX]);
                     mma128<true, true>(tb + kTS, lm(kK), lm(kK), 1u);         // S += K^T K
                     umma_commit(&ms->bar[bEvS]);
@@ -411,14 +446,14 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                         load_tile(kK, &tm_k, head, (t0 + j + 1) * kTile);
                         load_tile(qo, &tm_q, head, (t0 + j + 1) * kTile);
                     }
-                    if (!bar_wait(ms, bEpX, tp, p)) break;  // X_hi, X_lo and D_hi ready
-                    if (!wait_ld(kV)) break;
+                    if (!bar_wait(ms, bEpX, tp, p)) break;  // X_hi and X_lo ready
                     tc_fence_after();
                     mma128<false, false>(tb + kTA, lk(qs), lk(kSX), 0u);      // T = Q X_hi^T
                     mma128<false, false>(tb + kTA, lk(qs), lk(kW), 1u);       // += Q X_lo^T (X_lo in W)
                     umma_commit(&ms->bar[bEvT]);
                     // T (bf16) in W and D_p (bf16) in SD; TMEM A free; the epilogue has read D_p from TMEM
                     if (!bar_wait(ms, bEpT, tp, p)) break;
+                    if (!wait_ld(kV)) break;
                     tc_fence_after();
                     mma128<false, true>(tb + kTX, lk(qs), lm(kSD), 0u);       // O = Q D_p
                     mma128<false, true>(tb + kTX, lk(kW), lm(kV), 1u);        // += T V
@@ -496,6 +531,11 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
             float *ring_cur = p.ring + ((size_t)head * 2 + (sigma & 1)) * kRingFloats;
             const unsigned *flagS = p.flags, *flagD = p.flags + 2 * p.BH;
 
+            // Shift of the S split: cs = bf16(tr_s / d) with tr_s the trace of the carry S_p,
+            // kept up to date from the K tiles' sums of squares (trace K^T K); every epilogue
+            // thread holds the same value.  Any shift is exact (x = R q + cs q in fp32).
+            float tr_s = 0.f, cs = 0.f;
+
             // ---- 1. S chain: carry-in S of the segment, publish the inclusive prefix ----
             bar_wait(ms, bEvP, ip, p);
             tc_fence_after();
@@ -524,11 +564,9 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 s = warp_sum(s);
                 if (lane == 0) ms->red[warp] = s;
                 epi_sync();
-                float tr = 0.f;
 #pragma unroll
-                for (int w = 0; w < kEpiWarps; ++w) tr += ms->red[w];
-                const float c = bf16_round(tr / kD);
-                if (et == 0) ms->cshift[0] = c;
+                for (int w = 0; w < kEpiWarps; ++w) tr_s += ms->red[w];
+                cs = bf16_round(tr_s / kD);
                 {
                     // inclusive S prefix of this segment -> ring
                     float agg[32];
@@ -544,19 +582,9 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
 #pragma unroll
                 for (int j = 0; j < 32; ++j) u[j] = __float_as_uint(sp[j]);
                 tmem_st32(tb + lane_base + kTS + c0, u);
-                // split S_p = c I + R into R_hi (slot SX) and R_lo (slot SD)
-#pragma unroll
-                for (int j = 0; j < 32; j += 8) {
-                    float hi[8], lo[8];
-#pragma unroll
-                    for (int t = 0; t < 8; ++t) {
-                        const float rr = sp[j + t] - ((c0 + j + t) == r ? c : 0.f);
-                        hi[t] = bf16_round(rr);
-                        lo[t] = rr - hi[t];
-                    }
-                    store_row8(slot(kSX), r, c0 + j, hi);
-                    if (p.normalized) store_row8(slot(kSD), r, c0 + j, lo);
-                }
+                // split S_p = cs I + R into R_hi (slot SX) and R_lo (slot SD)
+                if (cq == qd) shift_diag32(sp, lane, cs);
+                store_split32(slot(kSX), slot(kSD), r, c0, sp, p.normalized);
                 // segment-local D carry: the initial state's D for the first segment
                 const float *d0 = (sigma == 0 && p.init_De) ? p.init_De + (size_t)head * (kD * kD + kD) : nullptr;
 #pragma unroll
@@ -583,15 +611,19 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 // W = L . A (hi, lo)
                 bar_wait(ms, bEvA, tp, p);
                 tc_fence_after();
+                // this tile's part of trace K^T K (slot K holds K_j until the X MMAs are done)
+                const float k2 = warp_sum(row_sumsq32(slot(kK), r, c0));
                 if (et == 0) tma_store_wait_read();  // the previous output tile has left slot W
                 epi_sync();
+                if (lane == 0) ms->red[warp] = k2;
                 if (blk_zero) {
                     store_zero32(slot(kW), r, c0);
                     if (p.normalized) store_zero32(wlo, r, c0);
                 } else {
                     float f[32];
                     ld32(tb + lane_base + kTA + c0, f);
-                    emit_w(slot(kW), wlo, r, c0, f, p.normalized);
+                    if (cq == qd) mask_upper32(f, r, c0);
+                    store_split32(slot(kW), wlo, r, c0, f, p.normalized);
                 }
                 fence_async_smem();
                 epi_arrive(ms, bEpW);
@@ -611,21 +643,16 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 // X -> X_hi (slot SX), X_lo (slot W)
                 bar_wait(ms, bEvX, tp, p);
                 tc_fence_after();
-                const float cs = ms->cshift[j & 1];
                 float x[32];
                 ld32(tb + lane_base + kTX + c0, x);
 #pragma unroll
                 for (int jj = 0; jj < 32; jj += 8) {
-                    float q8[8], lo8[8];
+                    float q8[8];
                     tile_row8(qt, r, c0 + jj, q8);
 #pragma unroll
-                    for (int u = 0; u < 8; ++u) {
-                        x[jj + u] += cs * q8[u];
-                        lo8[u] = x[jj + u] - bf16_round(x[jj + u]);
-                    }
-                    store_row8(slot(kSX), r, c0 + jj, x + jj);
-                    store_row8(slot(kW), r, c0 + jj, lo8);
+                    for (int u = 0; u < 8; ++u) x[jj + u] += cs * q8[u];
                 }
+                store_split32(slot(kSX), slot(kW), r, c0, x, true);
                 fence_async_smem();
                 epi_arrive(ms, bEpX);
 
@@ -648,16 +675,23 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 } else {
                     float f[32];
                     ld32(tb + lane_base + kTA + c0, f);
-                    den_part += emit_t(slot(kW), r, c0, f);
+                    if (cq == qd) mask_upper32(f, r, c0);
+                    den_part += store_sum32(slot(kW), r, c0, f);
                 }
                 fence_async_smem();
                 epi_arrive(ms, bEpT);
 
-                // denominators (sum over the four column quarters) and e carry += column sums of X
-                // (sum over the four lane quadrants), both in a fixed order
+                // trace of the updated S; denominators (sum over the four column quarters) and
+                // e carry += column sums of X (sum over the four lane quadrants), in a fixed order
+                if (p.normalized && cq > 0) ms->part[cq - 1][r] = den_part;
+                epi_sync();
+                {
+                    float t = 0.f;
+#pragma unroll
+                    for (int w = 0; w < kEpiWarps; ++w) t += ms->red[w];
+                    tr_s += t;
+                }
                 if (p.normalized) {
-                    if (cq > 0) ms->part[cq - 1][r] = den_part;
-                    epi_sync();
                     if (cq == 0) ms->den[r] = ((den_part + ms->part[0][r]) + ms->part[1][r]) + ms->part[2][r];
                     epi_sync();
                     if (qd > 0) ms->part[qd - 1][c0 + lane] = ecol;
@@ -690,34 +724,13 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 tc_fence_after();
                 if (j + 1 < nt) {
                     // split of the updated S for the next tile, shifted by the mean of its diagonal
+                    cs = bf16_round(tr_s / kD);
                     float f[32];
                     ld32(tb + lane_base + kTS + c0, f);
-                    float dg = 0.f;
-                    if (cq == qd) {
-#pragma unroll
-                        for (int jj = 0; jj < 32; ++jj)
-                            if (jj == lane) dg = f[jj];
-                    }
-                    dg = warp_sum(dg);
-                    if (lane == 0) ms->red[warp] = dg;
-                    epi_sync();
-                    float tr = 0.f;
-#pragma unroll
-                    for (int w = 0; w < kEpiWarps; ++w) tr += ms->red[w];
-                    const float c = bf16_round(tr / kD);
-                    if (et == 0) ms->cshift[(j + 1) & 1] = c;
-#pragma unroll
-                    for (int jj = 0; jj < 32; jj += 8) {
-                        float hi[8], lo[8];
-#pragma unroll
-                        for (int u = 0; u < 8; ++u) {
-                            const float rr = f[jj + u] - ((c0 + jj + u) == r ? c : 0.f);
-                            hi[u] = bf16_round(rr);
-                            lo[u] = rr - hi[u];
-                        }
-                        store_row8(slot(kSX), r, c0 + jj, hi);
-                        if (p.normalized) store_row8(slot(kSD), r, c0 + jj, lo);
-                    }
+                    if (cq == qd) shift_diag32(f, lane, cs);
+                    store_split32(slot(kSX), slot(kSD), r, c0, f, p.normalized);
+                    fence_async_smem();
+                    epi_arrive(ms, bEpR);  // R of the next tile ready, O read: Q R may start
                 }
                 fence_async_smem();
                 epi_sync();
