@@ -203,11 +203,6 @@ __device__ __forceinline__ void store_row8(uint8_t *tile, int r, int c, const fl
     *reinterpret_cast<uint4 *>(tile + tile_off(r, c)) = u;
 }
 
-__device__ __forceinline__ void store_zero32(uint8_t *tile, int r, int c0) {
-#pragma unroll
-    for (int j = 0; j < 32; j += 8) *reinterpret_cast<uint4 *>(tile + tile_off(r, c0 + j)) = make_uint4(0, 0, 0, 0);
-}
-
 __device__ __forceinline__ float bf16_round(float x) { return __bfloat162float(__float2bfloat16_rn(x)); }
 
 // a, b -> bf16 pair hi (a in the low half) and the bf16 pair of the remainders a - hi_a, b - hi_b
@@ -244,16 +239,16 @@ __device__ __forceinline__ void shift_diag32(float (&f)[32], int lane, float c) 
         if (jj == lane) f[jj] -= c;
 }
 
-// row r, columns c0..c0+31 -> bf16 tile; returns the fp32 sum of the values
-__device__ __forceinline__ float store_sum32(uint8_t *t, int r, int c0, const float (&f)[32]) {
-    float sum = 0.f;
+// 32 values -> 16 packed bf16 pairs (the tensor-memory A-operand layout)
+__device__ __forceinline__ void pack32(const float (&v)[32], uint32_t (&h)[16]) {
 #pragma unroll
-    for (int jj = 0; jj < 32; jj += 8) {
+    for (int i = 0; i < 16; ++i) h[i] = pack_bf16x2(v[2 * i], v[2 * i + 1]);
+}
+
+// 32 values -> packed bf16 pairs hi and packed bf16 remainders lo
+__device__ __forceinline__ void split_pack32(const float (&v)[32], uint32_t (&h)[16], uint32_t (&l)[16]) {
 #pragma unroll
-        for (int u = 0; u < 8; ++u) sum += f[jj + u];
-        store_row8(t, r, c0 + jj, f + jj);
-    }
-    return sum;
+    for (int i = 0; i < 16; ++i) split2(v[2 * i], v[2 * i + 1], h[i], l[i]);
 }
 
 __device__ __forceinline__ void ld32(uint32_t addr, float (&f)[32]) {
@@ -321,6 +316,20 @@ __device__ __forceinline__ void mma128(uint32_t d_tmem, uint32_t a_lo, uint32_t 
         const uint32_t kb = B_MN ? kk * 128u : (kk >> 2) * (kBlockBytes >> 4) + (kk & 3) * 2u;
         umma_bf16(d_tmem, (static_cast<uint64_t>(kDescHi) << 32) | (a_lo + ka),
                   (static_cast<uint64_t>(kDescHi) << 32) | (b_lo + kb), id, kk > 0 ? 1u : accumulate);
+    }
+}
+
+// The same product with A (128 x 128 bf16) in tensor memory, in the layout the epilogue
+// writes: K elements 32g .. 32g+31 of every row packed as bf16 pairs in columns
+// a_tmem + 32g .. +15 (g = 0..3), so that K step kk starts at column 32 (kk / 2) + 8 (kk % 2).
+template <bool B_MN>
+__device__ __forceinline__ void mma128_ts(uint32_t d_tmem, uint32_t a_tmem, uint32_t b_lo, uint32_t accumulate) {
+    constexpr uint32_t id = idesc_bf16(128, 128, 0, B_MN);
+#pragma unroll
+    for (int kk = 0; kk < 8; ++kk) {
+        const uint32_t kb = B_MN ? kk * 128u : (kk >> 2) * (kBlockBytes >> 4) + (kk & 3) * 2u;
+        umma_bf16_ts(d_tmem, a_tmem + 32u * (kk >> 1) + 8u * (kk & 1), (static_cast<uint64_t>(kDescHi) << 32) | (b_lo + kb),
+                     id, kk > 0 ? 1u : accumulate);
     }
 }
 
@@ -426,6 +435,8 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 for (int j = 0; j < nt && !ms->abort_flag; ++j) {
                     const uint32_t tp = n_tiles & 1;
                     const int qs = (j & 1) ? kQ1 : kQ0, qo = (j & 1) ? kQ0 : kQ1;
+                    // slot qo (Q of the previous tile, last read by its O MMA) takes the next Q
+                    if (j + 1 < nt) load_tile(qo, &tm_q, head, (t0 + j + 1) * kTile);
                     // X = Q R_hi + Q R_lo + W_hi K + W_lo K; the Q R part runs while W is built.  The
                     // split of S_p is ready (and O of the previous tile out of TMEM) at the R hand-off;
                     // for the first tile of a segment it comes with W.
@@ -436,16 +447,13 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                     if (p.normalized) mma128<false, false>(tb + kTX, lk(qs), lk(kSD), 1u);  // += Q R_lo
                     if (j > 0 && !bar_wait(ms, bEpW, tp, p)) break;  // W (hi, lo) ready
                     tc_fence_after();
-                    mma128<false, true>(tb + kTX, lk(kW), lm(kK), 1u);        // += W_hi K
-                    if (p.normalized) mma128<false, true>(tb + kTX, lk(qo), lm(kK), 1u);  // += W_lo K
+                    mma128_ts<true>(tb + kTX, tb + kTA, lm(kK), 1u);          // += W_hi K (W in TMEM)
+                    if (p.normalized) mma128_ts<true>(tb + kTX, tb + kTA + 16, lm(kK), 1u);  // += W_lo K
                     umma_commit(&ms->bar[bEvX]);
                     mma128<true, true>(tb + kTS, lm(kK), lm(kK), 1u);         // S += K^T K
                     umma_commit(&ms->bar[bEvS]);
-                    if (!bar_wait(ms, bEvS, tp, p)) break;  // X and S MMAs done: K and W_lo slots free
-                    if (j + 1 < nt) {
-                        load_tile(kK, &tm_k, head, (t0 + j + 1) * kTile);
-                        load_tile(qo, &tm_q, head, (t0 + j + 1) * kTile);
-                    }
+                    if (!bar_wait(ms, bEvS, tp, p)) break;  // X and S MMAs done: slot K free
+                    if (j + 1 < nt) load_tile(kK, &tm_k, head, (t0 + j + 1) * kTile);
                     if (!bar_wait(ms, bEpX, tp, p)) break;  // X_hi and X_lo ready
                     tc_fence_after();
                     mma128<false, false>(tb + kTA, lk(qs), lk(kSX), 0u);      // T = Q X_hi^T
@@ -456,11 +464,13 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                     if (!wait_ld(kV)) break;
                     tc_fence_after();
                     mma128<false, true>(tb + kTX, lk(qs), lm(kSD), 0u);       // O = Q D_p
-                    mma128<false, true>(tb + kTX, lk(kW), lm(kV), 1u);        // += T V
+                    mma128_ts<true>(tb + kTX, tb + kTA, lm(kV), 1u);          // += T V (T in TMEM)
                     umma_commit(&ms->bar[bEvO]);
                     mma128<true, true>(tb + kTD, lm(kSX), lm(kV), 1u);        // D += X^T V
                     umma_commit(&ms->bar[bEvD]);
                     if (j + 1 < nt) {  // next tile's A = Q K^T overlaps this tile's output epilogue
+                        // A goes to the TMEM columns O has just read T from
+                        if (!bar_wait(ms, bEvO, tp, p)) break;
                         if (!wait_ld(qo) || !wait_ld(kK)) break;
                         tc_fence_after();
                         mma128<false, false>(tb + kTA, lk(qo), lk(kK), 0u);
@@ -605,28 +615,34 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
             for (int j = 0; j < nt; ++j) {
                 const uint32_t tp = n_tiles & 1;
                 const uint8_t *qt = slot((j & 1) ? kQ1 : kQ0);
-                uint8_t *wlo = slot((j & 1) ? kQ0 : kQ1);  // W_lo staging (the other Q slot)
                 const int tok0 = (t0 + j) * kTile;
 
-                // W = L . A (hi, lo)
+                // W = L . A -> bf16 hi and lo, written over this thread's own A columns in TMEM
+                // (the A operand of X += W K): hi in columns c0 .. +15, lo in c0 + 16 .. +31
                 bar_wait(ms, bEvA, tp, p);
                 tc_fence_after();
                 // this tile's part of trace K^T K (slot K holds K_j until the X MMAs are done)
                 const float k2 = warp_sum(row_sumsq32(slot(kK), r, c0));
+                {
+                    uint32_t h[16], l[16];
+                    if (blk_zero) {
+#pragma unroll
+                        for (int i = 0; i < 16; ++i) h[i] = l[i] = 0u;
+                    } else {
+                        float f[32];
+                        ld32(tb + lane_base + kTA + c0, f);
+                        if (cq == qd) mask_upper32(f, r, c0);
+                        split_pack32(f, h, l);
+                    }
+                    tmem_st16(tb + lane_base + kTA + c0, h);
+                    if (p.normalized) tmem_st16(tb + lane_base + kTA + c0 + 16, l);
+                    tmem_st_wait();
+                }
+                epi_arrive(ms, bEpW);
+
                 if (et == 0) tma_store_wait_read();  // the previous output tile has left slot W
                 epi_sync();
                 if (lane == 0) ms->red[warp] = k2;
-                if (blk_zero) {
-                    store_zero32(slot(kW), r, c0);
-                    if (p.normalized) store_zero32(wlo, r, c0);
-                } else {
-                    float f[32];
-                    ld32(tb + lane_base + kTA + c0, f);
-                    if (cq == qd) mask_upper32(f, r, c0);
-                    store_split32(slot(kW), wlo, r, c0, f, p.normalized);
-                }
-                fence_async_smem();
-                epi_arrive(ms, bEpW);
 
                 // while X = W K + Q S_p runs: q_t . e_p, the carried part of the denominator
                 float den_part = 0.f;
@@ -670,15 +686,24 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 // T = L . (Q X^T) -> bf16 (slot W); row sums
                 bar_wait(ms, bEvT, tp, p);
                 tc_fence_after();
-                if (blk_zero) {
-                    store_zero32(slot(kW), r, c0);
-                } else {
-                    float f[32];
-                    ld32(tb + lane_base + kTA + c0, f);
-                    if (cq == qd) mask_upper32(f, r, c0);
-                    den_part += store_sum32(slot(kW), r, c0, f);
+                {
+                    // bf16 T over this thread's own T columns in TMEM (the A operand of O += T V)
+                    uint32_t h[16];
+                    if (blk_zero) {
+#pragma unroll
+                        for (int i = 0; i < 16; ++i) h[i] = 0u;
+                    } else {
+                        float f[32];
+                        ld32(tb + lane_base + kTA + c0, f);
+                        if (cq == qd) mask_upper32(f, r, c0);
+#pragma unroll
+                        for (int jj = 0; jj < 32; ++jj) den_part += f[jj];
+                        pack32(f, h);
+                    }
+                    tmem_st16(tb + lane_base + kTA + c0, h);
+                    tmem_st_wait();
                 }
-                fence_async_smem();
+                fence_async_smem();  // D_p (bf16) in SD
                 epi_arrive(ms, bEpT);
 
                 // trace of the updated S; denominators (sum over the four column quarters) and
