@@ -32,6 +32,13 @@
 // (TMEM -> registers -> shared memory): warp w reads TMEM lanes 32 (w % 4) ..
 // +31 (one row each) and columns 32 (w / 4) .. +31.
 //
+// Head sizes d, dv of 64 run as 128 with zero features 64..127: the TMA box of
+// those columns lies wholly outside the tensor and is zero-filled, so S, x_t,
+// D and e have zero rows / columns there (the S shift cancels exactly: q_f = 0)
+// and the padded output columns, which are zero, are not stored.  The tile is
+// 128 tokens whatever the requested chunk (Theorem 2: the result does not
+// depend on the chunking up to rounding).
+//
 // Precision: tokens are bf16, every product accumulates in fp32 (TMEM).  The S
 // operand is split as S = c I + R (c = bf16(trace S / d)) with c q_t added in
 // fp32, so x_t is accurate although |S| grows like t/d.  X enters T = Q X^T as
@@ -107,6 +114,7 @@ struct Params {
     WsHeader *err;
     unsigned long long wait_ns;  // budget of a cross-SM chain wait
     int inject_skip_item;        // testing: this item does not publish its S prefix
+    int out_blocks;              // 64-column blocks of an output row (dv / 64)
 };
 
 constexpr int kRingFloats = kD * kD + kD * kD + kD;
@@ -761,7 +769,7 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 epi_sync();
                 if (et == 0) {
                     tma_store_3d(&tm_o, slot(kW), 0, tok0, head);
-                    tma_store_3d(&tm_o, slot(kW) + kBlockBytes, 64, tok0, head);
+                    if (p.out_blocks > 1) tma_store_3d(&tm_o, slot(kW) + kBlockBytes, 64, tok0, head);
                     tma_store_commit();
                 }
                 ++n_tiles;
@@ -842,7 +850,7 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                         epi_sync();
                         if (et == 0) {
                             tma_store_3d(&tm_o, stg, 0, tok0, head);
-                            tma_store_3d(&tm_o, stg + kBlockBytes, 64, tok0, head);
+                            if (p.out_blocks > 1) tma_store_3d(&tm_o, stg + kBlockBytes, 64, tok0, head);
                             tma_store_commit();
                         }
                         epi_arrive(ms, bEpF + g);
@@ -906,12 +914,14 @@ EncodeTiledFn encode_fn() {
     return fn;
 }
 
-// [BH][n][128] bf16 tensor, boxes of 64 x 128 tokens, 128-byte swizzle, zero fill out of range
-bool make_map(CUtensorMap *m, const void *base, int BH, int n) {
+// [BH][n][inner] bf16 tensor (inner = 64 or 128), boxes of 64 columns x 128 tokens,
+// 128-byte swizzle, zero fill out of range (the box at column 64 of a 64-wide tensor
+// is all fill)
+bool make_map(CUtensorMap *m, const void *base, int BH, int n, int inner) {
     EncodeTiledFn fn = encode_fn();
     if (!fn) return false;
-    cuuint64_t dims[3] = {(cuuint64_t)kD, (cuuint64_t)n, (cuuint64_t)BH};
-    cuuint64_t strides[2] = {(cuuint64_t)kD * 2, (cuuint64_t)n * kD * 2};
+    cuuint64_t dims[3] = {(cuuint64_t)inner, (cuuint64_t)n, (cuuint64_t)BH};
+    cuuint64_t strides[2] = {(cuuint64_t)inner * 2, (cuuint64_t)n * inner * 2};
     cuuint32_t box[3] = {64, (cuuint32_t)kTile, 1};
     cuuint32_t es[3] = {1, 1, 1};
     return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(base), dims, strides, box, es,
@@ -950,16 +960,20 @@ int segment_tiles(int BH, int M, int sms) {
 
 }  // namespace
 
+// head sizes the fused kernel serves (64 as zero-padded 128)
+bool fused_dim(int x) { return x == 64 || x == kD; }
+
 size_t fused2_workspace_bytes(int BH, int n, int d, int dv, int chunk, hla_dtype dt) {
-    if (dt != HLA_BF16 || d != kD || dv != kD) return 0;
+    if (dt != HLA_BF16 || !fused_dim(d) || !fused_dim(dv)) return 0;
     (void)chunk;
     return fused_layout(BH, n).total;
 }
 
 bool fused2_applicable(const Fwd2 &p) {
     if (getenv("HLA_DISABLE_FUSED")) return false;
-    if (p.dt != HLA_BF16 || p.d != kD || p.dv != kD || !p.masked || p.chunk != kTile) return false;
+    if (p.dt != HLA_BF16 || !fused_dim(p.d) || !fused_dim(p.dv) || !p.masked) return false;
     if (p.state_out || p.n <= 0 || p.BH <= 0) return false;
+    if (p.state_in && (p.d != kD || p.dv != kD)) return false;  // initial states in the 128 x 128 layout only
     if (p.ws_bytes < fused_layout(p.BH, p.n).total) return false;
     int dev = 0, major = 0, minor = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return false;
@@ -971,8 +985,8 @@ bool fused2_applicable(const Fwd2 &p) {
 cudaError_t fused2_forward(const Fwd2 &p, cudaStream_t stream) {
     FusedLayout FL = fused_layout(p.BH, p.n);
     CUtensorMap mq, mk, mv, mo;
-    if (!make_map(&mq, p.q, p.BH, p.n) || !make_map(&mk, p.k, p.BH, p.n) || !make_map(&mv, p.v, p.BH, p.n) ||
-        !make_map(&mo, p.out, p.BH, p.n))
+    if (!make_map(&mq, p.q, p.BH, p.n, p.d) || !make_map(&mk, p.k, p.BH, p.n, p.d) ||
+        !make_map(&mv, p.v, p.BH, p.n, p.dv) || !make_map(&mo, p.out, p.BH, p.n, p.dv))
         return cudaErrorInvalidValue;
     int dev = 0, sms = 0;
     cudaGetDevice(&dev);
@@ -995,6 +1009,7 @@ cudaError_t fused2_forward(const Fwd2 &p, cudaStream_t stream) {
     kp.err = reinterpret_cast<WsHeader *>(p.ws);
     kp.wait_ns = 2000000000ull;
     kp.inject_skip_item = -1;
+    kp.out_blocks = p.dv / 64;
     if (const char *e = getenv("HLA_TEST_WAIT_NS")) kp.wait_ns = strtoull(e, nullptr, 10);
     if (const char *e = getenv("HLA_TEST_SKIP_PUBLISH_ITEM")) kp.inject_skip_item = atoi(e);
     cudaError_t e;

@@ -52,7 +52,8 @@ extern "C" hla_status hla2_forward_noalloc(const void *q, const void *k, const v
     if (path < 0) return fail(HLA_ERR_UNSUPPORTED, "arguments not supported by hla2_forward");
     if (path != 1)
         return fail(HLA_ERR_UNSUPPORTED,
-                    "hla2_forward_noalloc serves the fused path only (bf16, d = dv = 128, masked, chunk 128, sm_103)");
+                    "hla2_forward_noalloc serves the fused path only (bf16, d and dv in {64, 128}, masked, no "
+                    "state_out; an initial state only with d = dv = 128; sm_103)");
     if (!q || !k || !v || !out) return fail(HLA_ERR_INVALID_ARGUMENT, "null q/k/v/out pointer");
     const uintptr_t mis = (reinterpret_cast<uintptr_t>(q) | reinterpret_cast<uintptr_t>(k) |
                            reinterpret_cast<uintptr_t>(v) | reinterpret_cast<uintptr_t>(out) |

@@ -1,6 +1,7 @@
-"""The fused tcgen05 forward (bf16, d = dv = 128, masked, chunk 128) against the
-fp64 oracle, including its cross-SM chained scans (forced short segments),
-ragged tails, an initial state, and the device-side timeout path."""
+"""The fused tcgen05 forward (bf16, masked; d and dv in {64, 128}, 64 running as
+zero-padded 128; 128-token tiles for any requested chunk) against the fp64
+oracle, including its cross-SM chained scans (forced short segments), ragged
+tails, an initial state, and the device-side timeout path."""
 import numpy as np
 import pytest
 import torch
@@ -21,11 +22,11 @@ def hla():
     return binding
 
 
-def run(hla, q, k, v, normalized, state_in=None):
+def run(hla, q, k, v, normalized, state_in=None, chunk=128):
     tq, tk, tv = (hla_inputs.as_torch(x, "bf16", DEV) for x in (q, k, v))
     sin = None if state_in is None else torch.from_numpy(np.ascontiguousarray(state_in, np.float32)).to(DEV)
-    ws = hla.alloc_workspace(hla.hla2_workspace_bytes(*q.shape, v.shape[-1], 128, torch.bfloat16), DEV)
-    out = hla.hla2_forward(tq, tk, tv, masked=True, normalized=normalized, eps=hla_inputs.EPS, chunk=128,
+    ws = hla.alloc_workspace(hla.hla2_workspace_bytes(*q.shape, v.shape[-1], chunk, torch.bfloat16), DEV)
+    out = hla.hla2_forward(tq, tk, tv, masked=True, normalized=normalized, eps=hla_inputs.EPS, chunk=chunk,
                            state_in=sin, workspace=ws)
     torch.cuda.synchronize()
     assert hla.hla_poll_error(ws) == 0
@@ -33,18 +34,20 @@ def run(hla, q, k, v, normalized, state_in=None):
     return out.float().cpu().numpy().reshape(B * H, n, -1)
 
 
-def check(hla, q, k, v, normalized, state_in=None):
+def check(hla, q, k, v, normalized, state_in=None, chunk=128):
     B, H, n, d = q.shape
-    assert hla.hla2_forward_path(B, H, n, d, d, normalized=normalized, has_state_in=state_in is not None)[0] == 1
+    dv = v.shape[-1]
+    assert hla.hla2_forward_path(B, H, n, d, dv, normalized=normalized, chunk=chunk,
+                                 has_state_in=state_in is not None)[0] == 1
     sin = None if state_in is None else np.asarray(state_in, np.float64).reshape(B * H, -1)
-    num_ref, den_ref = oracle.hla2_serial(q.reshape(B * H, n, d), k.reshape(B * H, n, d), v.reshape(B * H, n, d),
+    num_ref, den_ref = oracle.hla2_serial(q.reshape(B * H, n, d), k.reshape(B * H, n, d), v.reshape(B * H, n, dv),
                                           masked=True, normalized=False, state_in=sin, return_den=True, nthreads=8)
-    num = run(hla, q, k, v, False, state_in)
+    num = run(hla, q, k, v, False, state_in, chunk)
     if not normalized:
         err = rowerr(num, num_ref)
         assert err < 2e-2, err
         return err
-    o = run(hla, q, k, v, True, state_in)
+    o = run(hla, q, k, v, True, state_in, chunk)
     return check_normalized(o, num, num_ref, den_ref, hla_inputs.EPS, 2e-2)
 
 
@@ -52,7 +55,26 @@ def test_fused_path_selected(hla):
     assert hla.hla2_forward_path(2, 16, 16384, 128, 128, normalized=True) == (1, 1)
     assert hla.hla2_forward_path(2, 16, 16384, 128, 128, normalized=True, has_state_out=True)[0] == 0
     assert hla.hla2_forward_path(2, 16, 16384, 128, 128, masked=False)[0] == 0
-    assert hla.hla2_forward_path(2, 16, 16384, 64, 64)[0] == 0
+    # d, dv of 64 as zero-padded 128, any chunk; an initial state only in the 128 x 128 layout
+    assert hla.hla2_forward_path(8, 16, 2048, 64, 64, chunk=64) == (1, 1)
+    assert hla.hla2_forward_path(1, 1, 100, 64, 128, chunk=7)[0] == 1
+    assert hla.hla2_forward_path(1, 1, 100, 128, 64, chunk=128)[0] == 1
+    assert hla.hla2_forward_path(1, 1, 100, 128, 128, chunk=32, has_state_in=True)[0] == 1
+    assert hla.hla2_forward_path(1, 1, 100, 64, 64, has_state_in=True)[0] == 0
+    assert hla.hla2_forward_path(1, 1, 100, 32, 32)[0] == 0
+    assert hla.hla2_forward_path(1, 1, 100, 128, 128, dtype=torch.float32)[0] == 0
+
+
+@pytest.mark.parametrize("d,dv", [(64, 64), (64, 128), (128, 64)])
+@pytest.mark.parametrize("B,H,n,chunk", [(1, 1, 1, 64), (1, 2, 129, 64), (2, 3, 600, 128), (1, 1, 1000, 32)])
+@pytest.mark.parametrize("seg", ["1", "default"])
+@pytest.mark.parametrize("normalized", [False, True])
+def test_fused_head_size_64(hla, monkeypatch, d, dv, B, H, n, chunk, seg, normalized):
+    """Head sizes of 64 run as 128 with zero features; the requested chunk changes nothing but rounding."""
+    if seg != "default":
+        monkeypatch.setenv("HLA_FUSED_SEGMENT_TILES", seg)
+    q, k, v = hla_inputs.make_qkv(B, H, n, d, dv, seed=n + 31 * d + dv, dtype="bf16")
+    check(hla, q, k, v, normalized, chunk=chunk)
 
 
 @pytest.mark.parametrize("B,H,n", [(1, 1, 1), (1, 2, 127), (1, 2, 128), (1, 3, 129), (2, 2, 600), (1, 1, 2000)])
