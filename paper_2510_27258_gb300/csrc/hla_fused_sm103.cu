@@ -951,10 +951,11 @@ int segment_tiles(int BH, int M, int sms) {
         if (v > 0) return v < M ? v : M;
     }
     // enough segments that the heads fill the SMs several times over, but long
-    // enough that the chained scans stay short; tuned on the long workload
-    int L = 4;
+    // enough that the chained scans and per-segment set-up stay short (measured
+    // on B2 H16 n16384: 4..6 tiles within 1%, 3 and 8+ slower)
+    int L = 6;
     if ((long long)BH * ((M + L - 1) / L) < 2LL * sms) L = 2;
-    if (BH >= 2 * sms) L = M;  // plenty of heads: one segment per head, no chains
+    if (2 * BH >= sms) L = M;  // heads enough to occupy the SMs: one segment per head, no chains
     return L < M ? L : M;
 }
 
