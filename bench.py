@@ -35,6 +35,32 @@ FWD = hla_inputs.WORKLOADS["long_bf16_norm"]
 DEC = hla_inputs.WORKLOADS["decode_bf16"]
 
 
+# DRAM traffic per launch (dram__bytes_read.sum + dram__bytes_write.sum) from one ncu
+# capture of the kernel sources (concatenated) whose SHA-256 starts with "sha256"
+# (summaries in profiles/); reported as null for any other source or workload.
+TRAFFIC = {
+    "hla2_fused_kernel": {"src": ["hla_fused_sm103.cu", "sm103_prims.cuh"], "sha256": "547299329d9401d2", "workload": "long_bf16_norm",
+                          "n": 16384, "bytes": 688.4e6,
+                          "how": "ncu capture at n=8192 (270.4 MB read + 73.8 MB written) scaled x2 to n=16384"},
+    "step2_kernel": {"src": ["hla_step.cu"], "sha256": "6b7c09075c2fc3a7", "workload": "decode_bf16", "n": 0,
+                     "bytes": 750.9e6, "how": "ncu capture of one step (406.4 MB read + 344.5 MB written)"},
+}
+
+
+def traffic(kernel, workload, n):
+    import hashlib
+    t = TRAFFIC.get(kernel)
+    if t is None or t["workload"] != workload or (t["n"] and t["n"] != n):
+        return None, None
+    h = hashlib.sha256()
+    for name in t["src"]:
+        with open(os.path.join(ROOT, "paper_2510_27258_gb300", "csrc", name), "rb") as f:
+            h.update(f.read())
+    if not h.hexdigest().startswith(t["sha256"]):
+        return None, None
+    return t["bytes"], t["how"]
+
+
 def peaks():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
@@ -276,6 +302,7 @@ def main():
     if args.workload != "long_bf16_norm" or args.n > 0:
         args.no_cpu_baseline = True  # the CPU baseline samples the long workload only
     value = tokens * world / (ms * 1e-3)
+    fwd_traffic, fwd_traffic_how = traffic("hla2_fused_kernel", w.name, w.n) if path == 1 else (None, None)
     achieved_gbs = fwd_bytes(w) / (ms * 1e-3) / 1e9
     achieved_tf = fwd_flops(w) / (ms * 1e-3) / 1e12
 
@@ -319,7 +346,8 @@ def main():
                        3 * w.BH * w.n * w.d * 2 / 1e6, w.BH * w.n * w.dv * 2 / 1e6)},
         "clocks": clocks,
         "roofline": {"bound": "hbm", "achieved": achieved_gbs, "peak": hbm_peak, "unit": "GB/s",
-                     "frac": achieved_gbs / hbm_peak, "traffic": None, "peak_kind": peak_kind,
+                     "frac": achieved_gbs / hbm_peak, "traffic": fwd_traffic, "traffic_how": fwd_traffic_how,
+                     "algorithmic_bytes": fwd_bytes(w), "peak_kind": peak_kind,
                      "kernel": "hla2_fused_kernel (the forward's only kernel)" if path == 1 else "hla2_forward (3 kernels)",
                      "tensor_view": {
                          "achieved_tflops": achieved_tf, "peak_tflops": tc_peak,
@@ -372,11 +400,13 @@ def bench_decode(hla, dev, stream, steps, hbm_peak, world):
     torch.cuda.synchronize()
     us = max_over_ranks(e0.elapsed_time(e1) * 1e3 / steps, world)
     gbs = dec_bytes(w) / (us * 1e-6) / 1e9
+    dec_traffic, dec_how = traffic("step2_kernel", "decode_bf16", 0)
     return {"workload": "decode_bf16", "B": w.B, "H": w.H, "d": w.d, "dv": w.dv, "prefix": w.decode_prefix,
             "steps": steps, "us_per_step": us, "value": gbs * world, "unit": "GB/s",
             "tokens_per_s": w.B * world / (us * 1e-6),
             "roofline": {"bound": "hbm", "achieved": gbs, "peak": hbm_peak, "unit": "GB/s", "frac": gbs / hbm_peak,
-                         "traffic": None, "kernel": "step2_kernel"},
+                         "traffic": dec_traffic, "traffic_how": dec_how, "algorithmic_bytes": dec_bytes(w),
+                         "kernel": "step2_kernel"},
             "launches": steps}
 
 
