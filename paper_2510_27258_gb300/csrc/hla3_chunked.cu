@@ -1,0 +1,472 @@
+// Chunk-parallel third-order HLA forward (Theorem 4, Algorithm 4 at gamma = 1)
+// in fp32 on CUDA cores; calls that ask for state_out take the serial kernel
+// (hla3_generic.cu), which also advances G1..G3 and h1..h3 of the state tuple.
+//
+// Per head, tokens are cut into chunks of W (W = min(chunk, 64), 32 for head
+// sizes of 128; the result does not depend on the chunking up to rounding).
+// Rows are tokens of one chunk, A = Q K^T (A_ts = q_t . k_s), a = diag(A),
+// L / Ls the lower triangle with / without the diagonal.
+//
+// Masked.  With o_t = q_t^T F_t for the corrected state F (and den_t = q_t^T eta_t),
+// the token update of Algorithm 3 is
+//   dF_s = k_s a_s q_s^T P_s + k_s (k_s^T S^Q_{s-1} k_s) v_s^T + S^K_{s-1} q_s a_s v_s^T,
+// so that, for a chunk with carry-in (S^K, S^Q, P, m, F, eta)_p,
+//   Y = Q P_p + (L.A) V,   b_s = k_s^T S^Q_p k_s + sum_{u<s} A_us^2,
+//   C_ts = q_t^T S^K_p q_s + sum_{i<s} A_ti A_si,
+//   num = Q F_p + (L.A)(diag(a) Y + diag(b) V) + (L.C) diag(a) V,
+//   den = Q eta_p + (L.A)(a . (Q m_p + (L.A) 1) + b) + (L.C) a.
+// The carries follow the concatenation of Eqs. hla3-base-concat and
+// hla3-corrected-concat: S^K, S^Q, P, m add up, and
+//   F_{A (x) B} = F_A + F_B + S^K_A R_B + M^KQP_B[S^Q_A] + U_B P_A
+// (eta likewise with r, M^KQm, m) with the chunk's R = Q^T diag(a) V,
+// r = Q^T a, U = K^T diag(a) Q and the segment map applied by contraction,
+// M^KQP_B[Z] = K^T diag(k_t^T Z k_t) V.  Every term is linear in the
+// exclusive prefixes of S^K, S^Q, P, m, so the carries are two rounds of
+// prefix sums with no sequential matrix chain:
+//   F_p(c) = F_0 + sum_{c'<c} [F_{c'} + S^K_p(c') R_{c'} + M_{c'}[S^Q_p(c')] + U_{c'} P_p(c')].
+// The chunk-local F of the bracket (zero carry-in) is
+//   F_c = K^T (diag(a) Y_loc + diag(b_loc) V + N V),  N_ts = [t < s] A_st a_s.
+//
+// Unmasked (Sec. 7.1): o_t = q_t^T S^K_t S^Q_t P_t with inclusive prefixes:
+//   X = Q S^K_p + (L.A) K,  Z = X S^Q_p + (L.(X Q^T)) Q,  num = Z P_p + (L.(Z K^T)) V,
+//   den = Z m_p + (L.(Z K^T)) 1.
+//
+// Launches: local summaries, prefix sums of (S^K, S^Q, P, m), brackets (masked),
+// prefix sums of the brackets (masked), outputs; plus the corrected initial
+// carry F_0 = S^K S^Q P - G1 - G2 - G3 (eta_0 likewise) when state_in is given.
+#include "hla_internal.h"
+
+namespace hla {
+namespace {
+
+constexpr int kT3c = 256;
+
+struct C3Layout {
+    int BH, n, d, dv, W, nc;
+    long long rec_loc, rec_pre, oSK, oSQ, oU, oP, oF, oR, om, oe, orr;  // local record offsets (floats)
+    long long pSK, pSQ, pP, pm, pF, pe;                                  // prefix record offsets
+    long long loc_base, pre_base, init_base, total;
+    __host__ __device__ float *loc(float *ws, int hd, int c) const { return ws + loc_base + ((long long)hd * nc + c) * rec_loc; }
+    __host__ __device__ float *pre(float *ws, int hd, int c) const { return ws + pre_base + ((long long)hd * nc + c) * rec_pre; }
+    __host__ __device__ float *init(float *ws, int hd) const {
+        return ws + init_base + (long long)hd * ((long long)d * dv + d);
+    }
+};
+
+inline long long up4(long long x) { return (x + 3) / 4 * 4; }
+
+int chunk3_width(int d, int dv, int chunk) {
+    const int cap = (d >= 128 || dv >= 128) ? 32 : 64;
+    return chunk < cap ? chunk : cap;
+}
+
+C3Layout c3_layout(int BH, int n, int d, int dv, int chunk) {
+    C3Layout L;
+    L.BH = BH; L.n = n; L.d = d; L.dv = dv;
+    L.W = chunk3_width(d, dv, chunk);
+    L.nc = (n + L.W - 1) / L.W;
+    const long long dd = (long long)d * d, ddv = (long long)d * dv;
+    long long o = 0;
+    L.oSK = o; o += up4(dd); L.oSQ = o; o += up4(dd); L.oU = o; o += up4(dd);
+    L.oP = o; o += up4(ddv); L.oF = o; o += up4(ddv); L.oR = o; o += up4(ddv);
+    L.om = o; o += up4(d); L.oe = o; o += up4(d); L.orr = o; o += up4(d);
+    L.rec_loc = o;
+    o = 0;
+    L.pSK = o; o += up4(dd); L.pSQ = o; o += up4(dd); L.pP = o; o += up4(ddv);
+    L.pm = o; o += up4(d); L.pF = o; o += up4(ddv); L.pe = o; o += up4(d);
+    L.rec_pre = o;
+    L.loc_base = 0;
+    L.pre_base = L.loc_base + (long long)BH * L.nc * L.rec_loc;
+    L.init_base = L.pre_base + (long long)BH * L.nc * L.rec_pre;
+    L.total = L.init_base + (long long)BH * (ddv + d);
+    return L;
+}
+
+template <typename T>
+__device__ __forceinline__ float ld_tok(const T *p) { return to_f32(*p); }
+
+// dst[r][c] (row-major, ld = cols) = sum_k A(r,k) B(k,c) with accessor lambdas
+template <typename FA, typename FB>
+__device__ __forceinline__ void smm(float *dst, int rows, int cols, int kdim, FA a, FB b) {
+    for (int i = threadIdx.x; i < rows * cols; i += blockDim.x) {
+        const int r = i / cols, c = i % cols;
+        float s = 0.f;
+        for (int k = 0; k < kdim; ++k) s += a(r, k) * b(k, c);
+        dst[i] = s;
+    }
+}
+
+// loads the chunk's Q, K (w x d) and V (w x dv) as fp32; rows past the sequence are zero
+template <typename T>
+__device__ void load_chunk(const T *q, const T *k, const T *v, float *Qs, float *Ks, float *Vs, int hd, int t0,
+                           int w, int W, int n, int d, int dv) {
+    const T *Qh = q + ((size_t)hd * n + t0) * d, *Kh = k + ((size_t)hd * n + t0) * d;
+    const T *Vh = v + ((size_t)hd * n + t0) * dv;
+    for (int i = threadIdx.x; i < W * d; i += blockDim.x) {
+        const int r = i / d;
+        Qs[i] = r < w ? ld_tok(Qh + i) : 0.f;
+        Ks[i] = r < w ? ld_tok(Kh + i) : 0.f;
+    }
+    for (int i = threadIdx.x; i < W * dv; i += blockDim.x) Vs[i] = (i / dv) < w ? ld_tok(Vh + i) : 0.f;
+}
+
+// ---------------------------------------------------------------------------
+// 1. chunk-local summaries
+// ---------------------------------------------------------------------------
+template <typename T>
+__global__ void __launch_bounds__(kT3c) c3_local_kernel(const T *__restrict__ q, const T *__restrict__ k,
+                                                        const T *__restrict__ v, float *ws, C3Layout L, int masked) {
+    extern __shared__ float sm[];
+    const int c = blockIdx.x, hd = blockIdx.y, W = L.W, d = L.d, dv = L.dv;
+    const int t0 = c * W, w = min(W, L.n - t0);
+    float *Qs = sm, *Ks = Qs + W * d, *Vs = Ks + W * d, *A = Vs + W * dv, *Z = A + W * W, *a = Z + W * dv;
+    float *zeta = a + W, *b = zeta + W, *ym = b + W;
+    load_chunk(q, k, v, Qs, Ks, Vs, hd, t0, w, W, L.n, d, dv);
+    __syncthreads();
+    float *rec = L.loc(ws, hd, c);
+    // first-order sums
+    smm(rec + L.oSK, d, d, W, [&](int r, int t) { return Ks[t * d + r]; }, [&](int t, int cc) { return Ks[t * d + cc]; });
+    smm(rec + L.oSQ, d, d, W, [&](int r, int t) { return Qs[t * d + r]; }, [&](int t, int cc) { return Qs[t * d + cc]; });
+    smm(rec + L.oP, d, dv, W, [&](int r, int t) { return Ks[t * d + r]; }, [&](int t, int cc) { return Vs[t * dv + cc]; });
+    for (int r = threadIdx.x; r < d; r += blockDim.x) {
+        float s = 0.f;
+        for (int t = 0; t < W; ++t) s += Ks[t * d + r];
+        rec[L.om + r] = s;
+    }
+    if (!masked) return;
+    smm(A, W, W, d, [&](int t, int j) { return Qs[t * d + j]; }, [&](int j, int s) { return Ks[s * d + j]; });
+    __syncthreads();
+    for (int t = threadIdx.x; t < W; t += blockDim.x) {
+        a[t] = A[t * W + t];
+        float bs = 0.f, ys = 0.f;
+        for (int u = 0; u < t; ++u) bs += A[u * W + t] * A[u * W + t];
+        for (int j = 0; j <= t; ++j) ys += A[t * W + j];
+        b[t] = bs;
+        ym[t] = ys;
+    }
+    __syncthreads();
+    // Z = diag(a) Y_loc + diag(b) V + N V with Y_loc = (L.A) V and (N V)_t = sum_{s>t} A_st a_s v_s
+    for (int i = threadIdx.x; i < W * dv; i += blockDim.x) {
+        const int t = i / dv, cc = i % dv;
+        float y = 0.f, nv = 0.f;
+        for (int j = 0; j <= t; ++j) y += A[t * W + j] * Vs[j * dv + cc];
+        for (int s = t + 1; s < W; ++s) nv += A[s * W + t] * a[s] * Vs[s * dv + cc];
+        Z[i] = a[t] * y + b[t] * Vs[i] + nv;
+    }
+    for (int t = threadIdx.x; t < W; t += blockDim.x) {
+        float nv = 0.f;
+        for (int s = t + 1; s < W; ++s) nv += A[s * W + t] * a[s];
+        zeta[t] = a[t] * ym[t] + b[t] + nv;
+    }
+    __syncthreads();
+    smm(rec + L.oF, d, dv, W, [&](int r, int t) { return Ks[t * d + r]; }, [&](int t, int cc) { return Z[t * dv + cc]; });
+    smm(rec + L.oR, d, dv, W, [&](int r, int t) { return Qs[t * d + r] * a[t]; },
+        [&](int t, int cc) { return Vs[t * dv + cc]; });
+    smm(rec + L.oU, d, d, W, [&](int r, int t) { return Ks[t * d + r] * a[t]; },
+        [&](int t, int cc) { return Qs[t * d + cc]; });
+    for (int r = threadIdx.x; r < d; r += blockDim.x) {
+        float se = 0.f, sr = 0.f;
+        for (int t = 0; t < W; ++t) {
+            se += Ks[t * d + r] * zeta[t];
+            sr += Qs[t * d + r] * a[t];
+        }
+        rec[L.oe + r] = se;
+        rec[L.orr + r] = sr;
+    }
+}
+
+// ---------------------------------------------------------------------------
+// 2. exclusive prefix sums over chunks of (S^K, S^Q, P, m), starting at state_in
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(kT3c) c3_prefix1_kernel(float *ws, C3Layout L, const float *state_in) {
+    const int hd = blockIdx.y, d = L.d, dv = L.dv;
+    const long long dd = (long long)d * d, ddv = (long long)d * dv;
+    const long long nel = 2 * dd + ddv + d;
+    const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= nel) return;
+    long long lo, po, so;  // local offset, prefix offset, offset in the state tuple [SK | SQ | P | mK | ...]
+    if (i < dd) { lo = L.oSK + i; po = L.pSK + i; so = i; }
+    else if (i < 2 * dd) { lo = L.oSQ + (i - dd); po = L.pSQ + (i - dd); so = i; }
+    else if (i < 2 * dd + ddv) { lo = L.oP + (i - 2 * dd); po = L.pP + (i - 2 * dd); so = i; }
+    else { lo = L.om + (i - 2 * dd - ddv); po = L.pm + (i - 2 * dd - ddv); so = i; }
+    const long long st_len = 2 * dd + 4 * ddv + 4 * (long long)d;
+    float run = state_in ? state_in[(long long)hd * st_len + so] : 0.f;
+    for (int c = 0; c < L.nc; ++c) {
+        L.pre(ws, hd, c)[po] = run;
+        run += L.loc(ws, hd, c)[lo];
+    }
+}
+
+// corrected initial carry F_0 = S^K S^Q P - G1 - G2 - G3, eta_0 = S^K S^Q m - h1 - h2 - h3
+__global__ void __launch_bounds__(kT3c) c3_init_kernel(float *ws, C3Layout L, const float *state_in) {
+    const int hd = blockIdx.x, d = L.d, dv = L.dv;
+    const long long dd = (long long)d * d, ddv = (long long)d * dv;
+    const float *st = state_in + (long long)hd * (2 * dd + 4 * ddv + 4 * (long long)d);
+    const float *SK = st, *SQ = SK + dd, *P = SQ + dd, *mK = P + ddv, *G1 = mK + d, *G2 = G1 + ddv, *G3 = G2 + ddv;
+    const float *h1 = G3 + ddv, *h2 = h1 + d, *h3 = h2 + d;
+    float *out = L.init(ws, hd);
+    for (long long i = threadIdx.x; i < ddv + d; i += blockDim.x) {
+        const bool isF = i < ddv;
+        const int r = isF ? (int)(i / dv) : (int)(i - ddv), cc = isF ? (int)(i % dv) : 0;
+        float acc = 0.f;
+        for (int x = 0; x < d; ++x) {
+            float skq = 0.f;
+            for (int y = 0; y < d; ++y) skq += SK[(long long)r * d + y] * SQ[(long long)y * d + x];
+            acc += skq * (isF ? P[(long long)x * dv + cc] : mK[x]);
+        }
+        out[i] = acc - (isF ? (G1[i] + G2[i] + G3[i]) : (h1[r] + h2[r] + h3[r]));
+    }
+}
+
+// ---------------------------------------------------------------------------
+// 3. brackets F_c + S^K_p R_c + M_c[S^Q_p] + U_c P_p (and eta), written over F_c / eta_c
+// ---------------------------------------------------------------------------
+template <typename T>
+__global__ void __launch_bounds__(kT3c) c3_bracket_kernel(const T *__restrict__ k, const T *__restrict__ v, float *ws,
+                                                          C3Layout L) {
+    extern __shared__ float sm[];
+    const int c = blockIdx.x, hd = blockIdx.y, W = L.W, d = L.d, dv = L.dv;
+    const int t0 = c * W, w = min(W, L.n - t0);
+    float *Ks = sm, *Vs = Ks + W * d, *T1 = Vs + W * dv, *bq = T1 + W * d, *tmp = bq + W;
+    const T *Kh = k + ((size_t)hd * L.n + t0) * d, *Vh = v + ((size_t)hd * L.n + t0) * dv;
+    for (int i = threadIdx.x; i < W * d; i += blockDim.x) Ks[i] = (i / d) < w ? ld_tok(Kh + i) : 0.f;
+    for (int i = threadIdx.x; i < W * dv; i += blockDim.x) Vs[i] = (i / dv) < w ? ld_tok(Vh + i) : 0.f;
+    __syncthreads();
+    float *rec = L.loc(ws, hd, c);
+    const float *pr = L.pre(ws, hd, c);
+    const float *SKp = pr + L.pSK, *SQp = pr + L.pSQ, *Pp = pr + L.pP, *mp = pr + L.pm;
+    // bq_t = k_t^T S^Q_p k_t
+    smm(T1, W, d, d, [&](int t, int j) { return Ks[t * d + j]; }, [&](int j, int cc) { return SQp[j * d + cc]; });
+    __syncthreads();
+    for (int t = threadIdx.x; t < W; t += blockDim.x) {
+        float s = 0.f;
+        for (int j = 0; j < d; ++j) s += T1[t * d + j] * Ks[t * d + j];
+        bq[t] = s;
+    }
+    __syncthreads();
+    const float *R = rec + L.oR, *U = rec + L.oU, *rr = rec + L.orr;
+    // new F (d x dv) into tmp, then over F_c (every thread reads only its own element of F_c)
+    for (int i = threadIdx.x; i < d * dv; i += blockDim.x) {
+        const int r = i / dv, cc = i % dv;
+        float s = rec[L.oF + i];
+        float a1 = 0.f, a2 = 0.f, a3 = 0.f;
+        for (int x = 0; x < d; ++x) {
+            a1 += SKp[r * d + x] * R[x * dv + cc];
+            a3 += U[r * d + x] * Pp[x * dv + cc];
+        }
+        for (int t = 0; t < W; ++t) a2 += Ks[t * d + r] * bq[t] * Vs[t * dv + cc];
+        rec[L.oF + i] = s + a1 + a2 + a3;
+    }
+    for (int r = threadIdx.x; r < d; r += blockDim.x) {
+        float a1 = 0.f, a2 = 0.f, a3 = 0.f;
+        for (int x = 0; x < d; ++x) {
+            a1 += SKp[r * d + x] * rr[x];
+            a3 += U[r * d + x] * mp[x];
+        }
+        for (int t = 0; t < W; ++t) a2 += Ks[t * d + r] * bq[t];
+        rec[L.oe + r] += a1 + a2 + a3;
+    }
+    (void)tmp;
+}
+
+// 4. exclusive prefix sums of the brackets, starting at F_0, eta_0
+__global__ void __launch_bounds__(kT3c) c3_prefix2_kernel(float *ws, C3Layout L, int has_init) {
+    const int hd = blockIdx.y, d = L.d, dv = L.dv;
+    const long long ddv = (long long)d * dv;
+    const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= ddv + d) return;
+    const bool isF = i < ddv;
+    const long long lo = isF ? L.oF + i : L.oe + (i - ddv), po = isF ? L.pF + i : L.pe + (i - ddv);
+    float run = has_init ? L.init(ws, hd)[i] : 0.f;
+    for (int c = 0; c < L.nc; ++c) {
+        L.pre(ws, hd, c)[po] = run;
+        run += L.loc(ws, hd, c)[lo];
+    }
+}
+
+// ---------------------------------------------------------------------------
+// 5. outputs of a chunk from its carry-in
+// ---------------------------------------------------------------------------
+template <typename T>
+__global__ void __launch_bounds__(kT3c) c3_out_kernel(const T *__restrict__ q, const T *__restrict__ k,
+                                                      const T *__restrict__ v, T *__restrict__ out, float *ws,
+                                                      C3Layout L, int masked, int normalized, float eps) {
+    extern __shared__ float sm[];
+    const int c = blockIdx.x, hd = blockIdx.y, W = L.W, d = L.d, dv = L.dv;
+    const int t0 = c * W, w = min(W, L.n - t0);
+    const int md = d > dv ? d : dv;
+    float *Qs = sm, *Ks = Qs + W * d, *Vs = Ks + W * d, *A = Vs + W * dv, *Cm = A + W * W;
+    float *M1 = Cm + W * W, *M2 = M1 + W * md, *a = M2 + W * md, *b = a + W, *x1 = b + W, *den = x1 + W;
+    load_chunk(q, k, v, Qs, Ks, Vs, hd, t0, w, W, L.n, d, dv);
+    __syncthreads();
+    const float *pr = L.pre(ws, hd, c);
+    const float *SKp = pr + L.pSK, *SQp = pr + L.pSQ, *Pp = pr + L.pP, *mp = pr + L.pm;
+    const float *Fp = pr + L.pF, *ep = pr + L.pe;
+    T *Oh = out + ((size_t)hd * L.n + t0) * dv;
+    if (masked) {
+        smm(A, W, W, d, [&](int t, int j) { return Qs[t * d + j]; }, [&](int j, int s) { return Ks[s * d + j]; });
+        // M1 = K S^Q_p, M2 = Q S^K_p  (W x d)
+        smm(M1, W, d, d, [&](int t, int j) { return Ks[t * d + j]; }, [&](int j, int cc) { return SQp[j * d + cc]; });
+        smm(M2, W, d, d, [&](int t, int j) { return Qs[t * d + j]; }, [&](int j, int cc) { return SKp[j * d + cc]; });
+        __syncthreads();
+        for (int s = threadIdx.x; s < W; s += blockDim.x) {
+            a[s] = A[s * W + s];
+            float bs = 0.f, ys = 0.f, qm = 0.f;
+            for (int j = 0; j < d; ++j) {
+                bs += M1[s * d + j] * Ks[s * d + j];
+                qm += Qs[s * d + j] * mp[j];
+            }
+            for (int u = 0; u < s; ++u) bs += A[u * W + s] * A[u * W + s];
+            for (int j = 0; j <= s; ++j) ys += A[s * W + j];
+            b[s] = bs;
+            x1[s] = qm + ys;  // (Q m_p + (L.A) 1)_s
+        }
+        // C_ts = q_t^T S^K_p q_s + sum_{i<s} A_ti A_si  (s <= t)
+        for (int i = threadIdx.x; i < W * W; i += blockDim.x) {
+            const int t = i / W, s = i % W;
+            float cv = 0.f;
+            if (s <= t) {
+                for (int j = 0; j < d; ++j) cv += M2[t * d + j] * Qs[s * d + j];
+                for (int x = 0; x < s; ++x) cv += A[t * W + x] * A[s * W + x];
+            }
+            Cm[i] = cv;
+        }
+        __syncthreads();
+        // M1 <- G1 = diag(a) Y + diag(b) V with Y = Q P_p + (L.A) V;  M2 <- G2 = diag(a) V
+        for (int i = threadIdx.x; i < W * dv; i += blockDim.x) {
+            const int s = i / dv, cc = i % dv;
+            float y = 0.f;
+            for (int j = 0; j < d; ++j) y += Qs[s * d + j] * Pp[j * dv + cc];
+            for (int j = 0; j <= s; ++j) y += A[s * W + j] * Vs[j * dv + cc];
+            M1[s * dv + cc] = a[s] * y + b[s] * Vs[i];
+            M2[s * dv + cc] = a[s] * Vs[i];
+        }
+        for (int t = threadIdx.x; t < W; t += blockDim.x) {
+            float dn = 0.f;
+            for (int j = 0; j < d; ++j) dn += Qs[t * d + j] * ep[j];
+            for (int s = 0; s <= t; ++s) dn += A[t * W + s] * (a[s] * x1[s] + b[s]) + Cm[t * W + s] * a[s];
+            den[t] = dn;
+        }
+        __syncthreads();
+        for (int i = threadIdx.x; i < w * dv; i += blockDim.x) {
+            const int t = i / dv, cc = i % dv;
+            float num = 0.f;
+            for (int j = 0; j < d; ++j) num += Qs[t * d + j] * Fp[j * dv + cc];
+            for (int s = 0; s <= t; ++s) num += A[t * W + s] * M1[s * dv + cc] + Cm[t * W + s] * M2[s * dv + cc];
+            from_f32(&Oh[i], normalized ? num / (den[t] + eps) : num);
+        }
+    } else {
+        // A = Q K^T; M1 = X = Q S^K_p + (L.A) K
+        smm(A, W, W, d, [&](int t, int j) { return Qs[t * d + j]; }, [&](int j, int s) { return Ks[s * d + j]; });
+        __syncthreads();
+        for (int i = threadIdx.x; i < W * d; i += blockDim.x) {
+            const int t = i / d, cc = i % d;
+            float x = 0.f;
+            for (int j = 0; j < d; ++j) x += Qs[t * d + j] * SKp[j * d + cc];
+            for (int s = 0; s <= t; ++s) x += A[t * W + s] * Ks[s * d + cc];
+            M1[i] = x;
+        }
+        __syncthreads();
+        // Cm = L.(X Q^T); M2 = Z = X S^Q_p + Cm Q
+        for (int i = threadIdx.x; i < W * W; i += blockDim.x) {
+            const int t = i / W, u = i % W;
+            float s = 0.f;
+            if (u <= t)
+                for (int j = 0; j < d; ++j) s += M1[t * d + j] * Qs[u * d + j];
+            Cm[i] = s;
+        }
+        __syncthreads();
+        for (int i = threadIdx.x; i < W * d; i += blockDim.x) {
+            const int t = i / d, cc = i % d;
+            float z = 0.f;
+            for (int j = 0; j < d; ++j) z += M1[t * d + j] * SQp[j * d + cc];
+            for (int u = 0; u <= t; ++u) z += Cm[t * W + u] * Qs[u * d + cc];
+            M2[i] = z;
+        }
+        __syncthreads();
+        // A <- L.(Z K^T); den = Z m_p + A 1
+        for (int i = threadIdx.x; i < W * W; i += blockDim.x) {
+            const int t = i / W, s = i % W;
+            float zk = 0.f;
+            if (s <= t)
+                for (int j = 0; j < d; ++j) zk += M2[t * d + j] * Ks[s * d + j];
+            A[i] = zk;
+        }
+        __syncthreads();
+        for (int t = threadIdx.x; t < W; t += blockDim.x) {
+            float dn = 0.f;
+            for (int j = 0; j < d; ++j) dn += M2[t * d + j] * mp[j];
+            for (int s = 0; s <= t; ++s) dn += A[t * W + s];
+            den[t] = dn;
+        }
+        __syncthreads();
+        for (int i = threadIdx.x; i < w * dv; i += blockDim.x) {
+            const int t = i / dv, cc = i % dv;
+            float num = 0.f;
+            for (int j = 0; j < d; ++j) num += M2[t * d + j] * Pp[j * dv + cc];
+            for (int s = 0; s <= t; ++s) num += A[t * W + s] * Vs[s * dv + cc];
+            from_f32(&Oh[i], normalized ? num / (den[t] + eps) : num);
+        }
+    }
+}
+
+size_t smem_local(const C3Layout &L) {
+    return sizeof(float) * ((size_t)L.W * (2 * L.d + 2 * L.dv) + (size_t)L.W * L.W + 4 * L.W);
+}
+size_t smem_bracket(const C3Layout &L) {
+    return sizeof(float) * ((size_t)L.W * (2 * L.d + L.dv) + 2 * L.W);
+}
+size_t smem_out(const C3Layout &L) {
+    const int md = L.d > L.dv ? L.d : L.dv;
+    return sizeof(float) * ((size_t)L.W * (2 * L.d + L.dv) + 2 * (size_t)L.W * L.W + 2 * (size_t)L.W * md + 4 * L.W);
+}
+
+template <typename T>
+cudaError_t launch_all(const Fwd2 &p, const C3Layout &L, float *ws, cudaStream_t s) {
+    const T *q = static_cast<const T *>(p.q), *k = static_cast<const T *>(p.k), *v = static_cast<const T *>(p.v);
+    T *out = static_cast<T *>(p.out);
+    cudaError_t e;
+    const dim3 grid(L.nc, L.BH);
+    if ((e = cudaFuncSetAttribute(c3_local_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_local(L))))
+        return e;
+    if ((e = cudaFuncSetAttribute(c3_bracket_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  (int)smem_bracket(L))))
+        return e;
+    if ((e = cudaFuncSetAttribute(c3_out_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_out(L))))
+        return e;
+    c3_local_kernel<T><<<grid, kT3c, smem_local(L), s>>>(q, k, v, ws, L, p.masked);
+    const long long n1 = 2LL * p.d * p.d + (long long)p.d * p.dv + p.d;
+    c3_prefix1_kernel<<<dim3((unsigned)((n1 + kT3c - 1) / kT3c), L.BH), kT3c, 0, s>>>(ws, L, p.state_in);
+    if (p.masked) {
+        if (p.state_in) c3_init_kernel<<<L.BH, kT3c, 0, s>>>(ws, L, p.state_in);
+        c3_bracket_kernel<T><<<grid, kT3c, smem_bracket(L), s>>>(k, v, ws, L);
+        const long long n2 = (long long)p.d * p.dv + p.d;
+        c3_prefix2_kernel<<<dim3((unsigned)((n2 + kT3c - 1) / kT3c), L.BH), kT3c, 0, s>>>(ws, L,
+                                                                                       p.state_in ? 1 : 0);
+    }
+    c3_out_kernel<T><<<grid, kT3c, smem_out(L), s>>>(q, k, v, out, ws, L, p.masked, p.normalized, p.eps);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+size_t chunked3_workspace_bytes(int BH, int n, int d, int dv, int chunk) {
+    if (n <= 0 || BH <= 0) return kWsHeaderBytes;
+    return kWsHeaderBytes + sizeof(float) * (size_t)c3_layout(BH, n, d, dv, chunk).total;
+}
+
+// the per-chunk records grow like (n / chunk) * (5 d^2 + 5 d dv); above 1 GiB the
+// serial kernel (whose scratch is one state per head) serves the call instead
+bool chunked3_eligible(int BH, int n, int d, int dv, int chunk) {
+    return BH <= 65535 && chunked3_workspace_bytes(BH, n, d, dv, chunk) <= (size_t(1) << 30);
+}
+
+cudaError_t chunked3_forward(const Fwd2 &p, cudaStream_t stream) {
+    if (p.n <= 0 || p.BH <= 0) return cudaSuccess;
+    const C3Layout L = c3_layout(p.BH, p.n, p.d, p.dv, p.chunk);
+    float *ws = reinterpret_cast<float *>(p.ws + kWsHeaderBytes);
+    if (p.dt == HLA_BF16) return launch_all<__nv_bfloat16>(p, L, ws, stream);
+    return launch_all<float>(p, L, ws, stream);
+}
+
+}  // namespace hla

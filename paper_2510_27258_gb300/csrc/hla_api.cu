@@ -102,7 +102,10 @@ size_t hla2_workspace_bytes(int B, int H, int n, int d, int dv, int chunk, hla_d
 size_t hla3_workspace_bytes(int B, int H, int n, int d, int dv, int chunk, hla_dtype dt) {
     if (B < 0 || H < 0 || n < 0 || !dim_ok(d) || !dim_ok(dv) || chunk < 1 || chunk > 128) return 0;
     if (dt != HLA_F32 && dt != HLA_BF16) return 0;
-    return align_up(generic3_workspace_bytes(B * H, n, d, dv, chunk), 256);
+    const int BH = B * H;
+    const size_t g = generic3_workspace_bytes(BH, n, d, dv, chunk);
+    const size_t c = chunked3_eligible(BH, n, d, dv, chunk) ? chunked3_workspace_bytes(BH, n, d, dv, chunk) : 0;
+    return align_up(g > c ? g : c, 256);
 }
 
 hla_status hla2_forward(const void *q, const void *k, const void *v, void *out, hla_dtype dt, int B, int H, int n,
@@ -178,6 +181,9 @@ hla_status hla3_forward(const void *q, const void *k, const void *v, void *out, 
     if (st != HLA_OK) return st;
     Fwd2 p{q, k, v, out, dt, B * H, n, d, dv, masked, normalized, eps, chunk, state_in, state_out,
            static_cast<char *>(workspace), workspace_bytes};
+    // chunk-parallel unless the final state is wanted (the serial kernel also carries G1..G3, h1..h3)
+    if (!state_out && chunked3_eligible(B * H, n, d, dv, chunk))
+        return cuda_status(chunked3_forward(p, s), "third-order forward (chunked)");
     return cuda_status(generic3_forward(p, s), "third-order forward");
 }
 

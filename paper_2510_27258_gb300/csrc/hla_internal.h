@@ -71,5 +71,9 @@ cudaError_t step2_launch(const void *q, const void *k, const void *v, void *out,
 // third order
 size_t generic3_workspace_bytes(int BH, int n, int d, int dv, int chunk);
 cudaError_t generic3_forward(const Fwd2 &p, cudaStream_t stream);
+// chunk-parallel third order (no state_out)
+size_t chunked3_workspace_bytes(int BH, int n, int d, int dv, int chunk);
+bool chunked3_eligible(int BH, int n, int d, int dv, int chunk);
+cudaError_t chunked3_forward(const Fwd2 &p, cudaStream_t stream);
 
 }  // namespace hla
