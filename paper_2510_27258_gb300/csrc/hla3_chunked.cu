@@ -43,6 +43,7 @@ constexpr int kT3c = 256;
 
 struct C3Layout {
     int BH, n, d, dv, W, nc;
+    int stage_bracket;  // the bracket kernel copies its d x d / d x dv operands to shared memory
     long long rec_loc, rec_pre, oSK, oSQ, oU, oP, oF, oR, om, oe, orr;  // local record offsets (floats)
     long long pSK, pSQ, pP, pm, pF, pe;                                  // prefix record offsets
     long long loc_base, pre_base, init_base, total;
@@ -79,68 +80,77 @@ C3Layout c3_layout(int BH, int n, int d, int dv, int chunk) {
     L.pre_base = L.loc_base + (long long)BH * L.nc * L.rec_loc;
     L.init_base = L.pre_base + (long long)BH * L.nc * L.rec_pre;
     L.total = L.init_base + (long long)BH * (ddv + d);
+    L.stage_bracket = (3 * dd + 2 * ddv) * 4 <= 96 * 1024;
     return L;
 }
 
 template <typename T>
 __device__ __forceinline__ float ld_tok(const T *p) { return to_f32(*p); }
 
-// dst[r][c] (row-major, ld = cols) = sum_k A(r,k) B(k,c) with accessor lambdas
+// dst[r * ld + c] = sum_k A(r,k) B(k,c) with accessor lambdas
 template <typename FA, typename FB>
-__device__ __forceinline__ void smm(float *dst, int rows, int cols, int kdim, FA a, FB b) {
+__device__ __forceinline__ void smm(float *dst, int ld, int rows, int cols, int kdim, FA a, FB b) {
     for (int i = threadIdx.x; i < rows * cols; i += blockDim.x) {
         const int r = i / cols, c = i % cols;
         float s = 0.f;
         for (int k = 0; k < kdim; ++k) s += a(r, k) * b(k, c);
-        dst[i] = s;
+        dst[r * ld + c] = s;
     }
 }
 
-// loads the chunk's Q, K (w x d) and V (w x dv) as fp32; rows past the sequence are zero
+// loads the chunk's Q, K (w x d) and V (w x dv) as fp32 with row strides d + 1 and dv + 1
+// (shared-memory rows one float longer than the data, so that column walks hit distinct
+// banks); rows past the sequence are zero
 template <typename T>
 __device__ void load_chunk(const T *q, const T *k, const T *v, float *Qs, float *Ks, float *Vs, int hd, int t0,
                            int w, int W, int n, int d, int dv) {
     const T *Qh = q + ((size_t)hd * n + t0) * d, *Kh = k + ((size_t)hd * n + t0) * d;
     const T *Vh = v + ((size_t)hd * n + t0) * dv;
     for (int i = threadIdx.x; i < W * d; i += blockDim.x) {
-        const int r = i / d;
-        Qs[i] = r < w ? ld_tok(Qh + i) : 0.f;
-        Ks[i] = r < w ? ld_tok(Kh + i) : 0.f;
+        const int r = i / d, c = i % d;
+        Qs[r * (d + 1) + c] = r < w ? ld_tok(Qh + i) : 0.f;
+        Ks[r * (d + 1) + c] = r < w ? ld_tok(Kh + i) : 0.f;
     }
-    for (int i = threadIdx.x; i < W * dv; i += blockDim.x) Vs[i] = (i / dv) < w ? ld_tok(Vh + i) : 0.f;
+    for (int i = threadIdx.x; i < W * dv; i += blockDim.x) {
+        const int r = i / dv, c = i % dv;
+        Vs[r * (dv + 1) + c] = r < w ? ld_tok(Vh + i) : 0.f;
+    }
 }
 
 // ---------------------------------------------------------------------------
 // 1. chunk-local summaries
 // ---------------------------------------------------------------------------
+// Shared-memory matrices use row strides one longer than their width (ld = d + 1,
+// lv = dv + 1, lw = W + 1, lm = max(d, dv) + 1).
 template <typename T>
 __global__ void __launch_bounds__(kT3c) c3_local_kernel(const T *__restrict__ q, const T *__restrict__ k,
                                                         const T *__restrict__ v, float *ws, C3Layout L, int masked) {
     extern __shared__ float sm[];
     const int c = blockIdx.x, hd = blockIdx.y, W = L.W, d = L.d, dv = L.dv;
+    const int ld = d + 1, lv = dv + 1, lw = W + 1;
     const int t0 = c * W, w = min(W, L.n - t0);
-    float *Qs = sm, *Ks = Qs + W * d, *Vs = Ks + W * d, *A = Vs + W * dv, *Z = A + W * W, *a = Z + W * dv;
+    float *Qs = sm, *Ks = Qs + W * ld, *Vs = Ks + W * ld, *A = Vs + W * lv, *Z = A + W * lw, *a = Z + W * lv;
     float *zeta = a + W, *b = zeta + W, *ym = b + W;
     load_chunk(q, k, v, Qs, Ks, Vs, hd, t0, w, W, L.n, d, dv);
     __syncthreads();
     float *rec = L.loc(ws, hd, c);
     // first-order sums
-    smm(rec + L.oSK, d, d, W, [&](int r, int t) { return Ks[t * d + r]; }, [&](int t, int cc) { return Ks[t * d + cc]; });
-    smm(rec + L.oSQ, d, d, W, [&](int r, int t) { return Qs[t * d + r]; }, [&](int t, int cc) { return Qs[t * d + cc]; });
-    smm(rec + L.oP, d, dv, W, [&](int r, int t) { return Ks[t * d + r]; }, [&](int t, int cc) { return Vs[t * dv + cc]; });
+    smm(rec + L.oSK, d, d, d, W, [&](int r, int t) { return Ks[t * ld + r]; }, [&](int t, int cc) { return Ks[t * ld + cc]; });
+    smm(rec + L.oSQ, d, d, d, W, [&](int r, int t) { return Qs[t * ld + r]; }, [&](int t, int cc) { return Qs[t * ld + cc]; });
+    smm(rec + L.oP, dv, d, dv, W, [&](int r, int t) { return Ks[t * ld + r]; }, [&](int t, int cc) { return Vs[t * lv + cc]; });
     for (int r = threadIdx.x; r < d; r += blockDim.x) {
         float s = 0.f;
-        for (int t = 0; t < W; ++t) s += Ks[t * d + r];
+        for (int t = 0; t < W; ++t) s += Ks[t * ld + r];
         rec[L.om + r] = s;
     }
     if (!masked) return;
-    smm(A, W, W, d, [&](int t, int j) { return Qs[t * d + j]; }, [&](int j, int s) { return Ks[s * d + j]; });
+    smm(A, lw, W, W, d, [&](int t, int j) { return Qs[t * ld + j]; }, [&](int j, int s) { return Ks[s * ld + j]; });
     __syncthreads();
     for (int t = threadIdx.x; t < W; t += blockDim.x) {
-        a[t] = A[t * W + t];
+        a[t] = A[t * lw + t];
         float bs = 0.f, ys = 0.f;
-        for (int u = 0; u < t; ++u) bs += A[u * W + t] * A[u * W + t];
-        for (int j = 0; j <= t; ++j) ys += A[t * W + j];
+        for (int u = 0; u < t; ++u) bs += A[u * lw + t] * A[u * lw + t];
+        for (int j = 0; j <= t; ++j) ys += A[t * lw + j];
         b[t] = bs;
         ym[t] = ys;
     }
@@ -149,29 +159,51 @@ __global__ void __launch_bounds__(kT3c) c3_local_kernel(const T *__restrict__ q,
     for (int i = threadIdx.x; i < W * dv; i += blockDim.x) {
         const int t = i / dv, cc = i % dv;
         float y = 0.f, nv = 0.f;
-        for (int j = 0; j <= t; ++j) y += A[t * W + j] * Vs[j * dv + cc];
-        for (int s = t + 1; s < W; ++s) nv += A[s * W + t] * a[s] * Vs[s * dv + cc];
-        Z[i] = a[t] * y + b[t] * Vs[i] + nv;
+        for (int j = 0; j <= t; ++j) y += A[t * lw + j] * Vs[j * lv + cc];
+        for (int s = t + 1; s < W; ++s) nv += A[s * lw + t] * a[s] * Vs[s * lv + cc];
+        Z[t * lv + cc] = a[t] * y + b[t] * Vs[t * lv + cc] + nv;
     }
     for (int t = threadIdx.x; t < W; t += blockDim.x) {
         float nv = 0.f;
-        for (int s = t + 1; s < W; ++s) nv += A[s * W + t] * a[s];
+        for (int s = t + 1; s < W; ++s) nv += A[s * lw + t] * a[s];
         zeta[t] = a[t] * ym[t] + b[t] + nv;
     }
     __syncthreads();
-    smm(rec + L.oF, d, dv, W, [&](int r, int t) { return Ks[t * d + r]; }, [&](int t, int cc) { return Z[t * dv + cc]; });
-    smm(rec + L.oR, d, dv, W, [&](int r, int t) { return Qs[t * d + r] * a[t]; },
-        [&](int t, int cc) { return Vs[t * dv + cc]; });
-    smm(rec + L.oU, d, d, W, [&](int r, int t) { return Ks[t * d + r] * a[t]; },
-        [&](int t, int cc) { return Qs[t * d + cc]; });
+    smm(rec + L.oF, dv, d, dv, W, [&](int r, int t) { return Ks[t * ld + r]; }, [&](int t, int cc) { return Z[t * lv + cc]; });
+    smm(rec + L.oR, dv, d, dv, W, [&](int r, int t) { return Qs[t * ld + r] * a[t]; },
+        [&](int t, int cc) { return Vs[t * lv + cc]; });
+    smm(rec + L.oU, d, d, d, W, [&](int r, int t) { return Ks[t * ld + r] * a[t]; },
+        [&](int t, int cc) { return Qs[t * ld + cc]; });
     for (int r = threadIdx.x; r < d; r += blockDim.x) {
         float se = 0.f, sr = 0.f;
         for (int t = 0; t < W; ++t) {
-            se += Ks[t * d + r] * zeta[t];
-            sr += Qs[t * d + r] * a[t];
+            se += Ks[t * ld + r] * zeta[t];
+            sr += Qs[t * ld + r] * a[t];
         }
         rec[L.oe + r] = se;
         rec[L.orr + r] = sr;
+    }
+}
+
+// exclusive scan of one element over the chunks of a head: pre[c][po] = run + sum_{c'<c} loc[c'][lo]
+// (eight loads in flight at a time; the additions stay in chunk order)
+__device__ __forceinline__ void scan_chunks(float *ws, const C3Layout &L, int hd, long long lo, long long po, float run) {
+    const float *src = L.loc(ws, hd, 0) + lo;
+    float *dst = L.pre(ws, hd, 0) + po;
+    int c = 0;
+    for (; c + 8 <= L.nc; c += 8) {
+        float x[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) x[u] = __ldcg(src + (long long)(c + u) * L.rec_loc);
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+            dst[(long long)(c + u) * L.rec_pre] = run;
+            run += x[u];
+        }
+    }
+    for (; c < L.nc; ++c) {
+        dst[(long long)c * L.rec_pre] = run;
+        run += __ldcg(src + (long long)c * L.rec_loc);
     }
 }
 
@@ -184,17 +216,14 @@ __global__ void __launch_bounds__(kT3c) c3_prefix1_kernel(float *ws, C3Layout L,
     const long long nel = 2 * dd + ddv + d;
     const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
     if (i >= nel) return;
-    long long lo, po, so;  // local offset, prefix offset, offset in the state tuple [SK | SQ | P | mK | ...]
-    if (i < dd) { lo = L.oSK + i; po = L.pSK + i; so = i; }
-    else if (i < 2 * dd) { lo = L.oSQ + (i - dd); po = L.pSQ + (i - dd); so = i; }
-    else if (i < 2 * dd + ddv) { lo = L.oP + (i - 2 * dd); po = L.pP + (i - 2 * dd); so = i; }
-    else { lo = L.om + (i - 2 * dd - ddv); po = L.pm + (i - 2 * dd - ddv); so = i; }
+    long long lo, po;  // local and prefix offsets; i is also the offset in the state tuple [SK | SQ | P | mK | ...]
+    if (i < dd) { lo = L.oSK + i; po = L.pSK + i; }
+    else if (i < 2 * dd) { lo = L.oSQ + (i - dd); po = L.pSQ + (i - dd); }
+    else if (i < 2 * dd + ddv) { lo = L.oP + (i - 2 * dd); po = L.pP + (i - 2 * dd); }
+    else { lo = L.om + (i - 2 * dd - ddv); po = L.pm + (i - 2 * dd - ddv); }
     const long long st_len = 2 * dd + 4 * ddv + 4 * (long long)d;
-    float run = state_in ? state_in[(long long)hd * st_len + so] : 0.f;
-    for (int c = 0; c < L.nc; ++c) {
-        L.pre(ws, hd, c)[po] = run;
-        run += L.loc(ws, hd, c)[lo];
-    }
+    float run = state_in ? state_in[(long long)hd * st_len + i] : 0.f;
+    scan_chunks(ws, L, hd, lo, po, run);
 }
 
 // corrected initial carry F_0 = S^K S^Q P - G1 - G2 - G3, eta_0 = S^K S^Q m - h1 - h2 - h3
@@ -226,36 +255,45 @@ __global__ void __launch_bounds__(kT3c) c3_bracket_kernel(const T *__restrict__ 
                                                           C3Layout L) {
     extern __shared__ float sm[];
     const int c = blockIdx.x, hd = blockIdx.y, W = L.W, d = L.d, dv = L.dv;
+    const int ld = d + 1, lv = dv + 1;
     const int t0 = c * W, w = min(W, L.n - t0);
-    float *Ks = sm, *Vs = Ks + W * d, *T1 = Vs + W * dv, *bq = T1 + W * d, *tmp = bq + W;
+    float *Ks = sm, *Vs = Ks + W * ld, *T1 = Vs + W * lv, *bq = T1 + W * ld, *stage = bq + W;
     const T *Kh = k + ((size_t)hd * L.n + t0) * d, *Vh = v + ((size_t)hd * L.n + t0) * dv;
-    for (int i = threadIdx.x; i < W * d; i += blockDim.x) Ks[i] = (i / d) < w ? ld_tok(Kh + i) : 0.f;
-    for (int i = threadIdx.x; i < W * dv; i += blockDim.x) Vs[i] = (i / dv) < w ? ld_tok(Vh + i) : 0.f;
+    for (int i = threadIdx.x; i < W * d; i += blockDim.x) Ks[(i / d) * ld + i % d] = (i / d) < w ? ld_tok(Kh + i) : 0.f;
+    for (int i = threadIdx.x; i < W * dv; i += blockDim.x)
+        Vs[(i / dv) * lv + i % dv] = (i / dv) < w ? ld_tok(Vh + i) : 0.f;
     __syncthreads();
     float *rec = L.loc(ws, hd, c);
     const float *pr = L.pre(ws, hd, c);
     const float *SKp = pr + L.pSK, *SQp = pr + L.pSQ, *Pp = pr + L.pP, *mp = pr + L.pm;
+    const float *R = rec + L.oR, *U = rec + L.oU, *rr = rec + L.orr;
+    if (L.stage_bracket) {  // copies of the d x d and d x dv operands in shared memory
+        const int dd = d * d, ddv = d * dv;
+        float *sSK = stage, *sSQ = sSK + dd, *sU = sSQ + dd, *sR = sU + dd, *sP = sR + ddv;
+        for (int i = threadIdx.x; i < dd; i += blockDim.x) { sSK[i] = SKp[i]; sSQ[i] = SQp[i]; sU[i] = U[i]; }
+        for (int i = threadIdx.x; i < ddv; i += blockDim.x) { sR[i] = R[i]; sP[i] = Pp[i]; }
+        SKp = sSK; SQp = sSQ; U = sU; R = sR; Pp = sP;
+        __syncthreads();
+    }
     // bq_t = k_t^T S^Q_p k_t
-    smm(T1, W, d, d, [&](int t, int j) { return Ks[t * d + j]; }, [&](int j, int cc) { return SQp[j * d + cc]; });
+    smm(T1, ld, W, d, d, [&](int t, int j) { return Ks[t * ld + j]; }, [&](int j, int cc) { return SQp[j * d + cc]; });
     __syncthreads();
     for (int t = threadIdx.x; t < W; t += blockDim.x) {
         float s = 0.f;
-        for (int j = 0; j < d; ++j) s += T1[t * d + j] * Ks[t * d + j];
+        for (int j = 0; j < d; ++j) s += T1[t * ld + j] * Ks[t * ld + j];
         bq[t] = s;
     }
     __syncthreads();
-    const float *R = rec + L.oR, *U = rec + L.oU, *rr = rec + L.orr;
-    // new F (d x dv) into tmp, then over F_c (every thread reads only its own element of F_c)
+    // every thread reads and rewrites only its own elements of F_c and eta_c
     for (int i = threadIdx.x; i < d * dv; i += blockDim.x) {
         const int r = i / dv, cc = i % dv;
-        float s = rec[L.oF + i];
         float a1 = 0.f, a2 = 0.f, a3 = 0.f;
         for (int x = 0; x < d; ++x) {
             a1 += SKp[r * d + x] * R[x * dv + cc];
             a3 += U[r * d + x] * Pp[x * dv + cc];
         }
-        for (int t = 0; t < W; ++t) a2 += Ks[t * d + r] * bq[t] * Vs[t * dv + cc];
-        rec[L.oF + i] = s + a1 + a2 + a3;
+        for (int t = 0; t < W; ++t) a2 += Ks[t * ld + r] * bq[t] * Vs[t * lv + cc];
+        rec[L.oF + i] += a1 + a2 + a3;
     }
     for (int r = threadIdx.x; r < d; r += blockDim.x) {
         float a1 = 0.f, a2 = 0.f, a3 = 0.f;
@@ -263,10 +301,9 @@ __global__ void __launch_bounds__(kT3c) c3_bracket_kernel(const T *__restrict__ 
             a1 += SKp[r * d + x] * rr[x];
             a3 += U[r * d + x] * mp[x];
         }
-        for (int t = 0; t < W; ++t) a2 += Ks[t * d + r] * bq[t];
+        for (int t = 0; t < W; ++t) a2 += Ks[t * ld + r] * bq[t];
         rec[L.oe + r] += a1 + a2 + a3;
     }
-    (void)tmp;
 }
 
 // 4. exclusive prefix sums of the brackets, starting at F_0, eta_0
@@ -278,10 +315,7 @@ __global__ void __launch_bounds__(kT3c) c3_prefix2_kernel(float *ws, C3Layout L,
     const bool isF = i < ddv;
     const long long lo = isF ? L.oF + i : L.oe + (i - ddv), po = isF ? L.pF + i : L.pe + (i - ddv);
     float run = has_init ? L.init(ws, hd)[i] : 0.f;
-    for (int c = 0; c < L.nc; ++c) {
-        L.pre(ws, hd, c)[po] = run;
-        run += L.loc(ws, hd, c)[lo];
-    }
+    scan_chunks(ws, L, hd, lo, po, run);
 }
 
 // ---------------------------------------------------------------------------
@@ -293,10 +327,10 @@ __global__ void __launch_bounds__(kT3c) c3_out_kernel(const T *__restrict__ q, c
                                                       C3Layout L, int masked, int normalized, float eps) {
     extern __shared__ float sm[];
     const int c = blockIdx.x, hd = blockIdx.y, W = L.W, d = L.d, dv = L.dv;
+    const int ld = d + 1, lv = dv + 1, lw = W + 1, lm = (d > dv ? d : dv) + 1;
     const int t0 = c * W, w = min(W, L.n - t0);
-    const int md = d > dv ? d : dv;
-    float *Qs = sm, *Ks = Qs + W * d, *Vs = Ks + W * d, *A = Vs + W * dv, *Cm = A + W * W;
-    float *M1 = Cm + W * W, *M2 = M1 + W * md, *a = M2 + W * md, *b = a + W, *x1 = b + W, *den = x1 + W;
+    float *Qs = sm, *Ks = Qs + W * ld, *Vs = Ks + W * ld, *A = Vs + W * lv, *Cm = A + W * lw;
+    float *M1 = Cm + W * lw, *M2 = M1 + W * lm, *a = M2 + W * lm, *b = a + W, *x1 = b + W, *den = x1 + W;
     load_chunk(q, k, v, Qs, Ks, Vs, hd, t0, w, W, L.n, d, dv);
     __syncthreads();
     const float *pr = L.pre(ws, hd, c);
@@ -304,20 +338,20 @@ __global__ void __launch_bounds__(kT3c) c3_out_kernel(const T *__restrict__ q, c
     const float *Fp = pr + L.pF, *ep = pr + L.pe;
     T *Oh = out + ((size_t)hd * L.n + t0) * dv;
     if (masked) {
-        smm(A, W, W, d, [&](int t, int j) { return Qs[t * d + j]; }, [&](int j, int s) { return Ks[s * d + j]; });
+        smm(A, lw, W, W, d, [&](int t, int j) { return Qs[t * ld + j]; }, [&](int j, int s) { return Ks[s * ld + j]; });
         // M1 = K S^Q_p, M2 = Q S^K_p  (W x d)
-        smm(M1, W, d, d, [&](int t, int j) { return Ks[t * d + j]; }, [&](int j, int cc) { return SQp[j * d + cc]; });
-        smm(M2, W, d, d, [&](int t, int j) { return Qs[t * d + j]; }, [&](int j, int cc) { return SKp[j * d + cc]; });
+        smm(M1, lm, W, d, d, [&](int t, int j) { return Ks[t * ld + j]; }, [&](int j, int cc) { return SQp[j * d + cc]; });
+        smm(M2, lm, W, d, d, [&](int t, int j) { return Qs[t * ld + j]; }, [&](int j, int cc) { return SKp[j * d + cc]; });
         __syncthreads();
         for (int s = threadIdx.x; s < W; s += blockDim.x) {
-            a[s] = A[s * W + s];
+            a[s] = A[s * lw + s];
             float bs = 0.f, ys = 0.f, qm = 0.f;
             for (int j = 0; j < d; ++j) {
-                bs += M1[s * d + j] * Ks[s * d + j];
-                qm += Qs[s * d + j] * mp[j];
+                bs += M1[s * lm + j] * Ks[s * ld + j];
+                qm += Qs[s * ld + j] * mp[j];
             }
-            for (int u = 0; u < s; ++u) bs += A[u * W + s] * A[u * W + s];
-            for (int j = 0; j <= s; ++j) ys += A[s * W + j];
+            for (int u = 0; u < s; ++u) bs += A[u * lw + s] * A[u * lw + s];
+            for (int j = 0; j <= s; ++j) ys += A[s * lw + j];
             b[s] = bs;
             x1[s] = qm + ys;  // (Q m_p + (L.A) 1)_s
         }
@@ -326,45 +360,45 @@ __global__ void __launch_bounds__(kT3c) c3_out_kernel(const T *__restrict__ q, c
             const int t = i / W, s = i % W;
             float cv = 0.f;
             if (s <= t) {
-                for (int j = 0; j < d; ++j) cv += M2[t * d + j] * Qs[s * d + j];
-                for (int x = 0; x < s; ++x) cv += A[t * W + x] * A[s * W + x];
+                for (int j = 0; j < d; ++j) cv += M2[t * lm + j] * Qs[s * ld + j];
+                for (int x = 0; x < s; ++x) cv += A[t * lw + x] * A[s * lw + x];
             }
-            Cm[i] = cv;
+            Cm[t * lw + s] = cv;
         }
         __syncthreads();
         // M1 <- G1 = diag(a) Y + diag(b) V with Y = Q P_p + (L.A) V;  M2 <- G2 = diag(a) V
         for (int i = threadIdx.x; i < W * dv; i += blockDim.x) {
             const int s = i / dv, cc = i % dv;
             float y = 0.f;
-            for (int j = 0; j < d; ++j) y += Qs[s * d + j] * Pp[j * dv + cc];
-            for (int j = 0; j <= s; ++j) y += A[s * W + j] * Vs[j * dv + cc];
-            M1[s * dv + cc] = a[s] * y + b[s] * Vs[i];
-            M2[s * dv + cc] = a[s] * Vs[i];
+            for (int j = 0; j < d; ++j) y += Qs[s * ld + j] * Pp[j * dv + cc];
+            for (int j = 0; j <= s; ++j) y += A[s * lw + j] * Vs[j * lv + cc];
+            M1[s * lm + cc] = a[s] * y + b[s] * Vs[s * lv + cc];
+            M2[s * lm + cc] = a[s] * Vs[s * lv + cc];
         }
         for (int t = threadIdx.x; t < W; t += blockDim.x) {
             float dn = 0.f;
-            for (int j = 0; j < d; ++j) dn += Qs[t * d + j] * ep[j];
-            for (int s = 0; s <= t; ++s) dn += A[t * W + s] * (a[s] * x1[s] + b[s]) + Cm[t * W + s] * a[s];
+            for (int j = 0; j < d; ++j) dn += Qs[t * ld + j] * ep[j];
+            for (int s = 0; s <= t; ++s) dn += A[t * lw + s] * (a[s] * x1[s] + b[s]) + Cm[t * lw + s] * a[s];
             den[t] = dn;
         }
         __syncthreads();
         for (int i = threadIdx.x; i < w * dv; i += blockDim.x) {
             const int t = i / dv, cc = i % dv;
             float num = 0.f;
-            for (int j = 0; j < d; ++j) num += Qs[t * d + j] * Fp[j * dv + cc];
-            for (int s = 0; s <= t; ++s) num += A[t * W + s] * M1[s * dv + cc] + Cm[t * W + s] * M2[s * dv + cc];
+            for (int j = 0; j < d; ++j) num += Qs[t * ld + j] * Fp[j * dv + cc];
+            for (int s = 0; s <= t; ++s) num += A[t * lw + s] * M1[s * lm + cc] + Cm[t * lw + s] * M2[s * lm + cc];
             from_f32(&Oh[i], normalized ? num / (den[t] + eps) : num);
         }
     } else {
         // A = Q K^T; M1 = X = Q S^K_p + (L.A) K
-        smm(A, W, W, d, [&](int t, int j) { return Qs[t * d + j]; }, [&](int j, int s) { return Ks[s * d + j]; });
+        smm(A, lw, W, W, d, [&](int t, int j) { return Qs[t * ld + j]; }, [&](int j, int s) { return Ks[s * ld + j]; });
         __syncthreads();
         for (int i = threadIdx.x; i < W * d; i += blockDim.x) {
             const int t = i / d, cc = i % d;
             float x = 0.f;
-            for (int j = 0; j < d; ++j) x += Qs[t * d + j] * SKp[j * d + cc];
-            for (int s = 0; s <= t; ++s) x += A[t * W + s] * Ks[s * d + cc];
-            M1[i] = x;
+            for (int j = 0; j < d; ++j) x += Qs[t * ld + j] * SKp[j * d + cc];
+            for (int s = 0; s <= t; ++s) x += A[t * lw + s] * Ks[s * ld + cc];
+            M1[t * lm + cc] = x;
         }
         __syncthreads();
         // Cm = L.(X Q^T); M2 = Z = X S^Q_p + Cm Q
@@ -372,16 +406,16 @@ __global__ void __launch_bounds__(kT3c) c3_out_kernel(const T *__restrict__ q, c
             const int t = i / W, u = i % W;
             float s = 0.f;
             if (u <= t)
-                for (int j = 0; j < d; ++j) s += M1[t * d + j] * Qs[u * d + j];
-            Cm[i] = s;
+                for (int j = 0; j < d; ++j) s += M1[t * lm + j] * Qs[u * ld + j];
+            Cm[t * lw + u] = s;
         }
         __syncthreads();
         for (int i = threadIdx.x; i < W * d; i += blockDim.x) {
             const int t = i / d, cc = i % d;
             float z = 0.f;
-            for (int j = 0; j < d; ++j) z += M1[t * d + j] * SQp[j * d + cc];
-            for (int u = 0; u <= t; ++u) z += Cm[t * W + u] * Qs[u * d + cc];
-            M2[i] = z;
+            for (int j = 0; j < d; ++j) z += M1[t * lm + j] * SQp[j * d + cc];
+            for (int u = 0; u <= t; ++u) z += Cm[t * lw + u] * Qs[u * ld + cc];
+            M2[t * lm + cc] = z;
         }
         __syncthreads();
         // A <- L.(Z K^T); den = Z m_p + A 1
@@ -389,36 +423,38 @@ __global__ void __launch_bounds__(kT3c) c3_out_kernel(const T *__restrict__ q, c
             const int t = i / W, s = i % W;
             float zk = 0.f;
             if (s <= t)
-                for (int j = 0; j < d; ++j) zk += M2[t * d + j] * Ks[s * d + j];
-            A[i] = zk;
+                for (int j = 0; j < d; ++j) zk += M2[t * lm + j] * Ks[s * ld + j];
+            A[t * lw + s] = zk;
         }
         __syncthreads();
         for (int t = threadIdx.x; t < W; t += blockDim.x) {
             float dn = 0.f;
-            for (int j = 0; j < d; ++j) dn += M2[t * d + j] * mp[j];
-            for (int s = 0; s <= t; ++s) dn += A[t * W + s];
+            for (int j = 0; j < d; ++j) dn += M2[t * lm + j] * mp[j];
+            for (int s = 0; s <= t; ++s) dn += A[t * lw + s];
             den[t] = dn;
         }
         __syncthreads();
         for (int i = threadIdx.x; i < w * dv; i += blockDim.x) {
             const int t = i / dv, cc = i % dv;
             float num = 0.f;
-            for (int j = 0; j < d; ++j) num += M2[t * d + j] * Pp[j * dv + cc];
-            for (int s = 0; s <= t; ++s) num += A[t * W + s] * Vs[s * dv + cc];
+            for (int j = 0; j < d; ++j) num += M2[t * lm + j] * Pp[j * dv + cc];
+            for (int s = 0; s <= t; ++s) num += A[t * lw + s] * Vs[s * lv + cc];
             from_f32(&Oh[i], normalized ? num / (den[t] + eps) : num);
         }
     }
 }
 
 size_t smem_local(const C3Layout &L) {
-    return sizeof(float) * ((size_t)L.W * (2 * L.d + 2 * L.dv) + (size_t)L.W * L.W + 4 * L.W);
+    return sizeof(float) * ((size_t)L.W * (2 * (L.d + 1) + 2 * (L.dv + 1)) + (size_t)L.W * (L.W + 1) + 4 * L.W);
 }
 size_t smem_bracket(const C3Layout &L) {
-    return sizeof(float) * ((size_t)L.W * (2 * L.d + L.dv) + 2 * L.W);
+    const size_t stage = L.stage_bracket ? 3 * (size_t)L.d * L.d + 2 * (size_t)L.d * L.dv : 0;
+    return sizeof(float) * ((size_t)L.W * (2 * (L.d + 1) + (L.dv + 1)) + L.W + stage);
 }
 size_t smem_out(const C3Layout &L) {
-    const int md = L.d > L.dv ? L.d : L.dv;
-    return sizeof(float) * ((size_t)L.W * (2 * L.d + L.dv) + 2 * (size_t)L.W * L.W + 2 * (size_t)L.W * md + 4 * L.W);
+    const int lm = (L.d > L.dv ? L.d : L.dv) + 1;
+    return sizeof(float) *
+           ((size_t)L.W * (2 * (L.d + 1) + (L.dv + 1)) + 2 * (size_t)L.W * (L.W + 1) + 2 * (size_t)L.W * lm + 4 * L.W);
 }
 
 template <typename T>
