@@ -127,9 +127,11 @@ hla_status hla2_step(const void *q, const void *k, const void *v, void *out, hla
  * on the current device, without launching anything:
  *   0  generic path: fp32 CUDA-core kernels (every supported shape);
  *   1  fused path: one persistent tcgen05/TMA kernel (bf16 tokens, d and dv
- *      in {64, 128}, masked, no state_out; state_in only with d = dv = 128)
- *      on sm_103.  It works in 128-token tiles whatever chunk is (chunk only
- *      changes the rounding, Theorem 2);
+ *      in {64, 128}, masked; state_in only with d = dv = 128) on sm_103, plus
+ *      two small kernels for state_out (C = Q^T V and m = Q^T 1 on the tensor
+ *      cores, then G = S C - D, h = S m - e from the forward's prefixes).  It
+ *      works in 128-token tiles whatever chunk is (chunk only changes the
+ *      rounding, Theorem 2);
  *  -1  the arguments are not supported.
  * *launches (if not NULL) receives the number of kernels the call launches.
  */
@@ -171,9 +173,9 @@ hla_status hla3_forward(const void *q, const void *k, const void *v, void *out, 
  * array in device memory that belongs to the library.  Every GPU on which the
  * library is used holds that array until the process exits.
  *
- * Scope: the arguments for which hla2_forward_path returns 1 (the fused path:
- * bf16 tokens, d and dv in {64, 128}, masked = 1, no state_out, state_in only
- * with d = dv = 128, an sm_103 device); other arguments return
+ * Scope: the arguments for which hla2_forward_path returns 1 without a final
+ * state (the fused path: bf16 tokens, d and dv in {64, 128}, masked = 1,
+ * state_in only with d = dv = 128, an sm_103 device); other arguments return
  * HLA_ERR_UNSUPPORTED.  Sizes whose scratch exceeds 16 MiB (it grows with
  * B*H, about 263 KiB per head, and with B*H*n*4 bytes when normalized) return
  * HLA_ERR_WORKSPACE before anything is launched.

@@ -95,7 +95,7 @@ size_t hla2_workspace_bytes(int B, int H, int n, int d, int dv, int chunk, hla_d
     if (dt != HLA_F32 && dt != HLA_BF16) return 0;
     const int BH = B * H;
     size_t g = generic2_workspace_bytes(BH, n, d, dv, chunk);
-    size_t f = fused2_workspace_bytes(BH, n, d, dv, chunk, dt);
+    size_t f = fused2_workspace_bytes(BH, n, d, dv, chunk, dt, true);
     return align_up(g > f ? g : f, 256);
 }
 
@@ -144,7 +144,7 @@ int hla2_forward_path(int B, int H, int n, int d, int dv, int masked, int normal
     const bool fused = (long long)B * H > 0 && fused2_applicable(p);
     if (launches) {
         if ((long long)B * H == 0) *launches = 0;
-        else if (fused) *launches = 1 + (has_state_in ? 1 : 0);
+        else if (fused) *launches = 1 + (has_state_in ? 1 : 0) + (has_state_out ? 2 : 0);
         else *launches = n > 0 ? 3 : 1;
     }
     return fused ? 1 : 0;

@@ -344,6 +344,10 @@ __device__ __forceinline__ void mma128_ts(uint32_t d_tmem, uint32_t a_tmem, uint
 // ---------------------------------------------------------------------------
 // the kernel
 // ---------------------------------------------------------------------------
+// kState: the final state is wanted.  Then W and R are split hi + lo and the e carry kept
+// whatever the output (as for the normalised output), and D += X_hi^T V + X_lo^T V is issued
+// before O (X_lo is still in slot W), so that the prefixes in the ring are accurate to fp32 level.
+template <bool kState>
 __global__ void __launch_bounds__(kThreads, 1)
 hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                   const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_o, Params p) {
@@ -353,6 +357,9 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const bool issuer = (warp == kIssuerWarp), publisher = (warp == kPubWarp);
+    const bool precise = kState || p.normalized;  // hi + lo splits of W and R
+    const bool need_e = kState || p.normalized;   // the e carry
+    constexpr bool d_lo = kState;                 // D with X_lo, issued before O
 
     // the tile layout needs 1 KiB alignment of the dynamic shared memory
     if (smem_u32(smem) & 1023u) {
@@ -452,11 +459,11 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                     if (j == 0 && !bar_wait(ms, bEpW, tp, p)) break;
                     tc_fence_after();
                     mma128<false, false>(tb + kTX, lk(qs), lk(kSX), 0u);      // X = Q R_hi
-                    if (p.normalized) mma128<false, false>(tb + kTX, lk(qs), lk(kSD), 1u);  // += Q R_lo
+                    if (precise) mma128<false, false>(tb + kTX, lk(qs), lk(kSD), 1u);  // += Q R_lo
                     if (j > 0 && !bar_wait(ms, bEpW, tp, p)) break;  // W (hi, lo) ready
                     tc_fence_after();
                     mma128_ts<true>(tb + kTX, tb + kTA, lm(kK), 1u);          // += W_hi K (W in TMEM)
-                    if (p.normalized) mma128_ts<true>(tb + kTX, tb + kTA + 16, lm(kK), 1u);  // += W_lo K
+                    if (precise) mma128_ts<true>(tb + kTX, tb + kTA + 16, lm(kK), 1u);  // += W_lo K
                     umma_commit(&ms->bar[bEvX]);
                     mma128<true, true>(tb + kTS, lm(kK), lm(kK), 1u);         // S += K^T K
                     umma_commit(&ms->bar[bEvS]);
@@ -471,11 +478,18 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                     if (!bar_wait(ms, bEpT, tp, p)) break;
                     if (!wait_ld(kV)) break;
                     tc_fence_after();
+                    if (d_lo) {  // D to fp32-level accuracy: X_lo is read from slot W before O's staging
+                        mma128<true, true>(tb + kTD, lm(kSX), lm(kV), 1u);    // D += X_hi^T V
+                        mma128<true, true>(tb + kTD, lm(kW), lm(kV), 1u);     // D += X_lo^T V
+                        umma_commit(&ms->bar[bEvD]);
+                    }
                     mma128<false, true>(tb + kTX, lk(qs), lm(kSD), 0u);       // O = Q D_p
                     mma128_ts<true>(tb + kTX, tb + kTA, lm(kV), 1u);          // += T V (T in TMEM)
                     umma_commit(&ms->bar[bEvO]);
-                    mma128<true, true>(tb + kTD, lm(kSX), lm(kV), 1u);        // D += X^T V
-                    umma_commit(&ms->bar[bEvD]);
+                    if (!d_lo) {
+                        mma128<true, true>(tb + kTD, lm(kSX), lm(kV), 1u);    // D += X^T V
+                        umma_commit(&ms->bar[bEvD]);
+                    }
                     if (j + 1 < nt) {  // next tile's A = Q K^T overlaps this tile's output epilogue
                         // A goes to the TMEM columns O has just read T from
                         if (!bar_wait(ms, bEvO, tp, p)) break;
@@ -484,7 +498,7 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                         mma128<false, false>(tb + kTA, lk(qo), lk(kK), 0u);
                         umma_commit(&ms->bar[bEvA]);
                     }
-                    if (!bar_wait(ms, bEvD, tp, p)) break;  // D += X^T V (the last reader of V) done
+                    if (!bar_wait(ms, d_lo ? bEvO : bEvD, tp, p)) break;  // the last reader of V done
                     if (j + 1 < nt) load_tile(kV, &tm_v, head, (t0 + j + 1) * kTile);
                     ++n_tiles;
                 }
@@ -602,7 +616,7 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 tmem_st32(tb + lane_base + kTS + c0, u);
                 // split S_p = cs I + R into R_hi (slot SX) and R_lo (slot SD)
                 if (cq == qd) shift_diag32(sp, lane, cs);
-                store_split32(slot(kSX), slot(kSD), r, c0, sp, p.normalized);
+                store_split32(slot(kSX), slot(kSD), r, c0, sp, precise);
                 // segment-local D carry: the initial state's D for the first segment
                 const float *d0 = (sigma == 0 && p.init_De) ? p.init_De + (size_t)head * (kD * kD + kD) : nullptr;
 #pragma unroll
@@ -643,7 +657,7 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                         split_pack32(f, h, l);
                     }
                     tmem_st16(tb + lane_base + kTA + c0, h);
-                    if (p.normalized) tmem_st16(tb + lane_base + kTA + c0 + 16, l);
+                    if (precise) tmem_st16(tb + lane_base + kTA + c0 + 16, l);
                     tmem_st_wait();
                 }
                 epi_arrive(ms, bEpW);
@@ -683,7 +697,7 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 // while T = Q X^T runs: column sums of X (e carry) and D_p -> bf16 (slot SD; R_lo
                 // there is dead once X is done; D += X^T V is issued after this tile's T hand-off)
                 float ecol = 0.f;
-                if (p.normalized) ecol = warp_colsum32(x);  // column c0 + lane over this warp's rows
+                if (need_e) ecol = warp_colsum32(x);  // column c0 + lane over this warp's rows
                 {
                     float f[32];
                     ld32(tb + lane_base + kTD + c0, f);
@@ -724,9 +738,10 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                     for (int w = 0; w < kEpiWarps; ++w) t += ms->red[w];
                     tr_s += t;
                 }
-                if (p.normalized) {
-                    if (cq == 0) ms->den[r] = ((den_part + ms->part[0][r]) + ms->part[1][r]) + ms->part[2][r];
-                    epi_sync();
+                if (p.normalized && cq == 0)
+                    ms->den[r] = ((den_part + ms->part[0][r]) + ms->part[1][r]) + ms->part[2][r];
+                if (need_e) {
+                    epi_sync();  // the denominator partials are read before part is reused
                     if (qd > 0) ms->part[qd - 1][c0 + lane] = ecol;
                     epi_sync();
                     if (qd == 0)
@@ -761,7 +776,7 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                     float f[32];
                     ld32(tb + lane_base + kTS + c0, f);
                     if (cq == qd) shift_diag32(f, lane, cs);
-                    store_split32(slot(kSX), slot(kSD), r, c0, f, p.normalized);
+                    store_split32(slot(kSX), slot(kSD), r, c0, f, precise);
                     fence_async_smem();
                     epi_arrive(ms, bEpR);  // R of the next tile ready, O read: Q R may start
                 }
@@ -930,8 +945,10 @@ bool make_map(CUtensorMap *m, const void *base, int BH, int n, int inner) {
 }
 
 struct FusedLayout {
-    size_t off_ticket, off_flags, off_ring, off_den, off_init, total;
+    size_t off_ticket, off_flags, off_ring, off_den, off_init, off_part, total, total_state;
 };
+
+int state_groups(int BH, int M);
 
 FusedLayout fused_layout(int BH, int n) {
     FusedLayout L;
@@ -942,6 +959,10 @@ FusedLayout fused_layout(int BH, int n) {
     L.off_den = o; o = align_up(o + sizeof(float) * (size_t)BH * n, 256);
     L.off_init = o; o = align_up(o + sizeof(float) * (size_t)BH * (kD * kD + kD), 256);
     L.total = o;
+    // C / m partials of the final state (only when state_out is asked for)
+    const int M = (n + kTile - 1) / kTile;
+    L.off_part = o; o = align_up(o + sizeof(float) * (size_t)BH * state_groups(BH, M) * (kD * kD + kD), 256);
+    L.total_state = o;
     return L;
 }
 
@@ -959,23 +980,202 @@ int segment_tiles(int BH, int M, int sms) {
     return L < M ? L : M;
 }
 
+
+// ---------------------------------------------------------------------------
+// final state (state_out): C = C_0 + Q^T V and m = m_0 + Q^T 1 on the tensor
+// cores, then the paper tuple from the prefixes the forward left in its ring:
+// S, D = S C - G and e = S m - h of the whole sequence, so G = S C - D and
+// h = S m - e (the D-form of Eq. semidirect read backwards)
+// ---------------------------------------------------------------------------
+constexpr int kCThreads = 160;            // 4 warps read TMEM (one lane quadrant each), warp 4 issues
+constexpr uint32_t kCOnesBytes = 4096;    // 16 x 128 bf16 ones operand (row 0 ones), K-major
+constexpr uint32_t kCSmemBytes = 4 * kTileBytes + kCOnesBytes + 1024;
+constexpr int kCPartFloats = kD * kD + kD;  // C (d x dv) then m (d) of one group of tiles
+
+// C and m of tiles [g * tiles_per, ...) of a head, from tiles of 128 tokens (Q^T V: A = Q^T and
+// B = V both MN-major; m: B = a 16-row K-major operand whose row 0 is ones)
+__global__ void __launch_bounds__(kCThreads, 1)
+state_c_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_v, float *part,
+               int M, int groups, int tiles_per, WsHeader *err) {
+    extern __shared__ __align__(1024) uint8_t csm[];
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int head = blockIdx.x / groups, g = blockIdx.x % groups;
+    const int j0 = g * tiles_per, j1 = min(M, j0 + tiles_per);
+    uint8_t *ones = csm + 4 * kTileBytes;
+    // after the tiles and the ones operand: loads of slot pair 0 / 1, MMAs of pair 0 / 1, all done
+    uint64_t *bars = reinterpret_cast<uint64_t *>(ones + kCOnesBytes);
+    uint32_t &tmem_base_s = *reinterpret_cast<uint32_t *>(bars + 5);
+    int &abort_c = *reinterpret_cast<int *>(bars + 6);
+    if (smem_u32(csm) & 1023u) {
+        if (tid == 0) set_error(err, 98, smem_u32(csm));
+        return;
+    }
+    // ones operand: element (row, token k) of the 128-byte swizzled K-major layout
+    for (int i = tid; i < 16 * 128; i += blockDim.x) {
+        const int row = i / 128, kk = i % 128;
+        const uint32_t off = (kk >> 6) * 2048 + row * 128 + ((((kk & 63) >> 3) ^ (row & 7)) << 4) + (kk & 7) * 2;
+        *reinterpret_cast<uint16_t *>(ones + off) = row == 0 ? (uint16_t)0x3F80 : (uint16_t)0;
+    }
+    if (tid == 0) {
+        for (int b = 0; b < 5; ++b) mbar_init(&bars[b], 1);
+        abort_c = 0;
+        fence_mbar_init();
+    }
+    if (warp == 4) {
+        tmem_alloc(&tmem_base_s, 256);
+        tmem_relinquish();
+    }
+    fence_async_smem();
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tb = tmem_base_s;
+    auto cwait = [&](int b, uint32_t par) {
+        if (abort_c) return false;
+        if (mbar_wait(&bars[b], par, kBarWaitNs)) return true;
+        set_error(err, 150 + b, par);
+        abort_c = 1;
+        return false;
+    };
+    if (warp == 4) {
+        if (lane == 0) {
+            const uint32_t sb4 = smem_u32(csm) >> 4;
+            auto lmn = [&](int s) { return sb4 + (uint32_t)s * (kTileBytes >> 4) + kLboMN; };
+            const uint32_t ones_lo = (smem_u32(ones) >> 4) + kLboK;
+            auto load_pair = [&](int j) {
+                const int sl = (j - j0) & 1;
+                mbar_arrive_expect_tx(&bars[sl], 2 * kTileBytes);
+                uint8_t *qs = csm + (2 * sl) * kTileBytes, *vs = csm + (2 * sl + 1) * kTileBytes;
+                tma_load_3d(qs, &tm_q, &bars[sl], 0, j * kTile, head);
+                tma_load_3d(qs + kBlockBytes, &tm_q, &bars[sl], 64, j * kTile, head);
+                tma_load_3d(vs, &tm_v, &bars[sl], 0, j * kTile, head);
+                tma_load_3d(vs + kBlockBytes, &tm_v, &bars[sl], 64, j * kTile, head);
+            };
+            if (j0 < j1) load_pair(j0);
+            if (j0 + 1 < j1) load_pair(j0 + 1);
+            constexpr uint32_t id_m = idesc_bf16(128, 16, 1, 0);
+            for (int j = j0; j < j1; ++j) {
+                const int i = j - j0, sl = i & 1;
+                if (!cwait(sl, (i >> 1) & 1)) break;
+                tc_fence_after();
+                mma128<true, true>(tb, lmn(2 * sl), lmn(2 * sl + 1), i > 0 ? 1u : 0u);  // C += Q^T V
+#pragma unroll
+                for (int kk = 0; kk < 8; ++kk)  // m += Q^T 1 (column 128)
+                    umma_bf16(tb + 128, (static_cast<uint64_t>(kDescHi) << 32) | (lmn(2 * sl) + kk * 128u),
+                              (static_cast<uint64_t>(kDescHi) << 32) | (ones_lo + (kk >> 2) * 128u + (kk & 3) * 2u),
+                              id_m, (i > 0 || kk > 0) ? 1u : 0u);
+                umma_commit(&bars[2 + sl]);
+                if (j + 2 < j1) {
+                    if (!cwait(2 + sl, (i >> 1) & 1)) break;
+                    load_pair(j + 2);
+                }
+            }
+            umma_commit(&bars[4]);
+        }
+        __syncwarp();
+    } else {
+        // C rows (features f = 32 warp + lane), 128 columns, then m
+        float *out = part + (size_t)blockIdx.x * kCPartFloats;
+        const uint32_t lb = (uint32_t)(32 * warp) << 16;
+        const int f = 32 * warp + lane;
+        const bool ok = (j0 < j1) && cwait(4, 0);
+        tc_fence_after();
+        for (int c0 = 0; c0 < kD; c0 += 32) {
+            float v[32];
+            if (ok) ld32(tb + lb + c0, v);
+            for (int jj = 0; jj < 32; ++jj) out[(size_t)f * kD + c0 + jj] = ok ? v[jj] : 0.f;
+        }
+        float mv[32];
+        if (ok) ld32(tb + lb + 128, mv);
+        out[kD * kD + f] = ok ? mv[0] : 0.f;
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 4) {
+        tc_fence_after();
+        tmem_dealloc(tb, 256);
+    }
+}
+
+// per head: the paper tuple [S | C | m | G | h] (d x d, d x dv, d, d x dv, d) from the ring slot of
+// the head's last segment and the C / m partials; state_in (may alias state_out) supplies C_0, m_0
+__global__ void __launch_bounds__(256) state_finalize_kernel(const float *ring, int last_slot, const float *part,
+                                                             int groups, const float *state_in, float *state_out,
+                                                             int d, int dv) {
+    extern __shared__ float fs[];
+    float *S = fs, *C = S + kD * kD, *m = C + kD * kD;  // 128 x 128, 128 x 128, 128 (zero outside d, dv)
+    const int hd = blockIdx.x, tid = threadIdx.x;
+    const float *rg = ring + ((size_t)hd * 2 + last_slot) * kRingFloats;
+    const size_t st_len = (size_t)d * d + 2 * (size_t)d * dv + 2 * (size_t)d;
+    const float *sin = state_in ? state_in + (size_t)hd * st_len : nullptr;
+    // the ring stores float4 c (columns c0 + 4c..) of epilogue thread et = 32 (qd + 4 cq) + lane at c * 512 + et
+    auto ring_at = [&](const float *base, int r, int col) {
+        const int et = 32 * ((r >> 5) + 4 * (col >> 5)) + (r & 31);
+        return base[(size_t)(((col & 31) >> 2) * kEpiThreads + et) * 4 + (col & 3)];
+    };
+    for (int i = tid; i < kD * kD; i += blockDim.x) {
+        const int r = i / kD, c = i % kD;
+        S[i] = ring_at(rg, r, c);
+        float cv = 0.f;
+        if (r < d && c < dv) {
+            for (int g = 0; g < groups; ++g) cv += part[((size_t)hd * groups + g) * kCPartFloats + (size_t)r * kD + c];
+            if (sin) cv += sin[(size_t)d * d + (size_t)r * dv + c];
+        }
+        C[i] = cv;
+    }
+    for (int r = tid; r < kD; r += blockDim.x) {
+        float mv = 0.f;
+        if (r < d) {
+            for (int g = 0; g < groups; ++g) mv += part[((size_t)hd * groups + g) * kCPartFloats + kD * kD + r];
+            if (sin) mv += sin[(size_t)d * d + (size_t)d * dv + r];
+        }
+        m[r] = mv;
+    }
+    __syncthreads();  // everything read from state_in before state_out (possibly the same memory) is written
+    float *so = state_out + (size_t)hd * st_len;
+    float *oS = so, *oC = oS + (size_t)d * d, *om = oC + (size_t)d * dv, *oG = om + d, *oh = oG + (size_t)d * dv;
+    for (int i = tid; i < d * d; i += blockDim.x) oS[i] = S[(i / d) * kD + i % d];
+    for (int i = tid; i < d * dv; i += blockDim.x) {
+        const int r = i / dv, c = i % dv;
+        float sc = 0.f;
+        for (int x = 0; x < d; ++x) sc += S[r * kD + x] * C[x * kD + c];
+        oC[i] = C[r * kD + c];
+        oG[i] = sc - ring_at(rg + kD * kD, r, c);  // G = S C - D
+    }
+    for (int r = tid; r < d; r += blockDim.x) {
+        float sm_ = 0.f;
+        for (int x = 0; x < d; ++x) sm_ += S[r * kD + x] * m[x];
+        om[r] = m[r];
+        oh[r] = sm_ - rg[2 * kD * kD + r];  // h = S m - e
+    }
+}
+
+int state_groups(int BH, int M) {
+    int g = 256 / (BH > 0 ? BH : 1);
+    if (g < 1) g = 1;
+    if (g > 8) g = 8;
+    return g < M ? g : M;
+}
+
 }  // namespace
 
 // head sizes the fused kernel serves (64 as zero-padded 128)
 bool fused_dim(int x) { return x == 64 || x == kD; }
 
-size_t fused2_workspace_bytes(int BH, int n, int d, int dv, int chunk, hla_dtype dt) {
+size_t fused2_workspace_bytes(int BH, int n, int d, int dv, int chunk, hla_dtype dt, bool with_state) {
     if (dt != HLA_BF16 || !fused_dim(d) || !fused_dim(dv)) return 0;
     (void)chunk;
-    return fused_layout(BH, n).total;
+    const FusedLayout L = fused_layout(BH, n);
+    return with_state ? L.total_state : L.total;
 }
 
 bool fused2_applicable(const Fwd2 &p) {
     if (getenv("HLA_DISABLE_FUSED")) return false;
     if (p.dt != HLA_BF16 || !fused_dim(p.d) || !fused_dim(p.dv) || !p.masked) return false;
-    if (p.state_out || p.n <= 0 || p.BH <= 0) return false;
+    if (p.n <= 0 || p.BH <= 0) return false;
     if (p.state_in && (p.d != kD || p.dv != kD)) return false;  // initial states in the 128 x 128 layout only
-    if (p.ws_bytes < fused_layout(p.BH, p.n).total) return false;
+    const FusedLayout FL = fused_layout(p.BH, p.n);
+    if (p.ws_bytes < (p.state_out ? FL.total_state : FL.total)) return false;
     int dev = 0, major = 0, minor = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return false;
     cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
@@ -1022,10 +1222,32 @@ cudaError_t fused2_forward(const Fwd2 &p, cudaStream_t stream) {
         if ((e = cudaGetLastError())) return e;
         kp.init_De = init;
     }
-    if ((e = cudaFuncSetAttribute(hla2_fused_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes)))
-        return e;
     const int grid = kp.n_items < sms ? kp.n_items : sms;
-    hla2_fused_kernel<<<grid, kThreads, kSmemBytes, stream>>>(mq, mk, mv, mo, kp);
+    if (p.state_out) {
+        if ((e = cudaFuncSetAttribute(hla2_fused_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                      (int)kSmemBytes)))
+            return e;
+        hla2_fused_kernel<true><<<grid, kThreads, kSmemBytes, stream>>>(mq, mk, mv, mo, kp);
+    } else {
+        if ((e = cudaFuncSetAttribute(hla2_fused_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                      (int)kSmemBytes)))
+            return e;
+        hla2_fused_kernel<false><<<grid, kThreads, kSmemBytes, stream>>>(mq, mk, mv, mo, kp);
+    }
+    if ((e = cudaGetLastError()) || !p.state_out) return e;
+    // final state: C and m partials, then the tuple (state_in, read by the kernel above, may alias)
+    const int groups = state_groups(p.BH, kp.M);
+    const int tiles_per = (kp.M + groups - 1) / groups;
+    float *part = reinterpret_cast<float *>(p.ws + FL.off_part);
+    if ((e = cudaFuncSetAttribute(state_c_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kCSmemBytes)))
+        return e;
+    state_c_kernel<<<p.BH * groups, kCThreads, kCSmemBytes, stream>>>(mq, mv, part, kp.M, groups, tiles_per, kp.err);
+    if ((e = cudaGetLastError())) return e;
+    const int fin_smem = (int)(sizeof(float) * (2 * kD * kD + kD));
+    if ((e = cudaFuncSetAttribute(state_finalize_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, fin_smem)))
+        return e;
+    state_finalize_kernel<<<p.BH, 256, fin_smem, stream>>>(kp.ring, (kp.G - 1) & 1, part, groups, p.state_in,
+                                                            p.state_out, p.d, p.dv);
     return cudaGetLastError();
 }
 

@@ -60,7 +60,7 @@ size_t generic2_workspace_bytes(int BH, int n, int d, int dv, int chunk);
 cudaError_t generic2_forward(const Fwd2 &p, cudaStream_t stream);
 
 // fused tcgen05 path (bf16, d = dv in {64, 128}); returns false if it does not apply
-size_t fused2_workspace_bytes(int BH, int n, int d, int dv, int chunk, hla_dtype dt);
+size_t fused2_workspace_bytes(int BH, int n, int d, int dv, int chunk, hla_dtype dt, bool with_state);
 bool fused2_applicable(const Fwd2 &p);
 cudaError_t fused2_forward(const Fwd2 &p, cudaStream_t stream);
 

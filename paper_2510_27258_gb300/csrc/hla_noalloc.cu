@@ -60,7 +60,7 @@ extern "C" hla_status hla2_forward_noalloc(const void *q, const void *k, const v
                            reinterpret_cast<uintptr_t>(state_in)) & 15u;
     if (mis) return fail(HLA_ERR_INVALID_ARGUMENT, "q, k, v, out and state_in must be 16-byte aligned");
     if (!std::isfinite(eps)) return fail(HLA_ERR_INVALID_ARGUMENT, "eps must be finite");
-    const size_t need = fused2_workspace_bytes(B * H, n, d, dv, chunk, dt);
+    const size_t need = fused2_workspace_bytes(B * H, n, d, dv, chunk, dt, false);
     if (need > kNoAllocScratchBytes)
         return fail(HLA_ERR_WORKSPACE, "these sizes need %zu bytes of scratch; hla2_forward_noalloc has %zu", need,
                     kNoAllocScratchBytes);

@@ -53,7 +53,8 @@ def check(hla, q, k, v, normalized, state_in=None, chunk=128):
 
 def test_fused_path_selected(hla):
     assert hla.hla2_forward_path(2, 16, 16384, 128, 128, normalized=True) == (1, 1)
-    assert hla.hla2_forward_path(2, 16, 16384, 128, 128, normalized=True, has_state_out=True)[0] == 0
+    assert hla.hla2_forward_path(2, 16, 16384, 128, 128, normalized=True, has_state_out=True) == (1, 3)
+    assert hla.hla2_forward_path(2, 16, 16384, 128, 128, has_state_in=True, has_state_out=True) == (1, 4)
     assert hla.hla2_forward_path(2, 16, 16384, 128, 128, masked=False)[0] == 0
     # d, dv of 64 as zero-padded 128, any chunk; an initial state only in the 128 x 128 layout
     assert hla.hla2_forward_path(8, 16, 2048, 64, 64, chunk=64) == (1, 1)
@@ -147,3 +148,53 @@ def test_fused_wait_timeout_is_reported_not_hung(hla, monkeypatch):
     assert hla.hla_poll_error(ws) == hla.HLA_OK
     ref = oracle.hla2_serial(q.reshape(1, 512, 128), k.reshape(1, 512, 128), v.reshape(1, 512, 128), masked=True)
     assert rowerr(out.float().cpu().numpy().reshape(1, 512, 128), ref) < 2e-2
+
+
+@pytest.mark.parametrize("d,dv", [(128, 128), (64, 64), (64, 128)])
+@pytest.mark.parametrize("n,seg", [(1, "default"), (200, "1"), (700, "2"), (1000, "default")])
+@pytest.mark.parametrize("normalized", [False, True])
+def test_fused_state_out(hla, monkeypatch, d, dv, n, seg, normalized):
+    """The final state tuple written by the fused path against the oracle's (parts S, C, m, G, h)."""
+    if seg != "default":
+        monkeypatch.setenv("HLA_FUSED_SEGMENT_TILES", seg)
+    B, H = 1, 2
+    q, k, v = hla_inputs.make_qkv(B, H, n, d, dv, seed=n + d + dv, dtype="bf16")
+    assert hla.hla2_forward_path(B, H, n, d, dv, normalized=normalized, has_state_out=True)[0] == 1
+    tq, tk, tv = (hla_inputs.as_torch(x, "bf16", DEV) for x in (q, k, v))
+    st = torch.zeros((B, H, hla.hla2_state_floats(d, dv)), dtype=torch.float32, device=DEV)
+    out = hla.hla2_forward(tq, tk, tv, masked=True, normalized=normalized, eps=hla_inputs.EPS, chunk=128, state_out=st)
+    torch.cuda.synchronize()
+    num_ref, rst = oracle.hla2_serial(q.reshape(B * H, n, d), k.reshape(B * H, n, d), v.reshape(B * H, n, dv),
+                                      masked=True, normalized=False, return_state=True, nthreads=4)
+    if not normalized:
+        assert rowerr(out.float().cpu().numpy().reshape(B * H, n, dv), num_ref) < 2e-2
+    gst = st.cpu().numpy().reshape(B * H, -1)
+    parts_g, parts_r = oracle.split_state2(gst, d, dv), oracle.split_state2(rst, d, dv)
+    for name in ("S", "C", "m", "G", "h"):
+        scale = max(np.abs(parts_r[name]).max(), np.abs(parts_r["S"]).max() * np.abs(parts_r["C"]).max())
+        err = np.abs(parts_g[name] - parts_r[name]).max()
+        assert err <= 2e-5 * max(scale, 1.0), (name, err, scale)
+
+
+@pytest.mark.parametrize("alias", [False, True])
+def test_fused_state_in_out(hla, monkeypatch, alias):
+    """state_in -> forward -> state_out on the fused path (state_out may be state_in), and the
+    next chunk of the sequence from that state equals the whole sequence at once."""
+    monkeypatch.setenv("HLA_FUSED_SEGMENT_TILES", "1")
+    B, H, n1, n2, d = 1, 2, 300, 260, 128
+    q, k, v = hla_inputs.make_qkv(B, H, n1 + n2, d, d, seed=77, dtype="bf16")
+    tq, tk, tv = (hla_inputs.as_torch(x, "bf16", DEV) for x in (q, k, v))
+    st1 = torch.zeros((B, H, hla.hla2_state_floats(d, d)), dtype=torch.float32, device=DEV)
+    hla.hla2_forward(tq[:, :, :n1].contiguous(), tk[:, :, :n1].contiguous(), tv[:, :, :n1].contiguous(),
+                     masked=True, chunk=128, state_out=st1)
+    st2 = st1 if alias else torch.zeros_like(st1)
+    out2 = hla.hla2_forward(tq[:, :, n1:].contiguous(), tk[:, :, n1:].contiguous(), tv[:, :, n1:].contiguous(),
+                            masked=True, chunk=128, state_in=st1, state_out=st2)
+    torch.cuda.synchronize()
+    num_ref, rst = oracle.hla2_serial(q.reshape(B * H, -1, d), k.reshape(B * H, -1, d), v.reshape(B * H, -1, d),
+                                      masked=True, normalized=False, return_state=True, nthreads=4)
+    assert rowerr(out2.float().cpu().numpy().reshape(B * H, n2, d), num_ref[:, n1:]) < 2e-2
+    parts_g, parts_r = oracle.split_state2(st2.cpu().numpy().reshape(B * H, -1), d, d), oracle.split_state2(rst, d, d)
+    for name in ("S", "C", "m", "G", "h"):
+        scale = max(np.abs(parts_r[name]).max(), np.abs(parts_r["S"]).max() * np.abs(parts_r["C"]).max())
+        assert np.abs(parts_g[name] - parts_r[name]).max() <= 2e-5 * max(scale, 1.0), name
