@@ -39,9 +39,9 @@ DEC = hla_inputs.WORKLOADS["decode_bf16"]
 # capture of the kernel sources (concatenated) whose SHA-256 starts with "sha256"
 # (summaries in profiles/); reported as null for any other source or workload.
 TRAFFIC = {
-    "hla2_fused_kernel": {"src": ["hla_fused_sm103.cu", "sm103_prims.cuh"], "sha256": "547299329d9401d2", "workload": "long_bf16_norm",
-                          "n": 16384, "bytes": 688.4e6,
-                          "how": "ncu capture at n=8192 (270.4 MB read + 73.8 MB written) scaled x2 to n=16384"},
+    "hla2_fused_kernel": {"src": ["hla_fused_sm103.cu", "sm103_prims.cuh"], "sha256": "cc4f69b0e001ea91", "workload": "long_bf16_norm",
+                          "n": 16384, "bytes": 688.0e6,
+                          "how": "ncu capture at n=8192 (270.2 MB read + 73.8 MB written) scaled x2 to n=16384"},
     "step2_kernel": {"src": ["hla_step.cu"], "sha256": "6b7c09075c2fc3a7", "workload": "decode_bf16", "n": 0,
                      "bytes": 750.9e6, "how": "ncu capture of one step (406.4 MB read + 344.5 MB written)"},
 }
@@ -307,32 +307,51 @@ def main():
     achieved_tf = fwd_flops(w) / (ms * 1e-3) / 1e12
 
     # ---------------- end to end: pinned host buffers, copies inside the timed region ----------
+    # Every step copies its inputs from pinned host memory and its output back.  Steps are
+    # independent, so they are pipelined over two sets of device buffers: the host-to-device
+    # copy of step i+1 and the read-back of step i-1 run on their own streams while step i's
+    # forward runs; the timed region spans all copies of all steps.
     hq, hk, hv = (t.cpu().pin_memory() for t in (tq, tk, tv))
     hout = torch.empty(out.shape, dtype=out.dtype).pin_memory()
-    dq, dk, dvv = (torch.empty_like(t) for t in (tq, tk, tv))
+    nb = 2
+    dins = [[torch.empty_like(t) for t in (tq, tk, tv)] for _ in range(nb)]
+    douts = [torch.empty_like(out) for _ in range(nb)]
+    s_in, s_out = torch.cuda.Stream(device=dev), torch.cuda.Stream(device=dev)
+    ev_in, ev_cmp, ev_out = ([torch.cuda.Event() for _ in range(nb)] for _ in range(3))
 
-    def e2e_step():
-        dq.copy_(hq, non_blocking=True)
-        dk.copy_(hk, non_blocking=True)
-        dvv.copy_(hv, non_blocking=True)
-        hla.hla2_forward(dq, dk, dvv, out, masked=w.masked, normalized=w.normalized, eps=hla_inputs.EPS,
+    def e2e_step(i):
+        b = i % nb
+        with torch.cuda.stream(s_in):
+            s_in.wait_event(ev_cmp[b])  # the forward that read this buffer set (step i - 2) is done
+            for dst, src in zip(dins[b], (hq, hk, hv)):
+                dst.copy_(src, non_blocking=True)
+            ev_in[b].record(s_in)
+        stream.wait_event(ev_in[b])
+        stream.wait_event(ev_out[b])  # the read-back of this output buffer (step i - 2) is done
+        hla.hla2_forward(*dins[b], douts[b], masked=w.masked, normalized=w.normalized, eps=hla_inputs.EPS,
                          chunk=w.chunk, workspace=ws, stream=stream)
-        hout.copy_(out, non_blocking=True)
+        ev_cmp[b].record(stream)
+        with torch.cuda.stream(s_out):
+            s_out.wait_event(ev_cmp[b])
+            hout.copy_(douts[b], non_blocking=True)
+            ev_out[b].record(s_out)
 
-    for _ in range(2):
-        e2e_step()
+    for i in range(2):
+        e2e_step(i)
     torch.cuda.synchronize()
     e2e_steps = max(3, min(args.steps, 50))
     barrier(world)
     e0.record(stream)
-    for _ in range(e2e_steps):
-        e2e_step()
+    s_in.wait_stream(stream)
+    for i in range(e2e_steps):
+        e2e_step(i)
+    stream.wait_stream(s_out)
     e1.record(stream)
     torch.cuda.synchronize()
     e2e_ms = max_over_ranks(e0.elapsed_time(e1) / e2e_steps, world)
     in_bytes = sum(t.numel() * t.element_size() for t in (hq, hk, hv))
     out_bytes = hout.numel() * hout.element_size()
-    del hq, hk, hv, hout, dq, dk, dvv
+    del hq, hk, hv, hout, dins, douts
 
     result = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
