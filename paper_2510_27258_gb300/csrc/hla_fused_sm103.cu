@@ -81,10 +81,11 @@ enum Bar {
     bEvP = 6, bEvA = 7, bEvX = 8, bEvS = 9, bEvT = 10, bEvO = 11, bEvD = 12,
     bEvF = 13,  // + TMEM region of the fix-up tile (0: A, 1: X)
     bEpW = 15, bEpX = 16, bEpT = 17,
-    bEpR = 18,  // next tile's S split written, O read out of TMEM
+    bEpR = 18,  // next tile's S split written
     bEpF = 19,  // + TMEM region of the fix-up tile
     bEpDF = 21,
-    kNumBars = 22
+    bEpO = 22,  // O read out of TMEM
+    kNumBars = 23
 };
 constexpr int kFirstEpiBar = bEpW;
 
@@ -284,19 +285,6 @@ __device__ __forceinline__ float warp_colsum32(float (&v)[32]) {
     return v[0];
 }
 
-// sum of squares of row r, columns c0..c0+31 of a bf16 tile
-__device__ __forceinline__ float row_sumsq32(const uint8_t *tile, int r, int c0) {
-    float acc = 0.f;
-#pragma unroll
-    for (int jj = 0; jj < 32; jj += 8) {
-        float k8[8];
-        tile_row8(tile, r, c0 + jj, k8);
-#pragma unroll
-        for (int u = 0; u < 8; ++u) acc += k8[u] * k8[u];
-    }
-    return acc;
-}
-
 __device__ __forceinline__ float warp_sum(float x) {
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
@@ -447,19 +435,24 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 }
 
                 // ---- 2. sweep ----
+                // Slots per tile: SX holds R_hi, then X_hi; W holds R_lo, then X_lo; SD holds D_p, then
+                // the output staging.  The split of the next tile's S_p is written once T and D have
+                // read X (while T V + Q D_p run), so that only the output read-out separates O from
+                // the next tile's Q R.
                 for (int j = 0; j < nt && !ms->abort_flag; ++j) {
                     const uint32_t tp = n_tiles & 1;
                     const int qs = (j & 1) ? kQ1 : kQ0, qo = (j & 1) ? kQ0 : kQ1;
                     // slot qo (Q of the previous tile, last read by its O MMA) takes the next Q
                     if (j + 1 < nt) load_tile(qo, &tm_q, head, (t0 + j + 1) * kTile);
-                    // X = Q R_hi + Q R_lo + W_hi K + W_lo K; the Q R part runs while W is built.  The
-                    // split of S_p is ready (and O of the previous tile out of TMEM) at the R hand-off;
-                    // for the first tile of a segment it comes with W.
+                    // X = Q R_hi + Q R_lo + W_hi K + W_lo K; the Q R part runs while W is built.  For the
+                    // first tile of a segment the split of S_p comes with W; later ones wait for the
+                    // split and for the previous output to have left TMEM columns X.
                     if (j > 0 && !bar_wait(ms, bEpR, (n_r++) & 1, p)) break;
+                    if (j > 0 && !bar_wait(ms, bEpO, tp ^ 1u, p)) break;
                     if (j == 0 && !bar_wait(ms, bEpW, tp, p)) break;
                     tc_fence_after();
                     mma128<false, false>(tb + kTX, lk(qs), lk(kSX), 0u);      // X = Q R_hi
-                    if (precise) mma128<false, false>(tb + kTX, lk(qs), lk(kSD), 1u);  // += Q R_lo
+                    if (precise) mma128<false, false>(tb + kTX, lk(qs), lk(kW), 1u);  // += Q R_lo
                     if (j > 0 && !bar_wait(ms, bEpW, tp, p)) break;  // W (hi, lo) ready
                     tc_fence_after();
                     mma128_ts<true>(tb + kTX, tb + kTA, lm(kK), 1u);          // += W_hi K (W in TMEM)
@@ -469,37 +462,30 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                     umma_commit(&ms->bar[bEvS]);
                     if (!bar_wait(ms, bEvS, tp, p)) break;  // X and S MMAs done: slot K free
                     if (j + 1 < nt) load_tile(kK, &tm_k, head, (t0 + j + 1) * kTile);
-                    if (!bar_wait(ms, bEpX, tp, p)) break;  // X_hi and X_lo ready
+                    if (!bar_wait(ms, bEpX, tp, p)) break;  // X_hi, X_lo in SX, W; D_p read out of TMEM
                     tc_fence_after();
                     mma128<false, false>(tb + kTA, lk(qs), lk(kSX), 0u);      // T = Q X_hi^T
-                    mma128<false, false>(tb + kTA, lk(qs), lk(kW), 1u);       // += Q X_lo^T (X_lo in W)
+                    mma128<false, false>(tb + kTA, lk(qs), lk(kW), 1u);       // += Q X_lo^T
                     umma_commit(&ms->bar[bEvT]);
-                    // T (bf16) in W and D_p (bf16) in SD; TMEM A free; the epilogue has read D_p from TMEM
-                    if (!bar_wait(ms, bEpT, tp, p)) break;
                     if (!wait_ld(kV)) break;
                     tc_fence_after();
-                    if (d_lo) {  // D to fp32-level accuracy: X_lo is read from slot W before O's staging
-                        mma128<true, true>(tb + kTD, lm(kSX), lm(kV), 1u);    // D += X_hi^T V
-                        mma128<true, true>(tb + kTD, lm(kW), lm(kV), 1u);     // D += X_lo^T V
-                        umma_commit(&ms->bar[bEvD]);
-                    }
+                    mma128<true, true>(tb + kTD, lm(kSX), lm(kV), 1u);        // D += X_hi^T V
+                    if (d_lo) mma128<true, true>(tb + kTD, lm(kW), lm(kV), 1u);  // D += X_lo^T V
+                    umma_commit(&ms->bar[bEvD]);
+                    // T (bf16) in TMEM A and D_p (bf16) in SD
+                    if (!bar_wait(ms, bEpT, tp, p)) break;
+                    tc_fence_after();
                     mma128<false, true>(tb + kTX, lk(qs), lm(kSD), 0u);       // O = Q D_p
                     mma128_ts<true>(tb + kTX, tb + kTA, lm(kV), 1u);          // += T V (T in TMEM)
                     umma_commit(&ms->bar[bEvO]);
-                    if (!d_lo) {
-                        mma128<true, true>(tb + kTD, lm(kSX), lm(kV), 1u);    // D += X^T V
-                        umma_commit(&ms->bar[bEvD]);
-                    }
+                    if (!bar_wait(ms, bEvO, tp, p)) break;  // T, V and D_p read
                     if (j + 1 < nt) {  // next tile's A = Q K^T overlaps this tile's output epilogue
-                        // A goes to the TMEM columns O has just read T from
-                        if (!bar_wait(ms, bEvO, tp, p)) break;
                         if (!wait_ld(qo) || !wait_ld(kK)) break;
                         tc_fence_after();
                         mma128<false, false>(tb + kTA, lk(qo), lk(kK), 0u);
                         umma_commit(&ms->bar[bEvA]);
+                        load_tile(kV, &tm_v, head, (t0 + j + 1) * kTile);
                     }
-                    if (!bar_wait(ms, d_lo ? bEvO : bEvD, tp, p)) break;  // the last reader of V done
-                    if (j + 1 < nt) load_tile(kV, &tm_v, head, (t0 + j + 1) * kTile);
                     ++n_tiles;
                 }
 
@@ -563,9 +549,9 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
             float *ring_cur = p.ring + ((size_t)head * 2 + (sigma & 1)) * kRingFloats;
             const unsigned *flagS = p.flags, *flagD = p.flags + 2 * p.BH;
 
-            // Shift of the S split: cs = bf16(tr_s / d) with tr_s the trace of the carry S_p,
-            // kept up to date from the K tiles' sums of squares (trace K^T K); every epilogue
-            // thread holds the same value.  Any shift is exact (x = R q + cs q in fp32).
+            // Shift of the S split: cs = bf16(trace S_p / d), from the carry-in here and from the
+            // diagonal of the S carry at each later split; every epilogue thread holds the same
+            // value.  Any shift is exact (x = R q + cs q in fp32).
             float tr_s = 0.f, cs = 0.f;
 
             // ---- 1. S chain: carry-in S of the segment, publish the inclusive prefix ----
@@ -614,9 +600,9 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
 #pragma unroll
                 for (int j = 0; j < 32; ++j) u[j] = __float_as_uint(sp[j]);
                 tmem_st32(tb + lane_base + kTS + c0, u);
-                // split S_p = cs I + R into R_hi (slot SX) and R_lo (slot SD)
+                // split S_p = cs I + R into R_hi (slot SX) and R_lo (slot W)
                 if (cq == qd) shift_diag32(sp, lane, cs);
-                store_split32(slot(kSX), slot(kSD), r, c0, sp, precise);
+                store_split32(slot(kSX), slot(kW), r, c0, sp, precise);
                 // segment-local D carry: the initial state's D for the first segment
                 const float *d0 = (sigma == 0 && p.init_De) ? p.init_De + (size_t)head * (kD * kD + kD) : nullptr;
 #pragma unroll
@@ -643,8 +629,6 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 // (the A operand of X += W K): hi in columns c0 .. +15, lo in c0 + 16 .. +31
                 bar_wait(ms, bEvA, tp, p);
                 tc_fence_after();
-                // this tile's part of trace K^T K (slot K holds K_j until the X MMAs are done)
-                const float k2 = warp_sum(row_sumsq32(slot(kK), r, c0));
                 {
                     uint32_t h[16], l[16];
                     if (blk_zero) {
@@ -662,11 +646,18 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 }
                 epi_arrive(ms, bEpW);
 
-                if (et == 0) tma_store_wait_read();  // the previous output tile has left slot W
+                if (et == 0) tma_store_wait_read();  // the previous output tile has left slot SD
                 epi_sync();
-                if (lane == 0) ms->red[warp] = k2;
 
-                // while X = W K + Q S_p runs: q_t . e_p, the carried part of the denominator
+                // while X = W K + Q S_p runs: D_p (bf16, final since the previous O) -> slot SD, read
+                // out of TMEM before this tile's D MMA (issued after the X hand-off), and q_t . e_p,
+                // the carried part of the denominator
+                {
+                    float f[32];
+                    ld32(tb + lane_base + kTD + c0, f);
+#pragma unroll
+                    for (int jj = 0; jj < 32; jj += 8) store_row8(slot(kSD), r, c0 + jj, f + jj);
+                }
                 float den_part = 0.f;
                 if (p.normalized) {
 #pragma unroll
@@ -694,18 +685,11 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 fence_async_smem();
                 epi_arrive(ms, bEpX);
 
-                // while T = Q X^T runs: column sums of X (e carry) and D_p -> bf16 (slot SD; R_lo
-                // there is dead once X is done; D += X^T V is issued after this tile's T hand-off)
+                // while T = Q X^T runs: column sums of X (e carry)
                 float ecol = 0.f;
                 if (need_e) ecol = warp_colsum32(x);  // column c0 + lane over this warp's rows
-                {
-                    float f[32];
-                    ld32(tb + lane_base + kTD + c0, f);
-#pragma unroll
-                    for (int jj = 0; jj < 32; jj += 8) store_row8(slot(kSD), r, c0 + jj, f + jj);
-                }
 
-                // T = L . (Q X^T) -> bf16 (slot W); row sums
+                // T = L . (Q X^T) -> bf16 in TMEM; row sums
                 bar_wait(ms, bEvT, tp, p);
                 tc_fence_after();
                 {
@@ -728,16 +712,10 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 fence_async_smem();  // D_p (bf16) in SD
                 epi_arrive(ms, bEpT);
 
-                // trace of the updated S; denominators (sum over the four column quarters) and
-                // e carry += column sums of X (sum over the four lane quadrants), in a fixed order
+                // denominators (sum over the four column quarters) and e carry += column sums of X
+                // (sum over the four lane quadrants), in a fixed order
                 if (p.normalized && cq > 0) ms->part[cq - 1][r] = den_part;
                 epi_sync();
-                {
-                    float t = 0.f;
-#pragma unroll
-                    for (int w = 0; w < kEpiWarps; ++w) t += ms->red[w];
-                    tr_s += t;
-                }
                 if (p.normalized && cq == 0)
                     ms->den[r] = ((den_part + ms->part[0][r]) + ms->part[1][r]) + ms->part[2][r];
                 if (need_e) {
@@ -749,7 +727,32 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                                                (ms->part[1][c0 + lane] + ms->part[2][c0 + lane]);
                 }
 
-                // O (provisional for segments > 0, final for the first) -> slot W, TMA store
+                // D += X^T V done (T too): slots SX and W are free, the S carry is current.  Split of
+                // S_p for the next tile, shifted by the mean of its diagonal, while T V + Q D_p run.
+                bar_wait(ms, bEvD, tp, p);
+                tc_fence_after();
+                if (j + 1 < nt) {
+                    float f[32];
+                    ld32(tb + lane_base + kTS + c0, f);
+                    {
+                        float dg = 0.f;
+                        if (cq == qd) {
+#pragma unroll
+                            for (int jj = 0; jj < 32; ++jj)
+                                if (jj == lane) dg = f[jj];
+                        }
+                        dg = warp_sum(dg);
+                        if (cq == qd && lane == 0) ms->red[qd] = dg;
+                    }
+                    epi_sync();
+                    cs = bf16_round(((ms->red[0] + ms->red[1]) + (ms->red[2] + ms->red[3])) / kD);
+                    if (cq == qd) shift_diag32(f, lane, cs);
+                    store_split32(slot(kSX), slot(kW), r, c0, f, precise);
+                    fence_async_smem();
+                    epi_arrive(ms, bEpR);  // R of the next tile ready: Q R may start once O is read
+                }
+
+                // O (provisional for segments > 0, final for the first) -> slot SD, TMA store
                 bar_wait(ms, bEvO, tp, p);
                 tc_fence_after();
                 {
@@ -757,34 +760,22 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                     const float den = p.normalized ? ms->den[r] : 1.f;
                     float f[32];
                     ld32(tb + lane_base + kTX + c0, f);
+                    epi_arrive(ms, bEpO);  // TMEM columns X are free for the next tile's X
                     if (final_out && p.normalized) {
                         const float inv = 1.f / (den + p.eps);
 #pragma unroll
                         for (int jj = 0; jj < 32; ++jj) f[jj] *= inv;
                     }
 #pragma unroll
-                    for (int jj = 0; jj < 32; jj += 8) store_row8(slot(kW), r, c0 + jj, f + jj);
+                    for (int jj = 0; jj < 32; jj += 8) store_row8(slot(kSD), r, c0 + jj, f + jj);
                     if (!final_out && p.normalized && cq == 0 && tok0 + r < p.n)
                         p.den_loc[(size_t)head * p.n + tok0 + r] = den;
-                }
-                // D += X^T V done: X_hi in SX and D_p (bf16) in SD are dead, the D carry is current
-                bar_wait(ms, bEvD, tp, p);
-                tc_fence_after();
-                if (j + 1 < nt) {
-                    // split of the updated S for the next tile, shifted by the mean of its diagonal
-                    cs = bf16_round(tr_s / kD);
-                    float f[32];
-                    ld32(tb + lane_base + kTS + c0, f);
-                    if (cq == qd) shift_diag32(f, lane, cs);
-                    store_split32(slot(kSX), slot(kSD), r, c0, f, precise);
-                    fence_async_smem();
-                    epi_arrive(ms, bEpR);  // R of the next tile ready, O read: Q R may start
                 }
                 fence_async_smem();
                 epi_sync();
                 if (et == 0) {
-                    tma_store_3d(&tm_o, slot(kW), 0, tok0, head);
-                    if (p.out_blocks > 1) tma_store_3d(&tm_o, slot(kW) + kBlockBytes, 64, tok0, head);
+                    tma_store_3d(&tm_o, slot(kSD), 0, tok0, head);
+                    if (p.out_blocks > 1) tma_store_3d(&tm_o, slot(kSD) + kBlockBytes, 64, tok0, head);
                     tma_store_commit();
                 }
                 ++n_tiles;
@@ -792,7 +783,10 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
 
             // ---- 3. D chain and fix-up ----
             {
-                if (sigma > 0 && et == 0) chain_wait(&flagD[head * 2 + ((sigma - 1) & 1)], (unsigned)sigma, p, 2, item);
+                if (et == 0) {
+                    tma_store_wait_read();  // the last output tile has left slot SD (D prefix below)
+                    if (sigma > 0) chain_wait(&flagD[head * 2 + ((sigma - 1) & 1)], (unsigned)sigma, p, 2, item);
+                }
                 epi_sync();
                 const float4 *dprev = sigma > 0 ? reinterpret_cast<const float4 *>(ring_prev + kD * kD) : nullptr;
                 float4 *dcur = reinterpret_cast<float4 *>(ring_cur + kD * kD);
