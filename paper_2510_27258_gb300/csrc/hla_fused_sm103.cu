@@ -99,6 +99,7 @@ struct Misc {
     float eloc[kD];      // segment-local e carry
     float den[kTile];    // denominators of the current tile
     float part[3][kD];   // partial sums of the other three column quarters / lane quadrants
+    float dtr[2][4];     // diagonal sums of the S carry per lane quadrant, by tile parity
 };
 static_assert(sizeof(Misc) <= kMiscBytes, "misc smem");
 
@@ -549,8 +550,9 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
             float *ring_cur = p.ring + ((size_t)head * 2 + (sigma & 1)) * kRingFloats;
             const unsigned *flagS = p.flags, *flagD = p.flags + 2 * p.BH;
 
-            // Shift of the S split: cs = bf16(trace S_p / d), from the carry-in here and from the
-            // diagonal of the S carry at each later split; every epilogue thread holds the same
+            // Shift of the S split: cs = bf16(trace / d) with the trace of the carry-in for the first
+            // tile and, for later ones, of the S carry one tile back (read at the previous split; a
+            // shift one tile stale keeps R small just the same); every epilogue thread holds the same
             // value.  Any shift is exact (x = R q + cs q in fp32).
             float tr_s = 0.f, cs = 0.f;
 
@@ -620,6 +622,15 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
             pub_arrive(kBarPubS);  // S prefix in the ring
 
             // ---- 2. sweep ----
+            // e carry += column sums of X (sum over the four lane quadrants, in a fixed order)
+            auto add_ecol = [&](float ec) {
+                if (qd > 0) ms->part[qd - 1][c0 + lane] = ec;
+                epi_sync();
+                if (qd == 0)
+                    ms->eloc[c0 + lane] += (ec + ms->part[0][c0 + lane]) + (ms->part[1][c0 + lane] + ms->part[2][c0 + lane]);
+                epi_sync();
+            };
+            float ecol = 0.f;  // this thread's column sum of the last tile's X, added in the next tile's X wait
             for (int j = 0; j < nt; ++j) {
                 const uint32_t tp = n_tiles & 1;
                 const uint8_t *qt = slot((j & 1) ? kQ1 : kQ0);
@@ -648,6 +659,7 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
 
                 if (et == 0) tma_store_wait_read();  // the previous output tile has left slot SD
                 epi_sync();
+                if (need_e && j > 0) add_ecol(ecol);  // the previous tile's X, before q_t . e_p below
 
                 // while X = W K + Q S_p runs: D_p (bf16, final since the previous O) -> slot SD, read
                 // out of TMEM before this tile's D MMA (issued after the X hand-off), and q_t . e_p,
@@ -686,7 +698,6 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 epi_arrive(ms, bEpX);
 
                 // while T = Q X^T runs: column sums of X (e carry)
-                float ecol = 0.f;
                 if (need_e) ecol = warp_colsum32(x);  // column c0 + lane over this warp's rows
 
                 // T = L . (Q X^T) -> bf16 in TMEM; row sums
@@ -712,28 +723,23 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 fence_async_smem();  // D_p (bf16) in SD
                 epi_arrive(ms, bEpT);
 
-                // denominators (sum over the four column quarters) and e carry += column sums of X
-                // (sum over the four lane quadrants), in a fixed order
-                if (p.normalized && cq > 0) ms->part[cq - 1][r] = den_part;
-                epi_sync();
-                if (p.normalized && cq == 0)
-                    ms->den[r] = ((den_part + ms->part[0][r]) + ms->part[1][r]) + ms->part[2][r];
-                if (need_e) {
-                    epi_sync();  // the denominator partials are read before part is reused
-                    if (qd > 0) ms->part[qd - 1][c0 + lane] = ecol;
-                    epi_sync();
-                    if (qd == 0)
-                        ms->eloc[c0 + lane] += (ecol + ms->part[0][c0 + lane]) +
-                                               (ms->part[1][c0 + lane] + ms->part[2][c0 + lane]);
+                // denominators: partial sums of the four column quarters, added in a fixed order
+                if (p.normalized) {
+                    if (cq == 0) ms->den[r] = den_part;
+                    else ms->part[cq - 1][r] = den_part;
                 }
+                epi_sync();
+                const float den = p.normalized ? ((ms->den[r] + ms->part[0][r]) + ms->part[1][r]) + ms->part[2][r] : 1.f;
 
                 // D += X^T V done (T too): slots SX and W are free, the S carry is current.  Split of
-                // S_p for the next tile, shifted by the mean of its diagonal, while T V + Q D_p run.
+                // S_p for the next tile while T V + Q D_p run.
                 bar_wait(ms, bEvD, tp, p);
                 tc_fence_after();
                 if (j + 1 < nt) {
                     float f[32];
                     ld32(tb + lane_base + kTS + c0, f);
+                    const float *dt = ms->dtr[(j + 1) & 1];
+                    cs = bf16_round((j == 0 ? tr_s : (dt[0] + dt[1]) + (dt[2] + dt[3])) / kD);
                     {
                         float dg = 0.f;
                         if (cq == qd) {
@@ -742,10 +748,8 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                                 if (jj == lane) dg = f[jj];
                         }
                         dg = warp_sum(dg);
-                        if (cq == qd && lane == 0) ms->red[qd] = dg;
+                        if (cq == qd && lane == 0) ms->dtr[j & 1][qd] = dg;
                     }
-                    epi_sync();
-                    cs = bf16_round(((ms->red[0] + ms->red[1]) + (ms->red[2] + ms->red[3])) / kD);
                     if (cq == qd) shift_diag32(f, lane, cs);
                     store_split32(slot(kSX), slot(kW), r, c0, f, precise);
                     fence_async_smem();
@@ -757,7 +761,6 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 tc_fence_after();
                 {
                     const bool final_out = (sigma == 0);
-                    const float den = p.normalized ? ms->den[r] : 1.f;
                     float f[32];
                     ld32(tb + lane_base + kTX + c0, f);
                     epi_arrive(ms, bEpO);  // TMEM columns X are free for the next tile's X
@@ -772,7 +775,7 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                         p.den_loc[(size_t)head * p.n + tok0 + r] = den;
                 }
                 fence_async_smem();
-                epi_sync();
+                epi_sync();  // also: every denominator read before part is reused
                 if (et == 0) {
                     tma_store_3d(&tm_o, slot(kSD), 0, tok0, head);
                     if (p.out_blocks > 1) tma_store_3d(&tm_o, slot(kSD) + kBlockBytes, 64, tok0, head);
@@ -780,6 +783,7 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 }
                 ++n_tiles;
             }
+            if (need_e && nt > 0) add_ecol(ecol);  // the last tile's X
 
             // ---- 3. D chain and fix-up ----
             {
