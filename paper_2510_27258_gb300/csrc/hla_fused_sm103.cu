@@ -394,8 +394,33 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
         return bar_wait(ms, bLd0 + s, par, p);
     };
 
+    // Pre-pass of an item: S aggregate of its tiles (sum of K^T K) into TMEM columns S, from K tiles
+    // in four slots (K, V, W, Q1).  It runs at the start of a CTA's first item and, for later items,
+    // while the previous item's epilogue waits for its D prefix (the S carry is dead by then and the
+    // fix-up has not started).  Returns false if a wait gave up.
+    bool pre_done = false;  // issuer: the current item's pre-pass ran in the previous item's tail
+    auto prepass = [&](int pitem) {
+        const int psig = pitem / p.BH, phead = pitem % p.BH;
+        const int pt0 = psig * p.L, pnt = min(p.L, p.M - pt0);
+        auto ps = [](int j) { return (j & 3) == 0 ? kK : (j & 3) == 1 ? kV : (j & 3) == 2 ? kW : kQ1; };
+        for (int j = 0; j < pnt && j < 4; ++j) load_tile(ps(j), &tm_k, phead, (pt0 + j) * kTile);
+        for (int j = 0; j < pnt; ++j) {
+            const int sl = ps(j);
+            if (!wait_ld(sl)) return false;
+            tc_fence_after();
+            mma128<true, true>(tb + kTS, lm(sl), lm(sl), j > 0 ? 1u : 0u);  // S_agg += K^T K
+            if (j + 4 < pnt) {  // long segment: reuse this slot once its MMA is done
+                umma_commit(&ms->bar[bPre]);
+                if (!bar_wait(ms, bPre, (n_pre++) & 1, p)) return false;
+                load_tile(sl, &tm_k, phead, (pt0 + j + 4) * kTile);
+            }
+        }
+        umma_commit(&ms->bar[bEvP]);
+        return true;
+    };
+
+    if (tid == 0) ms->item = (int)atomicAdd(p.ticket, 1u);  // later tickets are taken by the issuer
     while (true) {
-        if (tid == 0) ms->item = (int)atomicAdd(p.ticket, 1u);
         tc_fence_before();
         __syncthreads();
         tc_fence_after();
@@ -407,29 +432,21 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
         const int ip = n_items & 1;
 
         if (issuer) {
-            if (lane == 0) {
-                // ---- 1. pre-pass: S aggregate of the segment into TMEM cols kTX ----
-                // K tiles go to four idle slots (K, V, W, Q1); tile 0 stays in K for the sweep
-                const int ps[4] = {kK, kV, kW, kQ1};
-                load_tile(kQ0, &tm_q, head, t0 * kTile);
-                for (int j = 0; j < nt && j < 4; ++j) load_tile(ps[j], &tm_k, head, (t0 + j) * kTile);
-                for (int j = 0; j < nt; ++j) {
-                    const int s = ps[j & 3];
-                    if (!wait_ld(s)) break;
-                    tc_fence_after();
-                    mma128<true, true>(tb + kTX, lm(s), lm(s), j > 0 ? 1u : 0u);  // S_agg += K^T K
-                    if (j + 4 < nt) {  // long segment: reuse this slot once its MMA is done
-                        umma_commit(&ms->bar[bPre]);
-                        if (!bar_wait(ms, bPre, (n_pre++) & 1, p)) break;
-                        load_tile(s, &tm_k, head, (t0 + j + 4) * kTile);
-                    }
-                }
-                umma_commit(&ms->bar[bEvP]);
+            // one thread issues; a wait that gives up leaves this item's issuing (break) with the CTA
+            // marked aborted, so that every role runs on to the end of the item and the loop stops
+            if (lane == 0) do {
+                // ---- 1. pre-pass (unless it ran in the previous item's tail), first tile's A ----
+                const bool early = pre_done;
+                pre_done = false;
+                if (!early && !prepass(item)) break;
                 if (!bar_wait(ms, bEvP, ip, p)) break;  // the pre-pass slots are free again
-                // first tile's inputs (K tile 0 is still in slot K unless the segment is long)
-                if (nt > 4) load_tile(kK, &tm_k, head, t0 * kTile);
+                // first tile's inputs (K tile 0 is still in slot K after a pre-pass of <= 4 tiles that
+                // ran just now)
+                load_tile(kQ0, &tm_q, head, t0 * kTile);
+                const bool reload_k = early || nt > 4;
+                if (reload_k) load_tile(kK, &tm_k, head, t0 * kTile);
                 load_tile(kV, &tm_v, head, t0 * kTile);
-                if (wait_ld(kQ0) && (nt <= 4 || wait_ld(kK))) {
+                if (wait_ld(kQ0) && (!reload_k || wait_ld(kK))) {
                     tc_fence_after();
                     mma128<false, false>(tb + kTA, lk(kQ0), lk(kK), 0u);  // A = Q K^T
                     umma_commit(&ms->bar[bEvA]);
@@ -490,6 +507,17 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                     ++n_tiles;
                 }
 
+                // ---- next ticket; its pre-pass while the epilogue publishes this item's D prefix ----
+                if (!ms->abort_flag) {
+                    const int next = (int)atomicAdd(p.ticket, 1u);
+                    ms->item = next;  // every thread read this item's ticket at the top of the loop
+                    if (next < p.n_items) {
+                        if (!prepass(next)) break;
+                        pre_done = true;
+                        if (!bar_wait(ms, bEvP, ip ^ 1, p)) break;  // its slots are free for the fix-up
+                    }
+                }
+
                 // ---- 3. fix-up of segments > 0 ----
                 if (sigma > 0 && !ms->abort_flag) {
                     if (bar_wait(ms, bEpDF, n_dfix & 1, p)) {  // D prefix (bf16) in SD; outputs written
@@ -521,7 +549,7 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                         }
                     }
                 }
-            }
+            } while (0);
             __syncwarp();
         } else if (publisher) {
             // one S prefix and one D prefix per item (the epilogue arrives once at each, on every path)
@@ -590,7 +618,7 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 {
                     // inclusive S prefix of this segment -> ring
                     float agg[32];
-                    ld32(tb + lane_base + kTX + c0, agg);
+                    ld32(tb + lane_base + kTS + c0, agg);
                     float4 *rc = reinterpret_cast<float4 *>(ring_cur);
 #pragma unroll
                     for (int j = 0; j < 32; j += 4)
