@@ -74,18 +74,23 @@ enum Slot { kQ0 = 0, kQ1 = 1, kK = 2, kV = 3, kW = 4, kSX = 5, kSD = 6 };
 // TMEM columns: S carry, D carry, A -> T, X -> O
 constexpr uint32_t kTS = 0, kTD = 128, kTA = 256, kTX = 384;
 
+// fix-up buffers (three tiles in flight): Q slot, provisional output slot, TMEM columns of F
+__device__ __forceinline__ int fix_q(int i) { return i == 0 ? kQ0 : i == 1 ? kQ1 : kW; }
+__device__ __forceinline__ int fix_o(int i) { return i == 0 ? kK : i == 1 ? kV : kSX; }
+__device__ __forceinline__ uint32_t fix_t(int i) { return i == 0 ? kTA : i == 1 ? kTX : kTD; }
+
 // barrier indices
 enum Bar {
-    bLd0 = 0,  // + slot index for the TMA-loaded slots (Q0, Q1, K, V, W)
-    bPre = 5,  // pre-pass MMA done (per K tile)
-    bEvP = 6, bEvA = 7, bEvX = 8, bEvS = 9, bEvT = 10, bEvO = 11, bEvD = 12,
-    bEvF = 13,  // + TMEM region of the fix-up tile (0: A, 1: X)
-    bEpW = 15, bEpX = 16, bEpT = 17,
-    bEpR = 18,  // next tile's S split written
-    bEpF = 19,  // + TMEM region of the fix-up tile
-    bEpDF = 21,
-    bEpO = 22,  // O read out of TMEM
-    kNumBars = 23
+    bLd0 = 0,  // + slot index for the TMA-loaded slots (Q0, Q1, K, V, W, SX)
+    bPre = 6,  // pre-pass MMA done (per K tile)
+    bEvP = 7, bEvA = 8, bEvX = 9, bEvS = 10, bEvT = 11, bEvO = 12, bEvD = 13,
+    bEvF = 14,  // + fix-up buffer (0..2)
+    bEpW = 17, bEpX = 18, bEpT = 19,
+    bEpR = 20,  // next tile's S split written
+    bEpF = 21,  // + fix-up buffer: its slots and TMEM region are free again
+    bEpDF = 24,
+    bEpO = 25,  // O read out of TMEM
+    kNumBars = 26
 };
 constexpr int kFirstEpiBar = bEpW;
 
@@ -375,7 +380,7 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
     // per-CTA event counters (identical sequences on both sides)
     uint32_t n_tiles = 0, n_items = 0, n_pre = 0, n_dfix = 0;
     uint32_t ld_par = 0;  // bit s: parity of the next load completion of slot s
-    uint32_t fx_par = 0;  // bit g: parity of the next fix-up hand-off in TMEM region g
+    uint32_t fx_par = 0;  // bit i: parity of the next fix-up hand-off of buffer i
     uint32_t n_r = 0;     // S-split hand-offs (one per tile that has a successor in its segment)
 
     // descriptor low words of the slots, as K-major (lk) and MN-major (lm) operands
@@ -521,29 +526,30 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 // ---- 3. fix-up of segments > 0 ----
                 if (sigma > 0 && !ms->abort_flag) {
                     if (bar_wait(ms, bEpDF, n_dfix & 1, p)) {  // D prefix (bf16) in SD; outputs written
-                        // tile j: Q in slot Q(j&1), provisional output in slot K/V (j&1), F in TMEM A/X (j&1)
+                        // three tiles in flight: tile j uses buffer j % 3 (Q slot, provisional output slot,
+                        // which also stages the result, and TMEM region for F)
                         auto load_fix = [&](int j) {
-                            load_tile((j & 1) ? kQ1 : kQ0, &tm_q, head, (t0 + j) * kTile);
-                            load_tile((j & 1) ? kV : kK, &tm_o, head, (t0 + j) * kTile);
+                            const int i = j % 3;
+                            load_tile(fix_q(i), &tm_q, head, (t0 + j) * kTile);
+                            load_tile(fix_o(i), &tm_o, head, (t0 + j) * kTile);
                         };
-                        load_fix(0);
-                        if (nt > 1) load_fix(1);
+                        for (int j = 0; j < nt && j < 3; ++j) load_fix(j);
                         for (int j = 0; j < nt; ++j) {
-                            if (!wait_ld((j & 1) ? kQ1 : kQ0) || !wait_ld((j & 1) ? kV : kK)) break;
+                            const int i = j % 3;
+                            if (!wait_ld(fix_q(i)) || !wait_ld(fix_o(i))) break;
                             tc_fence_after();
-                            mma128<false, true>(tb + ((j & 1) ? kTX : kTA), lk((j & 1) ? kQ1 : kQ0), lm(kSD),
-                                                0u);  // F = Q D_prefix
-                            umma_commit(&ms->bar[bEvF + (j & 1)]);
-                            if (j >= 1) {  // tile j-1 done: its slots and TMEM region take tile j+1
-                                const int g = (j - 1) & 1;
+                            mma128<false, true>(tb + fix_t(i), lk(fix_q(i)), lm(kSD), 0u);  // F = Q D_prefix
+                            umma_commit(&ms->bar[bEvF + i]);
+                            if (j >= 1) {  // tile j-1 done: its buffer takes tile j+2
+                                const int g = (j - 1) % 3;
                                 const bool ok = bar_wait(ms, bEpF + g, (fx_par >> g) & 1u, p);
                                 fx_par ^= 1u << g;
                                 if (!ok) break;
-                                if (j + 1 < nt) load_fix(j + 1);
+                                if (j + 2 < nt) load_fix(j + 2);
                             }
                         }
                         {  // the last tile
-                            const int g = (nt - 1) & 1;
+                            const int g = (nt - 1) % 3;
                             bar_wait(ms, bEpF + g, (fx_par >> g) & 1u, p);
                             fx_par ^= 1u << g;
                         }
@@ -852,13 +858,13 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                     epi_sync();
                     epi_arrive(ms, bEpDF);
                     for (int j = 0; j < nt; ++j) {
-                        const uint8_t *qt = slot((j & 1) ? kQ1 : kQ0), *ot = slot((j & 1) ? kV : kK);
-                        uint8_t *stg = slot((j & 1) ? kSX : kW);  // output staging alternates W / SX
+                        const int i = j % 3;
+                        const uint8_t *qt = slot(fix_q(i));
+                        uint8_t *ot = slot(fix_o(i));  // provisional output, overwritten by the result
                         const int tok0 = (t0 + j) * kTile;
                         const float dl = (p.normalized && cq == 0 && tok0 + r < p.n)
                                              ? __ldcg(p.den_loc + (size_t)head * p.n + tok0 + r) : 0.f;
-                        const int g = j & 1;
-                        bar_wait(ms, bEvF + g, (fx_par >> g) & 1u, p);
+                        bar_wait(ms, bEvF + i, (fx_par >> i) & 1u, p);
                         tc_fence_after();
                         if (p.normalized) {
                             // den_t = provisional denominator + q_t . e_prefix (four column quarters)
@@ -870,33 +876,37 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
 #pragma unroll
                                 for (int u = 0; u < 8; ++u) qe += q8[u] * ms->eloc[c0 + jj + u];
                             }
-                            if (cq > 0) ms->part[cq - 1][r] = qe;
-                            epi_sync();
-                            if (cq == 0) ms->den[r] = dl + (((qe + ms->part[0][r]) + ms->part[1][r]) + ms->part[2][r]);
+                            if (cq == 0) ms->den[r] = dl + qe;
+                            else ms->part[cq - 1][r] = qe;
                         }
-                        if (et == 0) tma_store_wait_read1();  // the store that used stg two tiles ago is done
+                        if (j >= 1 && et == 0) tma_store_wait_read();  // tile j-1's result has left its slot
                         epi_sync();
-                        const float inv = p.normalized ? 1.f / (ms->den[r] + p.eps) : 1.f;
+                        if (j >= 1) epi_arrive(ms, bEpF + (j - 1) % 3);  // tile j-1's buffer is free
+                        const float inv = p.normalized
+                            ? 1.f / ((((ms->den[r] + ms->part[0][r]) + ms->part[1][r]) + ms->part[2][r]) + p.eps)
+                            : 1.f;
                         float f[32];
-                        ld32(tb + lane_base + (g ? kTX : kTA) + c0, f);
+                        ld32(tb + lane_base + fix_t(i) + c0, f);
 #pragma unroll
                         for (int jj = 0; jj < 32; jj += 8) {
                             float o8[8], w8[8];
                             tile_row8(ot, r, c0 + jj, o8);
 #pragma unroll
                             for (int u = 0; u < 8; ++u) w8[u] = (o8[u] + f[jj + u]) * inv;
-                            store_row8(stg, r, c0 + jj, w8);
+                            store_row8(ot, r, c0 + jj, w8);
                         }
                         fence_async_smem();
-                        epi_sync();
+                        epi_sync();  // also: every denominator read before the next tile's partials
                         if (et == 0) {
-                            tma_store_3d(&tm_o, stg, 0, tok0, head);
-                            if (p.out_blocks > 1) tma_store_3d(&tm_o, stg + kBlockBytes, 64, tok0, head);
+                            tma_store_3d(&tm_o, ot, 0, tok0, head);
+                            if (p.out_blocks > 1) tma_store_3d(&tm_o, ot + kBlockBytes, 64, tok0, head);
                             tma_store_commit();
                         }
-                        epi_arrive(ms, bEpF + g);
-                        fx_par ^= 1u << g;
+                        fx_par ^= 1u << i;
                     }
+                    if (et == 0) tma_store_wait_read();  // the last result has left its slot
+                    epi_sync();
+                    epi_arrive(ms, bEpF + (nt - 1) % 3);
                 }
             }
         }
