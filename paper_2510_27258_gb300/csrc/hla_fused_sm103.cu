@@ -495,11 +495,12 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                     mma128<true, true>(tb + kTD, lm(kSX), lm(kV), 1u);        // D += X_hi^T V
                     if (d_lo) mma128<true, true>(tb + kTD, lm(kW), lm(kV), 1u);  // D += X_lo^T V
                     umma_commit(&ms->bar[bEvD]);
-                    // T (bf16) in TMEM A and D_p (bf16) in SD
-                    if (!bar_wait(ms, bEpT, tp, p)) break;
+                    // O = Q D_p (D_p in SD since the X hand-off; TMEM X was read out then) runs while
+                    // the epilogue forms T
+                    mma128<false, true>(tb + kTX, lk(qs), lm(kSD), 0u);
+                    if (!bar_wait(ms, bEpT, tp, p)) break;  // T (bf16) in TMEM A
                     tc_fence_after();
-                    mma128<false, true>(tb + kTX, lk(qs), lm(kSD), 0u);       // O = Q D_p
-                    mma128_ts<true>(tb + kTX, tb + kTA, lm(kV), 1u);          // += T V (T in TMEM)
+                    mma128_ts<true>(tb + kTX, tb + kTA, lm(kV), 1u);          // O += T V (T in TMEM)
                     umma_commit(&ms->bar[bEvO]);
                     if (!bar_wait(ms, bEvO, tp, p)) break;  // T, V and D_p read
                     if (j + 1 < nt) {  // next tile's A = Q K^T overlaps this tile's output epilogue
@@ -728,7 +729,7 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                     for (int u = 0; u < 8; ++u) x[jj + u] += cs * q8[u];
                 }
                 store_split32(slot(kSX), slot(kW), r, c0, x, true);
-                fence_async_smem();
+                fence_async_smem();  // X_hi, X_lo and D_p (above) visible to the MMAs
                 epi_arrive(ms, bEpX);
 
                 // while T = Q X^T runs: column sums of X (e carry)
@@ -754,7 +755,6 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                     tmem_st16(tb + lane_base + kTA + c0, h);
                     tmem_st_wait();
                 }
-                fence_async_smem();  // D_p (bf16) in SD
                 epi_arrive(ms, bEpT);
 
                 // denominators: partial sums of the four column quarters, added in a fixed order
