@@ -48,6 +48,11 @@
 // R and W are also split into hi + lo, so X and T are accurate to ~2^-16 of
 // each term; the denominator is the fp32 row sum of T plus q_t . e_p, with the
 // e carry summed in fp32 on CUDA cores.  T and D enter T V and Q D as bf16.
+#include <algorithm>
+#include <functional>
+#include <queue>
+#include <vector>
+
 #include "hla_internal.h"
 #include "sm103_prims.cuh"
 
@@ -400,13 +405,18 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
     };
 
     // Pre-pass of an item: S aggregate of its tiles (sum of K^T K) into TMEM columns S, from K tiles
-    // in four slots (K, V, W, Q1).  It runs at the start of a CTA's first item and, for later items,
+    // in four slots (K, V, W, Q1); none for the last segment of a head unless the final state is
+    // wanted.  It runs at the start of a CTA's first item and, for later items,
     // while the previous item's epilogue waits for its D prefix (the S carry is dead by then and the
     // fix-up has not started).  Returns false if a wait gave up.
     bool pre_done = false;  // issuer: the current item's pre-pass ran in the previous item's tail
     auto prepass = [&](int pitem) {
         const int psig = pitem / p.BH, phead = pitem % p.BH;
         const int pt0 = psig * p.L, pnt = min(p.L, p.M - pt0);
+        if (!kState && psig + 1 >= p.G) {  // the last segment of a head: nothing reads its S prefix
+            mbar_arrive(&ms->bar[bEvP]);
+            return true;
+        }
         auto ps = [](int j) { return (j & 3) == 0 ? kK : (j & 3) == 1 ? kV : (j & 3) == 2 ? kW : kQ1; };
         for (int j = 0; j < pnt && j < 4; ++j) load_tile(ps(j), &tm_k, phead, (pt0 + j) * kTile);
         for (int j = 0; j < pnt; ++j) {
@@ -446,9 +456,9 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 if (!early && !prepass(item)) break;
                 if (!bar_wait(ms, bEvP, ip, p)) break;  // the pre-pass slots are free again
                 // first tile's inputs (K tile 0 is still in slot K after a pre-pass of <= 4 tiles that
-                // ran just now)
+                // ran just now, if there was one)
                 load_tile(kQ0, &tm_q, head, t0 * kTile);
-                const bool reload_k = early || nt > 4;
+                const bool reload_k = early || nt > 4 || (!kState && sigma + 1 >= p.G);
                 if (reload_k) load_tile(kK, &tm_k, head, t0 * kTile);
                 load_tile(kV, &tm_v, head, t0 * kTile);
                 if (wait_ld(kQ0) && (!reload_k || wait_ld(kK))) {
@@ -592,6 +602,8 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
             float tr_s = 0.f, cs = 0.f;
 
             // ---- 1. S chain: carry-in S of the segment, publish the inclusive prefix ----
+            // (the last segment of a head publishes none unless the final state is wanted)
+            const bool s_agg = kState || sigma + 1 < p.G;
             bar_wait(ms, bEvP, ip, p);
             tc_fence_after();
             if (sigma > 0 && et == 0) chain_wait(&flagS[head * 2 + ((sigma - 1) & 1)], (unsigned)sigma, p, 1, item);
@@ -609,6 +621,17 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                                             : st_row ? __ldcg(st_row + c) : make_float4(0.f, 0.f, 0.f, 0.f);
                     sp[4 * c] = v4.x; sp[4 * c + 1] = v4.y; sp[4 * c + 2] = v4.z; sp[4 * c + 3] = v4.w;
                 }
+                if (s_agg) {
+                    // inclusive S prefix of this segment -> ring, published before this segment's set-up
+                    float agg[32];
+                    ld32(tb + lane_base + kTS + c0, agg);
+                    float4 *rc = reinterpret_cast<float4 *>(ring_cur);
+#pragma unroll
+                    for (int j = 0; j < 32; j += 4)
+                        __stcg(rc + ring4(j / 4, et), make_float4(sp[j] + agg[j], sp[j + 1] + agg[j + 1],
+                                                                 sp[j + 2] + agg[j + 2], sp[j + 3] + agg[j + 3]));
+                }
+                pub_arrive(kBarPubS);  // S prefix in the ring
                 // trace -> shift (the diagonal element of row r lies in column block qd)
                 float s = 0.f;
                 if (cq == qd) {
@@ -622,16 +645,6 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
 #pragma unroll
                 for (int w = 0; w < kEpiWarps; ++w) tr_s += ms->red[w];
                 cs = bf16_round(tr_s / kD);
-                {
-                    // inclusive S prefix of this segment -> ring
-                    float agg[32];
-                    ld32(tb + lane_base + kTS + c0, agg);
-                    float4 *rc = reinterpret_cast<float4 *>(ring_cur);
-#pragma unroll
-                    for (int j = 0; j < 32; j += 4)
-                        __stcg(rc + ring4(j / 4, et), make_float4(sp[j] + agg[j], sp[j + 1] + agg[j + 1],
-                                                                 sp[j + 2] + agg[j + 2], sp[j + 3] + agg[j + 3]));
-                }
                 // S carry in TMEM
                 uint32_t u[32];
 #pragma unroll
@@ -654,7 +667,6 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 tmem_st_wait();
             }
             fence_async_smem();
-            pub_arrive(kBarPubS);  // S prefix in the ring
 
             // ---- 2. sweep ----
             // e carry += column sums of X (sum over the four lane quadrants, in a fixed order)
@@ -1002,20 +1014,50 @@ FusedLayout fused_layout(int BH, int n) {
     return L;
 }
 
+// Predicted duration (us) of the ticket schedule with segments of L tiles: items in ticket order go
+// to the SM that frees first; an item costs 5.5 us per tile of sweep and, for segments > 0, 2.1 us
+// per fix-up tile and 7 us of chain set-up (2 us for a first segment); in the first wave the S
+// prefix ripples through the concurrent segments of a head (about 5.6 us per segment, after a cold
+// pre-pass of 4.7 us).  Constants measured on B2 H16 n16384 d128.
+double predicted_span(int BH, int M, int L, int sms) {
+    std::priority_queue<double, std::vector<double>, std::greater<double>> free_at;
+    for (int i = 0; i < sms; ++i) free_at.push(0.0);
+    double span = 0.0;
+    const int G = (M + L - 1) / L;
+    for (int sg = 0; sg < G; ++sg) {
+        const int li = std::min(L, M - sg * L);
+        for (int h = 0; h < BH; ++h) {
+            const double t = free_at.top();
+            free_at.pop();
+            double c = 5.5 * li + (sg > 0 ? 2.1 * li + 7.0 : 2.0);
+            if (t == 0.0) c += 4.7 + 5.6 * sg;
+            free_at.push(t + c);
+            span = std::max(span, t + c);
+        }
+    }
+    return span;
+}
+
 int segment_tiles(int BH, int M, int sms) {
     if (const char *e = getenv("HLA_FUSED_SEGMENT_TILES")) {
         int v = atoi(e);
         if (v > 0) return v < M ? v : M;
     }
-    // enough segments that the heads fill the SMs several times over, but long
-    // enough that the chained scans and per-segment set-up stay short (measured
-    // on B2 H16 n16384: 4..6 tiles within 1%, 3 and 8+ slower)
-    int L = 6;
-    if ((long long)BH * ((M + L - 1) / L) < 2LL * sms) L = 2;
-    if (2 * BH >= sms) L = M;  // heads enough to occupy the SMs: one segment per head, no chains
-    return L < M ? L : M;
+    if (2 * BH >= sms) return M;  // heads enough to occupy the SMs: one segment per head, no chains
+    // Segments of 2..8 tiles (the range measured): the length whose schedule is predicted to end
+    // first (on B2 H16 n16384 the prediction picks 7, measured best among 4..13; 6 is 3.5 % slower
+    // there because 704 items leave the last wave of the 152 SMs partly idle).
+    int best = 2;
+    double best_t = 1e300;
+    for (int L = 2; L <= 8 && L <= M; ++L) {
+        const double t = predicted_span(BH, M, L, sms);
+        if (t < best_t) {
+            best_t = t;
+            best = L;
+        }
+    }
+    return best < M ? best : M;
 }
-
 
 // ---------------------------------------------------------------------------
 // final state (state_out): C = C_0 + Q^T V and m = m_0 + Q^T 1 on the tensor
