@@ -393,10 +393,14 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
     auto lk = [&](int s) { return sb4 + (uint32_t)s * (kTileBytes >> 4) + kLboK; };
     auto lm = [&](int s) { return sb4 + (uint32_t)s * (kTileBytes >> 4) + kLboMN; };
 
-    auto load_tile = [&](int s, const CUtensorMap *map, int head, int tok0) {
+    // L2 priorities: tiles read again later (Q and the provisional outputs of segments > 0, until the
+    // fix-up; K from the pre-pass to the sweep) are kept, tiles at their last use go first
+    const uint64_t pol_first = l2_policy_evict_first(), pol_last = l2_policy_evict_last();
+    const uint64_t pol_normal = l2_policy_evict_normal();
+    auto load_tile = [&](int s, const CUtensorMap *map, int head, int tok0, uint64_t pol) {
         mbar_arrive_expect_tx(&ms->bar[bLd0 + s], kTileBytes);
-        tma_load_3d(slot(s), map, &ms->bar[bLd0 + s], 0, tok0, head);
-        tma_load_3d(slot(s) + kBlockBytes, map, &ms->bar[bLd0 + s], 64, tok0, head);
+        tma_load_3d_hint(slot(s), map, &ms->bar[bLd0 + s], 0, tok0, head, pol);
+        tma_load_3d_hint(slot(s) + kBlockBytes, map, &ms->bar[bLd0 + s], 64, tok0, head, pol);
     };
     auto wait_ld = [&](int s) {
         const uint32_t par = (ld_par >> s) & 1u;
@@ -418,7 +422,7 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
             return true;
         }
         auto ps = [](int j) { return (j & 3) == 0 ? kK : (j & 3) == 1 ? kV : (j & 3) == 2 ? kW : kQ1; };
-        for (int j = 0; j < pnt && j < 4; ++j) load_tile(ps(j), &tm_k, phead, (pt0 + j) * kTile);
+        for (int j = 0; j < pnt && j < 4; ++j) load_tile(ps(j), &tm_k, phead, (pt0 + j) * kTile, pol_normal);
         for (int j = 0; j < pnt; ++j) {
             const int sl = ps(j);
             if (!wait_ld(sl)) return false;
@@ -427,7 +431,7 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
             if (j + 4 < pnt) {  // long segment: reuse this slot once its MMA is done
                 umma_commit(&ms->bar[bPre]);
                 if (!bar_wait(ms, bPre, (n_pre++) & 1, p)) return false;
-                load_tile(sl, &tm_k, phead, (pt0 + j + 4) * kTile);
+                load_tile(sl, &tm_k, phead, (pt0 + j + 4) * kTile, pol_normal);
             }
         }
         umma_commit(&ms->bar[bEvP]);
@@ -457,10 +461,11 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 if (!bar_wait(ms, bEvP, ip, p)) break;  // the pre-pass slots are free again
                 // first tile's inputs (K tile 0 is still in slot K after a pre-pass of <= 4 tiles that
                 // ran just now, if there was one)
-                load_tile(kQ0, &tm_q, head, t0 * kTile);
+                const uint64_t pol_q = sigma > 0 ? pol_last : pol_first;  // Q is read again by the fix-up
+                load_tile(kQ0, &tm_q, head, t0 * kTile, pol_q);
                 const bool reload_k = early || nt > 4 || (!kState && sigma + 1 >= p.G);
-                if (reload_k) load_tile(kK, &tm_k, head, t0 * kTile);
-                load_tile(kV, &tm_v, head, t0 * kTile);
+                if (reload_k) load_tile(kK, &tm_k, head, t0 * kTile, pol_first);
+                load_tile(kV, &tm_v, head, t0 * kTile, pol_first);
                 if (wait_ld(kQ0) && (!reload_k || wait_ld(kK))) {
                     tc_fence_after();
                     mma128<false, false>(tb + kTA, lk(kQ0), lk(kK), 0u);  // A = Q K^T
@@ -476,7 +481,7 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                     const uint32_t tp = n_tiles & 1;
                     const int qs = (j & 1) ? kQ1 : kQ0, qo = (j & 1) ? kQ0 : kQ1;
                     // slot qo (Q of the previous tile, last read by its O MMA) takes the next Q
-                    if (j + 1 < nt) load_tile(qo, &tm_q, head, (t0 + j + 1) * kTile);
+                    if (j + 1 < nt) load_tile(qo, &tm_q, head, (t0 + j + 1) * kTile, pol_q);
                     // X = Q R_hi + Q R_lo + W_hi K + W_lo K; the Q R part runs while W is built.  For the
                     // first tile of a segment the split of S_p comes with W; later ones wait for the
                     // split and for the previous output to have left TMEM columns X.
@@ -494,7 +499,7 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                     mma128<true, true>(tb + kTS, lm(kK), lm(kK), 1u);         // S += K^T K
                     umma_commit(&ms->bar[bEvS]);
                     if (!bar_wait(ms, bEvS, tp, p)) break;  // X and S MMAs done: slot K free
-                    if (j + 1 < nt) load_tile(kK, &tm_k, head, (t0 + j + 1) * kTile);
+                    if (j + 1 < nt) load_tile(kK, &tm_k, head, (t0 + j + 1) * kTile, pol_first);
                     if (!bar_wait(ms, bEpX, tp, p)) break;  // X_hi, X_lo in SX, W; D_p read out of TMEM
                     tc_fence_after();
                     mma128<false, false>(tb + kTA, lk(qs), lk(kSX), 0u);      // T = Q X_hi^T
@@ -518,7 +523,7 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                         tc_fence_after();
                         mma128<false, false>(tb + kTA, lk(qo), lk(kK), 0u);
                         umma_commit(&ms->bar[bEvA]);
-                        load_tile(kV, &tm_v, head, (t0 + j + 1) * kTile);
+                        load_tile(kV, &tm_v, head, (t0 + j + 1) * kTile, pol_first);
                     }
                     ++n_tiles;
                 }
@@ -541,8 +546,8 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                         // which also stages the result, and TMEM region for F)
                         auto load_fix = [&](int j) {
                             const int i = j % 3;
-                            load_tile(fix_q(i), &tm_q, head, (t0 + j) * kTile);
-                            load_tile(fix_o(i), &tm_o, head, (t0 + j) * kTile);
+                            load_tile(fix_q(i), &tm_q, head, (t0 + j) * kTile, pol_first);
+                            load_tile(fix_o(i), &tm_o, head, (t0 + j) * kTile, pol_first);
                         };
                         for (int j = 0; j < nt && j < 3; ++j) load_fix(j);
                         for (int j = 0; j < nt; ++j) {
@@ -822,9 +827,10 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 }
                 fence_async_smem();
                 epi_sync();  // also: every denominator read before part is reused
-                if (et == 0) {
-                    tma_store_3d(&tm_o, slot(kSD), 0, tok0, head);
-                    if (p.out_blocks > 1) tma_store_3d(&tm_o, slot(kSD) + kBlockBytes, 64, tok0, head);
+                if (et == 0) {  // provisional outputs stay in L2 for the fix-up
+                    const uint64_t pol = sigma > 0 ? l2_policy_evict_last() : l2_policy_evict_first();
+                    tma_store_3d_hint(&tm_o, slot(kSD), 0, tok0, head, pol);
+                    if (p.out_blocks > 1) tma_store_3d_hint(&tm_o, slot(kSD) + kBlockBytes, 64, tok0, head, pol);
                     tma_store_commit();
                 }
                 ++n_tiles;
@@ -910,8 +916,9 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                         fence_async_smem();
                         epi_sync();  // also: every denominator read before the next tile's partials
                         if (et == 0) {
-                            tma_store_3d(&tm_o, ot, 0, tok0, head);
-                            if (p.out_blocks > 1) tma_store_3d(&tm_o, ot + kBlockBytes, 64, tok0, head);
+                            const uint64_t pol = l2_policy_evict_first();
+                            tma_store_3d_hint(&tm_o, ot, 0, tok0, head, pol);
+                            if (p.out_blocks > 1) tma_store_3d_hint(&tm_o, ot + kBlockBytes, 64, tok0, head, pol);
                             tma_store_commit();
                         }
                         fx_par ^= 1u << i;
