@@ -95,7 +95,8 @@ enum Bar {
     bEpF = 21,  // + fix-up buffer: its slots and TMEM region are free again
     bEpDF = 24,
     bEpO = 25,  // O read out of TMEM
-    kNumBars = 26
+    bEpOut = 26,  // provisional outputs of the segment written (segments > 0)
+    kNumBars = 27
 };
 constexpr int kFirstEpiBar = bEpW;
 
@@ -541,15 +542,18 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
 
                 // ---- 3. fix-up of segments > 0 ----
                 if (sigma > 0 && !ms->abort_flag) {
-                    if (bar_wait(ms, bEpDF, n_dfix & 1, p)) {  // D prefix (bf16) in SD; outputs written
-                        // three tiles in flight: tile j uses buffer j % 3 (Q slot, provisional output slot,
-                        // which also stages the result, and TMEM region for F)
-                        auto load_fix = [&](int j) {
-                            const int i = j % 3;
-                            load_tile(fix_q(i), &tm_q, head, (t0 + j) * kTile, pol_first);
-                            load_tile(fix_o(i), &tm_o, head, (t0 + j) * kTile, pol_first);
-                        };
+                    // three tiles in flight: tile j uses buffer j % 3 (Q slot, provisional output slot,
+                    // which also stages the result, and TMEM region for F)
+                    auto load_fix = [&](int j) {
+                        const int i = j % 3;
+                        load_tile(fix_q(i), &tm_q, head, (t0 + j) * kTile, pol_first);
+                        load_tile(fix_o(i), &tm_o, head, (t0 + j) * kTile, pol_first);
+                    };
+                    // the first loads as soon as the provisional outputs are written, while the D
+                    // prefix may still be on its way
+                    if (bar_wait(ms, bEpOut, n_dfix & 1, p))
                         for (int j = 0; j < nt && j < 3; ++j) load_fix(j);
+                    if (bar_wait(ms, bEpDF, n_dfix & 1, p)) {  // D prefix (bf16) in SD
                         for (int j = 0; j < nt; ++j) {
                             const int i = j % 3;
                             if (!wait_ld(fix_q(i)) || !wait_ld(fix_o(i))) break;
@@ -836,6 +840,10 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 ++n_tiles;
             }
             if (need_e && nt > 0) add_ecol(ecol);  // the last tile's X
+            if (sigma > 0) {  // the fix-up may load the provisional outputs once they are written
+                if (et == 0) tma_store_wait_all();
+                epi_arrive(ms, bEpOut);
+            }
 
             // ---- 3. D chain and fix-up ----
             {
@@ -871,7 +879,6 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 pub_arrive(kBarPubD);  // D and e prefixes in the ring
                 if (sigma > 0) {
                     if (cq == 0) ms->eloc[r] = eprev;  // now e of the prefix, for the fix-up denominators
-                    if (et == 0) tma_store_wait_all();  // provisional outputs written before they are re-read
                     fence_async_smem();
                     epi_sync();
                     epi_arrive(ms, bEpDF);
