@@ -87,14 +87,78 @@ C3Layout c3_layout(int BH, int n, int d, int dv, int chunk) {
 template <typename T>
 __device__ __forceinline__ float ld_tok(const T *p) { return to_f32(*p); }
 
-// dst[r * ld + c] = sum_k A(r,k) B(k,c) with accessor lambdas
-template <typename FA, typename FB>
-__device__ __forceinline__ void smm(float *dst, int ld, int rows, int cols, int kdim, FA a, FB b) {
-    for (int i = threadIdx.x; i < rows * cols; i += blockDim.x) {
-        const int r = i / cols, c = i % cols;
-        float s = 0.f;
-        for (int k = 0; k < kdim; ++k) s += a(r, k) * b(k, c);
-        dst[r * ld + c] = s;
+// dst (row stride ld) = or += sum_k a(r, k) b(k, c) over rows x cols.  Each thread forms a 2 x 2 block of
+// outputs, rows r and r + rows/2, columns c and c + cols/2, so that every operand element it loads is used
+// twice (the products are bound by shared-memory loads); with an odd size, one output per thread.  The
+// same thread owns the same outputs in every call of the same shape, so accumulating calls need no barrier
+// between them.
+template <bool kAcc, typename FA, typename FB>
+__device__ __forceinline__ void smm2(float *dst, int ld, int rows, int cols, int kdim, FA a, FB b) {
+    if ((rows | cols) & 1) {
+        for (int i = threadIdx.x; i < rows * cols; i += blockDim.x) {
+            const int r = i / cols, c = i % cols;
+            float s = 0.f;
+            for (int k = 0; k < kdim; ++k) s += a(r, k) * b(k, c);
+            dst[r * ld + c] = kAcc ? dst[r * ld + c] + s : s;
+        }
+        return;
+    }
+    const int hr = rows >> 1, hc = cols >> 1;
+    for (int i = threadIdx.x; i < hr * hc; i += blockDim.x) {
+        const int r = i / hc, c = i % hc;
+        float s00 = 0.f, s01 = 0.f, s10 = 0.f, s11 = 0.f;
+        for (int k = 0; k < kdim; ++k) {
+            const float a0 = a(r, k), a1 = a(r + hr, k), b0 = b(k, c), b1 = b(k, c + hc);
+            s00 += a0 * b0;
+            s01 += a0 * b1;
+            s10 += a1 * b0;
+            s11 += a1 * b1;
+        }
+        float *d0 = dst + r * ld + c, *d1 = dst + (r + hr) * ld + c;
+        if (kAcc) {
+            d0[0] += s00; d0[hc] += s01; d1[0] += s10; d1[hc] += s11;
+        } else {
+            d0[0] = s00; d0[hc] = s01; d1[0] = s10; d1[hc] = s11;
+        }
+    }
+}
+
+// Triangular products, two outputs per thread that share one operand and their summation range:
+// rows:  dst[t][c] (+)= sum_{k in [lo(t), hi(t))} a(t, k) b(k, c), columns c and c + cols/2
+// cols:  dst[t][c] (+)= sum_{k in [0, hi(c))} a(t, k) b(k, c), rows t and t + rows/2
+// (odd widths: one output per thread)
+template <bool kAcc, typename FA, typename FB, typename FL, typename FH>
+__device__ __forceinline__ void smm_rows(float *dst, int ld, int rows, int cols, FA a, FB b, FL lo, FH hi) {
+    const int hc = (cols & 1) ? cols : cols >> 1, per = (cols & 1) ? 1 : 2;
+    for (int i = threadIdx.x; i < rows * hc; i += blockDim.x) {
+        const int t = i / hc, c = i % hc;
+        float s0 = 0.f, s1 = 0.f;
+        const int k1 = hi(t);
+        for (int k = lo(t); k < k1; ++k) {
+            const float av = a(t, k);
+            s0 += av * b(k, c);
+            if (per == 2) s1 += av * b(k, c + hc);
+        }
+        float *d0 = dst + t * ld + c;
+        d0[0] = kAcc ? d0[0] + s0 : s0;
+        if (per == 2) d0[hc] = kAcc ? d0[hc] + s1 : s1;
+    }
+}
+template <bool kAcc, typename FA, typename FB, typename FH>
+__device__ __forceinline__ void smm_cols(float *dst, int ld, int rows, int cols, FA a, FB b, FH hi) {
+    const int hr = (rows & 1) ? rows : rows >> 1, per = (rows & 1) ? 1 : 2;
+    for (int i = threadIdx.x; i < hr * cols; i += blockDim.x) {
+        const int t = i / cols, c = i % cols;
+        float s0 = 0.f, s1 = 0.f;
+        const int k1 = hi(c);
+        for (int k = 0; k < k1; ++k) {
+            const float bv = b(k, c);
+            s0 += a(t, k) * bv;
+            if (per == 2) s1 += a(t + hr, k) * bv;
+        }
+        float *d0 = dst + t * ld + c;
+        d0[0] = kAcc ? d0[0] + s0 : s0;
+        if (per == 2) d0[hr * ld] = kAcc ? d0[hr * ld] + s1 : s1;
     }
 }
 
@@ -135,16 +199,16 @@ __global__ void __launch_bounds__(kT3c) c3_local_kernel(const T *__restrict__ q,
     __syncthreads();
     float *rec = L.loc(ws, hd, c);
     // first-order sums
-    smm(rec + L.oSK, d, d, d, W, [&](int r, int t) { return Ks[t * ld + r]; }, [&](int t, int cc) { return Ks[t * ld + cc]; });
-    smm(rec + L.oSQ, d, d, d, W, [&](int r, int t) { return Qs[t * ld + r]; }, [&](int t, int cc) { return Qs[t * ld + cc]; });
-    smm(rec + L.oP, dv, d, dv, W, [&](int r, int t) { return Ks[t * ld + r]; }, [&](int t, int cc) { return Vs[t * lv + cc]; });
+    smm2<false>(rec + L.oSK, d, d, d, W, [&](int r, int t) { return Ks[t * ld + r]; }, [&](int t, int cc) { return Ks[t * ld + cc]; });
+    smm2<false>(rec + L.oSQ, d, d, d, W, [&](int r, int t) { return Qs[t * ld + r]; }, [&](int t, int cc) { return Qs[t * ld + cc]; });
+    smm2<false>(rec + L.oP, dv, d, dv, W, [&](int r, int t) { return Ks[t * ld + r]; }, [&](int t, int cc) { return Vs[t * lv + cc]; });
     for (int r = threadIdx.x; r < d; r += blockDim.x) {
         float s = 0.f;
         for (int t = 0; t < W; ++t) s += Ks[t * ld + r];
         rec[L.om + r] = s;
     }
     if (!masked) return;
-    smm(A, lw, W, W, d, [&](int t, int j) { return Qs[t * ld + j]; }, [&](int j, int s) { return Ks[s * ld + j]; });
+    smm2<false>(A, lw, W, W, d, [&](int t, int j) { return Qs[t * ld + j]; }, [&](int j, int s) { return Ks[s * ld + j]; });
     __syncthreads();
     for (int t = threadIdx.x; t < W; t += blockDim.x) {
         a[t] = A[t * lw + t];
@@ -154,14 +218,13 @@ __global__ void __launch_bounds__(kT3c) c3_local_kernel(const T *__restrict__ q,
         b[t] = bs;
         ym[t] = ys;
     }
+    // Z = diag(a) Y_loc + diag(b) V + N V with Y_loc = (L.A) V and N_ts = [s > t] A_st a_s
+    smm_rows<false>(Z, lv, W, dv, [&](int t, int j) { return A[t * lw + j]; }, [&](int j, int cc) { return Vs[j * lv + cc]; },
+                    [](int) { return 0; }, [](int t) { return t + 1; });
     __syncthreads();
-    // Z = diag(a) Y_loc + diag(b) V + N V with Y_loc = (L.A) V and (N V)_t = sum_{s>t} A_st a_s v_s
     for (int i = threadIdx.x; i < W * dv; i += blockDim.x) {
         const int t = i / dv, cc = i % dv;
-        float y = 0.f, nv = 0.f;
-        for (int j = 0; j <= t; ++j) y += A[t * lw + j] * Vs[j * lv + cc];
-        for (int s = t + 1; s < W; ++s) nv += A[s * lw + t] * a[s] * Vs[s * lv + cc];
-        Z[t * lv + cc] = a[t] * y + b[t] * Vs[t * lv + cc] + nv;
+        Z[t * lv + cc] = a[t] * Z[t * lv + cc] + b[t] * Vs[t * lv + cc];
     }
     for (int t = threadIdx.x; t < W; t += blockDim.x) {
         float nv = 0.f;
@@ -169,11 +232,14 @@ __global__ void __launch_bounds__(kT3c) c3_local_kernel(const T *__restrict__ q,
         zeta[t] = a[t] * ym[t] + b[t] + nv;
     }
     __syncthreads();
-    smm(rec + L.oF, dv, d, dv, W, [&](int r, int t) { return Ks[t * ld + r]; }, [&](int t, int cc) { return Z[t * lv + cc]; });
-    smm(rec + L.oR, dv, d, dv, W, [&](int r, int t) { return Qs[t * ld + r] * a[t]; },
-        [&](int t, int cc) { return Vs[t * lv + cc]; });
-    smm(rec + L.oU, d, d, d, W, [&](int r, int t) { return Ks[t * ld + r] * a[t]; },
-        [&](int t, int cc) { return Qs[t * ld + cc]; });
+    smm_rows<true>(Z, lv, W, dv, [&](int t, int s) { return A[s * lw + t] * a[s]; }, [&](int s, int cc) { return Vs[s * lv + cc]; },
+                   [](int t) { return t + 1; }, [&](int) { return W; });
+    __syncthreads();
+    smm2<false>(rec + L.oF, dv, d, dv, W, [&](int r, int t) { return Ks[t * ld + r]; }, [&](int t, int cc) { return Z[t * lv + cc]; });
+    smm2<false>(rec + L.oR, dv, d, dv, W, [&](int r, int t) { return Qs[t * ld + r] * a[t]; },
+                [&](int t, int cc) { return Vs[t * lv + cc]; });
+    smm2<false>(rec + L.oU, d, d, d, W, [&](int r, int t) { return Ks[t * ld + r] * a[t]; },
+                [&](int t, int cc) { return Qs[t * ld + cc]; });
     for (int r = threadIdx.x; r < d; r += blockDim.x) {
         float se = 0.f, sr = 0.f;
         for (int t = 0; t < W; ++t) {
@@ -276,7 +342,7 @@ __global__ void __launch_bounds__(kT3c) c3_bracket_kernel(const T *__restrict__ 
         __syncthreads();
     }
     // bq_t = k_t^T S^Q_p k_t
-    smm(T1, ld, W, d, d, [&](int t, int j) { return Ks[t * ld + j]; }, [&](int j, int cc) { return SQp[j * d + cc]; });
+    smm2<false>(T1, ld, W, d, d, [&](int t, int j) { return Ks[t * ld + j]; }, [&](int j, int cc) { return SQp[j * d + cc]; });
     __syncthreads();
     for (int t = threadIdx.x; t < W; t += blockDim.x) {
         float s = 0.f;
@@ -284,17 +350,12 @@ __global__ void __launch_bounds__(kT3c) c3_bracket_kernel(const T *__restrict__ 
         bq[t] = s;
     }
     __syncthreads();
-    // every thread reads and rewrites only its own elements of F_c and eta_c
-    for (int i = threadIdx.x; i < d * dv; i += blockDim.x) {
-        const int r = i / dv, cc = i % dv;
-        float a1 = 0.f, a2 = 0.f, a3 = 0.f;
-        for (int x = 0; x < d; ++x) {
-            a1 += SKp[r * d + x] * R[x * dv + cc];
-            a3 += U[r * d + x] * Pp[x * dv + cc];
-        }
-        for (int t = 0; t < W; ++t) a2 += Ks[t * ld + r] * bq[t] * Vs[t * lv + cc];
-        rec[L.oF + i] += a1 + a2 + a3;
-    }
+    // F_c += S^K_p R + U P_p + K^T diag(bq) V (each thread adds to the same elements of F_c in all three)
+    float *Fc = rec + L.oF;
+    smm2<true>(Fc, dv, d, dv, d, [&](int r, int x) { return SKp[r * d + x]; }, [&](int x, int cc) { return R[x * dv + cc]; });
+    smm2<true>(Fc, dv, d, dv, d, [&](int r, int x) { return U[r * d + x]; }, [&](int x, int cc) { return Pp[x * dv + cc]; });
+    smm2<true>(Fc, dv, d, dv, W, [&](int r, int t) { return Ks[t * ld + r] * bq[t]; },
+               [&](int t, int cc) { return Vs[t * lv + cc]; });
     for (int r = threadIdx.x; r < d; r += blockDim.x) {
         float a1 = 0.f, a2 = 0.f, a3 = 0.f;
         for (int x = 0; x < d; ++x) {
@@ -331,6 +392,7 @@ __global__ void __launch_bounds__(kT3c) c3_out_kernel(const T *__restrict__ q, c
     const int t0 = c * W, w = min(W, L.n - t0);
     float *Qs = sm, *Ks = Qs + W * ld, *Vs = Ks + W * ld, *A = Vs + W * lv, *Cm = A + W * lw;
     float *M1 = Cm + W * lw, *M2 = M1 + W * lm, *a = M2 + W * lm, *b = a + W, *x1 = b + W, *den = x1 + W;
+    float *Yb = den + W;  // W x dv (row stride dv + 1): Y, then the numerator
     load_chunk(q, k, v, Qs, Ks, Vs, hd, t0, w, W, L.n, d, dv);
     __syncthreads();
     const float *pr = L.pre(ws, hd, c);
@@ -338,10 +400,10 @@ __global__ void __launch_bounds__(kT3c) c3_out_kernel(const T *__restrict__ q, c
     const float *Fp = pr + L.pF, *ep = pr + L.pe;
     T *Oh = out + ((size_t)hd * L.n + t0) * dv;
     if (masked) {
-        smm(A, lw, W, W, d, [&](int t, int j) { return Qs[t * ld + j]; }, [&](int j, int s) { return Ks[s * ld + j]; });
+        smm2<false>(A, lw, W, W, d, [&](int t, int j) { return Qs[t * ld + j]; }, [&](int j, int s) { return Ks[s * ld + j]; });
         // M1 = K S^Q_p, M2 = Q S^K_p  (W x d)
-        smm(M1, lm, W, d, d, [&](int t, int j) { return Ks[t * ld + j]; }, [&](int j, int cc) { return SQp[j * d + cc]; });
-        smm(M2, lm, W, d, d, [&](int t, int j) { return Qs[t * ld + j]; }, [&](int j, int cc) { return SKp[j * d + cc]; });
+        smm2<false>(M1, lm, W, d, d, [&](int t, int j) { return Ks[t * ld + j]; }, [&](int j, int cc) { return SQp[j * d + cc]; });
+        smm2<false>(M2, lm, W, d, d, [&](int t, int j) { return Qs[t * ld + j]; }, [&](int j, int cc) { return SKp[j * d + cc]; });
         __syncthreads();
         for (int s = threadIdx.x; s < W; s += blockDim.x) {
             a[s] = A[s * lw + s];
@@ -355,43 +417,48 @@ __global__ void __launch_bounds__(kT3c) c3_out_kernel(const T *__restrict__ q, c
             b[s] = bs;
             x1[s] = qm + ys;  // (Q m_p + (L.A) 1)_s
         }
-        // C_ts = q_t^T S^K_p q_s + sum_{i<s} A_ti A_si  (s <= t)
+        // C_ts = q_t^T S^K_p q_s + sum_{i<s} A_ti A_si for s <= t, 0 above the diagonal; Y = Q P_p + (L.A) V
+        smm2<false>(Cm, lw, W, W, d, [&](int t, int j) { return M2[t * lm + j]; }, [&](int j, int s) { return Qs[s * ld + j]; });
+        smm2<false>(Yb, lv, W, dv, d, [&](int s, int j) { return Qs[s * ld + j]; }, [&](int j, int cc) { return Pp[j * dv + cc]; });
+        __syncthreads();  // the accumulating products below own other elements
+        smm_cols<true>(Cm, lw, W, W, [&](int t, int x) { return A[t * lw + x]; }, [&](int x, int s) { return A[s * lw + x]; },
+                       [](int s) { return s; });
+        smm_rows<true>(Yb, lv, W, dv, [&](int s, int j) { return A[s * lw + j]; }, [&](int j, int cc) { return Vs[j * lv + cc]; },
+                       [](int) { return 0; }, [](int s) { return s + 1; });
+        __syncthreads();
         for (int i = threadIdx.x; i < W * W; i += blockDim.x) {
             const int t = i / W, s = i % W;
-            float cv = 0.f;
-            if (s <= t) {
-                for (int j = 0; j < d; ++j) cv += M2[t * lm + j] * Qs[s * ld + j];
-                for (int x = 0; x < s; ++x) cv += A[t * lw + x] * A[s * lw + x];
-            }
-            Cm[t * lw + s] = cv;
+            if (s > t) Cm[t * lw + s] = 0.f;
         }
-        __syncthreads();
-        // M1 <- G1 = diag(a) Y + diag(b) V with Y = Q P_p + (L.A) V;  M2 <- G2 = diag(a) V
+        // M1 <- G1 = diag(a) Y + diag(b) V;  M2 <- G2 = diag(a) V
         for (int i = threadIdx.x; i < W * dv; i += blockDim.x) {
             const int s = i / dv, cc = i % dv;
-            float y = 0.f;
-            for (int j = 0; j < d; ++j) y += Qs[s * ld + j] * Pp[j * dv + cc];
-            for (int j = 0; j <= s; ++j) y += A[s * lw + j] * Vs[j * lv + cc];
-            M1[s * lm + cc] = a[s] * y + b[s] * Vs[s * lv + cc];
+            M1[s * lm + cc] = a[s] * Yb[s * lv + cc] + b[s] * Vs[s * lv + cc];
             M2[s * lm + cc] = a[s] * Vs[s * lv + cc];
         }
+        __syncthreads();
         for (int t = threadIdx.x; t < W; t += blockDim.x) {
             float dn = 0.f;
             for (int j = 0; j < d; ++j) dn += Qs[t * ld + j] * ep[j];
             for (int s = 0; s <= t; ++s) dn += A[t * lw + s] * (a[s] * x1[s] + b[s]) + Cm[t * lw + s] * a[s];
             den[t] = dn;
         }
+        // num = Q F_p + (L.A) G1 + C G2
+        smm2<false>(Yb, lv, W, dv, d, [&](int t, int j) { return Qs[t * ld + j]; }, [&](int j, int cc) { return Fp[j * dv + cc]; });
+        __syncthreads();
+        smm_rows<true>(Yb, lv, W, dv, [&](int t, int s) { return A[t * lw + s]; }, [&](int s, int cc) { return M1[s * lm + cc]; },
+                       [](int) { return 0; }, [](int t) { return t + 1; });
+        smm_rows<true>(Yb, lv, W, dv, [&](int t, int s) { return Cm[t * lw + s]; }, [&](int s, int cc) { return M2[s * lm + cc]; },
+                       [](int) { return 0; }, [](int t) { return t + 1; });
         __syncthreads();
         for (int i = threadIdx.x; i < w * dv; i += blockDim.x) {
             const int t = i / dv, cc = i % dv;
-            float num = 0.f;
-            for (int j = 0; j < d; ++j) num += Qs[t * ld + j] * Fp[j * dv + cc];
-            for (int s = 0; s <= t; ++s) num += A[t * lw + s] * M1[s * lm + cc] + Cm[t * lw + s] * M2[s * lm + cc];
+            const float num = Yb[t * lv + cc];
             from_f32(&Oh[i], normalized ? num / (den[t] + eps) : num);
         }
     } else {
         // A = Q K^T; M1 = X = Q S^K_p + (L.A) K
-        smm(A, lw, W, W, d, [&](int t, int j) { return Qs[t * ld + j]; }, [&](int j, int s) { return Ks[s * ld + j]; });
+        smm2<false>(A, lw, W, W, d, [&](int t, int j) { return Qs[t * ld + j]; }, [&](int j, int s) { return Ks[s * ld + j]; });
         __syncthreads();
         for (int i = threadIdx.x; i < W * d; i += blockDim.x) {
             const int t = i / d, cc = i % d;
@@ -453,8 +520,8 @@ size_t smem_bracket(const C3Layout &L) {
 }
 size_t smem_out(const C3Layout &L) {
     const int lm = (L.d > L.dv ? L.d : L.dv) + 1;
-    return sizeof(float) *
-           ((size_t)L.W * (2 * (L.d + 1) + (L.dv + 1)) + 2 * (size_t)L.W * (L.W + 1) + 2 * (size_t)L.W * lm + 4 * L.W);
+    return sizeof(float) * ((size_t)L.W * (2 * (L.d + 1) + (L.dv + 1)) + 2 * (size_t)L.W * (L.W + 1) +
+                            2 * (size_t)L.W * lm + 4 * L.W + (size_t)L.W * (L.dv + 1));
 }
 
 template <typename T>
