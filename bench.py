@@ -84,6 +84,23 @@ def fwd_flops(w):
     return w.BH * w.n * per
 
 
+def hla3_flops(w):
+    """FLOPs of one masked third-order forward in the chunk-parallel form the kernels compute
+    (Theorem 4; chunk W, 2 per multiply-add): chunk summaries, brackets and outputs."""
+    W, d, dv = min(w.chunk, 64 if max(w.d, w.dv) < 128 else 32), w.d, w.dv
+    tri, stri = W * (W + 1) // 2, W * (W - 1) // 2
+    local = 2 * d * d * W + 3 * d * dv * W + d * d * W + W * W * d + (tri + stri) * dv
+    bracket = W * d * d + 2 * d * d * dv + d * dv * W
+    out = W * W * d + 2 * W * d * d + W * W * d + W * W * W // 2 + W * d * dv + tri * dv + W * d * dv + 2 * tri * dv
+    chunks = w.B * w.H * ((w.n + W - 1) // W)
+    return 2 * chunks * (local + bracket + out)
+
+
+def alu_peak():
+    """fp32 CUDA-core peak: 152 SMs x 128 FP32 lanes x 2 FLOP x 2.07 GHz (maximum SM clock)."""
+    return 152 * 128 * 2 * 2.07e9 / 1e12
+
+
 def dec_bytes(w):
     """Algorithmic bytes of one decode step: read + write of the fp32 state tuple
     (S, C, m, G, h) of every head plus the token I/O."""
@@ -383,6 +400,9 @@ def main():
         result["decode"] = bench_decode(hla, dev, stream, args.decode_steps, hbm_peak, world)
         result["gpu_launches"] += result["decode"]["launches"]
 
+    # ---------------- the other configs: d = 64 forward and third order ----------------
+    if not args.no_decode:
+        result["mid"], result["hla3"] = bench_others(hla, dev, stream, hbm_peak, tc_peak, world)
     if rank == 0 and not args.no_cpu_baseline:
         result["cpu_baseline"] = cpu_baseline()
     if rank == 0:
@@ -390,6 +410,62 @@ def main():
     if world > 1:
         import torch.distributed as dist
         dist.destroy_process_group()
+
+
+def bench_others(hla, dev, stream, hbm_peak, tc_peak, world):
+    """Forward of mid_bf16 (B8 H16 n2048 d64 bf16) and of hla3_f32 (masked third order, B4 H8 n4096 d32
+    fp32): 20 timed calls each after 3 warm-ups, CUDA events on the launching stream."""
+    import torch
+    res = []
+    for name in ("mid_bf16", "hla3_f32"):
+        w = hla_inputs.WORKLOADS[name]
+        q, k, v = hla_inputs.make_workload(w)
+        tq, tk, tv = (hla_inputs.as_torch(x, w.dtype, dev) for x in (q, k, v))
+        out = torch.empty((w.B, w.H, w.n, w.dv), dtype=tq.dtype, device=dev)
+        third = w.order == 3
+        nbytes = (hla.hla3_workspace_bytes if third else hla.hla2_workspace_bytes)(w.B, w.H, w.n, w.d, w.dv, w.chunk,
+                                                                                  tq.dtype)
+        ws = hla.alloc_workspace(nbytes, dev)
+        fwd = hla.hla3_forward if third else hla.hla2_forward
+
+        def call():
+            fwd(tq, tk, tv, out, masked=w.masked, normalized=w.normalized, eps=hla_inputs.EPS, chunk=w.chunk,
+                workspace=ws, stream=stream)
+        for _ in range(3):
+            call()
+        torch.cuda.synchronize()
+        barrier(world)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        steps = 20
+        e0.record(stream)
+        for _ in range(steps):
+            call()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        ms = max_over_ranks(e0.elapsed_time(e1) / steps, world)
+        if hla.hla_poll_error(ws) != 0:
+            raise RuntimeError("device-side error flag set while timing " + name)
+        tok = w.B * w.n * world / (ms * 1e-3)
+        cfg = {"workload": name, "B": w.B, "H": w.H, "n": w.n, "d": w.d, "dv": w.dv, "chunk": w.chunk,
+               "masked": w.masked, "normalized": w.normalized, "tokens": w.dtype, "order": w.order,
+               "ms_per_step": ms, "value": tok, "unit": "tokens/s", "steps": steps}
+        if third:
+            tf = hla3_flops(w) / (ms * 1e-3) / 1e12
+            cfg["roofline"] = {"bound": "alu", "achieved": tf, "peak": alu_peak(), "unit": "TFLOP/s",
+                               "frac": tf / alu_peak(), "traffic": None, "flops": hla3_flops(w),
+                               "peak_kind": "derived (152 SMs x 128 fp32 lanes x 2 x 2.07 GHz)",
+                               "kernel": "c3_local/bracket/out (fp32 CUDA cores)"}
+            cfg["launches"] = steps * 5
+        else:
+            gbs = fwd_bytes(w) / (ms * 1e-3) / 1e9
+            tfl = fwd_flops(w) / (ms * 1e-3) / 1e12
+            cfg["roofline"] = {"bound": "hbm", "achieved": gbs, "peak": hbm_peak, "unit": "GB/s", "frac": gbs / hbm_peak,
+                               "traffic": None, "algorithmic_bytes": fwd_bytes(w), "kernel": "hla2_fused_kernel",
+                               "tensor_view": {"achieved_tflops": tfl, "peak_tflops": tc_peak, "frac": tfl / tc_peak}}
+            cfg["launches"] = steps
+        res.append(cfg)
+        del tq, tk, tv, out, ws
+    return res[0], res[1]
 
 
 def bench_decode(hla, dev, stream, steps, hbm_peak, world):

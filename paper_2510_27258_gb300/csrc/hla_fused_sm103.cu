@@ -310,14 +310,14 @@ constexpr uint32_t kDescHi = (1024u >> 4) | (1u << 14) | (2u << 29);
 // (stride between 64-element blocks) operands
 constexpr uint32_t kLboK = 1u << 16, kLboMN = (kBlockBytes >> 4) << 16;
 
-// One 128 x 128 x 128 product D (+)= A B as eight K = 16 steps, from the low
-// descriptor words of the two operand tiles (address >> 4 | LBO field).  The
-// step offsets are compile-time constants, so each MMA costs one add per operand.
-template <bool A_MN, bool B_MN>
+// One 128 x N x 16 KS product D (+)= A B as KS steps of K = 16 (N = 128, KS = 8 unless given), from the
+// low descriptor words of the two operand tiles (address >> 4 | LBO field).  The step offsets are
+// compile-time constants, so each MMA costs one add per operand.
+template <bool A_MN, bool B_MN, int N = 128, int KS = 8>
 __device__ __forceinline__ void mma128(uint32_t d_tmem, uint32_t a_lo, uint32_t b_lo, uint32_t accumulate) {
-    constexpr uint32_t id = idesc_bf16(128, 128, A_MN, B_MN);
+    constexpr uint32_t id = idesc_bf16(128, N, A_MN, B_MN);
 #pragma unroll
-    for (int kk = 0; kk < 8; ++kk) {
+    for (int kk = 0; kk < KS; ++kk) {
         // K-major: the second 64-element column block is 16 KiB on, 32 B per K step within a block;
         // MN-major: 8 K rows of 128 B (2 KiB with the swizzle atom) per K step
         const uint32_t ka = A_MN ? kk * 128u : (kk >> 2) * (kBlockBytes >> 4) + (kk & 3) * 2u;
@@ -330,9 +330,9 @@ __device__ __forceinline__ void mma128(uint32_t d_tmem, uint32_t a_lo, uint32_t 
 // The same product with A (128 x 128 bf16) in tensor memory, in the layout the epilogue
 // writes: K elements 32g .. 32g+31 of every row packed as bf16 pairs in columns
 // a_tmem + 32g .. +15 (g = 0..3), so that K step kk starts at column 32 (kk / 2) + 8 (kk % 2).
-template <bool B_MN>
+template <bool B_MN, int N = 128>
 __device__ __forceinline__ void mma128_ts(uint32_t d_tmem, uint32_t a_tmem, uint32_t b_lo, uint32_t accumulate) {
-    constexpr uint32_t id = idesc_bf16(128, 128, 0, B_MN);
+    constexpr uint32_t id = idesc_bf16(128, N, 0, B_MN);
 #pragma unroll
     for (int kk = 0; kk < 8; ++kk) {
         const uint32_t kb = B_MN ? kk * 128u : (kk >> 2) * (kBlockBytes >> 4) + (kk & 3) * 2u;
@@ -347,7 +347,7 @@ __device__ __forceinline__ void mma128_ts(uint32_t d_tmem, uint32_t a_tmem, uint
 // kState: the final state is wanted.  Then W and R are split hi + lo and the e carry kept
 // whatever the output (as for the normalised output), and D += X_hi^T V + X_lo^T V is issued
 // before O (X_lo is still in slot W), so that the prefixes in the ring are accurate to fp32 level.
-template <bool kState>
+template <bool kState, bool kNarrow>
 __global__ void __launch_bounds__(kThreads, 1)
 hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                   const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_o, Params p) {
@@ -358,6 +358,10 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const bool issuer = (warp == kIssuerWarp), publisher = (warp == kPubWarp);
     const bool precise = kState || p.normalized;  // hi + lo splits of W and R
+    // head size of the products: 128, or 64 for d = dv = 64 (then the feature columns 64..127 of the tiles,
+    // carries and TMEM regions are neither computed nor read; see the narrow notes in the epilogue)
+    constexpr int kF = kNarrow ? 64 : 128;
+    constexpr int kFS = kF / 16;  // K steps of a contraction over the head size
     const bool need_e = kState || p.normalized;   // the e carry
     constexpr bool d_lo = kState;                 // D with X_lo, issued before O
 
@@ -428,7 +432,7 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
             const int sl = ps(j);
             if (!wait_ld(sl)) return false;
             tc_fence_after();
-            mma128<true, true>(tb + kTS, lm(sl), lm(sl), j > 0 ? 1u : 0u);  // S_agg += K^T K
+            mma128<true, true, kF>(tb + kTS, lm(sl), lm(sl), j > 0 ? 1u : 0u);  // S_agg += K^T K
             if (j + 4 < pnt) {  // long segment: reuse this slot once its MMA is done
                 umma_commit(&ms->bar[bPre]);
                 if (!bar_wait(ms, bPre, (n_pre++) & 1, p)) return false;
@@ -469,7 +473,7 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 load_tile(kV, &tm_v, head, t0 * kTile, pol_first);
                 if (wait_ld(kQ0) && (!reload_k || wait_ld(kK))) {
                     tc_fence_after();
-                    mma128<false, false>(tb + kTA, lk(kQ0), lk(kK), 0u);  // A = Q K^T
+                    mma128<false, false, 128, kFS>(tb + kTA, lk(kQ0), lk(kK), 0u);  // A = Q K^T
                     umma_commit(&ms->bar[bEvA]);
                 }
 
@@ -490,39 +494,39 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                     if (j > 0 && !bar_wait(ms, bEpO, tp ^ 1u, p)) break;
                     if (j == 0 && !bar_wait(ms, bEpW, tp, p)) break;
                     tc_fence_after();
-                    mma128<false, false>(tb + kTX, lk(qs), lk(kSX), 0u);      // X = Q R_hi
-                    if (precise) mma128<false, false>(tb + kTX, lk(qs), lk(kW), 1u);  // += Q R_lo
+                    mma128<false, false, kF, kFS>(tb + kTX, lk(qs), lk(kSX), 0u);      // X = Q R_hi
+                    if (precise) mma128<false, false, kF, kFS>(tb + kTX, lk(qs), lk(kW), 1u);  // += Q R_lo
                     if (j > 0 && !bar_wait(ms, bEpW, tp, p)) break;  // W (hi, lo) ready
                     tc_fence_after();
-                    mma128_ts<true>(tb + kTX, tb + kTA, lm(kK), 1u);          // += W_hi K (W in TMEM)
-                    if (precise) mma128_ts<true>(tb + kTX, tb + kTA + 16, lm(kK), 1u);  // += W_lo K
+                    mma128_ts<true, kF>(tb + kTX, tb + kTA, lm(kK), 1u);          // += W_hi K (W in TMEM)
+                    if (precise) mma128_ts<true, kF>(tb + kTX, tb + kTA + 16, lm(kK), 1u);  // += W_lo K
                     umma_commit(&ms->bar[bEvX]);
-                    mma128<true, true>(tb + kTS, lm(kK), lm(kK), 1u);         // S += K^T K
+                    mma128<true, true, kF>(tb + kTS, lm(kK), lm(kK), 1u);         // S += K^T K
                     umma_commit(&ms->bar[bEvS]);
                     if (!bar_wait(ms, bEvS, tp, p)) break;  // X and S MMAs done: slot K free
                     if (j + 1 < nt) load_tile(kK, &tm_k, head, (t0 + j + 1) * kTile, pol_first);
                     if (!bar_wait(ms, bEpX, tp, p)) break;  // X_hi, X_lo in SX, W; D_p read out of TMEM
                     tc_fence_after();
-                    mma128<false, false>(tb + kTA, lk(qs), lk(kSX), 0u);      // T = Q X_hi^T
-                    mma128<false, false>(tb + kTA, lk(qs), lk(kW), 1u);       // += Q X_lo^T
+                    mma128<false, false, 128, kFS>(tb + kTA, lk(qs), lk(kSX), 0u);      // T = Q X_hi^T
+                    mma128<false, false, 128, kFS>(tb + kTA, lk(qs), lk(kW), 1u);       // += Q X_lo^T
                     umma_commit(&ms->bar[bEvT]);
                     if (!wait_ld(kV)) break;
                     tc_fence_after();
-                    mma128<true, true>(tb + kTD, lm(kSX), lm(kV), 1u);        // D += X_hi^T V
-                    if (d_lo) mma128<true, true>(tb + kTD, lm(kW), lm(kV), 1u);  // D += X_lo^T V
+                    mma128<true, true, kF>(tb + kTD, lm(kSX), lm(kV), 1u);        // D += X_hi^T V
+                    if (d_lo) mma128<true, true, kF>(tb + kTD, lm(kW), lm(kV), 1u);  // D += X_lo^T V
                     umma_commit(&ms->bar[bEvD]);
                     // O = Q D_p (D_p in SD since the X hand-off; TMEM X was read out then) runs while
                     // the epilogue forms T
-                    mma128<false, true>(tb + kTX, lk(qs), lm(kSD), 0u);
+                    mma128<false, true, kF, kFS>(tb + kTX, lk(qs), lm(kSD), 0u);
                     if (!bar_wait(ms, bEpT, tp, p)) break;  // T (bf16) in TMEM A
                     tc_fence_after();
-                    mma128_ts<true>(tb + kTX, tb + kTA, lm(kV), 1u);          // O += T V (T in TMEM)
+                    mma128_ts<true, kF>(tb + kTX, tb + kTA, lm(kV), 1u);          // O += T V (T in TMEM)
                     umma_commit(&ms->bar[bEvO]);
                     if (!bar_wait(ms, bEvO, tp, p)) break;  // T, V and D_p read
                     if (j + 1 < nt) {  // next tile's A = Q K^T overlaps this tile's output epilogue
                         if (!wait_ld(qo) || !wait_ld(kK)) break;
                         tc_fence_after();
-                        mma128<false, false>(tb + kTA, lk(qo), lk(kK), 0u);
+                        mma128<false, false, 128, kFS>(tb + kTA, lk(qo), lk(kK), 0u);
                         umma_commit(&ms->bar[bEvA]);
                         load_tile(kV, &tm_v, head, (t0 + j + 1) * kTile, pol_first);
                     }
@@ -558,7 +562,7 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                             const int i = j % 3;
                             if (!wait_ld(fix_q(i)) || !wait_ld(fix_o(i))) break;
                             tc_fence_after();
-                            mma128<false, true>(tb + fix_t(i), lk(fix_q(i)), lm(kSD), 0u);  // F = Q D_prefix
+                            mma128<false, true, kF, kFS>(tb + fix_t(i), lk(fix_q(i)), lm(kSD), 0u);  // F = Q D_prefix
                             umma_commit(&ms->bar[bEvF + i]);
                             if (j >= 1) {  // tile j-1 done: its buffer takes tile j+2
                                 const int g = (j - 1) % 3;
@@ -600,6 +604,11 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
             const uint32_t lane_base = (uint32_t)(32 * qd) << 16;
             // this thread's 32-column block of L . A and L . T lies above the diagonal (zero), on it, or below
             const bool blk_zero = cq > qd;
+            // Head size 64 (kNarrow): the products write feature columns 0..63 only, so the threads of
+            // column blocks 2, 3 (fcol false) hold zeros in the S carry and the e carry, skip their share
+            // of X, R, D_p, O and F, and never read the TMEM columns no product wrote.  Rows 64..127 of
+            // D (from the unwritten columns of X_hi / X_lo) are never read by a product over the head size.
+            const bool fcol = !kNarrow || cq < 2;
             const float *ring_prev = p.ring + ((size_t)head * 2 + ((sigma + 1) & 1)) * kRingFloats;
             float *ring_cur = p.ring + ((size_t)head * 2 + (sigma & 1)) * kRingFloats;
             const unsigned *flagS = p.flags, *flagD = p.flags + 2 * p.BH;
@@ -626,14 +635,19 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 float sp[32];
 #pragma unroll
                 for (int c = 0; c < 8; ++c) {
-                    const float4 v4 = ringS ? __ldcg(ringS + ring4(c, et))
-                                            : st_row ? __ldcg(st_row + c) : make_float4(0.f, 0.f, 0.f, 0.f);
+                    const float4 v4 = (ringS && fcol) ? __ldcg(ringS + ring4(c, et))
+                                      : st_row ? __ldcg(st_row + c) : make_float4(0.f, 0.f, 0.f, 0.f);
                     sp[4 * c] = v4.x; sp[4 * c + 1] = v4.y; sp[4 * c + 2] = v4.z; sp[4 * c + 3] = v4.w;
                 }
                 if (s_agg) {
                     // inclusive S prefix of this segment -> ring, published before this segment's set-up
                     float agg[32];
-                    ld32(tb + lane_base + kTS + c0, agg);
+                    if (fcol) {
+                        ld32(tb + lane_base + kTS + c0, agg);
+                    } else {
+#pragma unroll
+                        for (int j = 0; j < 32; ++j) agg[j] = 0.f;
+                    }
                     float4 *rc = reinterpret_cast<float4 *>(ring_cur);
 #pragma unroll
                     for (int j = 0; j < 32; j += 4)
@@ -661,7 +675,7 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 tmem_st32(tb + lane_base + kTS + c0, u);
                 // split S_p = cs I + R into R_hi (slot SX) and R_lo (slot W)
                 if (cq == qd) shift_diag32(sp, lane, cs);
-                store_split32(slot(kSX), slot(kW), r, c0, sp, precise);
+                if (fcol) store_split32(slot(kSX), slot(kW), r, c0, sp, precise);
                 // segment-local D carry: the initial state's D for the first segment
                 const float *d0 = (sigma == 0 && p.init_De) ? p.init_De + (size_t)head * (kD * kD + kD) : nullptr;
 #pragma unroll
@@ -720,14 +734,14 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 // while X = W K + Q S_p runs: D_p (bf16, final since the previous O) -> slot SD, read
                 // out of TMEM before this tile's D MMA (issued after the X hand-off), and q_t . e_p,
                 // the carried part of the denominator
-                {
+                if (fcol) {
                     float f[32];
                     ld32(tb + lane_base + kTD + c0, f);
 #pragma unroll
                     for (int jj = 0; jj < 32; jj += 8) store_row8(slot(kSD), r, c0 + jj, f + jj);
                 }
                 float den_part = 0.f;
-                if (p.normalized) {
+                if (p.normalized && fcol) {
 #pragma unroll
                     for (int jj = 0; jj < 32; jj += 8) {
                         float q8[8];
@@ -741,15 +755,20 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 bar_wait(ms, bEvX, tp, p);
                 tc_fence_after();
                 float x[32];
-                ld32(tb + lane_base + kTX + c0, x);
+                if (fcol) {
+                    ld32(tb + lane_base + kTX + c0, x);
 #pragma unroll
-                for (int jj = 0; jj < 32; jj += 8) {
-                    float q8[8];
-                    tile_row8(qt, r, c0 + jj, q8);
+                    for (int jj = 0; jj < 32; jj += 8) {
+                        float q8[8];
+                        tile_row8(qt, r, c0 + jj, q8);
 #pragma unroll
-                    for (int u = 0; u < 8; ++u) x[jj + u] += cs * q8[u];
+                        for (int u = 0; u < 8; ++u) x[jj + u] += cs * q8[u];
+                    }
+                    store_split32(slot(kSX), slot(kW), r, c0, x, true);
+                } else {
+#pragma unroll
+                    for (int jj = 0; jj < 32; ++jj) x[jj] = 0.f;
                 }
-                store_split32(slot(kSX), slot(kW), r, c0, x, true);
                 fence_async_smem();  // X_hi, X_lo and D_p (above) visible to the MMAs
                 epi_arrive(ms, bEpX);
 
@@ -792,7 +811,12 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 tc_fence_after();
                 if (j + 1 < nt) {
                     float f[32];
-                    ld32(tb + lane_base + kTS + c0, f);
+                    if (fcol) {
+                        ld32(tb + lane_base + kTS + c0, f);
+                    } else {
+#pragma unroll
+                        for (int jj = 0; jj < 32; ++jj) f[jj] = 0.f;
+                    }
                     const float *dt = ms->dtr[(j + 1) & 1];
                     cs = bf16_round((j == 0 ? tr_s : (dt[0] + dt[1]) + (dt[2] + dt[3])) / kD);
                     {
@@ -806,7 +830,7 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                         if (cq == qd && lane == 0) ms->dtr[j & 1][qd] = dg;
                     }
                     if (cq == qd) shift_diag32(f, lane, cs);
-                    store_split32(slot(kSX), slot(kW), r, c0, f, precise);
+                    if (fcol) store_split32(slot(kSX), slot(kW), r, c0, f, precise);
                     fence_async_smem();
                     epi_arrive(ms, bEpR);  // R of the next tile ready: Q R may start once O is read
                 }
@@ -817,15 +841,22 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 {
                     const bool final_out = (sigma == 0);
                     float f[32];
-                    ld32(tb + lane_base + kTX + c0, f);
+                    if (fcol) {
+                        ld32(tb + lane_base + kTX + c0, f);
+                    } else {
+#pragma unroll
+                        for (int jj = 0; jj < 32; ++jj) f[jj] = 0.f;
+                    }
                     epi_arrive(ms, bEpO);  // TMEM columns X are free for the next tile's X
                     if (final_out && p.normalized) {
                         const float inv = 1.f / (den + p.eps);
 #pragma unroll
                         for (int jj = 0; jj < 32; ++jj) f[jj] *= inv;
                     }
+                    if (fcol) {
 #pragma unroll
-                    for (int jj = 0; jj < 32; jj += 8) store_row8(slot(kSD), r, c0 + jj, f + jj);
+                        for (int jj = 0; jj < 32; jj += 8) store_row8(slot(kSD), r, c0 + jj, f + jj);
+                    }
                     if (!final_out && p.normalized && cq == 0 && tok0 + r < p.n)
                         p.den_loc[(size_t)head * p.n + tok0 + r] = den;
                 }
@@ -893,6 +924,7 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                         tc_fence_after();
                         if (p.normalized) {
                             // den_t = provisional denominator + q_t . e_prefix (four column quarters)
+                            // (q is zero beyond the head size)
                             float qe = 0.f;
 #pragma unroll
                             for (int jj = 0; jj < 32; jj += 8) {
@@ -910,15 +942,17 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                         const float inv = p.normalized
                             ? 1.f / ((((ms->den[r] + ms->part[0][r]) + ms->part[1][r]) + ms->part[2][r]) + p.eps)
                             : 1.f;
-                        float f[32];
-                        ld32(tb + lane_base + fix_t(i) + c0, f);
+                        if (fcol) {
+                            float f[32];
+                            ld32(tb + lane_base + fix_t(i) + c0, f);
 #pragma unroll
-                        for (int jj = 0; jj < 32; jj += 8) {
-                            float o8[8], w8[8];
-                            tile_row8(ot, r, c0 + jj, o8);
+                            for (int jj = 0; jj < 32; jj += 8) {
+                                float o8[8], w8[8];
+                                tile_row8(ot, r, c0 + jj, o8);
 #pragma unroll
-                            for (int u = 0; u < 8; ++u) w8[u] = (o8[u] + f[jj + u]) * inv;
-                            store_row8(ot, r, c0 + jj, w8);
+                                for (int u = 0; u < 8; ++u) w8[u] = (o8[u] + f[jj + u]) * inv;
+                                store_row8(ot, r, c0 + jj, w8);
+                            }
                         }
                         fence_async_smem();
                         epi_sync();  // also: every denominator read before the next tile's partials
@@ -1315,17 +1349,19 @@ cudaError_t fused2_forward(const Fwd2 &p, cudaStream_t stream) {
         kp.init_De = init;
     }
     const int grid = kp.n_items < sms ? kp.n_items : sms;
-    if (p.state_out) {
-        if ((e = cudaFuncSetAttribute(hla2_fused_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                      (int)kSmemBytes)))
-            return e;
-        hla2_fused_kernel<true><<<grid, kThreads, kSmemBytes, stream>>>(mq, mk, mv, mo, kp);
-    } else {
-        if ((e = cudaFuncSetAttribute(hla2_fused_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                      (int)kSmemBytes)))
-            return e;
-        hla2_fused_kernel<false><<<grid, kThreads, kSmemBytes, stream>>>(mq, mk, mv, mo, kp);
-    }
+    // instantiation: final state or not, head size 64 (d = dv = 64) or 128 (also 64 x 128 mixes, padded)
+    auto launch = [&](auto kern) -> cudaError_t {
+        cudaError_t err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
+        if (err) return err;
+        kern<<<grid, kThreads, kSmemBytes, stream>>>(mq, mk, mv, mo, kp);
+        return cudaGetLastError();
+    };
+    const bool narrow = p.d == 64 && p.dv == 64;
+    if (p.state_out)
+        e = narrow ? launch(hla2_fused_kernel<true, true>) : launch(hla2_fused_kernel<true, false>);
+    else
+        e = narrow ? launch(hla2_fused_kernel<false, true>) : launch(hla2_fused_kernel<false, false>);
+    if (e) return e;
     if ((e = cudaGetLastError()) || !p.state_out) return e;
     // final state: C and m partials, then the tuple (state_in, read by the kernel above, may alias)
     const int groups = state_groups(p.BH, kp.M);
