@@ -383,7 +383,7 @@ __global__ void __launch_bounds__(kT3c) c3_prefix2_kernel(float *ws, C3Layout L,
 // 5. outputs of a chunk from its carry-in
 // ---------------------------------------------------------------------------
 template <typename T>
-__global__ void __launch_bounds__(kT3c) c3_out_kernel(const T *__restrict__ q, const T *__restrict__ k,
+__global__ void __launch_bounds__(kT3c, 5) c3_out_kernel(const T *__restrict__ q, const T *__restrict__ k,
                                                       const T *__restrict__ v, T *__restrict__ out, float *ws,
                                                       C3Layout L, int masked, int normalized, float eps) {
     extern __shared__ float sm[];
@@ -537,6 +537,9 @@ cudaError_t launch_all(const Fwd2 &p, const C3Layout &L, float *ws, cudaStream_t
         return e;
     if ((e = cudaFuncSetAttribute(c3_out_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_out(L))))
         return e;
+    cudaFuncSetAttribute(c3_out_kernel<T>, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
+    cudaFuncSetAttribute(c3_local_kernel<T>, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
+    cudaFuncSetAttribute(c3_bracket_kernel<T>, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
     c3_local_kernel<T><<<grid, kT3c, smem_local(L), s>>>(q, k, v, ws, L, p.masked);
     const long long n1 = 2LL * p.d * p.d + (long long)p.d * p.dv + p.d;
     c3_prefix1_kernel<<<dim3((unsigned)((n1 + kT3c - 1) / kT3c), L.BH), kT3c, 0, s>>>(ws, L, p.state_in);
