@@ -251,6 +251,8 @@ def main():
     ap.add_argument("--workload", default="long_bf16_norm", choices=sorted(hla_inputs.WORKLOADS),
                     help="forward workload (default: the long-context one the metric is quoted on)")
     ap.add_argument("--n", type=int, default=0, help="override the sequence length (profiling runs)")
+    ap.add_argument("--only", default="", choices=["", "mid_bf16", "hla3_f32"],
+                    help="time only this secondary workload (the d = 64 forward or third order) and print its object")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
     if args.impl == "reference":
@@ -268,6 +270,13 @@ def main():
     dev = torch.device("cuda", local)
     torch.cuda.set_device(dev)
     hbm_peak, tc_peak, peak_kind = peaks()
+    if args.only:
+        stream = torch.cuda.current_stream()
+        res = bench_others(hla, dev, stream, hbm_peak, tc_peak, world, names=(args.only,),
+                           steps=args.steps if args.steps > 0 else 20, warmup=args.warmup)
+        if rank == 0:
+            print(json.dumps(res[0]))
+        return
 
     # ---------------- forward workload ----------------
     w = hla_inputs.WORKLOADS[args.workload]
@@ -413,12 +422,12 @@ def main():
         dist.destroy_process_group()
 
 
-def bench_others(hla, dev, stream, hbm_peak, tc_peak, world):
+def bench_others(hla, dev, stream, hbm_peak, tc_peak, world, names=("mid_bf16", "hla3_f32"), steps=20, warmup=3):
     """Forward of mid_bf16 (B8 H16 n2048 d64 bf16) and of hla3_f32 (masked third order, B4 H8 n4096 d32
-    fp32): 20 timed calls each after 3 warm-ups, CUDA events on the launching stream."""
+    fp32): `steps` timed calls each after `warmup` calls, CUDA events on the launching stream."""
     import torch
     res = []
-    for name in ("mid_bf16", "hla3_f32"):
+    for name in names:
         w = hla_inputs.WORKLOADS[name]
         q, k, v = hla_inputs.make_workload(w)
         tq, tk, tv = (hla_inputs.as_torch(x, w.dtype, dev) for x in (q, k, v))
@@ -432,12 +441,11 @@ def bench_others(hla, dev, stream, hbm_peak, tc_peak, world):
         def call():
             fwd(tq, tk, tv, out, masked=w.masked, normalized=w.normalized, eps=hla_inputs.EPS, chunk=w.chunk,
                 workspace=ws, stream=stream)
-        for _ in range(3):
+        for _ in range(warmup):
             call()
         torch.cuda.synchronize()
         barrier(world)
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        steps = 20
         e0.record(stream)
         for _ in range(steps):
             call()
@@ -466,7 +474,7 @@ def bench_others(hla, dev, stream, hbm_peak, tc_peak, world):
             cfg["launches"] = steps
         res.append(cfg)
         del tq, tk, tv, out, ws
-    return res[0], res[1]
+    return res
 
 
 def bench_decode(hla, dev, stream, steps, hbm_peak, world):
