@@ -96,7 +96,8 @@ enum Bar {
     bEpDF = 24,
     bEpO = 25,  // O read out of TMEM
     bEpOut = 26,  // provisional outputs of the segment written (segments > 0)
-    kNumBars = 27
+    bTear = 27,   // (count 1) all MMAs done, after a wait gave up
+    kNumBars = 28
 };
 constexpr int kFirstEpiBar = bEpW;
 
@@ -371,7 +372,7 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
         return;
     }
     if (tid == 0) {
-        for (int b = 0; b < kNumBars; ++b) mbar_init(&ms->bar[b], b >= kFirstEpiBar ? kEpiWarps : 1);
+        for (int b = 0; b < kNumBars; ++b) mbar_init(&ms->bar[b], (b >= kFirstEpiBar && b != bTear) ? kEpiWarps : 1);
         ms->abort_flag = 0;
         fence_mbar_init();
     }
@@ -390,6 +391,7 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
     // per-CTA event counters (identical sequences on both sides)
     uint32_t n_tiles = 0, n_items = 0, n_pre = 0, n_dfix = 0;
     uint32_t ld_par = 0;  // bit s: parity of the next load completion of slot s
+    uint32_t ld_pend = 0; // bit s: a load of slot s issued and not waited for yet
     uint32_t fx_par = 0;  // bit i: parity of the next fix-up hand-off of buffer i
     uint32_t n_r = 0;     // S-split hand-offs (one per tile that has a successor in its segment)
 
@@ -403,14 +405,16 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
     const uint64_t pol_first = l2_policy_evict_first(), pol_last = l2_policy_evict_last();
     const uint64_t pol_normal = l2_policy_evict_normal();
     auto load_tile = [&](int s, const CUtensorMap *map, int head, int tok0, uint64_t pol) {
+        ld_pend |= 1u << s;
         mbar_arrive_expect_tx(&ms->bar[bLd0 + s], kTileBytes);
         tma_load_3d_hint(slot(s), map, &ms->bar[bLd0 + s], 0, tok0, head, pol);
         tma_load_3d_hint(slot(s) + kBlockBytes, map, &ms->bar[bLd0 + s], 64, tok0, head, pol);
     };
     auto wait_ld = [&](int s) {
-        const uint32_t par = (ld_par >> s) & 1u;
+        if (!bar_wait(ms, bLd0 + s, (ld_par >> s) & 1u, p)) return false;  // still pending
         ld_par ^= 1u << s;
-        return bar_wait(ms, bLd0 + s, par, p);
+        ld_pend &= ~(1u << s);
+        return true;
     };
 
     // Pre-pass of an item: S aggregate of its tiles (sum of K^T K) into TMEM columns S, from K tiles
@@ -976,6 +980,14 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
         if (!issuer && tid == 0) tma_store_wait_all();
     }
 
+    if (issuer && lane == 0 && ms->abort_flag) {
+        // a wait gave up: the copies and MMAs this CTA still has in flight finish (each wait bounded)
+        // before its shared memory and TMEM are released
+        for (int s = 0; s <= kSX; ++s)
+            if ((ld_pend >> s) & 1u) mbar_wait(&ms->bar[bLd0 + s], (ld_par >> s) & 1u, kBarWaitNs);
+        umma_commit(&ms->bar[bTear]);
+        mbar_wait(&ms->bar[bTear], 0, kBarWaitNs);
+    }
     tc_fence_before();
     __syncthreads();
     if (issuer) {
