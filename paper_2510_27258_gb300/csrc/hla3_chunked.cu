@@ -44,6 +44,7 @@ constexpr int kT3c = 256;
 struct C3Layout {
     int BH, n, d, dv, W, nc;
     int stage_bracket;  // the bracket kernel copies its d x d / d x dv operands to shared memory
+    int stage_out;      // the output kernel copies its chunk's prefix record to shared memory
     long long rec_loc, rec_pre, oSK, oSQ, oU, oP, oF, oR, om, oe, orr;  // local record offsets (floats)
     long long pSK, pSQ, pP, pm, pF, pe;                                  // prefix record offsets
     long long loc_base, pre_base, init_base, total;
@@ -81,6 +82,7 @@ C3Layout c3_layout(int BH, int n, int d, int dv, int chunk) {
     L.init_base = L.pre_base + (long long)BH * L.nc * L.rec_pre;
     L.total = L.init_base + (long long)BH * (ddv + d);
     L.stage_bracket = (3 * dd + 2 * ddv) * 4 <= 96 * 1024;
+    L.stage_out = L.rec_pre * 4 <= 32 * 1024;
     return L;
 }
 
@@ -350,12 +352,14 @@ __global__ void __launch_bounds__(kT3c) c3_bracket_kernel(const T *__restrict__ 
         bq[t] = s;
     }
     __syncthreads();
-    // F_c += S^K_p R + U P_p + K^T diag(bq) V (each thread adds to the same elements of F_c in all three)
-    float *Fc = rec + L.oF;
-    smm2<true>(Fc, dv, d, dv, d, [&](int r, int x) { return SKp[r * d + x]; }, [&](int x, int cc) { return R[x * dv + cc]; });
-    smm2<true>(Fc, dv, d, dv, d, [&](int r, int x) { return U[r * d + x]; }, [&](int x, int cc) { return Pp[x * dv + cc]; });
-    smm2<true>(Fc, dv, d, dv, W, [&](int r, int t) { return Ks[t * ld + r] * bq[t]; },
+    // F_c += S^K_p R + U P_p + K^T diag(bq) V, summed in shared memory (same output owners in all three)
+    float *acc = bq + W + (L.stage_bracket ? 3 * d * d + 2 * d * dv : 0);
+    smm2<false>(acc, dv, d, dv, d, [&](int r, int x) { return SKp[r * d + x]; }, [&](int x, int cc) { return R[x * dv + cc]; });
+    smm2<true>(acc, dv, d, dv, d, [&](int r, int x) { return U[r * d + x]; }, [&](int x, int cc) { return Pp[x * dv + cc]; });
+    smm2<true>(acc, dv, d, dv, W, [&](int r, int t) { return Ks[t * ld + r] * bq[t]; },
                [&](int t, int cc) { return Vs[t * lv + cc]; });
+    __syncthreads();
+    for (int i = threadIdx.x; i < d * dv; i += blockDim.x) rec[L.oF + i] += acc[i];
     for (int r = threadIdx.x; r < d; r += blockDim.x) {
         float a1 = 0.f, a2 = 0.f, a3 = 0.f;
         for (int x = 0; x < d; ++x) {
@@ -379,6 +383,14 @@ __global__ void __launch_bounds__(kT3c) c3_prefix2_kernel(float *ws, C3Layout L,
     scan_chunks(ws, L, hd, lo, po, run);
 }
 
+// floats of the output kernel's working matrices, rounded up to 4: where the staged prefix record starts
+__host__ __device__ inline size_t out_stage_offset(const C3Layout &L) {
+    const int lm = (L.d > L.dv ? L.d : L.dv) + 1;
+    const size_t f = (size_t)L.W * (2 * (L.d + 1) + (L.dv + 1)) + 2 * (size_t)L.W * (L.W + 1) + 2 * (size_t)L.W * lm +
+                     4 * L.W + (size_t)L.W * (L.dv + 1);
+    return (f + 3) / 4 * 4;
+}
+
 // ---------------------------------------------------------------------------
 // 5. outputs of a chunk from its carry-in
 // ---------------------------------------------------------------------------
@@ -394,8 +406,14 @@ __global__ void __launch_bounds__(kT3c, 5) c3_out_kernel(const T *__restrict__ q
     float *M1 = Cm + W * lw, *M2 = M1 + W * lm, *a = M2 + W * lm, *b = a + W, *x1 = b + W, *den = x1 + W;
     float *Yb = den + W;  // W x dv (row stride dv + 1): Y, then the numerator
     load_chunk(q, k, v, Qs, Ks, Vs, hd, t0, w, W, L.n, d, dv);
-    __syncthreads();
     const float *pr = L.pre(ws, hd, c);
+    if (L.stage_out) {  // the chunk's prefix record (read many times below) from L2 once, 16-byte aligned
+        float *st = sm + out_stage_offset(L);
+        for (long long i = threadIdx.x; i < L.rec_pre / 4; i += blockDim.x)
+            reinterpret_cast<float4 *>(st)[i] = __ldcg(reinterpret_cast<const float4 *>(pr) + i);
+        pr = st;
+    }
+    __syncthreads();
     const float *SKp = pr + L.pSK, *SQp = pr + L.pSQ, *Pp = pr + L.pP, *mp = pr + L.pm;
     const float *Fp = pr + L.pF, *ep = pr + L.pe;
     T *Oh = out + ((size_t)hd * L.n + t0) * dv;
@@ -516,12 +534,10 @@ size_t smem_local(const C3Layout &L) {
 }
 size_t smem_bracket(const C3Layout &L) {
     const size_t stage = L.stage_bracket ? 3 * (size_t)L.d * L.d + 2 * (size_t)L.d * L.dv : 0;
-    return sizeof(float) * ((size_t)L.W * (2 * (L.d + 1) + (L.dv + 1)) + L.W + stage);
+    return sizeof(float) * ((size_t)L.W * (2 * (L.d + 1) + (L.dv + 1)) + L.W + stage + (size_t)L.d * L.dv);
 }
 size_t smem_out(const C3Layout &L) {
-    const int lm = (L.d > L.dv ? L.d : L.dv) + 1;
-    return sizeof(float) * ((size_t)L.W * (2 * (L.d + 1) + (L.dv + 1)) + 2 * (size_t)L.W * (L.W + 1) +
-                            2 * (size_t)L.W * lm + 4 * L.W + (size_t)L.W * (L.dv + 1));
+    return sizeof(float) * (out_stage_offset(L) + (L.stage_out ? (size_t)L.rec_pre : 0));
 }
 
 template <typename T>
