@@ -125,6 +125,52 @@ __device__ __forceinline__ void smm2(float *dst, int ld, int rows, int cols, int
     }
 }
 
+// One of up to four independent products of the same shape computed side by side: the block's threads
+// are split into ngrp groups and group grp forms this product with 4 x 4 output blocks per thread (rows
+// r + i rows/4, columns c + j cols/4), eight operand loads per sixteen multiply-adds; other threads return
+// at once.  Sizes that are not multiples of 4: one output per thread of the group.
+template <bool kAcc, typename FA, typename FB>
+__device__ __forceinline__ void smm44(int grp, int ngrp, float *dst, int ld, int rows, int cols, int kdim, FA a, FB b) {
+    const int per = blockDim.x / ngrp, t = (int)threadIdx.x - grp * per;
+    if (t < 0 || t >= per) return;
+    if ((rows | cols) & 3) {  // one output per thread of the group
+        for (int i = t; i < rows * cols; i += per) {
+            const int r = i / cols, c = i % cols;
+            float s = 0.f;
+            for (int k = 0; k < kdim; ++k) s += a(r, k) * b(k, c);
+            dst[r * ld + c] = kAcc ? dst[r * ld + c] + s : s;
+        }
+        return;
+    }
+    const int qr = rows >> 2, qc = cols >> 2;
+    for (int i = t; i < qr * qc; i += per) {
+        const int r = i / qc, c = i % qc;
+        float acc[4][4];
+#pragma unroll
+        for (int x = 0; x < 4; ++x)
+#pragma unroll
+            for (int y = 0; y < 4; ++y) acc[x][y] = 0.f;
+        for (int k = 0; k < kdim; ++k) {
+            float av[4], bv[4];
+#pragma unroll
+            for (int x = 0; x < 4; ++x) av[x] = a(r + x * qr, k);
+#pragma unroll
+            for (int y = 0; y < 4; ++y) bv[y] = b(k, c + y * qc);
+#pragma unroll
+            for (int x = 0; x < 4; ++x)
+#pragma unroll
+                for (int y = 0; y < 4; ++y) acc[x][y] += av[x] * bv[y];
+        }
+#pragma unroll
+        for (int x = 0; x < 4; ++x)
+#pragma unroll
+            for (int y = 0; y < 4; ++y) {
+                float *o = dst + (r + x * qr) * ld + c + y * qc;
+                *o = kAcc ? *o + acc[x][y] : acc[x][y];
+            }
+    }
+}
+
 // Triangular products, two outputs per thread that share one operand and their summation range:
 // rows:  dst[t][c] (+)= sum_{k in [lo(t), hi(t))} a(t, k) b(k, c), columns c and c + cols/2
 // cols:  dst[t][c] (+)= sum_{k in [0, hi(c))} a(t, k) b(k, c), rows t and t + rows/2
@@ -200,17 +246,17 @@ __global__ void __launch_bounds__(kT3c) c3_local_kernel(const T *__restrict__ q,
     load_chunk(q, k, v, Qs, Ks, Vs, hd, t0, w, W, L.n, d, dv);
     __syncthreads();
     float *rec = L.loc(ws, hd, c);
-    // first-order sums
-    smm2<false>(rec + L.oSK, d, d, d, W, [&](int r, int t) { return Ks[t * ld + r]; }, [&](int t, int cc) { return Ks[t * ld + cc]; });
-    smm2<false>(rec + L.oSQ, d, d, d, W, [&](int r, int t) { return Qs[t * ld + r]; }, [&](int t, int cc) { return Qs[t * ld + cc]; });
-    smm2<false>(rec + L.oP, dv, d, dv, W, [&](int r, int t) { return Ks[t * ld + r]; }, [&](int t, int cc) { return Vs[t * lv + cc]; });
+    // first-order sums (and A below), side by side in four thread groups
+    smm44<false>(0, 4, rec + L.oSK, d, d, d, W, [&](int r, int t) { return Ks[t * ld + r]; }, [&](int t, int cc) { return Ks[t * ld + cc]; });
+    smm44<false>(1, 4, rec + L.oSQ, d, d, d, W, [&](int r, int t) { return Qs[t * ld + r]; }, [&](int t, int cc) { return Qs[t * ld + cc]; });
+    smm44<false>(2, 4, rec + L.oP, dv, d, dv, W, [&](int r, int t) { return Ks[t * ld + r]; }, [&](int t, int cc) { return Vs[t * lv + cc]; });
     for (int r = threadIdx.x; r < d; r += blockDim.x) {
         float s = 0.f;
         for (int t = 0; t < W; ++t) s += Ks[t * ld + r];
         rec[L.om + r] = s;
     }
     if (!masked) return;
-    smm2<false>(A, lw, W, W, d, [&](int t, int j) { return Qs[t * ld + j]; }, [&](int j, int s) { return Ks[s * ld + j]; });
+    smm44<false>(3, 4, A, lw, W, W, d, [&](int t, int j) { return Qs[t * ld + j]; }, [&](int j, int s) { return Ks[s * ld + j]; });
     __syncthreads();
     for (int t = threadIdx.x; t < W; t += blockDim.x) {
         a[t] = A[t * lw + t];
@@ -237,11 +283,11 @@ __global__ void __launch_bounds__(kT3c) c3_local_kernel(const T *__restrict__ q,
     smm_rows<true>(Z, lv, W, dv, [&](int t, int s) { return A[s * lw + t] * a[s]; }, [&](int s, int cc) { return Vs[s * lv + cc]; },
                    [](int t) { return t + 1; }, [&](int) { return W; });
     __syncthreads();
-    smm2<false>(rec + L.oF, dv, d, dv, W, [&](int r, int t) { return Ks[t * ld + r]; }, [&](int t, int cc) { return Z[t * lv + cc]; });
-    smm2<false>(rec + L.oR, dv, d, dv, W, [&](int r, int t) { return Qs[t * ld + r] * a[t]; },
-                [&](int t, int cc) { return Vs[t * lv + cc]; });
-    smm2<false>(rec + L.oU, d, d, d, W, [&](int r, int t) { return Ks[t * ld + r] * a[t]; },
-                [&](int t, int cc) { return Qs[t * ld + cc]; });
+    smm44<false>(0, 4, rec + L.oF, dv, d, dv, W, [&](int r, int t) { return Ks[t * ld + r]; }, [&](int t, int cc) { return Z[t * lv + cc]; });
+    smm44<false>(1, 4, rec + L.oR, dv, d, dv, W, [&](int r, int t) { return Qs[t * ld + r] * a[t]; },
+                 [&](int t, int cc) { return Vs[t * lv + cc]; });
+    smm44<false>(2, 4, rec + L.oU, d, d, d, W, [&](int r, int t) { return Ks[t * ld + r] * a[t]; },
+                 [&](int t, int cc) { return Qs[t * ld + cc]; });
     for (int r = threadIdx.x; r < d; r += blockDim.x) {
         float se = 0.f, sr = 0.f;
         for (int t = 0; t < W; ++t) {
