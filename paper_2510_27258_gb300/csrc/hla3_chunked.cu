@@ -441,7 +441,7 @@ __host__ __device__ inline size_t out_stage_offset(const C3Layout &L) {
 // 5. outputs of a chunk from its carry-in
 // ---------------------------------------------------------------------------
 template <typename T>
-__global__ void __launch_bounds__(kT3c, 5) c3_out_kernel(const T *__restrict__ q, const T *__restrict__ k,
+__global__ void __launch_bounds__(kT3c, 4) c3_out_kernel(const T *__restrict__ q, const T *__restrict__ k,
                                                       const T *__restrict__ v, T *__restrict__ out, float *ws,
                                                       C3Layout L, int masked, int normalized, float eps) {
     extern __shared__ float sm[];
@@ -464,10 +464,11 @@ __global__ void __launch_bounds__(kT3c, 5) c3_out_kernel(const T *__restrict__ q
     const float *Fp = pr + L.pF, *ep = pr + L.pe;
     T *Oh = out + ((size_t)hd * L.n + t0) * dv;
     if (masked) {
-        smm2<false>(A, lw, W, W, d, [&](int t, int j) { return Qs[t * ld + j]; }, [&](int j, int s) { return Ks[s * ld + j]; });
-        // M1 = K S^Q_p, M2 = Q S^K_p  (W x d)
-        smm2<false>(M1, lm, W, d, d, [&](int t, int j) { return Ks[t * ld + j]; }, [&](int j, int cc) { return SQp[j * d + cc]; });
-        smm2<false>(M2, lm, W, d, d, [&](int t, int j) { return Qs[t * ld + j]; }, [&](int j, int cc) { return SKp[j * d + cc]; });
+        // A = Q K^T, M1 = K S^Q_p, M2 = Q S^K_p (W x d), Y = Q P_p: side by side in four thread groups
+        smm44<false>(0, 4, A, lw, W, W, d, [&](int t, int j) { return Qs[t * ld + j]; }, [&](int j, int s) { return Ks[s * ld + j]; });
+        smm44<false>(1, 4, M1, lm, W, d, d, [&](int t, int j) { return Ks[t * ld + j]; }, [&](int j, int cc) { return SQp[j * d + cc]; });
+        smm44<false>(2, 4, M2, lm, W, d, d, [&](int t, int j) { return Qs[t * ld + j]; }, [&](int j, int cc) { return SKp[j * d + cc]; });
+        smm44<false>(3, 4, Yb, lv, W, dv, d, [&](int s, int j) { return Qs[s * ld + j]; }, [&](int j, int cc) { return Pp[j * dv + cc]; });
         __syncthreads();
         for (int s = threadIdx.x; s < W; s += blockDim.x) {
             a[s] = A[s * lw + s];
@@ -481,9 +482,8 @@ __global__ void __launch_bounds__(kT3c, 5) c3_out_kernel(const T *__restrict__ q
             b[s] = bs;
             x1[s] = qm + ys;  // (Q m_p + (L.A) 1)_s
         }
-        // C_ts = q_t^T S^K_p q_s + sum_{i<s} A_ti A_si for s <= t, 0 above the diagonal; Y = Q P_p + (L.A) V
+        // C_ts = q_t^T S^K_p q_s + sum_{i<s} A_ti A_si for s <= t, 0 above the diagonal; Y += (L.A) V
         smm2<false>(Cm, lw, W, W, d, [&](int t, int j) { return M2[t * lm + j]; }, [&](int j, int s) { return Qs[s * ld + j]; });
-        smm2<false>(Yb, lv, W, dv, d, [&](int s, int j) { return Qs[s * ld + j]; }, [&](int j, int cc) { return Pp[j * dv + cc]; });
         __syncthreads();  // the accumulating products below own other elements
         smm_cols<true>(Cm, lw, W, W, [&](int t, int x) { return A[t * lw + x]; }, [&](int x, int s) { return A[s * lw + x]; },
                        [](int s) { return s; });
