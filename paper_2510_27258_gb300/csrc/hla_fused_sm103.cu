@@ -32,15 +32,18 @@
 // (TMEM -> registers -> shared memory): warp w reads TMEM lanes 32 (w % 4) ..
 // +31 (one row each) and columns 32 (w / 4) .. +31.
 //
-// Head sizes d, dv of 64 run as 128 with zero features 64..127: the TMA box of
-// those columns lies wholly outside the tensor and is zero-filled, so S, x_t,
-// D and e have zero rows / columns there (the S shift cancels exactly: q_f = 0)
-// and the padded output columns, which are zero, are not stored.  The tile is
-// 128 tokens whatever the requested chunk (Theorem 2: the result does not
-// depend on the chunking up to rounding).
+// Head sizes: d = dv = 64 has its own instantiation whose products run over 64
+// features (the tiles and TMEM regions keep their 128-column layout).  A mix of
+// 64 and 128 runs as 128 with zero features 64..127: the TMA box of those
+// columns lies wholly outside the tensor and is zero-filled, so S, x_t, D and e
+// have zero rows / columns there (the S shift cancels exactly: q_f = 0) and the
+// padded output columns, which are zero, are not stored.  The tile is 128
+// tokens whatever the requested chunk (Theorem 2: the result does not depend on
+// the chunking up to rounding).
 //
 // Precision: tokens are bf16, every product accumulates in fp32 (TMEM).  The S
-// operand is split as S = c I + R (c = bf16(trace S / d)) with c q_t added in
+// operand is split as S = c I + R (c = bf16(trace / d), the trace of the S carry
+// at most one tile old) with c q_t added in
 // fp32, so x_t is accurate although |S| grows like t/d.  X enters T = Q X^T as
 // bf16 hi + lo (with X rounded once, q_t . x_t = (q_t . k_t)^2 at t = 0 would
 // lose |q||k| / |q.k| times the bf16 rounding when q and k are nearly
@@ -61,7 +64,7 @@ namespace {
 
 using namespace sm103;
 
-constexpr int kD = 128;           // d = dv handled by this kernel
+constexpr int kD = 128;           // layout width of tiles, carries and TMEM regions (head sizes 64, 128)
 constexpr int kTile = 128;        // tokens per tile (MMA M)
 constexpr int kEpiWarps = 16;     // 4 per TMEM lane quadrant
 constexpr int kEpiThreads = kEpiWarps * 32;

@@ -71,7 +71,8 @@ def test_fused_path_selected(hla):
 @pytest.mark.parametrize("seg", ["1", "default"])
 @pytest.mark.parametrize("normalized", [False, True])
 def test_fused_head_size_64(hla, monkeypatch, d, dv, B, H, n, chunk, seg, normalized):
-    """Head sizes of 64 run as 128 with zero features; the requested chunk changes nothing but rounding."""
+    """Head sizes of 64: d = dv = 64 has its own instantiation (products over 64 features), mixes run as
+    128 with zero features; the requested chunk changes nothing but rounding."""
     if seg != "default":
         monkeypatch.setenv("HLA_FUSED_SEGMENT_TILES", seg)
     q, k, v = hla_inputs.make_qkv(B, H, n, d, dv, seed=n + 31 * d + dv, dtype="bf16")
