@@ -503,14 +503,15 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                     tc_fence_after();
                     mma128<false, false, kF, kFS>(tb + kTX, lk(qs), lk(kSX), 0u);      // X = Q R_hi
                     if (precise) mma128<false, false, kF, kFS>(tb + kTX, lk(qs), lk(kW), 1u);  // += Q R_lo
+                    // S += K^T K while the W epilogue runs (the S carry was read by the previous split,
+                    // before Q R could start)
+                    if (kState || j + 1 < nt) mma128<true, true, kF>(tb + kTS, lm(kK), lm(kK), 1u);
                     if (j > 0 && !bar_wait(ms, bEpW, tp, p)) break;  // W (hi, lo) ready
                     tc_fence_after();
                     mma128_ts<true, kF>(tb + kTX, tb + kTA, lm(kK), 1u);          // += W_hi K (W in TMEM)
                     if (precise) mma128_ts<true, kF>(tb + kTX, tb + kTA + 16, lm(kK), 1u);  // += W_lo K
                     umma_commit(&ms->bar[bEvX]);
-                    mma128<true, true, kF>(tb + kTS, lm(kK), lm(kK), 1u);         // S += K^T K
-                    umma_commit(&ms->bar[bEvS]);
-                    if (!bar_wait(ms, bEvS, tp, p)) break;  // X and S MMAs done: slot K free
+                    if (!bar_wait(ms, bEvX, tp, p)) break;  // X and S MMAs done: slot K free
                     if (j + 1 < nt) load_tile(kK, &tm_k, head, (t0 + j + 1) * kTile, pol_first);
                     if (!bar_wait(ms, bEpX, tp, p)) break;  // X_hi, X_lo in SX, W; D_p read out of TMEM
                     tc_fence_after();
