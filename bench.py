@@ -43,7 +43,7 @@ TRAFFIC = {
                           "n": 16384, "bytes": 526.2e6,
                           "how": "ncu capture at n=8192 (227.7 MB read + 35.4 MB written during the launch; outputs "
                                  "still dirty in L2 at its end are written later) scaled x2 to n=16384"},
-    "step2_kernel": {"src": ["hla_step.cu"], "sha256": "6b7c09075c2fc3a7", "workload": "decode_bf16", "n": 0,
+    "step2_kernel": {"src": ["hla_step.cu"], "sha256": "f6d2313a27dc36ee", "workload": "decode_bf16", "n": 0,
                      "bytes": 750.9e6, "how": "ncu capture of one step (406.4 MB read + 344.5 MB written)"},
 }
 

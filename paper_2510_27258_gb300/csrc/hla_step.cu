@@ -1,5 +1,5 @@
 // Streaming decode step of second-order HLA (online updates after Theorem 1,
-// outputs of Theorem 1 / Eq. hla-row), one block per head.
+// outputs of Theorem 1 / Eq. hla-row), one block per SM working through heads.
 //
 // The step is a read-modify-write of the fp32 state tuple (S, C, m, G, h):
 //   masked:  G' = G + k (k^T C),  h' = h + k (k^T m)       (previous C, m)
@@ -12,16 +12,16 @@
 // G' = G + k (k^T C) at once.  The unmasked form skips G and h (and leaves them
 // untouched).
 //
-// Memory access: every matrix is read and written once with 16-byte accesses,
-// consecutive threads on consecutive columns, all of a thread's loads of a
-// matrix issued before any of its arithmetic.
+// Memory access: every matrix is read once by 16-byte asynchronous copies into
+// shared memory, issued a pass or more ahead of its use, and written once with
+// 16-byte stores; consecutive threads on consecutive columns.
 #include "hla_internal.h"
 
 namespace hla {
 namespace {
 
-constexpr int kStepThreads = 256;
-constexpr int kMaxUnits = 16;  // float4 units per thread for a 128 x 128 matrix
+constexpr int kStepThreads = 512;
+constexpr int kMaxUnits = 128 * 128 / 4 / kStepThreads;  // float4 units per thread for a 128 x 128 matrix
 
 template <int W>
 __device__ __forceinline__ float group_sum(float x) {
@@ -51,159 +51,210 @@ __device__ __forceinline__ void block_sum3(float &a, float &b, float &c, float *
     for (int w = 0; w < kStepThreads / 32; ++w) { a += red[w * 3]; b += red[w * 3 + 1]; c += red[w * 3 + 2]; }
 }
 
+// 16-byte asynchronous copy global -> shared (L1 bypassed), and its group bookkeeping: each thread
+// waits for its own copies, a barrier then makes every thread's copies visible
+__device__ __forceinline__ void cp16(void *dst, const void *src) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"((uint32_t)__cvta_generic_to_shared(dst)), "l"(src)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
+
+__device__ __forceinline__ void store4(float4 *p, float4 v) { *p = v; }
+
+// One block per SM, heads hd = blockIdx.x, + gridDim.x, ...  The state of a head is staged in shared
+// memory in three buffers, one per pass (S; C with m; G with h), each refilled with the next head's
+// part as soon as its pass has read it, so that while one pass works the copies of the next two
+// parts (and of the next head's tokens) are in flight.  Updated values go to global memory straight
+// from registers.
 template <typename T>
-__global__ void __launch_bounds__(kStepThreads, 2)
+__global__ void __launch_bounds__(kStepThreads, 1)
 step2_kernel(const T *__restrict__ q, const T *__restrict__ k, const T *__restrict__ v, T *__restrict__ out,
-             float *__restrict__ state, int d, int dv, int masked, int normalized, float eps) {
-    __shared__ float qs[128], ks[128], vs[128], us[128], ms[128];
+             float *__restrict__ state, int BH, int d, int dv, int masked, int normalized, float eps) {
+    extern __shared__ float4 dyn[];
+    __shared__ float qs[128], ks[128], vs[128], us[128];
     __shared__ float red[3 * (kStepThreads / 32)];
     __shared__ float part[kStepThreads][12];
     __shared__ float kC[128], uC[128], qG[128];
 
-    const int hd = blockIdx.x, tid = threadIdx.x;
+    const int tid = threadIdx.x;
     const long long st_len = (long long)d * d + 2LL * d * dv + 2LL * d;
-    float *S = state + hd * st_len;
-    float *Cm = S + (long long)d * d;
-    float *m = Cm + (long long)d * dv;
-    float *G = m + d;
-    float *h = G + (long long)d * dv;
+    const int nS = (d * d) >> 2, nCm = (d * dv + d) >> 2;  // float4 units of S and of (C, m) / (G, h)
+    const int nt_q = d * (int)sizeof(T) / 16, nt_v = dv * (int)sizeof(T) / 16;  // 16-byte token chunks
+    float4 *bS = dyn, *bC = bS + nS, *bG = bC + nCm;
+    float4 *bT = bG + (masked ? nCm : 0);  // raw tokens q | k | v
+    const T *tq = reinterpret_cast<const T *>(bT), *tk = tq + d, *tv = tk + d;
 
-    float kq = 0.f, km = 0.f, qh = 0.f;
-    if (tid < d) {
-        const float qi = to_f32(q[(long long)hd * d + tid]), ki = to_f32(k[(long long)hd * d + tid]);
-        const float mi = m[tid];
-        qs[tid] = qi; ks[tid] = ki; ms[tid] = mi;
-        kq = ki * qi; km = ki * mi;
-        if (masked) qh = qi * h[tid];
-    }
-    if (tid < dv) vs[tid] = to_f32(v[(long long)hd * dv + tid]);
-    block_sum3(kq, km, qh, red);  // also a barrier: qs, ks, vs visible
+    auto load_S = [&](int hd) {  // S and the head's tokens
+        const float4 *src = reinterpret_cast<const float4 *>(state + hd * st_len);
+        for (int f = tid; f < nS; f += kStepThreads) cp16(bS + f, src + f);
+        if (tid < nt_q) {
+            cp16(bT + tid, reinterpret_cast<const float4 *>(q + (long long)hd * d) + tid);
+            cp16(bT + nt_q + tid, reinterpret_cast<const float4 *>(k + (long long)hd * d) + tid);
+        }
+        if (tid < nt_v) cp16(bT + 2 * nt_q + tid, reinterpret_cast<const float4 *>(v + (long long)hd * dv) + tid);
+        cp_commit();
+    };
+    auto load_part = [&](float4 *dst, int hd, long long off) {  // (C, m) or (G, h)
+        const float4 *src = reinterpret_cast<const float4 *>(state + hd * st_len + off);
+        for (int f = tid; f < nCm; f += kStepThreads) cp16(dst + f, src + f);
+        cp_commit();
+    };
+    const long long offC = (long long)d * d, offG = offC + (long long)d * dv + d;
 
-    // ---- pass over S: u = S q, S' = S + k k^T --------------------------------
-    {
-        const int w = d >> 2;  // float4 units per row of S
-        const int nunits = (d * d) >> 2;
-        const float4 *S4 = reinterpret_cast<const float4 *>(S);
-        float4 *S4w = reinterpret_cast<float4 *>(S);
-        float4 reg[kMaxUnits];
-#pragma unroll
-        for (int i = 0; i < kMaxUnits; ++i) {
-            const int f = tid + i * kStepThreads;
-            if (f < nunits) reg[i] = S4[f];
-        }
-#pragma unroll
-        for (int i = 0; i < kMaxUnits; ++i) {
-            const int f = tid + i * kStepThreads;
-            if (i * kStepThreads < nunits) {  // uniform per iteration: shuffles stay convergent
-                float part_u = 0.f;
-                if (f < nunits) {
-                    const int row = f / w, c4 = (f % w) * 4;
-                    const float4 s = reg[i];
-                    part_u = s.x * qs[c4] + s.y * qs[c4 + 1] + s.z * qs[c4 + 2] + s.w * qs[c4 + 3];
-                    const float kr = ks[row];
-                    S4w[f] = make_float4(s.x + kr * ks[c4], s.y + kr * ks[c4 + 1], s.z + kr * ks[c4 + 2],
-                                         s.w + kr * ks[c4 + 3]);
-                }
-                part_u = group_sum_rt(part_u, w);
-                if (f < nunits && (f % w) == 0) {
-                    const int row = f / w;
-                    us[row] = part_u + ks[row] * kq;  // u' = S q + k (k.q)
-                }
-            }
-        }
-    }
-    __syncthreads();
+    int hd = blockIdx.x;
+    if (hd >= BH) return;
+    load_S(hd);
+    load_part(bC, hd, offC);
+    if (masked) load_part(bG, hd, offG);
+    for (; hd < BH; hd += gridDim.x) {
+        const int nx = hd + gridDim.x;  // this block's next head (none: empty copy groups)
+        float *S = state + hd * st_len;
+        float *Cm = S + offC;
+        float *m = Cm + (long long)d * dv;
+        float *G = S + offG;
+        float *h = G + (long long)d * dv;
 
-    // u'.q and u'.(m + q)
-    float uq = 0.f, um = 0.f, dummy = 0.f;
-    if (tid < d) { uq = us[tid] * qs[tid]; um = us[tid] * (ms[tid] + qs[tid]); }
-    block_sum3(uq, um, dummy, red);
-
-    // ---- pass over C: column sums k^T C, u'^T C; C' = C + q v^T --------------
-    const int wv = dv >> 2;
-    const int nunits = (d * dv) >> 2;
-    const int c4 = (tid % wv) * 4;  // fixed column group of this thread
-    {
-        float4 acc_kC = make_float4(0.f, 0.f, 0.f, 0.f), acc_uC = acc_kC;
-        const float4 *C4 = reinterpret_cast<const float4 *>(Cm);
-        float4 *C4w = reinterpret_cast<float4 *>(Cm);
-        float4 creg[kMaxUnits];
-#pragma unroll
-        for (int i = 0; i < kMaxUnits; ++i) {
-            const int f = tid + i * kStepThreads;
-            if (f < nunits) creg[i] = C4[f];
-        }
-        const float v0 = vs[c4], v1 = vs[c4 + 1], v2 = vs[c4 + 2], v3 = vs[c4 + 3];
-#pragma unroll
-        for (int i = 0; i < kMaxUnits; ++i) {
-            const int f = tid + i * kStepThreads;
-            if (f < nunits) {
-                const int row = f / wv;
-                const float4 c = creg[i];
-                const float kr = ks[row], ur = us[row], qr = qs[row];
-                acc_kC.x += kr * c.x; acc_kC.y += kr * c.y; acc_kC.z += kr * c.z; acc_kC.w += kr * c.w;
-                acc_uC.x += ur * c.x; acc_uC.y += ur * c.y; acc_uC.z += ur * c.z; acc_uC.w += ur * c.w;
-                C4w[f] = make_float4(c.x + qr * v0, c.y + qr * v1, c.z + qr * v2, c.w + qr * v3);
-            }
-        }
-        part[tid][0] = acc_kC.x; part[tid][1] = acc_kC.y; part[tid][2] = acc_kC.z; part[tid][3] = acc_kC.w;
-        part[tid][4] = acc_uC.x; part[tid][5] = acc_uC.y; part[tid][6] = acc_uC.z; part[tid][7] = acc_uC.w;
-    }
-    __syncthreads();
-    if (tid < dv) {
-        const int grp = tid >> 2, comp = tid & 3;
-        float a = 0.f, b = 0.f;
-        for (int g = grp; g < kStepThreads; g += wv) { a += part[g][comp]; b += part[g][4 + comp]; }
-        kC[tid] = a; uC[tid] = b;
-    }
-    __syncthreads();
-
-    // ---- pass over G: column sums q^T G (old G); G' = G + k (k^T C) -----------
-    if (masked) {
-        float4 acc_qG = make_float4(0.f, 0.f, 0.f, 0.f);
-        const float4 *G4 = reinterpret_cast<const float4 *>(G);
-        float4 *G4w = reinterpret_cast<float4 *>(G);
-        float4 greg[kMaxUnits];
-#pragma unroll
-        for (int i = 0; i < kMaxUnits; ++i) {
-            const int f = tid + i * kStepThreads;
-            if (f < nunits) greg[i] = G4[f];
-        }
-        const float a0 = kC[c4], a1 = kC[c4 + 1], a2 = kC[c4 + 2], a3 = kC[c4 + 3];
-#pragma unroll
-        for (int i = 0; i < kMaxUnits; ++i) {
-            const int f = tid + i * kStepThreads;
-            if (f < nunits) {
-                const int row = f / wv;
-                const float kr = ks[row], qr = qs[row];
-                const float4 g = greg[i];
-                acc_qG.x += qr * g.x; acc_qG.y += qr * g.y; acc_qG.z += qr * g.z; acc_qG.w += qr * g.w;
-                G4w[f] = make_float4(g.x + kr * a0, g.y + kr * a1, g.z + kr * a2, g.w + kr * a3);
-            }
-        }
-        part[tid][8] = acc_qG.x; part[tid][9] = acc_qG.y; part[tid][10] = acc_qG.z; part[tid][11] = acc_qG.w;
-        if (tid < d) h[tid] += ks[tid] * km;
+        // ---- tokens, k.q ----
+        if (masked) cp_wait<2>(); else cp_wait<1>();  // S and tokens of this head
         __syncthreads();
+        float kq = 0.f, z0 = 0.f, z1 = 0.f;
+        if (tid < d) {
+            const float qi = to_f32(tq[tid]), ki = to_f32(tk[tid]);
+            qs[tid] = qi; ks[tid] = ki;
+            kq = ki * qi;
+        }
+        if (tid < dv) vs[tid] = to_f32(tv[tid]);
+        block_sum3(kq, z0, z1, red);  // also a barrier: qs, ks, vs visible
+
+        // ---- pass over S: u = S q, S' = S + k k^T ----
+        {
+            const int w = d >> 2;  // float4 units per row of S
+            float4 *Sg = reinterpret_cast<float4 *>(S);
+#pragma unroll
+            for (int i = 0; i < kMaxUnits; ++i) {
+                const int f = tid + i * kStepThreads;
+                if (i * kStepThreads < nS) {  // uniform per iteration: shuffles stay convergent
+                    float part_u = 0.f;
+                    if (f < nS) {
+                        const int row = f / w, c4 = (f % w) * 4;
+                        const float4 sv = bS[f];
+                        part_u = sv.x * qs[c4] + sv.y * qs[c4 + 1] + sv.z * qs[c4 + 2] + sv.w * qs[c4 + 3];
+                        const float kr = ks[row];
+                        store4(Sg + f, make_float4(sv.x + kr * ks[c4], sv.y + kr * ks[c4 + 1],
+                                                      sv.z + kr * ks[c4 + 2], sv.w + kr * ks[c4 + 3]));
+                    }
+                    part_u = group_sum_rt(part_u, w);
+                    if (f < nS && (f % w) == 0) {
+                        const int row = f / w;
+                        us[row] = part_u + ks[row] * kq;  // u' = S q + k (k.q)
+                    }
+                }
+            }
+        }
+        __syncthreads();  // S buffer read, u' complete
+        if (nx < BH) load_S(nx); else cp_commit();
+
+        // ---- pass over C: column sums k^T C, u'^T C; C' = C + q v^T; m' = m + q ----
+        if (masked) cp_wait<2>(); else cp_wait<1>();  // (C, m) of this head
+        __syncthreads();
+        const float *mv = reinterpret_cast<const float *>(bC + ((d * dv) >> 2));
+        float uq = 0.f, um = 0.f, km = 0.f;
+        if (tid < d) {
+            const float mi = mv[tid];
+            uq = us[tid] * qs[tid]; um = us[tid] * (mi + qs[tid]); km = ks[tid] * mi;
+            m[tid] = mi + qs[tid];
+        }
+        block_sum3(uq, um, km, red);
+        const int wv = dv >> 2;
+        const int nC = (d * dv) >> 2;
+        const int c4 = (tid % wv) * 4;  // fixed column group of this thread
+        {
+            float4 acc_kC = make_float4(0.f, 0.f, 0.f, 0.f), acc_uC = acc_kC;
+            float4 *Cg = reinterpret_cast<float4 *>(Cm);
+            const float v0 = vs[c4], v1 = vs[c4 + 1], v2 = vs[c4 + 2], v3 = vs[c4 + 3];
+#pragma unroll
+            for (int i = 0; i < kMaxUnits; ++i) {
+                const int f = tid + i * kStepThreads;
+                if (f < nC) {
+                    const int row = f / wv;
+                    const float4 c = bC[f];
+                    const float kr = ks[row], ur = us[row], qr = qs[row];
+                    acc_kC.x += kr * c.x; acc_kC.y += kr * c.y; acc_kC.z += kr * c.z; acc_kC.w += kr * c.w;
+                    acc_uC.x += ur * c.x; acc_uC.y += ur * c.y; acc_uC.z += ur * c.z; acc_uC.w += ur * c.w;
+                    store4(Cg + f, make_float4(c.x + qr * v0, c.y + qr * v1, c.z + qr * v2, c.w + qr * v3));
+                }
+            }
+            part[tid][0] = acc_kC.x; part[tid][1] = acc_kC.y; part[tid][2] = acc_kC.z; part[tid][3] = acc_kC.w;
+            part[tid][4] = acc_uC.x; part[tid][5] = acc_uC.y; part[tid][6] = acc_uC.z; part[tid][7] = acc_uC.w;
+        }
+        __syncthreads();  // (C, m) buffer read
+        if (nx < BH) load_part(bC, nx, offC); else cp_commit();
         if (tid < dv) {
             const int grp = tid >> 2, comp = tid & 3;
-            float c = 0.f;
-            for (int g = grp; g < kStepThreads; g += wv) c += part[g][8 + comp];
-            qG[tid] = c;
+            float a = 0.f, b = 0.f;
+            for (int g = grp; g < kStepThreads; g += wv) { a += part[g][comp]; b += part[g][4 + comp]; }
+            kC[tid] = a; uC[tid] = b;
         }
         __syncthreads();
-    }
 
-    // ---- m' = m + q; output ---------------------------------------------------
-    if (tid < d) m[tid] = ms[tid] + qs[tid];
-    if (tid < dv) {
-        float num = uC[tid] + uq * vs[tid];
-        float den = um;
+        // ---- pass over G: column sums q^T G (old G); G' = G + k (k^T C); h' = h + k (k.m) ----
+        float qh = 0.f;
         if (masked) {
-            num -= qG[tid] + kq * kC[tid];
-            den -= qh + kq * km;
+            cp_wait<2>();  // (G, h) of this head
+            __syncthreads();
+            const float *hv = reinterpret_cast<const float *>(bG + nC);
+            if (tid < d) {
+                const float hi = hv[tid];
+                qh = qs[tid] * hi;
+                h[tid] = hi + ks[tid] * km;
+            }
+            float4 acc_qG = make_float4(0.f, 0.f, 0.f, 0.f);
+            float4 *Gg = reinterpret_cast<float4 *>(G);
+            const float a0 = kC[c4], a1 = kC[c4 + 1], a2 = kC[c4 + 2], a3 = kC[c4 + 3];
+#pragma unroll
+            for (int i = 0; i < kMaxUnits; ++i) {
+                const int f = tid + i * kStepThreads;
+                if (f < nC) {
+                    const int row = f / wv;
+                    const float kr = ks[row], qr = qs[row];
+                    const float4 g = bG[f];
+                    acc_qG.x += qr * g.x; acc_qG.y += qr * g.y; acc_qG.z += qr * g.z; acc_qG.w += qr * g.w;
+                    store4(Gg + f, make_float4(g.x + kr * a0, g.y + kr * a1, g.z + kr * a2, g.w + kr * a3));
+                }
+            }
+            part[tid][8] = acc_qG.x; part[tid][9] = acc_qG.y; part[tid][10] = acc_qG.z; part[tid][11] = acc_qG.w;
+            block_sum3(qh, z0, z1, red);  // also a barrier: part and the (G, h) buffer read
+            if (nx < BH) load_part(bG, nx, offG); else cp_commit();
+            if (tid < dv) {
+                const int grp = tid >> 2, comp = tid & 3;
+                float c = 0.f;
+                for (int g = grp; g < kStepThreads; g += wv) c += part[g][8 + comp];
+                qG[tid] = c;
+            }
+            __syncthreads();
         }
-        from_f32(&out[(long long)hd * dv + tid], normalized ? num / (den + eps) : num);
+
+        // ---- output ----
+        if (tid < dv) {
+            float num = uC[tid] + uq * vs[tid];
+            float den = um;
+            if (masked) {
+                num -= qG[tid] + kq * kC[tid];
+                den -= qh + kq * km;
+            }
+            from_f32(&out[(long long)hd * dv + tid], normalized ? num / (den + eps) : num);
+        }
+        __syncthreads();  // qs, ks, vs, us, kC, uC, qG read before the next head rewrites them
     }
+    cp_wait<0>();  // (only empty groups remain)
+}
+
+// dynamic shared memory of step2_kernel: S, (C, m), (G, h) if masked, tokens
+size_t step2_smem(int d, int dv, int masked, size_t tsize) {
+    const size_t nS = (size_t)d * d / 4, nCm = ((size_t)d * dv + d) / 4;
+    return 16 * (nS + nCm * (masked ? 2 : 1)) + tsize * (2 * (size_t)d + dv);
 }
 
 }  // namespace
@@ -211,17 +262,28 @@ step2_kernel(const T *__restrict__ q, const T *__restrict__ k, const T *__restri
 cudaError_t step2_launch(const void *q, const void *k, const void *v, void *out, hla_dtype dt, int BH, int d, int dv,
                          int masked, int normalized, float eps, float *state, cudaStream_t stream) {
     if (BH == 0) return cudaSuccess;
-    if (dt == HLA_BF16)
-        step2_kernel<__nv_bfloat16><<<BH, kStepThreads, 0, stream>>>(
-            static_cast<const __nv_bfloat16 *>(q), static_cast<const __nv_bfloat16 *>(k),
-            static_cast<const __nv_bfloat16 *>(v), static_cast<__nv_bfloat16 *>(out), state, d, dv, masked,
-            normalized, eps);
-    else
-        step2_kernel<float><<<BH, kStepThreads, 0, stream>>>(static_cast<const float *>(q),
-                                                              static_cast<const float *>(k),
-                                                              static_cast<const float *>(v),
-                                                              static_cast<float *>(out), state, d, dv, masked,
-                                                              normalized, eps);
+    int dev = 0, sms = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return e;
+    const int grid = BH < sms ? BH : sms;
+    if (dt == HLA_BF16) {
+        auto kern = step2_kernel<__nv_bfloat16>;
+        const size_t sm = step2_smem(d, dv, masked, sizeof(__nv_bfloat16));
+        if ((e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm))) return e;
+        kern<<<grid, kStepThreads, sm, stream>>>(static_cast<const __nv_bfloat16 *>(q),
+                                                static_cast<const __nv_bfloat16 *>(k),
+                                                static_cast<const __nv_bfloat16 *>(v),
+                                                static_cast<__nv_bfloat16 *>(out), state, BH, d, dv, masked,
+                                                normalized, eps);
+    } else {
+        auto kern = step2_kernel<float>;
+        const size_t sm = step2_smem(d, dv, masked, sizeof(float));
+        if ((e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm))) return e;
+        kern<<<grid, kStepThreads, sm, stream>>>(static_cast<const float *>(q), static_cast<const float *>(k),
+                                                static_cast<const float *>(v), static_cast<float *>(out), state,
+                                                BH, d, dv, masked, normalized, eps);
+    }
     return cudaGetLastError();
 }
 

@@ -234,6 +234,21 @@ def test_decode_small(hla, d, dv, masked, normalized):
         assert np.abs(pg[name] - pr[name]).max() <= 2e-5 * max(scale, 1.0), name
 
 
+@pytest.mark.parametrize("d,dv,dtype", [(32, 64, "f32"), (64, 64, "bf16"), (128, 32, "f32")])
+@pytest.mark.parametrize("masked", [True, False])
+def test_decode_more_heads_than_sms(hla, d, dv, dtype, masked):
+    """320 heads (more than the SMs, so a block of the decode kernel works
+    through several heads with the next head's state staged while it computes):
+    every head's outputs and state against the oracle."""
+    B, H = 4, 80
+    got, ref, gst, rst = _decode_run(hla, B, H, d, dv, 20, 3, dtype, masked, False, seed=7 + d + dv)
+    assert rowerr(got, ref) < (1e-4 if dtype == "f32" else 2e-2)
+    pg, pr = oracle.split_state2(gst, d, dv), oracle.split_state2(rst, d, dv)
+    for name in ("S", "C", "m") + (("G", "h") if masked else ()):
+        scale = max(np.abs(pr[name]).max(), np.abs(pr["S"]).max() * np.abs(pr["C"]).max())
+        assert np.abs(pg[name] - pr[name]).max() <= 2e-5 * max(scale, 1.0), name
+
+
 def test_decode_workload_shape_sampled(hla):
     """The decode workload's shape (B64 H32 d128, bf16 tokens, fp32 state) with
     a shortened prefix; the oracle checks sampled heads."""
