@@ -39,16 +39,11 @@ __device__ __forceinline__ float group_sum_rt(float x, int w) {
     }
 }
 
-// block-wide sum of up to three values; every thread receives the result
-__device__ __forceinline__ void block_sum3(float &a, float &b, float &c, float *red) {
-    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
-    a = group_sum<32>(a); b = group_sum<32>(b); c = group_sum<32>(c);
-    __syncthreads();
-    if (lane == 0) { red[wid * 3 + 0] = a; red[wid * 3 + 1] = b; red[wid * 3 + 2] = c; }
-    __syncthreads();
-    a = b = c = 0.f;
-#pragma unroll
-    for (int w = 0; w < kStepThreads / 32; ++w) { a += red[w * 3]; b += red[w * 3 + 1]; c += red[w * 3 + 2]; }
+// sum_i a[i] b[i] over shared-memory vectors, computed by every warp on its own (no block barrier)
+__device__ __forceinline__ float warp_dot(const float *a, const float *b, int n) {
+    float s = 0.f;
+    for (int i = threadIdx.x & 31; i < n; i += 32) s += a[i] * b[i];
+    return group_sum<32>(s);
 }
 
 // 16-byte asynchronous copy global -> shared (L1 bypassed), and its group bookkeeping: each thread
@@ -74,7 +69,6 @@ step2_kernel(const T *__restrict__ q, const T *__restrict__ k, const T *__restri
              float *__restrict__ state, int BH, int d, int dv, int masked, int normalized, float eps) {
     extern __shared__ float4 dyn[];
     __shared__ float qs[128], ks[128], vs[128], us[128];
-    __shared__ float red[3 * (kStepThreads / 32)];
     __shared__ float part[kStepThreads][12];
     __shared__ float kC[128], uC[128], qG[128];
 
@@ -119,14 +113,13 @@ step2_kernel(const T *__restrict__ q, const T *__restrict__ k, const T *__restri
         // ---- tokens, k.q ----
         if (masked) cp_wait<2>(); else cp_wait<1>();  // S and tokens of this head
         __syncthreads();
-        float kq = 0.f, z0 = 0.f, z1 = 0.f;
         if (tid < d) {
-            const float qi = to_f32(tq[tid]), ki = to_f32(tk[tid]);
-            qs[tid] = qi; ks[tid] = ki;
-            kq = ki * qi;
+            qs[tid] = to_f32(tq[tid]);
+            ks[tid] = to_f32(tk[tid]);
         }
         if (tid < dv) vs[tid] = to_f32(tv[tid]);
-        block_sum3(kq, z0, z1, red);  // also a barrier: qs, ks, vs visible
+        __syncthreads();
+        const float kq = warp_dot(ks, qs, d);
 
         // ---- pass over S: u = S q, S' = S + k k^T ----
         {
@@ -160,13 +153,9 @@ step2_kernel(const T *__restrict__ q, const T *__restrict__ k, const T *__restri
         if (masked) cp_wait<2>(); else cp_wait<1>();  // (C, m) of this head
         __syncthreads();
         const float *mv = reinterpret_cast<const float *>(bC + ((d * dv) >> 2));
-        float uq = 0.f, um = 0.f, km = 0.f;
-        if (tid < d) {
-            const float mi = mv[tid];
-            uq = us[tid] * qs[tid]; um = us[tid] * (mi + qs[tid]); km = ks[tid] * mi;
-            m[tid] = mi + qs[tid];
-        }
-        block_sum3(uq, um, km, red);
+        if (tid < d) m[tid] = mv[tid] + qs[tid];
+        const float uq = warp_dot(us, qs, d), km = warp_dot(ks, mv, d);
+        const float um = warp_dot(us, mv, d) + uq;  // u'.(m + q)
         const int wv = dv >> 2;
         const int nC = (d * dv) >> 2;
         const int c4 = (tid % wv) * 4;  // fixed column group of this thread
@@ -205,11 +194,8 @@ step2_kernel(const T *__restrict__ q, const T *__restrict__ k, const T *__restri
             cp_wait<2>();  // (G, h) of this head
             __syncthreads();
             const float *hv = reinterpret_cast<const float *>(bG + nC);
-            if (tid < d) {
-                const float hi = hv[tid];
-                qh = qs[tid] * hi;
-                h[tid] = hi + ks[tid] * km;
-            }
+            if (tid < d) h[tid] = hv[tid] + ks[tid] * km;
+            qh = warp_dot(qs, hv, d);
             float4 acc_qG = make_float4(0.f, 0.f, 0.f, 0.f);
             float4 *Gg = reinterpret_cast<float4 *>(G);
             const float a0 = kC[c4], a1 = kC[c4 + 1], a2 = kC[c4 + 2], a3 = kC[c4 + 3];
@@ -225,7 +211,7 @@ step2_kernel(const T *__restrict__ q, const T *__restrict__ k, const T *__restri
                 }
             }
             part[tid][8] = acc_qG.x; part[tid][9] = acc_qG.y; part[tid][10] = acc_qG.z; part[tid][11] = acc_qG.w;
-            block_sum3(qh, z0, z1, red);  // also a barrier: part and the (G, h) buffer read
+            __syncthreads();  // part written, the (G, h) buffer read
             if (nx < BH) load_part(bG, nx, offG); else cp_commit();
             if (tid < dv) {
                 const int grp = tid >> 2, comp = tid & 3;
