@@ -39,6 +39,33 @@ __device__ __forceinline__ float group_sum_rt(float x, int w) {
     }
 }
 
+// Sums over the 32 lanes of a warp of eight values v[0..7] at once (9 shuffles instead of 40): on
+// return, lane l holds the sum of v[l >> 2] (each step keeps half of the values a lane still holds)
+__device__ __forceinline__ float warp_sum8(float (&v)[8]) {
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const bool up = (lane & 16) != 0;
+        const float send = up ? v[i] : v[i + 4], keep = up ? v[i + 4] : v[i];
+        v[i] = keep + __shfl_xor_sync(0xffffffffu, send, 16);
+    }
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+        const bool up = (lane & 8) != 0;
+        const float send = up ? v[i] : v[i + 2], keep = up ? v[i + 2] : v[i];
+        v[i] = keep + __shfl_xor_sync(0xffffffffu, send, 8);
+    }
+    {
+        const bool up = (lane & 4) != 0;
+        const float send = up ? v[0] : v[1], keep = up ? v[1] : v[0];
+        v[0] = keep + __shfl_xor_sync(0xffffffffu, send, 4);
+    }
+    float x = v[0];
+    x += __shfl_xor_sync(0xffffffffu, x, 2);
+    x += __shfl_xor_sync(0xffffffffu, x, 1);
+    return x;
+}
+
 // sum_i a[i] b[i] over shared-memory vectors, computed by every warp on its own (no block barrier)
 __device__ __forceinline__ float warp_dot(const float *a, const float *b, int n) {
     float s = 0.f;
@@ -122,7 +149,27 @@ step2_kernel(const T *__restrict__ q, const T *__restrict__ k, const T *__restri
         const float kq = warp_dot(ks, qs, d);
 
         // ---- pass over S: u = S q, S' = S + k k^T ----
-        {
+        if (d == 128 && kMaxUnits == 8) {
+            // a warp covers one row per unit (rows warp + 16 i): the eight row sums in one reduction
+            float4 *Sg = reinterpret_cast<float4 *>(S);
+            const int c4 = (tid & 31) * 4;
+            const float q0 = qs[c4], q1 = qs[c4 + 1], q2 = qs[c4 + 2], q3 = qs[c4 + 3];
+            const float k0 = ks[c4], k1 = ks[c4 + 1], k2 = ks[c4 + 2], k3 = ks[c4 + 3];
+            float pu[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                const int f = tid + i * kStepThreads;
+                const float4 sv = bS[f];
+                pu[i] = sv.x * q0 + sv.y * q1 + sv.z * q2 + sv.w * q3;
+                const float kr = ks[f >> 5];
+                store4(Sg + f, make_float4(sv.x + kr * k0, sv.y + kr * k1, sv.z + kr * k2, sv.w + kr * k3));
+            }
+            const float su = warp_sum8(pu);
+            if ((tid & 3) == 0) {
+                const int row = (tid >> 5) + 16 * ((tid & 31) >> 2);
+                us[row] = su + ks[row] * kq;  // u' = S q + k (k.q)
+            }
+        } else {
             const int w = d >> 2;  // float4 units per row of S
             float4 *Sg = reinterpret_cast<float4 *>(S);
 #pragma unroll
