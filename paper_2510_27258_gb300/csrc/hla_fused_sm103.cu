@@ -250,18 +250,47 @@ __device__ __forceinline__ void store_split32(uint8_t *th, uint8_t *tl, int r, i
 
 // zero the entries of columns c0..c0+31 above the diagonal of row r (c > r); for the
 // 32 x 32 diagonal block of the tile, r - c0 = lane
+// kSel: by selects (no branch that diverges the warp); else by a branch per element, which for the
+// 128-feature instantiation measured faster overall (it staggers the diagonal warps)
+template <bool kSel>
 __device__ __forceinline__ void mask_upper32(float (&f)[32], int r, int c0) {
 #pragma unroll
-    for (int jj = 0; jj < 32; ++jj)
-        if (c0 + jj > r) f[jj] = 0.f;
+    for (int jj = 0; jj < 32; ++jj) {
+        if constexpr (kSel) {
+            f[jj] = (c0 + jj > r) ? 0.f : f[jj];
+        } else {
+            if (c0 + jj > r) f[jj] = 0.f;
+        }
+    }
 }
 
 // subtract c from the entry of column r (the diagonal), which this thread holds when
 // its block is the diagonal block
+template <bool kSel>
 __device__ __forceinline__ void shift_diag32(float (&f)[32], int lane, float c) {
 #pragma unroll
-    for (int jj = 0; jj < 32; ++jj)
-        if (jj == lane) f[jj] -= c;
+    for (int jj = 0; jj < 32; ++jj) {
+        if constexpr (kSel) {
+            f[jj] -= (jj == lane) ? c : 0.f;
+        } else {
+            if (jj == lane) f[jj] -= c;
+        }
+    }
+}
+
+// f[lane] (the diagonal entry of row r when this thread's block is the diagonal block)
+template <bool kSel>
+__device__ __forceinline__ float pick_lane32(const float (&f)[32], int lane) {
+    float x = 0.f;
+#pragma unroll
+    for (int jj = 0; jj < 32; ++jj) {
+        if constexpr (kSel) {
+            x = (jj == lane) ? f[jj] : x;
+        } else {
+            if (jj == lane) x = f[jj];
+        }
+    }
+    return x;
 }
 
 // 32 values -> 16 packed bf16 pairs (the tensor-memory A-operand layout)
@@ -665,11 +694,7 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 pub_arrive(kBarPubS);  // S prefix in the ring
                 // trace -> shift (the diagonal element of row r lies in column block qd)
                 float s = 0.f;
-                if (cq == qd) {
-#pragma unroll
-                    for (int jj = 0; jj < 32; ++jj)
-                        if (jj == lane) s = sp[jj];
-                }
+                if (cq == qd) s = pick_lane32<kNarrow>(sp, lane);
                 s = warp_sum(s);
                 if (lane == 0) ms->red[warp] = s;
                 epi_sync();
@@ -682,7 +707,7 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 for (int j = 0; j < 32; ++j) u[j] = __float_as_uint(sp[j]);
                 tmem_st32(tb + lane_base + kTS + c0, u);
                 // split S_p = cs I + R into R_hi (slot SX) and R_lo (slot W)
-                if (cq == qd) shift_diag32(sp, lane, cs);
+                if (cq == qd) shift_diag32<kNarrow>(sp, lane, cs);
                 if (fcol) store_split32(slot(kSX), slot(kW), r, c0, sp, precise);
                 // segment-local D carry: the initial state's D for the first segment
                 const float *d0 = (sigma == 0 && p.init_De) ? p.init_De + (size_t)head * (kD * kD + kD) : nullptr;
@@ -726,7 +751,7 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                     } else {
                         float f[32];
                         ld32(tb + lane_base + kTA + c0, f);
-                        if (cq == qd) mask_upper32(f, r, c0);
+                        if (cq == qd) mask_upper32<kNarrow>(f, r, c0);
                         split_pack32(f, h, l);
                     }
                     tmem_st16(tb + lane_base + kTA + c0, h);
@@ -795,7 +820,7 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                     } else {
                         float f[32];
                         ld32(tb + lane_base + kTA + c0, f);
-                        if (cq == qd) mask_upper32(f, r, c0);
+                        if (cq == qd) mask_upper32<kNarrow>(f, r, c0);
 #pragma unroll
                         for (int jj = 0; jj < 32; ++jj) den_part += f[jj];
                         pack32(f, h);
@@ -829,15 +854,11 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                     cs = bf16_round((j == 0 ? tr_s : (dt[0] + dt[1]) + (dt[2] + dt[3])) / kD);
                     {
                         float dg = 0.f;
-                        if (cq == qd) {
-#pragma unroll
-                            for (int jj = 0; jj < 32; ++jj)
-                                if (jj == lane) dg = f[jj];
-                        }
+                        if (cq == qd) dg = pick_lane32<kNarrow>(f, lane);
                         dg = warp_sum(dg);
                         if (cq == qd && lane == 0) ms->dtr[j & 1][qd] = dg;
                     }
-                    if (cq == qd) shift_diag32(f, lane, cs);
+                    if (cq == qd) shift_diag32<kNarrow>(f, lane, cs);
                     if (fcol) store_split32(slot(kSX), slot(kW), r, c0, f, precise);
                     fence_async_smem();
                     epi_arrive(ms, bEpR);  // R of the next tile ready: Q R may start once O is read
