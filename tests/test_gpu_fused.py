@@ -103,6 +103,15 @@ def test_fused_initial_state(hla, monkeypatch, seg):
     check(hla, q, k, v, False, state_in=st0)
 
 
+@pytest.mark.parametrize("d", [64, 128])
+@pytest.mark.parametrize("normalized", [False, True])
+def test_fused_one_segment_per_head(hla, d, normalized):
+    """80 heads (at least half the SMs): the kernel gives each head one segment (no chains, no
+    fix-up), including the ragged last tile; every head against the oracle."""
+    q, k, v = hla_inputs.make_qkv(2, 40, 300, d, d, seed=77 + d, dtype="bf16")
+    check(hla, q, k, v, normalized)
+
+
 def test_fused_deterministic(hla, monkeypatch):
     monkeypatch.setenv("HLA_FUSED_SEGMENT_TILES", "2")
     q, k, v = hla_inputs.make_qkv(2, 3, 1500, 128, 128, seed=21, dtype="bf16")
