@@ -185,12 +185,22 @@ hla_status hla3_forward(const void *q, const void *k, const void *v, void *out, 
  * Sharing: all calls use the same array and it keeps the last call's contents
  * (each call clears what must start at zero).  Calls whose kernels overlap on
  * the GPU (different streams, or several host threads) race on it: order them
- * on one stream.  Device-side wait timeouts are not reported for this entry
- * point (hla_poll_error needs a workspace).
+ * on one stream.  A device-side wait that exceeds its budget sets the error
+ * word at the start of the array; hla_poll_error_noalloc reads it.
+ * An empty problem (B*H = 0 or n = 0) returns HLA_OK without launching.
  */
 hla_status hla2_forward_noalloc(const void *q, const void *k, const void *v, void *out, hla_dtype dt,
                                 int B, int H, int n, int d, int dv, int masked, int normalized, float eps,
                                 int chunk, const float *state_in, hla_stream_t stream);
+
+/*
+ * hla_poll_error_noalloc -- hla_poll_error for hla2_forward_noalloc (no
+ * counterpart in the paper): waits for `stream`, then reports and clears the
+ * device-side error word of the library's scratch array on the current device:
+ * HLA_OK, or HLA_ERR_TIMEOUT if a device-side wait of the last no-alloc call
+ * gave up.  Returns HLA_ERR_CUDA if synchronisation or the read fails.
+ */
+hla_status hla_poll_error_noalloc(hla_stream_t stream);
 
 /*
  * hla_poll_error -- wait for `stream`, then report the device-side error flag

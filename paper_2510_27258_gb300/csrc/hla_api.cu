@@ -20,6 +20,20 @@ hla_status fail(hla_status st, const char *fmt, ...) {
     return st;
 }
 
+void clear_last_error() { g_last_error[0] = 0; }
+
+hla_status poll_header(void *header, cudaStream_t s) {
+    WsHeader h{};
+    hla_status st = cuda_status(cudaMemcpyAsync(&h, header, sizeof(h), cudaMemcpyDeviceToHost, s), "reading flag");
+    if (st != HLA_OK) return st;
+    st = cuda_status(cudaStreamSynchronize(s), "synchronising");
+    if (st != HLA_OK) return st;
+    if (h.error == kDevOk) return HLA_OK;
+    st = cuda_status(cudaMemsetAsync(header, 0, sizeof(h), s), "clearing flag");
+    if (st != HLA_OK) return st;
+    return fail(HLA_ERR_TIMEOUT, "device-side wait gave up (where=%u detail=%u)", h.where, h.detail);
+}
+
 hla_status cuda_status(cudaError_t err, const char *what) {
     if (err == cudaSuccess) return HLA_OK;
     return fail(HLA_ERR_CUDA, "%s: %s (%s)", what, cudaGetErrorName(err), cudaGetErrorString(err));
@@ -190,16 +204,7 @@ hla_status hla3_forward(const void *q, const void *k, const void *v, void *out, 
 hla_status hla_poll_error(void *workspace, hla_stream_t stream) {
     g_last_error[0] = 0;
     if (!workspace) return fail(HLA_ERR_INVALID_ARGUMENT, "null workspace");
-    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-    WsHeader h{};
-    hla_status st = cuda_status(cudaMemcpyAsync(&h, workspace, sizeof(h), cudaMemcpyDeviceToHost, s), "reading flag");
-    if (st != HLA_OK) return st;
-    st = cuda_status(cudaStreamSynchronize(s), "synchronising");
-    if (st != HLA_OK) return st;
-    if (h.error == kDevOk) return HLA_OK;
-    st = cuda_status(cudaMemsetAsync(workspace, 0, sizeof(h), s), "clearing flag");
-    if (st != HLA_OK) return st;
-    return fail(HLA_ERR_TIMEOUT, "device-side wait gave up (where=%u detail=%u)", h.where, h.detail);
+    return poll_header(workspace, reinterpret_cast<cudaStream_t>(stream));
 }
 
 }  // extern "C"

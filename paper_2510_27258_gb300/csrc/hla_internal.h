@@ -28,6 +28,11 @@ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 // Records a host-side error message for hla_last_error() and returns `st`.
 hla_status fail(hla_status st, const char *fmt, ...);
+// Empties the message hla_last_error() returns (every entry point starts with it).
+void clear_last_error();
+// Reads the device-side error word of a workspace header (waiting for `stream`),
+// clears it, and maps it to HLA_OK / HLA_ERR_TIMEOUT (HLA_ERR_CUDA if a call fails).
+hla_status poll_header(void *header, cudaStream_t stream);
 // Maps a CUDA error to HLA_ERR_CUDA (recording the CUDA message), or HLA_OK.
 hla_status cuda_status(cudaError_t err, const char *what);
 

@@ -46,10 +46,12 @@ extern "C" hla_status hla2_forward_noalloc(const void *q, const void *k, const v
                                            int B, int H, int n, int d, int dv, int masked, int normalized,
                                            float eps, int chunk, const float *state_in, hla_stream_t stream) {
     // Same argument checks as hla2_forward; only the fused path is offered.
+    clear_last_error();
     int launches = 0;
     const int path = hla2_forward_path(B, H, n, d, dv, masked, normalized, chunk, dt, state_in != nullptr, 0,
                                        &launches);
     if (path < 0) return fail(HLA_ERR_UNSUPPORTED, "arguments not supported by hla2_forward");
+    if ((long long)B * H == 0 || n == 0) return HLA_OK;  // nothing to compute (no final state is written)
     if (path != 1)
         return fail(HLA_ERR_UNSUPPORTED,
                     "hla2_forward_noalloc serves the fused path only (bf16, d and dv in {64, 128}, masked, no "
@@ -74,4 +76,12 @@ extern "C" hla_status hla2_forward_noalloc(const void *q, const void *k, const v
     Fwd2 p{q, k, v, out, dt, B * H, n, d, dv, masked, normalized, eps, chunk, state_in, nullptr,
            static_cast<char *>(scratch), kNoAllocScratchBytes};
     return cuda_status(fused2_forward(p, s), "fused forward (no-alloc)");
+}
+
+extern "C" hla_status hla_poll_error_noalloc(hla_stream_t stream) {
+    clear_last_error();
+    void *scratch = nullptr;
+    hla_status st = scratch_address(&scratch);
+    if (st != HLA_OK) return st;
+    return poll_header(scratch, reinterpret_cast<cudaStream_t>(stream));
 }

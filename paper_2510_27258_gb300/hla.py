@@ -22,7 +22,7 @@ HLA_F32, HLA_BF16 = 0, 1
 # every symbol include/hla.h declares
 EXPORTS = ("hla_status_string", "hla_last_error", "hla2_state_floats", "hla2_workspace_bytes", "hla2_forward",
            "hla2_forward_path", "hla2_step", "hla3_state_floats", "hla3_workspace_bytes", "hla3_forward",
-           "hla2_forward_noalloc", "hla_poll_error")
+           "hla2_forward_noalloc", "hla_poll_error_noalloc", "hla_poll_error")
 
 _lib = None
 
@@ -64,6 +64,8 @@ def lib():
         L.hla2_step.restype = i
         L.hla_poll_error.argtypes = [vp, vp]
         L.hla_poll_error.restype = i
+        L.hla_poll_error_noalloc.argtypes = [vp]
+        L.hla_poll_error_noalloc.restype = i
         _lib = L
     return _lib
 
@@ -195,6 +197,12 @@ def hla2_step(q, k, v, state, out=None, *, masked=True, normalized=False, eps=1e
                            int(normalized), float(eps), _ptr(state), _stream(stream))
     _check(code, "hla2_step")
     return out
+
+
+def hla_poll_error_noalloc(stream=None) -> int:
+    """Synchronise and read the device-side error flag of the library's own scratch array, used by
+    hla2_forward_noalloc (include/hla.h: hla_poll_error_noalloc)."""
+    return int(lib().hla_poll_error_noalloc(_stream(stream)))
 
 
 def hla_poll_error(workspace, stream=None) -> int:

@@ -8,11 +8,16 @@ the denominator passes near zero: den_t is a sum of O(t) terms whose local
 magnitude s_t (RMS of den over neighbouring positions) is far larger than den_t
 itself on a few rows (on the long workload |den_t| / s_t reaches 1e-6).  Any
 fp32 evaluation of such a sum carries an absolute error of order
-u * sqrt(t) * s_t (u = 2^-24, random-walk bound for t rounded additions).  A
-sum evaluated in stages (tensor-core partial sums of split operands, cross-warp
-partial sums, a carried prefix) takes a few roundings per term, so the bound
-used is K u sqrt(t+1) s_t with K = 8.  The bar is applied as follows, all three
-checks required:
+u * sqrt(t) * s_t (u = 2^-24, random-walk bound for t rounded additions); the
+bound used is K u sqrt(t+1) s_t.  K is the envelope of an fp32 model of the
+fused kernel's own stages (tests/den_model.py: bf16 hi + lo operands, tensor-core
+partial sums, per-quarter partials, the carried e prefix): over the rows whose
+modelled denominator misses bar |den_t| on the cases the GPU tests run, the
+largest err_t / (u sqrt(t+1) s_t) is 6.1 (80 heads x 300 tokens, d = 128) and
+0.1 (sampled heads of the long workload); K = 8 covers it with a margin for the
+tensor cores' accumulation order (tests/test_den_model.py checks
+envelope <= K <= 2 envelope).  The bar is applied as follows, all three checks
+required:
   1. the numerator (the unnormalised output) meets the bar on every row;
   2. the normalised output meets the bar on every row whose denominator fp32
      can resolve to that bar:  |den_t + eps| >= K u sqrt(t+1) s_t / bar;
@@ -25,7 +30,7 @@ from __future__ import annotations
 import numpy as np
 
 U32 = 2.0 ** -24
-K_FP32 = 8.0  # roundings per term of a staged fp32 sum (see above)
+K_FP32 = 8.0  # envelope of the fp32 model of the kernel's denominator stages (see above)
 TOL = {"f32": 1e-4, "bf16": 2e-2}
 
 
@@ -69,8 +74,14 @@ def check_normalized(o_gpu, num_gpu, num_ref, den_ref, eps, tol):
     assert e_out < tol, "normalised output error %.3g >= %.3g on well-conditioned rows" % (e_out, tol)
     den_gpu = (num_gpu * o_gpu).sum(-1) / np.maximum((o_gpu * o_gpu).sum(-1), 1e-300) - eps
     allowed = np.maximum(tol * np.abs(den_ref + eps), bound)
-    excess = np.abs(den_gpu - den_ref) / allowed
+    err_den = np.abs(den_gpu - den_ref)
+    excess = err_den / allowed
     assert excess.max() <= 1.0, "implied denominator off by %.3g x its bound at row %s" % (
         excess.max(), np.unravel_index(int(excess.argmax()), excess.shape))
+    # the literal bar over every row, and the K the rows beyond it needed
+    lit = rowerr_rows(o_gpu, o_ref)
+    beyond = err_den > tol * np.abs(den_ref + eps)
+    k_used = float((err_den[beyond] / (bound[beyond] / K_FP32)).max()) if beyond.any() else 0.0
     return {"num": e_num, "out_well": e_out, "ill_rows": int((~well).sum()), "rows": int(well.size),
-            "den_excess": float(excess.max())}
+            "den_excess": float(excess.max()), "out_literal_max": float(lit.max()),
+            "rows_beyond_bar": int((lit >= tol).sum()), "k_used": k_used}

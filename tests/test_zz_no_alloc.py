@@ -1,9 +1,11 @@
 """hla2_forward_noalloc, the entry point for callers that cannot allocate device
 memory (they cannot call cudaMalloc or hand over a workspace, e.g. code running
-under someone else's memory pool or budget): it must give the same outputs as
-hla2_forward with a caller workspace, on consecutive calls that reuse the
-library's own scratch array.  Kept in the last test file so that a run stopping
-at its first failure has already run everything else."""
+under someone else's memory pool or budget).  Its outputs must match the fp64
+oracle within the bf16 bar and be bit-identical to hla2_forward with a caller
+workspace (the same kernel on the same inputs), on consecutive calls that reuse
+the library's own scratch array, also when a call of another shape has left
+its contents there.  Kept in the last test file so that a run stopping at its
+first failure has already run everything else."""
 import ctypes
 
 import numpy as np
@@ -11,7 +13,8 @@ import pytest
 import torch
 
 import hla_inputs
-from parity import TOL, rowerr
+import oracle
+from parity import TOL, check_normalized, rowerr
 
 pytestmark = pytest.mark.gpu
 DEV = "cuda:0"
@@ -25,30 +28,89 @@ def hla():
     return binding
 
 
-def _noalloc(hla, q, k, v, out, normalized):
+def _noalloc(hla, q, k, v, out, normalized, state_in=None):
+    """The C entry point through ctypes (no Python wrapper)."""
     B, H, n, d = q.shape
     L = hla.lib()
     stream = ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
     return L.hla2_forward_noalloc(ctypes.c_void_p(q.data_ptr()), ctypes.c_void_p(k.data_ptr()),
                                   ctypes.c_void_p(v.data_ptr()), ctypes.c_void_p(out.data_ptr()), hla.HLA_BF16,
                                   B, H, n, d, v.shape[-1], 1, int(normalized), ctypes.c_float(hla_inputs.EPS), 128,
-                                  None, stream)
+                                  None if state_in is None else ctypes.c_void_p(state_in.data_ptr()), stream)
 
 
+def _foreign_call(hla):
+    """A call of another shape, so that the scratch holds its counters, ring and denominators."""
+    q, k, v = hla_inputs.make_qkv(1, 3, 900, 64, 64, seed=5, dtype="bf16")
+    tq, tk, tv = (hla_inputs.as_torch(x, "bf16", DEV) for x in (q, k, v))
+    out = torch.empty((1, 3, 900, 64), dtype=torch.bfloat16, device=DEV)
+    assert _noalloc(hla, tq, tk, tv, out, True) == hla.HLA_OK, hla.lib().hla_last_error()
+
+
+def _check_oracle(q, k, v, got, normalized, state_in=None):
+    B, H, n, d = q.shape
+    dv = v.shape[-1]
+    qf, kf, vf = q.reshape(B * H, n, d), k.reshape(B * H, n, d), v.reshape(B * H, n, dv)
+    sin = None if state_in is None else state_in.reshape(B * H, -1).astype(np.float64)
+    num, den = oracle.hla2_serial(qf, kf, vf, masked=True, normalized=False, eps=hla_inputs.EPS, state_in=sin,
+                                  return_den=True, nthreads=4)
+    got = got.reshape(B * H, n, dv)
+    if not normalized:
+        assert rowerr(got, num) < TOL["bf16"]
+        return None
+    return num, den
+
+
+@pytest.mark.parametrize("d", [64, 128])
 @pytest.mark.parametrize("normalized", [False, True])
-def test_noalloc_matches_workspace_forward_on_two_calls(hla, normalized):
-    B, H, n, d = 1, 4, 1000, 128
-    q, k, v = hla_inputs.make_qkv(B, H, n, d, d, seed=77, dtype="bf16")
+def test_noalloc_matches_oracle_and_workspace_forward_on_two_calls(hla, d, normalized):
+    B, H, n = 1, 4, 1000
+    q, k, v = hla_inputs.make_qkv(B, H, n, d, d, seed=77 + d, dtype="bf16")
     tq, tk, tv = (hla_inputs.as_torch(x, "bf16", DEV) for x in (q, k, v))
     ref = hla.hla2_forward(tq, tk, tv, masked=True, normalized=normalized, eps=hla_inputs.EPS, chunk=128)
+    num_gpu = hla.hla2_forward(tq, tk, tv, masked=True, normalized=False, eps=hla_inputs.EPS, chunk=128)
     torch.cuda.synchronize()
-    ref = ref.float().cpu().numpy().reshape(B * H, n, d)
-    for call in range(2):  # the second call reuses the scratch left by the first
+    ref = ref.float().cpu().numpy()
+    num_gpu = num_gpu.float().cpu().numpy().reshape(B * H, n, d)
+    for call in range(2):  # the second call reuses the scratch left by a call of another shape
+        if call == 1:
+            _foreign_call(hla)
         out = torch.zeros((B, H, n, d), dtype=torch.bfloat16, device=DEV)
         assert _noalloc(hla, tq, tk, tv, out, normalized) == hla.HLA_OK, hla.lib().hla_last_error()
+        assert hla.hla_poll_error_noalloc() == hla.HLA_OK
+        got = out.float().cpu().numpy()
+        assert np.array_equal(got, ref), call
+        nd = _check_oracle(q, k, v, got, normalized)
+        if nd is not None:
+            check_normalized(got.reshape(B * H, n, d), num_gpu, nd[0], nd[1], hla_inputs.EPS, TOL["bf16"])
+
+
+def test_noalloc_python_wrapper_with_initial_state(hla):
+    """The Python wrapper with an initial state (d = dv = 128), twice in a row."""
+    B, H, n, d = 1, 2, 700, 128
+    pq, pk, pv = hla_inputs.make_qkv(B, H, 300, d, d, seed=31, dtype="bf16")
+    _, st0 = oracle.hla2_serial(pq.reshape(B * H, 300, d), pk.reshape(B * H, 300, d), pv.reshape(B * H, 300, d),
+                                masked=True, return_state=True)
+    st0 = st0.astype(np.float32)
+    q, k, v = hla_inputs.make_qkv(B, H, n, d, d, seed=32, dtype="bf16")
+    tq, tk, tv = (hla_inputs.as_torch(x, "bf16", DEV) for x in (q, k, v))
+    tst = torch.from_numpy(st0).to(DEV)
+    ref = hla.hla2_forward(tq, tk, tv, masked=True, normalized=False, eps=hla_inputs.EPS, chunk=128, state_in=tst)
+    torch.cuda.synchronize()
+    ref = ref.float().cpu().numpy()
+    for _ in range(2):
+        got = hla.hla2_forward_noalloc(tq, tk, tv, masked=True, normalized=False, eps=hla_inputs.EPS, chunk=128,
+                                       state_in=tst)
         torch.cuda.synchronize()
-        got = out.float().cpu().numpy().reshape(B * H, n, d)
-        assert rowerr(got, ref) < TOL["bf16"], (call, rowerr(got, ref))
+        got = got.float().cpu().numpy()
+        assert np.array_equal(got, ref)
+        _check_oracle(q, k, v, got, False, state_in=st0)
+
+
+def test_noalloc_empty_problem_is_ok(hla):
+    t = torch.zeros((1, 0, 256, 128), dtype=torch.bfloat16, device=DEV)
+    assert _noalloc(hla, t, t, t, t, False) == hla.HLA_OK
+    assert hla.lib().hla_last_error() == b""
 
 
 def test_noalloc_rejects_sizes_beyond_its_scratch(hla):
