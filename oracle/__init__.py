@@ -20,6 +20,16 @@ names the passage of the paper it follows:
   third-order factorisation of Sec. 7.1.
 * :func:`hla3_chunked`  -- Theorem 4 / Algorithm 4 with the segment maps
   applied by contraction.
+* :func:`hla2_state_to_sde` -- the masked tuple folded to (S, D = SC - G,
+  e = Sm - h), the quantities Theorem 1's outputs read.
+* :func:`ahla_serial`   -- the AHLA online updates (Theorem AHLA, Algorithm
+  AHLA-stream at gamma = 1).
+* :func:`ahla_combine`  -- Eq. AHLA-semidirect on (R, P, m, E, n).
+* :func:`ahla_chunked`  -- the AHLA scan route (exclusive Blelloch scans
+  under the AHLA product, then local inclusion; scan equivalence).
+* :func:`hla2_backward` -- gradients of second-order HLA by a reverse sweep
+  over the online updates, forward states checkpointed at tile boundaries
+  (Sec. "Chunk-parallel training via associative scans").
 
 Array conventions: q, k are ``[BH, n, d]``, v is ``[BH, n, dv]``; outputs are
 ``[BH, n, dv]``; the state tuple of one head is laid out as in
@@ -83,6 +93,16 @@ def _bind(lib):
     lib.hla3_chunked_f64.restype = i
     lib.hla3_state_len_f64.argtypes = [i, i]
     lib.hla3_state_len_f64.restype = ctypes.c_size_t
+    lib.hla2_state_to_sde_f64.argtypes = [_dp, _dp, i, i, i]
+    lib.hla2_state_to_sde_f64.restype = None
+    lib.ahla_serial_f64.argtypes = [_dp, _dp, _dp, _dp, _dp, i, i, i, i, i, d, _dp, _dp, i]
+    lib.ahla_serial_f64.restype = i
+    lib.ahla_chunked_f64.argtypes = [_dp, _dp, _dp, _dp, _dp, i, i, i, i, i, i, d, i]
+    lib.ahla_chunked_f64.restype = i
+    lib.ahla_combine_f64.argtypes = [_dp, _dp, _dp, i, i]
+    lib.ahla_combine_f64.restype = None
+    lib.hla2_backward_f64.argtypes = [_dp, _dp, _dp, _dp, _dp, _dp, _dp, i, i, i, i, i, i, d, i, i]
+    lib.hla2_backward_f64.restype = i
     return lib
 
 
@@ -214,3 +234,79 @@ def hla3_chunked(q, k, v, chunk, normalized=False, eps=1e-6, return_den=False, n
                                  float(eps), int(chunk), int(nthreads))
     assert rc == 0
     return (out, den) if return_den else out
+
+
+def hla2_sde_len(d: int, dv: int) -> int:
+    """Length of one head's (S, D, e) state: d*d + d*dv + d."""
+    return d * d + d * dv + d
+
+
+def hla2_state_to_sde(st, d: int, dv: int):
+    """(S, C, m, G, h) tuples [..., hla2_state_len] -> (S, D = S C - G, e = S m - h) [..., hla2_sde_len]."""
+    st = _f64(st)
+    lead = st.shape[:-1]
+    flat = np.ascontiguousarray(st.reshape(-1, hla2_state_len(d, dv)))
+    out = np.zeros((flat.shape[0], hla2_sde_len(d, dv)))
+    load().hla2_state_to_sde_f64(_ptr(flat), _ptr(out), flat.shape[0], d, dv)
+    return out.reshape(lead + (hla2_sde_len(d, dv),))
+
+
+def ahla_state_len(d: int, dv: int) -> int:
+    """Length of one head's AHLA streaming state [P | m | E | n]: 2 d dv + 2 d."""
+    return 2 * d * dv + 2 * d
+
+
+def ahla_summary_len(d: int, dv: int) -> int:
+    """Length of an AHLA segment summary [R | P | m | E | n]: d*d + 2 d dv + 2 d."""
+    return d * d + ahla_state_len(d, dv)
+
+
+def ahla_serial(q, k, v, normalized=False, eps=1e-6, state_in=None, return_state=False, return_den=False,
+                nthreads=1):
+    """Serial fp64 AHLA (Theorem AHLA online updates): out [BH, n, dv] (and, as requested, den [BH, n]
+    without eps and the final state [BH, ahla_state_len])."""
+    q, k, v, BH, n, d, dv = _shapes(q, k, v)
+    out = np.zeros((BH, n, dv))
+    den = np.zeros((BH, n)) if return_den else None
+    sin = None if state_in is None else _f64(state_in).reshape(BH, ahla_state_len(d, dv))
+    sout = np.zeros((BH, ahla_state_len(d, dv))) if return_state else None
+    rc = load().ahla_serial_f64(_ptr(q), _ptr(k), _ptr(v), _ptr(out), _ptr(den), BH, n, d, dv, int(normalized),
+                                float(eps), _ptr(sin), _ptr(sout), int(nthreads))
+    assert rc == 0
+    res = (out,)
+    if return_den:
+        res += (den,)
+    if return_state:
+        res += (sout,)
+    return res[0] if len(res) == 1 else res
+
+
+def ahla_chunked(q, k, v, chunk, normalized=False, eps=1e-6, return_den=False, nthreads=1):
+    """AHLA by exclusive scans under Eq. AHLA-semidirect (scan equivalence)."""
+    q, k, v, BH, n, d, dv = _shapes(q, k, v)
+    out = np.zeros((BH, n, dv))
+    den = np.zeros((BH, n)) if return_den else None
+    rc = load().ahla_chunked_f64(_ptr(q), _ptr(k), _ptr(v), _ptr(out), _ptr(den), BH, n, d, dv, int(chunk),
+                                 int(normalized), float(eps), int(nthreads))
+    assert rc == 0
+    return (out, den) if return_den else out
+
+
+def ahla_combine(A, B, d, dv):
+    """A (+)_AHLA B on summaries [R | P | m | E | n] (Eq. AHLA-semidirect)."""
+    A, B = _f64(A), _f64(B)
+    out = np.zeros(ahla_summary_len(d, dv))
+    load().ahla_combine_f64(_ptr(A), _ptr(B), _ptr(out), d, dv)
+    return out
+
+
+def hla2_backward(q, k, v, dout, masked=True, normalized=False, eps=1e-6, ckpt=64, nthreads=1):
+    """Gradients (dq, dk, dv) of L = sum_t dout_t . o_t for second-order HLA from a zero state, by the
+    reverse sweep of the online updates with checkpoints every `ckpt` tokens."""
+    q, k, v, BH, n, d, dv = _shapes(q, k, v)
+    g = _f64(dout).reshape(BH, n, dv)
+    dq, dk, dvv = np.zeros((BH, n, d)), np.zeros((BH, n, d)), np.zeros((BH, n, dv))
+    rc = load().hla2_backward_f64(_ptr(q), _ptr(k), _ptr(v), _ptr(g), _ptr(dq), _ptr(dk), _ptr(dvv), BH, n, d, dv,
+                                  int(masked), int(normalized), float(eps), int(ckpt), int(nthreads))
+    assert rc == 0
+    return dq, dk, dvv

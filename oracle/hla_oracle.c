@@ -34,6 +34,18 @@
  *                      third-order concatenation (Eqs. hla3-base-concat and
  *                      hla3-corrected-concat), segment maps applied by
  *                      contraction
+ *   hla2_state_to_sde_f64  the masked tuple folded to (S, D = S C - G,
+ *                      e = S m - h), what Theorem 1's num and den read
+ *   ahla_serial_f64    AHLA online updates (Theorem AHLA, Algorithm
+ *                      AHLA-stream at gamma = 1); state [P | m | E | n]
+ *   ahla_combine_f64   Eq. AHLA-semidirect on summaries [R | P | m | E | n]
+ *   ahla_chunked_f64   AHLA scan equivalence: exclusive Blelloch scans under
+ *                      the AHLA product within and across chunks
+ *   hla2_backward_f64  gradients of L = sum_t dout_t . o_t: the reverse sweep
+ *                      over the online updates after Theorem 1, with the
+ *                      forward states checkpointed at tile boundaries and
+ *                      recomputed within a tile (Sec. "Chunk-parallel
+ *                      training via associative scans")
  *
  * Threads: the serial functions spread the BH heads over nthreads POSIX
  * threads (heads are independent); each head is computed by one thread in
@@ -812,5 +824,429 @@ int hla3_chunked_f64(const double *q, const double *k, const double *v, double *
     if (BH < 0 || n < 0 || d < 1 || dv < 1 || chunk < 1) return 1;
     hla3_chunk_args a = {{q, k, v, out, den, n, d, dv, 1, normalized, eps, NULL, NULL}, chunk};
     run_heads(hla3_chunked_head, &a, BH, nthreads);
+    return 0;
+}
+
+/* ======================================================================== */
+/* (S, D, e) form of the masked second-order state                          */
+/* ======================================================================== */
+
+size_t hla2_sde_len_f64(int d, int dv)
+{
+    return (size_t)d * d + (size_t)d * dv + (size_t)d;
+}
+
+/*
+ * Theorem 1 reads the masked outputs as num_t = q_t^T (S_t C_t - G_t) and
+ * den_t = q_t^T (S_t m_t - h_t); this folds each head's tuple (S, C, m, G, h)
+ * into [ S | D = S C - G | e = S m - h ] (d*d, d*dv, d).
+ */
+void hla2_state_to_sde_f64(const double *st, double *out, int BH, int d, int dv)
+{
+    const size_t len = hla2_state_len_f64(d, dv), olen = hla2_sde_len_f64(d, dv);
+    for (int hd = 0; hd < BH; ++hd) {
+        const double *S = st + (size_t)hd * len, *C = S + (size_t)d * d, *m = C + (size_t)d * dv;
+        const double *G = m + d, *h = G + (size_t)d * dv;
+        double *oS = out + (size_t)hd * olen, *oD = oS + (size_t)d * d, *oe = oD + (size_t)d * dv;
+        memcpy(oS, S, sizeof(double) * (size_t)d * d);
+        mat_mul(S, C, d, d, dv, oD);
+        for (size_t i = 0; i < (size_t)d * dv; ++i) oD[i] -= G[i];
+        mat_vec(S, m, d, d, oe);
+        for (int r = 0; r < d; ++r) oe[r] -= h[r];
+    }
+}
+
+/* ======================================================================== */
+/* Asymmetric second order (AHLA), Sec. "Asymmetric Higher-order Linear      */
+/* Attention"                                                               */
+/* ======================================================================== */
+
+/* AHLA streaming state per head: [ P (d*dv) | m (d) | E (d*dv) | n (d) ] */
+size_t ahla_state_len_f64(int d, int dv)
+{
+    return 2 * (size_t)d * dv + 2 * (size_t)d;
+}
+
+typedef struct {
+    const double *q, *k, *v;
+    double *out, *den;
+    int n, d, dv, normalized;
+    double eps;
+    const double *state_in;
+    double *state_out;
+} ahla_args;
+
+/*
+ * One head of the AHLA recurrence (masked streaming identity, Theorem AHLA;
+ * Algorithm AHLA-stream at gamma = 1).  For t = 1..n:
+ *   P_t = P_{t-1} + k_t v_t^T,   m_t = m_{t-1} + k_t
+ *   E_t = E_{t-1} + k_t (q_t^T P_t),   n_t = n_{t-1} + k_t (q_t^T m_t)
+ *   num = q_t^T E_t,  den = q_t^T n_t,  out = num or num / (den + eps)
+ */
+static void ahla_serial_head(void *pargs, int hd)
+{
+    const ahla_args *a = (const ahla_args *)pargs;
+    const int n = a->n, d = a->d, dv = a->dv;
+    const double *q = a->q + (size_t)hd * n * d;
+    const double *k = a->k + (size_t)hd * n * d;
+    const double *v = a->v + (size_t)hd * n * dv;
+    double *out = a->out ? a->out + (size_t)hd * n * dv : NULL;
+    double *den_out = a->den ? a->den + (size_t)hd * n : NULL;
+    double *P = zalloc((size_t)d * dv), *m = zalloc(d), *E = zalloc((size_t)d * dv), *nn = zalloc(d);
+    double *r = zalloc(dv), *num = zalloc(dv);
+    if (a->state_in) {
+        const double *st = a->state_in + (size_t)hd * ahla_state_len_f64(d, dv);
+        memcpy(P, st, sizeof(double) * (size_t)d * dv);
+        memcpy(m, st + (size_t)d * dv, sizeof(double) * d);
+        memcpy(E, st + (size_t)d * dv + d, sizeof(double) * (size_t)d * dv);
+        memcpy(nn, st + 2 * (size_t)d * dv + d, sizeof(double) * d);
+    }
+    for (int t = 0; t < n; ++t) {
+        const double *qt = q + (size_t)t * d, *kt = k + (size_t)t * d, *vt = v + (size_t)t * dv;
+        for (int i = 0; i < d; ++i) {
+            for (int c = 0; c < dv; ++c) P[(size_t)i * dv + c] += kt[i] * vt[c];
+            m[i] += kt[i];
+        }
+        rowvec_mat(qt, P, d, dv, r);       /* r = q_t^T P_t  */
+        const double s = dot(qt, m, d);    /* s = q_t^T m_t  */
+        for (int i = 0; i < d; ++i) {
+            for (int c = 0; c < dv; ++c) E[(size_t)i * dv + c] += kt[i] * r[c];
+            nn[i] += s * kt[i];
+        }
+        rowvec_mat(qt, E, d, dv, num);     /* q_t^T E_t      */
+        const double den = dot(qt, nn, d); /* q_t^T n_t      */
+        if (out)
+            for (int c = 0; c < dv; ++c) out[(size_t)t * dv + c] = a->normalized ? num[c] / (den + a->eps) : num[c];
+        if (den_out) den_out[t] = den;
+    }
+    if (a->state_out) {
+        double *st = a->state_out + (size_t)hd * ahla_state_len_f64(d, dv);
+        memcpy(st, P, sizeof(double) * (size_t)d * dv);
+        memcpy(st + (size_t)d * dv, m, sizeof(double) * d);
+        memcpy(st + (size_t)d * dv + d, E, sizeof(double) * (size_t)d * dv);
+        memcpy(st + 2 * (size_t)d * dv + d, nn, sizeof(double) * d);
+    }
+    free(P); free(m); free(E); free(nn); free(r); free(num);
+}
+
+int ahla_serial_f64(const double *q, const double *k, const double *v, double *out, double *den,
+                    int BH, int n, int d, int dv, int normalized, double eps,
+                    const double *state_in, double *state_out, int nthreads)
+{
+    if (BH < 0 || n < 0 || d < 1 || dv < 1) return 1;
+    ahla_args a = {q, k, v, out, den, n, d, dv, normalized, eps, state_in, state_out};
+    run_heads(ahla_serial_head, &a, BH, nthreads);
+    return 0;
+}
+
+/* segment summary for the AHLA scan: [ R (d*d) | P (d*dv) | m (d) | E (d*dv) | n (d) ],
+ * R = sum over the segment of k_i q_i^T (Sec. "Chunk-parallel scans for AHLA") */
+size_t ahla_summary_len_f64(int d, int dv)
+{
+    return (size_t)d * d + ahla_state_len_f64(d, dv);
+}
+
+/*
+ * out = A (+)_AHLA B for adjacent segments, A first (Eq. AHLA-semidirect):
+ *   R = R_A + R_B,  P = P_A + P_B,  m = m_A + m_B,
+ *   E = E_A + E_B + R_B P_A,  n = n_A + n_B + R_B m_A.
+ */
+void ahla_combine_f64(const double *A, const double *B, double *out, int d, int dv)
+{
+    const size_t oR = 0, oP = (size_t)d * d, om = oP + (size_t)d * dv, oE = om + d, on = oE + (size_t)d * dv;
+    const size_t len = ahla_summary_len_f64(d, dv);
+    for (size_t i = 0; i < len; ++i) out[i] = A[i] + B[i];
+    double *RP = zalloc((size_t)d * dv), *Rm = zalloc(d);
+    mat_mul(B + oR, A + oP, d, d, dv, RP);   /* R_B P_A */
+    mat_vec(B + oR, A + om, d, d, Rm);       /* R_B m_A */
+    for (size_t i = 0; i < (size_t)d * dv; ++i) out[oE + i] += RP[i];
+    for (int i = 0; i < d; ++i) out[on + i] += Rm[i];
+    free(RP); free(Rm);
+}
+
+/* the summary of the single token (q, k, v): R = k q^T, P = k v^T, m = k, E = k (q . k) v^T, n = k (q . k) */
+static void ahla_token_summary(const double *qt, const double *kt, const double *vt, int d, int dv, double *T)
+{
+    const size_t oP = (size_t)d * d, om = oP + (size_t)d * dv, oE = om + d, on = oE + (size_t)d * dv;
+    const double qk = dot(qt, kt, d);
+    for (int i = 0; i < d; ++i) {
+        for (int j = 0; j < d; ++j) T[(size_t)i * d + j] = kt[i] * qt[j];
+        for (int c = 0; c < dv; ++c) {
+            T[oP + (size_t)i * dv + c] = kt[i] * vt[c];
+            T[oE + (size_t)i * dv + c] = kt[i] * qk * vt[c];
+        }
+        T[om + i] = kt[i];
+        T[on + i] = kt[i] * qk;
+    }
+}
+
+/* in-place exclusive Blelloch scan (up-sweep, down-sweep) of count summaries under (+)_AHLA */
+static void ahla_blelloch_exclusive(double *x, int count, int d, int dv)
+{
+    const size_t len = ahla_summary_len_f64(d, dv);
+    int p2 = 1;
+    while (p2 < count) p2 <<= 1;
+    double *buf = zalloc(len * (size_t)p2), *tmp = zalloc(len), *old_left = zalloc(len);
+    memcpy(buf, x, sizeof(double) * len * (size_t)count);   /* the padding stays the identity (zeros) */
+    for (int s = 1; s < p2; s <<= 1)
+        for (int i = 2 * s - 1; i < p2; i += 2 * s) {
+            ahla_combine_f64(buf + len * (size_t)(i - s), buf + len * (size_t)i, tmp, d, dv);
+            memcpy(buf + len * (size_t)i, tmp, sizeof(double) * len);
+        }
+    memset(buf + len * (size_t)(p2 - 1), 0, sizeof(double) * len);
+    for (int s = p2 >> 1; s >= 1; s >>= 1)
+        for (int i = 2 * s - 1; i < p2; i += 2 * s) {
+            double *l = buf + len * (size_t)(i - s), *r = buf + len * (size_t)i;
+            memcpy(old_left, l, sizeof(double) * len);
+            memcpy(l, r, sizeof(double) * len);
+            ahla_combine_f64(r, old_left, tmp, d, dv);
+            memcpy(r, tmp, sizeof(double) * len);
+        }
+    memcpy(x, buf, sizeof(double) * len * (size_t)count);
+    free(buf); free(tmp); free(old_left);
+}
+
+typedef struct {
+    const double *q, *k, *v;
+    double *out, *den;
+    int n, d, dv, chunk, normalized;
+    double eps;
+} ahla_chunk_args;
+
+/*
+ * One head by the scan route (Sec. "Chunk-parallel scans for AHLA", scan
+ * equivalence): token summaries; within each chunk an exclusive Blelloch scan
+ * gives the chunk-local prefix of every token; chunk summaries are scanned
+ * the same way across chunks; the state at token t is
+ *   carry(chunk) (+) local exclusive prefix (+) token t,
+ * and o_t = q_t^T E_t, den_t = q_t^T n_t.
+ */
+static void ahla_chunked_head(void *pargs, int hd)
+{
+    const ahla_chunk_args *a = (const ahla_chunk_args *)pargs;
+    const int n = a->n, d = a->d, dv = a->dv, C = a->chunk;
+    const size_t len = ahla_summary_len_f64(d, dv);
+    const size_t oE = (size_t)d * d + (size_t)d * dv + d, on = oE + (size_t)d * dv;
+    const double *q = a->q + (size_t)hd * n * d, *k = a->k + (size_t)hd * n * d, *v = a->v + (size_t)hd * n * dv;
+    const int nch = (n + C - 1) / C;
+    double *tok = zalloc(len * (size_t)(n > 0 ? n : 1)), *pre = zalloc(len * (size_t)(n > 0 ? n : 1));
+    double *summ = zalloc(len * (size_t)(nch > 0 ? nch : 1));
+    double *tmp = zalloc(len), *st = zalloc(len), *num = zalloc(dv);
+    for (int t = 0; t < n; ++t) ahla_token_summary(q + (size_t)t * d, k + (size_t)t * d, v + (size_t)t * dv, d, dv,
+                                                   tok + len * (size_t)t);
+    memcpy(pre, tok, sizeof(double) * len * (size_t)n);
+    for (int c = 0; c < nch; ++c) {
+        const int t0 = c * C, cnt = (n - t0 < C) ? n - t0 : C;
+        /* chunk summary = fold of its tokens */
+        double *sc = summ + len * (size_t)c;
+        memcpy(sc, tok + len * (size_t)t0, sizeof(double) * len);
+        for (int t = t0 + 1; t < t0 + cnt; ++t) {
+            ahla_combine_f64(sc, tok + len * (size_t)t, tmp, d, dv);
+            memcpy(sc, tmp, sizeof(double) * len);
+        }
+        ahla_blelloch_exclusive(pre + len * (size_t)t0, cnt, d, dv);
+    }
+    ahla_blelloch_exclusive(summ, nch, d, dv);
+    for (int t = 0; t < n; ++t) {
+        const double *carry = summ + len * (size_t)(t / C);
+        ahla_combine_f64(carry, pre + len * (size_t)t, tmp, d, dv);
+        ahla_combine_f64(tmp, tok + len * (size_t)t, st, d, dv);
+        const double *qt = q + (size_t)t * d;
+        rowvec_mat(qt, st + oE, d, dv, num);
+        const double den = dot(qt, st + on, d);
+        if (a->out)
+            for (int c = 0; c < dv; ++c)
+                a->out[((size_t)hd * n + t) * dv + c] = a->normalized ? num[c] / (den + a->eps) : num[c];
+        if (a->den) a->den[(size_t)hd * n + t] = den;
+    }
+    free(tok); free(pre); free(summ); free(tmp); free(st); free(num);
+}
+
+int ahla_chunked_f64(const double *q, const double *k, const double *v, double *out, double *den,
+                     int BH, int n, int d, int dv, int chunk, int normalized, double eps, int nthreads)
+{
+    if (BH < 0 || n < 0 || d < 1 || dv < 1 || chunk < 1) return 1;
+    ahla_chunk_args a = {q, k, v, out, den, n, d, dv, chunk, normalized, eps};
+    run_heads(ahla_chunked_head, &a, BH, nthreads);
+    return 0;
+}
+
+/* ======================================================================== */
+/* Gradients of second-order HLA (Sec. "Chunk-parallel training via          */
+/* associative scans": the reverse pass, with the forward states             */
+/* checkpointed at tile boundaries and recomputed within a tile)             */
+/* ======================================================================== */
+
+typedef struct {
+    const double *q, *k, *v, *dout;
+    double *dq, *dk, *dv;
+    int n, d, dvv, masked, normalized, ckpt;
+    double eps;
+} hla2_bwd_args;
+
+/* one forward token update of the tuple (online updates after Theorem 1) */
+static void hla2_token_update(double *st, const double *qt, const double *kt, const double *vt, int d, int dv,
+                              int masked, double *kC)
+{
+    double *S = st, *C = S + (size_t)d * d, *m = C + (size_t)d * dv, *G = m + d, *h = G + (size_t)d * dv;
+    if (masked) {
+        rowvec_mat(kt, C, d, dv, kC);
+        const double km = dot(kt, m, d);
+        for (int r = 0; r < d; ++r) {
+            for (int c = 0; c < dv; ++c) G[(size_t)r * dv + c] += kt[r] * kC[c];
+            h[r] += kt[r] * km;
+        }
+    }
+    for (int r = 0; r < d; ++r) {
+        for (int c = 0; c < d; ++c) S[(size_t)r * d + c] += kt[r] * kt[c];
+        for (int c = 0; c < dv; ++c) C[(size_t)r * dv + c] += qt[r] * vt[c];
+        m[r] += qt[r];
+    }
+}
+
+/*
+ * One head of the reverse sweep: the vector-Jacobian product of the serial
+ * recurrence for L = sum_t dout_t . o_t.  The forward states are kept at the
+ * start of every ckpt-token tile (checkpoints); each tile is recomputed
+ * forward from its checkpoint, then swept backward token by token.  With the
+ * adjoint tuple (dS, dC, dm, dG, dh) of the state after token t:
+ *   output (num = q^T S C - q^T G, den = q^T S m - q^T h on the state after t):
+ *     gnum = dout (unnormalised) or dout / (den + eps), gden = -(dout . o) / (den + eps)
+ *     dq += S C gnum - G gnum + gden (S m - h)
+ *     dS += q (C gnum)^T + gden q m^T,  dC += (S q) gnum^T,  dm += gden S q
+ *     dG -= q gnum^T,  dh -= gden q                     (masked only for G, h)
+ *   token update (state before t -> after t), in reverse:
+ *     S += k k^T:           dk += (dS + dS^T) k
+ *     C += q v^T:           dq += dC v,  dv += dC^T q
+ *     m += q:               dq += dm
+ *     G += k (k^T C_prev):  dk += dG (C_prev^T k) + C_prev (dG^T k),  dC += k (k^T dG)
+ *     h += k (k^T m_prev):  dk += dh (k . m_prev) + m_prev (k . dh),  dm += k (k . dh)
+ * (dS, dC, dm, dG, dh then belong to the state before t.)
+ */
+static void hla2_backward_head(void *pargs, int hd)
+{
+    const hla2_bwd_args *a = (const hla2_bwd_args *)pargs;
+    const int n = a->n, d = a->d, dv = a->dvv, ck = a->ckpt > 0 ? a->ckpt : 1;
+    const size_t len = hla2_state_len_f64(d, dv);
+    const size_t oC = (size_t)d * d, om = oC + (size_t)d * dv, oG = om + d, oh = oG + (size_t)d * dv;
+    const double *q = a->q + (size_t)hd * n * d, *k = a->k + (size_t)hd * n * d, *v = a->v + (size_t)hd * n * dv;
+    const double *g = a->dout + (size_t)hd * n * dv;
+    double *dq = a->dq + (size_t)hd * n * d, *dk = a->dk + (size_t)hd * n * d, *dvo = a->dv + (size_t)hd * n * dv;
+    const int ntile = (n + ck - 1) / ck;
+    double *cp = zalloc(len * (size_t)(ntile > 0 ? ntile : 1));   /* state before each tile */
+    double *tile = zalloc(len * (size_t)(ck + 1));                 /* states before / after the tile's tokens */
+    double *adj = zalloc(len), *kC = zalloc(dv);
+    double *u = zalloc(d), *Cg = zalloc(d), *Sm = zalloc(d), *num = zalloc(dv), *gnum = zalloc(dv), *tv = zalloc(d);
+    /* forward pass: checkpoints */
+    {
+        double *st = zalloc(len);
+        for (int t = 0; t < n; ++t) {
+            if (t % ck == 0) memcpy(cp + len * (size_t)(t / ck), st, sizeof(double) * len);
+            hla2_token_update(st, q + (size_t)t * d, k + (size_t)t * d, v + (size_t)t * dv, d, dv, a->masked, kC);
+        }
+        free(st);
+    }
+    memset(dq, 0, sizeof(double) * (size_t)n * d);
+    memset(dk, 0, sizeof(double) * (size_t)n * d);
+    memset(dvo, 0, sizeof(double) * (size_t)n * dv);
+    for (int ti = ntile - 1; ti >= 0; --ti) {
+        const int t0 = ti * ck, cnt = (n - t0 < ck) ? n - t0 : ck;
+        memcpy(tile, cp + len * (size_t)ti, sizeof(double) * len);
+        for (int j = 0; j < cnt; ++j) {
+            const int t = t0 + j;
+            memcpy(tile + len * (size_t)(j + 1), tile + len * (size_t)j, sizeof(double) * len);
+            hla2_token_update(tile + len * (size_t)(j + 1), q + (size_t)t * d, k + (size_t)t * d,
+                              v + (size_t)t * dv, d, dv, a->masked, kC);
+        }
+        for (int j = cnt - 1; j >= 0; --j) {
+            const int t = t0 + j;
+            const double *qt = q + (size_t)t * d, *kt = k + (size_t)t * d, *vt = v + (size_t)t * dv;
+            const double *gt = g + (size_t)t * dv;
+            const double *post = tile + len * (size_t)(j + 1), *prev = tile + len * (size_t)j;
+            const double *S = post, *C = post + oC, *m = post + om, *G = post + oG, *h = post + oh;
+            double *dS = adj, *dC = adj + oC, *dm = adj + om, *dG = adj + oG, *dh = adj + oh;
+            double *dqt = dq + (size_t)t * d, *dkt = dk + (size_t)t * d, *dvt = dvo + (size_t)t * dv;
+            /* forward values of the output at t */
+            mat_vec(S, qt, d, d, u);                     /* u = S q (S symmetric) */
+            rowvec_mat(u, C, d, dv, num);                /* u^T C     */
+            double den = dot(u, m, d);
+            if (a->masked) {
+                for (int c = 0; c < dv; ++c) {
+                    double s = 0.0;
+                    for (int r = 0; r < d; ++r) s += qt[r] * G[(size_t)r * dv + c];
+                    num[c] -= s;
+                }
+                den -= dot(qt, h, d);
+            }
+            double gden = 0.0;
+            for (int c = 0; c < dv; ++c) gnum[c] = a->normalized ? gt[c] / (den + a->eps) : gt[c];
+            if (a->normalized) {
+                double go = 0.0;
+                for (int c = 0; c < dv; ++c) go += gt[c] * num[c] / (den + a->eps);
+                gden = -go / (den + a->eps);
+            }
+            /* output adjoints */
+            mat_vec(C, gnum, d, dv, Cg);                 /* C gnum    */
+            mat_vec(S, Cg, d, d, tv);                    /* S C gnum  */
+            for (int r = 0; r < d; ++r) dqt[r] += tv[r];
+            mat_vec(S, m, d, d, Sm);                     /* S m       */
+            for (int r = 0; r < d; ++r) dqt[r] += gden * Sm[r];
+            if (a->masked) {
+                mat_vec(G, gnum, d, dv, tv);             /* G gnum    */
+                for (int r = 0; r < d; ++r) dqt[r] -= tv[r] + gden * h[r];
+            }
+            for (int r = 0; r < d; ++r) {
+                for (int c = 0; c < d; ++c) dS[(size_t)r * d + c] += qt[r] * Cg[c] + gden * qt[r] * m[c];
+                for (int c = 0; c < dv; ++c) dC[(size_t)r * dv + c] += u[r] * gnum[c];
+                dm[r] += gden * u[r];
+                if (a->masked) {
+                    for (int c = 0; c < dv; ++c) dG[(size_t)r * dv + c] -= qt[r] * gnum[c];
+                    dh[r] -= gden * qt[r];
+                }
+            }
+            /* reverse of the token update */
+            for (int r = 0; r < d; ++r) {
+                double s = 0.0;
+                for (int c = 0; c < d; ++c) s += (dS[(size_t)r * d + c] + dS[(size_t)c * d + r]) * kt[c];
+                dkt[r] += s;
+                double sc = 0.0;
+                for (int c = 0; c < dv; ++c) sc += dC[(size_t)r * dv + c] * vt[c];
+                dqt[r] += sc + dm[r];
+            }
+            for (int c = 0; c < dv; ++c) {
+                double s = 0.0;
+                for (int r = 0; r < d; ++r) s += dC[(size_t)r * dv + c] * qt[r];
+                dvt[c] += s;
+            }
+            if (a->masked) {
+                const double *Cp = prev + oC, *mp = prev + om;
+                double *kdG = zalloc(dv), *Ctk = zalloc(dv);
+                rowvec_mat(kt, dG, d, dv, kdG);          /* k^T dG       */
+                rowvec_mat(kt, Cp, d, dv, Ctk);          /* k^T C_prev   */
+                const double kdh = dot(kt, dh, d), kmp = dot(kt, mp, d);
+                for (int r = 0; r < d; ++r) {
+                    double s1 = 0.0, s2 = 0.0;
+                    for (int c = 0; c < dv; ++c) {
+                        s1 += dG[(size_t)r * dv + c] * Ctk[c];
+                        s2 += Cp[(size_t)r * dv + c] * kdG[c];
+                    }
+                    dkt[r] += s1 + s2 + dh[r] * kmp + mp[r] * kdh;
+                    for (int c = 0; c < dv; ++c) dC[(size_t)r * dv + c] += kt[r] * kdG[c];
+                    dm[r] += kt[r] * kdh;
+                }
+                free(kdG); free(Ctk);
+            }
+        }
+    }
+    free(cp); free(tile); free(adj); free(kC); free(u); free(Cg); free(Sm); free(num); free(gnum); free(tv);
+}
+
+int hla2_backward_f64(const double *q, const double *k, const double *v, const double *dout,
+                      double *dq, double *dk, double *dv, int BH, int n, int d, int dvv, int masked,
+                      int normalized, double eps, int ckpt, int nthreads)
+{
+    if (BH < 0 || n < 0 || d < 1 || dvv < 1) return 1;
+    hla2_bwd_args a = {q, k, v, dout, dq, dk, dv, n, d, dvv, masked, normalized, ckpt, eps};
+    run_heads(hla2_backward_head, &a, BH, nthreads);
     return 0;
 }

@@ -368,9 +368,206 @@ def pin_hla3_state_handoff():
         assert relerr(st2, rst) < 1e-12
 
 
+# --------------------------------------------------------------------------
+# (S, D, e) state, AHLA, gradients
+# --------------------------------------------------------------------------
+
+def pin_sde_definition():
+    """The (S, D, e) fold of the masked tuple: D_t = sum_{j<=t} x_j v_j^T and
+    e_t = sum_{j<=t} x_j with x_j = S_j q_j (proof of Theorem 1: num_t =
+    q_t^T sum_j S_j q_j v_j^T), built here token by token from the definitions
+    of S; and q_t^T D_t, q_t^T e_t are Theorem 1's num_t, den_t."""
+    n, d, dv = 9, 4, 3
+    q, k, v = rand_qkv(n, d, dv, seed=17)
+    st0 = oracle.hla2_serial(*rand_qkv(5, d, dv, seed=18), masked=True, return_state=True)[1]
+    for init in (None, st0):
+        out, den, st = oracle.hla2_serial(q, k, v, masked=True, state_in=init, return_state=True, return_den=True)
+        sde = oracle.hla2_state_to_sde(st[0], d, dv)
+        p0 = oracle.split_state2(st0[0], d, dv) if init is not None else None
+        S = p0["S"].copy() if p0 else np.zeros((d, d))
+        D = (p0["S"] @ p0["C"] - p0["G"]) if p0 else np.zeros((d, dv))
+        e = (p0["S"] @ p0["m"] - p0["h"]) if p0 else np.zeros(d)
+        for t in range(n):
+            S = S + np.outer(k[0, t], k[0, t])
+            x = S @ q[0, t]
+            D = D + np.outer(x, v[0, t])
+            e = e + x
+        assert relerr(sde[: d * d], S.ravel()) < 1e-13
+        assert relerr(sde[d * d: d * d + d * dv], D.ravel()) < 1e-12
+        assert relerr(sde[d * d + d * dv:], e) < 1e-12
+        assert relerr(q[0, -1] @ sde[d * d: d * d + d * dv].reshape(d, dv), out[0, -1]) < 1e-12
+        assert abs(q[0, -1] @ sde[d * d + d * dv:] - den[0, -1]) < 1e-12 * max(1.0, abs(den[0, -1]))
+
+
+def brute_ahla(q, k, v):
+    """AHLA from its definition (Eq. AHLA-explicit), one head: with A = L . (Q K^T),
+    (A A)_{tj} = sum_{i=j..t} (q_t.k_i)(q_i.k_j), o = (A A) V, den = (A A) 1."""
+    A = np.tril(q @ k.T)
+    AA = A @ A
+    return AA @ v, AA.sum(axis=1)
+
+
+def brute_ahla_loops(q, k, v):
+    """Eq. AHLA-explicit as nested loops over Python numbers (exact for integers)."""
+    n, d, dv = len(q), len(q[0]), len(v[0])
+    dotp = lambda a, b: sum(x * y for x, y in zip(a, b))
+    out, den = [], []
+    for t in range(n):
+        o = [0] * dv
+        s = 0
+        for j in range(t + 1):
+            w = sum(dotp(q[t], k[i]) * dotp(q[i], k[j]) for i in range(j, t + 1))
+            for c in range(dv):
+                o[c] += w * v[j][c]
+            s += w
+        out.append(o)
+        den.append(s)
+    return out, den
+
+
+def pin_ahla_bruteforce():
+    """The AHLA recurrence (Theorem AHLA) equals its defining sum, unnormalised
+    and ratio-normalised (v -> 1 gives the denominator)."""
+    n, d, dv = 10, 3, 2
+    q, k, v = rand_qkv(n, d, dv, seed=51, BH=2)
+    out, den = oracle.ahla_serial(q, k, v, return_den=True)
+    outn = oracle.ahla_serial(q, k, v, normalized=True, eps=0.3)
+    for h in range(2):
+        ref, rden = brute_ahla(q[h], k[h], v[h])
+        assert relerr(out[h], ref) < 1e-12
+        assert relerr(den[h], rden) < 1e-12
+        assert relerr(outn[h], ref / (rden + 0.3)[:, None]) < 1e-12
+
+
+def pin_ahla_exact_integers():
+    """Small-integer inputs: the fp64 recurrence equals the defining sum in Python integers bit for bit."""
+    rng = np.random.default_rng(52)
+    n, d, dv = 6, 3, 2
+    q, k, v = rng.integers(-2, 3, (n, d)), rng.integers(-2, 3, (n, d)), rng.integers(-3, 4, (n, dv))
+    ref, rden = brute_ahla_loops(q.tolist(), k.tolist(), v.tolist())
+    got, den = oracle.ahla_serial(q, k, v, return_den=True)
+    assert np.array_equal(got[0], np.array(ref, float))
+    assert np.array_equal(den[0], np.array(rden, float))
+
+
+def pin_ahla_scan_equals_serial():
+    """Scan equivalence for AHLA: exclusive Blelloch scans under Eq. AHLA-semidirect,
+    then local inclusion, reproduce the serial recurrence for every chunk size; and a
+    serial run resumed from a saved state equals one run over the concatenation."""
+    n, d, dv = 11, 3, 2
+    q, k, v = rand_qkv(n, d, dv, seed=53)
+    for normalized in (False, True):
+        ref, rden = oracle.ahla_serial(q, k, v, normalized=normalized, eps=0.25, return_den=True)
+        for chunk in range(1, n + 2):
+            got, den = oracle.ahla_chunked(q, k, v, chunk, normalized=normalized, eps=0.25, return_den=True)
+            assert relerr(got, ref) < 1e-11, (normalized, chunk)
+            assert relerr(den, rden) < 1e-11, chunk
+    ref, rst = oracle.ahla_serial(q, k, v, return_state=True)
+    o1, st = oracle.ahla_serial(q[:, :5], k[:, :5], v[:, :5], return_state=True)
+    o2, st2 = oracle.ahla_serial(q[:, 5:], k[:, 5:], v[:, 5:], state_in=st, return_state=True)
+    assert relerr(np.concatenate([o1, o2], axis=1), ref) < 1e-12
+    assert relerr(st2, rst) < 1e-12
+
+
+def pin_ahla_combine_algebra():
+    """Eq. AHLA-semidirect is associative with zero as identity, not commutative;
+    and the fold of single-token summaries (R = k q^T, P = k v^T, m = k,
+    E = (q.k) k v^T, n = (q.k) k) is the serial state (its P, m, E, n)."""
+    d, dv = 3, 2
+    L = oracle.ahla_summary_len(d, dv)
+    rng = np.random.default_rng(54)
+    A, B, C = (rng.standard_normal(L) for _ in range(3))
+    left = oracle.ahla_combine(oracle.ahla_combine(A, B, d, dv), C, d, dv)
+    right = oracle.ahla_combine(A, oracle.ahla_combine(B, C, d, dv), d, dv)
+    assert relerr(left, right) < 1e-13
+    Z = np.zeros(L)
+    assert relerr(oracle.ahla_combine(Z, A, d, dv), A) == 0.0 and relerr(oracle.ahla_combine(A, Z, d, dv), A) == 0.0
+    assert relerr(oracle.ahla_combine(A, B, d, dv), oracle.ahla_combine(B, A, d, dv)) > 1e-6
+    q, k, v = rand_qkv(7, d, dv, seed=55)
+    acc = np.zeros(L)
+    for t in range(7):
+        qt, kt, vt = q[0, t], k[0, t], v[0, t]
+        a = qt @ kt
+        T = np.concatenate([np.outer(kt, qt).ravel(), np.outer(kt, vt).ravel(), kt, a * np.outer(kt, vt).ravel(),
+                            a * kt])
+        acc = oracle.ahla_combine(acc, T, d, dv)
+    st = oracle.ahla_serial(q, k, v, return_state=True)[1][0]
+    assert relerr(acc[d * d:], st) < 1e-12
+
+
+def _loss2(q, k, v, g, masked, normalized, eps):
+    return float((oracle.hla2_serial(q, k, v, masked=masked, normalized=normalized, eps=eps) * g).sum())
+
+
+def pin_hla2_backward_finite_differences():
+    """Gradients of L = sum_t g_t . o_t from the reverse sweep equal central finite
+    differences of the forward (fp64, step 1e-6), masked and unmasked, plain and
+    ratio-normalised, for every entry of q, k and v."""
+    n, d, dv = 7, 3, 2
+    q, k, v = rand_qkv(n, d, dv, seed=61)
+    g = np.random.default_rng(62).standard_normal((1, n, dv))
+    hstep = 1e-6
+    for masked, normalized in itertools.product((True, False), (False, True)):
+        eps = 0.5
+        grads = oracle.hla2_backward(q, k, v, g, masked=masked, normalized=normalized, eps=eps, ckpt=3)
+        for x, gx in zip((q, k, v), grads):
+            fd = np.zeros_like(x)
+            for idx in np.ndindex(x.shape):
+                xp, xm = x.copy(), x.copy()
+                xp[idx] += hstep
+                xm[idx] -= hstep
+                args_p = [xp if y is x else y for y in (q, k, v)]
+                args_m = [xm if y is x else y for y in (q, k, v)]
+                fd[idx] = (_loss2(*args_p, g, masked, normalized, eps) - _loss2(*args_m, g, masked, normalized,
+                                                                               eps)) / (2 * hstep)
+            assert relerr(gx, fd) < 1e-6, (masked, normalized)
+
+
+def pin_hla2_backward_exact_integers():
+    """Integer inputs: L is a polynomial of degree at most 2 in each input entry
+    (each q_t, k_i occurs in at most two factors of the defining sums of Theorem 1 /
+    Eq. hla-unnorm), so the central difference with step 1 of the defining sum in
+    Python integers is the exact derivative; the reverse sweep must equal it bit for bit."""
+    rng = np.random.default_rng(63)
+    n, d, dv = 5, 2, 2
+    q, k, v = rng.integers(-2, 3, (n, d)), rng.integers(-2, 3, (n, d)), rng.integers(-2, 3, (n, dv))
+    g = rng.integers(-2, 3, (n, dv))
+    for masked in (True, False):
+        def loss(qq, kk, vv):
+            o, _ = brute2_loops(qq, kk, vv, masked)
+            return sum(o[t][c] * int(g[t, c]) for t in range(n) for c in range(dv))
+        grads = oracle.hla2_backward(q, k, v, g, masked=masked, ckpt=2)
+        for which, gx in enumerate(grads):
+            base = [q.tolist(), k.tolist(), v.tolist()]
+            for idx in np.ndindex(gx.shape[1:]):
+                plus = [list(map(list, a)) for a in base]
+                minus = [list(map(list, a)) for a in base]
+                plus[which][idx[0]][idx[1]] += 1
+                minus[which][idx[0]][idx[1]] -= 1
+                diff = loss(*plus) - loss(*minus)
+                assert diff % 2 == 0
+                assert gx[0][idx] == diff // 2, (masked, which, idx)
+
+
+def pin_hla2_backward_checkpoints():
+    """The reverse sweep does not depend on where the forward states are checkpointed."""
+    n, d, dv = 10, 3, 2
+    q, k, v = rand_qkv(n, d, dv, seed=64)
+    g = np.random.default_rng(65).standard_normal((1, n, dv))
+    for masked, normalized in ((True, False), (True, True), (False, True)):
+        ref = oracle.hla2_backward(q, k, v, g, masked=masked, normalized=normalized, eps=0.5, ckpt=1)
+        for ck in (3, 4, 10, 64):
+            got = oracle.hla2_backward(q, k, v, g, masked=masked, normalized=normalized, eps=0.5, ckpt=ck)
+            for a, b in zip(got, ref):
+                assert relerr(a, b) < 1e-13, ck
+
+
 ALL_PINS = [
     pin_hla2_bruteforce, pin_hla2_python_loops, pin_hla2_golden, pin_hla2_exact_integers,
     pin_hla2_masked_vs_unmasked, pin_hla2_state_definitions, pin_hla2_chunked_equals_serial,
     pin_hla2_combine_algebra, pin_hla2_special_cases, pin_hla2_causality, pin_hla2_state_handoff,
     pin_hla3_bruteforce, pin_hla3_golden, pin_hla3_chunked_equals_serial, pin_hla3_state_handoff,
+    pin_sde_definition, pin_ahla_bruteforce, pin_ahla_exact_integers, pin_ahla_scan_equals_serial,
+    pin_ahla_combine_algebra, pin_hla2_backward_finite_differences, pin_hla2_backward_exact_integers,
+    pin_hla2_backward_checkpoints,
 ]

@@ -40,6 +40,24 @@ MUTANTS = [
      "out->F[i] = A->F[i] + B->F[i] + t1[i] + t3[i];", 0),
     ("hla3_map_of_wrong_segment", "seg3_apply_maps(tk, B->t0, B->t1, A->SQ, t2, e2);",
      "seg3_apply_maps(tk, A->t0, A->t1, A->SQ, t2, e2);", 0),
+    ("sde_G_sign", "for (size_t i = 0; i < (size_t)d * dv; ++i) oD[i] -= G[i];",
+     "for (size_t i = 0; i < (size_t)d * dv; ++i) oD[i] += G[i];", 0),
+    ("sde_e_uses_m_only", "mat_vec(S, m, d, d, oe);", "memcpy(oe, m, sizeof(double) * d);", 0),
+    ("ahla_E_uses_exclusive_P", "rowvec_mat(qt, P, d, dv, r);       /* r = q_t^T P_t  */",
+     "rowvec_mat(qt, P, d, dv, r); for (int c = 0; c < dv; ++c) r[c] -= dot(qt, kt, d) * vt[c];", 0),
+    ("ahla_n_dropped_self_term", "const double s = dot(qt, m, d);    /* s = q_t^T m_t  */",
+     "const double s = dot(qt, m, d) - dot(qt, kt, d);", 0),
+    ("ahla_combine_cross_swapped", "mat_mul(B + oR, A + oP, d, d, dv, RP);   /* R_B P_A */",
+     "mat_mul(A + oR, B + oP, d, d, dv, RP);", 0),
+    ("ahla_combine_drop_Rm", "for (int i = 0; i < d; ++i) out[on + i] += Rm[i];",
+     "for (int i = 0; i < d; ++i) out[on + i] += 0.0 * Rm[i];", 0),
+    ("bwd_drop_G_adjoint_on_C", "for (int c = 0; c < dv; ++c) dC[(size_t)r * dv + c] += kt[r] * kdG[c];",
+     "for (int c = 0; c < dv; ++c) dC[(size_t)r * dv + c] += 0.0 * kdG[c];", 0),
+    ("bwd_drop_Cprev_term", "dkt[r] += s1 + s2 + dh[r] * kmp + mp[r] * kdh;", "dkt[r] += s1 + dh[r] * kmp + mp[r] * kdh;",
+     0),
+    ("bwd_gden_sign", "gden = -go / (den + a->eps);", "gden = go / (den + a->eps);", 0),
+    ("bwd_S_adjoint_not_symmetrised", "s += (dS[(size_t)r * d + c] + dS[(size_t)c * d + r]) * kt[c];",
+     "s += 2.0 * dS[(size_t)r * d + c] * kt[c];", 0),
 ]
 
 
