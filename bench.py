@@ -130,6 +130,14 @@ def dec_bytes(w):
     return w.BH * (2 * st * 4 + (2 * w.d + w.dv) * s + w.dv * s)
 
 
+def dec_sde_bytes(w):
+    """Algorithmic bytes of one decode step on (S, D, e) states: read + write of S, D, e of every
+    head plus the token I/O."""
+    st = w.d * w.d + w.d * w.dv + w.d
+    s = 2 if w.dtype == "bf16" else 4
+    return w.BH * (2 * st * 4 + (2 * w.d + w.dv) * s + w.dv * s)
+
+
 class ClockSampler:
     """nvidia-smi clock/throttle samples (every 100 ms) around a timed region."""
 
@@ -516,11 +524,10 @@ def bench_decode(hla, dev, stream, steps, hbm_peak, world):
     del tq, tk, tv
     toks = [[hla_inputs.as_torch(x[s], w.dtype, dev) for x in (qs, ks, vs)] for s in range(steps)]
     out = torch.empty((w.B, w.H, w.dv), dtype=toks[0][0].dtype, device=dev)
-    st0 = st.clone()
+    st_init = st.clone()
     for s in range(min(3, steps)):  # warm-up on a copy, then restore
         hla.hla2_step(*toks[s], st, out, masked=w.masked, normalized=w.normalized, eps=hla_inputs.EPS)
-    st.copy_(st0)
-    del st0
+    st.copy_(st_init)
     torch.cuda.synchronize()
     barrier(world)
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -533,13 +540,38 @@ def bench_decode(hla, dev, stream, steps, hbm_peak, world):
     us = max_over_ranks(e0.elapsed_time(e1) * 1e3 / steps, world)
     gbs = dec_bytes(w) / (us * 1e-6) / 1e9
     dec_traffic, dec_how = traffic("step2_kernel", "decode_bf16", 0)
-    return {"workload": "decode_bf16", "B": w.B, "H": w.H, "d": w.d, "dv": w.dv, "prefix": w.decode_prefix,
-            "steps": steps, "us_per_step": us, "value": gbs * world, "unit": "GB/s",
-            "tokens_per_s": w.B * world / (us * 1e-6),
-            "roofline": {"bound": "hbm", "achieved": gbs, "peak": hbm_peak, "unit": "GB/s", "frac": gbs / hbm_peak,
-                         "traffic": dec_traffic, "traffic_how": dec_how, "algorithmic_bytes": dec_bytes(w),
-                         "kernel": "step2_kernel"},
-            "launches": steps}
+    res = {"workload": "decode_bf16", "B": w.B, "H": w.H, "d": w.d, "dv": w.dv, "prefix": w.decode_prefix,
+           "steps": steps, "us_per_step": us, "value": gbs * world, "unit": "GB/s",
+           "tokens_per_s": w.B * world / (us * 1e-6),
+           "roofline": {"bound": "hbm", "achieved": gbs, "peak": hbm_peak, "unit": "GB/s", "frac": gbs / hbm_peak,
+                        "traffic": dec_traffic, "traffic_how": dec_how, "algorithmic_bytes": dec_bytes(w),
+                        "kernel": "step2_kernel"},
+           "launches": steps}
+
+    # the same steps on the (S, D, e) state (D = S C - G, e = S m - h): same outputs, a third fewer bytes
+    st.copy_(st_init)
+    sde = hla.hla2_state_to_sde(st, w.d, w.dv)
+    del st, st_init
+    torch.cuda.synchronize()
+    for s in range(min(3, steps)):
+        hla.hla2_step_sde(*toks[s], sde, out, normalized=w.normalized, eps=hla_inputs.EPS)
+    torch.cuda.synchronize()
+    barrier(world)
+    e0.record(stream)
+    for s in range(steps):
+        hla.hla2_step_sde(*toks[s], sde, out, normalized=w.normalized, eps=hla_inputs.EPS, stream=stream)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    us2 = max_over_ranks(e0.elapsed_time(e1) * 1e3 / steps, world)
+    gbs2 = dec_sde_bytes(w) / (us2 * 1e-6) / 1e9
+    res["sde"] = {"state": "(S, D, e)", "us_per_step": us2, "value": gbs2 * world, "unit": "GB/s",
+                  "tokens_per_s": w.B * world / (us2 * 1e-6),
+                  "roofline": {"bound": "hbm", "achieved": gbs2, "peak": hbm_peak, "unit": "GB/s",
+                               "frac": gbs2 / hbm_peak, "traffic": None, "algorithmic_bytes": dec_sde_bytes(w),
+                               "kernel": "step2_kernel (S, D, e)"},
+                  "launches": steps}
+    res["launches"] += steps
+    return res
 
 
 if __name__ == "__main__":

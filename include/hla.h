@@ -123,6 +123,47 @@ hla_status hla2_step(const void *q, const void *k, const void *v, void *out, hla
                      float *state, hla_stream_t stream);
 
 /*
+ * The (S, D, e) decode state of the masked operator (no counterpart printed in
+ * the paper; it follows from Theorem 1 and Eq. semidirect).  With
+ * D = S C - G (d x dv) and e = S m - h (d), Theorem 1's outputs read
+ * num_t = q_t^T D_t and den_t = q_t^T e_t, and the online updates after
+ * Theorem 1 collapse to
+ *   S' = S + k k^T,   x = S' q,   D' = D + x v^T,   e' = e + x.
+ * Per head (fp32, row-major): [ S (d*d) | D (d*dv) | e (d) ], heads in [B, H]
+ * order.  It carries exactly what the masked outputs need with d*d + d*dv + d
+ * floats instead of the tuple's d*d + 2*d*dv + 2*d (a third fewer bytes per
+ * decode step at d = dv); the tuple cannot be recovered from it (C, m, G, h
+ * are folded together).  This is one of the state-format options of the
+ * paper's implementation considerations (Sec. "Implementation details and
+ * complexity").
+ */
+size_t hla2_sde_state_floats(int d, int dv);
+
+/*
+ * hla2_state_to_sde -- convert B*H masked second-order tuples (S, C, m, G, h)
+ * (hla2_state_floats each, e.g. a state_out of hla2_forward) into (S, D, e)
+ * states: D = S C - G, e = S m - h, fp32 on the device.
+ * state : device fp32 [B*H * hla2_state_floats(d,dv)] (read only)
+ * sde   : device fp32 [B*H * hla2_sde_state_floats(d,dv)] (written); must not
+ *         overlap state.  Both 16-byte aligned.
+ * Errors: HLA_ERR_INVALID_ARGUMENT (null, misaligned, overlapping),
+ * HLA_ERR_UNSUPPORTED (d, dv outside {16, 32, 64, 128}), HLA_ERR_CUDA.
+ */
+hla_status hla2_state_to_sde(const float *state, float *sde, int B, int H, int d, int dv, hla_stream_t stream);
+
+/*
+ * hla2_step_sde -- hla2_step of the masked operator on (S, D, e) states:
+ *   S += k k^T;  x = S q;  D += x v^T;  e += x;
+ *   num = q^T D,  den = q^T e,  out = num or num / (den + eps).
+ * q, k : device [B, H, d] of type dt; v, out : device [B, H, dv] of type dt
+ * sde  : device fp32 [B*H * hla2_sde_state_floats(d,dv)], updated in place
+ * Errors as for hla2_step.
+ */
+hla_status hla2_step_sde(const void *q, const void *k, const void *v, void *out, hla_dtype dt,
+                         int B, int H, int d, int dv, int normalized, float eps,
+                         float *sde, hla_stream_t stream);
+
+/*
  * hla2_forward_path -- which CUDA path hla2_forward takes for these arguments
  * on the current device, without launching anything:
  *   0  generic path: fp32 CUDA-core kernels (every supported shape);
@@ -192,6 +233,45 @@ hla_status hla3_forward(const void *q, const void *k, const void *v, void *out, 
 hla_status hla2_forward_noalloc(const void *q, const void *k, const void *v, void *out, hla_dtype dt,
                                 int B, int H, int n, int d, int dv, int masked, int normalized, float eps,
                                 int chunk, const float *state_in, hla_stream_t stream);
+
+/*
+ * Asymmetric second-order HLA (AHLA), Sec. "Asymmetric Higher-order Linear
+ * Attention".  The operator is always causal:
+ *   o_t = sum_{j<=t} sum_{i=j..t} (q_t.k_i)(q_i.k_j) v_j   (Eq. AHLA-explicit),
+ * computed as q_t^T E_t with the streaming state of Theorem AHLA:
+ *   P_t = P_{t-1} + k_t v_t^T,  m_t = m_{t-1} + k_t,
+ *   E_t = E_{t-1} + k_t (q_t^T P_t),  n_t = n_{t-1} + k_t (q_t^T m_t),
+ *   out_t = q_t^T E_t, or q_t^T E_t / (q_t^T n_t + eps) if normalized.
+ * State of one head (fp32, row-major): [ P (d*dv) | m (d) | E (d*dv) | n (d) ].
+ */
+size_t ahla_state_floats(int d, int dv);
+
+/* Bytes of scratch workspace ahla_forward needs (0 if unsupported). */
+size_t ahla_workspace_bytes(int B, int H, int n, int d, int dv, int chunk, hla_dtype dt);
+
+/*
+ * ahla_forward -- chunk-parallel AHLA forward: chunk summaries composed with
+ * the AHLA semidirect product (Eq. AHLA-semidirect, with the segment cross
+ * moment R^KQ = sum k q^T of the later segment), which reproduces the serial
+ * recurrence (scan equivalence); chunk is the scan granularity (results do not
+ * depend on it up to rounding).  Arguments, layouts, shapes and errors as for
+ * hla2_forward (no masked flag), with the AHLA state layout for state_in /
+ * state_out (state_out may equal state_in).
+ */
+hla_status ahla_forward(const void *q, const void *k, const void *v, void *out, hla_dtype dt,
+                        int B, int H, int n, int d, int dv, int normalized, float eps, int chunk,
+                        const float *state_in, float *state_out,
+                        void *workspace, size_t workspace_bytes, hla_stream_t stream);
+
+/*
+ * ahla_step -- one AHLA decode step for B*H heads (the online updates of
+ * Theorem AHLA; Algorithm AHLA-stream at gamma = 1): q, k [B, H, d], v, out
+ * [B, H, dv] of type dt; state fp32 [B*H * ahla_state_floats(d,dv)], updated
+ * in place.  Errors as for hla2_step.
+ */
+hla_status ahla_step(const void *q, const void *k, const void *v, void *out, hla_dtype dt,
+                     int B, int H, int d, int dv, int normalized, float eps,
+                     float *state, hla_stream_t stream);
 
 /*
  * hla_poll_error_noalloc -- hla_poll_error for hla2_forward_noalloc (no

@@ -176,6 +176,81 @@ hla_status hla2_step(const void *q, const void *k, const void *v, void *out, hla
                        "decode step");
 }
 
+size_t hla2_sde_state_floats(int d, int dv) {
+    if (d <= 0 || dv <= 0) return 0;
+    return (size_t)d * d + (size_t)d * dv + (size_t)d;
+}
+
+hla_status hla2_state_to_sde(const float *state, float *sde, int B, int H, int d, int dv, hla_stream_t stream) {
+    g_last_error[0] = 0;
+    if (B < 0 || H < 0) return fail(HLA_ERR_INVALID_ARGUMENT, "negative size B=%d H=%d", B, H);
+    if (!dim_ok(d) || !dim_ok(dv))
+        return fail(HLA_ERR_UNSUPPORTED, "d=%d dv=%d: supported sizes are 16, 32, 64, 128", d, dv);
+    const long long BH = (long long)B * H;
+    if (BH == 0) return HLA_OK;
+    if (BH > (1LL << 31) - 1) return fail(HLA_ERR_UNSUPPORTED, "problem too large");
+    if (!state || !sde) return fail(HLA_ERR_INVALID_ARGUMENT, "null state pointer");
+    if (!aligned16(state) || !aligned16(sde)) return fail(HLA_ERR_INVALID_ARGUMENT, "states must be 16-byte aligned");
+    const uintptr_t a0 = reinterpret_cast<uintptr_t>(state), a1 = a0 + sizeof(float) * BH * hla2_state_floats(d, dv);
+    const uintptr_t b0 = reinterpret_cast<uintptr_t>(sde), b1 = b0 + sizeof(float) * BH * hla2_sde_state_floats(d, dv);
+    if (a0 < b1 && b0 < a1) return fail(HLA_ERR_INVALID_ARGUMENT, "state and sde must not overlap");
+    return cuda_status(state_to_sde_launch(state, sde, (int)BH, d, dv, reinterpret_cast<cudaStream_t>(stream)),
+                       "state conversion");
+}
+
+hla_status hla2_step_sde(const void *q, const void *k, const void *v, void *out, hla_dtype dt, int B, int H, int d,
+                         int dv, int normalized, float eps, float *sde, hla_stream_t stream) {
+    g_last_error[0] = 0;
+    hla_status st = check_forward(q, k, v, out, dt, B, H, 1, d, dv, 1, normalized, eps, 1, sde, sde);
+    if (st != HLA_OK) return st;
+    if ((long long)B * H == 0) return HLA_OK;
+    if (!sde) return fail(HLA_ERR_INVALID_ARGUMENT, "null state pointer");
+    return cuda_status(step2_sde_launch(q, k, v, out, dt, B * H, d, dv, normalized, eps, sde,
+                                        reinterpret_cast<cudaStream_t>(stream)),
+                       "decode step (S, D, e)");
+}
+
+size_t ahla_state_floats(int d, int dv) {
+    if (d <= 0 || dv <= 0) return 0;
+    return 2 * (size_t)d * dv + 2 * (size_t)d;
+}
+
+size_t ahla_workspace_bytes(int B, int H, int n, int d, int dv, int chunk, hla_dtype dt) {
+    if (B < 0 || H < 0 || n < 0 || !dim_ok(d) || !dim_ok(dv) || chunk < 1 || chunk > 128) return 0;
+    if (dt != HLA_F32 && dt != HLA_BF16) return 0;
+    return align_up(ahla_workspace_bytes_internal(B * H, n, d, dv, chunk), 256);
+}
+
+hla_status ahla_forward(const void *q, const void *k, const void *v, void *out, hla_dtype dt, int B, int H, int n,
+                        int d, int dv, int normalized, float eps, int chunk, const float *state_in, float *state_out,
+                        void *workspace, size_t workspace_bytes, hla_stream_t stream) {
+    g_last_error[0] = 0;
+    hla_status st = check_forward(q, k, v, out, dt, B, H, n, d, dv, 1, normalized, eps, chunk, state_in, state_out);
+    if (st != HLA_OK) return st;
+    const size_t need = ahla_workspace_bytes(B, H, n, d, dv, chunk, dt);
+    if (!workspace || workspace_bytes < need)
+        return fail(HLA_ERR_WORKSPACE, "workspace of %zu bytes needed, %zu given", need,
+                    workspace ? workspace_bytes : (size_t)0);
+    if ((reinterpret_cast<uintptr_t>(workspace) & 255u) != 0)
+        return fail(HLA_ERR_INVALID_ARGUMENT, "workspace must be 256-byte aligned");
+    if ((long long)B * H == 0) return HLA_OK;
+    Fwd2 p{q, k, v, out, dt, B * H, n, d, dv, 1, normalized, eps, chunk, state_in, state_out,
+           static_cast<char *>(workspace), workspace_bytes};
+    return cuda_status(ahla_forward_launch(p, reinterpret_cast<cudaStream_t>(stream)), "AHLA forward");
+}
+
+hla_status ahla_step(const void *q, const void *k, const void *v, void *out, hla_dtype dt, int B, int H, int d,
+                     int dv, int normalized, float eps, float *state, hla_stream_t stream) {
+    g_last_error[0] = 0;
+    hla_status st = check_forward(q, k, v, out, dt, B, H, 1, d, dv, 1, normalized, eps, 1, state, state);
+    if (st != HLA_OK) return st;
+    if ((long long)B * H == 0) return HLA_OK;
+    if (!state) return fail(HLA_ERR_INVALID_ARGUMENT, "null state pointer");
+    return cuda_status(ahla_step_launch(q, k, v, out, dt, B * H, d, dv, normalized, eps, state,
+                                        reinterpret_cast<cudaStream_t>(stream)),
+                       "AHLA decode step");
+}
+
 hla_status hla3_forward(const void *q, const void *k, const void *v, void *out, hla_dtype dt, int B, int H, int n,
                         int d, int dv, int masked, int normalized, float eps, int chunk, const float *state_in,
                         float *state_out, void *workspace, size_t workspace_bytes, hla_stream_t stream) {

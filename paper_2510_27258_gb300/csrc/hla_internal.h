@@ -73,6 +73,17 @@ cudaError_t fused2_forward(const Fwd2 &p, cudaStream_t stream);
 cudaError_t step2_launch(const void *q, const void *k, const void *v, void *out, hla_dtype dt, int BH, int d,
                          int dv, int masked, int normalized, float eps, float *state, cudaStream_t stream);
 
+// decode step on the (S, D, e) state, and the conversion of paper tuples to it
+cudaError_t step2_sde_launch(const void *q, const void *k, const void *v, void *out, hla_dtype dt, int BH, int d,
+                             int dv, int normalized, float eps, float *state, cudaStream_t stream);
+cudaError_t state_to_sde_launch(const float *src, float *dst, int BH, int d, int dv, cudaStream_t stream);
+
+// AHLA (asymmetric second order): chunk-parallel forward and decode step
+size_t ahla_workspace_bytes_internal(int BH, int n, int d, int dv, int chunk);
+cudaError_t ahla_forward_launch(const Fwd2 &p, cudaStream_t stream);
+cudaError_t ahla_step_launch(const void *q, const void *k, const void *v, void *out, hla_dtype dt, int BH, int d,
+                             int dv, int normalized, float eps, float *state, cudaStream_t stream);
+
 // third order
 size_t generic3_workspace_bytes(int BH, int n, int d, int dv, int chunk);
 cudaError_t generic3_forward(const Fwd2 &p, cudaStream_t stream);

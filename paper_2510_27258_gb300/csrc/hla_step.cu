@@ -90,7 +90,12 @@ __device__ __forceinline__ void store4(float4 *p, float4 v) { *p = v; }
 // part as soon as its pass has read it, so that while one pass works the copies of the next two
 // parts (and of the next head's tokens) are in flight.  Updated values go to global memory straight
 // from registers.
-template <typename T>
+//
+// kSDE: the state is (S, D, e) with D = S C - G and e = S m - h (masked operator only; rows of the
+// per-head record: S d*d | D d*dv | e d).  A token then updates
+//   S' = S + k k^T,  u' = S' q,  D' = D + u' v^T,  e' = e + u'
+// and num = q^T D' = q^T D + (q.u') v^T, den = q.e' = q.e + q.u': one pass over S and one over D.
+template <typename T, bool kSDE>
 __global__ void __launch_bounds__(kStepThreads, 1)
 step2_kernel(const T *__restrict__ q, const T *__restrict__ k, const T *__restrict__ v, T *__restrict__ out,
              float *__restrict__ state, int BH, int d, int dv, int masked, int normalized, float eps) {
@@ -100,7 +105,8 @@ step2_kernel(const T *__restrict__ q, const T *__restrict__ k, const T *__restri
     __shared__ float kC[128], uC[128], qG[128];
 
     const int tid = threadIdx.x;
-    const long long st_len = (long long)d * d + 2LL * d * dv + 2LL * d;
+    if (kSDE) masked = 0;  // staging as for (S, C, m): no third buffer
+    const long long st_len = kSDE ? (long long)d * d + (long long)d * dv + d : (long long)d * d + 2LL * d * dv + 2LL * d;
     const int nS = (d * d) >> 2, nCm = (d * dv + d) >> 2;  // float4 units of S and of (C, m) / (G, h)
     const int nt_q = d * (int)sizeof(T) / 16, nt_v = dv * (int)sizeof(T) / 16;  // 16-byte token chunks
     float4 *bS = dyn, *bC = bS + nS, *bG = bC + nCm;
@@ -196,6 +202,45 @@ step2_kernel(const T *__restrict__ q, const T *__restrict__ k, const T *__restri
         __syncthreads();  // S buffer read, u' complete
         if (nx < BH) load_S(nx); else cp_commit();
 
+        if constexpr (kSDE) {
+            // ---- pass over D: column sums q^T D (old D); D' = D + u' v^T; e' = e + u' ----
+            cp_wait<1>();  // (D, e) of this head
+            __syncthreads();
+            const float *ev = reinterpret_cast<const float *>(bC + ((d * dv) >> 2));
+            float *eg = Cm + (long long)d * dv;
+            if (tid < d) eg[tid] = ev[tid] + us[tid];
+            const float qe = warp_dot(qs, ev, d), uq = warp_dot(us, qs, d);
+            const int wv = dv >> 2, nD = (d * dv) >> 2, c4 = (tid % wv) * 4;
+            {
+                float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+                float4 *Dg = reinterpret_cast<float4 *>(Cm);
+                const float v0 = vs[c4], v1 = vs[c4 + 1], v2 = vs[c4 + 2], v3 = vs[c4 + 3];
+#pragma unroll
+                for (int i = 0; i < kMaxUnits; ++i) {
+                    const int f = tid + i * kStepThreads;
+                    if (f < nD) {
+                        const int row = f / wv;
+                        const float4 c = bC[f];
+                        const float qr = qs[row], ur = us[row];
+                        acc.x += qr * c.x; acc.y += qr * c.y; acc.z += qr * c.z; acc.w += qr * c.w;
+                        store4(Dg + f, make_float4(c.x + ur * v0, c.y + ur * v1, c.z + ur * v2, c.w + ur * v3));
+                    }
+                }
+                part[tid][0] = acc.x; part[tid][1] = acc.y; part[tid][2] = acc.z; part[tid][3] = acc.w;
+            }
+            __syncthreads();  // (D, e) buffer read
+            if (nx < BH) load_part(bC, nx, offC); else cp_commit();
+            if (tid < dv) {
+                const int grp = tid >> 2, comp = tid & 3;
+                float a = 0.f;
+                for (int g = grp; g < kStepThreads; g += wv) a += part[g][comp];
+                const float num = a + uq * vs[tid];
+                from_f32(&out[(long long)hd * dv + tid], normalized ? num / (qe + uq + eps) : num);
+            }
+            __syncthreads();  // qs, ks, vs, us, part read before the next head rewrites them
+            continue;
+        }
+
         // ---- pass over C: column sums k^T C, u'^T C; C' = C + q v^T; m' = m + q ----
         if (masked) cp_wait<2>(); else cp_wait<1>();  // (C, m) of this head
         __syncthreads();
@@ -290,18 +335,18 @@ size_t step2_smem(int d, int dv, int masked, size_t tsize) {
     return 16 * (nS + nCm * (masked ? 2 : 1)) + tsize * (2 * (size_t)d + dv);
 }
 
-}  // namespace
-
-cudaError_t step2_launch(const void *q, const void *k, const void *v, void *out, hla_dtype dt, int BH, int d, int dv,
-                         int masked, int normalized, float eps, float *state, cudaStream_t stream) {
+template <bool kSDE>
+cudaError_t step2_launch_t(const void *q, const void *k, const void *v, void *out, hla_dtype dt, int BH, int d,
+                           int dv, int masked, int normalized, float eps, float *state, cudaStream_t stream) {
     if (BH == 0) return cudaSuccess;
     int dev = 0, sms = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     if (e != cudaSuccess) return e;
     const int grid = BH < sms ? BH : sms;
+    if (kSDE) masked = 0;  // shared-memory staging of (S, D, e) is that of (S, C, m)
     if (dt == HLA_BF16) {
-        auto kern = step2_kernel<__nv_bfloat16>;
+        auto kern = step2_kernel<__nv_bfloat16, kSDE>;
         const size_t sm = step2_smem(d, dv, masked, sizeof(__nv_bfloat16));
         if ((e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm))) return e;
         kern<<<grid, kStepThreads, sm, stream>>>(static_cast<const __nv_bfloat16 *>(q),
@@ -310,13 +355,60 @@ cudaError_t step2_launch(const void *q, const void *k, const void *v, void *out,
                                                 static_cast<__nv_bfloat16 *>(out), state, BH, d, dv, masked,
                                                 normalized, eps);
     } else {
-        auto kern = step2_kernel<float>;
+        auto kern = step2_kernel<float, kSDE>;
         const size_t sm = step2_smem(d, dv, masked, sizeof(float));
         if ((e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm))) return e;
         kern<<<grid, kStepThreads, sm, stream>>>(static_cast<const float *>(q), static_cast<const float *>(k),
                                                 static_cast<const float *>(v), static_cast<float *>(out), state,
                                                 BH, d, dv, masked, normalized, eps);
     }
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t step2_launch(const void *q, const void *k, const void *v, void *out, hla_dtype dt, int BH, int d, int dv,
+                         int masked, int normalized, float eps, float *state, cudaStream_t stream) {
+    return step2_launch_t<false>(q, k, v, out, dt, BH, d, dv, masked, normalized, eps, state, stream);
+}
+
+cudaError_t step2_sde_launch(const void *q, const void *k, const void *v, void *out, hla_dtype dt, int BH, int d,
+                             int dv, int normalized, float eps, float *state, cudaStream_t stream) {
+    return step2_launch_t<true>(q, k, v, out, dt, BH, d, dv, 1, normalized, eps, state, stream);
+}
+
+namespace {
+
+// (S, C, m, G, h) -> (S, D = S C - G, e = S m - h) per head, one block per head, the tuple staged in
+// shared memory (dst must not overlap src: blocks of other heads may still be reading it).
+__global__ void __launch_bounds__(256) state_to_sde_kernel(const float *src, float *dst, int d, int dv) {
+    extern __shared__ float st[];
+    const int hd = blockIdx.x, tid = threadIdx.x;
+    const long long len = (long long)d * d + 2LL * d * dv + 2LL * d;
+    const float4 *s4 = reinterpret_cast<const float4 *>(src + hd * len);
+    float4 *st4 = reinterpret_cast<float4 *>(st);
+    for (int i = tid; i < (int)(len >> 2); i += blockDim.x) st4[i] = s4[i];
+    __syncthreads();
+    const float *S = st, *C = S + d * d, *m = C + d * dv, *G = m + d, *h = G + d * dv;
+    float *o = dst + hd * ((long long)d * d + (long long)d * dv + d);
+    for (int i = tid; i < d * d; i += blockDim.x) o[i] = S[i];
+    for (int i = tid; i < d * dv + d; i += blockDim.x) {
+        const bool is_e = i >= d * dv;
+        const int a = is_e ? i - d * dv : i / dv, b = is_e ? 0 : i % dv;
+        float acc = 0.f;
+        for (int j = 0; j < d; ++j) acc += S[a * d + j] * (is_e ? m[j] : C[j * dv + b]);
+        o[d * d + i] = acc - (is_e ? h[a] : G[i]);
+    }
+}
+
+}  // namespace
+
+cudaError_t state_to_sde_launch(const float *src, float *dst, int BH, int d, int dv, cudaStream_t stream) {
+    if (BH == 0) return cudaSuccess;
+    const size_t smem = sizeof(float) * ((size_t)d * d + 2 * (size_t)d * dv + 2 * (size_t)d);
+    cudaError_t e = cudaFuncSetAttribute(state_to_sde_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e) return e;
+    state_to_sde_kernel<<<BH, 256, smem, stream>>>(src, dst, d, dv);
     return cudaGetLastError();
 }
 

@@ -22,7 +22,9 @@ HLA_F32, HLA_BF16 = 0, 1
 # every symbol include/hla.h declares
 EXPORTS = ("hla_status_string", "hla_last_error", "hla2_state_floats", "hla2_workspace_bytes", "hla2_forward",
            "hla2_forward_path", "hla2_step", "hla3_state_floats", "hla3_workspace_bytes", "hla3_forward",
-           "hla2_forward_noalloc", "hla_poll_error_noalloc", "hla_poll_error")
+           "hla2_forward_noalloc", "hla_poll_error_noalloc", "hla_poll_error", "hla2_sde_state_floats",
+           "hla2_state_to_sde", "hla2_step_sde", "ahla_state_floats", "ahla_workspace_bytes", "ahla_forward",
+           "ahla_step")
 
 _lib = None
 
@@ -50,7 +52,13 @@ def lib():
         for name in ("hla2_state_floats", "hla3_state_floats"):
             getattr(L, name).argtypes = [i, i]
             getattr(L, name).restype = sz
-        for name in ("hla2_workspace_bytes", "hla3_workspace_bytes"):
+        L.ahla_state_floats.argtypes = [i, i]
+        L.ahla_state_floats.restype = sz
+        L.ahla_forward.argtypes = [vp, vp, vp, vp, i, i, i, i, i, i, i, f, i, vp, vp, vp, sz, vp]
+        L.ahla_forward.restype = i
+        L.ahla_step.argtypes = [vp, vp, vp, vp, i, i, i, i, i, i, f, vp, vp]
+        L.ahla_step.restype = i
+        for name in ("hla2_workspace_bytes", "hla3_workspace_bytes", "ahla_workspace_bytes"):
             getattr(L, name).argtypes = [i, i, i, i, i, i, i]
             getattr(L, name).restype = sz
         for name in ("hla2_forward", "hla3_forward"):
@@ -66,6 +74,12 @@ def lib():
         L.hla_poll_error.restype = i
         L.hla_poll_error_noalloc.argtypes = [vp]
         L.hla_poll_error_noalloc.restype = i
+        L.hla2_sde_state_floats.argtypes = [i, i]
+        L.hla2_sde_state_floats.restype = sz
+        L.hla2_state_to_sde.argtypes = [vp, vp, i, i, i, i, vp]
+        L.hla2_state_to_sde.restype = i
+        L.hla2_step_sde.argtypes = [vp, vp, vp, vp, i, i, i, i, i, i, f, vp, vp]
+        L.hla2_step_sde.restype = i
         _lib = L
     return _lib
 
@@ -196,6 +210,80 @@ def hla2_step(q, k, v, state, out=None, *, masked=True, normalized=False, eps=1e
     code = lib().hla2_step(_ptr(q), _ptr(k), _ptr(v), _ptr(out), _dtype_code(q), B, H, d, dv, int(masked),
                            int(normalized), float(eps), _ptr(state), _stream(stream))
     _check(code, "hla2_step")
+    return out
+
+
+def ahla_state_floats(d: int, dv: int) -> int:
+    return int(lib().ahla_state_floats(d, dv))
+
+
+def ahla_workspace_bytes(B, H, n, d, dv, chunk, dtype) -> int:
+    code = dtype if isinstance(dtype, int) else (HLA_BF16 if dtype == torch.bfloat16 else HLA_F32)
+    return int(lib().ahla_workspace_bytes(B, H, n, d, dv, chunk, code))
+
+
+def ahla_forward(q, k, v, out=None, *, normalized=False, eps=1e-6, chunk=64, state_in=None, state_out=None,
+                 workspace=None, stream=None):
+    """AHLA forward (include/hla.h: ahla_forward). Returns ``out``."""
+    if q.dim() != 4:
+        raise ValueError("q, k, v must be [B, H, n, d]")
+    B, H, n, d = q.shape
+    dv = v.shape[-1]
+    for t in (q, k, v):
+        if not t.is_cuda or not t.is_contiguous() or t.dtype != q.dtype:
+            raise ValueError("q, k, v must be contiguous CUDA tensors of one dtype")
+    if out is None:
+        out = torch.empty((B, H, n, dv), dtype=q.dtype, device=q.device)
+    dt = _dtype_code(q)
+    if workspace is None:
+        workspace = alloc_workspace(ahla_workspace_bytes(B, H, n, d, dv, chunk, dt), q.device)
+    code = lib().ahla_forward(_ptr(q), _ptr(k), _ptr(v), _ptr(out), dt, B, H, n, d, dv, int(normalized), float(eps),
+                              int(chunk), _ptr(state_in), _ptr(state_out), _ptr(workspace),
+                              workspace.numel() * workspace.element_size(), _stream(stream))
+    _check(code, "ahla_forward")
+    return out
+
+
+def ahla_step(q, k, v, state, out=None, *, normalized=False, eps=1e-6, stream=None):
+    """One AHLA decode step for every head (include/hla.h: ahla_step); ``state`` is updated in place."""
+    B, H, d = q.shape
+    dv = v.shape[-1]
+    if out is None:
+        out = torch.empty((B, H, dv), dtype=q.dtype, device=q.device)
+    if state.dtype != torch.float32 or not state.is_contiguous():
+        raise ValueError("state must be contiguous float32")
+    code = lib().ahla_step(_ptr(q), _ptr(k), _ptr(v), _ptr(out), _dtype_code(q), B, H, d, dv, int(normalized),
+                           float(eps), _ptr(state), _stream(stream))
+    _check(code, "ahla_step")
+    return out
+
+
+def hla2_sde_state_floats(d: int, dv: int) -> int:
+    return int(lib().hla2_sde_state_floats(d, dv))
+
+
+def hla2_state_to_sde(state, d: int, dv: int, sde=None, *, stream=None):
+    """(S, C, m, G, h) tuples [B, H, hla2_state_floats(d, dv)] -> (S, D, e) states
+    [B, H, hla2_sde_state_floats(d, dv)] (include/hla.h: hla2_state_to_sde)."""
+    B, H = state.shape[:2]
+    if sde is None:
+        sde = torch.empty((B, H, hla2_sde_state_floats(d, dv)), dtype=torch.float32, device=state.device)
+    _check(lib().hla2_state_to_sde(_ptr(state), _ptr(sde), B, H, d, dv, _stream(stream)), "hla2_state_to_sde")
+    return sde
+
+
+def hla2_step_sde(q, k, v, sde, out=None, *, normalized=False, eps=1e-6, stream=None):
+    """One decode step of the masked operator on (S, D, e) states, updated in place
+    (include/hla.h: hla2_step_sde).  q, k: [B, H, d]; v: [B, H, dv]."""
+    B, H, d = q.shape
+    dv = v.shape[-1]
+    if out is None:
+        out = torch.empty((B, H, dv), dtype=q.dtype, device=q.device)
+    if sde.dtype != torch.float32 or not sde.is_contiguous():
+        raise ValueError("state must be contiguous float32")
+    code = lib().hla2_step_sde(_ptr(q), _ptr(k), _ptr(v), _ptr(out), _dtype_code(q), B, H, d, dv, int(normalized),
+                               float(eps), _ptr(sde), _stream(stream))
+    _check(code, "hla2_step_sde")
     return out
 
 

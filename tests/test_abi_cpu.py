@@ -21,7 +21,7 @@ def L():
 def declared_functions():
     text = open(HEADER).read()
     text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
-    return sorted(set(re.findall(r"\b(hla\w+)\s*\(", text)))
+    return sorted(set(re.findall(r"\b((?:hla|ahla)\w+)\s*\(", text)))
 
 
 def test_header_declares_expected_entry_points():
@@ -95,3 +95,28 @@ def test_step_argument_errors(L):
 def test_poll_error_null_workspace(L):
     from paper_2510_27258_gb300 import hla as H
     assert L.hla_poll_error(None, None) == H.HLA_ERR_INVALID_ARGUMENT
+
+
+def test_sde_sizes_and_argument_errors(L):
+    from paper_2510_27258_gb300 import hla as H
+    assert L.hla2_sde_state_floats(128, 128) == 128 * 128 + 128 * 128 + 128
+    assert L.hla2_sde_state_floats(16, 32) == 16 * 16 + 16 * 32 + 16
+    f = ctypes.c_float(0.0)
+    # conversion: null, misaligned, unsupported head size, overlapping buffers, empty problem
+    assert L.hla2_state_to_sde(None, 4096, 1, 1, 16, 16, None) == H.HLA_ERR_INVALID_ARGUMENT
+    assert L.hla2_state_to_sde(4100, 1 << 20, 1, 1, 16, 16, None) == H.HLA_ERR_INVALID_ARGUMENT
+    assert L.hla2_state_to_sde(4096, 1 << 20, 1, 1, 24, 16, None) == H.HLA_ERR_UNSUPPORTED
+    assert L.hla2_state_to_sde(4096, 4096 + 64, 1, 1, 16, 16, None) == H.HLA_ERR_INVALID_ARGUMENT
+    assert "overlap" in L.hla_last_error().decode()
+    assert L.hla2_state_to_sde(4096, 4096, 0, 1, 16, 16, None) == H.HLA_OK
+    # decode step on (S, D, e): as hla2_step
+    assert L.hla2_step_sde(16, 16, 16, 16, 1, 1, 1, 128, 128, 0, f, None, None) == H.HLA_ERR_INVALID_ARGUMENT
+    assert L.hla2_step_sde(16, 16, 16, 16, 1, 1, 1, 100, 128, 0, f, 16, None) == H.HLA_ERR_UNSUPPORTED
+    assert L.hla2_step_sde(16, 16, 16, 16, 1, 0, 1, 128, 128, 0, f, 16, None) == H.HLA_OK
+
+
+def test_noalloc_empty_problem_without_gpu(L):
+    from paper_2510_27258_gb300 import hla as H
+    f = ctypes.c_float(1e-6)
+    assert L.hla2_forward_noalloc(None, None, None, None, 1, 1, 0, 256, 128, 128, 1, 0, f, 128, None, None) == H.HLA_OK
+    assert L.hla_last_error() == b""
