@@ -117,6 +117,22 @@ def hla3_flops(w):
     return 2 * chunks * (local + bracket + out)
 
 
+def ahla_flops(w):
+    """Algorithmic FLOPs of one AHLA forward (masks exploited, chunk C): per token-head
+    2 * [C d / 2 (Q K^T) + C dv / 2 (A V) + C dv / 2 (A R) + C / 2 (A 1, A s)
+         + 4 d dv (Q P_p, Q E_p, K^T V, K^T R) + 2 d (Q m_p, Q n_p) + d^2 dv / C (R^KQ P_p)]."""
+    C, d, dv = min(w.chunk, 64), w.d, w.dv
+    per = 2 * (C * d / 2 + C * dv + C / 2 + 4 * d * dv + 2 * d + d * d * dv / C)
+    return w.BH * w.n * per
+
+
+def ahla_dec_bytes(w):
+    """Algorithmic bytes of one AHLA decode step: read + write of (P, m, E, n) of every head plus token I/O."""
+    st = 2 * w.d * w.dv + 2 * w.d
+    s = 2 if w.dtype == "bf16" else 4
+    return w.BH * (2 * st * 4 + (2 * w.d + w.dv) * s + w.dv * s)
+
+
 def alu_peak():
     """fp32 CUDA-core peak: 152 SMs x 128 FP32 lanes x 2 FLOP x 2.07 GHz (maximum SM clock)."""
     return 152 * 128 * 2 * 2.07e9 / 1e12
@@ -279,7 +295,7 @@ def main():
     ap.add_argument("--workload", default="long_bf16_norm", choices=sorted(hla_inputs.WORKLOADS),
                     help="forward workload (default: the long-context one the metric is quoted on)")
     ap.add_argument("--n", type=int, default=0, help="override the sequence length (profiling runs)")
-    ap.add_argument("--only", default="", choices=["", "mid_bf16", "hla3_f32"],
+    ap.add_argument("--only", default="", choices=["", "mid_bf16", "hla3_f32", "ahla"],
                     help="time only this secondary workload (the d = 64 forward or third order) and print its object")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
@@ -298,6 +314,11 @@ def main():
     dev = torch.device("cuda", local)
     torch.cuda.set_device(dev)
     hbm_peak, tc_peak, peak_kind = peaks()
+    if args.only == "ahla":
+        res = bench_ahla(hla, dev, torch.cuda.current_stream(), hbm_peak, world)
+        if rank == 0:
+            print(json.dumps(res))
+        return
     if args.only:
         stream = torch.cuda.current_stream()
         res = bench_others(hla, dev, stream, hbm_peak, tc_peak, world, names=(args.only,),
@@ -453,6 +474,9 @@ def main():
     # ---------------- the other configs: d = 64 forward and third order ----------------
     if not args.no_decode:
         result["mid"], result["hla3"] = bench_others(hla, dev, stream, hbm_peak, tc_peak, world)
+        result["gpu_launches"] += result["mid"]["launches"] + result["hla3"]["launches"]
+        result["ahla"] = bench_ahla(hla, dev, stream, hbm_peak, world)
+        result["gpu_launches"] += result["ahla"]["forward"]["launches"] + result["ahla"]["decode"]["launches"]
     if rank == 0 and not args.no_cpu_baseline:
         result["cpu_baseline"] = cpu_baseline()
     if rank == 0:
@@ -510,6 +534,78 @@ def bench_others(hla, dev, stream, hbm_peak, tc_peak, world, names=("mid_bf16", 
             cfg["launches"] = steps
         res.append(cfg)
         del tq, tk, tv, out, ws
+    return res
+
+
+def bench_ahla(hla, dev, stream, hbm_peak, world, steps=20, warmup=3, decode_steps=256):
+    """AHLA: the forward on ahla_bf16 (B8 H16 n2048 d64 bf16, chunk 64) and the decode step on
+    ahla_decode_bf16 (B64 H32 d128, state built from a 4096-token prefix), CUDA events on the
+    launching stream."""
+    import torch
+    res = {}
+    w = hla_inputs.WORKLOADS["ahla_bf16"]
+    q, k, v = hla_inputs.make_workload(w)
+    tq, tk, tv = (hla_inputs.as_torch(x, w.dtype, dev) for x in (q, k, v))
+    out = torch.empty((w.B, w.H, w.n, w.dv), dtype=tq.dtype, device=dev)
+    ws = hla.alloc_workspace(hla.ahla_workspace_bytes(w.B, w.H, w.n, w.d, w.dv, w.chunk, tq.dtype), dev)
+
+    def call():
+        hla.ahla_forward(tq, tk, tv, out, normalized=w.normalized, eps=hla_inputs.EPS, chunk=w.chunk, workspace=ws,
+                         stream=stream)
+    for _ in range(warmup):
+        call()
+    torch.cuda.synchronize()
+    barrier(world)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(steps):
+        call()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = max_over_ranks(e0.elapsed_time(e1) / steps, world)
+    tf = ahla_flops(w) / (ms * 1e-3) / 1e12
+    gbs = fwd_bytes(w) / (ms * 1e-3) / 1e9
+    res["forward"] = {"workload": w.name, "B": w.B, "H": w.H, "n": w.n, "d": w.d, "dv": w.dv, "chunk": w.chunk,
+                      "tokens": w.dtype, "ms_per_step": ms, "value": w.B * w.n * world / (ms * 1e-3),
+                      "unit": "tokens/s", "steps": steps,
+                      "roofline": {"bound": "alu", "achieved": tf, "peak": alu_peak(), "unit": "TFLOP/s",
+                                   "frac": tf / alu_peak(), "traffic": None, "flops": ahla_flops(w),
+                                   "peak_kind": "derived (152 SMs x 128 fp32 lanes x 2 x 2.07 GHz)",
+                                   "kernel": "ahla_local/scan/out (fp32 CUDA cores)",
+                                   "hbm_view": {"achieved": gbs, "peak": hbm_peak, "unit": "GB/s",
+                                                "frac": gbs / hbm_peak}},
+                      "launches": 3 * steps}
+    del tq, tk, tv, out, ws
+    # decode step
+    w = hla_inputs.WORKLOADS["ahla_decode_bf16"]
+    (qp, kp, vp), (qs, ks, vs) = hla_inputs.make_decode(w, steps=decode_steps)
+    st = torch.zeros((w.B, w.H, hla.ahla_state_floats(w.d, w.dv)), dtype=torch.float32, device=dev)
+    tq, tk, tv = (hla_inputs.as_torch(x, w.dtype, dev) for x in (qp, kp, vp))
+    hla.ahla_forward(tq, tk, tv, chunk=w.chunk, state_out=st)
+    del tq, tk, tv, qp, kp, vp
+    toks = [[hla_inputs.as_torch(x[s], w.dtype, dev) for x in (qs, ks, vs)] for s in range(decode_steps)]
+    out = torch.empty((w.B, w.H, w.dv), dtype=toks[0][0].dtype, device=dev)
+    st0 = st.clone()
+    for s in range(min(3, decode_steps)):
+        hla.ahla_step(*toks[s], st, out, normalized=w.normalized, eps=hla_inputs.EPS)
+    st.copy_(st0)
+    del st0
+    torch.cuda.synchronize()
+    barrier(world)
+    e0.record(stream)
+    for s in range(decode_steps):
+        hla.ahla_step(*toks[s], st, out, normalized=w.normalized, eps=hla_inputs.EPS, stream=stream)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    us = max_over_ranks(e0.elapsed_time(e1) * 1e3 / decode_steps, world)
+    gbs = ahla_dec_bytes(w) / (us * 1e-6) / 1e9
+    res["decode"] = {"workload": w.name, "B": w.B, "H": w.H, "d": w.d, "dv": w.dv, "prefix": w.decode_prefix,
+                     "steps": decode_steps, "us_per_step": us, "value": gbs * world, "unit": "GB/s",
+                     "tokens_per_s": w.B * world / (us * 1e-6),
+                     "roofline": {"bound": "hbm", "achieved": gbs, "peak": hbm_peak, "unit": "GB/s",
+                                  "frac": gbs / hbm_peak, "traffic": None, "algorithmic_bytes": ahla_dec_bytes(w),
+                                  "kernel": "ahla_step_kernel"},
+                     "launches": decode_steps}
     return res
 
 

@@ -37,7 +37,7 @@ class Workload:
     masked: bool
     normalized: bool
     seed: int
-    order: int = 2      # 2 = second-order HLA, 3 = third-order HLA
+    order: int = 2      # 2 = second-order HLA, 3 = third-order HLA, 22 = asymmetric second order (AHLA)
     decode_prefix: int = 0
     decode_steps: int = 0
 
@@ -55,6 +55,11 @@ WORKLOADS = {
     "decode_bf16": Workload("decode_bf16", 64, 32, 0, 128, 128, 128, "bf16", True, False, 3,
                             decode_prefix=4096, decode_steps=256),
     "hla3_f32": Workload("hla3_f32", 4, 8, 4096, 32, 32, 32, "f32", True, False, 4, order=3),
+    # asymmetric second order (AHLA) at the shapes of the d = 64 forward, and its decode step at the
+    # shapes of the second-order decode workload
+    "ahla_bf16": Workload("ahla_bf16", 8, 16, 2048, 64, 64, 64, "bf16", True, False, 5, order=22),
+    "ahla_decode_bf16": Workload("ahla_decode_bf16", 64, 32, 0, 128, 128, 64, "bf16", True, False, 6, order=22,
+                                 decode_prefix=4096, decode_steps=256),
 }
 
 EPS = 1e-6  # the stability constant of the ratio-normalised output, used on both sides

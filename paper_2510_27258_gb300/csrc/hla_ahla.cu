@@ -1,0 +1,414 @@
+// Asymmetric second-order HLA (AHLA): chunk-parallel forward and decode step,
+// fp32 SIMT kernels (Sec. "Asymmetric Higher-order Linear Attention").
+//
+// AHLA is causal linear attention applied twice: with A = L . (Q K^T) (L lower
+// triangular incl. the diagonal), r_t = q_t^T P_t = (A V)_t and
+// o_t = q_t^T E_t = (A R)_t (Theorem AHLA: P_t = sum_{j<=t} k_j v_j^T,
+// E_t = sum_{i<=t} k_i r_i^T; denominators with v -> 1).  Per chunk, rows are
+// its tokens and "p" the carry-in prefix:
+//   R = A V + Q P_p,   s = A 1 + Q m_p,   O = A R + Q E_p,   den = A s + Q n_p.
+// Chunk summaries compose with Eq. AHLA-semidirect,
+//   E_AB = E_A + E_B + R^KQ_B P_A,  n_AB = n_A + n_B + R^KQ_B m_A,
+// with R^KQ = sum_i k_i q_i^T over the later chunk, so a chunk's local
+// summary (zero carry) is R^KQ = K^T Q, P = K^T V, m = K^T 1, E = K^T (A V),
+// n = K^T (A 1).  Three launches: chunk-local summaries (all chunks in
+// parallel), the carry scan (sequential over chunks, parallel over column
+// blocks of [P | m] and [E | n]), outputs (all chunks in parallel).  The
+// chunk argument is the scan granularity; chunks are at most 64 tokens here
+// (the result does not depend on it up to rounding).
+#include <algorithm>
+
+#include "hla_internal.h"
+
+namespace hla {
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int kCols = 32;  // columns of [P | m] / [E | n] per scan block
+
+struct ALayout {
+    int BH, n, d, dv, C, nch;
+    // local record per (head, chunk), floats: R^KQ d*d | P d*dv | m d | E d*dv | n d | Rloc C*dv | sloc C
+    long long oR, oP, om, oE, on, oRl, osl, rec_local;
+    // carry record per (head, chunk): P d*dv | m d | E d*dv | n d  (the state before the chunk)
+    long long rec_carry, carry_base;
+};
+
+inline long long up16(long long x) { return (x + 15) / 16 * 16; }
+
+ALayout make_layout(int BH, int n, int d, int dv, int chunk) {
+    ALayout L;
+    L.BH = BH; L.n = n; L.d = d; L.dv = dv;
+    L.C = std::min(chunk, 64);
+    L.nch = (n + L.C - 1) / L.C;
+    long long o = 0;
+    L.oR = o; o += up16((long long)d * d);
+    L.oP = o; o += up16((long long)d * dv);
+    L.om = o; o += up16(d);
+    L.oE = o; o += up16((long long)d * dv);
+    L.on = o; o += up16(d);
+    L.oRl = o; o += up16((long long)L.C * dv);
+    L.osl = o; o += up16(L.C);
+    L.rec_local = o;
+    L.rec_carry = up16(2LL * d * dv + 2LL * d);
+    L.carry_base = (long long)BH * L.nch * L.rec_local;
+    return L;
+}
+
+long long scratch_floats(const ALayout &L) { return L.carry_base + (long long)L.BH * L.nch * L.rec_carry; }
+
+__device__ __forceinline__ float *local_rec(float *ws, const ALayout &L, int hd, int c) {
+    return ws + ((long long)hd * L.nch + c) * L.rec_local;
+}
+__device__ __forceinline__ float *carry_rec(float *ws, const ALayout &L, int hd, int c) {
+    return ws + L.carry_base + ((long long)hd * L.nch + c) * L.rec_carry;
+}
+
+template <typename T>
+__device__ void load_tokens(const T *src, float *dst, int rows, int width, int Crows) {
+    for (int i = threadIdx.x; i < Crows * width; i += blockDim.x) dst[i] = i < rows * width ? to_f32(src[i]) : 0.f;
+}
+
+// ---------------------------------------------------------------------------
+// kernel 1: chunk-local summaries (zero carry)
+// ---------------------------------------------------------------------------
+template <typename T>
+__global__ void __launch_bounds__(kThreads) ahla_local_kernel(const T *__restrict__ q, const T *__restrict__ k,
+                                                              const T *__restrict__ v, float *ws, ALayout L) {
+    extern __shared__ float sm[];
+    const int c = blockIdx.x, hd = blockIdx.y, d = L.d, dv = L.dv, C = L.C;
+    const int t0 = c * C, len = min(C, L.n - t0);
+    float *Qs = sm, *Ks = Qs + C * d, *Vs = Ks + C * d, *As = Vs + C * dv, *Rs = As + C * C, *ss = Rs + C * dv;
+    load_tokens(q + ((long long)hd * L.n + t0) * d, Qs, len, d, C);
+    load_tokens(k + ((long long)hd * L.n + t0) * d, Ks, len, d, C);
+    load_tokens(v + ((long long)hd * L.n + t0) * dv, Vs, len, dv, C);
+    __syncthreads();
+    // A_ti = q_t . k_i for i <= t
+    for (int idx = threadIdx.x; idx < C * C; idx += blockDim.x) {
+        const int t = idx / C, i = idx % C;
+        float s = 0.f;
+        if (i <= t)
+            for (int f = 0; f < d; ++f) s += Qs[t * d + f] * Ks[i * d + f];
+        As[idx] = s;
+    }
+    __syncthreads();
+    // R_loc = A V, s_loc = A 1
+    float *rec = local_rec(ws, L, hd, c);
+    for (int idx = threadIdx.x; idx < C * (dv + 1); idx += blockDim.x) {
+        const int t = idx / (dv + 1), col = idx % (dv + 1);
+        float s = 0.f;
+        for (int i = 0; i <= t; ++i) s += As[t * C + i] * (col < dv ? Vs[i * dv + col] : 1.f);
+        if (col < dv) {
+            Rs[t * dv + col] = s;
+            rec[L.oRl + t * dv + col] = s;
+        } else {
+            ss[t] = s;
+            rec[L.osl + t] = s;
+        }
+    }
+    __syncthreads();
+    // R^KQ = K^T Q, P = K^T V, m = K^T 1, E = K^T R_loc, n = K^T s_loc
+    for (int idx = threadIdx.x; idx < d * d; idx += blockDim.x) {
+        const int a = idx / d, b = idx % d;
+        float s = 0.f;
+        for (int t = 0; t < len; ++t) s += Ks[t * d + a] * Qs[t * d + b];
+        rec[L.oR + idx] = s;
+    }
+    for (int idx = threadIdx.x; idx < d * (dv + 1); idx += blockDim.x) {
+        const int a = idx / (dv + 1), col = idx % (dv + 1);
+        float sp = 0.f, se = 0.f;
+        for (int t = 0; t < len; ++t) {
+            const float kt = Ks[t * d + a];
+            sp += kt * (col < dv ? Vs[t * dv + col] : 1.f);
+            se += kt * (col < dv ? Rs[t * dv + col] : ss[t]);
+        }
+        if (col < dv) {
+            rec[L.oP + a * dv + col] = sp;
+            rec[L.oE + a * dv + col] = se;
+        } else {
+            rec[L.om + a] = sp;
+            rec[L.on + a] = se;
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------
+// kernel 2: carry scan.  Block (column block, head) keeps columns [j0, j0 + 32) of
+// the augmented P' = [P | m] and E' = [E | n] (d x (dv + 1)); for every chunk it
+// records the carry-in, then E' += E'_c + R^KQ_c P'  (old P') and P' += P'_c.
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(kThreads) ahla_scan_kernel(float *ws, ALayout L, const float *state_in,
+                                                             float *state_out) {
+    extern __shared__ float sm[];
+    const int hd = blockIdx.y, d = L.d, dv = L.dv, j0 = blockIdx.x * kCols;
+    float *Pp = sm, *Ep = Pp + d * kCols, *Rq = Ep + d * kCols;  // d x 32, d x 32, d x d
+    const int ncol = min(kCols, dv + 1 - j0);
+    const long long st_len = 2LL * d * dv + 2LL * d;
+    auto P_at = [&](const float *base, int a, int j) { return j < dv ? base[a * dv + j] : base[(long long)d * dv + a]; };
+    // base layout of a state / carry record: P d*dv | m d | E d*dv | n d
+    const float *sin = state_in ? state_in + hd * st_len : nullptr;
+    for (int idx = threadIdx.x; idx < d * kCols; idx += blockDim.x) {
+        const int a = idx / kCols, j = idx % kCols;
+        const bool ok = j < ncol;
+        Pp[idx] = (ok && sin) ? P_at(sin, a, j0 + j) : 0.f;
+        Ep[idx] = (ok && sin) ? P_at(sin + (long long)d * dv + d, a, j0 + j) : 0.f;
+    }
+    __syncthreads();
+    for (int c = 0; c < L.nch; ++c) {
+        float *cr = carry_rec(ws, L, hd, c);
+        const float *lr = local_rec(ws, L, hd, c);
+        for (int idx = threadIdx.x; idx < d * ncol; idx += blockDim.x) {
+            const int a = idx / ncol, j = idx % ncol, col = j0 + j;
+            if (col < dv) {
+                cr[a * dv + col] = Pp[a * kCols + j];
+                cr[(long long)d * dv + d + a * dv + col] = Ep[a * kCols + j];
+            } else {
+                cr[(long long)d * dv + a] = Pp[a * kCols + j];
+                cr[2LL * d * dv + d + a] = Ep[a * kCols + j];
+            }
+        }
+        for (int idx = threadIdx.x; idx < d * d; idx += blockDim.x) Rq[idx] = lr[L.oR + idx];
+        __syncthreads();
+        // E' += E'_c + R^KQ_c P' (each thread owns elements (a, j); P' is read before it changes)
+        float newE[128 * kCols / kThreads], newP[128 * kCols / kThreads];
+        int cnt = 0;
+        for (int idx = threadIdx.x; idx < d * kCols; idx += blockDim.x, ++cnt) {
+            const int a = idx / kCols, j = idx % kCols;
+            float e = Ep[idx], p = Pp[idx];
+            if (j < ncol) {
+                float s = 0.f;
+                for (int b = 0; b < d; ++b) s += Rq[a * d + b] * Pp[b * kCols + j];
+                const int col = j0 + j;
+                e += s + (col < dv ? lr[L.oE + a * dv + col] : lr[L.on + a]);
+                p += col < dv ? lr[L.oP + a * dv + col] : lr[L.om + a];
+            }
+            newE[cnt] = e;
+            newP[cnt] = p;
+        }
+        __syncthreads();  // every P' read before it is updated
+        cnt = 0;
+        for (int idx = threadIdx.x; idx < d * kCols; idx += blockDim.x, ++cnt) {
+            Ep[idx] = newE[cnt];
+            Pp[idx] = newP[cnt];
+        }
+        __syncthreads();
+    }
+    if (state_out) {
+        float *so = state_out + hd * st_len;
+        for (int idx = threadIdx.x; idx < d * ncol; idx += blockDim.x) {
+            const int a = idx / ncol, j = idx % ncol, col = j0 + j;
+            if (col < dv) {
+                so[a * dv + col] = Pp[a * kCols + j];
+                so[(long long)d * dv + d + a * dv + col] = Ep[a * kCols + j];
+            } else {
+                so[(long long)d * dv + a] = Pp[a * kCols + j];
+                so[2LL * d * dv + d + a] = Ep[a * kCols + j];
+            }
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------
+// kernel 3: outputs.  R = R_loc + Q P_p, s = s_loc + Q m_p, O = A R + Q E_p,
+// den = A s + Q n_p.
+// ---------------------------------------------------------------------------
+template <typename T>
+__global__ void __launch_bounds__(kThreads) ahla_out_kernel(const T *__restrict__ q, const T *__restrict__ k,
+                                                            T *__restrict__ out, float *ws, ALayout L, int normalized,
+                                                            float eps) {
+    extern __shared__ float sm[];
+    const int c = blockIdx.x, hd = blockIdx.y, d = L.d, dv = L.dv, C = L.C;
+    const int t0 = c * C, len = min(C, L.n - t0);
+    float *Qs = sm, *Ks = Qs + C * d, *Rs = Ks + C * d, *As = Rs + C * (dv + 1);  // Rs: C x (dv + 1), col dv = s
+    load_tokens(q + ((long long)hd * L.n + t0) * d, Qs, len, d, C);
+    load_tokens(k + ((long long)hd * L.n + t0) * d, Ks, len, d, C);
+    const float *lr = local_rec(ws, L, hd, c), *cr = carry_rec(ws, L, hd, c);
+    const float *Pp = cr, *mp = cr + (long long)d * dv, *Ep = mp + d, *np = Ep + (long long)d * dv;
+    __syncthreads();
+    for (int idx = threadIdx.x; idx < C * (dv + 1); idx += blockDim.x) {
+        const int t = idx / (dv + 1), col = idx % (dv + 1);
+        float s = col < dv ? lr[L.oRl + t * dv + col] : lr[L.osl + t];
+        for (int f = 0; f < d; ++f) s += Qs[t * d + f] * (col < dv ? Pp[f * dv + col] : mp[f]);
+        Rs[idx] = s;
+    }
+    for (int idx = threadIdx.x; idx < C * C; idx += blockDim.x) {
+        const int t = idx / C, i = idx % C;
+        float s = 0.f;
+        if (i <= t)
+            for (int f = 0; f < d; ++f) s += Qs[t * d + f] * Ks[i * d + f];
+        As[idx] = s;
+    }
+    __syncthreads();
+    // den first (column dv), then the numerator columns; rows handled by warps
+    T *o = out + ((long long)hd * L.n + t0) * dv;
+    for (int t = threadIdx.x >> 5; t < len; t += kThreads / 32) {
+        const int lane = threadIdx.x & 31;
+        float den = 0.f;
+        if (normalized) {
+            float s = 0.f;
+            for (int i = lane; i <= t; i += 32) s += As[t * C + i] * Rs[i * (dv + 1) + dv];
+            for (int f = lane; f < d; f += 32) s += Qs[t * d + f] * np[f];
+#pragma unroll
+            for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
+            den = s;
+        }
+        for (int col = lane; col < dv; col += 32) {
+            float s = 0.f;
+            for (int i = 0; i <= t; ++i) s += As[t * C + i] * Rs[i * (dv + 1) + col];
+            for (int f = 0; f < d; ++f) s += Qs[t * d + f] * Ep[f * dv + col];
+            from_f32(&o[t * dv + col], normalized ? s / (den + eps) : s);
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------
+// decode step: P' = P + k v^T, m' = m + k, r = q^T P', s = q . m',
+// E' = E + k r^T, n' = n + s k, o = q^T E', den = q . n'.  One block per head;
+// P and E are read and written once with 16-byte accesses, consecutive threads
+// on consecutive column groups; every thread keeps one column group of the
+// column sums q^T P' (then q^T E'), combined across row groups in shared memory.
+// ---------------------------------------------------------------------------
+template <typename T>
+__global__ void __launch_bounds__(kThreads) ahla_step_kernel(const T *__restrict__ q, const T *__restrict__ k,
+                                                             const T *__restrict__ v, T *__restrict__ out,
+                                                             float *__restrict__ state, int d, int dv, int normalized,
+                                                             float eps) {
+    __shared__ float qs[128], ks[128], vs[128], rs[128], part[kThreads][4], red[kThreads / 32];
+    __shared__ float s_sc;
+    const int hd = blockIdx.x, tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+    float *P = state + (long long)hd * (2LL * d * dv + 2 * d), *m = P + (long long)d * dv, *E = m + d,
+          *nn = E + (long long)d * dv;
+    if (tid < d) {
+        qs[tid] = to_f32(q[(long long)hd * d + tid]);
+        ks[tid] = to_f32(k[(long long)hd * d + tid]);
+    }
+    if (tid < dv) vs[tid] = to_f32(v[(long long)hd * dv + tid]);
+    __syncthreads();
+    const int wv = dv >> 2, n4 = (d * dv) >> 2, c4 = (tid % wv) * 4;  // kThreads is a multiple of wv
+    // block sum of one value per thread (all threads call it)
+    auto block_sum = [&](float x) {
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+        if (lane == 0) red[wid] = x;
+        __syncthreads();
+        float t = 0.f;
+        for (int w = 0; w < kThreads / 32; ++w) t += red[w];
+        __syncthreads();
+        return t;
+    };
+    // ---- [P | m] ----
+    {
+        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+        float4 *P4 = reinterpret_cast<float4 *>(P);
+        const float v0 = vs[c4], v1 = vs[c4 + 1], v2 = vs[c4 + 2], v3 = vs[c4 + 3];
+        for (int f = tid; f < n4; f += kThreads) {
+            const int row = f / wv;
+            float4 p = P4[f];
+            const float kr = ks[row], qr = qs[row];
+            p.x += kr * v0; p.y += kr * v1; p.z += kr * v2; p.w += kr * v3;
+            P4[f] = p;
+            acc.x += qr * p.x; acc.y += qr * p.y; acc.z += qr * p.z; acc.w += qr * p.w;
+        }
+        part[tid][0] = acc.x; part[tid][1] = acc.y; part[tid][2] = acc.z; part[tid][3] = acc.w;
+        float sm = 0.f;
+        if (tid < d) {
+            const float mv = m[tid] + ks[tid];
+            m[tid] = mv;
+            sm = qs[tid] * mv;
+        }
+        const float s_tot = block_sum(sm);  // s = q . m' (also orders part[] before the reads below)
+        if (tid < dv) {
+            const int grp = tid >> 2, comp = tid & 3;
+            float a = 0.f;
+            for (int g = grp; g < kThreads; g += wv) a += part[g][comp];
+            rs[tid] = a;  // r = q^T P'
+        }
+        if (tid == 0) s_sc = s_tot;
+        __syncthreads();
+    }
+    // ---- [E | n] ----
+    {
+        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+        float4 *E4 = reinterpret_cast<float4 *>(E);
+        const float r0 = rs[c4], r1 = rs[c4 + 1], r2 = rs[c4 + 2], r3 = rs[c4 + 3];
+        for (int f = tid; f < n4; f += kThreads) {
+            const int row = f / wv;
+            float4 e = E4[f];
+            const float kr = ks[row], qr = qs[row];
+            e.x += kr * r0; e.y += kr * r1; e.z += kr * r2; e.w += kr * r3;
+            E4[f] = e;
+            acc.x += qr * e.x; acc.y += qr * e.y; acc.z += qr * e.z; acc.w += qr * e.w;
+        }
+        part[tid][0] = acc.x; part[tid][1] = acc.y; part[tid][2] = acc.z; part[tid][3] = acc.w;
+        float sn = 0.f;
+        if (tid < d) {
+            const float nv = nn[tid] + s_sc * ks[tid];
+            nn[tid] = nv;
+            sn = qs[tid] * nv;
+        }
+        const float den = block_sum(sn);  // den = q . n'
+        if (tid < dv) {
+            const int grp = tid >> 2, comp = tid & 3;
+            float a = 0.f;
+            for (int g = grp; g < kThreads; g += wv) a += part[g][comp];
+            from_f32(&out[(long long)hd * dv + tid], normalized ? a / (den + eps) : a);
+        }
+    }
+}
+
+template <typename T>
+cudaError_t forward_t(const Fwd2 &p, cudaStream_t stream) {
+    const ALayout L = make_layout(p.BH, p.n, p.d, p.dv, p.chunk);
+    float *ws = reinterpret_cast<float *>(p.ws + kWsHeaderBytes);
+    const T *q = static_cast<const T *>(p.q), *k = static_cast<const T *>(p.k), *v = static_cast<const T *>(p.v);
+    cudaError_t e;
+    if (L.nch > 0) {
+        const size_t sm1 = sizeof(float) * ((size_t)L.C * (2 * L.d + 2 * L.dv) + (size_t)L.C * L.C + L.C);
+        if ((e = cudaFuncSetAttribute(ahla_local_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm1)))
+            return e;
+        ahla_local_kernel<T><<<dim3(L.nch, p.BH), kThreads, sm1, stream>>>(q, k, v, ws, L);
+        if ((e = cudaGetLastError())) return e;
+    }
+    const size_t sm2 = sizeof(float) * ((size_t)2 * p.d * kCols + (size_t)p.d * p.d);
+    if ((e = cudaFuncSetAttribute(ahla_scan_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm2))) return e;
+    ahla_scan_kernel<<<dim3((p.dv + 1 + kCols - 1) / kCols, p.BH), kThreads, sm2, stream>>>(ws, L, p.state_in,
+                                                                                            p.state_out);
+    if ((e = cudaGetLastError())) return e;
+    if (L.nch > 0) {
+        const size_t sm3 = sizeof(float) * ((size_t)L.C * (2 * L.d + L.dv + 1) + (size_t)L.C * L.C);
+        if ((e = cudaFuncSetAttribute(ahla_out_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm3)))
+            return e;
+        ahla_out_kernel<T><<<dim3(L.nch, p.BH), kThreads, sm3, stream>>>(q, k, static_cast<T *>(p.out), ws, L,
+                                                                         p.normalized, p.eps);
+        if ((e = cudaGetLastError())) return e;
+    }
+    return cudaSuccess;
+}
+
+}  // namespace
+
+size_t ahla_workspace_bytes_internal(int BH, int n, int d, int dv, int chunk) {
+    const ALayout L = make_layout(BH, n, d, dv, chunk);
+    return kWsHeaderBytes + sizeof(float) * (size_t)scratch_floats(L);
+}
+
+cudaError_t ahla_forward_launch(const Fwd2 &p, cudaStream_t stream) {
+    return p.dt == HLA_BF16 ? forward_t<__nv_bfloat16>(p, stream) : forward_t<float>(p, stream);
+}
+
+cudaError_t ahla_step_launch(const void *q, const void *k, const void *v, void *out, hla_dtype dt, int BH, int d,
+                             int dv, int normalized, float eps, float *state, cudaStream_t stream) {
+    if (BH == 0) return cudaSuccess;
+    if (dt == HLA_BF16)
+        ahla_step_kernel<__nv_bfloat16><<<BH, kThreads, 0, stream>>>(
+            static_cast<const __nv_bfloat16 *>(q), static_cast<const __nv_bfloat16 *>(k),
+            static_cast<const __nv_bfloat16 *>(v), static_cast<__nv_bfloat16 *>(out), state, d, dv, normalized, eps);
+    else
+        ahla_step_kernel<float><<<BH, kThreads, 0, stream>>>(static_cast<const float *>(q),
+                                                             static_cast<const float *>(k),
+                                                             static_cast<const float *>(v), static_cast<float *>(out),
+                                                             state, d, dv, normalized, eps);
+    return cudaGetLastError();
+}
+
+}  // namespace hla
