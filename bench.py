@@ -295,7 +295,7 @@ def main():
     ap.add_argument("--workload", default="long_bf16_norm", choices=sorted(hla_inputs.WORKLOADS),
                     help="forward workload (default: the long-context one the metric is quoted on)")
     ap.add_argument("--n", type=int, default=0, help="override the sequence length (profiling runs)")
-    ap.add_argument("--only", default="", choices=["", "mid_bf16", "hla3_f32", "ahla"],
+    ap.add_argument("--only", default="", choices=["", "mid_bf16", "hla3_f32", "ahla", "backward"],
                     help="time only this secondary workload (the d = 64 forward or third order) and print its object")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
@@ -314,8 +314,9 @@ def main():
     dev = torch.device("cuda", local)
     torch.cuda.set_device(dev)
     hbm_peak, tc_peak, peak_kind = peaks()
-    if args.only == "ahla":
-        res = bench_ahla(hla, dev, torch.cuda.current_stream(), hbm_peak, world)
+    if args.only in ("ahla", "backward"):
+        st = torch.cuda.current_stream()
+        res = bench_ahla(hla, dev, st, hbm_peak, world) if args.only == "ahla" else bench_backward(hla, dev, st, world)
         if rank == 0:
             print(json.dumps(res))
         return
@@ -477,6 +478,8 @@ def main():
         result["gpu_launches"] += result["mid"]["launches"] + result["hla3"]["launches"]
         result["ahla"] = bench_ahla(hla, dev, stream, hbm_peak, world)
         result["gpu_launches"] += result["ahla"]["forward"]["launches"] + result["ahla"]["decode"]["launches"]
+        result["backward"] = bench_backward(hla, dev, stream, world)
+        result["gpu_launches"] += result["backward"]["launches"]
     if rank == 0 and not args.no_cpu_baseline:
         result["cpu_baseline"] = cpu_baseline()
     if rank == 0:
@@ -535,6 +538,52 @@ def bench_others(hla, dev, stream, hbm_peak, tc_peak, world, names=("mid_bf16", 
         res.append(cfg)
         del tq, tk, tv, out, ws
     return res
+
+
+def bwd_flops(w):
+    """Algorithmic FLOPs of one masked second-order backward (chunk C, augmented width
+    W = dv + 1): the forward recompute (as fwd_flops) plus, per token-head,
+    2 [C W / 2 (P) + C d / 2 (P^T Q) + d W (V' Gam) + C d / 2 (Y K^T) + C W / 2 (T^T G')
+       + d W (X Gam^T) + C d / 2 (P X) + 2 d W (G' D^T, Gam, M) + d^2 (Y S_p) + C d / 2 (B K)
+       + d^2 (K Lam) + C d (W^T Y, B^T Q) + 2 d^2 (Lam) + 2 d^2 W / C (scans)]."""
+    C, d, W = min(w.chunk, 32 if max(w.d, w.dv) == 128 else 64), w.d, w.dv + 1
+    per = 2 * (C * W / 2 + C * d / 2 + d * W + C * d / 2 + C * W / 2 + d * W + C * d / 2 + 2 * d * W + d * d
+               + C * d / 2 + d * d + C * d + 2 * d * d + 2 * d * d * W / C)
+    return fwd_flops(w) + w.BH * w.n * per
+
+
+def bench_backward(hla, dev, stream, world, steps=10, warmup=3):
+    """hla2_backward on mid_bf16 (B8 H16 n2048 d64 bf16, chunk 64), CUDA events on the launching stream."""
+    import torch
+    w = hla_inputs.WORKLOADS["mid_bf16"]
+    q, k, v = hla_inputs.make_workload(w)
+    g = hla_inputs.round_to(np.random.default_rng(w.seed + 1).standard_normal((w.B, w.H, w.n, w.dv)), w.dtype)
+    tq, tk, tv, tg = (hla_inputs.as_torch(x, w.dtype, dev) for x in (q, k, v, g))
+    ws = hla.alloc_workspace(hla.hla2_backward_workspace_bytes(w.B, w.H, w.n, w.d, w.dv, w.chunk, tq.dtype), dev)
+
+    def call():
+        hla.hla2_backward(tq, tk, tv, tg, normalized=w.normalized, eps=hla_inputs.EPS, chunk=w.chunk, workspace=ws,
+                          stream=stream)
+    for _ in range(warmup):
+        call()
+    torch.cuda.synchronize()
+    barrier(world)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(steps):
+        call()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = max_over_ranks(e0.elapsed_time(e1) / steps, world)
+    tf = bwd_flops(w) / (ms * 1e-3) / 1e12
+    return {"workload": w.name, "B": w.B, "H": w.H, "n": w.n, "d": w.d, "dv": w.dv, "chunk": w.chunk,
+            "tokens": w.dtype, "ms_per_step": ms, "value": w.B * w.n * world / (ms * 1e-3), "unit": "tokens/s",
+            "steps": steps,
+            "roofline": {"bound": "alu", "achieved": tf, "peak": alu_peak(), "unit": "TFLOP/s", "frac": tf / alu_peak(),
+                         "traffic": None, "flops": bwd_flops(w),
+                         "peak_kind": "derived (152 SMs x 128 fp32 lanes x 2 x 2.07 GHz)",
+                         "kernel": "bwd_fwd_local/fwd_scan/local1/scan/local2 (fp32 CUDA cores)"},
+            "launches": 5 * steps}
 
 
 def bench_ahla(hla, dev, stream, hbm_peak, world, steps=20, warmup=3, decode_steps=256):

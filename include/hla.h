@@ -122,6 +122,28 @@ hla_status hla2_step(const void *q, const void *k, const void *v, void *out, hla
                      int B, int H, int d, int dv, int masked, int normalized, float eps,
                      float *state, hla_stream_t stream);
 
+/* Bytes of scratch workspace hla2_backward needs (0 if unsupported). */
+size_t hla2_backward_workspace_bytes(int B, int H, int n, int d, int dv, int chunk, hla_dtype dt);
+
+/*
+ * hla2_backward -- gradients of the masked second-order forward (from a zero
+ * state) for L = sum_t dout_t . out_t: dq, dk, dv.  The paper's training
+ * route (Sec. "Chunk-parallel training via associative scans"): the forward
+ * prefixes are checkpointed at chunk boundaries and recomputed within a
+ * chunk, and the gradient suffixes are carried by a reverse scan with the
+ * adjoint of the semidirect product (Eq. semidirect); the result equals the
+ * gradients of the serial recurrence (Theorem 2 and the chain rule) up to
+ * rounding.  normalized selects out = num / (den + eps) (Eq. masked).
+ * q, k, v : device [B, H, n, d] / [B, H, n, d] / [B, H, n, dv] of type dt
+ * dout    : device [B, H, n, dv] of type dt (the gradient of the output)
+ * dq, dk  : device [B, H, n, d] of type dt (written); dv : [B, H, n, dv] (written)
+ * workspace : at least hla2_backward_workspace_bytes(...) bytes, 256-byte aligned.
+ * Errors as for hla2_forward.
+ */
+hla_status hla2_backward(const void *q, const void *k, const void *v, const void *dout, void *dq, void *dk,
+                         void *dv, hla_dtype dt, int B, int H, int n, int d, int dv_size, int normalized,
+                         float eps, int chunk, void *workspace, size_t workspace_bytes, hla_stream_t stream);
+
 /*
  * The (S, D, e) decode state of the masked operator (no counterpart printed in
  * the paper; it follows from Theorem 1 and Eq. semidirect).  With

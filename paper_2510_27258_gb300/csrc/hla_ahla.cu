@@ -14,8 +14,10 @@
 // n = K^T (A 1).  Three launches: chunk-local summaries (all chunks in
 // parallel), the carry scan (sequential over chunks, parallel over column
 // blocks of [P | m] and [E | n]), outputs (all chunks in parallel).  The
-// chunk argument is the scan granularity; chunks are at most 64 tokens here
-// (the result does not depend on it up to rounding).
+// chunk argument is the scan granularity; chunks are at most 64 tokens here,
+// 32 with a 128-wide head (the result does not depend on it up to rounding).
+// Token rows of K are staged with a stride of d + 1 floats, so that the lanes
+// of a warp, which take consecutive keys, read distinct banks.
 #include <algorithm>
 
 #include "hla_internal.h"
@@ -39,7 +41,7 @@ inline long long up16(long long x) { return (x + 15) / 16 * 16; }
 ALayout make_layout(int BH, int n, int d, int dv, int chunk) {
     ALayout L;
     L.BH = BH; L.n = n; L.d = d; L.dv = dv;
-    L.C = std::min(chunk, 64);
+    L.C = std::min(chunk, (d == 128 || dv == 128) ? 32 : 64);  // shared-memory staging of the output kernel
     L.nch = (n + L.C - 1) / L.C;
     long long o = 0;
     L.oR = o; o += up16((long long)d * d);
@@ -65,8 +67,11 @@ __device__ __forceinline__ float *carry_rec(float *ws, const ALayout &L, int hd,
 }
 
 template <typename T>
-__device__ void load_tokens(const T *src, float *dst, int rows, int width, int Crows) {
-    for (int i = threadIdx.x; i < Crows * width; i += blockDim.x) dst[i] = i < rows * width ? to_f32(src[i]) : 0.f;
+__device__ void load_tokens(const T *src, float *dst, int rows, int width, int Crows, int stride) {
+    for (int i = threadIdx.x; i < Crows * width; i += blockDim.x) {
+        const int r = i / width, c = i % width;
+        dst[r * stride + c] = i < rows * width ? to_f32(src[i]) : 0.f;
+    }
 }
 
 // ---------------------------------------------------------------------------
@@ -78,17 +83,18 @@ __global__ void __launch_bounds__(kThreads) ahla_local_kernel(const T *__restric
     extern __shared__ float sm[];
     const int c = blockIdx.x, hd = blockIdx.y, d = L.d, dv = L.dv, C = L.C;
     const int t0 = c * C, len = min(C, L.n - t0);
-    float *Qs = sm, *Ks = Qs + C * d, *Vs = Ks + C * d, *As = Vs + C * dv, *Rs = As + C * C, *ss = Rs + C * dv;
-    load_tokens(q + ((long long)hd * L.n + t0) * d, Qs, len, d, C);
-    load_tokens(k + ((long long)hd * L.n + t0) * d, Ks, len, d, C);
-    load_tokens(v + ((long long)hd * L.n + t0) * dv, Vs, len, dv, C);
+    const int kd = d + 1;  // row stride of K in shared memory
+    float *Qs = sm, *Ks = Qs + C * d, *Vs = Ks + C * kd, *As = Vs + C * dv, *Rs = As + C * C, *ss = Rs + C * dv;
+    load_tokens(q + ((long long)hd * L.n + t0) * d, Qs, len, d, C, d);
+    load_tokens(k + ((long long)hd * L.n + t0) * d, Ks, len, d, C, kd);
+    load_tokens(v + ((long long)hd * L.n + t0) * dv, Vs, len, dv, C, dv);
     __syncthreads();
     // A_ti = q_t . k_i for i <= t
     for (int idx = threadIdx.x; idx < C * C; idx += blockDim.x) {
         const int t = idx / C, i = idx % C;
         float s = 0.f;
         if (i <= t)
-            for (int f = 0; f < d; ++f) s += Qs[t * d + f] * Ks[i * d + f];
+            for (int f = 0; f < d; ++f) s += Qs[t * d + f] * Ks[i * kd + f];
         As[idx] = s;
     }
     __syncthreads();
@@ -111,14 +117,14 @@ __global__ void __launch_bounds__(kThreads) ahla_local_kernel(const T *__restric
     for (int idx = threadIdx.x; idx < d * d; idx += blockDim.x) {
         const int a = idx / d, b = idx % d;
         float s = 0.f;
-        for (int t = 0; t < len; ++t) s += Ks[t * d + a] * Qs[t * d + b];
+        for (int t = 0; t < len; ++t) s += Ks[t * kd + a] * Qs[t * d + b];
         rec[L.oR + idx] = s;
     }
     for (int idx = threadIdx.x; idx < d * (dv + 1); idx += blockDim.x) {
         const int a = idx / (dv + 1), col = idx % (dv + 1);
         float sp = 0.f, se = 0.f;
         for (int t = 0; t < len; ++t) {
-            const float kt = Ks[t * d + a];
+            const float kt = Ks[t * kd + a];
             sp += kt * (col < dv ? Vs[t * dv + col] : 1.f);
             se += kt * (col < dv ? Rs[t * dv + col] : ss[t]);
         }
@@ -219,23 +225,29 @@ __global__ void __launch_bounds__(kThreads) ahla_out_kernel(const T *__restrict_
     extern __shared__ float sm[];
     const int c = blockIdx.x, hd = blockIdx.y, d = L.d, dv = L.dv, C = L.C;
     const int t0 = c * C, len = min(C, L.n - t0);
-    float *Qs = sm, *Ks = Qs + C * d, *Rs = Ks + C * d, *As = Rs + C * (dv + 1);  // Rs: C x (dv + 1), col dv = s
-    load_tokens(q + ((long long)hd * L.n + t0) * d, Qs, len, d, C);
-    load_tokens(k + ((long long)hd * L.n + t0) * d, Ks, len, d, C);
+    const int kd = d + 1, w1 = dv + 1;
+    // Rs: C x (dv + 1), column dv = s; Ps = [P_p | m_p], Es = [E_p | n_p]: d x (dv + 1)
+    float *Qs = sm, *Ks = Qs + C * d, *Rs = Ks + C * kd, *As = Rs + C * w1, *Ps = As + C * C, *Es = Ps + d * w1;
+    load_tokens(q + ((long long)hd * L.n + t0) * d, Qs, len, d, C, d);
+    load_tokens(k + ((long long)hd * L.n + t0) * d, Ks, len, d, C, kd);
     const float *lr = local_rec(ws, L, hd, c), *cr = carry_rec(ws, L, hd, c);
-    const float *Pp = cr, *mp = cr + (long long)d * dv, *Ep = mp + d, *np = Ep + (long long)d * dv;
+    for (int idx = threadIdx.x; idx < d * w1; idx += blockDim.x) {
+        const int f = idx / w1, col = idx % w1;
+        Ps[idx] = col < dv ? cr[f * dv + col] : cr[(long long)d * dv + f];
+        Es[idx] = col < dv ? cr[(long long)d * dv + d + f * dv + col] : cr[2LL * d * dv + d + f];
+    }
     __syncthreads();
-    for (int idx = threadIdx.x; idx < C * (dv + 1); idx += blockDim.x) {
-        const int t = idx / (dv + 1), col = idx % (dv + 1);
+    for (int idx = threadIdx.x; idx < C * w1; idx += blockDim.x) {
+        const int t = idx / w1, col = idx % w1;
         float s = col < dv ? lr[L.oRl + t * dv + col] : lr[L.osl + t];
-        for (int f = 0; f < d; ++f) s += Qs[t * d + f] * (col < dv ? Pp[f * dv + col] : mp[f]);
+        for (int f = 0; f < d; ++f) s += Qs[t * d + f] * Ps[f * w1 + col];
         Rs[idx] = s;
     }
     for (int idx = threadIdx.x; idx < C * C; idx += blockDim.x) {
         const int t = idx / C, i = idx % C;
         float s = 0.f;
         if (i <= t)
-            for (int f = 0; f < d; ++f) s += Qs[t * d + f] * Ks[i * d + f];
+            for (int f = 0; f < d; ++f) s += Qs[t * d + f] * Ks[i * kd + f];
         As[idx] = s;
     }
     __syncthreads();
@@ -246,16 +258,16 @@ __global__ void __launch_bounds__(kThreads) ahla_out_kernel(const T *__restrict_
         float den = 0.f;
         if (normalized) {
             float s = 0.f;
-            for (int i = lane; i <= t; i += 32) s += As[t * C + i] * Rs[i * (dv + 1) + dv];
-            for (int f = lane; f < d; f += 32) s += Qs[t * d + f] * np[f];
+            for (int i = lane; i <= t; i += 32) s += As[t * C + i] * Rs[i * w1 + dv];
+            for (int f = lane; f < d; f += 32) s += Qs[t * d + f] * Es[f * w1 + dv];
 #pragma unroll
             for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
             den = s;
         }
         for (int col = lane; col < dv; col += 32) {
             float s = 0.f;
-            for (int i = 0; i <= t; ++i) s += As[t * C + i] * Rs[i * (dv + 1) + col];
-            for (int f = 0; f < d; ++f) s += Qs[t * d + f] * Ep[f * dv + col];
+            for (int i = 0; i <= t; ++i) s += As[t * C + i] * Rs[i * w1 + col];
+            for (int f = 0; f < d; ++f) s += Qs[t * d + f] * Es[f * w1 + col];
             from_f32(&o[t * dv + col], normalized ? s / (den + eps) : s);
         }
     }
@@ -363,7 +375,7 @@ cudaError_t forward_t(const Fwd2 &p, cudaStream_t stream) {
     const T *q = static_cast<const T *>(p.q), *k = static_cast<const T *>(p.k), *v = static_cast<const T *>(p.v);
     cudaError_t e;
     if (L.nch > 0) {
-        const size_t sm1 = sizeof(float) * ((size_t)L.C * (2 * L.d + 2 * L.dv) + (size_t)L.C * L.C + L.C);
+        const size_t sm1 = sizeof(float) * ((size_t)L.C * (2 * L.d + 1 + 2 * L.dv) + (size_t)L.C * L.C + L.C);
         if ((e = cudaFuncSetAttribute(ahla_local_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm1)))
             return e;
         ahla_local_kernel<T><<<dim3(L.nch, p.BH), kThreads, sm1, stream>>>(q, k, v, ws, L);
@@ -375,7 +387,8 @@ cudaError_t forward_t(const Fwd2 &p, cudaStream_t stream) {
                                                                                             p.state_out);
     if ((e = cudaGetLastError())) return e;
     if (L.nch > 0) {
-        const size_t sm3 = sizeof(float) * ((size_t)L.C * (2 * L.d + L.dv + 1) + (size_t)L.C * L.C);
+        const size_t sm3 = sizeof(float) * ((size_t)L.C * (2 * L.d + 1 + L.dv + 1) + (size_t)L.C * L.C +
+                                            2 * (size_t)L.d * (L.dv + 1));
         if ((e = cudaFuncSetAttribute(ahla_out_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm3)))
             return e;
         ahla_out_kernel<T><<<dim3(L.nch, p.BH), kThreads, sm3, stream>>>(q, k, static_cast<T *>(p.out), ws, L,

@@ -210,6 +210,34 @@ hla_status hla2_step_sde(const void *q, const void *k, const void *v, void *out,
                        "decode step (S, D, e)");
 }
 
+size_t hla2_backward_workspace_bytes(int B, int H, int n, int d, int dv, int chunk, hla_dtype dt) {
+    if (B < 0 || H < 0 || n < 0 || !dim_ok(d) || !dim_ok(dv) || chunk < 1 || chunk > 128) return 0;
+    if (dt != HLA_F32 && dt != HLA_BF16) return 0;
+    return align_up(backward2_workspace_bytes(B * H, n, d, dv, chunk), 256);
+}
+
+hla_status hla2_backward(const void *q, const void *k, const void *v, const void *dout, void *dq, void *dk, void *dv_,
+                         hla_dtype dt, int B, int H, int n, int d, int dv, int normalized, float eps, int chunk,
+                         void *workspace, size_t workspace_bytes, hla_stream_t stream) {
+    g_last_error[0] = 0;
+    hla_status st = check_forward(q, k, v, dv_, dt, B, H, n, d, dv, 1, normalized, eps, chunk, nullptr, nullptr);
+    if (st != HLA_OK) return st;
+    const long long tokens = (long long)B * H * n;
+    if (tokens > 0 && (!dout || !dq || !dk)) return fail(HLA_ERR_INVALID_ARGUMENT, "null dout/dq/dk pointer");
+    if (!aligned16(dout) || !aligned16(dq) || !aligned16(dk))
+        return fail(HLA_ERR_INVALID_ARGUMENT, "dout, dq, dk and dv must be 16-byte aligned");
+    const size_t need = hla2_backward_workspace_bytes(B, H, n, d, dv, chunk, dt);
+    if (!workspace || workspace_bytes < need)
+        return fail(HLA_ERR_WORKSPACE, "workspace of %zu bytes needed, %zu given", need,
+                    workspace ? workspace_bytes : (size_t)0);
+    if ((reinterpret_cast<uintptr_t>(workspace) & 255u) != 0)
+        return fail(HLA_ERR_INVALID_ARGUMENT, "workspace must be 256-byte aligned");
+    if (tokens == 0) return HLA_OK;
+    Bwd2 p{q, k, v, dout, dq, dk, dv_, dt, B * H, n, d, dv, normalized, eps, chunk, static_cast<char *>(workspace),
+           workspace_bytes};
+    return cuda_status(backward2_launch(p, reinterpret_cast<cudaStream_t>(stream)), "backward");
+}
+
 size_t ahla_state_floats(int d, int dv) {
     if (d <= 0 || dv <= 0) return 0;
     return 2 * (size_t)d * dv + 2 * (size_t)d;

@@ -78,6 +78,20 @@ cudaError_t step2_sde_launch(const void *q, const void *k, const void *v, void *
                              int dv, int normalized, float eps, float *state, cudaStream_t stream);
 cudaError_t state_to_sde_launch(const float *src, float *dst, int BH, int d, int dv, cudaStream_t stream);
 
+// gradients of masked second order (reverse chunk scan)
+struct Bwd2 {
+    const void *q, *k, *v, *dout;
+    void *dq, *dk, *dval;
+    hla_dtype dt;
+    int BH, n, d, dv, normalized;
+    float eps;
+    int chunk;
+    char *ws;
+    size_t ws_bytes;
+};
+size_t backward2_workspace_bytes(int BH, int n, int d, int dv, int chunk);
+cudaError_t backward2_launch(const Bwd2 &p, cudaStream_t stream);
+
 // AHLA (asymmetric second order): chunk-parallel forward and decode step
 size_t ahla_workspace_bytes_internal(int BH, int n, int d, int dv, int chunk);
 cudaError_t ahla_forward_launch(const Fwd2 &p, cudaStream_t stream);

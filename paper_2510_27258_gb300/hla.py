@@ -24,7 +24,7 @@ EXPORTS = ("hla_status_string", "hla_last_error", "hla2_state_floats", "hla2_wor
            "hla2_forward_path", "hla2_step", "hla3_state_floats", "hla3_workspace_bytes", "hla3_forward",
            "hla2_forward_noalloc", "hla_poll_error_noalloc", "hla_poll_error", "hla2_sde_state_floats",
            "hla2_state_to_sde", "hla2_step_sde", "ahla_state_floats", "ahla_workspace_bytes", "ahla_forward",
-           "ahla_step")
+           "ahla_step", "hla2_backward_workspace_bytes", "hla2_backward")
 
 _lib = None
 
@@ -58,7 +58,10 @@ def lib():
         L.ahla_forward.restype = i
         L.ahla_step.argtypes = [vp, vp, vp, vp, i, i, i, i, i, i, f, vp, vp]
         L.ahla_step.restype = i
-        for name in ("hla2_workspace_bytes", "hla3_workspace_bytes", "ahla_workspace_bytes"):
+        L.hla2_backward.argtypes = [vp, vp, vp, vp, vp, vp, vp, i, i, i, i, i, i, i, f, i, vp, sz, vp]
+        L.hla2_backward.restype = i
+        for name in ("hla2_workspace_bytes", "hla3_workspace_bytes", "ahla_workspace_bytes",
+                     "hla2_backward_workspace_bytes"):
             getattr(L, name).argtypes = [i, i, i, i, i, i, i]
             getattr(L, name).restype = sz
         for name in ("hla2_forward", "hla3_forward"):
@@ -211,6 +214,30 @@ def hla2_step(q, k, v, state, out=None, *, masked=True, normalized=False, eps=1e
                            int(normalized), float(eps), _ptr(state), _stream(stream))
     _check(code, "hla2_step")
     return out
+
+
+def hla2_backward_workspace_bytes(B, H, n, d, dv, chunk, dtype) -> int:
+    code = dtype if isinstance(dtype, int) else (HLA_BF16 if dtype == torch.bfloat16 else HLA_F32)
+    return int(lib().hla2_backward_workspace_bytes(B, H, n, d, dv, chunk, code))
+
+
+def hla2_backward(q, k, v, dout, *, normalized=False, eps=1e-6, chunk=64, workspace=None, stream=None):
+    """Gradients (dq, dk, dv) of sum(dout * out) for the masked second-order forward
+    (include/hla.h: hla2_backward)."""
+    B, H, n, d = q.shape
+    dv = v.shape[-1]
+    for t in (q, k, v, dout):
+        if not t.is_cuda or not t.is_contiguous() or t.dtype != q.dtype:
+            raise ValueError("q, k, v, dout must be contiguous CUDA tensors of one dtype")
+    dt = _dtype_code(q)
+    gq, gk, gv = torch.empty_like(q), torch.empty_like(k), torch.empty_like(v)
+    if workspace is None:
+        workspace = alloc_workspace(hla2_backward_workspace_bytes(B, H, n, d, dv, chunk, dt), q.device)
+    code = lib().hla2_backward(_ptr(q), _ptr(k), _ptr(v), _ptr(dout), _ptr(gq), _ptr(gk), _ptr(gv), dt, B, H, n, d,
+                               dv, int(normalized), float(eps), int(chunk), _ptr(workspace),
+                               workspace.numel() * workspace.element_size(), _stream(stream))
+    _check(code, "hla2_backward")
+    return gq, gk, gv
 
 
 def ahla_state_floats(d: int, dv: int) -> int:
