@@ -200,15 +200,21 @@ class ClockSampler:
                 "reasons": reasons, "samples": len(rows)}
 
 
-def dist_setup(gpus):
+def dist_setup(gpus, backend=None):
+    """One process per GPU (torchrun sets RANK / LOCAL_RANK / WORLD_SIZE / MASTER_*): NCCL on GPUs,
+    gloo without one (the host-side logic of the replica mode, tested on CPU)."""
     import torch
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
     if world > 1:
         import torch.distributed as dist
-        torch.cuda.set_device(local)
-        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+        backend = backend or ("nccl" if torch.cuda.is_available() else "gloo")
+        if backend == "nccl":
+            torch.cuda.set_device(local)
+            dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+        else:
+            dist.init_process_group(backend)
     return rank, world, local
 
 
@@ -219,13 +225,21 @@ def barrier(world):
 
 
 def max_over_ranks(x, world):
+    """The largest of the ranks' values (the step time of a weak-scaling job is its slowest rank's)."""
     if world == 1:
         return x
     import torch
     import torch.distributed as dist
-    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
     return float(t.item())
+
+
+def weak_scaling_value(units_per_rank, world, ms):
+    """Whole-job throughput: every rank processes its own copy of the workload (heads are
+    independent), so the job processes world x units in the slowest rank's time."""
+    return units_per_rank * world / (ms * 1e-3)
 
 
 def cpu_baseline(budget_s=15.0):
@@ -394,7 +408,7 @@ def main():
     tokens = w.B * w.n  # sequence positions per forward (every head processed)
     if args.workload != "long_bf16_norm" or args.n > 0:
         args.no_cpu_baseline = True  # the CPU baseline samples the long workload only
-    value = tokens * world / (ms * 1e-3)
+    value = weak_scaling_value(tokens, world, ms)
     fwd_traffic, fwd_traffic_how = traffic("hla2_fused_kernel", w.name, w.n) if path == 1 else (None, None)
 
     # ---------------- end to end: pinned host buffers, copies inside the timed region ----------
