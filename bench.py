@@ -43,8 +43,12 @@ TRAFFIC = {
                           "n": 16384, "bytes": 526.6e6,
                           "how": "ncu capture at n=8192 (227.1 MB read + 36.2 MB written during the launch; outputs "
                                  "still dirty in L2 at its end are written later) scaled x2 to n=16384"},
-    "step2_kernel": {"src": ["hla_step.cu"], "sha256": "766bb0084dcd285e", "workload": "decode_bf16", "n": 0,
-                     "bytes": 751.2e6, "how": "ncu capture of one step (406.5 MB read + 344.7 MB written)"},
+    "step2_kernel": {"src": ["hla_step.cu"], "sha256": "5542daa4b35fe2f4", "workload": "decode_bf16", "n": 0,
+                     "bytes": 750.6e6, "how": "ncu capture of one step at B64 H32 d128 (bench.py --profile-case "
+                                              "tuple_step): 406.4 MB read + 344.2 MB written"},
+    "step2_kernel_sde": {"src": ["hla_step.cu"], "sha256": "5542daa4b35fe2f4", "workload": "decode_bf16", "n": 0,
+                         "bytes": 481.3e6, "how": "ncu capture of one step at B64 H32 d128 (bench.py --profile-case "
+                                                  "sde_step): 271.2 MB read + 210.1 MB written"},
 }
 
 
@@ -309,6 +313,9 @@ def main():
     ap.add_argument("--workload", default="long_bf16_norm", choices=sorted(hla_inputs.WORKLOADS),
                     help="forward workload (default: the long-context one the metric is quoted on)")
     ap.add_argument("--n", type=int, default=0, help="override the sequence length (profiling runs)")
+    ap.add_argument("--profile-case", default="", choices=["", "sde_step", "tuple_step", "ahla_step", "ahla_fwd",
+                                                             "backward"],
+                    help="run a few launches of one kernel family on a small case (for ncu captures) and exit")
     ap.add_argument("--only", default="", choices=["", "mid_bf16", "hla3_f32", "ahla", "backward"],
                     help="time only this secondary workload (the d = 64 forward or third order) and print its object")
     args = ap.parse_args()
@@ -328,6 +335,8 @@ def main():
     dev = torch.device("cuda", local)
     torch.cuda.set_device(dev)
     hbm_peak, tc_peak, peak_kind = peaks()
+    if args.profile_case:
+        return profile_case(hla, dev, args.profile_case)
     if args.only in ("ahla", "backward"):
         st = torch.cuda.current_stream()
         res = bench_ahla(hla, dev, st, hbm_peak, world) if args.only == "ahla" else bench_backward(hla, dev, st, world)
@@ -554,6 +563,36 @@ def bench_others(hla, dev, stream, hbm_peak, tc_peak, world, names=("mid_bf16", 
     return res
 
 
+def profile_case(hla, dev, case):
+    """A few launches of one kernel family on a case small enough for an ncu capture (state or
+    inputs of a few hundred MB, larger than L2): the decode steps on B64 H32 d128 states (random
+    values), the AHLA forward on ahla_bf16, the backward on mid_bf16."""
+    import torch
+    torch.manual_seed(0)
+    if case in ("sde_step", "tuple_step", "ahla_step"):
+        B, H, d, dv = 64, 32, 128, 128
+        q = (torch.randn(B, H, d, device=dev) / d ** 0.5).to(torch.bfloat16)
+        k = (torch.randn(B, H, d, device=dev) / d ** 0.5).to(torch.bfloat16)
+        v = torch.randn(B, H, dv, device=dev).to(torch.bfloat16)
+        floats = {"sde_step": hla.hla2_sde_state_floats, "tuple_step": hla.hla2_state_floats,
+                  "ahla_step": hla.ahla_state_floats}[case](d, dv)
+        st = torch.randn(B, H, floats, device=dev)
+        step = {"sde_step": lambda: hla.hla2_step_sde(q, k, v, st), "tuple_step": lambda: hla.hla2_step(q, k, v, st),
+                "ahla_step": lambda: hla.ahla_step(q, k, v, st)}[case]
+        for _ in range(4):
+            step()
+    else:
+        w = hla_inputs.WORKLOADS["ahla_bf16" if case == "ahla_fwd" else "mid_bf16"]
+        q, k, v = (hla_inputs.as_torch(x, w.dtype, dev) for x in hla_inputs.make_workload(w))
+        for _ in range(2):
+            if case == "ahla_fwd":
+                hla.ahla_forward(q, k, v, chunk=w.chunk)
+            else:
+                hla.hla2_backward(q, k, v, torch.randn_like(v), chunk=w.chunk)
+    torch.cuda.synchronize()
+    print(json.dumps({"profile_case": case, "ok": True}))
+
+
 def bwd_flops(w):
     """Algorithmic FLOPs of one masked second-order backward (chunk C, augmented width
     W = dv + 1): the forward recompute (as fwd_flops) plus, per token-head,
@@ -723,11 +762,12 @@ def bench_decode(hla, dev, stream, steps, hbm_peak, world):
     torch.cuda.synchronize()
     us2 = max_over_ranks(e0.elapsed_time(e1) * 1e3 / steps, world)
     gbs2 = dec_sde_bytes(w) / (us2 * 1e-6) / 1e9
+    sde_traffic, sde_how = traffic("step2_kernel_sde", "decode_bf16", 0)
     res["sde"] = {"state": "(S, D, e)", "us_per_step": us2, "value": gbs2 * world, "unit": "GB/s",
                   "tokens_per_s": w.B * world / (us2 * 1e-6),
                   "roofline": {"bound": "hbm", "achieved": gbs2, "peak": hbm_peak, "unit": "GB/s",
-                               "frac": gbs2 / hbm_peak, "traffic": None, "algorithmic_bytes": dec_sde_bytes(w),
-                               "kernel": "step2_kernel (S, D, e)"},
+                               "frac": gbs2 / hbm_peak, "traffic": sde_traffic, "traffic_how": sde_how,
+                               "algorithmic_bytes": dec_sde_bytes(w), "kernel": "step2_kernel (S, D, e)"},
                   "launches": steps}
     res["launches"] += steps
     return res

@@ -21,6 +21,7 @@
 #include <algorithm>
 
 #include "hla_internal.h"
+#include "simt_gemm.cuh"
 
 namespace hla {
 namespace {
@@ -83,59 +84,28 @@ __global__ void __launch_bounds__(kThreads) ahla_local_kernel(const T *__restric
     extern __shared__ float sm[];
     const int c = blockIdx.x, hd = blockIdx.y, d = L.d, dv = L.dv, C = L.C;
     const int t0 = c * C, len = min(C, L.n - t0);
-    const int kd = d + 1;  // row stride of K in shared memory
-    float *Qs = sm, *Ks = Qs + C * d, *Vs = Ks + C * kd, *As = Vs + C * dv, *Rs = As + C * C, *ss = Rs + C * dv;
+    const int kd = d + 1, w1 = dv + 1;  // row strides of K and of the augmented [V | 1], [R | s]
+    float *Qs = sm, *Ks = Qs + C * d, *Vs = Ks + C * kd, *As = Vs + C * w1, *Rs = As + C * C;
     load_tokens(q + ((long long)hd * L.n + t0) * d, Qs, len, d, C, d);
     load_tokens(k + ((long long)hd * L.n + t0) * d, Ks, len, d, C, kd);
-    load_tokens(v + ((long long)hd * L.n + t0) * dv, Vs, len, dv, C, dv);
+    load_tokens(v + ((long long)hd * L.n + t0) * dv, Vs, len, dv, C, w1);
+    for (int t = threadIdx.x; t < C; t += blockDim.x) Vs[t * w1 + dv] = t < len ? 1.f : 0.f;
     __syncthreads();
-    // A_ti = q_t . k_i for i <= t
-    for (int idx = threadIdx.x; idx < C * C; idx += blockDim.x) {
-        const int t = idx / C, i = idx % C;
-        float s = 0.f;
-        if (i <= t)
-            for (int f = 0; f < d; ++f) s += Qs[t * d + f] * Ks[i * kd + f];
-        As[idx] = s;
-    }
+    bgemm(As, C, Qs, d, 1, Ks, 1, kd, C, C, d, false, 1);          // A = L . Q K^T
     __syncthreads();
-    // R_loc = A V, s_loc = A 1
+    bgemm(Rs, w1, As, C, 1, Vs, w1, 1, C, w1, C, false, 0, 1);     // [R_loc | s_loc] = A [V | 1]
+    __syncthreads();
     float *rec = local_rec(ws, L, hd, c);
-    for (int idx = threadIdx.x; idx < C * (dv + 1); idx += blockDim.x) {
-        const int t = idx / (dv + 1), col = idx % (dv + 1);
-        float s = 0.f;
-        for (int i = 0; i <= t; ++i) s += As[t * C + i] * (col < dv ? Vs[i * dv + col] : 1.f);
-        if (col < dv) {
-            Rs[t * dv + col] = s;
-            rec[L.oRl + t * dv + col] = s;
-        } else {
-            ss[t] = s;
-            rec[L.osl + t] = s;
-        }
+    for (int idx = threadIdx.x; idx < C * w1; idx += blockDim.x) {
+        const int t = idx / w1, col = idx % w1;
+        if (col < dv) rec[L.oRl + t * dv + col] = Rs[idx];
+        else rec[L.osl + t] = Rs[idx];
     }
-    __syncthreads();
-    // R^KQ = K^T Q, P = K^T V, m = K^T 1, E = K^T R_loc, n = K^T s_loc
-    for (int idx = threadIdx.x; idx < d * d; idx += blockDim.x) {
-        const int a = idx / d, b = idx % d;
-        float s = 0.f;
-        for (int t = 0; t < len; ++t) s += Ks[t * kd + a] * Qs[t * d + b];
-        rec[L.oR + idx] = s;
-    }
-    for (int idx = threadIdx.x; idx < d * (dv + 1); idx += blockDim.x) {
-        const int a = idx / (dv + 1), col = idx % (dv + 1);
-        float sp = 0.f, se = 0.f;
-        for (int t = 0; t < len; ++t) {
-            const float kt = Ks[t * kd + a];
-            sp += kt * (col < dv ? Vs[t * dv + col] : 1.f);
-            se += kt * (col < dv ? Rs[t * dv + col] : ss[t]);
-        }
-        if (col < dv) {
-            rec[L.oP + a * dv + col] = sp;
-            rec[L.oE + a * dv + col] = se;
-        } else {
-            rec[L.om + a] = sp;
-            rec[L.on + a] = se;
-        }
-    }
+    bgemm(rec + L.oR, d, Ks, 1, kd, Qs, d, 1, d, d, C, false);      // R^KQ = K^T Q
+    bgemm(rec + L.oP, dv, Ks, 1, kd, Vs, w1, 1, d, dv, C, false);   // P = K^T V
+    bgemm(rec + L.om, 1, Ks, 1, kd, Vs + dv, w1, 1, d, 1, C, false); // m = K^T 1
+    bgemm(rec + L.oE, dv, Ks, 1, kd, Rs, w1, 1, d, dv, C, false);   // E = K^T R_loc
+    bgemm(rec + L.on, 1, Ks, 1, kd, Rs + dv, w1, 1, d, 1, C, false); // n = K^T s_loc
 }
 
 // ---------------------------------------------------------------------------
@@ -226,8 +196,11 @@ __global__ void __launch_bounds__(kThreads) ahla_out_kernel(const T *__restrict_
     const int c = blockIdx.x, hd = blockIdx.y, d = L.d, dv = L.dv, C = L.C;
     const int t0 = c * C, len = min(C, L.n - t0);
     const int kd = d + 1, w1 = dv + 1;
-    // Rs: C x (dv + 1), column dv = s; Ps = [P_p | m_p], Es = [E_p | n_p]: d x (dv + 1)
-    float *Qs = sm, *Ks = Qs + C * d, *Rs = Ks + C * kd, *As = Rs + C * w1, *Ps = As + C * C, *Es = Ps + d * w1;
+    // Rs = [R | s] and Os = [O | den] (C x (dv + 1)); Ps = [P_p | m_p], Es = [E_p | n_p] (d x (dv + 1));
+    // Os takes the place of K, which is dead once A is formed
+    const int kw = kd > w1 ? kd : w1;
+    float *Qs = sm, *Ks = Qs + C * d, *Rs = Ks + C * kw, *As = Rs + C * w1, *Ps = As + C * C, *Es = Ps + d * w1;
+    float *Os = Ks;
     load_tokens(q + ((long long)hd * L.n + t0) * d, Qs, len, d, C, d);
     load_tokens(k + ((long long)hd * L.n + t0) * d, Ks, len, d, C, kd);
     const float *lr = local_rec(ws, L, hd, c), *cr = carry_rec(ws, L, hd, c);
@@ -236,40 +209,22 @@ __global__ void __launch_bounds__(kThreads) ahla_out_kernel(const T *__restrict_
         Ps[idx] = col < dv ? cr[f * dv + col] : cr[(long long)d * dv + f];
         Es[idx] = col < dv ? cr[(long long)d * dv + d + f * dv + col] : cr[2LL * d * dv + d + f];
     }
-    __syncthreads();
     for (int idx = threadIdx.x; idx < C * w1; idx += blockDim.x) {
         const int t = idx / w1, col = idx % w1;
-        float s = col < dv ? lr[L.oRl + t * dv + col] : lr[L.osl + t];
-        for (int f = 0; f < d; ++f) s += Qs[t * d + f] * Ps[f * w1 + col];
-        Rs[idx] = s;
-    }
-    for (int idx = threadIdx.x; idx < C * C; idx += blockDim.x) {
-        const int t = idx / C, i = idx % C;
-        float s = 0.f;
-        if (i <= t)
-            for (int f = 0; f < d; ++f) s += Qs[t * d + f] * Ks[i * kd + f];
-        As[idx] = s;
+        Rs[idx] = col < dv ? lr[L.oRl + t * dv + col] : lr[L.osl + t];
     }
     __syncthreads();
-    // den first (column dv), then the numerator columns; rows handled by warps
+    bgemm(Rs, w1, Qs, d, 1, Ps, w1, 1, C, w1, d, true);             // [R | s] += Q [P_p | m_p]
+    bgemm(As, C, Qs, d, 1, Ks, 1, kd, C, C, d, false, 1);           // A = L . Q K^T
+    __syncthreads();
+    bgemm(Os, w1, As, C, 1, Rs, w1, 1, C, w1, C, false, 0, 1);      // [O | den] = A [R | s]
+    bgemm(Os, w1, Qs, d, 1, Es, w1, 1, C, w1, d, true);             //   + Q [E_p | n_p]
+    __syncthreads();
     T *o = out + ((long long)hd * L.n + t0) * dv;
-    for (int t = threadIdx.x >> 5; t < len; t += kThreads / 32) {
-        const int lane = threadIdx.x & 31;
-        float den = 0.f;
-        if (normalized) {
-            float s = 0.f;
-            for (int i = lane; i <= t; i += 32) s += As[t * C + i] * Rs[i * w1 + dv];
-            for (int f = lane; f < d; f += 32) s += Qs[t * d + f] * Es[f * w1 + dv];
-#pragma unroll
-            for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
-            den = s;
-        }
-        for (int col = lane; col < dv; col += 32) {
-            float s = 0.f;
-            for (int i = 0; i <= t; ++i) s += As[t * C + i] * Rs[i * w1 + col];
-            for (int f = 0; f < d; ++f) s += Qs[t * d + f] * Es[f * w1 + col];
-            from_f32(&o[t * dv + col], normalized ? s / (den + eps) : s);
-        }
+    for (int idx = threadIdx.x; idx < len * dv; idx += blockDim.x) {
+        const int t = idx / dv, col = idx % dv;
+        const float x = Os[t * w1 + col];
+        from_f32(&o[idx], normalized ? x / (Os[t * w1 + dv] + eps) : x);
     }
 }
 
@@ -375,7 +330,7 @@ cudaError_t forward_t(const Fwd2 &p, cudaStream_t stream) {
     const T *q = static_cast<const T *>(p.q), *k = static_cast<const T *>(p.k), *v = static_cast<const T *>(p.v);
     cudaError_t e;
     if (L.nch > 0) {
-        const size_t sm1 = sizeof(float) * ((size_t)L.C * (2 * L.d + 1 + 2 * L.dv) + (size_t)L.C * L.C + L.C);
+        const size_t sm1 = sizeof(float) * ((size_t)L.C * (2 * L.d + 1 + 2 * (L.dv + 1)) + (size_t)L.C * L.C);
         if ((e = cudaFuncSetAttribute(ahla_local_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm1)))
             return e;
         ahla_local_kernel<T><<<dim3(L.nch, p.BH), kThreads, sm1, stream>>>(q, k, v, ws, L);
@@ -387,8 +342,8 @@ cudaError_t forward_t(const Fwd2 &p, cudaStream_t stream) {
                                                                                             p.state_out);
     if ((e = cudaGetLastError())) return e;
     if (L.nch > 0) {
-        const size_t sm3 = sizeof(float) * ((size_t)L.C * (2 * L.d + 1 + L.dv + 1) + (size_t)L.C * L.C +
-                                            2 * (size_t)L.d * (L.dv + 1));
+        const size_t sm3 = sizeof(float) * ((size_t)L.C * (L.d + std::max(L.d + 1, L.dv + 1) + L.dv + 1) +
+                                            (size_t)L.C * L.C + 2 * (size_t)L.d * (L.dv + 1));
         if ((e = cudaFuncSetAttribute(ahla_out_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm3)))
             return e;
         ahla_out_kernel<T><<<dim3(L.nch, p.BH), kThreads, sm3, stream>>>(q, k, static_cast<T *>(p.out), ws, L,

@@ -32,6 +32,7 @@
 #include <algorithm>
 
 #include "hla_internal.h"
+#include "simt_gemm.cuh"
 
 namespace hla {
 namespace {
@@ -42,9 +43,9 @@ constexpr int kCols = 32;
 struct BLayout {
     int BH, n, d, dv, W, C, nch;
     long long fl_S, fl_DL, fl_C, fl_len;            // forward local: S_c d*d | DL_c d*W | C_c d*W
-    long long fc_S, fc_D, fc_len;                   // forward carry: S_p d*d | D_p d*W
+    long long fc_S, fc_D, fc_DT, fc_len;            // forward carry: S_p d*d | D_p d*W | D_p^T W*d
     long long bl_G, bl_Gam, bl_M, bl_Lam, bl_len;   // backward local: G' C*W | Gam_c W*d | M_c W*d | Lam_c d*d
-    long long bc_Gam, bc_Lam, bc_len;               // backward carry: Gam_s W*d | Lam_s d*d
+    long long bc_Gam, bc_Lam, bc_GamT, bc_len;      // backward carry: Gam_s W*d | Lam_s d*d | Gam_s^T d*W
     long long o_fl, o_fc, o_bl, o_bc, total;        // floats from the scratch start
 };
 
@@ -57,10 +58,10 @@ BLayout make_layout(int BH, int n, int d, int dv, int chunk) {
     L.nch = (n + L.C - 1) / L.C;
     const long long dd = (long long)d * d, dW = (long long)d * L.W;
     L.fl_S = 0; L.fl_DL = up16(dd); L.fl_C = L.fl_DL + up16(dW); L.fl_len = L.fl_C + up16(dW);
-    L.fc_S = 0; L.fc_D = up16(dd); L.fc_len = L.fc_D + up16(dW);
+    L.fc_S = 0; L.fc_D = up16(dd); L.fc_DT = L.fc_D + up16(dW); L.fc_len = L.fc_DT + up16(dW);
     L.bl_G = 0; L.bl_Gam = up16((long long)L.C * L.W); L.bl_M = L.bl_Gam + up16(dW); L.bl_Lam = L.bl_M + up16(dW);
     L.bl_len = L.bl_Lam + up16(dd);
-    L.bc_Gam = 0; L.bc_Lam = up16(dW); L.bc_len = L.bc_Lam + up16(dd);
+    L.bc_Gam = 0; L.bc_Lam = up16(dW); L.bc_GamT = L.bc_Lam + up16(dd); L.bc_len = L.bc_GamT + up16(dW);
     const long long chunks = (long long)BH * L.nch;
     L.o_fl = 0;
     L.o_fc = L.o_fl + chunks * L.fl_len;
@@ -72,29 +73,6 @@ BLayout make_layout(int BH, int n, int d, int dv, int chunk) {
 
 __device__ __forceinline__ float *rec(float *ws, long long base, long long len, const BLayout &L, int hd, int c) {
     return ws + base + ((long long)hd * L.nch + c) * len;
-}
-
-// C[r][c] (+)= sum_k A(r, k) B(k, c) for r < M, c < N over the block's threads, with
-// A(r, k) = A[r * ar + k * ak], B(k, c) = B[k * bk + c * bc], C[r * ldc + c].
-// mask 1: only c <= r (others set to 0 unless accumulating); the k range may be cut to
-// [klo(r, c), khi(r, c)) by kmode: 0 all, 1 k <= r (A lower triangular by rows),
-// 2 k >= c (B lower triangular: B(k, c) = 0 for k < c), 3 k >= r (A(r,k) = 0 for k < r).
-__device__ void bgemm(float *Cm, int ldc, const float *A, int ar, int ak, const float *B, int bk, int bc, int M, int N,
-                      int K, bool accumulate, int mask = 0, int kmode = 0) {
-    for (int idx = threadIdx.x; idx < M * N; idx += blockDim.x) {
-        const int r = idx / N, c = idx % N;
-        if (mask == 1 && c > r) {
-            if (!accumulate) Cm[r * ldc + c] = 0.f;
-            continue;
-        }
-        int k0 = 0, k1 = K;
-        if (kmode == 1) k1 = min(K, r + 1);
-        else if (kmode == 2) k0 = c;
-        else if (kmode == 3) k0 = r;
-        float s = accumulate ? Cm[r * ldc + c] : 0.f;
-        for (int kk = k0; kk < k1; ++kk) s += A[r * ar + kk * ak] * B[kk * bk + c * bc];
-        Cm[r * ldc + c] = s;
-    }
 }
 
 // token rows of a chunk into shared memory (zero beyond the sequence); with ones, column
@@ -140,7 +118,8 @@ __global__ void __launch_bounds__(kThreads) bwd_fwd_local(const T *q, const T *k
 __global__ void __launch_bounds__(kThreads) bwd_fwd_scan(float *ws, BLayout L) {
     extern __shared__ float sm[];
     const int hd = blockIdx.y, d = L.d, W = L.W, j0 = blockIdx.x * kCols, ncol = min(kCols, W - j0);
-    float *Sp = sm, *Dp = Sp + d * d, *Dn = Dp + d * kCols;
+    // S_p (d x d), D_p columns (d x 32), the chunk's C_c and DL_c columns staged per chunk (d x 32 each)
+    float *Sp = sm, *Dp = Sp + d * d, *Cc = Dp + d * kCols, *DLc = Cc + d * kCols;
     for (int i = threadIdx.x; i < d * d; i += blockDim.x) Sp[i] = 0.f;
     for (int i = threadIdx.x; i < d * kCols; i += blockDim.x) Dp[i] = 0.f;
     __syncthreads();
@@ -149,19 +128,34 @@ __global__ void __launch_bounds__(kThreads) bwd_fwd_scan(float *ws, BLayout L) {
         const float *fl = rec(ws, L.o_fl, L.fl_len, L, hd, c);
         if (blockIdx.x == 0)
             for (int i = threadIdx.x; i < d * d; i += blockDim.x) fc[L.fc_S + i] = Sp[i];
-        for (int i = threadIdx.x; i < d * ncol; i += blockDim.x) {
-            const int a = i / ncol, j = i % ncol;
-            fc[L.fc_D + a * W + j0 + j] = Dp[a * kCols + j];
+        for (int i = threadIdx.x; i < d * kCols; i += blockDim.x) {
+            const int a = i / kCols, j = i % kCols;
+            if (j < ncol) {
+                fc[L.fc_D + a * W + j0 + j] = Dp[i];
+                Cc[i] = fl[L.fl_C + a * W + j0 + j];
+                DLc[i] = fl[L.fl_DL + a * W + j0 + j];
+            }
         }
-        // D_new = D_p + DL_c + S_p C_c (old S_p)
-        for (int i = threadIdx.x; i < d * ncol; i += blockDim.x) {
-            const int a = i / ncol, j = i % ncol;
-            float s = Dp[a * kCols + j] + fl[L.fl_DL + a * W + j0 + j];
-            for (int b = 0; b < d; ++b) s += Sp[a * d + b] * fl[L.fl_C + b * W + j0 + j];
-            Dn[a * kCols + j] = s;
+        for (int i = threadIdx.x; i < d * ncol; i += blockDim.x) {  // D_p^T, consecutive threads on consecutive a
+            const int j = i / d, a = i % d;
+            fc[L.fc_DT + (long long)(j0 + j) * d + a] = Dp[a * kCols + j];
         }
         __syncthreads();
-        for (int i = threadIdx.x; i < d * ncol; i += blockDim.x) Dp[(i / ncol) * kCols + i % ncol] = Dn[(i / ncol) * kCols + i % ncol];
+        // D_new = D_p + DL_c + S_p C_c (old S_p); each thread keeps its results in registers
+        float dn[128 * kCols / kThreads];
+        int cnt = 0;
+        for (int i = threadIdx.x; i < d * kCols; i += blockDim.x, ++cnt) {
+            const int a = i / kCols, j = i % kCols;
+            float x = 0.f;
+            if (j < ncol) {
+                x = Dp[i] + DLc[i];
+                for (int b = 0; b < d; ++b) x += Sp[a * d + b] * Cc[b * kCols + j];
+            }
+            dn[cnt] = x;
+        }
+        __syncthreads();
+        cnt = 0;
+        for (int i = threadIdx.x; i < d * kCols; i += blockDim.x, ++cnt) Dp[i] = dn[cnt];
         for (int i = threadIdx.x; i < d * d; i += blockDim.x) Sp[i] += fl[L.fl_S + i];
         __syncthreads();
     }
@@ -243,28 +237,41 @@ __global__ void __launch_bounds__(kThreads) bwd_local1(const T *q, const T *k, c
 __global__ void __launch_bounds__(kThreads) bwd_scan(float *ws, BLayout L) {
     extern __shared__ float sm[];
     const int hd = blockIdx.y, d = L.d, W = L.W, j0 = blockIdx.x * kCols, ncol = min(kCols, d - j0);
-    float *Gm = sm, *Lm = Gm + W * d, *Ln = Lm + d * kCols;
+    // Gam_s (W x d), Lam_s columns (d x 32), the chunk's M_c (W x d) staged per chunk
+    float *Gm = sm, *Lm = Gm + W * d, *Mc = Lm + d * kCols;
     for (int i = threadIdx.x; i < W * d; i += blockDim.x) Gm[i] = 0.f;
     for (int i = threadIdx.x; i < d * kCols; i += blockDim.x) Lm[i] = 0.f;
     __syncthreads();
     for (int c = L.nch - 1; c >= 0; --c) {
         float *bc = rec(ws, L.o_bc, L.bc_len, L, hd, c);
         const float *bl = rec(ws, L.o_bl, L.bl_len, L, hd, c);
-        if (blockIdx.x == 0)
+        if (blockIdx.x == 0) {
             for (int i = threadIdx.x; i < W * d; i += blockDim.x) bc[L.bc_Gam + i] = Gm[i];
+            for (int i = threadIdx.x; i < W * d; i += blockDim.x) {  // Gam_s^T, consecutive threads on consecutive w
+                const int f = i / W, w = i % W;
+                bc[L.bc_GamT + i] = Gm[w * d + f];
+            }
+        }
         for (int i = threadIdx.x; i < d * ncol; i += blockDim.x) {
             const int a = i / ncol, j = i % ncol;
             bc[L.bc_Lam + a * d + j0 + j] = Lm[a * kCols + j];
         }
-        for (int i = threadIdx.x; i < d * ncol; i += blockDim.x) {
-            const int a = i / ncol, j = i % ncol, b = j0 + j;
-            float s = Lm[a * kCols + j] + bl[L.bl_Lam + a * d + b];
-            for (int w = 0; w < W; ++w)
-                s += Gm[w * d + a] * bl[L.bl_M + w * d + b] + bl[L.bl_M + w * d + a] * Gm[w * d + b];
-            Ln[a * kCols + j] = s;
+        for (int i = threadIdx.x; i < W * d; i += blockDim.x) Mc[i] = bl[L.bl_M + i];
+        __syncthreads();
+        float ln[128 * kCols / kThreads];
+        int cnt = 0;
+        for (int i = threadIdx.x; i < d * kCols; i += blockDim.x, ++cnt) {
+            const int a = i / kCols, j = i % kCols, b = j0 + j;
+            float x = 0.f;
+            if (j < ncol) {
+                x = Lm[i] + bl[L.bl_Lam + a * d + b];
+                for (int w = 0; w < W; ++w) x += Gm[w * d + a] * Mc[w * d + b] + Mc[w * d + a] * Gm[w * d + b];
+            }
+            ln[cnt] = x;
         }
         __syncthreads();
-        for (int i = threadIdx.x; i < d * ncol; i += blockDim.x) Lm[(i / ncol) * kCols + i % ncol] = Ln[(i / ncol) * kCols + i % ncol];
+        cnt = 0;
+        for (int i = threadIdx.x; i < d * kCols; i += blockDim.x, ++cnt) Lm[i] = ln[cnt];
         for (int i = threadIdx.x; i < W * d; i += blockDim.x) Gm[i] += bl[L.bl_Gam + i];
         __syncthreads();
     }
@@ -297,14 +304,14 @@ __global__ void __launch_bounds__(kThreads) bwd_local2(const T *q, const T *k, c
     bgemm(Bs, C, Ys, d, 1, Ks, 1, kd, C, C, d, false, 1);         // B = L . Y K^T
     // dV' = T^T G' + X Gam_s^T   (columns < dv)
     bgemm(Os, W, Ts, 1, C, Gs, W, 1, C, W, C, false, 0, 3);
-    bgemm(Os, W, Xs, d, 1, bc + L.bc_Gam, 1, d, C, W, d, true);
+    bgemm(Os, W, Xs, d, 1, bc + L.bc_GamT, W, 1, C, W, d, true);
     __syncthreads();
     T *gv = dvo + ((long long)hd * L.n + t0) * dv;
     for (int i = threadIdx.x; i < len * dv; i += blockDim.x) from_f32(&gv[i], Os[(i / dv) * W + i % dv]);
     __syncthreads();
     // dQ = P X + G' D_p^T + Y S_p + B K
     bgemm(Os, d, Ps, C, 1, Xs, d, 1, C, d, C, false, 0, 1);
-    bgemm(Os, d, Gs, W, 1, fc + L.fc_D, 1, W, C, d, W, true);
+    bgemm(Os, d, Gs, W, 1, fc + L.fc_DT, d, 1, C, d, W, true);
     bgemm(Os, d, Ys, d, 1, fc + L.fc_S, d, 1, C, d, d, true);
     bgemm(Os, d, Bs, C, 1, Ks, kd, 1, C, d, C, true, 0, 1);
     __syncthreads();
@@ -335,7 +342,7 @@ cudaError_t backward_t(const Bwd2 &p, cudaStream_t s) {
     if ((e = cudaFuncSetAttribute(bwd_fwd_local<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm1))) return e;
     bwd_fwd_local<T><<<grid, kThreads, sm1, s>>>(q, k, v, ws, L);
     if ((e = cudaGetLastError())) return e;
-    const int sm2 = smem((size_t)d * d + 2 * (size_t)d * kCols);
+    const int sm2 = smem((size_t)d * d + 3 * (size_t)d * kCols);
     if ((e = cudaFuncSetAttribute(bwd_fwd_scan, cudaFuncAttributeMaxDynamicSharedMemorySize, sm2))) return e;
     bwd_fwd_scan<<<dim3((W + kCols - 1) / kCols, p.BH), kThreads, sm2, s>>>(ws, L);
     if ((e = cudaGetLastError())) return e;
@@ -344,7 +351,7 @@ cudaError_t backward_t(const Bwd2 &p, cudaStream_t s) {
     if ((e = cudaFuncSetAttribute(bwd_local1<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm3))) return e;
     bwd_local1<T><<<grid, kThreads, sm3, s>>>(q, k, v, g, ws, L, p.normalized, p.eps);
     if ((e = cudaGetLastError())) return e;
-    const int sm4 = smem((size_t)W * d + 2 * (size_t)d * kCols);
+    const int sm4 = smem(2 * (size_t)W * d + (size_t)d * kCols);
     if ((e = cudaFuncSetAttribute(bwd_scan, cudaFuncAttributeMaxDynamicSharedMemorySize, sm4))) return e;
     bwd_scan<<<dim3((d + kCols - 1) / kCols, p.BH), kThreads, sm4, s>>>(ws, L);
     if ((e = cudaGetLastError())) return e;
