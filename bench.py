@@ -465,6 +465,19 @@ def main():
     e2e_ms = max_over_ranks(e0.elapsed_time(e1) / e2e_steps, world)
     in_bytes = sum(t.numel() * t.element_size() for t in (hq, hk, hv))
     out_bytes = hout.numel() * hout.element_size()
+    # the host link alone: the same pinned buffers copied in (and the output back), 5 times each
+    link = {}
+    for name, copies, nbytes in (("h2d_gbs", [(d_, h_) for d_, h_ in zip(dins[0], (hq, hk, hv))], in_bytes),
+                                 ("d2h_gbs", [(hout, douts[0])], out_bytes)):
+        torch.cuda.synchronize()
+        e0.record(stream)
+        for _ in range(5):
+            for dst, src in copies:
+                dst.copy_(src, non_blocking=True)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        link[name] = nbytes * 5 / (e0.elapsed_time(e1) * 1e-3) / 1e9
+    link["how"] = "pinned host buffers of the e2e leg, one stream, 5 x the per-step bytes, CUDA events"
     del hq, hk, hv, hout, dins, douts
 
     result = {
@@ -484,7 +497,7 @@ def main():
         "median_flushed": {"ms": med_ms, "runs": len(per_ms), "value": tokens * world / (med_ms * 1e-3),
                            "how": "median of single launches, each after a 256 MB write that flushes L2"},
         "e2e": {"value": tokens * world / (e2e_ms * 1e-3), "unit": "tokens/s", "ms_per_step": e2e_ms,
-                "h2d_bytes_per_step": in_bytes, "d2h_bytes_per_step": out_bytes},
+                "h2d_bytes_per_step": in_bytes, "d2h_bytes_per_step": out_bytes, "host_link": link},
         "gpu_launches": launches_per_step * args.steps,
     }
     del tq, tk, tv, out, ws
