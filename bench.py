@@ -339,7 +339,8 @@ def main():
         return profile_case(hla, dev, args.profile_case)
     if args.only in ("ahla", "backward"):
         st = torch.cuda.current_stream()
-        res = bench_ahla(hla, dev, st, hbm_peak, world) if args.only == "ahla" else bench_backward(hla, dev, st, world)
+        res = (bench_ahla(hla, dev, st, hbm_peak, world, tc_peak=tc_peak) if args.only == "ahla"
+               else bench_backward(hla, dev, st, world))
         if rank == 0:
             print(json.dumps(res))
         return
@@ -512,7 +513,7 @@ def main():
     if not args.no_decode:
         result["mid"], result["hla3"] = bench_others(hla, dev, stream, hbm_peak, tc_peak, world)
         result["gpu_launches"] += result["mid"]["launches"] + result["hla3"]["launches"]
-        result["ahla"] = bench_ahla(hla, dev, stream, hbm_peak, world)
+        result["ahla"] = bench_ahla(hla, dev, stream, hbm_peak, world, tc_peak=tc_peak)
         result["gpu_launches"] += result["ahla"]["forward"]["launches"] + result["ahla"]["decode"]["launches"]
         result["backward"] = bench_backward(hla, dev, stream, world)
         result["gpu_launches"] += result["backward"]["launches"]
@@ -652,7 +653,7 @@ def bench_backward(hla, dev, stream, world, steps=10, warmup=3):
             "launches": 5 * steps}
 
 
-def bench_ahla(hla, dev, stream, hbm_peak, world, steps=20, warmup=3, decode_steps=256):
+def bench_ahla(hla, dev, stream, hbm_peak, world, steps=20, warmup=3, decode_steps=256, tc_peak=None):
     """AHLA: the forward on ahla_bf16 (B8 H16 n2048 d64 bf16, chunk 64) and the decode step on
     ahla_decode_bf16 (B64 H32 d128, state built from a 4096-token prefix), CUDA events on the
     launching stream."""
@@ -678,18 +679,28 @@ def bench_ahla(hla, dev, stream, hbm_peak, world, steps=20, warmup=3, decode_ste
     e1.record(stream)
     torch.cuda.synchronize()
     ms = max_over_ranks(e0.elapsed_time(e1) / steps, world)
+    tensor_path = hla.ahla_forward_path(w.B, w.H, w.n, w.d, w.dv, normalized=w.normalized, chunk=w.chunk,
+                                        dtype=tq.dtype) == 1
     tf = ahla_flops(w) / (ms * 1e-3) / 1e12
     gbs = fwd_bytes(w) / (ms * 1e-3) / 1e9
+    if tensor_path:  # the slower of the bytes at HBM bandwidth and the FLOPs at the bf16 tensor peak
+        t_bytes, t_flops = fwd_bytes(w) / (hbm_peak * 1e9), ahla_flops(w) / (tc_peak * 1e12)
+        hbm = {"achieved": gbs, "peak": hbm_peak, "unit": "GB/s", "frac": gbs / hbm_peak}
+        ten = {"achieved": tf, "peak": tc_peak, "unit": "TFLOP/s", "frac": tf / tc_peak}
+        main, other, bound = (hbm, ten, "hbm") if t_bytes >= t_flops else (ten, hbm, "tensor")
+        roof = dict(main, bound=bound, traffic=None, flops=ahla_flops(w), algorithmic_bytes=fwd_bytes(w),
+                    kernel="ahla_tc_kernel (tcgen05, one launch)")
+        roof["tensor_view" if bound == "hbm" else "hbm_view"] = other
+    else:
+        roof = {"bound": "alu", "achieved": tf, "peak": alu_peak(), "unit": "TFLOP/s", "frac": tf / alu_peak(),
+                "traffic": None, "flops": ahla_flops(w),
+                "peak_kind": "derived (152 SMs x 128 fp32 lanes x 2 x 2.07 GHz)",
+                "kernel": "ahla_local/scan/out (fp32 CUDA cores)",
+                "hbm_view": {"achieved": gbs, "peak": hbm_peak, "unit": "GB/s", "frac": gbs / hbm_peak}}
     res["forward"] = {"workload": w.name, "B": w.B, "H": w.H, "n": w.n, "d": w.d, "dv": w.dv, "chunk": w.chunk,
                       "tokens": w.dtype, "ms_per_step": ms, "value": w.B * w.n * world / (ms * 1e-3),
-                      "unit": "tokens/s", "steps": steps,
-                      "roofline": {"bound": "alu", "achieved": tf, "peak": alu_peak(), "unit": "TFLOP/s",
-                                   "frac": tf / alu_peak(), "traffic": None, "flops": ahla_flops(w),
-                                   "peak_kind": "derived (152 SMs x 128 fp32 lanes x 2 x 2.07 GHz)",
-                                   "kernel": "ahla_local/scan/out (fp32 CUDA cores)",
-                                   "hbm_view": {"achieved": gbs, "peak": hbm_peak, "unit": "GB/s",
-                                                "frac": gbs / hbm_peak}},
-                      "launches": 3 * steps}
+                      "unit": "tokens/s", "steps": steps, "roofline": roof,
+                      "launches": (1 if tensor_path else 3) * steps}
     del tq, tk, tv, out, ws
     # decode step
     w = hla_inputs.WORKLOADS["ahla_decode_bf16"]

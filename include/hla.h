@@ -278,12 +278,24 @@ size_t ahla_workspace_bytes(int B, int H, int n, int d, int dv, int chunk, hla_d
  * recurrence (scan equivalence); chunk is the scan granularity (results do not
  * depend on it up to rounding).  Arguments, layouts, shapes and errors as for
  * hla2_forward (no masked flag), with the AHLA state layout for state_in /
- * state_out (state_out may equal state_in).
+ * state_out (state_out may equal state_in).  bf16 tokens with d and dv in
+ * {64, 128}, the plain output and no states run on the tensor cores (one
+ * persistent tcgen05 kernel sweeping each head's 128-token tiles with the P
+ * and E carries in tensor memory); every other call runs three fp32 kernels.
+ * A device-side wait that exceeds its budget sets the flag hla_poll_error reads.
  */
 hla_status ahla_forward(const void *q, const void *k, const void *v, void *out, hla_dtype dt,
                         int B, int H, int n, int d, int dv, int normalized, float eps, int chunk,
                         const float *state_in, float *state_out,
                         void *workspace, size_t workspace_bytes, hla_stream_t stream);
+
+/*
+ * ahla_forward_path -- which CUDA path ahla_forward takes for these arguments on
+ * the current device, without launching anything: 1 the tensor-core kernel,
+ * 0 the fp32 kernels, -1 the arguments are not supported.
+ */
+int ahla_forward_path(int B, int H, int n, int d, int dv, int normalized, int chunk, hla_dtype dt, int has_state_in,
+                      int has_state_out);
 
 /*
  * ahla_step -- one AHLA decode step for B*H heads (the online updates of

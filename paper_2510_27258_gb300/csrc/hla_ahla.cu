@@ -361,6 +361,7 @@ size_t ahla_workspace_bytes_internal(int BH, int n, int d, int dv, int chunk) {
 }
 
 cudaError_t ahla_forward_launch(const Fwd2 &p, cudaStream_t stream) {
+    if (ahla_tc_applicable(p)) return ahla_tc_forward(p, stream);
     return p.dt == HLA_BF16 ? forward_t<__nv_bfloat16>(p, stream) : forward_t<float>(p, stream);
 }
 

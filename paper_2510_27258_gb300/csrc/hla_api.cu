@@ -262,9 +262,25 @@ hla_status ahla_forward(const void *q, const void *k, const void *v, void *out, 
     if ((reinterpret_cast<uintptr_t>(workspace) & 255u) != 0)
         return fail(HLA_ERR_INVALID_ARGUMENT, "workspace must be 256-byte aligned");
     if ((long long)B * H == 0) return HLA_OK;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    st = cuda_status(cudaMemsetAsync(workspace, 0, kWsHeaderBytes, s), "clearing the workspace header");
+    if (st != HLA_OK) return st;
     Fwd2 p{q, k, v, out, dt, B * H, n, d, dv, 1, normalized, eps, chunk, state_in, state_out,
            static_cast<char *>(workspace), workspace_bytes};
-    return cuda_status(ahla_forward_launch(p, reinterpret_cast<cudaStream_t>(stream)), "AHLA forward");
+    return cuda_status(ahla_forward_launch(p, s), "AHLA forward");
+}
+
+int ahla_forward_path(int B, int H, int n, int d, int dv, int normalized, int chunk, hla_dtype dt, int has_state_in,
+                      int has_state_out) {
+    const void *dummy = reinterpret_cast<const void *>(uintptr_t(256));
+    if (check_forward(dummy, dummy, dummy, const_cast<void *>(dummy), dt, B, H, n, d, dv, 1, normalized, 0.f, chunk,
+                      nullptr, nullptr) != HLA_OK)
+        return -1;
+    Fwd2 p{dummy, dummy, dummy, const_cast<void *>(dummy), dt, B * H, n, d, dv, 1, normalized, 0.f, chunk,
+           has_state_in ? static_cast<const float *>(dummy) : nullptr,
+           has_state_out ? static_cast<float *>(const_cast<void *>(dummy)) : nullptr, nullptr,
+           ahla_workspace_bytes(B, H, n, d, dv, chunk, dt)};
+    return ((long long)B * H > 0 && ahla_tc_applicable(p)) ? 1 : 0;
 }
 
 hla_status ahla_step(const void *q, const void *k, const void *v, void *out, hla_dtype dt, int B, int H, int d,

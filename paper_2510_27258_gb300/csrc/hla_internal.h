@@ -94,6 +94,9 @@ cudaError_t backward2_launch(const Bwd2 &p, cudaStream_t stream);
 
 // AHLA (asymmetric second order): chunk-parallel forward and decode step
 size_t ahla_workspace_bytes_internal(int BH, int n, int d, int dv, int chunk);
+// tensor-core AHLA forward (bf16, d and dv in {64, 128}, plain output, no states, sm_103)
+bool ahla_tc_applicable(const Fwd2 &p);
+cudaError_t ahla_tc_forward(const Fwd2 &p, cudaStream_t stream);
 cudaError_t ahla_forward_launch(const Fwd2 &p, cudaStream_t stream);
 cudaError_t ahla_step_launch(const void *q, const void *k, const void *v, void *out, hla_dtype dt, int BH, int d,
                              int dv, int normalized, float eps, float *state, cudaStream_t stream);

@@ -145,3 +145,55 @@ def test_ahla_step(hla, d, dv, normalized):
     else:
         assert rowerr(got, num[:, prefix:]) < TOL["f32"]
     assert np.abs(st.cpu().numpy().reshape(B * H, -1) - rst).max() <= 2e-5 * np.abs(rst).max()
+
+
+# ----------------------------------------------------------------------------
+# the tensor-core path (bf16, d and dv in {64, 128}, plain output, no states)
+# ----------------------------------------------------------------------------
+
+TC_SHAPES = [
+    # (B, H, n, d, dv)
+    (1, 1, 1, 128, 128),
+    (1, 2, 127, 128, 128),
+    (2, 3, 300, 64, 64),
+    (1, 2, 700, 64, 128),
+    (1, 1, 1000, 128, 64),
+]
+
+
+@pytest.mark.parametrize("shape", TC_SHAPES, ids=lambda s: "B%dH%dn%dd%ddv%d" % s)
+def test_ahla_tensor_core_path(hla, shape, monkeypatch):
+    """Every head against the oracle, and against the CUDA-core path on the same inputs."""
+    B, H, n, d, dv = shape
+    q, k, v = hla_inputs.make_qkv(B, H, n, d, dv, seed=4000 + n + d, dtype="bf16")
+    ref, _, _ = ref_ahla(q, k, v)
+    got = gpu_ahla(hla, q, k, v, "bf16", False, 64)
+    assert rowerr(got, ref) < TOL["bf16"]
+    monkeypatch.setenv("HLA_DISABLE_FUSED", "1")
+    generic = gpu_ahla(hla, q, k, v, "bf16", False, 64)
+    assert rowerr(generic, ref) < TOL["bf16"]
+
+
+def test_ahla_tensor_core_more_heads_than_sms(hla):
+    """200 heads: a CTA sweeps several heads one after the other (carries restarted per head)."""
+    B, H, n, d = 2, 100, 260, 128
+    q, k, v = hla_inputs.make_qkv(B, H, n, d, d, seed=4100, dtype="bf16")
+    got = gpu_ahla(hla, q, k, v, "bf16", False, 64)
+    heads = [0, 1, 151, 152, 153, 199]
+    ref = oracle.ahla_serial(q.reshape(B * H, n, d)[heads], k.reshape(B * H, n, d)[heads],
+                             v.reshape(B * H, n, d)[heads], nthreads=6)
+    assert rowerr(got[heads], ref) < TOL["bf16"]
+
+
+def test_ahla_tensor_core_causality_and_determinism(hla):
+    B, H, n, d, t = 1, 2, 512, 128, 300
+    q, k, v = hla_inputs.make_qkv(B, H, n, d, d, seed=4200, dtype="bf16")
+    a = gpu_ahla(hla, q, k, v, "bf16", False, 64)
+    assert np.array_equal(a, gpu_ahla(hla, q, k, v, "bf16", False, 64))
+    q2, k2, v2 = q.copy(), k.copy(), v.copy()
+    rng = np.random.default_rng(3)
+    for x in (q2, k2, v2):
+        x[:, :, t + 1:] = hla_inputs.round_to(rng.standard_normal(x[:, :, t + 1:].shape), "bf16")
+    b = gpu_ahla(hla, q2, k2, v2, "bf16", False, 64)
+    assert np.array_equal(a[:, : t + 1], b[:, : t + 1])
+    assert not np.array_equal(a[:, t + 1:], b[:, t + 1:])

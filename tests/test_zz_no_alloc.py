@@ -107,6 +107,27 @@ def test_noalloc_python_wrapper_with_initial_state(hla):
         _check_oracle(q, k, v, got, False, state_in=st0)
 
 
+def test_noalloc_wait_timeout_is_reported(hla, monkeypatch):
+    """A segment that never publishes its S prefix (injected on the host side, as in
+    the fused tests): the next segment's 20 ms wait runs out, the call finishes,
+    hla_poll_error_noalloc reports HLA_ERR_TIMEOUT and clears it, and the next call
+    on the same scratch is correct."""
+    monkeypatch.setenv("HLA_FUSED_SEGMENT_TILES", "1")
+    monkeypatch.setenv("HLA_TEST_WAIT_NS", "20000000")
+    monkeypatch.setenv("HLA_TEST_SKIP_PUBLISH_ITEM", "0")
+    B, H, n, d = 1, 1, 512, 128
+    q, k, v = hla_inputs.make_qkv(B, H, n, d, d, seed=51, dtype="bf16")
+    tq, tk, tv = (hla_inputs.as_torch(x, "bf16", DEV) for x in (q, k, v))
+    out = torch.zeros((B, H, n, d), dtype=torch.bfloat16, device=DEV)
+    assert _noalloc(hla, tq, tk, tv, out, False) == hla.HLA_OK
+    assert hla.hla_poll_error_noalloc() == hla.HLA_ERR_TIMEOUT
+    assert hla.hla_poll_error_noalloc() == hla.HLA_OK  # cleared
+    monkeypatch.delenv("HLA_TEST_SKIP_PUBLISH_ITEM")
+    assert _noalloc(hla, tq, tk, tv, out, False) == hla.HLA_OK
+    assert hla.hla_poll_error_noalloc() == hla.HLA_OK
+    _check_oracle(q, k, v, out.float().cpu().numpy(), False)
+
+
 def test_noalloc_empty_problem_is_ok(hla):
     t = torch.zeros((1, 0, 256, 128), dtype=torch.bfloat16, device=DEV)
     assert _noalloc(hla, t, t, t, t, False) == hla.HLA_OK
