@@ -46,6 +46,9 @@ TRAFFIC = {
     "step2_kernel": {"src": ["hla_step.cu"], "sha256": "5542daa4b35fe2f4", "workload": "decode_bf16", "n": 0,
                      "bytes": 750.6e6, "how": "ncu capture of one step at B64 H32 d128 (bench.py --profile-case "
                                               "tuple_step): 406.4 MB read + 344.2 MB written"},
+    "c3_kernels": {"src": ["hla3_chunked.cu"], "sha256": "17ac1acd5c9202d1", "workload": "hla3_f32", "n": 4096,
+                   "bytes": 432.5e6, "how": "ncu capture of one forward's five launches (bench.py --only hla3_f32): "
+                                            "373.0 MB read + 59.5 MB written, 6.4 x the token I/O (per-chunk records)"},
     "step2_kernel_sde": {"src": ["hla_step.cu"], "sha256": "5542daa4b35fe2f4", "workload": "decode_bf16", "n": 0,
                          "bytes": 481.3e6, "how": "ncu capture of one step at B64 H32 d128 (bench.py --profile-case "
                                                   "sde_step): 271.2 MB read + 210.1 MB written"},
@@ -564,8 +567,10 @@ def bench_others(hla, dev, stream, hbm_peak, tc_peak, world, names=("mid_bf16", 
                "ms_per_step": ms, "value": tok, "unit": "tokens/s", "steps": steps}
         if third:
             tf = hla3_flops(w) / (ms * 1e-3) / 1e12
+            h3_traffic, h3_how = traffic("c3_kernels", w.name, w.n)
             cfg["roofline"] = {"bound": "alu", "achieved": tf, "peak": alu_peak(), "unit": "TFLOP/s",
-                               "frac": tf / alu_peak(), "traffic": None, "flops": hla3_flops(w),
+                               "frac": tf / alu_peak(), "traffic": h3_traffic, "traffic_how": h3_how,
+                               "algorithmic_bytes": fwd_bytes(w), "flops": hla3_flops(w),
                                "peak_kind": "derived (152 SMs x 128 fp32 lanes x 2 x 2.07 GHz)",
                                "kernel": "c3_local/bracket/out (fp32 CUDA cores)"}
             cfg["launches"] = steps * 5

@@ -120,3 +120,35 @@ def test_noalloc_empty_problem_without_gpu(L):
     f = ctypes.c_float(1e-6)
     assert L.hla2_forward_noalloc(None, None, None, None, 1, 1, 0, 256, 128, 128, 1, 0, f, 128, None, None) == H.HLA_OK
     assert L.hla_last_error() == b""
+
+
+def test_ahla_and_backward_argument_errors(L):
+    from paper_2510_27258_gb300 import hla as H
+    f = ctypes.c_float(1e-6)
+    assert L.ahla_state_floats(128, 64) == 2 * 128 * 64 + 2 * 128
+    assert L.ahla_workspace_bytes(1, 1, 64, 16, 16, 16, 0) > 0
+    assert L.ahla_workspace_bytes(1, 1, 64, 48, 16, 16, 0) == 0
+    assert L.hla2_backward_workspace_bytes(1, 1, 64, 16, 16, 16, 1) > 0
+    assert L.hla2_backward_workspace_bytes(1, 1, 64, 16, 16, 0, 1) == 0
+
+    def ahla(q=16, B=1, n=64, d=16, chunk=16, ws=256, ws_bytes=1 << 30):
+        return L.ahla_forward(q, 16, 16, 16, 1, B, 1, n, d, 16, 0, f, chunk, None, None, ws, ws_bytes, None)
+    assert ahla(q=None) == H.HLA_ERR_INVALID_ARGUMENT
+    assert ahla(q=8) == H.HLA_ERR_INVALID_ARGUMENT
+    assert ahla(d=24) == H.HLA_ERR_UNSUPPORTED
+    assert ahla(chunk=129) == H.HLA_ERR_UNSUPPORTED
+    assert ahla(ws=None) == H.HLA_ERR_WORKSPACE
+    assert ahla(ws=272) == H.HLA_ERR_INVALID_ARGUMENT
+    assert ahla(B=0) == H.HLA_OK
+    assert L.ahla_step(16, 16, 16, 16, 1, 1, 1, 128, 128, 0, f, None, None) == H.HLA_ERR_INVALID_ARGUMENT
+    assert L.ahla_step(16, 16, 16, 16, 1, 0, 1, 128, 128, 0, f, 16, None) == H.HLA_OK
+    assert L.ahla_forward_path(1, 1, 64, 24, 16, 0, 16, 1, 0, 0) == -1
+    assert L.ahla_forward_path(1, 1, 64, 16, 16, 0, 16, 0, 0, 0) == 0  # fp32 tokens: the CUDA-core kernels
+
+    def bwd(dout=16, dq=16, n=64, d=16, ws=256, ws_bytes=1 << 30):
+        return L.hla2_backward(16, 16, 16, dout, dq, 16, 16, 1, 1, 1, n, d, 16, 0, f, 16, ws, ws_bytes, None)
+    assert bwd(dout=None) == H.HLA_ERR_INVALID_ARGUMENT
+    assert bwd(dq=24) == H.HLA_ERR_INVALID_ARGUMENT
+    assert bwd(d=100) == H.HLA_ERR_UNSUPPORTED
+    assert bwd(ws_bytes=16) == H.HLA_ERR_WORKSPACE
+    assert bwd(n=0) == H.HLA_OK
