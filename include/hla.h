@@ -224,6 +224,17 @@ hla_status hla3_forward(const void *q, const void *k, const void *v, void *out, 
                         void *workspace, size_t workspace_bytes, hla_stream_t stream);
 
 /*
+ * hla3_forward_path -- which CUDA path hla3_forward takes for these arguments on
+ * the current device, without launching anything: 2 the tensor-core kernels
+ * (fp32 tokens, d = dv = 32, masked = 1, normalized = 0, no states, an sm_103
+ * device), 1 the chunk-parallel fp32 kernels, 0 the serial kernel, -1 the
+ * arguments are not supported.  *launches (if not null) receives the number of
+ * kernel launches of one call (0 when B*H = 0).
+ */
+int hla3_forward_path(int B, int H, int n, int d, int dv, int masked, int normalized, int chunk, hla_dtype dt,
+                      int has_state_in, int has_state_out, int *launches);
+
+/*
  * hla2_forward_noalloc -- hla2_forward for callers that cannot allocate device
  * memory (no counterpart in the paper: it only changes where scratch lives).
  *

@@ -119,7 +119,9 @@ size_t hla3_workspace_bytes(int B, int H, int n, int d, int dv, int chunk, hla_d
     const int BH = B * H;
     const size_t g = generic3_workspace_bytes(BH, n, d, dv, chunk);
     const size_t c = chunked3_eligible(BH, n, d, dv, chunk) ? chunked3_workspace_bytes(BH, n, d, dv, chunk) : 0;
-    return align_up(g > c ? g : c, 256);
+    const size_t t = hla3_tc_workspace_bytes(BH, n);
+    const size_t gc = g > c ? g : c;
+    return align_up(gc > t ? gc : t, 256);
 }
 
 hla_status hla2_forward(const void *q, const void *k, const void *v, void *out, hla_dtype dt, int B, int H, int n,
@@ -295,6 +297,32 @@ hla_status ahla_step(const void *q, const void *k, const void *v, void *out, hla
                        "AHLA decode step");
 }
 
+int hla3_forward_path(int B, int H, int n, int d, int dv, int masked, int normalized, int chunk, hla_dtype dt,
+                      int has_state_in, int has_state_out, int *launches) {
+    const void *dummy = reinterpret_cast<const void *>(uintptr_t(256));
+    if (check_forward(dummy, dummy, dummy, const_cast<void *>(dummy), dt, B, H, n, d, dv, masked, normalized, 0.f,
+                      chunk, nullptr, nullptr) != HLA_OK)
+        return -1;
+    Fwd2 p{dummy, dummy, dummy, const_cast<void *>(dummy), dt, B * H, n, d, dv, masked, normalized, 0.f, chunk,
+           has_state_in ? static_cast<const float *>(dummy) : nullptr,
+           has_state_out ? static_cast<float *>(const_cast<void *>(dummy)) : nullptr, nullptr,
+           hla3_workspace_bytes(B, H, n, d, dv, chunk, dt)};
+    int path = 0, nl = 0;
+    if ((long long)B * H == 0) {
+        path = 0;
+    } else if (hla3_tc_applicable(p)) {
+        path = 2;
+        nl = hla3_tc_launches(B * H, n);
+    } else if (!has_state_out && chunked3_eligible(B * H, n, d, dv, chunk)) {
+        path = 1;
+        nl = masked ? 5 + (has_state_in ? 1 : 0) : 3;
+    } else {
+        nl = 1;
+    }
+    if (launches) *launches = nl;
+    return path;
+}
+
 hla_status hla3_forward(const void *q, const void *k, const void *v, void *out, hla_dtype dt, int B, int H, int n,
                         int d, int dv, int masked, int normalized, float eps, int chunk, const float *state_in,
                         float *state_out, void *workspace, size_t workspace_bytes, hla_stream_t stream) {
@@ -314,6 +342,7 @@ hla_status hla3_forward(const void *q, const void *k, const void *v, void *out, 
     if (st != HLA_OK) return st;
     Fwd2 p{q, k, v, out, dt, B * H, n, d, dv, masked, normalized, eps, chunk, state_in, state_out,
            static_cast<char *>(workspace), workspace_bytes};
+    if (hla3_tc_applicable(p)) return cuda_status(hla3_tc_forward(p, s), "third-order forward (tensor cores)");
     // chunk-parallel unless the final state is wanted (the serial kernel also carries G1..G3, h1..h3)
     if (!state_out && chunked3_eligible(B * H, n, d, dv, chunk))
         return cuda_status(chunked3_forward(p, s), "third-order forward (chunked)");

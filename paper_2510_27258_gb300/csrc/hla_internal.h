@@ -109,4 +109,11 @@ size_t chunked3_workspace_bytes(int BH, int n, int d, int dv, int chunk);
 bool chunked3_eligible(int BH, int n, int d, int dv, int chunk);
 cudaError_t chunked3_forward(const Fwd2 &p, cudaStream_t stream);
 
+// Masked third-order forward on the tensor cores (hla3_sm103.cu): fp32, d = dv = 32,
+// plain output, no states
+size_t hla3_tc_workspace_bytes(int BH, int n);
+bool hla3_tc_applicable(const Fwd2 &p);
+int hla3_tc_launches(int BH, int n);
+cudaError_t hla3_tc_forward(const Fwd2 &p, cudaStream_t stream);
+
 }  // namespace hla

@@ -22,6 +22,7 @@ HLA_F32, HLA_BF16 = 0, 1
 # every symbol include/hla.h declares
 EXPORTS = ("hla_status_string", "hla_last_error", "hla2_state_floats", "hla2_workspace_bytes", "hla2_forward",
            "hla2_forward_path", "hla2_step", "hla3_state_floats", "hla3_workspace_bytes", "hla3_forward",
+           "hla3_forward_path",
            "hla2_forward_noalloc", "hla_poll_error_noalloc", "hla_poll_error", "hla2_sde_state_floats",
            "hla2_state_to_sde", "hla2_step_sde", "ahla_state_floats", "ahla_workspace_bytes", "ahla_forward",
            "ahla_step", "hla2_backward_workspace_bytes", "hla2_backward", "ahla_forward_path")
@@ -71,8 +72,9 @@ def lib():
             getattr(L, name).restype = i
         L.hla2_forward_noalloc.argtypes = [vp, vp, vp, vp, i, i, i, i, i, i, i, i, f, i, vp, vp]
         L.hla2_forward_noalloc.restype = i
-        L.hla2_forward_path.argtypes = [i, i, i, i, i, i, i, i, i, i, i, ctypes.POINTER(i)]
-        L.hla2_forward_path.restype = i
+        for name in ("hla2_forward_path", "hla3_forward_path"):
+            getattr(L, name).argtypes = [i, i, i, i, i, i, i, i, i, i, i, ctypes.POINTER(i)]
+            getattr(L, name).restype = i
         L.hla2_step.argtypes = [vp, vp, vp, vp, i, i, i, i, i, i, i, f, vp, vp]
         L.hla2_step.restype = i
         L.hla_poll_error.argtypes = [vp, vp]
@@ -197,6 +199,17 @@ def hla2_forward_path(B, H, n, d, dv, *, masked=True, normalized=False, chunk=12
     code = dtype if isinstance(dtype, int) else (HLA_BF16 if dtype == torch.bfloat16 else HLA_F32)
     n_launch = ctypes.c_int(0)
     path = lib().hla2_forward_path(B, H, n, d, dv, int(masked), int(normalized), int(chunk), code,
+                                   int(has_state_in), int(has_state_out), ctypes.byref(n_launch))
+    return int(path), int(n_launch.value)
+
+
+def hla3_forward_path(B, H, n, d, dv, *, masked=True, normalized=False, chunk=32, dtype=torch.float32,
+                      has_state_in=False, has_state_out=False):
+    """(path, launches) that hla3_forward takes: path 2 = tensor-core kernels, 1 = chunk-parallel fp32
+    kernels, 0 = serial kernel, -1 = unsupported."""
+    code = dtype if isinstance(dtype, int) else (HLA_BF16 if dtype == torch.bfloat16 else HLA_F32)
+    n_launch = ctypes.c_int(0)
+    path = lib().hla3_forward_path(B, H, n, d, dv, int(masked), int(normalized), int(chunk), code,
                                    int(has_state_in), int(has_state_out), ctypes.byref(n_launch))
     return int(path), int(n_launch.value)
 

@@ -144,6 +144,14 @@ def test_ahla_and_backward_argument_errors(L):
     assert L.ahla_step(16, 16, 16, 16, 1, 0, 1, 128, 128, 0, f, 16, None) == H.HLA_OK
     assert L.ahla_forward_path(1, 1, 64, 24, 16, 0, 16, 1, 0, 0) == -1
     assert L.ahla_forward_path(1, 1, 64, 16, 16, 0, 16, 0, 0, 0) == 0  # fp32 tokens: the CUDA-core kernels
+    # third order: no device here, so never the tensor-core path; chunk-parallel or serial otherwise
+    nl = ctypes.c_int(-7)
+    assert L.hla3_forward_path(1, 1, 64, 24, 32, 1, 0, 32, 0, 0, 0, ctypes.byref(nl)) == -1
+    assert L.hla3_forward_path(2, 4, 4096, 32, 32, 1, 0, 32, 0, 0, 0, ctypes.byref(nl)) == 1 and nl.value == 5
+    assert L.hla3_forward_path(2, 4, 4096, 32, 32, 1, 0, 32, 0, 1, 0, ctypes.byref(nl)) == 1 and nl.value == 6
+    assert L.hla3_forward_path(2, 4, 4096, 32, 32, 0, 0, 32, 0, 0, 0, ctypes.byref(nl)) == 1 and nl.value == 3
+    assert L.hla3_forward_path(2, 4, 4096, 32, 32, 1, 0, 32, 0, 0, 1, ctypes.byref(nl)) == 0 and nl.value == 1
+    assert L.hla3_forward_path(0, 4, 4096, 32, 32, 1, 0, 32, 0, 0, 0, ctypes.byref(nl)) == 0 and nl.value == 0
 
     def bwd(dout=16, dq=16, n=64, d=16, ws=256, ws_bytes=1 << 30):
         return L.hla2_backward(16, 16, 16, dout, dq, 16, 16, 1, 1, 1, n, d, 16, 0, f, 16, ws, ws_bytes, None)
