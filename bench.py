@@ -124,6 +124,34 @@ def hla3_flops(w):
     return 2 * chunks * (local + bracket + out)
 
 
+def hla3_tc_flops(w):
+    """FLOPs of one masked third-order forward in the 128-token tile form of the tensor-core path
+    (2 per multiply-add, triangles counted once): per tile of T tokens, A = Q K^T (T^2 d, the
+    squares above the diagonal enter b), Y (T d dv + T^2 dv / 2), Q S^K_p and K S^Q_p (2 T d^2),
+    C' on the lower triangle (T^3 / 6 + T^2 d / 2), LA^T aV, LA Z', (L.C') aV (3 T^2 dv / 2),
+    Q F_p (T d dv) and the carries K^T K, Q^T Q, K^T V, K^T G', (Q S^K_p)^T aV (2 T d^2 + 3 T d dv)."""
+    T, d, dv = 128, w.d, w.dv
+    tiles = w.B * w.H * ((w.n + T - 1) // T)
+    per_tile = (T * T * d + T * d * dv + T * T * dv / 2 + 2 * T * d * d + T ** 3 / 6 + T * T * d / 2
+                + 3 * T * T * dv / 2 + T * d * dv + 2 * T * d * d + 3 * T * d * dv)
+    return 2 * tiles * per_tile
+
+
+def hla3_tc_issued_flops(w, sms=152):
+    """Tensor FLOPs the tensor-core path issues (bf16 hi/lo splits, full 128-row tiles): per
+    sweep tile 36 K = 16 steps at N = 128, 104 at N = 64 and 24 at N = 32; per pre-pass tile 24
+    at N = 64 (segments as the library plans them: sms // (B H) per head, at most one per tile)."""
+    T = 128
+    M = (w.n + T - 1) // T
+    BH = w.B * w.H
+    G = max(1, min(M, sms // BH, 160))
+    L = (M + G - 1) // G
+    G = (M + L - 1) // L
+    pre_tiles = BH * (M - (M - (G - 1) * L)) if G > 1 else 0
+    step = lambda N: 2 * 128 * N * 16
+    return BH * M * (36 * step(128) + 104 * step(64) + 24 * step(32)) + pre_tiles * 24 * step(64)
+
+
 def ahla_flops(w):
     """Algorithmic FLOPs of one AHLA forward (masks exploited, chunk C): per token-head
     2 * [C d / 2 (Q K^T) + C dv / 2 (A V) + C dv / 2 (A R) + C / 2 (A 1, A s)
@@ -565,7 +593,27 @@ def bench_others(hla, dev, stream, hbm_peak, tc_peak, world, names=("mid_bf16", 
         cfg = {"workload": name, "B": w.B, "H": w.H, "n": w.n, "d": w.d, "dv": w.dv, "chunk": w.chunk,
                "masked": w.masked, "normalized": w.normalized, "tokens": w.dtype, "order": w.order,
                "ms_per_step": ms, "value": tok, "unit": "tokens/s", "steps": steps}
-        if third:
+        path, n_launch = (hla.hla3_forward_path(w.B, w.H, w.n, w.d, w.dv, masked=w.masked, normalized=w.normalized,
+                                                chunk=w.chunk, dtype=tq.dtype) if third else (None, 1))
+        if third and path == 2:
+            gbs = fwd_bytes(w) / (ms * 1e-3) / 1e9
+            tc_traffic, tc_how = traffic("hla3_tc_kernels", w.name, w.n)
+            issued = hla3_tc_issued_flops(w)
+            cfg["roofline"] = {
+                "bound": "hbm", "achieved": gbs, "peak": hbm_peak, "unit": "GB/s", "frac": gbs / hbm_peak,
+                "traffic": tc_traffic, "traffic_how": tc_how, "algorithmic_bytes": fwd_bytes(w),
+                "algorithmic_flops": hla3_tc_flops(w),
+                "roofline_us": max(fwd_bytes(w) / (hbm_peak * 1e9), hla3_tc_flops(w) / (tc_peak * 1e12)) * 1e6,
+                "tensor_view": {"achieved": hla3_tc_flops(w) / (ms * 1e-3) / 1e12, "peak": tc_peak,
+                                "unit": "TFLOP/s", "frac": hla3_tc_flops(w) / (ms * 1e-3) / 1e12 / tc_peak},
+                "issued_tensor": {"flops": issued, "achieved": issued / (ms * 1e-3) / 1e12, "peak": tc_peak,
+                                  "unit": "TFLOP/s", "frac": issued / (ms * 1e-3) / 1e12 / tc_peak,
+                                  "note": "bf16 hi.hi + hi.lo + lo.hi products on full 128-row tiles"},
+                "peak_kind": "measured",
+                "kernel": "hla3_tc_kernel (tcgen05 pre-pass and sweep) + hla3_tc_fixup_kernel"}
+            cfg["path"] = "tensor cores"
+            cfg["launches"] = steps * n_launch
+        elif third:
             tf = hla3_flops(w) / (ms * 1e-3) / 1e12
             h3_traffic, h3_how = traffic("c3_kernels", w.name, w.n)
             cfg["roofline"] = {"bound": "alu", "achieved": tf, "peak": alu_peak(), "unit": "TFLOP/s",
@@ -573,7 +621,8 @@ def bench_others(hla, dev, stream, hbm_peak, tc_peak, world, names=("mid_bf16", 
                                "algorithmic_bytes": fwd_bytes(w), "flops": hla3_flops(w),
                                "peak_kind": "derived (152 SMs x 128 fp32 lanes x 2 x 2.07 GHz)",
                                "kernel": "c3_local/bracket/out (fp32 CUDA cores)"}
-            cfg["launches"] = steps * 5
+            cfg["path"] = "fp32 CUDA cores"
+            cfg["launches"] = steps * n_launch
         else:
             cfg["roofline"] = roofline_record(w, ms, hbm_peak, tc_peak, "measured", None, None, "hla2_fused_kernel")
             cfg["launches"] = steps

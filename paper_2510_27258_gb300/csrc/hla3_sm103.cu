@@ -66,6 +66,9 @@ constexpr int kMaxSegments = 160;
 enum Block { bQ = 0, bK = 1, bV = 2, bQS = 3, bAV = 4, bZ = 5, bG = 6, bLh = 7, bLl = 9, bCar = 11, kBlocks = 12 };
 // bLh / bLl: 128 x 128 tiles (two blocks each): LA, then L . C', hi and lo parts.
 // bCar: four 32-row K-major operands (hi | lo): S^K_p, S^Q_p, P_p^T, F_p^T.
+// The pre-pass uses Q, K, V only; blocks kStage.. hold its two stages of fp32 tokens
+// (Q, K, V of one tile: 128 rows of 128 bytes each, copied as one contiguous piece).
+constexpr int kStage = 4;
 constexpr uint32_t kSmemBlocks = kBlocks * kBlockBytes;
 
 // TMEM columns
@@ -75,7 +78,8 @@ enum Bar {
     bEvA = 0, bEvQ = 1, bEvY = 2, bEvC = 3, bEvO = 4,  // MMA commits
     bEp0 = 5, bEp1 = 6, bEp2 = 7, bEp3 = 8,            // epilogue hand-offs (16 warp arrivals)
     bTear = 9,
-    kNumBars = 10
+    bSt0 = 10,                                         // + stage: pre-pass token copies
+    kNumBars = 12
 };
 
 struct Misc {
@@ -126,34 +130,69 @@ __device__ __forceinline__ void epi_arrive(Misc *ms, int b) {
     if ((threadIdx.x & 31) == 0) mbar_arrive(&ms->bar[b]);
 }
 
+// 32 lanes x 8 consecutive TMEM columns
+__device__ __forceinline__ void tmem_ld8(uint32_t taddr, uint32_t (&v)[8]) {
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];"
+                 : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7])
+                 : "r"(taddr));
+}
+
+// 1-D bulk copy global -> shared (both addresses 16-byte aligned, size a multiple of 16),
+// completing as transaction bytes on `bar`
+__device__ __forceinline__ void bulk_load(void *dst, const void *src, uint32_t bytes, uint64_t *bar) {
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+                 ::"r"(smem_u32(dst)), "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(smem_u32(bar))
+                 : "memory");
+}
+
 // ------------------------------- MMA issue -------------------------------
-__device__ __forceinline__ uint64_t dsc(uint32_t saddr, uint32_t lbo) { return desc_sw128(saddr, lbo, 1024); }
+// Shared-memory descriptors: the high word is fixed (1 KiB between 8-row groups, tcgen05
+// version, 128-byte swizzle); the low word is the start address / 16 plus the leading-byte
+// offset (unused for K-major operands; 16 KiB between the 64-element blocks of an MN-major
+// operand), so every K step adds a constant to a per-block low word.
+constexpr uint32_t kDescHi = (1024u >> 4) | (1u << 14) | (2u << 29);
+constexpr uint32_t kLboK = 1u << 16, kLboMN = (kBlockBytes >> 4) << 16;
+constexpr uint32_t kBlk16 = kBlockBytes >> 4;  // one block in 16-byte units
+
+__device__ __forceinline__ uint64_t dsc(uint32_t lo) { return (static_cast<uint64_t>(kDescHi) << 32) | lo; }
 
 // D (+)= A B over the 32 features, both operands K-major blocks with hi in columns
-// 0..31 and lo in columns 32..63: hi.hi + hi.lo + lo.hi (six K = 16 steps).
+// 0..31 and lo in columns 32..63: hi.hi + hi.lo + lo.hi (six K = 16 steps; a step of 16
+// columns is 32 bytes).  a, b: low descriptor words of K-major blocks.
 template <int N>
 __device__ __forceinline__ void mma_feat3(uint32_t d, uint32_t a, uint32_t b, uint32_t acc) {
     constexpr uint32_t id = idesc_bf16(128, N, 0, 0);
-    umma_bf16(d, dsc(a, 16), dsc(b, 16), id, acc);
-    umma_bf16(d, dsc(a + 32, 16), dsc(b + 32, 16), id, 1u);
-    umma_bf16(d, dsc(a, 16), dsc(b + 64, 16), id, 1u);
-    umma_bf16(d, dsc(a + 32, 16), dsc(b + 96, 16), id, 1u);
-    umma_bf16(d, dsc(a + 64, 16), dsc(b, 16), id, 1u);
-    umma_bf16(d, dsc(a + 96, 16), dsc(b + 32, 16), id, 1u);
+    umma_bf16(d, dsc(a), dsc(b), id, acc);
+    umma_bf16(d, dsc(a + 2), dsc(b + 2), id, 1u);
+    umma_bf16(d, dsc(a), dsc(b + 4), id, 1u);
+    umma_bf16(d, dsc(a + 2), dsc(b + 6), id, 1u);
+    umma_bf16(d, dsc(a + 4), dsc(b), id, 1u);
+    umma_bf16(d, dsc(a + 6), dsc(b + 2), id, 1u);
 }
 
 // D (+)= A B over the 128 tokens of a tile (eight K = 16 steps).  K-major operands
 // span a 128 x 128 tile (two blocks); MN-major ones hold the tokens in their rows
-// (M = 128 reads the block after as columns 64..127).
+// (16 rows = 2 KiB per step; M = 128 reads the block after as columns 64..127).
 template <bool A_MN, bool B_MN, int N>
 __device__ __forceinline__ void mma_tok(uint32_t d, uint32_t a, uint32_t b, uint32_t acc) {
     constexpr uint32_t id = idesc_bf16(128, N, A_MN, B_MN);
 #pragma unroll
     for (int kk = 0; kk < 8; ++kk) {
-        const uint64_t ad = A_MN ? dsc(a + kk * 2048, kBlockBytes) : dsc(a + (kk >> 2) * kBlockBytes + (kk & 3) * 32, 16);
-        const uint64_t bd = B_MN ? dsc(b + kk * 2048, kBlockBytes) : dsc(b + (kk >> 2) * kBlockBytes + (kk & 3) * 32, 16);
-        umma_bf16(d, ad, bd, id, kk > 0 ? 1u : acc);
+        const uint32_t ka = A_MN ? kk * 128u : (kk >> 2) * kBlk16 + (kk & 3) * 2u;
+        const uint32_t kb = B_MN ? kk * 128u : (kk >> 2) * kBlk16 + (kk & 3) * 2u;
+        umma_bf16(d, dsc(a + ka), dsc(b + kb), id, kk > 0 ? 1u : acc);
     }
+}
+
+// D (+)= A B over the 128 tokens with A in TMEM (bf16 pairs packed in the first 16 of each 32
+// columns: K elements 32g .. 32g + 31 of a row in columns a + 32g .. +15, so K step kk starts at
+// column 32 (kk / 2) + 8 (kk % 2)); B MN-major
+template <int N>
+__device__ __forceinline__ void mma_ts_tok(uint32_t d, uint32_t a_tmem, uint32_t b, uint32_t acc) {
+    constexpr uint32_t id = idesc_bf16(128, N, 0, 1);
+#pragma unroll
+    for (int kk = 0; kk < 8; ++kk)
+        umma_bf16_ts(d, a_tmem + 32u * (kk >> 1) + 8u * (kk & 1), dsc(b + kk * 128u), id, kk > 0 ? 1u : acc);
 }
 
 // ------------------------------- epilogue helpers -------------------------------
@@ -205,6 +244,13 @@ __device__ __forceinline__ void load_row8(const float *base, int n, int head, in
     }
 }
 
+// 8 staged fp32 values, or zeros for a row beyond the sequence
+__device__ __forceinline__ void ld_stage8(const float *src, bool ok, float (&x)[8]) {
+    const float4 u = *reinterpret_cast<const float4 *>(src), w = *reinterpret_cast<const float4 *>(src + 4);
+    x[0] = ok ? u.x : 0.f; x[1] = ok ? u.y : 0.f; x[2] = ok ? u.z : 0.f; x[3] = ok ? u.w : 0.f;
+    x[4] = ok ? w.x : 0.f; x[5] = ok ? w.y : 0.f; x[6] = ok ? w.z : 0.f; x[7] = ok ? w.w : 0.f;
+}
+
 // the 32 column sums of a warp's 32 x 32 values: lane i returns the sum of column i
 __device__ __forceinline__ float reduce_scatter32(float (&x)[32], int lane) {
 #pragma unroll
@@ -248,61 +294,85 @@ __global__ void __launch_bounds__(kThreads, 1) hla3_tc_kernel(Params p) {
 
     if (issuer) {
         if (lane == 0) {
-            const uint32_t sb = smem_u32(smem);
-            auto ba = [&](int b) { return sb + (uint32_t)b * kBlockBytes; };
-            const uint32_t car = ba(bCar);
-            uint32_t n_tiles = 0;
+            const uint32_t sb4 = smem_u32(smem) >> 4;
+            auto lk = [&](int b) { return sb4 + (uint32_t)b * kBlk16 + kLboK; };   // K-major block
+            auto lm = [&](int b) { return sb4 + (uint32_t)b * kBlk16 + kLboMN; };  // MN-major block
+            const uint32_t car = lk(bCar);  // + 256 per 32-row carry operand
+            uint32_t n_tiles = 0, st_pend = 0, st_iss = 0;  // st_iss bit s: copies into stage s, mod 2
+            auto stage_copy = [&](int s, int head, int j) {  // pre-pass: tile j's Q, K, V into stage s
+                const int tok0 = j * kTile, rows = min(kTile, p.n - tok0);
+                const uint32_t bytes = (uint32_t)rows * kD * sizeof(float);
+                const size_t off = ((size_t)head * p.n + tok0) * kD;
+                uint8_t *dst = blk(kStage + 3 * s);
+                st_pend |= 1u << s;
+                st_iss ^= 1u << s;
+                mbar_arrive_expect_tx(&ms->bar[bSt0 + s], 3 * bytes);
+                bulk_load(dst, p.q + off, bytes, &ms->bar[bSt0 + s]);
+                bulk_load(dst + kBlockBytes, p.k + off, bytes, &ms->bar[bSt0 + s]);
+                bulk_load(dst + 2 * kBlockBytes, p.v + off, bytes, &ms->bar[bSt0 + s]);
+            };
             for (int item = blockIdx.x; item < items && !ms->abort_flag; item += gridDim.x) {
-                const int g = item % p.G;
+                const int head = item / p.G, g = item % p.G;
                 if (kPre && g == p.G - 1) continue;  // nobody reads the last segment's sums
                 const int j0 = g * p.L, j1 = min(p.M, j0 + p.L);
+                if (kPre) {  // the first two tiles' copies (both stages are free between items)
+                    stage_copy(n_tiles & 1, head, j0);
+                    if (j0 + 1 < j1) stage_copy((n_tiles + 1) & 1, head, j0 + 1);
+                }
                 for (int j = j0; j < j1; ++j, ++n_tiles) {
                     const uint32_t tp = n_tiles & 1;
                     if (!bar_wait(ms, bEp0, tp, p)) break;  // Q, K, V (and the carries) in shared memory
                     tc_fence_after();
                     if (kPre) {
-                        mma_tok<true, true, 64>(tb + kTCar + 0, ba(bK), ba(bK), 1u);    // S^K += K^T K
-                        mma_tok<true, true, 64>(tb + kTCar + 64, ba(bQ), ba(bQ), 1u);   // S^Q += Q^T Q
-                        mma_tok<true, true, 64>(tb + kTCar + 128, ba(bV), ba(bK), 1u);  // P^T += V^T K
+                        st_pend &= ~(1u << (n_tiles & 1));  // read by the epilogue
+                        if (j + 2 < j1) stage_copy(n_tiles & 1, head, j + 2);
+                        mma_tok<true, true, 64>(tb + kTCar + 0, lm(bK), lm(bK), 1u);    // S^K += K^T K
+                        mma_tok<true, true, 64>(tb + kTCar + 64, lm(bQ), lm(bQ), 1u);   // S^Q += Q^T Q
+                        mma_tok<true, true, 64>(tb + kTCar + 128, lm(bV), lm(bK), 1u);  // P^T += V^T K
                         umma_commit(&ms->bar[bEvO]);
                         continue;
                     }
-                    mma_feat3<128>(tb + kTA, ba(bQ), ba(bK), 0u);        // A = Q K^T
+                    mma_feat3<128>(tb + kTA, lk(bQ), lk(bK), 0u);        // A = Q K^T
                     umma_commit(&ms->bar[bEvA]);
-                    mma_feat3<32>(tb + kTQS, ba(bQ), car, 0u);           // Q S^K_p
-                    mma_feat3<32>(tb + kTKS, ba(bK), car + 4096, 0u);    // K S^Q_p
+                    mma_feat3<32>(tb + kTQS, lk(bQ), car, 0u);           // Q S^K_p
+                    mma_feat3<32>(tb + kTKS, lk(bK), car + 256, 0u);     // K S^Q_p
                     umma_commit(&ms->bar[bEvQ]);
+                    // carries that need only this tile's tokens, while the epilogue forms LA
+                    mma_tok<true, true, 64>(tb + kTCar + 0, lm(bK), lm(bK), 1u);      // S^K += K^T K
+                    mma_tok<true, true, 64>(tb + kTCar + 64, lm(bQ), lm(bQ), 1u);     // S^Q += Q^T Q
+                    mma_tok<true, true, 64>(tb + kTCar + 128, lm(bV), lm(bK), 1u);    // P^T += V^T K
                     if (!bar_wait(ms, bEp1, tp, p)) break;              // LA (hi, lo)
                     tc_fence_after();
-                    mma_tok<false, true, 64>(tb + kTY, ba(bLh), ba(bV), 0u);   // Y = LA V (hi | lo halves)
-                    mma_tok<false, true, 64>(tb + kTY, ba(bLl), ba(bV), 1u);
-                    mma_feat3<32>(tb + kTY, ba(bQ), car + 8192, 1u);           //   + Q P_p
-                    mma_tok<false, false, 128>(tb + kTA, ba(bLh), ba(bLh), 0u);  // C' = LA LA^T
-                    mma_tok<false, false, 128>(tb + kTA, ba(bLh), ba(bLl), 1u);
-                    mma_tok<false, false, 128>(tb + kTA, ba(bLl), ba(bLh), 1u);
+                    mma_tok<false, true, 64>(tb + kTY, lk(bLh), lm(bV), 0u);   // Y = LA V (hi | lo halves)
+                    mma_tok<false, true, 64>(tb + kTY, lk(bLl), lm(bV), 1u);
+                    mma_feat3<32>(tb + kTY, lk(bQ), car + 512, 1u);           //   + Q P_p
                     umma_commit(&ms->bar[bEvY]);
+                    // C' = LA LA^T while the epilogue forms Z', aV and Q S^K_p
+                    mma_tok<false, false, 128>(tb + kTA, lk(bLh), lk(bLh), 0u);
+                    mma_tok<false, false, 128>(tb + kTA, lk(bLh), lk(bLl), 1u);
+                    mma_tok<false, false, 128>(tb + kTA, lk(bLl), lk(bLh), 1u);
                     if (!bar_wait(ms, bEp2, tp, p)) break;              // Q S^K_p, aV, Z' (hi | lo)
                     tc_fence_after();
-                    mma_feat3<128>(tb + kTA, ba(bQS), ba(bQ), 1u);             // C' += (Q S^K_p) Q^T
-                    mma_tok<true, true, 64>(tb + kTG, ba(bLh), ba(bAV), 0u);   // G'' = LA^T aV
-                    mma_tok<true, true, 64>(tb + kTG, ba(bLl), ba(bAV), 1u);
-                    mma_tok<false, true, 64>(tb + kTY, ba(bLh), ba(bZ), 0u);   // num = LA Z'
-                    mma_tok<false, true, 64>(tb + kTY, ba(bLl), ba(bZ), 1u);
-                    mma_feat3<32>(tb + kTY, ba(bQ), car + 12288, 1u);          //   + Q F_p
-                    mma_tok<true, true, 64>(tb + kTCar + 0, ba(bK), ba(bK), 1u);      // S^K += K^T K
-                    mma_tok<true, true, 64>(tb + kTCar + 64, ba(bQ), ba(bQ), 1u);     // S^Q += Q^T Q
-                    mma_tok<true, true, 64>(tb + kTCar + 128, ba(bV), ba(bK), 1u);    // P^T += V^T K
-                    mma_tok<true, true, 64>(tb + kTCar + 192, ba(bAV), ba(bQS), 1u);  // F^T += aV^T (Q S^K_p)
+                    mma_feat3<128>(tb + kTA, lk(bQS), lk(bQ), 1u);             // C' += (Q S^K_p) Q^T
+                    mma_tok<true, true, 64>(tb + kTG, lm(bLh), lm(bAV), 0u);   // G'' = LA^T aV
+                    mma_tok<true, true, 64>(tb + kTG, lm(bLl), lm(bAV), 1u);
                     umma_commit(&ms->bar[bEvC]);
-                    if (!bar_wait(ms, bEp3, tp, p)) break;              // L . C' over LA, G'
+                    // while the epilogue forms L . C' and G': num = LA Z' + Q F_p, F^T += aV^T (Q S^K_p)
+                    mma_tok<false, true, 64>(tb + kTY, lk(bLh), lm(bZ), 0u);
+                    mma_tok<false, true, 64>(tb + kTY, lk(bLl), lm(bZ), 1u);
+                    mma_feat3<32>(tb + kTY, lk(bQ), car + 768, 1u);
+                    mma_tok<true, true, 64>(tb + kTCar + 192, lm(bAV), lm(bQS), 1u);
+                    if (!bar_wait(ms, bEp3, tp, p)) break;              // L . C' (packed over C'), G'
                     tc_fence_after();
-                    mma_tok<false, true, 64>(tb + kTY, ba(bLh), ba(bAV), 1u);  // num += (L . C') aV
-                    mma_tok<false, true, 64>(tb + kTY, ba(bLl), ba(bAV), 1u);
-                    mma_tok<true, true, 64>(tb + kTCar + 192, ba(bG), ba(bK), 1u);    // F^T += G'^T K
+                    mma_ts_tok<64>(tb + kTY, tb + kTA, lm(bAV), 1u);        // num += (L . C') aV: hi
+                    mma_ts_tok<64>(tb + kTY, tb + kTA + 16, lm(bAV), 1u);   //   and lo (packed in TMEM)
+                    mma_tok<true, true, 64>(tb + kTCar + 192, lm(bG), lm(bK), 1u);    // F^T += G'^T K
                     umma_commit(&ms->bar[bEvO]);
                 }
             }
-            if (ms->abort_flag) {  // MMAs in flight finish (bounded) before TMEM is released
+            if (ms->abort_flag) {  // copies and MMAs in flight finish (bounded) before release
+                for (int st = 0; st < 2; ++st)
+                    if ((st_pend >> st) & 1u) mbar_wait(&ms->bar[bSt0 + st], ((st_iss >> st) & 1u) ^ 1u, kBarWaitNs);
                 umma_commit(&ms->bar[bTear]);
                 mbar_wait(&ms->bar[bTear], 0, kBarWaitNs);
             }
@@ -314,8 +384,10 @@ __global__ void __launch_bounds__(kThreads, 1) hla3_tc_kernel(Params p) {
         const int r = 32 * qd + lane;
         const uint32_t lb = (uint32_t)(32 * qd) << 16;
         const uint32_t treg = tb + lb + kTCar + 64u * (uint32_t)cq;  // carry region cq, this warp's lanes
-        uint32_t n_tiles = 0;
-        float pq[8], pk[8], pv[8];  // fp32 rows (8 columns) of the tile to come
+        uint32_t n_tiles = 0, st_par = 0;
+        // tokens are read 4 threads to a row (a warp covers 8 consecutive rows, 1 KiB)
+        const int e_row = tid >> 2, e_c = (tid & 3) * 8;
+        float pq[8], pk[8], pv[8];  // sweep: fp32 (8 columns) of the tile to come
 
         // rows 0..63 of carry region cq (lanes of the quadrant-0 and -1 warps) folded into
         // ms->fold[cq] as the fp32 32 x 32 carry: hi and lo columns added, rows 32..63 onto 0..31
@@ -374,9 +446,11 @@ __global__ void __launch_bounds__(kThreads, 1) hla3_tc_kernel(Params p) {
                 tmem_st32(treg + 32, z);
                 tmem_st_wait();
             }
-            load_row8(p.q, p.n, head, j0 * kTile + r, 8 * cq, pq);
-            load_row8(p.k, p.n, head, j0 * kTile + r, 8 * cq, pk);
-            load_row8(p.v, p.n, head, j0 * kTile + r, 8 * cq, pv);
+            if (!kPre) {
+                load_row8(p.q, p.n, head, j0 * kTile + e_row, e_c, pq);
+                load_row8(p.k, p.n, head, j0 * kTile + e_row, e_c, pk);
+                load_row8(p.v, p.n, head, j0 * kTile + e_row, e_c, pv);
+            }
 
             // tiles j0 .. j1 - 1, then (j = j1) the segment totals once the last tile's MMAs are done
             for (int j = j0; j <= j1; ++j) {
@@ -385,14 +459,24 @@ __global__ void __launch_bounds__(kThreads, 1) hla3_tc_kernel(Params p) {
                 const bool totals = j == j1;
                 // ---- E0: Q, K, V -> hi | lo blocks; carries -> bf16 operands ----
                 if (!totals) {
-                    store_hl8(blk(bQ), r, 8 * cq, pq);
-                    store_hl8(blk(bK), r, 8 * cq, pk);
-                    store_hl8(blk(bV), r, 8 * cq, pv);
+                    if (kPre) {  // this tile's copies in stage n_tiles % 2 (rows beyond n are stale: zero)
+                        const int st = n_tiles & 1;
+                        bar_wait(ms, bSt0 + st, (st_par >> st) & 1u, p);
+                        st_par ^= 1u << st;
+                        const float *stg = reinterpret_cast<const float *>(blk(kStage + 3 * st)) + e_row * kD + e_c;
+                        const bool ok = tok0 + e_row < p.n;
+                        ld_stage8(stg, ok, pq);
+                        ld_stage8(stg + kBlockBytes / 4, ok, pk);
+                        ld_stage8(stg + kBlockBytes / 2, ok, pv);
+                    }
+                    store_hl8(blk(bQ), e_row, e_c, pq);
+                    store_hl8(blk(bK), e_row, e_c, pk);
+                    store_hl8(blk(bV), e_row, e_c, pv);
                     if (!kPre) {
                         float dp = 0.f;
 #pragma unroll
                         for (int u = 0; u < 8; ++u) dp = fmaf(pq[u], pk[u], dp);
-                        ms->sdp[cq][r] = dp;
+                        ms->sdp[e_c / 8][e_row] = dp;
                     }
                 }
                 if (!kPre || totals) {
@@ -418,13 +502,12 @@ __global__ void __launch_bounds__(kThreads, 1) hla3_tc_kernel(Params p) {
                 epi_arrive(ms, bEp0);
                 auto prefetch = [&]() {  // the next tile's rows load while this one is worked on
                     if (j + 1 < j1) {
-                        load_row8(p.q, p.n, head, tok0 + kTile + r, 8 * cq, pq);
-                        load_row8(p.k, p.n, head, tok0 + kTile + r, 8 * cq, pk);
-                        load_row8(p.v, p.n, head, tok0 + kTile + r, 8 * cq, pv);
+                        load_row8(p.q, p.n, head, tok0 + kTile + e_row, e_c, pq);
+                        load_row8(p.k, p.n, head, tok0 + kTile + e_row, e_c, pk);
+                        load_row8(p.v, p.n, head, tok0 + kTile + e_row, e_c, pv);
                     }
                 };
                 if (kPre) {
-                    prefetch();
                     bar_wait(ms, bEvO, tp, p);
                     tc_fence_after();
                     ++n_tiles;
@@ -507,29 +590,13 @@ __global__ void __launch_bounds__(kThreads, 1) hla3_tc_kernel(Params p) {
                 }
                 fence_async_smem();
                 epi_arrive(ms, bEp2);
-                prefetch();  // (after E2: K and V of this tile are no longer held)
-                // ---- E3: L . C' -> hi, lo (over LA); G' = Z' + LA^T aV -> hi | lo ----
+                // ---- E3: G' = Z' + LA^T aV -> hi | lo; L . C' -> hi, lo packed over C' in TMEM ----
+                // (each thread packs its own 32 columns into their first 16 (hi) and last 16 (lo),
+                // so no thread overwrites columns another still reads; LA stays in shared memory
+                // for the products issued meanwhile)
                 bar_wait(ms, bEvC, tp, p);
                 tc_fence_after();
                 {
-                    const bool blk_zero = cq > qd;
-#pragma unroll
-                    for (int hh = 0; hh < 32; hh += 16) {
-                        uint32_t c[16];
-                        tmem_ld16(tb + lb + kTA + 32 * cq + hh, c);
-                        tmem_ld_wait();
-#pragma unroll
-                        for (int jj = 0; jj < 16; jj += 8) {
-                            float x[8];
-#pragma unroll
-                            for (int u = 0; u < 8; ++u)
-                                x[u] = (!blk_zero && 32 * cq + hh + jj + u <= r) ? __uint_as_float(c[jj + u]) : 0.f;
-                            uint4 h, l;
-                            split8(x, h, l);
-                            st16(blk(bLh), r, 32 * cq + hh + jj, h);
-                            st16(blk(bLl), r, 32 * cq + hh + jj, l);
-                        }
-                    }
                     uint32_t g0[8], g1[8];
                     tmem_ld8(tb + lb + kTG + 8 * cq, g0);
                     tmem_ld8(tb + lb + kTG + 32 + 8 * cq, g1);
@@ -539,8 +606,27 @@ __global__ void __launch_bounds__(kThreads, 1) hla3_tc_kernel(Params p) {
                     for (int u = 0; u < 8; ++u) gf[u] = zf[u] + (__uint_as_float(g0[u]) + __uint_as_float(g1[u]));
                     store_hl8(blk(bG), r, 8 * cq, gf);
                 }
+                {
+                    uint32_t c[32];
+                    tmem_ld32(tb + lb + kTA + 32 * cq, c);
+                    tmem_ld_wait();
+                    const bool blk_zero = cq > qd;
+                    uint32_t hp[16], lp[16];
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) {
+                        const int c0 = 32 * cq + 2 * i;
+                        const float x0 = (!blk_zero && c0 <= r) ? __uint_as_float(c[2 * i]) : 0.f;
+                        const float x1 = (!blk_zero && c0 + 1 <= r) ? __uint_as_float(c[2 * i + 1]) : 0.f;
+                        hp[i] = pack_bf16x2(x0, x1);
+                        lp[i] = pack_bf16x2(x0 - __uint_as_float(hp[i] << 16), x1 - __uint_as_float(hp[i] & 0xFFFF0000u));
+                    }
+                    tmem_st16(tb + lb + kTA + 32 * cq, hp);
+                    tmem_st16(tb + lb + kTA + 32 * cq + 16, lp);
+                    tmem_st_wait();
+                }
                 fence_async_smem();
                 epi_arrive(ms, bEp3);
+                prefetch();
                 // ---- E4: outputs ----
                 bar_wait(ms, bEvO, tp, p);
                 tc_fence_after();
@@ -570,38 +656,57 @@ __global__ void __launch_bounds__(kThreads, 1) hla3_tc_kernel(Params p) {
     }
 }
 
-// out[t] += q_t^T F_start(g) for the tiles of segments g >= 1 (F_start: F^T totals of
-// the segments before g); one block per tile of a head
+// out[t] += q_t^T F_start(g) for the tiles of segments g >= 1 (F_start: the F^T totals of the
+// segments before g); one block per tile of a head: the tile's Q rows and F_start staged in
+// shared memory, each thread forms 4 tokens x 4 outputs
 __global__ void __launch_bounds__(256) hla3_tc_fixup_kernel(const float *__restrict__ q, float *__restrict__ out,
                                                              const float *__restrict__ dF, int n, int G, int L) {
-    __shared__ float F[kD][kD + 1];  // F^T[j][f]
-    const int head = blockIdx.y, j = blockIdx.x + L, g = j / L;
-    for (int i = threadIdx.x; i < kD * kD; i += blockDim.x) {
+    __shared__ __align__(16) float Qs[kTile][kD + 4];
+    __shared__ __align__(16) float Fs[kD][kD + 4];  // Fs[f][j] = F_start[f][j]
+    const int head = blockIdx.y, j = blockIdx.x + L, g = j / L, tok0 = j * kTile;
+    for (int e = threadIdx.x; e < kD * kD; e += blockDim.x) {
+        const float *src = dF + (size_t)head * G * 1024 + e;  // F^T[jv][f], e = jv * 32 + f
         float s = 0.f;
-        for (int h = 0; h < g; ++h) s += __ldcg(dF + ((size_t)head * G + h) * 1024 + i);
-        F[i / kD][i % kD] = s;
+#pragma unroll 4
+        for (int h = 0; h < g; ++h) s += __ldcg(src + (size_t)h * 1024);
+        Fs[e % kD][e / kD] = s;
+    }
+    for (int e = threadIdx.x; e < kTile * kD / 4; e += blockDim.x) {
+        const int row = e / (kD / 4), c4 = (e % (kD / 4)) * 4;
+        float4 x = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (tok0 + row < n) x = __ldg(reinterpret_cast<const float4 *>(q + ((size_t)head * n + tok0 + row) * kD + c4));
+        *reinterpret_cast<float4 *>(&Qs[row][c4]) = x;
     }
     __syncthreads();
-    const int t = j * kTile + (threadIdx.x >> 1), c0 = (threadIdx.x & 1) * 16;
-    if (t >= n) return;
-    const float4 *qr = reinterpret_cast<const float4 *>(q + ((size_t)head * n + t) * kD);
-    float x[kD];
+    const int tg = threadIdx.x >> 3, c0 = (threadIdx.x & 7) * 4;  // tokens 4 tg .. +3, outputs c0 .. +3
+    float acc[4][4] = {};
+#pragma unroll 8
+    for (int f = 0; f < kD; f += 4) {
+        float4 qv[4], fv[4];
 #pragma unroll
-    for (int f = 0; f < kD / 4; ++f) {
-        const float4 u = __ldg(qr + f);
-        x[4 * f] = u.x; x[4 * f + 1] = u.y; x[4 * f + 2] = u.z; x[4 * f + 3] = u.w;
+        for (int i = 0; i < 4; ++i) qv[i] = *reinterpret_cast<const float4 *>(&Qs[4 * tg + i][f]);
+#pragma unroll
+        for (int u = 0; u < 4; ++u) fv[u] = *reinterpret_cast<const float4 *>(&Fs[f + u][c0]);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const float qq[4] = {qv[i].x, qv[i].y, qv[i].z, qv[i].w};
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                acc[i][0] += qq[u] * fv[u].x;
+                acc[i][1] += qq[u] * fv[u].y;
+                acc[i][2] += qq[u] * fv[u].z;
+                acc[i][3] += qq[u] * fv[u].w;
+            }
+        }
     }
-    float4 *orow = reinterpret_cast<float4 *>(out + ((size_t)head * n + t) * kD + c0);
 #pragma unroll
-    for (int c = 0; c < 16; c += 4) {
-        float4 o = orow[c / 4];
-        float a[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-        for (int f = 0; f < kD; ++f)
-#pragma unroll
-            for (int u = 0; u < 4; ++u) a[u] += x[f] * F[c0 + c + u][f];
-        o.x += a[0]; o.y += a[1]; o.z += a[2]; o.w += a[3];
-        orow[c / 4] = o;
+    for (int i = 0; i < 4; ++i) {
+        const int t = tok0 + 4 * tg + i;
+        if (t >= n) break;
+        float4 *o = reinterpret_cast<float4 *>(out + ((size_t)head * n + t) * kD + c0);
+        float4 x = *o;
+        x.x += acc[i][0]; x.y += acc[i][1]; x.z += acc[i][2]; x.w += acc[i][3];
+        *o = x;
     }
 }
 
