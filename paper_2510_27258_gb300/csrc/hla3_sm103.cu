@@ -34,11 +34,12 @@
 //     side by side (or the four hi/lo quadrants), summed by the epilogue.
 // The 128 x 128 operands (LA, then L . C') are separate hi and lo tiles.
 //
-// TMEM (512 columns): A -> C' (128), Y -> num (64), Q S^K_p and K S^Q_p (32 + 32,
-// then G'' = LA^T aV over them), and four 64-column carry regions holding the
-// hi/lo quadrants of K^T K, Q^T Q, V^T K (= P^T) and G'^T K + aV^T (Q S^K_p)
-// (= F^T).  Rows 64..127 of the carry products read the block after the
-// operand's own and are never used.
+// TMEM (512 columns): A -> C' -> L . C' packed (128), Y -> num (64), Q S^K_p and
+// K S^Q_p (32 + 32, then G'' = LA^T aV over them), and 64-column carry regions
+// holding the hi/lo quadrants of [K V]^T K (rows 0..63: S^K, rows 64..127: P^T, V's
+// block following K's), Q^T Q (= S^Q) and G'^T K + aV^T (Q S^K_p) (= F^T).  Rows
+// 64..127 of the other carry products read the block after the operand's own and
+// are never used.
 //
 // Roles: warp 16 issues the MMAs (one thread); warps 0..15 are the epilogue
 // (warp w: TMEM lanes 32 (w % 4) .. +31, one token row each; column block w / 4),
@@ -66,9 +67,12 @@ constexpr int kMaxSegments = 160;
 enum Block { bQ = 0, bK = 1, bV = 2, bQS = 3, bAV = 4, bZ = 5, bG = 6, bLh = 7, bLl = 9, bCar = 11, kBlocks = 12 };
 // bLh / bLl: 128 x 128 tiles (two blocks each): LA, then L . C', hi and lo parts.
 // bCar: four 32-row K-major operands (hi | lo): S^K_p, S^Q_p, P_p^T, F_p^T.
-// The pre-pass uses Q, K, V only; blocks kStage.. hold its two stages of fp32 tokens
-// (Q, K, V of one tile: 128 rows of 128 bytes each, copied as one contiguous piece).
-constexpr int kStage = 4;
+// The pre-pass alternates two sets of Q, K, V blocks (0..2 and 3..5: a tile's split runs
+// while the products of the tile before read the other set) and holds two stages of fp32
+// tokens in blocks 6..11 (Q, K, V of one tile: 128 rows of 128 bytes each, copied as one
+// contiguous piece per operand).
+constexpr int kStages = 2;
+__device__ __forceinline__ int stage_block(int s, int t) { return 6 + 3 * s + t; }
 constexpr uint32_t kSmemBlocks = kBlocks * kBlockBytes;
 
 // TMEM columns
@@ -79,7 +83,8 @@ enum Bar {
     bEp0 = 5, bEp1 = 6, bEp2 = 7, bEp3 = 8,            // epilogue hand-offs (16 warp arrivals)
     bTear = 9,
     bSt0 = 10,                                         // + stage: pre-pass token copies
-    kNumBars = 12
+    bEvO1 = 12,                                        // pre-pass: products of the second block set
+    kNumBars = 13
 };
 
 struct Misc {
@@ -303,33 +308,30 @@ __global__ void __launch_bounds__(kThreads, 1) hla3_tc_kernel(Params p) {
                 const int tok0 = j * kTile, rows = min(kTile, p.n - tok0);
                 const uint32_t bytes = (uint32_t)rows * kD * sizeof(float);
                 const size_t off = ((size_t)head * p.n + tok0) * kD;
-                uint8_t *dst = blk(kStage + 3 * s);
                 st_pend |= 1u << s;
                 st_iss ^= 1u << s;
                 mbar_arrive_expect_tx(&ms->bar[bSt0 + s], 3 * bytes);
-                bulk_load(dst, p.q + off, bytes, &ms->bar[bSt0 + s]);
-                bulk_load(dst + kBlockBytes, p.k + off, bytes, &ms->bar[bSt0 + s]);
-                bulk_load(dst + 2 * kBlockBytes, p.v + off, bytes, &ms->bar[bSt0 + s]);
+                bulk_load(blk(stage_block(s, 0)), p.q + off, bytes, &ms->bar[bSt0 + s]);
+                bulk_load(blk(stage_block(s, 1)), p.k + off, bytes, &ms->bar[bSt0 + s]);
+                bulk_load(blk(stage_block(s, 2)), p.v + off, bytes, &ms->bar[bSt0 + s]);
             };
             for (int item = blockIdx.x; item < items && !ms->abort_flag; item += gridDim.x) {
                 const int head = item / p.G, g = item % p.G;
                 if (kPre && g == p.G - 1) continue;  // nobody reads the last segment's sums
                 const int j0 = g * p.L, j1 = min(p.M, j0 + p.L);
-                if (kPre) {  // the first two tiles' copies (both stages are free between items)
-                    stage_copy(n_tiles & 1, head, j0);
-                    if (j0 + 1 < j1) stage_copy((n_tiles + 1) & 1, head, j0 + 1);
-                }
+                if (kPre)  // the first tiles' copies (every stage is free between items)
+                    for (int t = 0; t < kStages && j0 + t < j1; ++t) stage_copy((n_tiles + t) % kStages, head, j0 + t);
                 for (int j = j0; j < j1; ++j, ++n_tiles) {
                     const uint32_t tp = n_tiles & 1;
                     if (!bar_wait(ms, bEp0, tp, p)) break;  // Q, K, V (and the carries) in shared memory
                     tc_fence_after();
                     if (kPre) {
-                        st_pend &= ~(1u << (n_tiles & 1));  // read by the epilogue
-                        if (j + 2 < j1) stage_copy(n_tiles & 1, head, j + 2);
-                        mma_tok<true, true, 64>(tb + kTCar + 0, lm(bK), lm(bK), 1u);    // S^K += K^T K
-                        mma_tok<true, true, 64>(tb + kTCar + 64, lm(bQ), lm(bQ), 1u);   // S^Q += Q^T Q
-                        mma_tok<true, true, 64>(tb + kTCar + 128, lm(bV), lm(bK), 1u);  // P^T += V^T K
-                        umma_commit(&ms->bar[bEvO]);
+                        st_pend &= ~(1u << (n_tiles % kStages));  // read by the epilogue
+                        if (j + kStages < j1) stage_copy(n_tiles % kStages, head, j + kStages);
+                        const int o = 3 * (int)(n_tiles & 1);  // block set of this tile
+                        mma_tok<true, true, 64>(tb + kTCar + 0, lm(o + 1), lm(o + 1), 1u);   // [S^K; P^T] += [K V]^T K
+                        mma_tok<true, true, 64>(tb + kTCar + 64, lm(o), lm(o), 1u);          // S^Q += Q^T Q
+                        umma_commit(&ms->bar[(n_tiles & 1) ? bEvO1 : bEvO]);
                         continue;
                     }
                     mma_feat3<128>(tb + kTA, lk(bQ), lk(bK), 0u);        // A = Q K^T
@@ -338,9 +340,8 @@ __global__ void __launch_bounds__(kThreads, 1) hla3_tc_kernel(Params p) {
                     mma_feat3<32>(tb + kTKS, lk(bK), car + 256, 0u);     // K S^Q_p
                     umma_commit(&ms->bar[bEvQ]);
                     // carries that need only this tile's tokens, while the epilogue forms LA
-                    mma_tok<true, true, 64>(tb + kTCar + 0, lm(bK), lm(bK), 1u);      // S^K += K^T K
-                    mma_tok<true, true, 64>(tb + kTCar + 64, lm(bQ), lm(bQ), 1u);     // S^Q += Q^T Q
-                    mma_tok<true, true, 64>(tb + kTCar + 128, lm(bV), lm(bK), 1u);    // P^T += V^T K
+                    mma_tok<true, true, 64>(tb + kTCar + 0, lm(bK), lm(bK), 1u);   // [S^K; P^T] += [K V]^T K
+                    mma_tok<true, true, 64>(tb + kTCar + 64, lm(bQ), lm(bQ), 1u);  // S^Q += Q^T Q
                     if (!bar_wait(ms, bEp1, tp, p)) break;              // LA (hi, lo)
                     tc_fence_after();
                     mma_tok<false, true, 64>(tb + kTY, lk(bLh), lm(bV), 0u);   // Y = LA V (hi | lo halves)
@@ -371,7 +372,7 @@ __global__ void __launch_bounds__(kThreads, 1) hla3_tc_kernel(Params p) {
                 }
             }
             if (ms->abort_flag) {  // copies and MMAs in flight finish (bounded) before release
-                for (int st = 0; st < 2; ++st)
+                for (int st = 0; st < kStages; ++st)
                     if ((st_pend >> st) & 1u) mbar_wait(&ms->bar[bSt0 + st], ((st_iss >> st) & 1u) ^ 1u, kBarWaitNs);
                 umma_commit(&ms->bar[bTear]);
                 mbar_wait(&ms->bar[bTear], 0, kBarWaitNs);
@@ -383,7 +384,12 @@ __global__ void __launch_bounds__(kThreads, 1) hla3_tc_kernel(Params p) {
         const int qd = warp & 3, cq = warp >> 2;
         const int r = 32 * qd + lane;
         const uint32_t lb = (uint32_t)(32 * qd) << 16;
-        const uint32_t treg = tb + lb + kTCar + 64u * (uint32_t)cq;  // carry region cq, this warp's lanes
+        // carry cq (S^K, S^Q, P^T, F^T) lives in TMEM region 0, 1, 0, 3 (P^T in lanes 64..127 of the
+        // [K; V]^T K product); the two warps on its lanes fold it (c_half: rows 0..31 or 32..63)
+        const int c_reg = cq == 2 ? 0 : cq;
+        const bool c_act = cq == 2 ? qd >= 2 : qd < 2;
+        const int c_half = qd & 1;
+        const uint32_t treg = tb + lb + kTCar + 64u * (uint32_t)c_reg;  // this warp's lanes of it
         uint32_t n_tiles = 0, st_par = 0;
         // tokens are read 4 threads to a row (a warp covers 8 consecutive rows, 1 KiB)
         const int e_row = tid >> 2, e_c = (tid & 3) * 8;
@@ -394,7 +400,7 @@ __global__ void __launch_bounds__(kThreads, 1) hla3_tc_kernel(Params p) {
         auto carry_fold = [&]() {
 #pragma unroll
             for (int pass = 1; pass >= 0; --pass) {
-                if (qd == pass) {
+                if (c_act && c_half == pass) {
 #pragma unroll
                     for (int h = 0; h < 32; h += 16) {
                         uint32_t d0[16], d1[16];
@@ -420,11 +426,11 @@ __global__ void __launch_bounds__(kThreads, 1) hla3_tc_kernel(Params p) {
             if (kPre && g == p.G - 1) continue;
             const int j0 = g * p.L, j1 = min(p.M, j0 + p.L);
             // carries at the segment start: S^K, S^Q, P^T summed over the earlier segments, F = 0
-            if (qd < 2) {
+            if (c_act) {
                 uint32_t z[32];
 #pragma unroll
                 for (int f = 0; f < 32; ++f) z[f] = 0u;
-                if (!kPre && qd == 0 && cq < 3) {
+                if (!kPre && c_half == 0 && cq < 3) {
                     float s[32];
 #pragma unroll
                     for (int f = 0; f < 32; ++f) s[f] = 0.f;
@@ -460,24 +466,34 @@ __global__ void __launch_bounds__(kThreads, 1) hla3_tc_kernel(Params p) {
                 // ---- E0: Q, K, V -> hi | lo blocks; carries -> bf16 operands ----
                 if (!totals) {
                     if (kPre) {  // this tile's copies in stage n_tiles % 2 (rows beyond n are stale: zero)
-                        const int st = n_tiles & 1;
+                        const int st = n_tiles % kStages;
+                        if (n_tiles >= 2) {  // the products of tile n_tiles - 2 have read this block set
+                            bar_wait(ms, (n_tiles & 1) ? bEvO1 : bEvO, ((n_tiles >> 1) + 1) & 1, p);
+                            tc_fence_after();
+                        }
                         bar_wait(ms, bSt0 + st, (st_par >> st) & 1u, p);
                         st_par ^= 1u << st;
-                        const float *stg = reinterpret_cast<const float *>(blk(kStage + 3 * st)) + e_row * kD + e_c;
+                        const int so = e_row * kD + e_c;
                         const bool ok = tok0 + e_row < p.n;
-                        ld_stage8(stg, ok, pq);
-                        ld_stage8(stg + kBlockBytes / 4, ok, pk);
-                        ld_stage8(stg + kBlockBytes / 2, ok, pv);
+                        ld_stage8(reinterpret_cast<const float *>(blk(stage_block(st, 0))) + so, ok, pq);
+                        ld_stage8(reinterpret_cast<const float *>(blk(stage_block(st, 1))) + so, ok, pk);
+                        ld_stage8(reinterpret_cast<const float *>(blk(stage_block(st, 2))) + so, ok, pv);
                     }
-                    store_hl8(blk(bQ), e_row, e_c, pq);
-                    store_hl8(blk(bK), e_row, e_c, pk);
-                    store_hl8(blk(bV), e_row, e_c, pv);
+                    const int o = kPre ? 3 * (int)(n_tiles & 1) : 0;  // block set (Q, K, V at o, o + 1, o + 2)
+                    store_hl8(blk(o + bQ), e_row, e_c, pq);
+                    store_hl8(blk(o + bK), e_row, e_c, pk);
+                    store_hl8(blk(o + bV), e_row, e_c, pv);
                     if (!kPre) {
                         float dp = 0.f;
 #pragma unroll
                         for (int u = 0; u < 8; ++u) dp = fmaf(pq[u], pk[u], dp);
                         ms->sdp[e_c / 8][e_row] = dp;
                     }
+                }
+                if (kPre && totals && n_tiles > 0) {  // the last tile's products (and so all) are done
+                    const uint32_t c = n_tiles - 1;
+                    bar_wait(ms, (c & 1) ? bEvO1 : bEvO, (c >> 1) & 1, p);
+                    tc_fence_after();
                 }
                 if (!kPre || totals) {
                     carry_fold();
@@ -508,8 +524,6 @@ __global__ void __launch_bounds__(kThreads, 1) hla3_tc_kernel(Params p) {
                     }
                 };
                 if (kPre) {
-                    bar_wait(ms, bEvO, tp, p);
-                    tc_fence_after();
                     ++n_tiles;
                     continue;
                 }
@@ -658,44 +672,56 @@ __global__ void __launch_bounds__(kThreads, 1) hla3_tc_kernel(Params p) {
 
 // out[t] += q_t^T F_start(g) for the tiles of segments g >= 1 (F_start: the F^T totals of the
 // segments before g); one block per tile of a head: the tile's Q rows and F_start staged in
-// shared memory, each thread forms 4 tokens x 4 outputs
+// shared memory, each thread forms 4 tokens x 4 outputs.  Every global load (Q rows, the
+// thread's outputs, the totals) is issued before the first shared-memory store.
 __global__ void __launch_bounds__(256) hla3_tc_fixup_kernel(const float *__restrict__ q, float *__restrict__ out,
                                                              const float *__restrict__ dF, int n, int G, int L) {
     __shared__ __align__(16) float Qs[kTile][kD + 4];
     __shared__ __align__(16) float Fs[kD][kD + 4];  // Fs[f][j] = F_start[f][j]
     const int head = blockIdx.y, j = blockIdx.x + L, g = j / L, tok0 = j * kTile;
-    for (int e = threadIdx.x; e < kD * kD; e += blockDim.x) {
-        const float *src = dF + (size_t)head * G * 1024 + e;  // F^T[jv][f], e = jv * 32 + f
-        float s = 0.f;
-#pragma unroll 4
-        for (int h = 0; h < g; ++h) s += __ldcg(src + (size_t)h * 1024);
-        Fs[e % kD][e / kD] = s;
+    const int tid = threadIdx.x;
+    const int tg = tid >> 3, c0 = (tid & 7) * 4;  // tokens 4 tg .. +3, outputs c0 .. +3
+    float4 qv[4], ov[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {  // Q rows: element e = tid + 256 i of the tile's 128 x 8 float4
+        const int e = tid + 256 * i, row = e >> 3, c4 = (e & 7) * 4;
+        qv[i] = tok0 + row < n ? __ldg(reinterpret_cast<const float4 *>(q + ((size_t)head * n + tok0 + row) * kD + c4))
+                               : make_float4(0.f, 0.f, 0.f, 0.f);
     }
-    for (int e = threadIdx.x; e < kTile * kD / 4; e += blockDim.x) {
-        const int row = e / (kD / 4), c4 = (e % (kD / 4)) * 4;
-        float4 x = make_float4(0.f, 0.f, 0.f, 0.f);
-        if (tok0 + row < n) x = __ldg(reinterpret_cast<const float4 *>(q + ((size_t)head * n + tok0 + row) * kD + c4));
-        *reinterpret_cast<float4 *>(&Qs[row][c4]) = x;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const int t = tok0 + 4 * tg + i;
+        ov[i] = t < n ? *reinterpret_cast<const float4 *>(out + ((size_t)head * n + t) * kD + c0)
+                      : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+    float fs[4] = {0.f, 0.f, 0.f, 0.f};  // F^T elements tid + 256 i summed over the earlier segments
+    for (int h = 0; h < g; ++h)
+#pragma unroll
+        for (int i = 0; i < 4; ++i) fs[i] += __ldcg(dF + ((size_t)head * G + h) * 1024 + tid + 256 * i);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const int e = tid + 256 * i;
+        *reinterpret_cast<float4 *>(&Qs[e >> 3][(e & 7) * 4]) = qv[i];
+        Fs[e % kD][e / kD] = fs[i];
     }
     __syncthreads();
-    const int tg = threadIdx.x >> 3, c0 = (threadIdx.x & 7) * 4;  // tokens 4 tg .. +3, outputs c0 .. +3
     float acc[4][4] = {};
 #pragma unroll 8
     for (int f = 0; f < kD; f += 4) {
-        float4 qv[4], fv[4];
+        float4 a4[4], f4[4];
 #pragma unroll
-        for (int i = 0; i < 4; ++i) qv[i] = *reinterpret_cast<const float4 *>(&Qs[4 * tg + i][f]);
+        for (int i = 0; i < 4; ++i) a4[i] = *reinterpret_cast<const float4 *>(&Qs[4 * tg + i][f]);
 #pragma unroll
-        for (int u = 0; u < 4; ++u) fv[u] = *reinterpret_cast<const float4 *>(&Fs[f + u][c0]);
+        for (int u = 0; u < 4; ++u) f4[u] = *reinterpret_cast<const float4 *>(&Fs[f + u][c0]);
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
-            const float qq[4] = {qv[i].x, qv[i].y, qv[i].z, qv[i].w};
+            const float qq[4] = {a4[i].x, a4[i].y, a4[i].z, a4[i].w};
 #pragma unroll
             for (int u = 0; u < 4; ++u) {
-                acc[i][0] += qq[u] * fv[u].x;
-                acc[i][1] += qq[u] * fv[u].y;
-                acc[i][2] += qq[u] * fv[u].z;
-                acc[i][3] += qq[u] * fv[u].w;
+                acc[i][0] += qq[u] * f4[u].x;
+                acc[i][1] += qq[u] * f4[u].y;
+                acc[i][2] += qq[u] * f4[u].z;
+                acc[i][3] += qq[u] * f4[u].w;
             }
         }
     }
@@ -703,10 +729,9 @@ __global__ void __launch_bounds__(256) hla3_tc_fixup_kernel(const float *__restr
     for (int i = 0; i < 4; ++i) {
         const int t = tok0 + 4 * tg + i;
         if (t >= n) break;
-        float4 *o = reinterpret_cast<float4 *>(out + ((size_t)head * n + t) * kD + c0);
-        float4 x = *o;
+        float4 x = ov[i];
         x.x += acc[i][0]; x.y += acc[i][1]; x.z += acc[i][2]; x.w += acc[i][3];
-        *o = x;
+        *reinterpret_cast<float4 *>(out + ((size_t)head * n + t) * kD + c0) = x;
     }
 }
 
