@@ -235,6 +235,15 @@ int hla3_forward_path(int B, int H, int n, int d, int dv, int masked, int normal
                       int has_state_in, int has_state_out, int *launches);
 
 /*
+ * hla2_backward_path -- which CUDA path hla2_backward takes for these arguments
+ * on the current device, without launching anything: 1 the tensor-core kernel
+ * (bf16 tokens, d = dv = 64, normalized = 0, an sm_103 device; one launch),
+ * 0 the fp32 CUDA-core kernels (five launches), -1 the arguments are not
+ * supported.
+ */
+int hla2_backward_path(int B, int H, int n, int d, int dv, int normalized, int chunk, hla_dtype dt);
+
+/*
  * hla2_forward_noalloc -- hla2_forward for callers that cannot allocate device
  * memory (no counterpart in the paper: it only changes where scratch lives).
  *

@@ -240,6 +240,17 @@ hla_status hla2_backward(const void *q, const void *k, const void *v, const void
     return cuda_status(backward2_launch(p, reinterpret_cast<cudaStream_t>(stream)), "backward");
 }
 
+int hla2_backward_path(int B, int H, int n, int d, int dv, int normalized, int chunk, hla_dtype dt) {
+    const void *dummy = reinterpret_cast<const void *>(uintptr_t(256));
+    if (check_forward(dummy, dummy, dummy, const_cast<void *>(dummy), dt, B, H, n, d, dv, 1, normalized, 0.f, chunk,
+                      nullptr, nullptr) != HLA_OK)
+        return -1;
+    Bwd2 p{dummy, dummy, dummy, dummy, const_cast<void *>(dummy), const_cast<void *>(dummy),
+           const_cast<void *>(dummy), dt, B * H, n, d, dv, normalized, 0.f, chunk, nullptr,
+           hla2_backward_workspace_bytes(B, H, n, d, dv, chunk, dt)};
+    return ((long long)B * H > 0 && backward2_tc_applicable(p)) ? 1 : 0;
+}
+
 size_t ahla_state_floats(int d, int dv) {
     if (d <= 0 || dv <= 0) return 0;
     return 2 * (size_t)d * dv + 2 * (size_t)d;

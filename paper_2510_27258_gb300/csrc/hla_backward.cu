@@ -367,10 +367,12 @@ cudaError_t backward_t(const Bwd2 &p, cudaStream_t s) {
 
 size_t backward2_workspace_bytes(int BH, int n, int d, int dv, int chunk) {
     const BLayout L = make_layout(BH, n, d, dv, chunk);
-    return kWsHeaderBytes + sizeof(float) * (size_t)L.total;
+    const size_t simt = kWsHeaderBytes + sizeof(float) * (size_t)L.total, tc = backward2_tc_workspace_bytes(BH, n);
+    return simt > tc ? simt : tc;
 }
 
 cudaError_t backward2_launch(const Bwd2 &p, cudaStream_t stream) {
+    if (backward2_tc_applicable(p)) return backward2_tc_launch(p, stream);
     return p.dt == HLA_BF16 ? backward_t<__nv_bfloat16>(p, stream) : backward_t<float>(p, stream);
 }
 

@@ -1,0 +1,609 @@
+// Backward of masked second-order HLA on the tensor cores (sm_103a): tcgen05 MMAs
+// with TMEM accumulators, TMA tile loads, one persistent CTA per head.
+//
+// The gradients are the adjoint of the chunked forward (Sec. "Chunk-parallel
+// training via associative scans": the reverse scan with the adjoint of the
+// semidirect product, checkpoints at tile boundaries).  With x_j = S_j q_j,
+// T_tj = q_t . x_j and P_tj = g_t . v_j (both for j <= t), per 128-token tile
+// (rows = tokens; p = prefix before the tile, s = suffix after it):
+//   forward:  W = L . (Q K^T),  X = W K + Q S_p,  T = L . (Q X^T)
+//   backward: P = L . (G V^T),  Y = P^T Q + V Gam_s     (y_j = sum_{t>=j} P_tj q_t)
+//             dV = T^T G + X Gam_s^T
+//             B = L . (Y K^T)
+//             dQ = P X + G D_p^T + Y S_p + B K
+//             dK = K Lam_s + W^T Y + B^T Q
+// with the forward prefixes S_p = sum k k^T, D_p = sum x v^T and the suffix sums
+// Gam_s^T = sum q g^T and Lam_s = sum (y q^T + q y^T), which the reverse sweep
+// carries as Gam^T += Q^T G, Lam += Y^T Q + Q^T Y.
+//
+// One kernel, per head: a forward sweep over the tiles carries S and D in TMEM
+// and stores, before each tile, S_p and D_p as bf16 checkpoints (the swizzled
+// shared-memory image, by 1-D bulk copies); a reverse sweep reloads them and
+// carries Gam^T and Lam in TMEM.  No CTA waits on another.
+//
+// Operands are bf16 in the 128-byte-swizzled layout TMA writes (128 rows x 64
+// columns per 16 KiB block; 64 x 64 matrices in the first 64 rows of an 8 KiB
+// half); every product accumulates in fp32.  The transposed uses (P^T, T^T, W^T,
+// B^T, and X^T, Y^T, Q^T, K^T of the carries) read the same tiles MN-major; a
+// 64-wide operand read as the M side of an M = 128 product takes the block after
+// it as rows 64..127, which land in TMEM lanes nobody reads.
+//
+// TMEM (512 columns): R0 (128) A -> T -> [dQ | dK]; R1 (128) G V^T -> B;
+// R2 (64) X -> dV; R3 (64) Y; R4, R5 (64 each) the carries (forward S, D;
+// reverse Gam^T, Lam), rows 0..63.
+//
+// Roles: warp 16 issues TMA copies and MMAs (one thread); warps 0..15 are the
+// epilogue (warp w: TMEM lanes 32 (w % 4) .. +31, one token row each; column
+// quarter w / 4).
+//
+// Scope: bf16 tokens, d = dv = 64, masked, plain (unnormalised) output.
+#include <cstdlib>
+
+#include "hla_internal.h"
+#include "sm103_prims.cuh"
+
+namespace hla {
+namespace {
+
+using namespace sm103;
+
+constexpr int kTile = 128, kD = 64;
+constexpr int kEpiWarps = 16, kEpiThreads = kEpiWarps * 32, kIssuerWarp = kEpiWarps;
+constexpr int kThreads = kEpiThreads + 32;
+
+// shared-memory blocks of 16 KiB (128 rows x 64 bf16)
+enum Block {
+    bQ = 0, bK = 1, bV = 2, bG = 3,
+    bW = 4,    // 4..5: W = L . (Q K^T), 128 x 128
+    bP = 6,    // 6..7: P = L . (G V^T); forward sweep: the second Q, K, V set at 6, 7, 8
+    bT = 8,    // 8..9: T, then B
+    bX = 10, bY = 11,
+    bCk = 12,  // S_p (rows 0..63 of the first 8 KiB), D_p (the second 8 KiB): the checkpoint image
+    bCar = 13, // Gam_s^T (first 8 KiB), Lam_s (second 8 KiB), bf16 copies of the reverse carries
+    kBlocks = 14
+};
+constexpr uint32_t kHalf = kBlockBytes / 2;
+constexpr uint32_t kSmemBlocks = kBlocks * kBlockBytes;
+constexpr uint32_t kCkBytes = kBlockBytes;  // one checkpoint: S_p and D_p images
+
+constexpr uint32_t kR0 = 0, kR1 = 128, kR2 = 256, kR3 = 320, kR4 = 384, kR5 = 448;  // TMEM columns
+
+enum Bar {
+    bLd0 = 0, bLd1 = 1,                                        // tile copies (forward: two sets)
+    bEvA = 2, bEvX = 3, bEvT = 4, bEvB = 5, bEvV = 6, bEvO = 7, bEvC = 8,  // MMA commits
+    bEp0 = 9, bEp1 = 10, bEp2 = 11, bEp3 = 12, bEp4 = 13,    // epilogue hand-offs (16 warp arrivals)
+    bTear = 14,
+    bCkDone = 15,                                              // a head's checkpoints are in global memory
+    kNumBars = 16
+};
+
+struct Misc {
+    uint64_t bar[kNumBars];
+    uint32_t tmem_base;
+    int abort_flag;
+};
+constexpr uint32_t kMiscBytes = 1024;
+static_assert(sizeof(Misc) <= kMiscBytes, "misc smem");
+constexpr uint32_t kSmemBytes = kSmemBlocks + kMiscBytes;
+
+struct Params {
+    __nv_bfloat16 *dq, *dk, *dv;
+    uint8_t *ck;  // [BH][M] checkpoints of kCkBytes
+    int BH, n, M;
+    WsHeader *err;
+};
+
+constexpr unsigned long long kBarWaitNs = 2000000000ull;
+
+__device__ __forceinline__ void set_error(WsHeader *err, unsigned where, unsigned detail) {
+    if (atomicCAS(&err->error, 0u, (unsigned)kDevTimeout) == 0u) {
+        err->where = where;
+        err->detail = detail;
+    }
+}
+
+__device__ __forceinline__ bool bar_wait(Misc *ms, int b, uint32_t parity, const Params &p) {
+    if (ms->abort_flag) return false;
+    if (mbar_wait(&ms->bar[b], parity, kBarWaitNs)) return true;
+    set_error(p.err, 500 + b, parity);
+    ms->abort_flag = 1;
+    return false;
+}
+
+__device__ __forceinline__ void epi_sync() { asm volatile("bar.sync 1, %0;" ::"n"(kEpiThreads) : "memory"); }
+
+__device__ __forceinline__ void epi_arrive(Misc *ms, int b) {
+    tc_fence_before();
+    __syncwarp();
+    if ((threadIdx.x & 31) == 0) mbar_arrive(&ms->bar[b]);
+}
+
+// 1-D bulk copies between global and shared memory (16-byte aligned, sizes a multiple of 16)
+__device__ __forceinline__ void bulk_load(void *dst, const void *src, uint32_t bytes, uint64_t *bar) {
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+                 ::"r"(smem_u32(dst)), "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(smem_u32(bar))
+                 : "memory");
+}
+__device__ __forceinline__ void bulk_store(void *dst, const void *src, uint32_t bytes) {
+    asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;"
+                 ::"l"(reinterpret_cast<uint64_t>(dst)), "r"(smem_u32(src)), "r"(bytes)
+                 : "memory");
+}
+__device__ __forceinline__ void bulk_prefetch_l2(const void *src, uint32_t bytes) {
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(reinterpret_cast<uint64_t>(src)), "r"(bytes)
+                 : "memory");
+}
+
+// ------------------------------- MMA issue -------------------------------
+constexpr uint32_t kDescHi = (1024u >> 4) | (1u << 14) | (2u << 29);
+constexpr uint32_t kLboK = 1u << 16, kLboMN = (kBlockBytes >> 4) << 16;
+constexpr uint32_t kBlk16 = kBlockBytes >> 4;
+
+__device__ __forceinline__ uint64_t dsc(uint32_t lo) { return (static_cast<uint64_t>(kDescHi) << 32) | lo; }
+
+// D (+)= A B over KS steps of K = 16.  K-major operands: 64 K elements per 128-byte row,
+// the next 64 in the next block; MN-major operands: 16 K rows (2 KiB) per step.
+template <bool A_MN, bool B_MN, int N, int KS>
+__device__ __forceinline__ void mma(uint32_t d, uint32_t a, uint32_t b, uint32_t acc) {
+    constexpr uint32_t id = idesc_bf16(128, N, A_MN, B_MN);
+#pragma unroll
+    for (int kk = 0; kk < KS; ++kk) {
+        const uint32_t ka = A_MN ? kk * 128u : (kk >> 2) * kBlk16 + (kk & 3) * 2u;
+        const uint32_t kb = B_MN ? kk * 128u : (kk >> 2) * kBlk16 + (kk & 3) * 2u;
+        umma_bf16(d, dsc(a + ka), dsc(b + kb), id, kk > 0 ? 1u : acc);
+    }
+}
+
+// ------------------------------- epilogue helpers -------------------------------
+__device__ __forceinline__ uint4 pack8(const float *x) {
+    return make_uint4(pack_bf16x2(x[0], x[1]), pack_bf16x2(x[2], x[3]), pack_bf16x2(x[4], x[5]),
+                      pack_bf16x2(x[6], x[7]));
+}
+
+__device__ __forceinline__ void st16(uint8_t *tile, int r, int c, const uint4 &v) {
+    *reinterpret_cast<uint4 *>(tile + tile_off(r, c)) = v;
+}
+
+// 32 fp32 TMEM values of row r (columns c0 .. c0 + 31 of a 128-wide result), masked to the
+// lower triangle (column <= r), as bf16 into a 128 x 128 tile
+__device__ __forceinline__ void store_masked32(uint8_t *tile, int r, int c0, const uint32_t (&a)[32]) {
+    const bool zero = c0 > r;
+#pragma unroll
+    for (int jj = 0; jj < 32; jj += 8) {
+        float x[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) x[u] = (!zero && c0 + jj + u <= r) ? __uint_as_float(a[jj + u]) : 0.f;
+        st16(tile, r, c0 + jj, pack8(x));
+    }
+}
+
+// 16 fp32 TMEM values (columns c0 .. c0 + 15 of a 64-wide result) as bf16 into row r of a block
+__device__ __forceinline__ void store16(uint8_t *blk, int r, int c0, const uint32_t (&a)[16]) {
+    float x[16];
+#pragma unroll
+    for (int u = 0; u < 16; ++u) x[u] = __uint_as_float(a[u]);
+    st16(blk, r, c0, pack8(x));
+    st16(blk, r, c0 + 8, pack8(x + 8));
+}
+
+// 16 fp32 TMEM values as bf16 into row `tok` of a [n][64] global array
+__device__ __forceinline__ void out16(__nv_bfloat16 *dst, const uint32_t (&a)[16]) {
+    float x[16];
+#pragma unroll
+    for (int u = 0; u < 16; ++u) x[u] = __uint_as_float(a[u]);
+    uint4 *d4 = reinterpret_cast<uint4 *>(dst);
+    d4[0] = pack8(x);
+    d4[1] = pack8(x + 8);
+}
+
+struct Tok {  // raw token pointers, for the L2 prefetch of the next reverse tile
+    const __nv_bfloat16 *q, *k, *v, *g;
+};
+
+__global__ void __launch_bounds__(kThreads, 1)
+bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
+              const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_g, Params p, Tok tok) {
+    extern __shared__ __align__(1024) uint8_t smem[];
+    Misc *ms = reinterpret_cast<Misc *>(smem + kSmemBlocks);
+    auto blk = [&](int b) { return smem + b * kBlockBytes; };
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const bool issuer = warp == kIssuerWarp;
+
+    if (smem_u32(smem) & 1023u) {  // the swizzled layout needs 1 KiB alignment
+        if (tid == 0) set_error(p.err, 499, smem_u32(smem));
+        return;
+    }
+    if (tid == 0) {
+        for (int b = 0; b < kNumBars; ++b) mbar_init(&ms->bar[b], (b >= bEp0 && b <= bEp4) ? kEpiWarps : 1);
+        ms->abort_flag = 0;
+        fence_mbar_init();
+    }
+    if (issuer) {
+        tmem_alloc(&ms->tmem_base, 512);
+        tmem_relinquish();
+        if (lane == 0) {
+            prefetch_tmap(&tm_q); prefetch_tmap(&tm_k); prefetch_tmap(&tm_v); prefetch_tmap(&tm_g);
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tb = ms->tmem_base;
+    const int M = p.M;
+
+    if (issuer) {
+        if (lane == 0) {
+            const uint32_t sb4 = smem_u32(smem) >> 4;
+            auto lk = [&](int b) { return sb4 + (uint32_t)b * kBlk16 + kLboK; };   // K-major block
+            auto lm = [&](int b) { return sb4 + (uint32_t)b * kBlk16 + kLboMN; };  // MN-major block
+            constexpr uint32_t kH16 = kHalf >> 4;  // the second 8 KiB of a block
+            // tile counters: n_s every tile of both sweeps (the barriers both use), n_f forward
+            // tiles, n_b reverse tiles
+            uint32_t ld_par = 0, ld_pend = 0, n_s = 0, n_f = 0, n_b = 0, n_head = 0;
+            auto load_fwd = [&](int set, int head, int j) {  // Q, K, V of tile j into blocks 0..2 or 6..8
+                const int b0 = set ? bP : bQ;
+                ld_pend |= 1u << set;
+                mbar_arrive_expect_tx(&ms->bar[bLd0 + set], 3 * kBlockBytes);
+                tma_load_3d(blk(b0), &tm_q, &ms->bar[bLd0 + set], 0, j * kTile, head);
+                tma_load_3d(blk(b0 + 1), &tm_k, &ms->bar[bLd0 + set], 0, j * kTile, head);
+                tma_load_3d(blk(b0 + 2), &tm_v, &ms->bar[bLd0 + set], 0, j * kTile, head);
+            };
+            auto load_bwd = [&](int head, int j) {  // Q, K, V, G of tile j and its checkpoint
+                ld_pend |= 1u;
+                mbar_arrive_expect_tx(&ms->bar[bLd0], 4 * kBlockBytes + kCkBytes);
+                tma_load_3d(blk(bQ), &tm_q, &ms->bar[bLd0], 0, j * kTile, head);
+                tma_load_3d(blk(bK), &tm_k, &ms->bar[bLd0], 0, j * kTile, head);
+                tma_load_3d(blk(bV), &tm_v, &ms->bar[bLd0], 0, j * kTile, head);
+                tma_load_3d(blk(bG), &tm_g, &ms->bar[bLd0], 0, j * kTile, head);
+                bulk_load(blk(bCk), p.ck + ((size_t)head * M + j) * kCkBytes, kCkBytes, &ms->bar[bLd0]);
+            };
+            auto wait_ld = [&](int set) {
+                if (!bar_wait(ms, bLd0 + set, (ld_par >> set) & 1u, p)) return false;
+                ld_par ^= 1u << set;
+                ld_pend &= ~(1u << set);
+                return true;
+            };
+            for (int head = blockIdx.x; head < p.BH && !ms->abort_flag; head += gridDim.x, ++n_head) {
+                // ---------------- forward sweep: checkpoints of S and D ----------------
+                load_fwd(0, head, 0);
+                if (M > 1) load_fwd(1, head, 1);
+                bool ok = true;
+                for (int j = 0; j < M && ok; ++j, ++n_f, ++n_s) {
+                    const uint32_t tp = n_s & 1, tf = n_f & 1;
+                    const int set = j & 1, qb = set ? bP : bQ;
+                    ok = false;
+                    if (!bar_wait(ms, bEp0, tp, p) || !wait_ld(set)) break;  // S_p (bf16) in bCk; tokens
+                    tc_fence_after();
+                    mma<false, false, 128, 4>(tb + kR0, lk(qb), lk(qb + 1), 0u);   // A = Q K^T
+                    umma_commit(&ms->bar[bEvA]);
+                    if (!bar_wait(ms, bEp1, tp, p)) break;                        // W in bW
+                    tc_fence_after();
+                    mma<false, true, 64, 8>(tb + kR2, lk(bW), lm(qb + 1), 0u);     // X = W K
+                    mma<false, false, 64, 4>(tb + kR2, lk(qb), lk(bCk), 1u);       //   + Q S_p
+                    umma_commit(&ms->bar[bEvX]);
+                    if (!bar_wait(ms, bEp2, tp, p)) break;                        // X (bf16) in bX
+                    tc_fence_after();
+                    mma<true, true, 64, 8>(tb + kR4, lm(qb + 1), lm(qb + 1), 1u);  // S += K^T K
+                    mma<true, true, 64, 8>(tb + kR5, lm(bX), lm(qb + 2), 1u);      // D += X^T V
+                    umma_commit(&ms->bar[bEvC]);
+                    if (!bar_wait(ms, bEvC, tf, p)) break;                        // this set is free again
+                    if (j + 2 < M) load_fwd(set, head, j + 2);
+                    ok = true;
+                }
+                if (!ok) break;
+                // the checkpoints are in global memory (the epilogue waited for its copies)
+                if (!bar_wait(ms, bCkDone, n_head & 1, p)) break;
+                // ---------------- reverse sweep: gradients ----------------
+                load_bwd(head, M - 1);
+                for (int j = M - 1; j >= 0 && ok; --j, ++n_b, ++n_s) {
+                    const uint32_t ts = n_s & 1, tp = n_b & 1;
+                    ok = false;
+                    if (j > 0) {  // the next tile's tokens and checkpoint towards L2
+                        const size_t t0 = (size_t)head * p.n + (size_t)(j - 1) * kTile;
+                        const uint32_t bytes = (uint32_t)min(kTile, p.n - (j - 1) * kTile) * kD * 2;
+                        bulk_prefetch_l2(tok.q + t0 * kD, bytes);
+                        bulk_prefetch_l2(tok.k + t0 * kD, bytes);
+                        bulk_prefetch_l2(tok.v + t0 * kD, bytes);
+                        bulk_prefetch_l2(tok.g + t0 * kD, bytes);
+                        bulk_prefetch_l2(p.ck + ((size_t)head * M + j - 1) * kCkBytes, kCkBytes);
+                    }
+                    if (!bar_wait(ms, bEp0, ts, p) || !wait_ld(0)) break;  // Gam^T, Lam (bf16); tokens
+                    tc_fence_after();
+                    mma<false, false, 128, 4>(tb + kR0, lk(bQ), lk(bK), 0u);        // A = Q K^T
+                    mma<false, false, 128, 4>(tb + kR1, lk(bG), lk(bV), 0u);        // G V^T
+                    umma_commit(&ms->bar[bEvA]);
+                    if (!bar_wait(ms, bEp1, ts, p)) break;            // W, P (bf16)
+                    tc_fence_after();
+                    mma<false, true, 64, 8>(tb + kR2, lk(bW), lm(bK), 0u);          // X = W K
+                    mma<false, false, 64, 4>(tb + kR2, lk(bQ), lk(bCk), 1u);        //   + Q S_p
+                    mma<true, true, 64, 8>(tb + kR3, lm(bP), lm(bQ), 0u);           // Y = P^T Q
+                    mma<false, false, 64, 4>(tb + kR3, lk(bV), lk(bCar), 1u);       //   + V Gam_s
+                    umma_commit(&ms->bar[bEvX]);
+                    if (!bar_wait(ms, bEp2, ts, p)) break;            // X, Y (bf16)
+                    tc_fence_after();
+                    mma<false, false, 128, 4>(tb + kR0, lk(bQ), lk(bX), 0u);        // T = Q X^T
+                    umma_commit(&ms->bar[bEvT]);
+                    mma<false, false, 128, 4>(tb + kR1, lk(bY), lk(bK), 0u);        // B = Y K^T
+                    umma_commit(&ms->bar[bEvB]);
+                    if (!bar_wait(ms, bEp3, tp, p)) break;                         // T (bf16) in bT
+                    tc_fence_after();
+                    mma<true, true, 64, 8>(tb + kR2, lm(bT), lm(bG), 0u);           // dV = T^T G
+                    mma<false, true, 64, 4>(tb + kR2, lk(bX), lm(bCar), 1u);        //   + X Gam_s^T
+                    umma_commit(&ms->bar[bEvV]);
+                    if (!bar_wait(ms, bEp4, tp, p)) break;                         // B (bf16) in bT
+                    tc_fence_after();
+                    mma<false, true, 64, 8>(tb + kR0, lk(bP), lm(bX), 0u);          // dQ = P X
+                    mma<false, false, 64, 4>(tb + kR0, lk(bG), lk(bCk) + kH16, 1u); //   + G D_p^T
+                    mma<false, false, 64, 4>(tb + kR0, lk(bY), lk(bCk), 1u);        //   + Y S_p
+                    mma<false, true, 64, 8>(tb + kR0, lk(bT), lm(bK), 1u);          //   + B K
+                    mma<false, false, 64, 4>(tb + kR0 + 64, lk(bK), lk(bCar) + kH16, 0u);  // dK = K Lam_s
+                    mma<true, true, 64, 8>(tb + kR0 + 64, lm(bW), lm(bY), 1u);      //   + W^T Y
+                    mma<true, true, 64, 8>(tb + kR0 + 64, lm(bT), lm(bQ), 1u);      //   + B^T Q
+                    mma<true, true, 64, 8>(tb + kR4, lm(bQ), lm(bG), 1u);           // Gam^T += Q^T G
+                    mma<true, true, 64, 8>(tb + kR5, lm(bY), lm(bQ), 1u);           // Lam += Y^T Q
+                    mma<true, true, 64, 8>(tb + kR5, lm(bQ), lm(bY), 1u);           //   + Q^T Y
+                    umma_commit(&ms->bar[bEvO]);
+                    if (!bar_wait(ms, bEvO, tp, p)) break;                         // every operand read
+                    if (j > 0) load_bwd(head, j - 1);
+                    ok = true;
+                }
+                if (!ok) break;
+            }
+            if (ms->abort_flag) {  // copies and MMAs in flight finish (bounded) before release
+                for (int s = 0; s < 2; ++s)
+                    if ((ld_pend >> s) & 1u) mbar_wait(&ms->bar[bLd0 + s], (ld_par >> s) & 1u, kBarWaitNs);
+                umma_commit(&ms->bar[bTear]);
+                mbar_wait(&ms->bar[bTear], 0, kBarWaitNs);
+            }
+        }
+        __syncwarp();
+    } else {
+        // ================================ epilogue ================================
+        const int qd = warp & 3, cq = warp >> 2;
+        const int r = 32 * qd + lane;
+        const uint32_t lb = (uint32_t)(32 * qd) << 16;
+        uint32_t n_s = 0, n_f = 0, n_b = 0, n_head = 0;
+        auto zero_carries = [&]() {  // rows 0..63 of R4 and R5
+            if (qd < 2) {
+                uint32_t z[16];
+#pragma unroll
+                for (int u = 0; u < 16; ++u) z[u] = 0u;
+                tmem_st16(tb + lb + kR4 + 16 * cq, z);
+                tmem_st16(tb + lb + kR5 + 16 * cq, z);
+                tmem_st_wait();
+            }
+        };
+        // rows 0..63 of R4 and R5 as bf16 into the two 8 KiB halves of a block
+        auto carries_bf16 = [&](uint8_t *dst) {
+            if (qd < 2) {
+                uint32_t a[16], b[16];
+                tmem_ld16(tb + lb + kR4 + 16 * cq, a);
+                tmem_ld16(tb + lb + kR5 + 16 * cq, b);
+                tmem_ld_wait();
+                store16(dst, r, 16 * cq, a);
+                store16(dst + kHalf, r, 16 * cq, b);
+            }
+        };
+        for (int head = blockIdx.x; head < p.BH; head += gridDim.x, ++n_head) {
+            // ---------------- forward sweep ----------------
+            zero_carries();
+            for (int j = 0; j < M; ++j, ++n_f, ++n_s) {
+                const uint32_t tp = n_s & 1, tf = n_f & 1;
+                // E0: S_p, D_p -> bf16 checkpoint image (also the B operand of Q S_p) -> global
+                if (j > 0) {
+                    bar_wait(ms, bEvC, tf ^ 1u, p);  // the previous tile's carry products
+                    tc_fence_after();
+                    if (tid == 0) tma_store_wait_read();  // its checkpoint copy has left bCk
+                    epi_sync();
+                }
+                carries_bf16(blk(bCk));
+                fence_async_smem();
+                epi_sync();
+                if (tid == 0) {
+                    bulk_store(p.ck + ((size_t)head * M + j) * kCkBytes, blk(bCk), kCkBytes);
+                    tma_store_commit();
+                }
+                epi_arrive(ms, bEp0);
+                // E1: W = L . A
+                bar_wait(ms, bEvA, tp, p);
+                tc_fence_after();
+                {
+                    uint32_t a[32];
+                    tmem_ld32(tb + lb + kR0 + 32 * cq, a);
+                    tmem_ld_wait();
+                    store_masked32(blk(bW), r, 32 * cq, a);
+                }
+                fence_async_smem();
+                epi_arrive(ms, bEp1);
+                // E2: X -> bf16
+                bar_wait(ms, bEvX, tp, p);
+                tc_fence_after();
+                {
+                    uint32_t x[16];
+                    tmem_ld16(tb + lb + kR2 + 16 * cq, x);
+                    tmem_ld_wait();
+                    store16(blk(bX), r, 16 * cq, x);
+                }
+                fence_async_smem();
+                epi_arrive(ms, bEp2);
+            }
+            bar_wait(ms, bEvC, (n_f - 1) & 1u, p);  // the last carry products (before R4, R5 are reset)
+            tc_fence_after();
+            if (tid == 0) {
+                tma_store_wait_all();  // every checkpoint is in global memory
+                mbar_arrive(&ms->bar[bCkDone]);
+            }
+            // ---------------- reverse sweep ----------------
+            zero_carries();
+            for (int j = M - 1; j >= 0; --j, ++n_b, ++n_s) {
+                const uint32_t ts = n_s & 1, tp = n_b & 1;
+                const int tok0 = j * kTile;
+                const bool row_ok = tok0 + r < p.n;
+                const size_t orow = ((size_t)head * p.n + tok0 + r) * kD + 16 * cq;
+                // E0: Gam_s^T, Lam_s -> bf16 (the previous tile's products are done: waited in E4)
+                carries_bf16(blk(bCar));
+                fence_async_smem();
+                epi_arrive(ms, bEp0);
+                // E1: W = L . A, P = L . (G V^T)
+                bar_wait(ms, bEvA, ts, p);
+                tc_fence_after();
+                {
+                    uint32_t a[32];
+                    tmem_ld32(tb + lb + kR0 + 32 * cq, a);
+                    tmem_ld_wait();
+                    store_masked32(blk(bW), r, 32 * cq, a);
+                    tmem_ld32(tb + lb + kR1 + 32 * cq, a);
+                    tmem_ld_wait();
+                    store_masked32(blk(bP), r, 32 * cq, a);
+                }
+                fence_async_smem();
+                epi_arrive(ms, bEp1);
+                // E2: X, Y -> bf16
+                bar_wait(ms, bEvX, ts, p);
+                tc_fence_after();
+                {
+                    uint32_t x[16];
+                    tmem_ld16(tb + lb + kR2 + 16 * cq, x);
+                    tmem_ld_wait();
+                    store16(blk(bX), r, 16 * cq, x);
+                    tmem_ld16(tb + lb + kR3 + 16 * cq, x);
+                    tmem_ld_wait();
+                    store16(blk(bY), r, 16 * cq, x);
+                }
+                fence_async_smem();
+                epi_arrive(ms, bEp2);
+                // E3: T = L . (Q X^T) -> bf16
+                bar_wait(ms, bEvT, tp, p);
+                tc_fence_after();
+                {
+                    uint32_t a[32];
+                    tmem_ld32(tb + lb + kR0 + 32 * cq, a);
+                    tmem_ld_wait();
+                    store_masked32(blk(bT), r, 32 * cq, a);
+                }
+                fence_async_smem();
+                epi_arrive(ms, bEp3);
+                // dV out; then B = L . (Y K^T) -> bf16 over T (the dV products have read T)
+                bar_wait(ms, bEvV, tp, p);
+                tc_fence_after();
+                {
+                    uint32_t x[16];
+                    tmem_ld16(tb + lb + kR2 + 16 * cq, x);
+                    tmem_ld_wait();
+                    if (row_ok) out16(p.dv + orow, x);
+                }
+                bar_wait(ms, bEvB, tp, p);
+                tc_fence_after();
+                {
+                    uint32_t a[32];
+                    tmem_ld32(tb + lb + kR1 + 32 * cq, a);
+                    tmem_ld_wait();
+                    store_masked32(blk(bT), r, 32 * cq, a);
+                }
+                fence_async_smem();
+                epi_arrive(ms, bEp4);
+                // dQ, dK out
+                bar_wait(ms, bEvO, tp, p);
+                tc_fence_after();
+                {
+                    uint32_t x[16];
+                    tmem_ld16(tb + lb + kR0 + 16 * cq, x);
+                    tmem_ld_wait();
+                    if (row_ok) out16(p.dq + orow, x);
+                    tmem_ld16(tb + lb + kR0 + 64 + 16 * cq, x);
+                    tmem_ld_wait();
+                    if (row_ok) out16(p.dk + orow, x);
+                }
+            }
+        }
+        if (tid == 0) tma_store_wait_all();
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (issuer) {
+        tc_fence_after();
+        tmem_dealloc(tb, 512);
+    }
+}
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
+                                  const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+    static EncodeTiledFn fn = nullptr;
+    if (!fn) {
+        cudaDriverEntryPointQueryResult qr;
+        void *f = nullptr;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &qr) ==
+                cudaSuccess &&
+            qr == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(f);
+    }
+    return fn;
+}
+
+// [BH][n][64] bf16, boxes of 64 columns x 128 tokens, 128-byte swizzle, zero fill beyond n
+bool make_map(CUtensorMap *m, const void *base, int BH, int n) {
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return false;
+    cuuint64_t dims[3] = {(cuuint64_t)kD, (cuuint64_t)n, (cuuint64_t)BH};
+    cuuint64_t strides[2] = {(cuuint64_t)kD * 2, (cuuint64_t)n * kD * 2};
+    cuuint32_t box[3] = {(cuuint32_t)kD, (cuuint32_t)kTile, 1};
+    cuuint32_t es[3] = {1, 1, 1};
+    return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(base), dims, strides, box, es,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+bool aligned16(const void *q) { return (reinterpret_cast<uintptr_t>(q) & 15u) == 0; }
+
+}  // namespace
+
+size_t backward2_tc_workspace_bytes(int BH, int n) {
+    if (BH <= 0 || n <= 0) return kWsHeaderBytes;
+    return kWsHeaderBytes + (size_t)BH * ((n + kTile - 1) / kTile) * kCkBytes;
+}
+
+bool backward2_tc_applicable(const Bwd2 &p) {
+    if (getenv("HLA_DISABLE_FUSED")) return false;
+    if (p.dt != HLA_BF16 || p.d != kD || p.dv != kD || p.normalized || p.n <= 0 || p.BH <= 0) return false;
+    if (!aligned16(p.q) || !aligned16(p.k) || !aligned16(p.v) || !aligned16(p.dout)) return false;
+    if (!aligned16(p.dq) || !aligned16(p.dk) || !aligned16(p.dval)) return false;
+    if (p.ws_bytes < backward2_tc_workspace_bytes(p.BH, p.n)) return false;
+    int dev = 0, major = 0, minor = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return false;
+    cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
+    cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
+    return major == 10 && minor == 3 && encode_fn() != nullptr;
+}
+
+cudaError_t backward2_tc_launch(const Bwd2 &p, cudaStream_t stream) {
+    CUtensorMap mq, mk, mv, mg;
+    if (!make_map(&mq, p.q, p.BH, p.n) || !make_map(&mk, p.k, p.BH, p.n) || !make_map(&mv, p.v, p.BH, p.n) ||
+        !make_map(&mg, p.dout, p.BH, p.n))
+        return cudaErrorInvalidValue;
+    int dev = 0, sms = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    Params kp{};
+    kp.dq = static_cast<__nv_bfloat16 *>(p.dq);
+    kp.dk = static_cast<__nv_bfloat16 *>(p.dk);
+    kp.dv = static_cast<__nv_bfloat16 *>(p.dval);
+    kp.ck = reinterpret_cast<uint8_t *>(p.ws + kWsHeaderBytes);
+    kp.BH = p.BH;
+    kp.n = p.n;
+    kp.M = (p.n + kTile - 1) / kTile;
+    kp.err = reinterpret_cast<WsHeader *>(p.ws);
+    Tok tok{static_cast<const __nv_bfloat16 *>(p.q), static_cast<const __nv_bfloat16 *>(p.k),
+            static_cast<const __nv_bfloat16 *>(p.v), static_cast<const __nv_bfloat16 *>(p.dout)};
+    cudaError_t e = cudaMemsetAsync(p.ws, 0, kWsHeaderBytes, stream);
+    if (e) return e;
+    if ((e = cudaFuncSetAttribute(bwd_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes)))
+        return e;
+    const int grid = p.BH < sms ? p.BH : sms;
+    bwd_tc_kernel<<<grid, kThreads, kSmemBytes, stream>>>(mq, mk, mv, mg, kp, tok);
+    return cudaGetLastError();
+}
+
+}  // namespace hla

@@ -91,6 +91,10 @@ struct Bwd2 {
 };
 size_t backward2_workspace_bytes(int BH, int n, int d, int dv, int chunk);
 cudaError_t backward2_launch(const Bwd2 &p, cudaStream_t stream);
+// the backward on the tensor cores (hla_backward_sm103.cu): bf16, d = dv = 64, plain output
+size_t backward2_tc_workspace_bytes(int BH, int n);
+bool backward2_tc_applicable(const Bwd2 &p);
+cudaError_t backward2_tc_launch(const Bwd2 &p, cudaStream_t stream);
 
 // AHLA (asymmetric second order): chunk-parallel forward and decode step
 size_t ahla_workspace_bytes_internal(int BH, int n, int d, int dv, int chunk);

@@ -22,7 +22,7 @@ HLA_F32, HLA_BF16 = 0, 1
 # every symbol include/hla.h declares
 EXPORTS = ("hla_status_string", "hla_last_error", "hla2_state_floats", "hla2_workspace_bytes", "hla2_forward",
            "hla2_forward_path", "hla2_step", "hla3_state_floats", "hla3_workspace_bytes", "hla3_forward",
-           "hla3_forward_path",
+           "hla3_forward_path", "hla2_backward_path",
            "hla2_forward_noalloc", "hla_poll_error_noalloc", "hla_poll_error", "hla2_sde_state_floats",
            "hla2_state_to_sde", "hla2_step_sde", "ahla_state_floats", "ahla_workspace_bytes", "ahla_forward",
            "ahla_step", "hla2_backward_workspace_bytes", "hla2_backward", "ahla_forward_path")
@@ -61,6 +61,8 @@ def lib():
         L.ahla_step.restype = i
         L.ahla_forward_path.argtypes = [i, i, i, i, i, i, i, i, i, i]
         L.ahla_forward_path.restype = i
+        L.hla2_backward_path.argtypes = [i, i, i, i, i, i, i, i]
+        L.hla2_backward_path.restype = i
         L.hla2_backward.argtypes = [vp, vp, vp, vp, vp, vp, vp, i, i, i, i, i, i, i, f, i, vp, sz, vp]
         L.hla2_backward.restype = i
         for name in ("hla2_workspace_bytes", "hla3_workspace_bytes", "ahla_workspace_bytes",
@@ -284,6 +286,12 @@ def ahla_forward(q, k, v, out=None, *, normalized=False, eps=1e-6, chunk=64, sta
                               workspace.numel() * workspace.element_size(), _stream(stream))
     _check(code, "ahla_forward")
     return out
+
+
+def hla2_backward_path(B, H, n, d, dv, *, normalized=False, chunk=64, dtype=torch.bfloat16) -> int:
+    """1 if hla2_backward runs on the tensor cores for these arguments, 0 on the fp32 kernels, -1 unsupported."""
+    code = dtype if isinstance(dtype, int) else (HLA_BF16 if dtype == torch.bfloat16 else HLA_F32)
+    return int(lib().hla2_backward_path(B, H, n, d, dv, int(normalized), int(chunk), code))
 
 
 def ahla_forward_path(B, H, n, d, dv, *, normalized=False, chunk=64, dtype=torch.bfloat16, has_state_in=False,

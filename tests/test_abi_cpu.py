@@ -144,6 +144,8 @@ def test_ahla_and_backward_argument_errors(L):
     assert L.ahla_step(16, 16, 16, 16, 1, 0, 1, 128, 128, 0, f, 16, None) == H.HLA_OK
     assert L.ahla_forward_path(1, 1, 64, 24, 16, 0, 16, 1, 0, 0) == -1
     assert L.ahla_forward_path(1, 1, 64, 16, 16, 0, 16, 0, 0, 0) == 0  # fp32 tokens: the CUDA-core kernels
+    assert L.hla2_backward_path(1, 1, 64, 24, 64, 0, 64, 1) == -1
+    assert L.hla2_backward_path(8, 16, 2048, 64, 64, 0, 64, 1) == 0  # no device here: the CUDA-core kernels
     # third order: no device here, so never the tensor-core path; chunk-parallel or serial otherwise
     nl = ctypes.c_int(-7)
     assert L.hla3_forward_path(1, 1, 64, 24, 32, 1, 0, 32, 0, 0, 0, ctypes.byref(nl)) == -1

@@ -95,3 +95,45 @@ def test_backward_mid_workload_sampled(hla):
     errs = _check(hla, w.B, w.H, w.n, w.d, w.dv, w.chunk, w.dtype, False, hla_inputs.EPS, seed=w.seed,
                   heads=[0, 65, w.BH - 1])
     print("\nbackward on mid_bf16 sampled heads: dq %.3g dk %.3g dv %.3g" % tuple(errs))
+
+
+# ----------------------------------------------------------------------------
+# the tensor-core kernel (bf16 tokens, d = dv = 64, plain output)
+# ----------------------------------------------------------------------------
+
+TC_SHAPES = [(1, 1, 1), (1, 2, 127), (1, 2, 128), (2, 1, 129), (1, 3, 300), (1, 2, 700)]
+
+
+@pytest.mark.parametrize("shape", TC_SHAPES, ids=lambda s: "B%dH%dn%d" % s)
+def test_backward_tensor_core_path(hla, shape, monkeypatch):
+    """Every head against the oracle, and against the CUDA-core kernels on the same inputs."""
+    B, H, n = shape
+    assert hla.hla2_backward_path(B, H, n, 64, 64) == 1
+    q, k, v = hla_inputs.make_qkv(B, H, n, 64, 64, seed=6000 + n, dtype="bf16")
+    g = hla_inputs.round_to(np.random.default_rng(6001 + n).standard_normal((B, H, n, 64)), "bf16")
+    got = _grads(hla, q, k, v, g, "bf16", False, hla_inputs.EPS, 64)
+    flat = lambda x: x.reshape(B * H, n, -1)
+    ref = oracle.hla2_backward(flat(q), flat(k), flat(v), flat(g), masked=True, ckpt=64, nthreads=8)
+    for name, a, b in zip(("dq", "dk", "dv"), got, ref):
+        assert rowerr(flat(a), b) < TOL["bf16"], (name, rowerr(flat(a), b))
+    monkeypatch.setenv("HLA_DISABLE_FUSED", "1")
+    assert hla.hla2_backward_path(B, H, n, 64, 64) == 0
+    cc = _grads(hla, q, k, v, g, "bf16", False, hla_inputs.EPS, 64)
+    for name, a, b in zip(("dq", "dk", "dv"), got, cc):
+        assert rowerr(flat(a), flat(b)) < TOL["bf16"], (name, rowerr(flat(a), flat(b)))
+
+
+def test_backward_tensor_core_more_heads_than_sms(hla):
+    """200 heads: a CTA takes several heads in turn (both sweeps restart per head)."""
+    B, H, n = 2, 100, 260
+    errs = _check(hla, B, H, n, 64, 64, 64, "bf16", False, hla_inputs.EPS, seed=6100, heads=[0, 1, 151, 152, 199])
+    print("\nbackward, 200 heads: dq %.3g dk %.3g dv %.3g" % tuple(errs))
+
+
+def test_backward_tensor_core_deterministic(hla):
+    q, k, v = hla_inputs.make_qkv(1, 2, 500, 64, 64, seed=6200, dtype="bf16")
+    g = hla_inputs.round_to(np.random.default_rng(6201).standard_normal((1, 2, 500, 64)), "bf16")
+    a = _grads(hla, q, k, v, g, "bf16", False, hla_inputs.EPS, 64)
+    b = _grads(hla, q, k, v, g, "bf16", False, hla_inputs.EPS, 64)
+    for x, y in zip(a, b):
+        assert np.array_equal(x, y)
