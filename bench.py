@@ -376,7 +376,7 @@ def main():
     if args.only in ("ahla", "backward"):
         st = torch.cuda.current_stream()
         res = (bench_ahla(hla, dev, st, hbm_peak, world, tc_peak=tc_peak) if args.only == "ahla"
-               else bench_backward(hla, dev, st, world))
+               else bench_backward(hla, dev, st, world, hbm_peak, tc_peak))
         if rank == 0:
             print(json.dumps(res))
         return
@@ -551,7 +551,7 @@ def main():
         result["gpu_launches"] += result["mid"]["launches"] + result["hla3"]["launches"]
         result["ahla"] = bench_ahla(hla, dev, stream, hbm_peak, world, tc_peak=tc_peak)
         result["gpu_launches"] += result["ahla"]["forward"]["launches"] + result["ahla"]["decode"]["launches"]
-        result["backward"] = bench_backward(hla, dev, stream, world)
+        result["backward"] = bench_backward(hla, dev, stream, world, hbm_peak, tc_peak)
         result["gpu_launches"] += result["backward"]["launches"]
     if rank == 0 and not args.no_cpu_baseline:
         result["cpu_baseline"] = cpu_baseline()
@@ -666,19 +666,22 @@ def profile_case(hla, dev, case):
     print(json.dumps({"profile_case": case, "ok": True}))
 
 
-def bwd_flops(w):
-    """Algorithmic FLOPs of one masked second-order backward (chunk C, augmented width
-    W = dv + 1): the forward recompute (as fwd_flops) plus, per token-head,
+def bwd_flops(w, C=None, W=None):
+    """Algorithmic FLOPs of one masked second-order backward (chunk C, value width W: dv + 1
+    on the CUDA-core kernels, which always carry the denominator column; dv on the tensor-core
+    kernel, plain output, C = 128): the forward recompute (as fwd_flops) plus, per token-head,
     2 [C W / 2 (P) + C d / 2 (P^T Q) + d W (V' Gam) + C d / 2 (Y K^T) + C W / 2 (T^T G')
        + d W (X Gam^T) + C d / 2 (P X) + 2 d W (G' D^T, Gam, M) + d^2 (Y S_p) + C d / 2 (B K)
        + d^2 (K Lam) + C d (W^T Y, B^T Q) + 2 d^2 (Lam) + 2 d^2 W / C (scans)]."""
-    C, d, W = min(w.chunk, 32 if max(w.d, w.dv) == 128 else 64), w.d, w.dv + 1
+    d = w.d
+    C = min(w.chunk, 32 if max(w.d, w.dv) == 128 else 64) if C is None else C
+    W = w.dv + 1 if W is None else W
     per = 2 * (C * W / 2 + C * d / 2 + d * W + C * d / 2 + C * W / 2 + d * W + C * d / 2 + 2 * d * W + d * d
                + C * d / 2 + d * d + C * d + 2 * d * d + 2 * d * d * W / C)
     return fwd_flops(w) + w.BH * w.n * per
 
 
-def bench_backward(hla, dev, stream, world, steps=10, warmup=3):
+def bench_backward(hla, dev, stream, world, hbm_peak, tc_peak, steps=10, warmup=3):
     """hla2_backward on mid_bf16 (B8 H16 n2048 d64 bf16, chunk 64), CUDA events on the launching stream."""
     import torch
     w = hla_inputs.WORKLOADS["mid_bf16"]
@@ -701,15 +704,34 @@ def bench_backward(hla, dev, stream, world, steps=10, warmup=3):
     e1.record(stream)
     torch.cuda.synchronize()
     ms = max_over_ranks(e0.elapsed_time(e1) / steps, world)
-    tf = bwd_flops(w) / (ms * 1e-3) / 1e12
-    return {"workload": w.name, "B": w.B, "H": w.H, "n": w.n, "d": w.d, "dv": w.dv, "chunk": w.chunk,
-            "tokens": w.dtype, "ms_per_step": ms, "value": w.B * w.n * world / (ms * 1e-3), "unit": "tokens/s",
-            "steps": steps,
-            "roofline": {"bound": "alu", "achieved": tf, "peak": alu_peak(), "unit": "TFLOP/s", "frac": tf / alu_peak(),
-                         "traffic": None, "flops": bwd_flops(w),
-                         "peak_kind": "derived (152 SMs x 128 fp32 lanes x 2 x 2.07 GHz)",
-                         "kernel": "bwd_fwd_local/fwd_scan/local1/scan/local2 (fp32 CUDA cores)"},
-            "launches": 5 * steps}
+    rec = {"workload": w.name, "B": w.B, "H": w.H, "n": w.n, "d": w.d, "dv": w.dv, "chunk": w.chunk,
+           "tokens": w.dtype, "ms_per_step": ms, "value": w.B * w.n * world / (ms * 1e-3), "unit": "tokens/s",
+           "steps": steps}
+    if hla.hla2_backward_path(w.B, w.H, w.n, w.d, w.dv, normalized=w.normalized, chunk=w.chunk, dtype=tq.dtype) == 1:
+        # q, k, v, dout read once, dq, dk, dv written once (the checkpoints are the kernel's own traffic)
+        nbytes = w.BH * w.n * (3 * w.d + 4 * w.dv) * (2 if w.dtype == "bf16" else 4)
+        flops = bwd_flops(w, C=128, W=w.dv)
+        t_b, t_f = nbytes / (hbm_peak * 1e9), flops / (tc_peak * 1e12)
+        gbs, tfl = nbytes / (ms * 1e-3) / 1e9, flops / (ms * 1e-3) / 1e12
+        hbm = {"achieved": gbs, "peak": hbm_peak, "unit": "GB/s", "frac": gbs / hbm_peak}
+        ten = {"achieved": tfl, "peak": tc_peak, "unit": "TFLOP/s", "frac": tfl / tc_peak}
+        bound, main, other = ("hbm", hbm, ten) if t_b >= t_f else ("tensor", ten, hbm)
+        rec["roofline"] = {"bound": bound, "achieved": main["achieved"], "peak": main["peak"], "unit": main["unit"],
+                           "frac": main["frac"], "traffic": None, "algorithmic_bytes": nbytes, "flops": flops,
+                           "roofline_us": max(t_b, t_f) * 1e6, "peak_kind": "measured",
+                           ("tensor_view" if bound == "hbm" else "hbm_view"): other,
+                           "kernel": "bwd_tc_kernel (tcgen05, one launch)"}
+        rec["path"] = "tensor cores"
+        rec["launches"] = steps
+    else:
+        tf = bwd_flops(w) / (ms * 1e-3) / 1e12
+        rec["roofline"] = {"bound": "alu", "achieved": tf, "peak": alu_peak(), "unit": "TFLOP/s",
+                           "frac": tf / alu_peak(), "traffic": None, "flops": bwd_flops(w),
+                           "peak_kind": "derived (152 SMs x 128 fp32 lanes x 2 x 2.07 GHz)",
+                           "kernel": "bwd_fwd_local/fwd_scan/local1/scan/local2 (fp32 CUDA cores)"}
+        rec["path"] = "fp32 CUDA cores"
+        rec["launches"] = 5 * steps
+    return rec
 
 
 def bench_ahla(hla, dev, stream, hbm_peak, world, steps=20, warmup=3, decode_steps=256, tc_peak=None):
