@@ -28,9 +28,11 @@
 // 64-wide operand read as the M side of an M = 128 product takes the block after
 // it as rows 64..127, which land in TMEM lanes nobody reads.
 //
-// TMEM (512 columns): R0 (128) A -> T -> [dQ | dK]; R1 (128) G V^T -> B;
-// R2 (64) X -> dV; R3 (64) Y; R4, R5 (64 each) the carries (forward S, D;
-// reverse Gam^T, Lam), rows 0..63.
+// TMEM (512 columns): R0 (128) A -> T -> dV; R1 (128) G V^T -> B; R2 (64) X -> dK;
+// R3 (64) Y -> dQ; R4, R5 (64 each) the carries (forward S, D; reverse Gam^T,
+// Lam), rows 0..63.  The products that do not need T or B (the carries, and the
+// parts of dQ and dK without B) are issued so that they run while the epilogue
+// forms the operands of the next ones.
 //
 // Roles: warp 16 issues TMA copies and MMAs (one thread); warps 0..15 are the
 // epilogue (warp w: TMEM lanes 32 (w % 4) .. +31, one token row each; column
@@ -276,6 +278,7 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                     tc_fence_after();
                     mma<false, false, 128, 4>(tb + kR0, lk(qb), lk(qb + 1), 0u);   // A = Q K^T
                     umma_commit(&ms->bar[bEvA]);
+                    mma<true, true, 64, 8>(tb + kR4, lm(qb + 1), lm(qb + 1), 1u);  // S += K^T K (under E1)
                     if (!bar_wait(ms, bEp1, tp, p)) break;                        // W in bW
                     tc_fence_after();
                     mma<false, true, 64, 8>(tb + kR2, lk(bW), lm(qb + 1), 0u);     // X = W K
@@ -283,7 +286,6 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                     umma_commit(&ms->bar[bEvX]);
                     if (!bar_wait(ms, bEp2, tp, p)) break;                        // X (bf16) in bX
                     tc_fence_after();
-                    mma<true, true, 64, 8>(tb + kR4, lm(qb + 1), lm(qb + 1), 1u);  // S += K^T K
                     mma<true, true, 64, 8>(tb + kR5, lm(bX), lm(qb + 2), 1u);      // D += X^T V
                     umma_commit(&ms->bar[bEvC]);
                     if (!bar_wait(ms, bEvC, tf, p)) break;                        // this set is free again
@@ -312,6 +314,7 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                     mma<false, false, 128, 4>(tb + kR0, lk(bQ), lk(bK), 0u);        // A = Q K^T
                     mma<false, false, 128, 4>(tb + kR1, lk(bG), lk(bV), 0u);        // G V^T
                     umma_commit(&ms->bar[bEvA]);
+                    mma<true, true, 64, 8>(tb + kR4, lm(bQ), lm(bG), 1u);           // Gam^T += Q^T G (under E1)
                     if (!bar_wait(ms, bEp1, ts, p)) break;            // W, P (bf16)
                     tc_fence_after();
                     mma<false, true, 64, 8>(tb + kR2, lk(bW), lm(bK), 0u);          // X = W K
@@ -319,29 +322,29 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                     mma<true, true, 64, 8>(tb + kR3, lm(bP), lm(bQ), 0u);           // Y = P^T Q
                     mma<false, false, 64, 4>(tb + kR3, lk(bV), lk(bCar), 1u);       //   + V Gam_s
                     umma_commit(&ms->bar[bEvX]);
-                    if (!bar_wait(ms, bEp2, ts, p)) break;            // X, Y (bf16)
+                    if (!bar_wait(ms, bEp2, ts, p)) break;            // X, Y (bf16); R2, R3 read
                     tc_fence_after();
                     mma<false, false, 128, 4>(tb + kR0, lk(bQ), lk(bX), 0u);        // T = Q X^T
                     umma_commit(&ms->bar[bEvT]);
                     mma<false, false, 128, 4>(tb + kR1, lk(bY), lk(bK), 0u);        // B = Y K^T
                     umma_commit(&ms->bar[bEvB]);
-                    if (!bar_wait(ms, bEp3, tp, p)) break;                         // T (bf16) in bT
+                    if (!bar_wait(ms, bEp3, tp, p)) break;                         // T (bf16) in bT; R0 read
                     tc_fence_after();
-                    mma<true, true, 64, 8>(tb + kR2, lm(bT), lm(bG), 0u);           // dV = T^T G
-                    mma<false, true, 64, 4>(tb + kR2, lk(bX), lm(bCar), 1u);        //   + X Gam_s^T
+                    mma<true, true, 64, 8>(tb + kR0, lm(bT), lm(bG), 0u);           // dV = T^T G
+                    mma<false, true, 64, 4>(tb + kR0, lk(bX), lm(bCar), 1u);        //   + X Gam_s^T
                     umma_commit(&ms->bar[bEvV]);
-                    if (!bar_wait(ms, bEp4, tp, p)) break;                         // B (bf16) in bT
-                    tc_fence_after();
-                    mma<false, true, 64, 8>(tb + kR0, lk(bP), lm(bX), 0u);          // dQ = P X
-                    mma<false, false, 64, 4>(tb + kR0, lk(bG), lk(bCk) + kH16, 1u); //   + G D_p^T
-                    mma<false, false, 64, 4>(tb + kR0, lk(bY), lk(bCk), 1u);        //   + Y S_p
-                    mma<false, true, 64, 8>(tb + kR0, lk(bT), lm(bK), 1u);          //   + B K
-                    mma<false, false, 64, 4>(tb + kR0 + 64, lk(bK), lk(bCar) + kH16, 0u);  // dK = K Lam_s
-                    mma<true, true, 64, 8>(tb + kR0 + 64, lm(bW), lm(bY), 1u);      //   + W^T Y
-                    mma<true, true, 64, 8>(tb + kR0 + 64, lm(bT), lm(bQ), 1u);      //   + B^T Q
-                    mma<true, true, 64, 8>(tb + kR4, lm(bQ), lm(bG), 1u);           // Gam^T += Q^T G
+                    // while dV goes out and the epilogue forms B: the parts of dQ and dK without B, Lam
+                    mma<false, true, 64, 8>(tb + kR3, lk(bP), lm(bX), 0u);          // dQ = P X
+                    mma<false, false, 64, 4>(tb + kR3, lk(bG), lk(bCk) + kH16, 1u); //   + G D_p^T
+                    mma<false, false, 64, 4>(tb + kR3, lk(bY), lk(bCk), 1u);        //   + Y S_p
+                    mma<false, false, 64, 4>(tb + kR2, lk(bK), lk(bCar) + kH16, 0u);  // dK = K Lam_s
+                    mma<true, true, 64, 8>(tb + kR2, lm(bW), lm(bY), 1u);           //   + W^T Y
                     mma<true, true, 64, 8>(tb + kR5, lm(bY), lm(bQ), 1u);           // Lam += Y^T Q
                     mma<true, true, 64, 8>(tb + kR5, lm(bQ), lm(bY), 1u);           //   + Q^T Y
+                    if (!bar_wait(ms, bEp4, tp, p)) break;                         // B (bf16) in bT
+                    tc_fence_after();
+                    mma<false, true, 64, 8>(tb + kR3, lk(bT), lm(bK), 1u);          // dQ += B K
+                    mma<true, true, 64, 8>(tb + kR2, lm(bT), lm(bQ), 1u);           // dK += B^T Q
                     umma_commit(&ms->bar[bEvO]);
                     if (!bar_wait(ms, bEvO, tp, p)) break;                         // every operand read
                     if (j > 0) load_bwd(head, j - 1);
@@ -488,7 +491,7 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                 tc_fence_after();
                 {
                     uint32_t x[16];
-                    tmem_ld16(tb + lb + kR2 + 16 * cq, x);
+                    tmem_ld16(tb + lb + kR0 + 16 * cq, x);
                     tmem_ld_wait();
                     if (row_ok) out16(p.dv + orow, x);
                 }
@@ -507,10 +510,10 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                 tc_fence_after();
                 {
                     uint32_t x[16];
-                    tmem_ld16(tb + lb + kR0 + 16 * cq, x);
+                    tmem_ld16(tb + lb + kR3 + 16 * cq, x);
                     tmem_ld_wait();
                     if (row_ok) out16(p.dq + orow, x);
-                    tmem_ld16(tb + lb + kR0 + 64 + 16 * cq, x);
+                    tmem_ld16(tb + lb + kR2 + 16 * cq, x);
                     tmem_ld_wait();
                     if (row_ok) out16(p.dk + orow, x);
                 }
