@@ -76,7 +76,8 @@ enum Bar {
     bEp0 = 9, bEp1 = 10, bEp2 = 11, bEp3 = 12, bEp4 = 13,    // epilogue hand-offs (16 warp arrivals)
     bTear = 14,
     bCkDone = 15,                                              // a head's checkpoints are in global memory
-    kNumBars = 16
+    bEp5 = 16,                                                 // reverse sweep: P (bf16) formed after W
+    kNumBars = 17
 };
 
 struct Misc {
@@ -216,7 +217,8 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
         return;
     }
     if (tid == 0) {
-        for (int b = 0; b < kNumBars; ++b) mbar_init(&ms->bar[b], (b >= bEp0 && b <= bEp4) ? kEpiWarps : 1);
+        for (int b = 0; b < kNumBars; ++b)
+            mbar_init(&ms->bar[b], ((b >= bEp0 && b <= bEp4) || b == bEp5) ? kEpiWarps : 1);
         ms->abort_flag = 0;
         fence_mbar_init();
     }
@@ -315,10 +317,12 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                     mma<false, false, 128, 4>(tb + kR1, lk(bG), lk(bV), 0u);        // G V^T
                     umma_commit(&ms->bar[bEvA]);
                     mma<true, true, 64, 8>(tb + kR4, lm(bQ), lm(bG), 1u);           // Gam^T += Q^T G (under E1)
-                    if (!bar_wait(ms, bEp1, ts, p)) break;            // W, P (bf16)
+                    if (!bar_wait(ms, bEp1, ts, p)) break;            // W (bf16)
                     tc_fence_after();
                     mma<false, true, 64, 8>(tb + kR2, lk(bW), lm(bK), 0u);          // X = W K
                     mma<false, false, 64, 4>(tb + kR2, lk(bQ), lk(bCk), 1u);        //   + Q S_p
+                    if (!bar_wait(ms, bEp5, tp, p)) break;            // P (bf16)
+                    tc_fence_after();
                     mma<true, true, 64, 8>(tb + kR3, lm(bP), lm(bQ), 0u);           // Y = P^T Q
                     mma<false, false, 64, 4>(tb + kR3, lk(bV), lk(bCar), 1u);       //   + V Gam_s
                     umma_commit(&ms->bar[bEvX]);
@@ -447,7 +451,7 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                 carries_bf16(blk(bCar));
                 fence_async_smem();
                 epi_arrive(ms, bEp0);
-                // E1: W = L . A, P = L . (G V^T)
+                // E1: W = L . A (X = W K starts on it), then P = L . (G V^T)
                 bar_wait(ms, bEvA, ts, p);
                 tc_fence_after();
                 {
@@ -455,12 +459,14 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                     tmem_ld32(tb + lb + kR0 + 32 * cq, a);
                     tmem_ld_wait();
                     store_masked32(blk(bW), r, 32 * cq, a);
+                    fence_async_smem();
+                    epi_arrive(ms, bEp1);
                     tmem_ld32(tb + lb + kR1 + 32 * cq, a);
                     tmem_ld_wait();
                     store_masked32(blk(bP), r, 32 * cq, a);
                 }
                 fence_async_smem();
-                epi_arrive(ms, bEp1);
+                epi_arrive(ms, bEp5);
                 // E2: X, Y -> bf16
                 bar_wait(ms, bEvX, ts, p);
                 tc_fence_after();
@@ -486,15 +492,8 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                 }
                 fence_async_smem();
                 epi_arrive(ms, bEp3);
-                // dV out; then B = L . (Y K^T) -> bf16 over T (the dV products have read T)
+                // B = L . (Y K^T) -> bf16 over T (the dV products have read T), then dV out
                 bar_wait(ms, bEvV, tp, p);
-                tc_fence_after();
-                {
-                    uint32_t x[16];
-                    tmem_ld16(tb + lb + kR0 + 16 * cq, x);
-                    tmem_ld_wait();
-                    if (row_ok) out16(p.dv + orow, x);
-                }
                 bar_wait(ms, bEvB, tp, p);
                 tc_fence_after();
                 {
@@ -505,6 +504,12 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                 }
                 fence_async_smem();
                 epi_arrive(ms, bEp4);
+                {
+                    uint32_t x[16];
+                    tmem_ld16(tb + lb + kR0 + 16 * cq, x);
+                    tmem_ld_wait();
+                    if (row_ok) out16(p.dv + orow, x);
+                }
                 // dQ, dK out
                 bar_wait(ms, bEvO, tp, p);
                 tc_fence_after();
