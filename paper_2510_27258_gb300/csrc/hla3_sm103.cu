@@ -84,7 +84,8 @@ enum Bar {
     bTear = 9,
     bSt0 = 10,                                         // + stage: pre-pass token copies
     bEvO1 = 12,                                        // pre-pass: products of the second block set
-    kNumBars = 13
+    bEpQK = 13,                                        // sweep: Q, K, V (hi | lo) stored (16 warp arrivals)
+    kNumBars = 14
 };
 
 struct Misc {
@@ -283,7 +284,8 @@ __global__ void __launch_bounds__(kThreads, 1) hla3_tc_kernel(Params p) {
         return;
     }
     if (tid == 0) {
-        for (int b = 0; b < kNumBars; ++b) mbar_init(&ms->bar[b], (b >= bEp0 && b <= bEp3) ? kEpiWarps : 1);
+        for (int b = 0; b < kNumBars; ++b)
+            mbar_init(&ms->bar[b], ((b >= bEp0 && b <= bEp3) || b == bEpQK) ? kEpiWarps : 1);
         ms->abort_flag = 0;
         fence_mbar_init();
     }
@@ -323,7 +325,7 @@ __global__ void __launch_bounds__(kThreads, 1) hla3_tc_kernel(Params p) {
                     for (int t = 0; t < kStages && j0 + t < j1; ++t) stage_copy((n_tiles + t) % kStages, head, j0 + t);
                 for (int j = j0; j < j1; ++j, ++n_tiles) {
                     const uint32_t tp = n_tiles & 1;
-                    if (!bar_wait(ms, bEp0, tp, p)) break;  // Q, K, V (and the carries) in shared memory
+                    if (!bar_wait(ms, kPre ? bEp0 : bEpQK, tp, p)) break;  // Q, K, V in shared memory
                     tc_fence_after();
                     if (kPre) {
                         st_pend &= ~(1u << (n_tiles % kStages));  // read by the epilogue
@@ -334,8 +336,10 @@ __global__ void __launch_bounds__(kThreads, 1) hla3_tc_kernel(Params p) {
                         umma_commit(&ms->bar[(n_tiles & 1) ? bEvO1 : bEvO]);
                         continue;
                     }
-                    mma_feat3<128>(tb + kTA, lk(bQ), lk(bK), 0u);        // A = Q K^T
+                    mma_feat3<128>(tb + kTA, lk(bQ), lk(bK), 0u);        // A = Q K^T (under the carry fold)
                     umma_commit(&ms->bar[bEvA]);
+                    if (!bar_wait(ms, bEp0, tp, p)) break;              // the carries (bf16) in shared memory
+                    tc_fence_after();
                     mma_feat3<32>(tb + kTQS, lk(bQ), car, 0u);           // Q S^K_p
                     mma_feat3<32>(tb + kTKS, lk(bK), car + 256, 0u);     // K S^Q_p
                     umma_commit(&ms->bar[bEvQ]);
@@ -463,7 +467,12 @@ __global__ void __launch_bounds__(kThreads, 1) hla3_tc_kernel(Params p) {
                 const uint32_t tp = n_tiles & 1;
                 const int tok0 = j * kTile;
                 const bool totals = j == j1;
-                // ---- E0: Q, K, V -> hi | lo blocks; carries -> bf16 operands ----
+                if (!kPre && j > j0) {  // the previous tile's products are done (its outputs are read below)
+                    bar_wait(ms, bEvO, tp ^ 1u, p);
+                    tc_fence_after();
+                }
+                // ---- E0: Q, K, V -> hi | lo blocks (A = Q K^T starts on them); the previous tile's
+                // outputs; carries -> bf16 operands ----
                 if (!totals) {
                     if (kPre) {  // this tile's copies in stage n_tiles % 2 (rows beyond n are stale: zero)
                         const int st = n_tiles % kStages;
@@ -488,6 +497,23 @@ __global__ void __launch_bounds__(kThreads, 1) hla3_tc_kernel(Params p) {
 #pragma unroll
                         for (int u = 0; u < 8; ++u) dp = fmaf(pq[u], pk[u], dp);
                         ms->sdp[e_c / 8][e_row] = dp;
+                        fence_async_smem();
+                        epi_arrive(ms, bEpQK);
+                    }
+                }
+                if (!kPre && j > j0) {  // ---- E4 of the previous tile: its outputs ----
+                    uint32_t o0[8], o1[8];
+                    tmem_ld8(tb + lb + kTY + 8 * cq, o0);
+                    tmem_ld8(tb + lb + kTY + 32 + 8 * cq, o1);
+                    tmem_ld_wait();
+                    const int t = tok0 - kTile + r;
+                    if (t < p.n) {
+                        float4 *dst = reinterpret_cast<float4 *>(p.out + ((size_t)head * p.n + t) * kD + 8 * cq);
+                        float o[8];
+#pragma unroll
+                        for (int u = 0; u < 8; ++u) o[u] = __uint_as_float(o0[u]) + __uint_as_float(o1[u]);
+                        dst[0] = make_float4(o[0], o[1], o[2], o[3]);
+                        dst[1] = make_float4(o[4], o[5], o[6], o[7]);
                     }
                 }
                 if (kPre && totals && n_tiles > 0) {  // the last tile's products (and so all) are done
@@ -641,23 +667,6 @@ __global__ void __launch_bounds__(kThreads, 1) hla3_tc_kernel(Params p) {
                 fence_async_smem();
                 epi_arrive(ms, bEp3);
                 prefetch();
-                // ---- E4: outputs ----
-                bar_wait(ms, bEvO, tp, p);
-                tc_fence_after();
-                {
-                    uint32_t o0[8], o1[8];
-                    tmem_ld8(tb + lb + kTY + 8 * cq, o0);
-                    tmem_ld8(tb + lb + kTY + 32 + 8 * cq, o1);
-                    tmem_ld_wait();
-                    if (tok0 + r < p.n) {
-                        float4 *dst = reinterpret_cast<float4 *>(p.out + ((size_t)head * p.n + tok0 + r) * kD + 8 * cq);
-                        float o[8];
-#pragma unroll
-                        for (int u = 0; u < 8; ++u) o[u] = __uint_as_float(o0[u]) + __uint_as_float(o1[u]);
-                        dst[0] = make_float4(o[0], o[1], o[2], o[3]);
-                        dst[1] = make_float4(o[4], o[5], o[6], o[7]);
-                    }
-                }
                 ++n_tiles;
             }
         }
