@@ -46,6 +46,16 @@ def rowerr(got, ref):
     return float(r.max()) if r.size else 0.0
 
 
+def rowerr_stats(got, ref):
+    """max, median and 99.9th percentile of the per-row error (the reading of the error metric
+    asks for all three), as a short string and a tuple."""
+    r = rowerr_rows(got, ref).ravel()
+    if r.size == 0:
+        return "max 0 median 0 p99.9 0", (0.0, 0.0, 0.0)
+    t = (float(r.max()), float(np.median(r)), float(np.quantile(r, 0.999)))
+    return "max %.3g median %.3g p99.9 %.3g" % t, t
+
+
 def local_rms(den, window=512):
     """RMS of den over positions [t - window, t + window] (per head), den: [..., n]."""
     den = np.asarray(den, np.float64)
@@ -84,4 +94,5 @@ def check_normalized(o_gpu, num_gpu, num_ref, den_ref, eps, tol):
     k_used = float((err_den[beyond] / (bound[beyond] / K_FP32)).max()) if beyond.any() else 0.0
     return {"num": e_num, "out_well": e_out, "ill_rows": int((~well).sum()), "rows": int(well.size),
             "den_excess": float(excess.max()), "out_literal_max": float(lit.max()),
+            "out_literal_median": float(np.median(lit)), "out_literal_p999": float(np.quantile(lit, 0.999)),
             "rows_beyond_bar": int((lit >= tol).sum()), "k_used": k_used}

@@ -12,7 +12,7 @@ import torch
 
 import hla_inputs
 import oracle
-from parity import TOL, check_normalized, rowerr, rowerr_rows
+from parity import TOL, check_normalized, rowerr, rowerr_rows, rowerr_stats
 
 pytestmark = pytest.mark.gpu
 
@@ -194,9 +194,10 @@ def test_workload_full_size_sampled(hla, name):
     num_gpu = gpu_forward(hla, q, k, v, w.dtype, w.masked, False, w.chunk).reshape(w.BH, w.n, w.dv)[heads]
     num_ref = ref_forward(q, k, v, w.masked, False, heads=heads)
     tiles = _tile_errors(num_gpu, num_ref)
-    print("\n%s sampled heads %s: %s; numerator row error by tile: first %.3g, max %.3g (tile %d), "
-          "tiles 0-6 %.3g, tiles 7+ %.3g" % (name, heads, res, tiles[0], max(tiles), int(np.argmax(tiles)),
-                                             max(tiles[:7]), max(tiles[7:]) if len(tiles) > 7 else 0.0))
+    print("\n%s sampled heads %s: %s; numerator row error %s; by tile: first %.3g, max %.3g (tile %d), "
+          "tiles 0-6 %.3g, tiles 7+ %.3g" % (name, heads, res, rowerr_stats(num_gpu, num_ref)[0], tiles[0],
+                                             max(tiles), int(np.argmax(tiles)), max(tiles[:7]),
+                                             max(tiles[7:]) if len(tiles) > 7 else 0.0))
     if w.normalized:
         assert res["ill_rows"] <= 0.01 * res["rows"], res
 
@@ -296,7 +297,8 @@ def test_decode_workload_full_depth_sampled(hla):
     ref, rst = oracle.hla2_serial(*cat, masked=w.masked, normalized=w.normalized, eps=hla_inputs.EPS,
                                   return_state=True, nthreads=4)
     err = rowerr(got, ref[:, w.decode_prefix:])
-    print("\ndecode at depth %d, %d steps, heads %s: max row error %.3g" % (w.decode_prefix, steps, heads, err))
+    print("\ndecode at depth %d, %d steps, heads %s: row error %s" % (w.decode_prefix, steps, heads,
+                                                                      rowerr_stats(got, ref[:, w.decode_prefix:])[0]))
     assert err < TOL["bf16"], err
     pg, pr = oracle.split_state2(gst, w.d, w.dv), oracle.split_state2(rst, w.d, w.dv)
     for name in ("S", "C", "m", "G", "h"):
