@@ -49,10 +49,10 @@ TRAFFIC = {
     "c3_kernels": {"src": ["hla3_chunked.cu"], "sha256": "17ac1acd5c9202d1", "workload": "hla3_f32", "n": 4096,
                    "bytes": 432.5e6, "how": "ncu capture of one forward's five launches (bench.py --only hla3_f32): "
                                             "373.0 MB read + 59.5 MB written, 6.4 x the token I/O (per-chunk records)"},
-    "hla3_tc_kernels": {"src": ["hla3_sm103.cu", "sm103_prims.cuh"], "sha256": "2638848aa44b37f5", "workload": "hla3_f32",
+    "hla3_tc_kernels": {"src": ["hla3_sm103.cu", "sm103_prims.cuh"], "sha256": "a0d8a1593e2f3545", "workload": "hla3_f32",
                         "n": 4096, "bytes": 115.2e6,
                         "how": "ncu capture of one forward's three launches (bench.py --only hla3_f32), caches "
-                               "flushed per launch: pre-pass 37.8 MB read, sweep 51.7 MB read + 0.2 MB written "
+                               "flushed per launch: pre-pass 37.8 MB read, sweep 51.7 MB read + 0.1 MB written "
                                "(outputs still dirty in L2 at its end), fix-up 25.6 MB read"},
     "step2_kernel_sde": {"src": ["hla_step.cu"], "sha256": "5542daa4b35fe2f4", "workload": "decode_bf16", "n": 0,
                          "bytes": 481.3e6, "how": "ncu capture of one step at B64 H32 d128 (bench.py --profile-case "
