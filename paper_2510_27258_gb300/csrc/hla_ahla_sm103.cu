@@ -56,7 +56,8 @@ enum Bar {
     bEvA = 5, bEvR = 6, bEvO = 7,  // MMA commits
     bEpW = 8, bEpR = 9,            // epilogue hand-offs (16 warp arrivals)
     bTear = 10,
-    kNumBars = 11
+    bEvV = 11, bEvE = 12,          // commits: V read (after P += K^T V); E += K^T R done
+    kNumBars = 13
 };
 
 struct Misc {
@@ -201,7 +202,10 @@ ahla_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
                     const int qs = (j & 1) ? kQ1 : kQ0, ks = (j & 1) ? kK1 : kK0;
                     const int qo = (j & 1) ? kQ0 : kQ1, ko = (j & 1) ? kK0 : kK1;
                     const bool more = j + 1 < p.M;
-                    if (more) {  // slots qo, ko were last read by the previous tile's MMAs (done)
+                    if (more) {
+                        // slots qo, ko were last read by the previous tile's products, the last of
+                        // them E += K^T R (bEvE)
+                        if (j > 0 && !bar_wait(ms, bEvE, tp ^ 1u, p)) break;
                         load_tile(qo, &tm_q, head, (j + 1) * kTile);
                         load_tile(ko, &tm_k, head, (j + 1) * kTile);
                     }
@@ -209,22 +213,25 @@ ahla_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
                     tc_fence_after();
                     mma_ts(tb + kTR, tb + kTA, lm(kV), 0u);              // R = W V
                     mma_ss<false, true>(tb + kTR, lk(qs), lm(kC), 1u);   //   + Q P_p
-                    mma_ss<true, true>(tb + kTP, lm(ks), lm(kV), 1u);    // P += K^T V
                     umma_commit(&ms->bar[bEvR]);
-                    if (!bar_wait(ms, bEvR, tp, p)) break;                // V and P_p read
+                    mma_ss<true, true>(tb + kTP, lm(ks), lm(kV), 1u);    // P += K^T V (under the R epilogue)
+                    umma_commit(&ms->bar[bEvV]);
+                    if (!bar_wait(ms, bEvV, tp, p)) break;                // V read
                     if (more) load_tile(kV, &tm_v, head, (j + 1) * kTile);
                     if (!bar_wait(ms, bEpR, tp, p)) break;                // R and E_p (bf16) ready
                     tc_fence_after();
                     mma_ts(tb + kTR, tb + kTA, lm(kR), 0u);              // O = W R
                     mma_ss<false, true>(tb + kTR, lk(qs), lm(kC), 1u);   //   + Q E_p
-                    mma_ss<true, true>(tb + kTE, lm(ks), lm(kR), 1u);    // E += K^T R
                     umma_commit(&ms->bar[bEvO]);
-                    if (!bar_wait(ms, bEvO, tp, p)) break;                // W, R, E_p, Q, K read
-                    if (more) {
+                    mma_ss<true, true>(tb + kTE, lm(ks), lm(kR), 1u);    // E += K^T R (under the O epilogue)
+                    umma_commit(&ms->bar[bEvE]);
+                    if (more) {  // the next A runs behind them (the products execute in issue order)
                         if (!wait_ld(qo) || !wait_ld(ko)) break;
                         tc_fence_after();
                         mma_ss<false, false>(tb + kTA, lk(qo), lk(ko), 0u);  // next A = Q K^T
                         umma_commit(&ms->bar[bEvA]);
+                    } else if (!bar_wait(ms, bEvE, tp, p)) {  // every product of the head is done
+                        break;
                     }
                     ++n_tiles;
                 }
@@ -246,6 +253,10 @@ ahla_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
         const uint32_t lane_base = (uint32_t)(32 * qd) << 16;
         const bool blk_zero = cq > qd;  // this 32-column block of W lies above the diagonal
         for (int head = blockIdx.x; head < p.BH; head += gridDim.x) {
+            if (n_tiles > 0) {  // the previous head's last E += K^T R is done before E is reset
+                bar_wait(ms, bEvE, (n_tiles - 1) & 1u, p);
+                tc_fence_after();
+            }
             {  // carries start at zero
                 uint32_t z[32];
 #pragma unroll
