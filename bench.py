@@ -49,7 +49,7 @@ TRAFFIC = {
     "c3_kernels": {"src": ["hla3_chunked.cu"], "sha256": "17ac1acd5c9202d1", "workload": "hla3_f32", "n": 4096,
                    "bytes": 432.5e6, "how": "ncu capture of one forward's five launches (bench.py --only hla3_f32): "
                                             "373.0 MB read + 59.5 MB written, 6.4 x the token I/O (per-chunk records)"},
-    "hla3_tc_kernels": {"src": ["hla3_sm103.cu", "sm103_prims.cuh"], "sha256": "a0d8a1593e2f3545", "workload": "hla3_f32",
+    "hla3_tc_kernels": {"src": ["hla3_sm103.cu", "sm103_prims.cuh"], "sha256": "0bf5b53339f19510", "workload": "hla3_f32",
                         "n": 4096, "bytes": 115.2e6,
                         "how": "ncu capture of one forward's three launches (bench.py --only hla3_f32), caches "
                                "flushed per launch: pre-pass 37.8 MB read, sweep 51.7 MB read + 0.1 MB written "

@@ -32,7 +32,9 @@
 //   * products over the 128 tokens read such a block MN-major with N = 64 (or
 //     M = 64 of an M = 128 product), so the result holds the hi and lo halves
 //     side by side (or the four hi/lo quadrants), summed by the epilogue.
-// The 128 x 128 operands (LA, then L . C') are separate hi and lo tiles.
+// LA (128 x 128) has separate hi and lo tiles.  L . C' is packed as bf16 into TMEM over
+// C' itself (each thread's 32 columns: hi in the first 16, lo in the last 16) and read
+// from there as the A operand of its product.
 //
 // TMEM (512 columns): A -> C' -> L . C' packed (128), Y -> num (64), Q S^K_p and
 // K S^Q_p (32 + 32, then G'' = LA^T aV over them), and 64-column carry regions
@@ -44,7 +46,9 @@
 // Roles: warp 16 issues the MMAs (one thread); warps 0..15 are the epilogue
 // (warp w: TMEM lanes 32 (w % 4) .. +31, one token row each; column block w / 4),
 // which also loads the fp32 tokens (the next tile's during this one) and splits
-// them into hi + lo.
+// them into hi + lo.  A tile's outputs are read out while the next tile's first
+// product (A = Q K^T) runs, and that product starts on the split tokens while the
+// epilogue folds the carries.
 //
 // Scope: fp32 tokens, d = dv = 32, masked, plain (unnormalised) output, no
 // initial or final state.
@@ -65,7 +69,7 @@ constexpr int kMaxSegments = 160;
 
 // shared-memory blocks of 16 KiB
 enum Block { bQ = 0, bK = 1, bV = 2, bQS = 3, bAV = 4, bZ = 5, bG = 6, bLh = 7, bLl = 9, bCar = 11, kBlocks = 12 };
-// bLh / bLl: 128 x 128 tiles (two blocks each): LA, then L . C', hi and lo parts.
+// bLh / bLl: 128 x 128 tiles (two blocks each): LA, hi and lo parts.
 // bCar: four 32-row K-major operands (hi | lo): S^K_p, S^Q_p, P_p^T, F_p^T.
 // The pre-pass alternates two sets of Q, K, V blocks (0..2 and 3..5: a tile's split runs
 // while the products of the tile before read the other set) and holds two stages of fp32
@@ -96,7 +100,7 @@ struct Misc {
     float sdp[4][kTile];      // per column block: partial q_t . k_t in fp32
     float sbp[4][kTile];      // per lane quadrant: column sums of A_us^2 over u < s
     float sbp2[4][kTile];     // per column block: partial k_s^T S^Q_p k_s
-    float fold[4][32][33];    // carry read-out: rows 32..63 of each carry region, folded
+    float fold[4][32][33];    // carry read-out: each carry folded to 32 x 32 (hi/lo rows, columns added)
 };
 constexpr uint32_t kMiscBytes = 24 * 1024;
 static_assert(sizeof(Misc) <= kMiscBytes, "misc smem");
