@@ -21,18 +21,28 @@
 // shared-memory image, by 1-D bulk copies); a reverse sweep reloads them and
 // carries Gam^T and Lam in TMEM.  No CTA waits on another.
 //
-// Operands are bf16 in the 128-byte-swizzled layout TMA writes (128 rows x 64
-// columns per 16 KiB block; 64 x 64 matrices in the first 64 rows of an 8 KiB
-// half); every product accumulates in fp32.  The transposed uses (P^T, T^T, W^T,
-// B^T, and X^T, Y^T, Q^T, K^T of the carries) read the same tiles MN-major; a
-// 64-wide operand read as the M side of an M = 128 product takes the block after
-// it as rows 64..127, which land in TMEM lanes nobody reads.
+// Precision.  A gradient row can be a small difference of large terms (dq_0 is
+// k_0 times k_0 . y_0 plus a P X term, for one), so an intermediate rounded once
+// to bf16 can miss the row by far more than its own 2^-9.  Every intermediate
+// that feeds such a sum is therefore an exact pair hi + lo of bf16 values
+// (lo = bf16(x - hi), 2^-17 together) and its products take the terms hi.hi,
+// hi.lo and lo.hi: W, P, X, Y, B and the carries Gam_s, Lam_s.  T (it only
+// scales rows of G) and the checkpoints S_p, D_p stay single.
 //
-// TMEM (512 columns): R0 (128) A -> T -> dV; R1 (128) G V^T -> B; R2 (64) X -> dK;
-// R3 (64) Y -> dQ; R4, R5 (64 each) the carries (forward S, D; reverse Gam^T,
-// Lam), rows 0..63.  The products that do not need T or B (the carries, and the
-// parts of dQ and dK without B) are issued so that they run while the epilogue
-// forms the operands of the next ones.
+// Layout.  Token operands are bf16 in the 128-byte-swizzled layout TMA writes
+// (128 rows x 64 columns per 16 KiB block; 64 x 64 matrices in the first 64
+// rows of an 8 KiB half); X and Y go to shared memory as hi and lo blocks.  The
+// 128 x 128 masked tiles never touch shared memory: each is formed in TMEM, the
+// epilogue masks it and writes it back over its own columns as packed bf16
+// hi/lo, and the next product reads it there as its A operand.  A transposed
+// use (P^T, T^T, W^T, B^T) is its own product (V G^T, X Q^T, K Q^T, K Y^T) with
+// the mask turned over.  Products on the carries read X^T, Y^T, Q^T MN-major
+// as the M side of an M = 128 product; rows 64..127 come from the next block
+// and land in TMEM lanes nobody reads.
+//
+// TMEM (512 columns): DQ (64) Y -> dQ; DK (64) X -> dV -> dK; GAM, LAM (64 each)
+// the carries (forward S, D; reverse Gam^T, Lam), rows 0..63; T0, T1 (128 each)
+// the masked tiles: W, T^T, B, W^T in T0 and P^T, P, B^T in T1.
 //
 // Roles: warp 16 issues TMA copies and MMAs (one thread); warps 0..15 are the
 // epilogue (warp w: TMEM lanes 32 (w % 4) .. +31, one token row each; column
@@ -56,29 +66,32 @@ constexpr int kThreads = kEpiThreads + 32;
 // shared-memory blocks of 16 KiB (128 rows x 64 bf16)
 enum Block {
     bQ = 0, bK = 1, bV = 2, bG = 3,
-    bW = 4,    // 4..5: W = L . (Q K^T), 128 x 128
-    bP = 6,    // 6..7: P = L . (G V^T); forward sweep: the second Q, K, V set at 6, 7, 8
-    bT = 8,    // 8..9: T, then B
-    bX = 10, bY = 11,
-    bCk = 12,  // S_p (rows 0..63 of the first 8 KiB), D_p (the second 8 KiB): the checkpoint image
-    bCar = 13, // Gam_s^T (first 8 KiB), Lam_s (second 8 KiB), bf16 copies of the reverse carries
+    bXh = 4, bXl = 5,  // X = hi + lo
+    bYh = 6, bYl = 7,  // Y = hi + lo
+    bCk = 8,           // S_p (rows 0..63 of the first 8 KiB), D_p (the second 8 KiB): the checkpoint image
+    bGam = 9,          // Gam_s^T: hi (first 8 KiB), lo (second 8 KiB)
+    bLam = 10,         // Lam_s: hi, lo
+    bQ2 = 11,          // forward sweep: the second Q, K, V set at 11, 12, 13
     kBlocks = 14
 };
 constexpr uint32_t kHalf = kBlockBytes / 2;
 constexpr uint32_t kSmemBlocks = kBlocks * kBlockBytes;
 constexpr uint32_t kCkBytes = kBlockBytes;  // one checkpoint: S_p and D_p images
 
-constexpr uint32_t kR0 = 0, kR1 = 128, kR2 = 256, kR3 = 320, kR4 = 384, kR5 = 448;  // TMEM columns
+constexpr uint32_t kDQ = 0, kDK = 64, kGAM = 128, kLAM = 192, kT0 = 256, kT1 = 384;  // TMEM columns
 
 enum Bar {
-    bLd0 = 0, bLd1 = 1,                                        // tile copies (forward: two sets)
-    bEvA = 2, bEvX = 3, bEvT = 4, bEvB = 5, bEvV = 6, bEvO = 7, bEvC = 8,  // MMA commits
-    bEp0 = 9, bEp1 = 10, bEp2 = 11, bEp3 = 12, bEp4 = 13,    // epilogue hand-offs (16 warp arrivals)
-    bTear = 14,
-    bCkDone = 15,                                              // a head's checkpoints are in global memory
-    bEp5 = 16,                                                 // reverse sweep: P (bf16) formed after W
-    kNumBars = 17
+    bLd0 = 0, bLd1 = 1,  // tile copies (forward: two sets)
+    // MMA commits
+    bEvA = 2, bEvX = 3, bEvC = 4, bEvT = 5, bEvV = 6, bEvB = 7, bEvW = 8, bEvO = 9,
+    // epilogue hand-offs (16 warp arrivals each)
+    bEp0 = 10, bEp1 = 11, bEp2 = 12,                 // both sweeps
+    bEp1b = 13, bEp3a = 14, bEp3b = 15, bEp4a = 16, bEp4b = 17, bEp5 = 18,  // reverse sweep
+    bTear = 19,
+    bCkDone = 20,  // a head's checkpoints are in global memory
+    kNumBars = 21
 };
+__host__ __device__ constexpr bool epi_bar(int b) { return b >= bEp0 && b <= bEp5; }
 
 struct Misc {
     uint64_t bar[kNumBars];
@@ -141,11 +154,13 @@ __device__ __forceinline__ void bulk_prefetch_l2(const void *src, uint32_t bytes
 constexpr uint32_t kDescHi = (1024u >> 4) | (1u << 14) | (2u << 29);
 constexpr uint32_t kLboK = 1u << 16, kLboMN = (kBlockBytes >> 4) << 16;
 constexpr uint32_t kBlk16 = kBlockBytes >> 4;
+constexpr uint32_t kH16 = kHalf >> 4;  // the second 8 KiB of a block, in descriptor units
 
 __device__ __forceinline__ uint64_t dsc(uint32_t lo) { return (static_cast<uint64_t>(kDescHi) << 32) | lo; }
 
-// D (+)= A B over KS steps of K = 16.  K-major operands: 64 K elements per 128-byte row,
-// the next 64 in the next block; MN-major operands: 16 K rows (2 KiB) per step.
+// D (+)= A B over KS steps of K = 16, both operands in shared memory.  K-major operands:
+// 64 K elements per 128-byte row, the next 64 in the next block; MN-major operands: 16 K
+// rows (2 KiB) per step.
 template <bool A_MN, bool B_MN, int N, int KS>
 __device__ __forceinline__ void mma(uint32_t d, uint32_t a, uint32_t b, uint32_t acc) {
     constexpr uint32_t id = idesc_bf16(128, N, A_MN, B_MN);
@@ -155,6 +170,17 @@ __device__ __forceinline__ void mma(uint32_t d, uint32_t a, uint32_t b, uint32_t
         const uint32_t kb = B_MN ? kk * 128u : (kk >> 2) * kBlk16 + (kk & 3) * 2u;
         umma_bf16(d, dsc(a + ka), dsc(b + kb), id, kk > 0 ? 1u : acc);
     }
+}
+
+// D (+)= A B over the 128 tokens of a tile, A a masked tile in TMEM (bf16 pairs packed in
+// the first 16 of each 32 columns: K elements 32g .. 32g + 31 of a row in columns
+// a + 32g .. +15, so K step kk starts at column 32 (kk / 2) + 8 (kk % 2); the lo parts sit
+// 16 columns further), B a token block read MN-major, N = 64
+__device__ __forceinline__ void mma_ts(uint32_t d, uint32_t a_tmem, uint32_t b, uint32_t acc) {
+    constexpr uint32_t id = idesc_bf16(128, 64, 0, 1);
+#pragma unroll
+    for (int kk = 0; kk < 8; ++kk)
+        umma_bf16_ts(d, a_tmem + 32u * (kk >> 1) + 8u * (kk & 1), dsc(b + kk * 128u), id, kk > 0 ? 1u : acc);
 }
 
 // ------------------------------- epilogue helpers -------------------------------
@@ -167,20 +193,45 @@ __device__ __forceinline__ void st16(uint8_t *tile, int r, int c, const uint4 &v
     *reinterpret_cast<uint4 *>(tile + tile_off(r, c)) = v;
 }
 
-// 32 fp32 TMEM values of row r (columns c0 .. c0 + 31 of a 128-wide result), masked to the
-// lower triangle (column <= r), as bf16 into a 128 x 128 tile
-__device__ __forceinline__ void store_masked32(uint8_t *tile, int r, int c0, const uint32_t (&a)[32]) {
-    const bool zero = c0 > r;
-#pragma unroll
-    for (int jj = 0; jj < 32; jj += 8) {
-        float x[8];
-#pragma unroll
-        for (int u = 0; u < 8; ++u) x[u] = (!zero && c0 + jj + u <= r) ? __uint_as_float(a[jj + u]) : 0.f;
-        st16(tile, r, c0 + jj, pack8(x));
-    }
+// bf16 hi of a pair and lo = bf16(x - hi), packed
+__device__ __forceinline__ void split2(float x0, float x1, uint32_t &h, uint32_t &l) {
+    h = pack_bf16x2(x0, x1);
+    l = pack_bf16x2(x0 - __uint_as_float(h << 16), x1 - __uint_as_float(h & 0xFFFF0000u));
 }
 
-// 16 fp32 TMEM values (columns c0 .. c0 + 15 of a 64-wide result) as bf16 into row r of a block
+// One warp's 32 columns (c0 .. c0 + 31) of row r of a 128 x 128 product in TMEM at `t`:
+// masked (kUpper: column >= r, else column <= r) and written back over the same columns
+// as packed bf16, hi at c0 and (kLo) lo at c0 + 16.
+template <bool kUpper, bool kLo>
+__device__ __forceinline__ void mask_pack(uint32_t t, int r, int c0) {
+    uint32_t a[32];
+    tmem_ld32(t + c0, a);
+    tmem_ld_wait();
+    uint32_t hp[16], lp[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+        const int c = c0 + 2 * i;
+        const bool k0 = kUpper ? c >= r : c <= r, k1 = kUpper ? c + 1 >= r : c + 1 <= r;
+        split2(k0 ? __uint_as_float(a[2 * i]) : 0.f, k1 ? __uint_as_float(a[2 * i + 1]) : 0.f, hp[i], lp[i]);
+    }
+    tmem_st16(t + c0, hp);
+    if (kLo) tmem_st16(t + c0 + 16, lp);
+    tmem_st_wait();
+}
+
+// 16 fp32 TMEM values (columns c0 .. c0 + 15 of a 64-wide result) of row r as bf16 hi and
+// lo into the same row of two blocks
+__device__ __forceinline__ void store16_hl(uint8_t *hi, uint8_t *lo, int r, int c0, const uint32_t (&a)[16]) {
+    uint32_t h[8], l[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) split2(__uint_as_float(a[2 * i]), __uint_as_float(a[2 * i + 1]), h[i], l[i]);
+    st16(hi, r, c0, make_uint4(h[0], h[1], h[2], h[3]));
+    st16(hi, r, c0 + 8, make_uint4(h[4], h[5], h[6], h[7]));
+    st16(lo, r, c0, make_uint4(l[0], l[1], l[2], l[3]));
+    st16(lo, r, c0 + 8, make_uint4(l[4], l[5], l[6], l[7]));
+}
+
+// the same, bf16 only
 __device__ __forceinline__ void store16(uint8_t *blk, int r, int c0, const uint32_t (&a)[16]) {
     float x[16];
 #pragma unroll
@@ -217,8 +268,7 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
         return;
     }
     if (tid == 0) {
-        for (int b = 0; b < kNumBars; ++b)
-            mbar_init(&ms->bar[b], ((b >= bEp0 && b <= bEp4) || b == bEp5) ? kEpiWarps : 1);
+        for (int b = 0; b < kNumBars; ++b) mbar_init(&ms->bar[b], epi_bar(b) ? kEpiWarps : 1);
         ms->abort_flag = 0;
         fence_mbar_init();
     }
@@ -240,12 +290,13 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
             const uint32_t sb4 = smem_u32(smem) >> 4;
             auto lk = [&](int b) { return sb4 + (uint32_t)b * kBlk16 + kLboK; };   // K-major block
             auto lm = [&](int b) { return sb4 + (uint32_t)b * kBlk16 + kLboMN; };  // MN-major block
-            constexpr uint32_t kH16 = kHalf >> 4;  // the second 8 KiB of a block
+            const uint32_t DQ = tb + kDQ, DK = tb + kDK, GAM = tb + kGAM, LAM = tb + kLAM;
+            const uint32_t T0 = tb + kT0, T1 = tb + kT1;
             // tile counters: n_s every tile of both sweeps (the barriers both use), n_f forward
             // tiles, n_b reverse tiles
             uint32_t ld_par = 0, ld_pend = 0, n_s = 0, n_f = 0, n_b = 0, n_head = 0;
-            auto load_fwd = [&](int set, int head, int j) {  // Q, K, V of tile j into blocks 0..2 or 6..8
-                const int b0 = set ? bP : bQ;
+            auto load_fwd = [&](int set, int head, int j) {  // Q, K, V of tile j into blocks 0..2 or 11..13
+                const int b0 = set ? bQ2 : bQ;
                 ld_pend |= 1u << set;
                 mbar_arrive_expect_tx(&ms->bar[bLd0 + set], 3 * kBlockBytes);
                 tma_load_3d(blk(b0), &tm_q, &ms->bar[bLd0 + set], 0, j * kTile, head);
@@ -274,23 +325,25 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                 bool ok = true;
                 for (int j = 0; j < M && ok; ++j, ++n_f, ++n_s) {
                     const uint32_t tp = n_s & 1, tf = n_f & 1;
-                    const int set = j & 1, qb = set ? bP : bQ;
+                    const int set = j & 1, qb = set ? bQ2 : bQ, kb = qb + 1, vb = qb + 2;
                     ok = false;
                     if (!bar_wait(ms, bEp0, tp, p) || !wait_ld(set)) break;  // S_p (bf16) in bCk; tokens
                     tc_fence_after();
-                    mma<false, false, 128, 4>(tb + kR0, lk(qb), lk(qb + 1), 0u);   // A = Q K^T
+                    mma<false, false, 128, 4>(T0, lk(qb), lk(kb), 0u);  // A = Q K^T
                     umma_commit(&ms->bar[bEvA]);
-                    mma<true, true, 64, 8>(tb + kR4, lm(qb + 1), lm(qb + 1), 1u);  // S += K^T K (under E1)
-                    if (!bar_wait(ms, bEp1, tp, p)) break;                        // W in bW
+                    mma<true, true, 64, 8>(GAM, lm(kb), lm(kb), 1u);  // S += K^T K (under E1)
+                    if (!bar_wait(ms, bEp1, tp, p)) break;           // W (hi, lo) packed in T0
                     tc_fence_after();
-                    mma<false, true, 64, 8>(tb + kR2, lk(bW), lm(qb + 1), 0u);     // X = W K
-                    mma<false, false, 64, 4>(tb + kR2, lk(qb), lk(bCk), 1u);       //   + Q S_p
+                    mma_ts(DK, T0, lm(kb), 0u);                       // X = W K
+                    mma_ts(DK, T0 + 16, lm(kb), 1u);
+                    mma<false, false, 64, 4>(DK, lk(qb), lk(bCk), 1u);  //   + Q S_p
                     umma_commit(&ms->bar[bEvX]);
-                    if (!bar_wait(ms, bEp2, tp, p)) break;                        // X (bf16) in bX
+                    if (!bar_wait(ms, bEp2, tp, p)) break;  // X (hi, lo) in bXh, bXl
                     tc_fence_after();
-                    mma<true, true, 64, 8>(tb + kR5, lm(bX), lm(qb + 2), 1u);      // D += X^T V
+                    mma<true, true, 64, 8>(LAM, lm(bXh), lm(vb), 1u);  // D += X^T V
+                    mma<true, true, 64, 8>(LAM, lm(bXl), lm(vb), 1u);
                     umma_commit(&ms->bar[bEvC]);
-                    if (!bar_wait(ms, bEvC, tf, p)) break;                        // this set is free again
+                    if (!bar_wait(ms, bEvC, tf, p)) break;  // this set is free again
                     if (j + 2 < M) load_fwd(set, head, j + 2);
                     ok = true;
                 }
@@ -311,46 +364,73 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                         bulk_prefetch_l2(tok.g + t0 * kD, bytes);
                         bulk_prefetch_l2(p.ck + ((size_t)head * M + j - 1) * kCkBytes, kCkBytes);
                     }
-                    if (!bar_wait(ms, bEp0, ts, p) || !wait_ld(0)) break;  // Gam^T, Lam (bf16); tokens
+                    if (!bar_wait(ms, bEp0, ts, p) || !wait_ld(0)) break;  // Gam_s, Lam_s (hi, lo); tokens
                     tc_fence_after();
-                    mma<false, false, 128, 4>(tb + kR0, lk(bQ), lk(bK), 0u);        // A = Q K^T
-                    mma<false, false, 128, 4>(tb + kR1, lk(bG), lk(bV), 0u);        // G V^T
+                    mma<false, false, 128, 4>(T0, lk(bQ), lk(bK), 0u);  // A = Q K^T
+                    mma<false, false, 128, 4>(T1, lk(bV), lk(bG), 0u);  // P^T = V G^T
                     umma_commit(&ms->bar[bEvA]);
-                    mma<true, true, 64, 8>(tb + kR4, lm(bQ), lm(bG), 1u);           // Gam^T += Q^T G (under E1)
-                    if (!bar_wait(ms, bEp1, ts, p)) break;            // W (bf16)
+                    if (!bar_wait(ms, bEp1, ts, p)) break;  // W in T0
                     tc_fence_after();
-                    mma<false, true, 64, 8>(tb + kR2, lk(bW), lm(bK), 0u);          // X = W K
-                    mma<false, false, 64, 4>(tb + kR2, lk(bQ), lk(bCk), 1u);        //   + Q S_p
-                    if (!bar_wait(ms, bEp5, tp, p)) break;            // P (bf16)
+                    mma_ts(DK, T0, lm(bK), 0u);  // X = W K
+                    mma_ts(DK, T0 + 16, lm(bK), 1u);
+                    mma<false, false, 64, 4>(DK, lk(bQ), lk(bCk), 1u);  //   + Q S_p
+                    if (!bar_wait(ms, bEp1b, tp, p)) break;             // P^T in T1
                     tc_fence_after();
-                    mma<true, true, 64, 8>(tb + kR3, lm(bP), lm(bQ), 0u);           // Y = P^T Q
-                    mma<false, false, 64, 4>(tb + kR3, lk(bV), lk(bCar), 1u);       //   + V Gam_s
+                    mma_ts(DQ, T1, lm(bQ), 0u);  // Y = P^T Q
+                    mma_ts(DQ, T1 + 16, lm(bQ), 1u);
+                    mma<false, false, 64, 4>(DQ, lk(bV), lk(bGam), 1u);  //   + V Gam_s
+                    mma<false, false, 64, 4>(DQ, lk(bV), lk(bGam) + kH16, 1u);
                     umma_commit(&ms->bar[bEvX]);
-                    if (!bar_wait(ms, bEp2, ts, p)) break;            // X, Y (bf16); R2, R3 read
+                    if (!bar_wait(ms, bEp2, ts, p)) break;  // X, Y (hi, lo) in shared memory; DK, DQ read
                     tc_fence_after();
-                    mma<false, false, 128, 4>(tb + kR0, lk(bQ), lk(bX), 0u);        // T = Q X^T
+                    mma<false, false, 128, 4>(T0, lk(bXh), lk(bQ), 0u);  // T^T = X Q^T
+                    mma<false, false, 128, 4>(T0, lk(bXl), lk(bQ), 1u);
+                    mma<false, false, 128, 4>(T1, lk(bG), lk(bV), 0u);   // P = G V^T
                     umma_commit(&ms->bar[bEvT]);
-                    mma<false, false, 128, 4>(tb + kR1, lk(bY), lk(bK), 0u);        // B = Y K^T
-                    umma_commit(&ms->bar[bEvB]);
-                    if (!bar_wait(ms, bEp3, tp, p)) break;                         // T (bf16) in bT; R0 read
+                    mma<true, true, 64, 8>(GAM, lm(bQ), lm(bG), 1u);   // Gam^T += Q^T G
+                    mma<true, true, 64, 8>(LAM, lm(bYh), lm(bQ), 1u);  // Lam += Y^T Q
+                    mma<true, true, 64, 8>(LAM, lm(bYl), lm(bQ), 1u);
+                    mma<true, true, 64, 8>(LAM, lm(bQ), lm(bYh), 1u);  //   + Q^T Y
+                    mma<true, true, 64, 8>(LAM, lm(bQ), lm(bYl), 1u);
+                    if (!bar_wait(ms, bEp3a, tp, p)) break;  // T^T in T0
                     tc_fence_after();
-                    mma<true, true, 64, 8>(tb + kR0, lm(bT), lm(bG), 0u);           // dV = T^T G
-                    mma<false, true, 64, 4>(tb + kR0, lk(bX), lm(bCar), 1u);        //   + X Gam_s^T
+                    mma_ts(DK, T0, lm(bG), 0u);                                 // dV = T^T G
+                    mma<false, true, 64, 4>(DK, lk(bXh), lm(bGam), 1u);         //   + X Gam_s^T
+                    mma<false, true, 64, 4>(DK, lk(bXh), lm(bGam) + kH16, 1u);
+                    mma<false, true, 64, 4>(DK, lk(bXl), lm(bGam), 1u);
                     umma_commit(&ms->bar[bEvV]);
-                    // while dV goes out and the epilogue forms B: the parts of dQ and dK without B, Lam
-                    mma<false, true, 64, 8>(tb + kR3, lk(bP), lm(bX), 0u);          // dQ = P X
-                    mma<false, false, 64, 4>(tb + kR3, lk(bG), lk(bCk) + kH16, 1u); //   + G D_p^T
-                    mma<false, false, 64, 4>(tb + kR3, lk(bY), lk(bCk), 1u);        //   + Y S_p
-                    mma<false, false, 64, 4>(tb + kR2, lk(bK), lk(bCar) + kH16, 0u);  // dK = K Lam_s
-                    mma<true, true, 64, 8>(tb + kR2, lm(bW), lm(bY), 1u);           //   + W^T Y
-                    mma<true, true, 64, 8>(tb + kR5, lm(bY), lm(bQ), 1u);           // Lam += Y^T Q
-                    mma<true, true, 64, 8>(tb + kR5, lm(bQ), lm(bY), 1u);           //   + Q^T Y
-                    if (!bar_wait(ms, bEp4, tp, p)) break;                         // B (bf16) in bT
+                    mma<false, false, 128, 4>(T0, lk(bYh), lk(bK), 0u);  // B = Y K^T
+                    mma<false, false, 128, 4>(T0, lk(bYl), lk(bK), 1u);
+                    if (!bar_wait(ms, bEp3b, tp, p)) break;  // P in T1
                     tc_fence_after();
-                    mma<false, true, 64, 8>(tb + kR3, lk(bT), lm(bK), 1u);          // dQ += B K
-                    mma<true, true, 64, 8>(tb + kR2, lm(bT), lm(bQ), 1u);           // dK += B^T Q
+                    mma_ts(DQ, T1, lm(bXh), 0u);  // dQ = P X
+                    mma_ts(DQ, T1, lm(bXl), 1u);
+                    mma_ts(DQ, T1 + 16, lm(bXh), 1u);
+                    mma<false, false, 64, 4>(DQ, lk(bG), lk(bCk) + kH16, 1u);  //   + G D_p^T
+                    mma<false, false, 64, 4>(DQ, lk(bYh), lk(bCk), 1u);        //   + Y S_p
+                    mma<false, false, 64, 4>(DQ, lk(bYl), lk(bCk), 1u);
+                    mma<false, false, 128, 4>(T1, lk(bK), lk(bYh), 0u);  // B^T = K Y^T
+                    mma<false, false, 128, 4>(T1, lk(bK), lk(bYl), 1u);
+                    umma_commit(&ms->bar[bEvB]);
+                    if (!bar_wait(ms, bEp4a, tp, p)) break;  // B in T0; dV out of DK
+                    tc_fence_after();
+                    mma_ts(DQ, T0, lm(bK), 1u);  // dQ += B K
+                    mma_ts(DQ, T0 + 16, lm(bK), 1u);
+                    mma<false, false, 128, 4>(T0, lk(bK), lk(bQ), 0u);  // W^T = K Q^T
+                    if (!bar_wait(ms, bEp4b, tp, p)) break;             // B^T in T1
+                    tc_fence_after();
+                    mma<false, false, 64, 4>(DK, lk(bK), lk(bLam), 0u);  // dK = K Lam_s
+                    mma<false, false, 64, 4>(DK, lk(bK), lk(bLam) + kH16, 1u);
+                    mma_ts(DK, T1, lm(bQ), 1u);  //   + B^T Q
+                    mma_ts(DK, T1 + 16, lm(bQ), 1u);
+                    umma_commit(&ms->bar[bEvW]);
+                    if (!bar_wait(ms, bEp5, tp, p)) break;  // W^T in T0
+                    tc_fence_after();
+                    mma_ts(DK, T0, lm(bYh), 1u);  //   + W^T Y
+                    mma_ts(DK, T0, lm(bYl), 1u);
+                    mma_ts(DK, T0 + 16, lm(bYh), 1u);
                     umma_commit(&ms->bar[bEvO]);
-                    if (!bar_wait(ms, bEvO, tp, p)) break;                         // every operand read
+                    if (!bar_wait(ms, bEvO, tp, p)) break;  // every operand read
                     if (j > 0) load_bwd(head, j - 1);
                     ok = true;
                 }
@@ -369,27 +449,30 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
         const int qd = warp & 3, cq = warp >> 2;
         const int r = 32 * qd + lane;
         const uint32_t lb = (uint32_t)(32 * qd) << 16;
+        const uint32_t t0 = tb + lb + kT0, t1 = tb + lb + kT1, c32 = 32u * cq, c16 = 16u * cq;
         uint32_t n_s = 0, n_f = 0, n_b = 0, n_head = 0;
-        auto zero_carries = [&]() {  // rows 0..63 of R4 and R5
+        auto zero_carries = [&]() {  // rows 0..63 of GAM and LAM
             if (qd < 2) {
                 uint32_t z[16];
 #pragma unroll
                 for (int u = 0; u < 16; ++u) z[u] = 0u;
-                tmem_st16(tb + lb + kR4 + 16 * cq, z);
-                tmem_st16(tb + lb + kR5 + 16 * cq, z);
+                tmem_st16(tb + lb + kGAM + c16, z);
+                tmem_st16(tb + lb + kLAM + c16, z);
                 tmem_st_wait();
             }
         };
-        // rows 0..63 of R4 and R5 as bf16 into the two 8 KiB halves of a block
-        auto carries_bf16 = [&](uint8_t *dst) {
-            if (qd < 2) {
-                uint32_t a[16], b[16];
-                tmem_ld16(tb + lb + kR4 + 16 * cq, a);
-                tmem_ld16(tb + lb + kR5 + 16 * cq, b);
-                tmem_ld_wait();
-                store16(dst, r, 16 * cq, a);
-                store16(dst + kHalf, r, 16 * cq, b);
-            }
+        // a 64-wide result in TMEM at column `col` -> row r of a block as bf16 hi and lo
+        auto to_smem_hl = [&](uint32_t col, int bh, int bl) {
+            uint32_t a[16];
+            tmem_ld16(tb + lb + col + c16, a);
+            tmem_ld_wait();
+            store16_hl(blk(bh), blk(bl), r, c16, a);
+        };
+        auto drain = [&](uint32_t col, __nv_bfloat16 *dst, bool ok) {  // a 64-wide result -> global
+            uint32_t a[16];
+            tmem_ld16(tb + lb + col + c16, a);
+            tmem_ld_wait();
+            if (ok) out16(dst, a);
         };
         for (int head = blockIdx.x; head < p.BH; head += gridDim.x, ++n_head) {
             // ---------------- forward sweep ----------------
@@ -403,7 +486,14 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                     if (tid == 0) tma_store_wait_read();  // its checkpoint copy has left bCk
                     epi_sync();
                 }
-                carries_bf16(blk(bCk));
+                if (qd < 2) {
+                    uint32_t a[16], b[16];
+                    tmem_ld16(tb + lb + kGAM + c16, a);
+                    tmem_ld16(tb + lb + kLAM + c16, b);
+                    tmem_ld_wait();
+                    store16(blk(bCk), r, c16, a);
+                    store16(blk(bCk) + kHalf, r, c16, b);
+                }
                 fence_async_smem();
                 epi_sync();
                 if (tid == 0) {
@@ -411,30 +501,19 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                     tma_store_commit();
                 }
                 epi_arrive(ms, bEp0);
-                // E1: W = L . A
+                // E1: W = L . A, packed hi/lo over A
                 bar_wait(ms, bEvA, tp, p);
                 tc_fence_after();
-                {
-                    uint32_t a[32];
-                    tmem_ld32(tb + lb + kR0 + 32 * cq, a);
-                    tmem_ld_wait();
-                    store_masked32(blk(bW), r, 32 * cq, a);
-                }
-                fence_async_smem();
+                mask_pack<false, true>(t0, r, c32);
                 epi_arrive(ms, bEp1);
-                // E2: X -> bf16
+                // E2: X -> hi, lo
                 bar_wait(ms, bEvX, tp, p);
                 tc_fence_after();
-                {
-                    uint32_t x[16];
-                    tmem_ld16(tb + lb + kR2 + 16 * cq, x);
-                    tmem_ld_wait();
-                    store16(blk(bX), r, 16 * cq, x);
-                }
+                to_smem_hl(kDK, bXh, bXl);
                 fence_async_smem();
                 epi_arrive(ms, bEp2);
             }
-            bar_wait(ms, bEvC, (n_f - 1) & 1u, p);  // the last carry products (before R4, R5 are reset)
+            bar_wait(ms, bEvC, (n_f - 1) & 1u, p);  // the last carry products (before GAM, LAM are reset)
             tc_fence_after();
             if (tid == 0) {
                 tma_store_wait_all();  // every checkpoint is in global memory
@@ -446,82 +525,59 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                 const uint32_t ts = n_s & 1, tp = n_b & 1;
                 const int tok0 = j * kTile;
                 const bool row_ok = tok0 + r < p.n;
-                const size_t orow = ((size_t)head * p.n + tok0 + r) * kD + 16 * cq;
-                // E0: Gam_s^T, Lam_s -> bf16 (the previous tile's products are done: waited in E4)
-                carries_bf16(blk(bCar));
+                const size_t orow = ((size_t)head * p.n + tok0 + r) * kD + c16;
+                // E0: Gam_s^T, Lam_s -> hi, lo (the previous tile's products are done: waited in E6)
+                if (qd < 2) {
+                    uint32_t a[16], b[16];
+                    tmem_ld16(tb + lb + kGAM + c16, a);
+                    tmem_ld16(tb + lb + kLAM + c16, b);
+                    tmem_ld_wait();
+                    store16_hl(blk(bGam), blk(bGam) + kHalf, r, c16, a);
+                    store16_hl(blk(bLam), blk(bLam) + kHalf, r, c16, b);
+                }
                 fence_async_smem();
                 epi_arrive(ms, bEp0);
-                // E1: W = L . A (X = W K starts on it), then P = L . (G V^T)
+                // E1: W = L . A over T0 (X = W K starts on it), then P^T = L^T . (V G^T) over T1
                 bar_wait(ms, bEvA, ts, p);
                 tc_fence_after();
-                {
-                    uint32_t a[32];
-                    tmem_ld32(tb + lb + kR0 + 32 * cq, a);
-                    tmem_ld_wait();
-                    store_masked32(blk(bW), r, 32 * cq, a);
-                    fence_async_smem();
-                    epi_arrive(ms, bEp1);
-                    tmem_ld32(tb + lb + kR1 + 32 * cq, a);
-                    tmem_ld_wait();
-                    store_masked32(blk(bP), r, 32 * cq, a);
-                }
-                fence_async_smem();
-                epi_arrive(ms, bEp5);
-                // E2: X, Y -> bf16
+                mask_pack<false, true>(t0, r, c32);
+                epi_arrive(ms, bEp1);
+                mask_pack<true, true>(t1, r, c32);
+                epi_arrive(ms, bEp1b);
+                // E2: X, Y -> hi, lo
                 bar_wait(ms, bEvX, ts, p);
                 tc_fence_after();
-                {
-                    uint32_t x[16];
-                    tmem_ld16(tb + lb + kR2 + 16 * cq, x);
-                    tmem_ld_wait();
-                    store16(blk(bX), r, 16 * cq, x);
-                    tmem_ld16(tb + lb + kR3 + 16 * cq, x);
-                    tmem_ld_wait();
-                    store16(blk(bY), r, 16 * cq, x);
-                }
+                to_smem_hl(kDK, bXh, bXl);
+                to_smem_hl(kDQ, bYh, bYl);
                 fence_async_smem();
                 epi_arrive(ms, bEp2);
-                // E3: T = L . (Q X^T) -> bf16
+                // E3: T^T = L^T . (X Q^T) over T0 (bf16 only), P = L . (G V^T) over T1
                 bar_wait(ms, bEvT, tp, p);
                 tc_fence_after();
-                {
-                    uint32_t a[32];
-                    tmem_ld32(tb + lb + kR0 + 32 * cq, a);
-                    tmem_ld_wait();
-                    store_masked32(blk(bT), r, 32 * cq, a);
-                }
-                fence_async_smem();
-                epi_arrive(ms, bEp3);
-                // B = L . (Y K^T) -> bf16 over T (the dV products have read T), then dV out
+                mask_pack<true, false>(t0, r, c32);
+                epi_arrive(ms, bEp3a);
+                mask_pack<false, true>(t1, r, c32);
+                epi_arrive(ms, bEp3b);
+                // E4: dV out, then B = L . (Y K^T) over T0 and B^T over T1
                 bar_wait(ms, bEvV, tp, p);
+                tc_fence_after();
+                drain(kDK, p.dv + orow, row_ok);
                 bar_wait(ms, bEvB, tp, p);
                 tc_fence_after();
-                {
-                    uint32_t a[32];
-                    tmem_ld32(tb + lb + kR1 + 32 * cq, a);
-                    tmem_ld_wait();
-                    store_masked32(blk(bT), r, 32 * cq, a);
-                }
-                fence_async_smem();
-                epi_arrive(ms, bEp4);
-                {
-                    uint32_t x[16];
-                    tmem_ld16(tb + lb + kR0 + 16 * cq, x);
-                    tmem_ld_wait();
-                    if (row_ok) out16(p.dv + orow, x);
-                }
-                // dQ, dK out
+                mask_pack<false, true>(t0, r, c32);
+                epi_arrive(ms, bEp4a);
+                mask_pack<true, true>(t1, r, c32);
+                epi_arrive(ms, bEp4b);
+                // E5: W^T = L^T . (K Q^T) over T0, then dQ out
+                bar_wait(ms, bEvW, tp, p);
+                tc_fence_after();
+                mask_pack<true, true>(t0, r, c32);
+                epi_arrive(ms, bEp5);
+                drain(kDQ, p.dq + orow, row_ok);
+                // E6: dK out
                 bar_wait(ms, bEvO, tp, p);
                 tc_fence_after();
-                {
-                    uint32_t x[16];
-                    tmem_ld16(tb + lb + kR3 + 16 * cq, x);
-                    tmem_ld_wait();
-                    if (row_ok) out16(p.dq + orow, x);
-                    tmem_ld16(tb + lb + kR2 + 16 * cq, x);
-                    tmem_ld_wait();
-                    if (row_ok) out16(p.dk + orow, x);
-                }
+                drain(kDK, p.dk + orow, row_ok);
             }
         }
         if (tid == 0) tma_store_wait_all();
