@@ -71,7 +71,7 @@ enum Block {
     bCk = 8,           // S_p (rows 0..63 of the first 8 KiB), D_p (the second 8 KiB): the checkpoint image
     bGam = 9,          // Gam_s^T: hi (first 8 KiB), lo (second 8 KiB)
     bLam = 10,         // Lam_s: hi, lo
-    bQ2 = 11,          // forward sweep: the second Q, K, V set at 11, 12, 13
+    bQ2 = 11,          // the second Q, K, V set at 11, 12, 13 (tiles alternate between the sets)
     kBlocks = 14
 };
 constexpr uint32_t kHalf = kBlockBytes / 2;
@@ -81,15 +81,16 @@ constexpr uint32_t kCkBytes = kBlockBytes;  // one checkpoint: S_p and D_p image
 constexpr uint32_t kDQ = 0, kDK = 64, kGAM = 128, kLAM = 192, kT0 = 256, kT1 = 384;  // TMEM columns
 
 enum Bar {
-    bLd0 = 0, bLd1 = 1,  // tile copies (forward: two sets)
+    bLd0 = 0, bLd1 = 1,  // tile copies: the two Q, K, V sets
+    bLdG = 2,            // reverse sweep: G and the checkpoint
     // MMA commits
-    bEvA = 2, bEvX = 3, bEvC = 4, bEvT = 5, bEvV = 6, bEvB = 7, bEvW = 8, bEvO = 9,
+    bEvA = 3, bEvA2 = 4, bEvX = 5, bEvC = 6, bEvT = 7, bEvV = 8, bEvB = 9, bEvW = 10, bEvO = 11,
     // epilogue hand-offs (16 warp arrivals each)
-    bEp0 = 10, bEp1 = 11, bEp2 = 12,                 // both sweeps
-    bEp1b = 13, bEp3a = 14, bEp3b = 15, bEp4a = 16, bEp4b = 17, bEp5 = 18,  // reverse sweep
-    bTear = 19,
-    bCkDone = 20,  // a head's checkpoints are in global memory
-    kNumBars = 21
+    bEp0 = 12, bEp1 = 13, bEp2 = 14,                 // both sweeps
+    bEp1b = 15, bEp3a = 16, bEp3b = 17, bEp4a = 18, bEp4b = 19, bEp5 = 20,  // reverse sweep
+    bTear = 21,
+    bCkDone = 22,  // a head's checkpoints are in global memory
+    kNumBars = 23
 };
 __host__ __device__ constexpr bool epi_bar(int b) { return b >= bEp0 && b <= bEp5; }
 
@@ -303,16 +304,13 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                 tma_load_3d(blk(b0 + 1), &tm_k, &ms->bar[bLd0 + set], 0, j * kTile, head);
                 tma_load_3d(blk(b0 + 2), &tm_v, &ms->bar[bLd0 + set], 0, j * kTile, head);
             };
-            auto load_bwd = [&](int head, int j) {  // Q, K, V, G of tile j and its checkpoint
-                ld_pend |= 1u;
-                mbar_arrive_expect_tx(&ms->bar[bLd0], 4 * kBlockBytes + kCkBytes);
-                tma_load_3d(blk(bQ), &tm_q, &ms->bar[bLd0], 0, j * kTile, head);
-                tma_load_3d(blk(bK), &tm_k, &ms->bar[bLd0], 0, j * kTile, head);
-                tma_load_3d(blk(bV), &tm_v, &ms->bar[bLd0], 0, j * kTile, head);
-                tma_load_3d(blk(bG), &tm_g, &ms->bar[bLd0], 0, j * kTile, head);
-                bulk_load(blk(bCk), p.ck + ((size_t)head * M + j) * kCkBytes, kCkBytes, &ms->bar[bLd0]);
+            auto load_gck = [&](int head, int j) {  // G of tile j and its checkpoint
+                ld_pend |= 4u;
+                mbar_arrive_expect_tx(&ms->bar[bLdG], kBlockBytes + kCkBytes);
+                tma_load_3d(blk(bG), &tm_g, &ms->bar[bLdG], 0, j * kTile, head);
+                bulk_load(blk(bCk), p.ck + ((size_t)head * M + j) * kCkBytes, kCkBytes, &ms->bar[bLdG]);
             };
-            auto wait_ld = [&](int set) {
+            auto wait_ld = [&](int set) {  // set 0, 1: a Q, K, V set; 2: G and the checkpoint
                 if (!bar_wait(ms, bLd0 + set, (ld_par >> set) & 1u, p)) return false;
                 ld_par ^= 1u << set;
                 ld_pend &= ~(1u << set);
@@ -351,47 +349,45 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                 // the checkpoints are in global memory (the epilogue waited for its copies)
                 if (!bar_wait(ms, bCkDone, n_head & 1, p)) break;
                 // ---------------- reverse sweep: gradients ----------------
-                load_bwd(head, M - 1);
+                load_fwd(0, head, M - 1);
+                load_gck(head, M - 1);
                 for (int j = M - 1; j >= 0 && ok; --j, ++n_b, ++n_s) {
                     const uint32_t ts = n_s & 1, tp = n_b & 1;
+                    const int set = (M - 1 - j) & 1, qb = set ? bQ2 : bQ, kb = qb + 1, vb = qb + 2;
                     ok = false;
-                    if (j > 0) {  // the next tile's tokens and checkpoint towards L2
+                    if (j > 0) {  // the other set is free (the previous tile's products are done)
+                        load_fwd(set ^ 1, head, j - 1);
                         const size_t t0 = (size_t)head * p.n + (size_t)(j - 1) * kTile;
                         const uint32_t bytes = (uint32_t)min(kTile, p.n - (j - 1) * kTile) * kD * 2;
-                        bulk_prefetch_l2(tok.q + t0 * kD, bytes);
-                        bulk_prefetch_l2(tok.k + t0 * kD, bytes);
-                        bulk_prefetch_l2(tok.v + t0 * kD, bytes);
-                        bulk_prefetch_l2(tok.g + t0 * kD, bytes);
+                        bulk_prefetch_l2(tok.g + t0 * kD, bytes);  // G and the checkpoint towards L2
                         bulk_prefetch_l2(p.ck + ((size_t)head * M + j - 1) * kCkBytes, kCkBytes);
                     }
-                    if (!bar_wait(ms, bEp0, ts, p) || !wait_ld(0)) break;  // Gam_s, Lam_s (hi, lo); tokens
+                    if (!bar_wait(ms, bEp0, ts, p) || !wait_ld(set)) break;  // Gam_s, Lam_s (hi, lo); Q, K, V
                     tc_fence_after();
-                    mma<false, false, 128, 4>(T0, lk(bQ), lk(bK), 0u);  // A = Q K^T
-                    mma<false, false, 128, 4>(T1, lk(bV), lk(bG), 0u);  // P^T = V G^T
+                    mma<false, false, 128, 4>(T0, lk(qb), lk(kb), 0u);  // A = Q K^T
                     umma_commit(&ms->bar[bEvA]);
-                    if (!bar_wait(ms, bEp1, ts, p)) break;  // W in T0
+                    if (!wait_ld(2)) break;  // G, checkpoint
+                    mma<false, false, 128, 4>(T1, lk(vb), lk(bG), 0u);  // P^T = V G^T
+                    umma_commit(&ms->bar[bEvA2]);
+                    mma<true, true, 64, 8>(GAM, lm(qb), lm(bG), 1u);  // Gam^T += Q^T G
+                    if (!bar_wait(ms, bEp1, ts, p)) break;           // W in T0
                     tc_fence_after();
-                    mma_ts(DK, T0, lm(bK), 0u);  // X = W K
-                    mma_ts(DK, T0 + 16, lm(bK), 1u);
-                    mma<false, false, 64, 4>(DK, lk(bQ), lk(bCk), 1u);  //   + Q S_p
+                    mma_ts(DK, T0, lm(kb), 0u);  // X = W K
+                    mma_ts(DK, T0 + 16, lm(kb), 1u);
+                    mma<false, false, 64, 4>(DK, lk(qb), lk(bCk), 1u);  //   + Q S_p
                     if (!bar_wait(ms, bEp1b, tp, p)) break;             // P^T in T1
                     tc_fence_after();
-                    mma_ts(DQ, T1, lm(bQ), 0u);  // Y = P^T Q
-                    mma_ts(DQ, T1 + 16, lm(bQ), 1u);
-                    mma<false, false, 64, 4>(DQ, lk(bV), lk(bGam), 1u);  //   + V Gam_s
-                    mma<false, false, 64, 4>(DQ, lk(bV), lk(bGam) + kH16, 1u);
+                    mma_ts(DQ, T1, lm(qb), 0u);  // Y = P^T Q
+                    mma_ts(DQ, T1 + 16, lm(qb), 1u);
+                    mma<false, false, 64, 4>(DQ, lk(vb), lk(bGam), 1u);  //   + V Gam_s
+                    mma<false, false, 64, 4>(DQ, lk(vb), lk(bGam) + kH16, 1u);
                     umma_commit(&ms->bar[bEvX]);
                     if (!bar_wait(ms, bEp2, ts, p)) break;  // X, Y (hi, lo) in shared memory; DK, DQ read
                     tc_fence_after();
-                    mma<false, false, 128, 4>(T0, lk(bXh), lk(bQ), 0u);  // T^T = X Q^T
-                    mma<false, false, 128, 4>(T0, lk(bXl), lk(bQ), 1u);
-                    mma<false, false, 128, 4>(T1, lk(bG), lk(bV), 0u);   // P = G V^T
+                    mma<false, false, 128, 4>(T0, lk(bXh), lk(qb), 0u);  // T^T = X Q^T
+                    mma<false, false, 128, 4>(T0, lk(bXl), lk(qb), 1u);
+                    mma<false, false, 128, 4>(T1, lk(bG), lk(vb), 0u);   // P = G V^T
                     umma_commit(&ms->bar[bEvT]);
-                    mma<true, true, 64, 8>(GAM, lm(bQ), lm(bG), 1u);   // Gam^T += Q^T G
-                    mma<true, true, 64, 8>(LAM, lm(bYh), lm(bQ), 1u);  // Lam += Y^T Q
-                    mma<true, true, 64, 8>(LAM, lm(bYl), lm(bQ), 1u);
-                    mma<true, true, 64, 8>(LAM, lm(bQ), lm(bYh), 1u);  //   + Q^T Y
-                    mma<true, true, 64, 8>(LAM, lm(bQ), lm(bYl), 1u);
                     if (!bar_wait(ms, bEp3a, tp, p)) break;  // T^T in T0
                     tc_fence_after();
                     mma_ts(DK, T0, lm(bG), 0u);                                 // dV = T^T G
@@ -399,8 +395,8 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                     mma<false, true, 64, 4>(DK, lk(bXh), lm(bGam) + kH16, 1u);
                     mma<false, true, 64, 4>(DK, lk(bXl), lm(bGam), 1u);
                     umma_commit(&ms->bar[bEvV]);
-                    mma<false, false, 128, 4>(T0, lk(bYh), lk(bK), 0u);  // B = Y K^T
-                    mma<false, false, 128, 4>(T0, lk(bYl), lk(bK), 1u);
+                    mma<false, false, 128, 4>(T0, lk(bYh), lk(kb), 0u);  // B = Y K^T
+                    mma<false, false, 128, 4>(T0, lk(bYl), lk(kb), 1u);
                     if (!bar_wait(ms, bEp3b, tp, p)) break;  // P in T1
                     tc_fence_after();
                     mma_ts(DQ, T1, lm(bXh), 0u);  // dQ = P X
@@ -409,29 +405,33 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                     mma<false, false, 64, 4>(DQ, lk(bG), lk(bCk) + kH16, 1u);  //   + G D_p^T
                     mma<false, false, 64, 4>(DQ, lk(bYh), lk(bCk), 1u);        //   + Y S_p
                     mma<false, false, 64, 4>(DQ, lk(bYl), lk(bCk), 1u);
-                    mma<false, false, 128, 4>(T1, lk(bK), lk(bYh), 0u);  // B^T = K Y^T
-                    mma<false, false, 128, 4>(T1, lk(bK), lk(bYl), 1u);
+                    mma<false, false, 128, 4>(T1, lk(kb), lk(bYh), 0u);  // B^T = K Y^T
+                    mma<false, false, 128, 4>(T1, lk(kb), lk(bYl), 1u);
                     umma_commit(&ms->bar[bEvB]);
-                    if (!bar_wait(ms, bEp4a, tp, p)) break;  // B in T0; dV out of DK
+                    if (!bar_wait(ms, bEp4a, tp, p)) break;  // B in T0; dV out of DK; G, checkpoint read
                     tc_fence_after();
-                    mma_ts(DQ, T0, lm(bK), 1u);  // dQ += B K
-                    mma_ts(DQ, T0 + 16, lm(bK), 1u);
-                    mma<false, false, 128, 4>(T0, lk(bK), lk(bQ), 0u);  // W^T = K Q^T
+                    if (j > 0) load_gck(head, j - 1);
+                    mma_ts(DQ, T0, lm(kb), 1u);  // dQ += B K
+                    mma_ts(DQ, T0 + 16, lm(kb), 1u);
+                    mma<false, false, 128, 4>(T0, lk(kb), lk(qb), 0u);  // W^T = K Q^T
                     if (!bar_wait(ms, bEp4b, tp, p)) break;             // B^T in T1
                     tc_fence_after();
-                    mma<false, false, 64, 4>(DK, lk(bK), lk(bLam), 0u);  // dK = K Lam_s
-                    mma<false, false, 64, 4>(DK, lk(bK), lk(bLam) + kH16, 1u);
-                    mma_ts(DK, T1, lm(bQ), 1u);  //   + B^T Q
-                    mma_ts(DK, T1 + 16, lm(bQ), 1u);
+                    mma<false, false, 64, 4>(DK, lk(kb), lk(bLam), 0u);  // dK = K Lam_s
+                    mma<false, false, 64, 4>(DK, lk(kb), lk(bLam) + kH16, 1u);
+                    mma_ts(DK, T1, lm(qb), 1u);  //   + B^T Q
+                    mma_ts(DK, T1 + 16, lm(qb), 1u);
                     umma_commit(&ms->bar[bEvW]);
+                    mma<true, true, 64, 8>(LAM, lm(bYh), lm(qb), 1u);  // Lam += Y^T Q (under E5)
+                    mma<true, true, 64, 8>(LAM, lm(bYl), lm(qb), 1u);
+                    mma<true, true, 64, 8>(LAM, lm(qb), lm(bYh), 1u);  //   + Q^T Y
+                    mma<true, true, 64, 8>(LAM, lm(qb), lm(bYl), 1u);
                     if (!bar_wait(ms, bEp5, tp, p)) break;  // W^T in T0
                     tc_fence_after();
                     mma_ts(DK, T0, lm(bYh), 1u);  //   + W^T Y
                     mma_ts(DK, T0, lm(bYl), 1u);
                     mma_ts(DK, T0 + 16, lm(bYh), 1u);
                     umma_commit(&ms->bar[bEvO]);
-                    if (!bar_wait(ms, bEvO, tp, p)) break;  // every operand read
-                    if (j > 0) load_bwd(head, j - 1);
+                    if (!bar_wait(ms, bEvO, tp, p)) break;  // every operand of this set read
                     ok = true;
                 }
                 if (!ok) break;
@@ -439,6 +439,7 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
             if (ms->abort_flag) {  // copies and MMAs in flight finish (bounded) before release
                 for (int s = 0; s < 2; ++s)
                     if ((ld_pend >> s) & 1u) mbar_wait(&ms->bar[bLd0 + s], (ld_par >> s) & 1u, kBarWaitNs);
+                if ((ld_pend >> 2) & 1u) mbar_wait(&ms->bar[bLdG], (ld_par >> 2) & 1u, kBarWaitNs);
                 umma_commit(&ms->bar[bTear]);
                 mbar_wait(&ms->bar[bTear], 0, kBarWaitNs);
             }
@@ -542,6 +543,8 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                 tc_fence_after();
                 mask_pack<false, true>(t0, r, c32);
                 epi_arrive(ms, bEp1);
+                bar_wait(ms, bEvA2, tp, p);
+                tc_fence_after();
                 mask_pack<true, true>(t1, r, c32);
                 epi_arrive(ms, bEp1b);
                 // E2: X, Y -> hi, lo
