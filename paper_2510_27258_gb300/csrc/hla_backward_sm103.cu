@@ -14,11 +14,13 @@
 //             dK = K Lam_s + W^T Y + B^T Q
 // with the forward prefixes S_p = sum k k^T, D_p = sum x v^T and the suffix sums
 // Gam_s^T = sum q g^T and Lam_s = sum (y q^T + q y^T), which the reverse sweep
-// carries as Gam^T += Q^T G, Lam += Y^T Q + Q^T Y.
+// carries as Gam^T += Q^T G and Lam'' += Q^T Y with Lam_s = Lam'' + Lam''^T (K Lam_s
+// reads Lam'' once K-major and once MN-major; one N = 128 product serves both carries).
 //
 // One kernel, per head: a forward sweep over the tiles carries S and D in TMEM
-// and stores, before each tile, S_p and D_p as bf16 checkpoints (the swizzled
-// shared-memory image, by 1-D bulk copies); a reverse sweep reloads them and
+// and stores per tile a record of X (hi, lo) and the bf16 checkpoints S_p, D_p
+// (the swizzled shared-memory image of three blocks, one 1-D bulk copy); a
+// reverse sweep reloads the records, so it never forms W or X again, and
 // carries Gam^T and Lam in TMEM.  No CTA waits on another.
 //
 // Precision.  A gradient row can be a small difference of large terms (dq_0 is
@@ -36,13 +38,14 @@
 // epilogue masks it and writes it back over its own columns as packed bf16
 // hi/lo, and the next product reads it there as its A operand.  A transposed
 // use (P^T, T^T, W^T, B^T) is its own product (V G^T, X Q^T, K Q^T, K Y^T) with
-// the mask turned over.  Products on the carries read X^T, Y^T, Q^T MN-major
+// the mask turned over.  Products on the carries read K^T, X^T, Q^T MN-major
 // as the M side of an M = 128 product; rows 64..127 come from the next block
 // and land in TMEM lanes nobody reads.
 //
-// TMEM (512 columns): DQ (64) Y -> dQ; DK (64) X -> dV -> dK; GAM, LAM (64 each)
-// the carries (forward S, D; reverse Gam^T, Lam), rows 0..63; T0, T1 (128 each)
-// the masked tiles: W, T^T, B, W^T in T0 and P^T, P, B^T in T1.
+// TMEM (512 columns): DQ (64) dQ; DK (64) X (forward), Y -> dV -> dK (reverse);
+// GAM, LAM (64 each) the carries (forward S, D; reverse Gam^T, Lam''), rows
+// 0..63; T0, T1 (128 each) the masked tiles: forward W in T0; reverse P^T, T^T,
+// B^T in T0 and P, B, W^T in T1.
 //
 // Roles: warp 16 issues TMA copies and MMAs (one thread); warps 0..15 are the
 // epilogue (warp w: TMEM lanes 32 (w % 4) .. +31, one token row each; column
@@ -66,30 +69,32 @@ constexpr int kThreads = kEpiThreads + 32;
 // shared-memory blocks of 16 KiB (128 rows x 64 bf16)
 enum Block {
     bQ = 0, bK = 1, bV = 2, bG = 3,
-    bXh = 4, bXl = 5,  // X = hi + lo
-    bYh = 6, bYl = 7,  // Y = hi + lo
+    bYh = 4, bYl = 5,  // Y = hi + lo (Y_hi right after G: Q^T [G | Y_hi] is one N = 128 product)
+    bXh = 6, bXl = 7,  // X = hi + lo
     bCk = 8,           // S_p (rows 0..63 of the first 8 KiB), D_p (the second 8 KiB): the checkpoint image
     bGam = 9,          // Gam_s^T: hi (first 8 KiB), lo (second 8 KiB)
-    bLam = 10,         // Lam_s: hi, lo
+    bLam = 10,         // Lam''_s (Lam_s = Lam'' + Lam''^T): hi, lo
     bQ2 = 11,          // the second Q, K, V set at 11, 12, 13 (tiles alternate between the sets)
     kBlocks = 14
 };
+static_assert(bXl == bXh + 1 && bCk == bXh + 2, "a tile's record is three consecutive blocks");
 constexpr uint32_t kHalf = kBlockBytes / 2;
 constexpr uint32_t kSmemBlocks = kBlocks * kBlockBytes;
-constexpr uint32_t kCkBytes = kBlockBytes;  // one checkpoint: S_p and D_p images
+// one record per tile, the image of blocks bXh, bXl, bCk: X (hi, lo), then S_p and D_p
+constexpr uint32_t kCkBytes = 3 * kBlockBytes;
 
 constexpr uint32_t kDQ = 0, kDK = 64, kGAM = 128, kLAM = 192, kT0 = 256, kT1 = 384;  // TMEM columns
 
 enum Bar {
     bLd0 = 0, bLd1 = 1,  // tile copies: the two Q, K, V sets
-    bLdG = 2,            // reverse sweep: G and the checkpoint
-    // MMA commits
-    bEvA = 3, bEvA2 = 4, bEvX = 5, bEvC = 6, bEvT = 7, bEvV = 8, bEvB = 9, bEvW = 10, bEvO = 11,
+    bLdG = 2,            // reverse sweep: G and the tile's record
+    // MMA commits (forward: A, X, the carries; reverse: P^T, P, Y, T^T, B, dV, B^T, W^T, all)
+    bEvA = 3, bEvA2 = 4, bEvX = 5, bEvC = 6, bEvT = 7, bEvB = 8, bEvV = 9, bEvB2 = 10, bEvW = 11, bEvO = 12,
     // epilogue hand-offs (16 warp arrivals each)
-    bEp0 = 12, bEp1 = 13, bEp2 = 14,                 // both sweeps
-    bEp1b = 15, bEp3a = 16, bEp3b = 17, bEp4a = 18, bEp4b = 19, bEp5 = 20,  // reverse sweep
+    bEp0 = 13, bEp1 = 14, bEp2 = 15,                             // both sweeps
+    bEp1b = 16, bEp3 = 17, bEp4a = 18, bEp4b = 19, bEp5 = 20,  // reverse sweep
     bTear = 21,
-    bCkDone = 22,  // a head's checkpoints are in global memory
+    bCkDone = 22,  // a head's records are in global memory
     kNumBars = 23
 };
 __host__ __device__ constexpr bool epi_bar(int b) { return b >= bEp0 && b <= bEp5; }
@@ -304,13 +309,13 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                 tma_load_3d(blk(b0 + 1), &tm_k, &ms->bar[bLd0 + set], 0, j * kTile, head);
                 tma_load_3d(blk(b0 + 2), &tm_v, &ms->bar[bLd0 + set], 0, j * kTile, head);
             };
-            auto load_gck = [&](int head, int j) {  // G of tile j and its checkpoint
+            auto load_gck = [&](int head, int j) {  // G of tile j and its record (X hi, lo; S_p, D_p)
                 ld_pend |= 4u;
                 mbar_arrive_expect_tx(&ms->bar[bLdG], kBlockBytes + kCkBytes);
                 tma_load_3d(blk(bG), &tm_g, &ms->bar[bLdG], 0, j * kTile, head);
-                bulk_load(blk(bCk), p.ck + ((size_t)head * M + j) * kCkBytes, kCkBytes, &ms->bar[bLdG]);
+                bulk_load(blk(bXh), p.ck + ((size_t)head * M + j) * kCkBytes, kCkBytes, &ms->bar[bLdG]);
             };
-            auto wait_ld = [&](int set) {  // set 0, 1: a Q, K, V set; 2: G and the checkpoint
+            auto wait_ld = [&](int set) {  // set 0, 1: a Q, K, V set; 2: G and the record
                 if (!bar_wait(ms, bLd0 + set, (ld_par >> set) & 1u, p)) return false;
                 ld_par ^= 1u << set;
                 ld_pend &= ~(1u << set);
@@ -359,77 +364,73 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                         load_fwd(set ^ 1, head, j - 1);
                         const size_t t0 = (size_t)head * p.n + (size_t)(j - 1) * kTile;
                         const uint32_t bytes = (uint32_t)min(kTile, p.n - (j - 1) * kTile) * kD * 2;
-                        bulk_prefetch_l2(tok.g + t0 * kD, bytes);  // G and the checkpoint towards L2
+                        bulk_prefetch_l2(tok.g + t0 * kD, bytes);  // G and the record towards L2
                         bulk_prefetch_l2(p.ck + ((size_t)head * M + j - 1) * kCkBytes, kCkBytes);
                     }
-                    if (!bar_wait(ms, bEp0, ts, p) || !wait_ld(set)) break;  // Gam_s, Lam_s (hi, lo); Q, K, V
+                    // Gam_s, Lam_s (hi, lo); Q, K, V; G and the record
+                    if (!bar_wait(ms, bEp0, ts, p) || !wait_ld(set) || !wait_ld(2)) break;
                     tc_fence_after();
-                    mma<false, false, 128, 4>(T0, lk(qb), lk(kb), 0u);  // A = Q K^T
+                    mma<false, false, 128, 4>(T0, lk(vb), lk(bG), 0u);  // P^T = V G^T
                     umma_commit(&ms->bar[bEvA]);
-                    if (!wait_ld(2)) break;  // G, checkpoint
-                    mma<false, false, 128, 4>(T1, lk(vb), lk(bG), 0u);  // P^T = V G^T
+                    mma<false, false, 128, 4>(T1, lk(bG), lk(vb), 0u);  // P = G V^T
                     umma_commit(&ms->bar[bEvA2]);
-                    mma<true, true, 64, 8>(GAM, lm(qb), lm(bG), 1u);  // Gam^T += Q^T G
-                    if (!bar_wait(ms, bEp1, ts, p)) break;           // W in T0
+                    if (!bar_wait(ms, bEp1, ts, p)) break;  // P^T in T0
                     tc_fence_after();
-                    mma_ts(DK, T0, lm(kb), 0u);  // X = W K
-                    mma_ts(DK, T0 + 16, lm(kb), 1u);
-                    mma<false, false, 64, 4>(DK, lk(qb), lk(bCk), 1u);  //   + Q S_p
-                    if (!bar_wait(ms, bEp1b, tp, p)) break;             // P^T in T1
-                    tc_fence_after();
-                    mma_ts(DQ, T1, lm(qb), 0u);  // Y = P^T Q
-                    mma_ts(DQ, T1 + 16, lm(qb), 1u);
-                    mma<false, false, 64, 4>(DQ, lk(vb), lk(bGam), 1u);  //   + V Gam_s
-                    mma<false, false, 64, 4>(DQ, lk(vb), lk(bGam) + kH16, 1u);
+                    mma_ts(DK, T0, lm(qb), 0u);  // Y = P^T Q
+                    mma_ts(DK, T0 + 16, lm(qb), 1u);
+                    mma<false, false, 64, 4>(DK, lk(vb), lk(bGam), 1u);  //   + V Gam_s
+                    mma<false, false, 64, 4>(DK, lk(vb), lk(bGam) + kH16, 1u);
                     umma_commit(&ms->bar[bEvX]);
-                    if (!bar_wait(ms, bEp2, ts, p)) break;  // X, Y (hi, lo) in shared memory; DK, DQ read
-                    tc_fence_after();
                     mma<false, false, 128, 4>(T0, lk(bXh), lk(qb), 0u);  // T^T = X Q^T
                     mma<false, false, 128, 4>(T0, lk(bXl), lk(qb), 1u);
-                    mma<false, false, 128, 4>(T1, lk(bG), lk(vb), 0u);   // P = G V^T
                     umma_commit(&ms->bar[bEvT]);
-                    if (!bar_wait(ms, bEp3a, tp, p)) break;  // T^T in T0
+                    if (!bar_wait(ms, bEp1b, tp, p)) break;  // P in T1
+                    tc_fence_after();
+                    mma_ts(DQ, T1, lm(bXh), 0u);  // dQ = P X
+                    mma_ts(DQ, T1, lm(bXl), 1u);
+                    mma_ts(DQ, T1 + 16, lm(bXh), 1u);
+                    mma<false, false, 64, 4>(DQ, lk(bG), lk(bCk) + kH16, 1u);  //   + G D_p^T
+                    if (!bar_wait(ms, bEp2, ts, p)) break;  // Y (hi, lo) in shared memory; DK read
+                    tc_fence_after();
+                    mma<false, false, 64, 4>(DQ, lk(bYh), lk(bCk), 1u);  //   + Y S_p
+                    mma<false, false, 64, 4>(DQ, lk(bYl), lk(bCk), 1u);
+                    mma<false, false, 128, 4>(T1, lk(bYh), lk(kb), 0u);  // B = Y K^T
+                    mma<false, false, 128, 4>(T1, lk(bYl), lk(kb), 1u);
+                    umma_commit(&ms->bar[bEvB]);
+                    // the carries, under the B epilogue: [Gam^T | Lam''] += Q^T [G | Y_hi], Lam'' += Q^T Y_lo
+                    mma<true, true, 128, 8>(GAM, lm(qb), lm(bG), 1u);
+                    mma<true, true, 64, 8>(LAM, lm(qb), lm(bYl), 1u);
+                    if (!bar_wait(ms, bEp3, tp, p)) break;  // T^T in T0
                     tc_fence_after();
                     mma_ts(DK, T0, lm(bG), 0u);                                 // dV = T^T G
                     mma<false, true, 64, 4>(DK, lk(bXh), lm(bGam), 1u);         //   + X Gam_s^T
                     mma<false, true, 64, 4>(DK, lk(bXh), lm(bGam) + kH16, 1u);
                     mma<false, true, 64, 4>(DK, lk(bXl), lm(bGam), 1u);
                     umma_commit(&ms->bar[bEvV]);
-                    mma<false, false, 128, 4>(T0, lk(bYh), lk(kb), 0u);  // B = Y K^T
-                    mma<false, false, 128, 4>(T0, lk(bYl), lk(kb), 1u);
-                    if (!bar_wait(ms, bEp3b, tp, p)) break;  // P in T1
+                    mma<false, false, 128, 4>(T0, lk(kb), lk(bYh), 0u);  // B^T = K Y^T
+                    mma<false, false, 128, 4>(T0, lk(kb), lk(bYl), 1u);
+                    umma_commit(&ms->bar[bEvB2]);
+                    if (!bar_wait(ms, bEp4a, tp, p)) break;  // B in T1
                     tc_fence_after();
-                    mma_ts(DQ, T1, lm(bXh), 0u);  // dQ = P X
-                    mma_ts(DQ, T1, lm(bXl), 1u);
-                    mma_ts(DQ, T1 + 16, lm(bXh), 1u);
-                    mma<false, false, 64, 4>(DQ, lk(bG), lk(bCk) + kH16, 1u);  //   + G D_p^T
-                    mma<false, false, 64, 4>(DQ, lk(bYh), lk(bCk), 1u);        //   + Y S_p
-                    mma<false, false, 64, 4>(DQ, lk(bYl), lk(bCk), 1u);
-                    mma<false, false, 128, 4>(T1, lk(kb), lk(bYh), 0u);  // B^T = K Y^T
-                    mma<false, false, 128, 4>(T1, lk(kb), lk(bYl), 1u);
-                    umma_commit(&ms->bar[bEvB]);
-                    if (!bar_wait(ms, bEp4a, tp, p)) break;  // B in T0; dV out of DK; G, checkpoint read
+                    mma_ts(DQ, T1, lm(kb), 1u);  // dQ += B K
+                    mma_ts(DQ, T1 + 16, lm(kb), 1u);
+                    mma<false, false, 128, 4>(T1, lk(kb), lk(qb), 0u);  // W^T = K Q^T
+                    umma_commit(&ms->bar[bEvW]);
+                    // B^T in T0; dV out of DK; every product that reads G or the record is done
+                    if (!bar_wait(ms, bEp4b, tp, p)) break;
                     tc_fence_after();
                     if (j > 0) load_gck(head, j - 1);
-                    mma_ts(DQ, T0, lm(kb), 1u);  // dQ += B K
-                    mma_ts(DQ, T0 + 16, lm(kb), 1u);
-                    mma<false, false, 128, 4>(T0, lk(kb), lk(qb), 0u);  // W^T = K Q^T
-                    if (!bar_wait(ms, bEp4b, tp, p)) break;             // B^T in T1
-                    tc_fence_after();
-                    mma<false, false, 64, 4>(DK, lk(kb), lk(bLam), 0u);  // dK = K Lam_s
+                    mma<false, false, 64, 4>(DK, lk(kb), lk(bLam), 0u);  // dK = K Lam''^T
                     mma<false, false, 64, 4>(DK, lk(kb), lk(bLam) + kH16, 1u);
-                    mma_ts(DK, T1, lm(qb), 1u);  //   + B^T Q
-                    mma_ts(DK, T1 + 16, lm(qb), 1u);
-                    umma_commit(&ms->bar[bEvW]);
-                    mma<true, true, 64, 8>(LAM, lm(bYh), lm(qb), 1u);  // Lam += Y^T Q (under E5)
-                    mma<true, true, 64, 8>(LAM, lm(bYl), lm(qb), 1u);
-                    mma<true, true, 64, 8>(LAM, lm(qb), lm(bYh), 1u);  //   + Q^T Y
-                    mma<true, true, 64, 8>(LAM, lm(qb), lm(bYl), 1u);
-                    if (!bar_wait(ms, bEp5, tp, p)) break;  // W^T in T0
+                    mma<false, true, 64, 4>(DK, lk(kb), lm(bLam), 1u);  //   + K Lam''
+                    mma<false, true, 64, 4>(DK, lk(kb), lm(bLam) + kH16, 1u);
+                    mma_ts(DK, T0, lm(qb), 1u);  //   + B^T Q
+                    mma_ts(DK, T0 + 16, lm(qb), 1u);
+                    if (!bar_wait(ms, bEp5, tp, p)) break;  // W^T in T1
                     tc_fence_after();
-                    mma_ts(DK, T0, lm(bYh), 1u);  //   + W^T Y
-                    mma_ts(DK, T0, lm(bYl), 1u);
-                    mma_ts(DK, T0 + 16, lm(bYh), 1u);
+                    mma_ts(DK, T1, lm(bYh), 1u);  //   + W^T Y
+                    mma_ts(DK, T1, lm(bYl), 1u);
+                    mma_ts(DK, T1 + 16, lm(bYh), 1u);
                     umma_commit(&ms->bar[bEvO]);
                     if (!bar_wait(ms, bEvO, tp, p)) break;  // every operand of this set read
                     ok = true;
@@ -480,11 +481,11 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
             zero_carries();
             for (int j = 0; j < M; ++j, ++n_f, ++n_s) {
                 const uint32_t tp = n_s & 1, tf = n_f & 1;
-                // E0: S_p, D_p -> bf16 checkpoint image (also the B operand of Q S_p) -> global
+                // E0: S_p, D_p -> bf16 checkpoint image in bCk (also the B operand of Q S_p)
                 if (j > 0) {
                     bar_wait(ms, bEvC, tf ^ 1u, p);  // the previous tile's carry products
                     tc_fence_after();
-                    if (tid == 0) tma_store_wait_read();  // its checkpoint copy has left bCk
+                    if (tid == 0) tma_store_wait_read();  // its record has left bXh, bXl, bCk
                     epi_sync();
                 }
                 if (qd < 2) {
@@ -496,28 +497,28 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                     store16(blk(bCk) + kHalf, r, c16, b);
                 }
                 fence_async_smem();
-                epi_sync();
-                if (tid == 0) {
-                    bulk_store(p.ck + ((size_t)head * M + j) * kCkBytes, blk(bCk), kCkBytes);
-                    tma_store_commit();
-                }
                 epi_arrive(ms, bEp0);
                 // E1: W = L . A, packed hi/lo over A
                 bar_wait(ms, bEvA, tp, p);
                 tc_fence_after();
                 mask_pack<false, true>(t0, r, c32);
                 epi_arrive(ms, bEp1);
-                // E2: X -> hi, lo
+                // E2: X -> hi, lo; the tile's record (X hi, lo; S_p, D_p) -> global
                 bar_wait(ms, bEvX, tp, p);
                 tc_fence_after();
                 to_smem_hl(kDK, bXh, bXl);
                 fence_async_smem();
+                epi_sync();
+                if (tid == 0) {
+                    bulk_store(p.ck + ((size_t)head * M + j) * kCkBytes, blk(bXh), kCkBytes);
+                    tma_store_commit();
+                }
                 epi_arrive(ms, bEp2);
             }
             bar_wait(ms, bEvC, (n_f - 1) & 1u, p);  // the last carry products (before GAM, LAM are reset)
             tc_fence_after();
             if (tid == 0) {
-                tma_store_wait_all();  // every checkpoint is in global memory
+                tma_store_wait_all();  // every record is in global memory
                 mbar_arrive(&ms->bar[bCkDone]);
             }
             // ---------------- reverse sweep ----------------
@@ -527,7 +528,7 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                 const int tok0 = j * kTile;
                 const bool row_ok = tok0 + r < p.n;
                 const size_t orow = ((size_t)head * p.n + tok0 + r) * kD + c16;
-                // E0: Gam_s^T, Lam_s -> hi, lo (the previous tile's products are done: waited in E6)
+                // E0: Gam_s^T, Lam''_s -> hi, lo (the previous tile's products are done: waited in E6)
                 if (qd < 2) {
                     uint32_t a[16], b[16];
                     tmem_ld16(tb + lb + kGAM + c16, a);
@@ -538,43 +539,42 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                 }
                 fence_async_smem();
                 epi_arrive(ms, bEp0);
-                // E1: W = L . A over T0 (X = W K starts on it), then P^T = L^T . (V G^T) over T1
+                // E1: P^T = L^T . (V G^T) over T0, P = L . (G V^T) over T1
                 bar_wait(ms, bEvA, ts, p);
                 tc_fence_after();
-                mask_pack<false, true>(t0, r, c32);
+                mask_pack<true, true>(t0, r, c32);
                 epi_arrive(ms, bEp1);
                 bar_wait(ms, bEvA2, tp, p);
                 tc_fence_after();
-                mask_pack<true, true>(t1, r, c32);
+                mask_pack<false, true>(t1, r, c32);
                 epi_arrive(ms, bEp1b);
-                // E2: X, Y -> hi, lo
+                // E2: Y -> hi, lo
                 bar_wait(ms, bEvX, ts, p);
                 tc_fence_after();
-                to_smem_hl(kDK, bXh, bXl);
-                to_smem_hl(kDQ, bYh, bYl);
+                to_smem_hl(kDK, bYh, bYl);
                 fence_async_smem();
                 epi_arrive(ms, bEp2);
-                // E3: T^T = L^T . (X Q^T) over T0 (bf16 only), P = L . (G V^T) over T1
+                // E3: T^T = L^T . (X Q^T) over T0 (bf16 only)
                 bar_wait(ms, bEvT, tp, p);
                 tc_fence_after();
                 mask_pack<true, false>(t0, r, c32);
-                epi_arrive(ms, bEp3a);
+                epi_arrive(ms, bEp3);
+                // E4: B = L . (Y K^T) over T1; dV out; B^T over T0
+                bar_wait(ms, bEvB, tp, p);
+                tc_fence_after();
                 mask_pack<false, true>(t1, r, c32);
-                epi_arrive(ms, bEp3b);
-                // E4: dV out, then B = L . (Y K^T) over T0 and B^T over T1
+                epi_arrive(ms, bEp4a);
                 bar_wait(ms, bEvV, tp, p);
                 tc_fence_after();
                 drain(kDK, p.dv + orow, row_ok);
-                bar_wait(ms, bEvB, tp, p);
-                tc_fence_after();
-                mask_pack<false, true>(t0, r, c32);
-                epi_arrive(ms, bEp4a);
-                mask_pack<true, true>(t1, r, c32);
-                epi_arrive(ms, bEp4b);
-                // E5: W^T = L^T . (K Q^T) over T0, then dQ out
-                bar_wait(ms, bEvW, tp, p);
+                bar_wait(ms, bEvB2, tp, p);
                 tc_fence_after();
                 mask_pack<true, true>(t0, r, c32);
+                epi_arrive(ms, bEp4b);
+                // E5: W^T = L^T . (K Q^T) over T1, then dQ out
+                bar_wait(ms, bEvW, tp, p);
+                tc_fence_after();
+                mask_pack<true, true>(t1, r, c32);
                 epi_arrive(ms, bEp5);
                 drain(kDQ, p.dq + orow, row_ok);
                 // E6: dK out
