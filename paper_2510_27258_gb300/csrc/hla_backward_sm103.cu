@@ -47,7 +47,10 @@
 // 0..63; T0, T1 (128 each) the masked tiles: forward W in T0; reverse P^T, T^T,
 // B^T in T0 and P, B, W^T in T1.
 //
-// Roles: warp 16 issues TMA copies and MMAs (one thread); warps 0..15 are the
+// Roles: warp 16 issues TMA copies and MMAs (one thread); in the reverse sweep
+// warp 17 issues the second half of the MMAs (P, B, W^T in T1, dQ, the carries),
+// since one thread issues a 128 x 64 x 16 MMA with A in TMEM no faster than
+// about one per 55 cycles and two threads overlap them; warps 0..15 are the
 // epilogue (warp w: TMEM lanes 32 (w % 4) .. +31, one token row each; column
 // quarter w / 4).
 //
@@ -63,8 +66,8 @@ namespace {
 using namespace sm103;
 
 constexpr int kTile = 128, kD = 64;
-constexpr int kEpiWarps = 16, kEpiThreads = kEpiWarps * 32, kIssuerWarp = kEpiWarps;
-constexpr int kThreads = kEpiThreads + 32;
+constexpr int kEpiWarps = 16, kEpiThreads = kEpiWarps * 32, kIssuerWarp = kEpiWarps, kIssuer2Warp = kEpiWarps + 1;
+constexpr int kThreads = kEpiThreads + 64;
 
 // shared-memory blocks of 16 KiB (128 rows x 64 bf16)
 enum Block {
@@ -95,7 +98,9 @@ enum Bar {
     bEp1b = 16, bEp3 = 17, bEp4a = 18, bEp4b = 19, bEp5 = 20,  // reverse sweep
     bTear = 21,
     bCkDone = 22,  // a head's records are in global memory
-    kNumBars = 23
+    bEvCar = 23,   // reverse sweep, second issuer: the carries (its last reads of G, X and the checkpoint)
+    bTear2 = 24,
+    kNumBars = 25
 };
 __host__ __device__ constexpr bool epi_bar(int b) { return b >= bEp0 && b <= bEp5; }
 
@@ -109,7 +114,6 @@ static_assert(sizeof(Misc) <= kMiscBytes, "misc smem");
 constexpr uint32_t kSmemBytes = kSmemBlocks + kMiscBytes;
 
 struct Params {
-    __nv_bfloat16 *dq, *dk, *dv;
     uint8_t *ck;  // [BH][M] checkpoints of kCkBytes
     int BH, n, M;
     WsHeader *err;
@@ -127,6 +131,33 @@ __device__ __forceinline__ void set_error(WsHeader *err, unsigned where, unsigne
 __device__ __forceinline__ bool bar_wait(Misc *ms, int b, uint32_t parity, const Params &p) {
     if (ms->abort_flag) return false;
     if (mbar_wait(&ms->bar[b], parity, kBarWaitNs)) return true;
+    set_error(p.err, 500 + b, parity);
+    ms->abort_flag = 1;
+    return false;
+}
+
+// The issuers' wait: a non-suspending poll (a suspended try_wait was seen to resume up to
+// ~900 cycles after the phase completed), bounded like mbar_wait.
+__device__ __forceinline__ bool mbar_test(uint64_t *bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+__device__ __forceinline__ bool bar_poll(Misc *ms, int b, uint32_t parity, const Params &p) {
+    if (ms->abort_flag) return false;
+    if (mbar_test(&ms->bar[b], parity)) return true;
+    const uint64_t t0 = globaltimer_ns();
+    while (true) {
+        for (int i = 0; i < 32; ++i)
+            if (mbar_test(&ms->bar[b], parity)) return true;
+        if (globaltimer_ns() - t0 > kBarWaitNs) break;
+    }
     set_error(p.err, 500 + b, parity);
     ms->abort_flag = 1;
     return false;
@@ -246,28 +277,20 @@ __device__ __forceinline__ void store16(uint8_t *blk, int r, int c0, const uint3
     st16(blk, r, c0 + 8, pack8(x + 8));
 }
 
-// 16 fp32 TMEM values as bf16 into row `tok` of a [n][64] global array
-__device__ __forceinline__ void out16(__nv_bfloat16 *dst, const uint32_t (&a)[16]) {
-    float x[16];
-#pragma unroll
-    for (int u = 0; u < 16; ++u) x[u] = __uint_as_float(a[u]);
-    uint4 *d4 = reinterpret_cast<uint4 *>(dst);
-    d4[0] = pack8(x);
-    d4[1] = pack8(x + 8);
-}
-
 struct Tok {  // raw token pointers, for the L2 prefetch of the next reverse tile
     const __nv_bfloat16 *q, *k, *v, *g;
 };
 
 __global__ void __launch_bounds__(kThreads, 1)
 bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
-              const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_g, Params p, Tok tok) {
+              const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_g,
+              const __grid_constant__ CUtensorMap tm_dq, const __grid_constant__ CUtensorMap tm_dk,
+              const __grid_constant__ CUtensorMap tm_dv, Params p, Tok tok) {
     extern __shared__ __align__(1024) uint8_t smem[];
     Misc *ms = reinterpret_cast<Misc *>(smem + kSmemBlocks);
     auto blk = [&](int b) { return smem + b * kBlockBytes; };
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const bool issuer = warp == kIssuerWarp;
+    const bool issuer = warp == kIssuerWarp, issuer2 = warp == kIssuer2Warp;
 
     if (smem_u32(smem) & 1023u) {  // the swizzled layout needs 1 KiB alignment
         if (tid == 0) set_error(p.err, 499, smem_u32(smem));
@@ -296,7 +319,7 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
             const uint32_t sb4 = smem_u32(smem) >> 4;
             auto lk = [&](int b) { return sb4 + (uint32_t)b * kBlk16 + kLboK; };   // K-major block
             auto lm = [&](int b) { return sb4 + (uint32_t)b * kBlk16 + kLboMN; };  // MN-major block
-            const uint32_t DQ = tb + kDQ, DK = tb + kDK, GAM = tb + kGAM, LAM = tb + kLAM;
+            const uint32_t DK = tb + kDK, GAM = tb + kGAM, LAM = tb + kLAM;
             const uint32_t T0 = tb + kT0, T1 = tb + kT1;
             // tile counters: n_s every tile of both sweeps (the barriers both use), n_f forward
             // tiles, n_b reverse tiles
@@ -316,7 +339,7 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                 bulk_load(blk(bXh), p.ck + ((size_t)head * M + j) * kCkBytes, kCkBytes, &ms->bar[bLdG]);
             };
             auto wait_ld = [&](int set) {  // set 0, 1: a Q, K, V set; 2: G and the record
-                if (!bar_wait(ms, bLd0 + set, (ld_par >> set) & 1u, p)) return false;
+                if (!bar_poll(ms, bLd0 + set, (ld_par >> set) & 1u, p)) return false;
                 ld_par ^= 1u << set;
                 ld_pend &= ~(1u << set);
                 return true;
@@ -330,29 +353,29 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                     const uint32_t tp = n_s & 1, tf = n_f & 1;
                     const int set = j & 1, qb = set ? bQ2 : bQ, kb = qb + 1, vb = qb + 2;
                     ok = false;
-                    if (!bar_wait(ms, bEp0, tp, p) || !wait_ld(set)) break;  // S_p (bf16) in bCk; tokens
+                    if (!bar_poll(ms, bEp0, tp, p) || !wait_ld(set)) break;  // S_p (bf16) in bCk; tokens
                     tc_fence_after();
                     mma<false, false, 128, 4>(T0, lk(qb), lk(kb), 0u);  // A = Q K^T
                     umma_commit(&ms->bar[bEvA]);
                     mma<true, true, 64, 8>(GAM, lm(kb), lm(kb), 1u);  // S += K^T K (under E1)
-                    if (!bar_wait(ms, bEp1, tp, p)) break;           // W (hi, lo) packed in T0
+                    if (!bar_poll(ms, bEp1, tp, p)) break;           // W (hi, lo) packed in T0
                     tc_fence_after();
                     mma_ts(DK, T0, lm(kb), 0u);                       // X = W K
                     mma_ts(DK, T0 + 16, lm(kb), 1u);
                     mma<false, false, 64, 4>(DK, lk(qb), lk(bCk), 1u);  //   + Q S_p
                     umma_commit(&ms->bar[bEvX]);
-                    if (!bar_wait(ms, bEp2, tp, p)) break;  // X (hi, lo) in bXh, bXl
+                    if (!bar_poll(ms, bEp2, tp, p)) break;  // X (hi, lo) in bXh, bXl
                     tc_fence_after();
                     mma<true, true, 64, 8>(LAM, lm(bXh), lm(vb), 1u);  // D += X^T V
                     mma<true, true, 64, 8>(LAM, lm(bXl), lm(vb), 1u);
                     umma_commit(&ms->bar[bEvC]);
-                    if (!bar_wait(ms, bEvC, tf, p)) break;  // this set is free again
+                    if (!bar_poll(ms, bEvC, tf, p)) break;  // this set is free again
                     if (j + 2 < M) load_fwd(set, head, j + 2);
                     ok = true;
                 }
                 if (!ok) break;
                 // the checkpoints are in global memory (the epilogue waited for its copies)
-                if (!bar_wait(ms, bCkDone, n_head & 1, p)) break;
+                if (!bar_poll(ms, bCkDone, n_head & 1, p)) break;
                 // ---------------- reverse sweep: gradients ----------------
                 load_fwd(0, head, M - 1);
                 load_gck(head, M - 1);
@@ -368,13 +391,11 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                         bulk_prefetch_l2(p.ck + ((size_t)head * M + j - 1) * kCkBytes, kCkBytes);
                     }
                     // Gam_s, Lam_s (hi, lo); Q, K, V; G and the record
-                    if (!bar_wait(ms, bEp0, ts, p) || !wait_ld(set) || !wait_ld(2)) break;
+                    if (!bar_poll(ms, bEp0, ts, p) || !wait_ld(set) || !wait_ld(2)) break;
                     tc_fence_after();
                     mma<false, false, 128, 4>(T0, lk(vb), lk(bG), 0u);  // P^T = V G^T
                     umma_commit(&ms->bar[bEvA]);
-                    mma<false, false, 128, 4>(T1, lk(bG), lk(vb), 0u);  // P = G V^T
-                    umma_commit(&ms->bar[bEvA2]);
-                    if (!bar_wait(ms, bEp1, ts, p)) break;  // P^T in T0
+                    if (!bar_poll(ms, bEp1, ts, p)) break;  // P^T in T0
                     tc_fence_after();
                     mma_ts(DK, T0, lm(qb), 0u);  // Y = P^T Q
                     mma_ts(DK, T0 + 16, lm(qb), 1u);
@@ -384,23 +405,7 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                     mma<false, false, 128, 4>(T0, lk(bXh), lk(qb), 0u);  // T^T = X Q^T
                     mma<false, false, 128, 4>(T0, lk(bXl), lk(qb), 1u);
                     umma_commit(&ms->bar[bEvT]);
-                    if (!bar_wait(ms, bEp1b, tp, p)) break;  // P in T1
-                    tc_fence_after();
-                    mma_ts(DQ, T1, lm(bXh), 0u);  // dQ = P X
-                    mma_ts(DQ, T1, lm(bXl), 1u);
-                    mma_ts(DQ, T1 + 16, lm(bXh), 1u);
-                    mma<false, false, 64, 4>(DQ, lk(bG), lk(bCk) + kH16, 1u);  //   + G D_p^T
-                    if (!bar_wait(ms, bEp2, ts, p)) break;  // Y (hi, lo) in shared memory; DK read
-                    tc_fence_after();
-                    mma<false, false, 64, 4>(DQ, lk(bYh), lk(bCk), 1u);  //   + Y S_p
-                    mma<false, false, 64, 4>(DQ, lk(bYl), lk(bCk), 1u);
-                    mma<false, false, 128, 4>(T1, lk(bYh), lk(kb), 0u);  // B = Y K^T
-                    mma<false, false, 128, 4>(T1, lk(bYl), lk(kb), 1u);
-                    umma_commit(&ms->bar[bEvB]);
-                    // the carries, under the B epilogue: [Gam^T | Lam''] += Q^T [G | Y_hi], Lam'' += Q^T Y_lo
-                    mma<true, true, 128, 8>(GAM, lm(qb), lm(bG), 1u);
-                    mma<true, true, 64, 8>(LAM, lm(qb), lm(bYl), 1u);
-                    if (!bar_wait(ms, bEp3, tp, p)) break;  // T^T in T0
+                    if (!bar_poll(ms, bEp3, tp, p)) break;  // T^T in T0
                     tc_fence_after();
                     mma_ts(DK, T0, lm(bG), 0u);                                 // dV = T^T G
                     mma<false, true, 64, 4>(DK, lk(bXh), lm(bGam), 1u);         //   + X Gam_s^T
@@ -410,14 +415,8 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                     mma<false, false, 128, 4>(T0, lk(kb), lk(bYh), 0u);  // B^T = K Y^T
                     mma<false, false, 128, 4>(T0, lk(kb), lk(bYl), 1u);
                     umma_commit(&ms->bar[bEvB2]);
-                    if (!bar_wait(ms, bEp4a, tp, p)) break;  // B in T1
-                    tc_fence_after();
-                    mma_ts(DQ, T1, lm(kb), 1u);  // dQ += B K
-                    mma_ts(DQ, T1 + 16, lm(kb), 1u);
-                    mma<false, false, 128, 4>(T1, lk(kb), lk(qb), 0u);  // W^T = K Q^T
-                    umma_commit(&ms->bar[bEvW]);
-                    // B^T in T0; dV out of DK; every product that reads G or the record is done
-                    if (!bar_wait(ms, bEp4b, tp, p)) break;
+                    // B^T in T0 and dV out of DK; the second issuer's reads of G and the record done
+                    if (!bar_poll(ms, bEp4b, tp, p) || !bar_poll(ms, bEvCar, tp, p)) break;
                     tc_fence_after();
                     if (j > 0) load_gck(head, j - 1);
                     mma<false, false, 64, 4>(DK, lk(kb), lk(bLam), 0u);  // dK = K Lam''^T
@@ -426,13 +425,13 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                     mma<false, true, 64, 4>(DK, lk(kb), lm(bLam) + kH16, 1u);
                     mma_ts(DK, T0, lm(qb), 1u);  //   + B^T Q
                     mma_ts(DK, T0 + 16, lm(qb), 1u);
-                    if (!bar_wait(ms, bEp5, tp, p)) break;  // W^T in T1
+                    if (!bar_poll(ms, bEp5, tp, p)) break;  // W^T in T1
                     tc_fence_after();
                     mma_ts(DK, T1, lm(bYh), 1u);  //   + W^T Y
                     mma_ts(DK, T1, lm(bYl), 1u);
                     mma_ts(DK, T1 + 16, lm(bYh), 1u);
                     umma_commit(&ms->bar[bEvO]);
-                    if (!bar_wait(ms, bEvO, tp, p)) break;  // every operand of this set read
+                    if (!bar_poll(ms, bEvO, tp, p)) break;  // every operand of this set read
                     ok = true;
                 }
                 if (!ok) break;
@@ -443,6 +442,67 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                 if ((ld_pend >> 2) & 1u) mbar_wait(&ms->bar[bLdG], (ld_par >> 2) & 1u, kBarWaitNs);
                 umma_commit(&ms->bar[bTear]);
                 mbar_wait(&ms->bar[bTear], 0, kBarWaitNs);
+            }
+        }
+        __syncwarp();
+    } else if (issuer2) {
+        // ====== second issuer: the reverse sweep's P, B, W^T tiles (T1), dQ (DQ) and the carries ======
+        if (lane == 0) {
+            const uint32_t sb4 = smem_u32(smem) >> 4;
+            auto lk = [&](int b) { return sb4 + (uint32_t)b * kBlk16 + kLboK; };
+            auto lm = [&](int b) { return sb4 + (uint32_t)b * kBlk16 + kLboMN; };
+            const uint32_t DQ = tb + kDQ, GAM = tb + kGAM, LAM = tb + kLAM, T1 = tb + kT1;
+            // the same tile counters as the first issuer; ld_par follows every completed copy phase,
+            // the forward sweep's included (set j % 2 for forward tile j)
+            uint32_t ld_par = 0, n_s = 0, n_b = 0, n_head = 0;
+            auto wait_ld = [&](int set) {
+                if (!bar_poll(ms, bLd0 + set, (ld_par >> set) & 1u, p)) return false;
+                ld_par ^= 1u << set;
+                return true;
+            };
+            for (int head = blockIdx.x; head < p.BH && !ms->abort_flag; head += gridDim.x, ++n_head) {
+                n_s += (uint32_t)M;
+                ld_par ^= (uint32_t)(((M + 1) / 2) & 1) | ((uint32_t)((M / 2) & 1) << 1);
+                if (!bar_poll(ms, bCkDone, n_head & 1, p)) break;
+                bool ok = true;
+                for (int j = M - 1; j >= 0 && ok; --j, ++n_b, ++n_s) {
+                    const uint32_t ts = n_s & 1, tp = n_b & 1;
+                    const int set = (M - 1 - j) & 1, qb = set ? bQ2 : bQ, kb = qb + 1, vb = qb + 2;
+                    ok = false;
+                    if (!bar_poll(ms, bEp0, ts, p) || !wait_ld(set) || !wait_ld(2)) break;
+                    tc_fence_after();
+                    mma<false, false, 128, 4>(T1, lk(bG), lk(vb), 0u);  // P = G V^T
+                    umma_commit(&ms->bar[bEvA2]);
+                    if (!bar_poll(ms, bEp1b, tp, p)) break;  // P in T1
+                    tc_fence_after();
+                    mma_ts(DQ, T1, lm(bXh), 0u);  // dQ = P X
+                    mma_ts(DQ, T1, lm(bXl), 1u);
+                    mma_ts(DQ, T1 + 16, lm(bXh), 1u);
+                    mma<false, false, 64, 4>(DQ, lk(bG), lk(bCk) + kH16, 1u);  //   + G D_p^T
+                    if (!bar_poll(ms, bEp2, ts, p)) break;  // Y (hi, lo) in shared memory
+                    tc_fence_after();
+                    mma<false, false, 64, 4>(DQ, lk(bYh), lk(bCk), 1u);  //   + Y S_p
+                    mma<false, false, 64, 4>(DQ, lk(bYl), lk(bCk), 1u);
+                    mma<false, false, 128, 4>(T1, lk(bYh), lk(kb), 0u);  // B = Y K^T
+                    mma<false, false, 128, 4>(T1, lk(bYl), lk(kb), 1u);
+                    umma_commit(&ms->bar[bEvB]);
+                    // the carries, under the B epilogue: [Gam^T | Lam''] += Q^T [G | Y_hi], Lam'' += Q^T Y_lo
+                    mma<true, true, 128, 8>(GAM, lm(qb), lm(bG), 1u);
+                    mma<true, true, 64, 8>(LAM, lm(qb), lm(bYl), 1u);
+                    umma_commit(&ms->bar[bEvCar]);
+                    if (!bar_poll(ms, bEp4a, tp, p)) break;  // B in T1
+                    tc_fence_after();
+                    mma_ts(DQ, T1, lm(kb), 1u);  // dQ += B K
+                    mma_ts(DQ, T1 + 16, lm(kb), 1u);
+                    mma<false, false, 128, 4>(T1, lk(kb), lk(qb), 0u);  // W^T = K Q^T
+                    umma_commit(&ms->bar[bEvW]);
+                    ok = true;
+                }
+                if (!ok) break;
+            }
+            if (ms->abort_flag) {  // this thread's MMAs in flight finish (bounded) before release
+                umma_commit(&ms->bar[bTear2]);
+                mbar_wait(&ms->bar[bTear2], 0, kBarWaitNs);
             }
         }
         __syncwarp();
@@ -470,11 +530,21 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
             tmem_ld_wait();
             store16_hl(blk(bh), blk(bl), r, c16, a);
         };
-        auto drain = [&](uint32_t col, __nv_bfloat16 *dst, bool ok) {  // a 64-wide result -> global
+        // a 64-wide result -> bf16 in a free block -> one TMA store of the tile (rows past n are
+        // not written); row-wise stores from the threads would cost a 16-byte piece per row
+        auto drain = [&](uint32_t col, int stage, const CUtensorMap *map, int tok0, int head) {
             uint32_t a[16];
             tmem_ld16(tb + lb + col + c16, a);
             tmem_ld_wait();
-            if (ok) out16(dst, a);
+            if (tid == 0) tma_store_wait_read();  // the block's previous copy has read it
+            epi_sync();
+            store16(blk(stage), r, c16, a);
+            fence_async_smem();
+            epi_sync();
+            if (tid == 0) {
+                tma_store_3d(map, blk(stage), 0, tok0, head);
+                tma_store_commit();
+            }
         };
         for (int head = blockIdx.x; head < p.BH; head += gridDim.x, ++n_head) {
             // ---------------- forward sweep ----------------
@@ -526,9 +596,10 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
             for (int j = M - 1; j >= 0; --j, ++n_b, ++n_s) {
                 const uint32_t ts = n_s & 1, tp = n_b & 1;
                 const int tok0 = j * kTile;
-                const bool row_ok = tok0 + r < p.n;
-                const size_t orow = ((size_t)head * p.n + tok0 + r) * kD + c16;
-                // E0: Gam_s^T, Lam''_s -> hi, lo (the previous tile's products are done: waited in E6)
+                // E0: Gam_s^T, Lam''_s -> hi, lo (the previous tile's products are done: waited in E6;
+                // the copies of its dV and dQ have read bGam, the one of dK may still read bYh)
+                if (tid == 0) tma_store_wait_read1();
+                epi_sync();
                 if (qd < 2) {
                     uint32_t a[16], b[16];
                     tmem_ld16(tb + lb + kGAM + c16, a);
@@ -548,9 +619,11 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                 tc_fence_after();
                 mask_pack<false, true>(t1, r, c32);
                 epi_arrive(ms, bEp1b);
-                // E2: Y -> hi, lo
+                // E2: Y -> hi, lo (the previous dK copy has read bYh)
                 bar_wait(ms, bEvX, ts, p);
                 tc_fence_after();
+                if (tid == 0) tma_store_wait_read();
+                epi_sync();
                 to_smem_hl(kDK, bYh, bYl);
                 fence_async_smem();
                 epi_arrive(ms, bEp2);
@@ -566,7 +639,7 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                 epi_arrive(ms, bEp4a);
                 bar_wait(ms, bEvV, tp, p);
                 tc_fence_after();
-                drain(kDK, p.dv + orow, row_ok);
+                drain(kDK, bGam, &tm_dv, tok0, head);  // Gam_s read by its last product (dV)
                 bar_wait(ms, bEvB2, tp, p);
                 tc_fence_after();
                 mask_pack<true, true>(t0, r, c32);
@@ -576,11 +649,11 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                 tc_fence_after();
                 mask_pack<true, true>(t1, r, c32);
                 epi_arrive(ms, bEp5);
-                drain(kDQ, p.dq + orow, row_ok);
+                drain(kDQ, bGam, &tm_dq, tok0, head);
                 // E6: dK out
                 bar_wait(ms, bEvO, tp, p);
                 tc_fence_after();
-                drain(kDK, p.dk + orow, row_ok);
+                drain(kDK, bYh, &tm_dk, tok0, head);  // Y read by its last product (W^T Y)
             }
         }
         if (tid == 0) tma_store_wait_all();
@@ -646,17 +719,15 @@ bool backward2_tc_applicable(const Bwd2 &p) {
 }
 
 cudaError_t backward2_tc_launch(const Bwd2 &p, cudaStream_t stream) {
-    CUtensorMap mq, mk, mv, mg;
+    CUtensorMap mq, mk, mv, mg, mdq, mdk, mdv;
     if (!make_map(&mq, p.q, p.BH, p.n) || !make_map(&mk, p.k, p.BH, p.n) || !make_map(&mv, p.v, p.BH, p.n) ||
-        !make_map(&mg, p.dout, p.BH, p.n))
+        !make_map(&mg, p.dout, p.BH, p.n) || !make_map(&mdq, p.dq, p.BH, p.n) || !make_map(&mdk, p.dk, p.BH, p.n) ||
+        !make_map(&mdv, p.dval, p.BH, p.n))
         return cudaErrorInvalidValue;
     int dev = 0, sms = 0;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     Params kp{};
-    kp.dq = static_cast<__nv_bfloat16 *>(p.dq);
-    kp.dk = static_cast<__nv_bfloat16 *>(p.dk);
-    kp.dv = static_cast<__nv_bfloat16 *>(p.dval);
     kp.ck = reinterpret_cast<uint8_t *>(p.ws + kWsHeaderBytes);
     kp.BH = p.BH;
     kp.n = p.n;
@@ -669,7 +740,7 @@ cudaError_t backward2_tc_launch(const Bwd2 &p, cudaStream_t stream) {
     if ((e = cudaFuncSetAttribute(bwd_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes)))
         return e;
     const int grid = p.BH < sms ? p.BH : sms;
-    bwd_tc_kernel<<<grid, kThreads, kSmemBytes, stream>>>(mq, mk, mv, mg, kp, tok);
+    bwd_tc_kernel<<<grid, kThreads, kSmemBytes, stream>>>(mq, mk, mv, mg, mdq, mdk, mdv, kp, tok);
     return cudaGetLastError();
 }
 
