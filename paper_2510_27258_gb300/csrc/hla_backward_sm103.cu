@@ -390,12 +390,14 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                         bulk_prefetch_l2(tok.g + t0 * kD, bytes);  // G and the record towards L2
                         bulk_prefetch_l2(p.ck + ((size_t)head * M + j - 1) * kCkBytes, kCkBytes);
                     }
-                    // Gam_s, Lam_s (hi, lo); Q, K, V; G and the record
-                    if (!bar_poll(ms, bEp0, ts, p) || !wait_ld(set) || !wait_ld(2)) break;
+                    // Q, K, V; G and the record.  P^T starts at once (T0 was last read by this
+                    // thread's B^T Q); the epilogue packs it after the carry hand-off E0, so the
+                    // arrival of E1 also says Gam_s, Lam_s (hi, lo) are in shared memory.
+                    if (!wait_ld(set) || !wait_ld(2)) break;
                     tc_fence_after();
                     mma<false, false, 128, 4>(T0, lk(vb), lk(bG), 0u);  // P^T = V G^T
                     umma_commit(&ms->bar[bEvA]);
-                    if (!bar_poll(ms, bEp1, ts, p)) break;  // P^T in T0
+                    if (!bar_poll(ms, bEp1, ts, p)) break;  // P^T in T0; E0 done
                     tc_fence_after();
                     mma_ts(DK, T0, lm(qb), 0u);  // Y = P^T Q
                     mma_ts(DK, T0 + 16, lm(qb), 1u);
@@ -415,16 +417,18 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                     mma<false, false, 128, 4>(T0, lk(kb), lk(bYh), 0u);  // B^T = K Y^T
                     mma<false, false, 128, 4>(T0, lk(kb), lk(bYl), 1u);
                     umma_commit(&ms->bar[bEvB2]);
-                    // B^T in T0 and dV out of DK; the second issuer's reads of G and the record done
-                    if (!bar_poll(ms, bEp4b, tp, p) || !bar_poll(ms, bEvCar, tp, p)) break;
+                    if (!bar_poll(ms, bEp4b, tp, p)) break;  // B^T in T0 and dV out of DK
                     tc_fence_after();
-                    if (j > 0) load_gck(head, j - 1);
                     mma<false, false, 64, 4>(DK, lk(kb), lk(bLam), 0u);  // dK = K Lam''^T
                     mma<false, false, 64, 4>(DK, lk(kb), lk(bLam) + kH16, 1u);
                     mma<false, true, 64, 4>(DK, lk(kb), lm(bLam), 1u);  //   + K Lam''
                     mma<false, true, 64, 4>(DK, lk(kb), lm(bLam) + kH16, 1u);
                     mma_ts(DK, T0, lm(qb), 1u);  //   + B^T Q
                     mma_ts(DK, T0 + 16, lm(qb), 1u);
+                    // every product that reads G or the record is done (this thread's by the B^T
+                    // hand-off, the second issuer's by its carry commit)
+                    if (!bar_poll(ms, bEvCar, tp, p)) break;
+                    if (j > 0) load_gck(head, j - 1);
                     if (!bar_poll(ms, bEp5, tp, p)) break;  // W^T in T1
                     tc_fence_after();
                     mma_ts(DK, T1, lm(bYh), 1u);  //   + W^T Y
@@ -469,7 +473,9 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                     const uint32_t ts = n_s & 1, tp = n_b & 1;
                     const int set = (M - 1 - j) & 1, qb = set ? bQ2 : bQ, kb = qb + 1, vb = qb + 2;
                     ok = false;
-                    if (!bar_poll(ms, bEp0, ts, p) || !wait_ld(set) || !wait_ld(2)) break;
+                    // T1 free (the previous tile's W^T Y has read it); Q, K, V; G and the record
+                    if (j < M - 1 && !bar_poll(ms, bEvO, tp ^ 1u, p)) break;
+                    if (!wait_ld(set) || !wait_ld(2)) break;
                     tc_fence_after();
                     mma<false, false, 128, 4>(T1, lk(bG), lk(vb), 0u);  // P = G V^T
                     umma_commit(&ms->bar[bEvA2]);
