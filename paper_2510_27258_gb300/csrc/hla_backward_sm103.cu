@@ -241,15 +241,29 @@ __device__ __forceinline__ void split2(float x0, float x1, uint32_t &h, uint32_t
 // as packed bf16, hi at c0 and (kLo) lo at c0 + 16.
 template <bool kUpper, bool kLo>
 __device__ __forceinline__ void mask_pack(uint32_t t, int r, int c0) {
-    uint32_t a[32];
-    tmem_ld32(t + c0, a);
-    tmem_ld_wait();
+    // the warp's 32 x 32 block (rows 32 qd .., columns c0 ..) lies wholly outside the mask, wholly
+    // inside it, or on the diagonal (warp-uniform)
+    const int qd = r >> 5, cq = c0 >> 5;
+    const bool zero = kUpper ? cq < qd : cq > qd, full = kUpper ? cq > qd : cq < qd;
     uint32_t hp[16], lp[16];
+    if (zero) {
 #pragma unroll
-    for (int i = 0; i < 16; ++i) {
-        const int c = c0 + 2 * i;
-        const bool k0 = kUpper ? c >= r : c <= r, k1 = kUpper ? c + 1 >= r : c + 1 <= r;
-        split2(k0 ? __uint_as_float(a[2 * i]) : 0.f, k1 ? __uint_as_float(a[2 * i + 1]) : 0.f, hp[i], lp[i]);
+        for (int i = 0; i < 16; ++i) hp[i] = lp[i] = 0u;
+    } else {
+        uint32_t a[32];
+        tmem_ld32(t + c0, a);
+        tmem_ld_wait();
+        if (full) {
+#pragma unroll
+            for (int i = 0; i < 16; ++i) split2(__uint_as_float(a[2 * i]), __uint_as_float(a[2 * i + 1]), hp[i], lp[i]);
+        } else {
+#pragma unroll
+            for (int i = 0; i < 16; ++i) {
+                const int c = c0 + 2 * i;
+                const bool k0 = kUpper ? c >= r : c <= r, k1 = kUpper ? c + 1 >= r : c + 1 <= r;
+                split2(k0 ? __uint_as_float(a[2 * i]) : 0.f, k1 ? __uint_as_float(a[2 * i + 1]) : 0.f, hp[i], lp[i]);
+            }
+        }
     }
     tmem_st16(t + c0, hp);
     if (kLo) tmem_st16(t + c0 + 16, lp);
