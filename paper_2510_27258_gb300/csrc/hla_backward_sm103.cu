@@ -100,9 +100,11 @@ enum Bar {
     bCkDone = 22,  // a head's records are in global memory
     bEvCar = 23,   // reverse sweep, second issuer: the carries (its last reads of G, X and the checkpoint)
     bTear2 = 24,
-    kNumBars = 25
+    bEp5b = 25,   // reverse sweep: dQ read out of TMEM (DQ free for K Lam_s)
+    bEvKL = 26,   // reverse sweep, second issuer: K Lam_s in DQ
+    kNumBars = 27
 };
-__host__ __device__ constexpr bool epi_bar(int b) { return b >= bEp0 && b <= bEp5; }
+__host__ __device__ constexpr bool epi_bar(int b) { return (b >= bEp0 && b <= bEp5) || b == bEp5b; }
 
 struct Misc {
     uint64_t bar[kNumBars];
@@ -346,12 +348,6 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                 tma_load_3d(blk(b0 + 1), &tm_k, &ms->bar[bLd0 + set], 0, j * kTile, head);
                 tma_load_3d(blk(b0 + 2), &tm_v, &ms->bar[bLd0 + set], 0, j * kTile, head);
             };
-            auto load_gck = [&](int head, int j) {  // G of tile j and its record (X hi, lo; S_p, D_p)
-                ld_pend |= 4u;
-                mbar_arrive_expect_tx(&ms->bar[bLdG], kBlockBytes + kCkBytes);
-                tma_load_3d(blk(bG), &tm_g, &ms->bar[bLdG], 0, j * kTile, head);
-                bulk_load(blk(bXh), p.ck + ((size_t)head * M + j) * kCkBytes, kCkBytes, &ms->bar[bLdG]);
-            };
             auto wait_ld = [&](int set) {  // set 0, 1: a Q, K, V set; 2: G and the record
                 if (!bar_poll(ms, bLd0 + set, (ld_par >> set) & 1u, p)) return false;
                 ld_par ^= 1u << set;
@@ -390,20 +386,11 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                 if (!ok) break;
                 // the checkpoints are in global memory (the epilogue waited for its copies)
                 if (!bar_poll(ms, bCkDone, n_head & 1, p)) break;
-                // ---------------- reverse sweep: gradients ----------------
-                load_fwd(0, head, M - 1);
-                load_gck(head, M - 1);
+                // ---------------- reverse sweep: gradients (the second issuer makes the copies) ----
                 for (int j = M - 1; j >= 0 && ok; --j, ++n_b, ++n_s) {
                     const uint32_t ts = n_s & 1, tp = n_b & 1;
                     const int set = (M - 1 - j) & 1, qb = set ? bQ2 : bQ, kb = qb + 1, vb = qb + 2;
                     ok = false;
-                    if (j > 0) {  // the other set is free (the previous tile's products are done)
-                        load_fwd(set ^ 1, head, j - 1);
-                        const size_t t0 = (size_t)head * p.n + (size_t)(j - 1) * kTile;
-                        const uint32_t bytes = (uint32_t)min(kTile, p.n - (j - 1) * kTile) * kD * 2;
-                        bulk_prefetch_l2(tok.g + t0 * kD, bytes);  // G and the record towards L2
-                        bulk_prefetch_l2(p.ck + ((size_t)head * M + j - 1) * kCkBytes, kCkBytes);
-                    }
                     // Q, K, V; G and the record.  P^T starts at once (T0 was last read by this
                     // thread's B^T Q); the epilogue packs it after the carry hand-off E0, so the
                     // arrival of E1 also says Gam_s, Lam_s (hi, lo) are in shared memory.
@@ -433,16 +420,8 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                     umma_commit(&ms->bar[bEvB2]);
                     if (!bar_poll(ms, bEp4b, tp, p)) break;  // B^T in T0 and dV out of DK
                     tc_fence_after();
-                    mma<false, false, 64, 4>(DK, lk(kb), lk(bLam), 0u);  // dK = K Lam''^T
-                    mma<false, false, 64, 4>(DK, lk(kb), lk(bLam) + kH16, 1u);
-                    mma<false, true, 64, 4>(DK, lk(kb), lm(bLam), 1u);  //   + K Lam''
-                    mma<false, true, 64, 4>(DK, lk(kb), lm(bLam) + kH16, 1u);
-                    mma_ts(DK, T0, lm(qb), 1u);  //   + B^T Q
+                    mma_ts(DK, T0, lm(qb), 0u);  // dK = B^T Q (+ W^T Y below; K Lam_s goes to DQ)
                     mma_ts(DK, T0 + 16, lm(qb), 1u);
-                    // every product that reads G or the record is done (this thread's by the B^T
-                    // hand-off, the second issuer's by its carry commit)
-                    if (!bar_poll(ms, bEvCar, tp, p)) break;
-                    if (j > 0) load_gck(head, j - 1);
                     if (!bar_poll(ms, bEp5, tp, p)) break;  // W^T in T1
                     tc_fence_after();
                     mma_ts(DK, T1, lm(bYh), 1u);  //   + W^T Y
@@ -452,7 +431,8 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                     if (!bar_poll(ms, bEvO, tp, p)) break;  // every operand of this set read
                     ok = true;
                 }
-                if (!ok) break;
+                // the second issuer's last K Lam_s has read its set before the next head's copies
+                if (!ok || !bar_poll(ms, bEvKL, (n_b - 1) & 1u, p)) break;
             }
             if (ms->abort_flag) {  // copies and MMAs in flight finish (bounded) before release
                 for (int s = 0; s < 2; ++s)
@@ -472,23 +452,48 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
             const uint32_t DQ = tb + kDQ, GAM = tb + kGAM, LAM = tb + kLAM, T1 = tb + kT1;
             // the same tile counters as the first issuer; ld_par follows every completed copy phase,
             // the forward sweep's included (set j % 2 for forward tile j)
-            uint32_t ld_par = 0, n_s = 0, n_b = 0, n_head = 0;
+            uint32_t ld_par = 0, ld_pend = 0, n_s = 0, n_b = 0, n_head = 0;
             auto wait_ld = [&](int set) {
                 if (!bar_poll(ms, bLd0 + set, (ld_par >> set) & 1u, p)) return false;
                 ld_par ^= 1u << set;
+                ld_pend &= ~(1u << set);
                 return true;
+            };
+            auto load_qkv = [&](int set, int head, int j) {  // Q, K, V of tile j into blocks 0..2 or 11..13
+                const int b0 = set ? bQ2 : bQ;
+                ld_pend |= 1u << set;
+                mbar_arrive_expect_tx(&ms->bar[bLd0 + set], 3 * kBlockBytes);
+                tma_load_3d(blk(b0), &tm_q, &ms->bar[bLd0 + set], 0, j * kTile, head);
+                tma_load_3d(blk(b0 + 1), &tm_k, &ms->bar[bLd0 + set], 0, j * kTile, head);
+                tma_load_3d(blk(b0 + 2), &tm_v, &ms->bar[bLd0 + set], 0, j * kTile, head);
+            };
+            auto load_gck = [&](int head, int j) {  // G of tile j and its record (X hi, lo; S_p, D_p)
+                ld_pend |= 4u;
+                mbar_arrive_expect_tx(&ms->bar[bLdG], kBlockBytes + kCkBytes);
+                tma_load_3d(blk(bG), &tm_g, &ms->bar[bLdG], 0, j * kTile, head);
+                bulk_load(blk(bXh), p.ck + ((size_t)head * M + j) * kCkBytes, kCkBytes, &ms->bar[bLdG]);
             };
             for (int head = blockIdx.x; head < p.BH && !ms->abort_flag; head += gridDim.x, ++n_head) {
                 n_s += (uint32_t)M;
                 ld_par ^= (uint32_t)(((M + 1) / 2) & 1) | ((uint32_t)((M / 2) & 1) << 1);
-                if (!bar_poll(ms, bCkDone, n_head & 1, p)) break;
+                if (!bar_poll(ms, bCkDone, n_head & 1, p)) break;  // every record written, every forward product done
+                load_qkv(0, head, M - 1);
+                load_gck(head, M - 1);
                 bool ok = true;
                 for (int j = M - 1; j >= 0 && ok; --j, ++n_b, ++n_s) {
                     const uint32_t ts = n_s & 1, tp = n_b & 1;
                     const int set = (M - 1 - j) & 1, qb = set ? bQ2 : bQ, kb = qb + 1, vb = qb + 2;
                     ok = false;
-                    // T1 free (the previous tile's W^T Y has read it); Q, K, V; G and the record
-                    if (j < M - 1 && !bar_poll(ms, bEvO, tp ^ 1u, p)) break;
+                    // the previous tile's products are done (the first issuer's, the last of which
+                    // read T1, and this thread's K Lam_s): its set takes the next tile's Q, K, V
+                    if (j < M - 1 && (!bar_poll(ms, bEvO, tp ^ 1u, p) || !bar_poll(ms, bEvKL, tp ^ 1u, p))) break;
+                    if (j > 0) {
+                        load_qkv(set ^ 1, head, j - 1);
+                        const size_t t0 = (size_t)head * p.n + (size_t)(j - 1) * kTile;
+                        const uint32_t bytes = (uint32_t)min(kTile, p.n - (j - 1) * kTile) * kD * 2;
+                        bulk_prefetch_l2(tok.g + t0 * kD, bytes);  // G and the record towards L2
+                        bulk_prefetch_l2(p.ck + ((size_t)head * M + j - 1) * kCkBytes, kCkBytes);
+                    }
                     if (!wait_ld(set) || !wait_ld(2)) break;
                     tc_fence_after();
                     mma<false, false, 128, 4>(T1, lk(bG), lk(vb), 0u);  // P = G V^T
@@ -516,11 +521,24 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                     mma_ts(DQ, T1 + 16, lm(kb), 1u);
                     mma<false, false, 128, 4>(T1, lk(kb), lk(qb), 0u);  // W^T = K Q^T
                     umma_commit(&ms->bar[bEvW]);
+                    // every product that reads G or the record is done (the first issuer's by the
+                    // B^T hand-off, this thread's by its carry commit): the next tile's G and record
+                    if (!bar_poll(ms, bEp4b, tp, p) || !bar_poll(ms, bEvCar, tp, p)) break;
+                    if (j > 0) load_gck(head, j - 1);
+                    if (!bar_poll(ms, bEp5b, tp, p)) break;  // dQ read out of DQ
+                    tc_fence_after();
+                    mma<false, false, 64, 4>(DQ, lk(kb), lk(bLam), 0u);  // K Lam_s = K Lam''^T
+                    mma<false, false, 64, 4>(DQ, lk(kb), lk(bLam) + kH16, 1u);
+                    mma<false, true, 64, 4>(DQ, lk(kb), lm(bLam), 1u);  //   + K Lam''
+                    mma<false, true, 64, 4>(DQ, lk(kb), lm(bLam) + kH16, 1u);
+                    umma_commit(&ms->bar[bEvKL]);
                     ok = true;
                 }
                 if (!ok) break;
             }
-            if (ms->abort_flag) {  // this thread's MMAs in flight finish (bounded) before release
+            if (ms->abort_flag) {  // this thread's copies and MMAs in flight finish (bounded) before release
+                for (int s = 0; s < 3; ++s)
+                    if ((ld_pend >> s) & 1u) mbar_wait(&ms->bar[bLd0 + s], (ld_par >> s) & 1u, kBarWaitNs);
                 umma_commit(&ms->bar[bTear2]);
                 mbar_wait(&ms->bar[bTear2], 0, kBarWaitNs);
             }
@@ -552,6 +570,23 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
         };
         // a 64-wide result -> bf16 in a free block -> one TMA store of the tile (rows past n are
         // not written); row-wise stores from the threads would cost a 16-byte piece per row
+        auto drain2 = [&](uint32_t col, uint32_t col2, int stage, const CUtensorMap *map, int tok0, int head) {
+            uint32_t a[16], b[16];
+            tmem_ld16(tb + lb + col + c16, a);
+            tmem_ld16(tb + lb + col2 + c16, b);
+            tmem_ld_wait();
+#pragma unroll
+            for (int u = 0; u < 16; ++u) a[u] = __float_as_uint(__uint_as_float(a[u]) + __uint_as_float(b[u]));
+            if (tid == 0) tma_store_wait_read();
+            epi_sync();
+            store16(blk(stage), r, c16, a);
+            fence_async_smem();
+            epi_sync();
+            if (tid == 0) {
+                tma_store_3d(map, blk(stage), 0, tok0, head);
+                tma_store_commit();
+            }
+        };
         auto drain = [&](uint32_t col, int stage, const CUtensorMap *map, int tok0, int head) {
             uint32_t a[16];
             tmem_ld16(tb + lb + col + c16, a);
@@ -670,10 +705,12 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                 mask_pack<true, true>(t1, r, c32);
                 epi_arrive(ms, bEp5);
                 drain(kDQ, bGam, &tm_dq, tok0, head);
-                // E6: dK out
+                epi_arrive(ms, bEp5b);
+                // E6: dK = (B^T Q + W^T Y from DK) + (K Lam_s from DQ) out
                 bar_wait(ms, bEvO, tp, p);
+                bar_wait(ms, bEvKL, tp, p);
                 tc_fence_after();
-                drain(kDK, bYh, &tm_dk, tok0, head);  // Y read by its last product (W^T Y)
+                drain2(kDK, kDQ, bYh, &tm_dk, tok0, head);  // Y read by its last product (W^T Y)
             }
         }
         if (tid == 0) tma_store_wait_all();
