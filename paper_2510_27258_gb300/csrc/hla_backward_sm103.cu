@@ -138,33 +138,6 @@ __device__ __forceinline__ bool bar_wait(Misc *ms, int b, uint32_t parity, const
     return false;
 }
 
-// The issuers' wait: a non-suspending poll (a suspended try_wait was seen to resume up to
-// ~900 cycles after the phase completed), bounded like mbar_wait.
-__device__ __forceinline__ bool mbar_test(uint64_t *bar, uint32_t parity) {
-    uint32_t ok;
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-        "selp.u32 %0, 1, 0, p;\n\t}"
-        : "=r"(ok)
-        : "r"(smem_u32(bar)), "r"(parity)
-        : "memory");
-    return ok != 0;
-}
-__device__ __forceinline__ bool bar_poll(Misc *ms, int b, uint32_t parity, const Params &p) {
-    if (ms->abort_flag) return false;
-    if (mbar_test(&ms->bar[b], parity)) return true;
-    const uint64_t t0 = globaltimer_ns();
-    while (true) {
-        for (int i = 0; i < 32; ++i)
-            if (mbar_test(&ms->bar[b], parity)) return true;
-        if (globaltimer_ns() - t0 > kBarWaitNs) break;
-    }
-    set_error(p.err, 500 + b, parity);
-    ms->abort_flag = 1;
-    return false;
-}
-
 __device__ __forceinline__ void epi_sync() { asm volatile("bar.sync 1, %0;" ::"n"(kEpiThreads) : "memory"); }
 
 __device__ __forceinline__ void epi_arrive(Misc *ms, int b) {
@@ -349,7 +322,7 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                 tma_load_3d(blk(b0 + 2), &tm_v, &ms->bar[bLd0 + set], 0, j * kTile, head);
             };
             auto wait_ld = [&](int set) {  // set 0, 1: a Q, K, V set; 2: G and the record
-                if (!bar_poll(ms, bLd0 + set, (ld_par >> set) & 1u, p)) return false;
+                if (!bar_wait(ms, bLd0 + set, (ld_par >> set) & 1u, p)) return false;
                 ld_par ^= 1u << set;
                 ld_pend &= ~(1u << set);
                 return true;
@@ -363,29 +336,29 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                     const uint32_t tp = n_s & 1, tf = n_f & 1;
                     const int set = j & 1, qb = set ? bQ2 : bQ, kb = qb + 1, vb = qb + 2;
                     ok = false;
-                    if (!bar_poll(ms, bEp0, tp, p) || !wait_ld(set)) break;  // S_p (bf16) in bCk; tokens
+                    if (!bar_wait(ms, bEp0, tp, p) || !wait_ld(set)) break;  // S_p (bf16) in bCk; tokens
                     tc_fence_after();
                     mma<false, false, 128, 4>(T0, lk(qb), lk(kb), 0u);  // A = Q K^T
                     umma_commit(&ms->bar[bEvA]);
                     mma<true, true, 64, 8>(GAM, lm(kb), lm(kb), 1u);  // S += K^T K (under E1)
-                    if (!bar_poll(ms, bEp1, tp, p)) break;           // W (hi, lo) packed in T0
+                    if (!bar_wait(ms, bEp1, tp, p)) break;           // W (hi, lo) packed in T0
                     tc_fence_after();
                     mma_ts(DK, T0, lm(kb), 0u);                       // X = W K
                     mma_ts(DK, T0 + 16, lm(kb), 1u);
                     mma<false, false, 64, 4>(DK, lk(qb), lk(bCk), 1u);  //   + Q S_p
                     umma_commit(&ms->bar[bEvX]);
-                    if (!bar_poll(ms, bEp2, tp, p)) break;  // X (hi, lo) in bXh, bXl
+                    if (!bar_wait(ms, bEp2, tp, p)) break;  // X (hi, lo) in bXh, bXl
                     tc_fence_after();
                     mma<true, true, 64, 8>(LAM, lm(bXh), lm(vb), 1u);  // D += X^T V
                     mma<true, true, 64, 8>(LAM, lm(bXl), lm(vb), 1u);
                     umma_commit(&ms->bar[bEvC]);
-                    if (!bar_poll(ms, bEvC, tf, p)) break;  // this set is free again
+                    if (!bar_wait(ms, bEvC, tf, p)) break;  // this set is free again
                     if (j + 2 < M) load_fwd(set, head, j + 2);
                     ok = true;
                 }
                 if (!ok) break;
                 // the checkpoints are in global memory (the epilogue waited for its copies)
-                if (!bar_poll(ms, bCkDone, n_head & 1, p)) break;
+                if (!bar_wait(ms, bCkDone, n_head & 1, p)) break;
                 // ---------------- reverse sweep: gradients (the second issuer makes the copies) ----
                 for (int j = M - 1; j >= 0 && ok; --j, ++n_b, ++n_s) {
                     const uint32_t ts = n_s & 1, tp = n_b & 1;
@@ -398,7 +371,7 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                     tc_fence_after();
                     mma<false, false, 128, 4>(T0, lk(vb), lk(bG), 0u);  // P^T = V G^T
                     umma_commit(&ms->bar[bEvA]);
-                    if (!bar_poll(ms, bEp1, ts, p)) break;  // P^T in T0; E0 done
+                    if (!bar_wait(ms, bEp1, ts, p)) break;  // P^T in T0; E0 done
                     tc_fence_after();
                     mma_ts(DK, T0, lm(qb), 0u);  // Y = P^T Q
                     mma_ts(DK, T0 + 16, lm(qb), 1u);
@@ -408,7 +381,7 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                     mma<false, false, 128, 4>(T0, lk(bXh), lk(qb), 0u);  // T^T = X Q^T
                     mma<false, false, 128, 4>(T0, lk(bXl), lk(qb), 1u);
                     umma_commit(&ms->bar[bEvT]);
-                    if (!bar_poll(ms, bEp3, tp, p)) break;  // T^T in T0
+                    if (!bar_wait(ms, bEp3, tp, p)) break;  // T^T in T0
                     tc_fence_after();
                     mma_ts(DK, T0, lm(bG), 0u);                                 // dV = T^T G
                     mma<false, true, 64, 4>(DK, lk(bXh), lm(bGam), 1u);         //   + X Gam_s^T
@@ -418,21 +391,21 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                     mma<false, false, 128, 4>(T0, lk(kb), lk(bYh), 0u);  // B^T = K Y^T
                     mma<false, false, 128, 4>(T0, lk(kb), lk(bYl), 1u);
                     umma_commit(&ms->bar[bEvB2]);
-                    if (!bar_poll(ms, bEp4b, tp, p)) break;  // B^T in T0 and dV out of DK
+                    if (!bar_wait(ms, bEp4b, tp, p)) break;  // B^T in T0 and dV out of DK
                     tc_fence_after();
                     mma_ts(DK, T0, lm(qb), 0u);  // dK = B^T Q (+ W^T Y below; K Lam_s goes to DQ)
                     mma_ts(DK, T0 + 16, lm(qb), 1u);
-                    if (!bar_poll(ms, bEp5, tp, p)) break;  // W^T in T1
+                    if (!bar_wait(ms, bEp5, tp, p)) break;  // W^T in T1
                     tc_fence_after();
                     mma_ts(DK, T1, lm(bYh), 1u);  //   + W^T Y
                     mma_ts(DK, T1, lm(bYl), 1u);
                     mma_ts(DK, T1 + 16, lm(bYh), 1u);
                     umma_commit(&ms->bar[bEvO]);
-                    if (!bar_poll(ms, bEvO, tp, p)) break;  // every operand of this set read
+                    if (!bar_wait(ms, bEvO, tp, p)) break;  // every operand of this set read
                     ok = true;
                 }
                 // the second issuer's last K Lam_s has read its set before the next head's copies
-                if (!ok || !bar_poll(ms, bEvKL, (n_b - 1) & 1u, p)) break;
+                if (!ok || !bar_wait(ms, bEvKL, (n_b - 1) & 1u, p)) break;
             }
             if (ms->abort_flag) {  // copies and MMAs in flight finish (bounded) before release
                 for (int s = 0; s < 2; ++s)
@@ -454,7 +427,7 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
             // the forward sweep's included (set j % 2 for forward tile j)
             uint32_t ld_par = 0, ld_pend = 0, n_s = 0, n_b = 0, n_head = 0;
             auto wait_ld = [&](int set) {
-                if (!bar_poll(ms, bLd0 + set, (ld_par >> set) & 1u, p)) return false;
+                if (!bar_wait(ms, bLd0 + set, (ld_par >> set) & 1u, p)) return false;
                 ld_par ^= 1u << set;
                 ld_pend &= ~(1u << set);
                 return true;
@@ -476,7 +449,7 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
             for (int head = blockIdx.x; head < p.BH && !ms->abort_flag; head += gridDim.x, ++n_head) {
                 n_s += (uint32_t)M;
                 ld_par ^= (uint32_t)(((M + 1) / 2) & 1) | ((uint32_t)((M / 2) & 1) << 1);
-                if (!bar_poll(ms, bCkDone, n_head & 1, p)) break;  // every record written, every forward product done
+                if (!bar_wait(ms, bCkDone, n_head & 1, p)) break;  // every record written, every forward product done
                 load_qkv(0, head, M - 1);
                 load_gck(head, M - 1);
                 bool ok = true;
@@ -486,7 +459,7 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                     ok = false;
                     // the previous tile's products are done (the first issuer's, the last of which
                     // read T1, and this thread's K Lam_s): its set takes the next tile's Q, K, V
-                    if (j < M - 1 && (!bar_poll(ms, bEvO, tp ^ 1u, p) || !bar_poll(ms, bEvKL, tp ^ 1u, p))) break;
+                    if (j < M - 1 && (!bar_wait(ms, bEvO, tp ^ 1u, p) || !bar_wait(ms, bEvKL, tp ^ 1u, p))) break;
                     if (j > 0) {
                         load_qkv(set ^ 1, head, j - 1);
                         const size_t t0 = (size_t)head * p.n + (size_t)(j - 1) * kTile;
@@ -498,13 +471,13 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                     tc_fence_after();
                     mma<false, false, 128, 4>(T1, lk(bG), lk(vb), 0u);  // P = G V^T
                     umma_commit(&ms->bar[bEvA2]);
-                    if (!bar_poll(ms, bEp1b, tp, p)) break;  // P in T1
+                    if (!bar_wait(ms, bEp1b, tp, p)) break;  // P in T1
                     tc_fence_after();
                     mma_ts(DQ, T1, lm(bXh), 0u);  // dQ = P X
                     mma_ts(DQ, T1, lm(bXl), 1u);
                     mma_ts(DQ, T1 + 16, lm(bXh), 1u);
                     mma<false, false, 64, 4>(DQ, lk(bG), lk(bCk) + kH16, 1u);  //   + G D_p^T
-                    if (!bar_poll(ms, bEp2, ts, p)) break;  // Y (hi, lo) in shared memory
+                    if (!bar_wait(ms, bEp2, ts, p)) break;  // Y (hi, lo) in shared memory
                     tc_fence_after();
                     mma<false, false, 64, 4>(DQ, lk(bYh), lk(bCk), 1u);  //   + Y S_p
                     mma<false, false, 64, 4>(DQ, lk(bYl), lk(bCk), 1u);
@@ -515,7 +488,7 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                     mma<true, true, 128, 8>(GAM, lm(qb), lm(bG), 1u);
                     mma<true, true, 64, 8>(LAM, lm(qb), lm(bYl), 1u);
                     umma_commit(&ms->bar[bEvCar]);
-                    if (!bar_poll(ms, bEp4a, tp, p)) break;  // B in T1
+                    if (!bar_wait(ms, bEp4a, tp, p)) break;  // B in T1
                     tc_fence_after();
                     mma_ts(DQ, T1, lm(kb), 1u);  // dQ += B K
                     mma_ts(DQ, T1 + 16, lm(kb), 1u);
@@ -523,9 +496,9 @@ bwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ 
                     umma_commit(&ms->bar[bEvW]);
                     // every product that reads G or the record is done (the first issuer's by the
                     // B^T hand-off, this thread's by its carry commit): the next tile's G and record
-                    if (!bar_poll(ms, bEp4b, tp, p) || !bar_poll(ms, bEvCar, tp, p)) break;
+                    if (!bar_wait(ms, bEp4b, tp, p) || !bar_wait(ms, bEvCar, tp, p)) break;
                     if (j > 0) load_gck(head, j - 1);
-                    if (!bar_poll(ms, bEp5b, tp, p)) break;  // dQ read out of DQ
+                    if (!bar_wait(ms, bEp5b, tp, p)) break;  // dQ read out of DQ
                     tc_fence_after();
                     mma<false, false, 64, 4>(DQ, lk(kb), lk(bLam), 0u);  // K Lam_s = K Lam''^T
                     mma<false, false, 64, 4>(DQ, lk(kb), lk(bLam) + kH16, 1u);
