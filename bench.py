@@ -54,6 +54,11 @@ TRAFFIC = {
                         "how": "ncu capture of one forward's three launches (bench.py --only hla3_f32), caches "
                                "flushed per launch: pre-pass 37.8 MB read, sweep 51.7 MB read + 0.1 MB written "
                                "(outputs still dirty in L2 at its end), fix-up 25.6 MB read"},
+    "bwd_tc_kernel": {"src": ["hla_backward_sm103.cu", "sm103_prims.cuh"], "sha256": "e1940b86e729b1d1",
+                      "workload": "mid_bf16", "n": 2048, "bytes": 448.4e6,
+                      "how": "ncu capture of one backward (bench.py --only backward): 278.0 MB read + 170.4 MB "
+                             "written; the per-tile records (X hi, lo; S_p, D_p: 96 MB) are written once and read "
+                             "back once"},
     "step2_kernel_sde": {"src": ["hla_step.cu"], "sha256": "5542daa4b35fe2f4", "workload": "decode_bf16", "n": 0,
                          "bytes": 481.3e6, "how": "ncu capture of one step at B64 H32 d128 (bench.py --profile-case "
                                                   "sde_step): 271.2 MB read + 210.1 MB written"},
@@ -681,6 +686,15 @@ def bwd_flops(w, C=None, W=None):
     return fwd_flops(w) + w.BH * w.n * per
 
 
+def bwd_tc_issued_flops(w):
+    """Tensor FLOPs the tensor-core backward issues (bf16 hi/lo pairs, full 128-row tiles): per
+    128-token tile 48 K = 16 steps at N = 128 and 204 at N = 64 (forward sweep 4 and 44, reverse
+    sweep 44 and 160)."""
+    M = (w.n + 127) // 128
+    step = lambda N: 2 * 128 * N * 16
+    return w.BH * M * (48 * step(128) + 204 * step(64))
+
+
 def bench_backward(hla, dev, stream, world, hbm_peak, tc_peak, steps=10, warmup=3):
     """hla2_backward on mid_bf16 (B8 H16 n2048 d64 bf16, chunk 64), CUDA events on the launching stream."""
     import torch
@@ -716,10 +730,14 @@ def bench_backward(hla, dev, stream, world, hbm_peak, tc_peak, steps=10, warmup=
         hbm = {"achieved": gbs, "peak": hbm_peak, "unit": "GB/s", "frac": gbs / hbm_peak}
         ten = {"achieved": tfl, "peak": tc_peak, "unit": "TFLOP/s", "frac": tfl / tc_peak}
         bound, main, other = ("hbm", hbm, ten) if t_b >= t_f else ("tensor", ten, hbm)
+        tr, tr_how = traffic("bwd_tc_kernel", w.name, w.n)
+        issued = bwd_tc_issued_flops(w)
         rec["roofline"] = {"bound": bound, "achieved": main["achieved"], "peak": main["peak"], "unit": main["unit"],
-                           "frac": main["frac"], "traffic": None, "algorithmic_bytes": nbytes, "flops": flops,
-                           "roofline_us": max(t_b, t_f) * 1e6, "peak_kind": "measured",
+                           "frac": main["frac"], "traffic": tr, "traffic_how": tr_how, "algorithmic_bytes": nbytes,
+                           "flops": flops, "roofline_us": max(t_b, t_f) * 1e6, "peak_kind": "measured",
                            ("tensor_view" if bound == "hbm" else "hbm_view"): other,
+                           "issued_tensor": {"flops": issued, "achieved": issued / (ms * 1e-3) / 1e12, "peak": tc_peak,
+                                             "unit": "TFLOP/s", "frac": issued / (ms * 1e-3) / 1e12 / tc_peak},
                            "kernel": "bwd_tc_kernel (tcgen05, one launch)"}
         rec["path"] = "tensor cores"
         rec["launches"] = steps
