@@ -279,11 +279,16 @@ ahla_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
                         uint32_t a[32];
                         tmem_ld32(tb + lane_base + kTA + c0, a);
                         tmem_ld_wait();
+                        if (cq < qd) {  // wholly below the diagonal: no compares
 #pragma unroll
-                        for (int i = 0; i < 16; ++i) {
-                            const float x0 = (c0 + 2 * i <= r) ? __uint_as_float(a[2 * i]) : 0.f;
-                            const float x1 = (c0 + 2 * i + 1 <= r) ? __uint_as_float(a[2 * i + 1]) : 0.f;
-                            h[i] = pack_bf16x2(x0, x1);
+                            for (int i = 0; i < 16; ++i) h[i] = pack_bf16x2(__uint_as_float(a[2 * i]), __uint_as_float(a[2 * i + 1]));
+                        } else {
+#pragma unroll
+                            for (int i = 0; i < 16; ++i) {
+                                const float x0 = (c0 + 2 * i <= r) ? __uint_as_float(a[2 * i]) : 0.f;
+                                const float x1 = (c0 + 2 * i + 1 <= r) ? __uint_as_float(a[2 * i + 1]) : 0.f;
+                                h[i] = pack_bf16x2(x0, x1);
+                            }
                         }
                     }
                     tmem_st16(tb + lane_base + kTA + c0, h);
