@@ -575,25 +575,32 @@ __global__ void __launch_bounds__(kThreads, 1) hla3_tc_kernel(Params p) {
                         for (int i = 0; i < 32; ++i) a[i] = (i == lane) ? __float_as_uint(dg) : a[i];
                         ms->sa[r] = dg;
                     }
-                    const bool blk_zero = cq > qd;  // columns all above the diagonal
+                    // this warp's 32 x 32 block lies above the diagonal (blk_zero), below it (blk_full) or on it
+                    const bool blk_zero = cq > qd, blk_full = cq < qd;
 #pragma unroll
                     for (int jj = 0; jj < 32; jj += 8) {
-                        float x[8];
+                        uint4 h = make_uint4(0u, 0u, 0u, 0u), l = h;
+                        if (!blk_zero) {
+                            float x[8];
 #pragma unroll
-                        for (int u = 0; u < 8; ++u)
-                            x[u] = (!blk_zero && 32 * cq + jj + u <= r) ? __uint_as_float(a[jj + u]) : 0.f;
-                        uint4 h, l;
-                        split8(x, h, l);
+                            for (int u = 0; u < 8; ++u)
+                                x[u] = (blk_full || 32 * cq + jj + u <= r) ? __uint_as_float(a[jj + u]) : 0.f;
+                            split8(x, h, l);
+                        }
                         st16(blk(bLh), r, 32 * cq + jj, h);
                         st16(blk(bLl), r, 32 * cq + jj, l);
                     }
-                    float x[32];
+                    if (blk_full) {  // no entry above the diagonal
+                        ms->sbp[qd][32 * cq + lane] = 0.f;
+                    } else {
+                        float x[32];
 #pragma unroll
-                    for (int i = 0; i < 32; ++i) {
-                        const float av = __uint_as_float(a[i]);
-                        x[i] = (r < 32 * cq + i) ? av * av : 0.f;
+                        for (int i = 0; i < 32; ++i) {
+                            const float av = __uint_as_float(a[i]);
+                            x[i] = (blk_zero || r < 32 * cq + i) ? av * av : 0.f;
+                        }
+                        ms->sbp[qd][32 * cq + lane] = reduce_scatter32(x, lane);
                     }
-                    ms->sbp[qd][32 * cq + lane] = reduce_scatter32(x, lane);
                 }
                 fence_async_smem();
                 epi_arrive(ms, bEp1);
@@ -651,18 +658,23 @@ __global__ void __launch_bounds__(kThreads, 1) hla3_tc_kernel(Params p) {
                     store_hl8(blk(bG), r, 8 * cq, gf);
                 }
                 {
-                    uint32_t c[32];
-                    tmem_ld32(tb + lb + kTA + 32 * cq, c);
-                    tmem_ld_wait();
-                    const bool blk_zero = cq > qd;
+                    const bool blk_zero = cq > qd, blk_full = cq < qd;  // above, below or on the diagonal
                     uint32_t hp[16], lp[16];
+                    if (blk_zero) {
 #pragma unroll
-                    for (int i = 0; i < 16; ++i) {
-                        const int c0 = 32 * cq + 2 * i;
-                        const float x0 = (!blk_zero && c0 <= r) ? __uint_as_float(c[2 * i]) : 0.f;
-                        const float x1 = (!blk_zero && c0 + 1 <= r) ? __uint_as_float(c[2 * i + 1]) : 0.f;
-                        hp[i] = pack_bf16x2(x0, x1);
-                        lp[i] = pack_bf16x2(x0 - __uint_as_float(hp[i] << 16), x1 - __uint_as_float(hp[i] & 0xFFFF0000u));
+                        for (int i = 0; i < 16; ++i) hp[i] = lp[i] = 0u;
+                    } else {
+                        uint32_t c[32];
+                        tmem_ld32(tb + lb + kTA + 32 * cq, c);
+                        tmem_ld_wait();
+#pragma unroll
+                        for (int i = 0; i < 16; ++i) {
+                            const int c0 = 32 * cq + 2 * i;
+                            const float x0 = (blk_full || c0 <= r) ? __uint_as_float(c[2 * i]) : 0.f;
+                            const float x1 = (blk_full || c0 + 1 <= r) ? __uint_as_float(c[2 * i + 1]) : 0.f;
+                            hp[i] = pack_bf16x2(x0, x1);
+                            lp[i] = pack_bf16x2(x0 - __uint_as_float(hp[i] << 16), x1 - __uint_as_float(hp[i] & 0xFFFF0000u));
+                        }
                     }
                     tmem_st16(tb + lb + kTA + 32 * cq, hp);
                     tmem_st16(tb + lb + kTA + 32 * cq + 16, lp);
