@@ -49,10 +49,10 @@ TRAFFIC = {
     "c3_kernels": {"src": ["hla3_chunked.cu"], "sha256": "17ac1acd5c9202d1", "workload": "hla3_f32", "n": 4096,
                    "bytes": 432.5e6, "how": "ncu capture of one forward's five launches (bench.py --only hla3_f32): "
                                             "373.0 MB read + 59.5 MB written, 6.4 x the token I/O (per-chunk records)"},
-    "hla3_tc_kernels": {"src": ["hla3_sm103.cu", "sm103_prims.cuh"], "sha256": "0bf5b53339f19510", "workload": "hla3_f32",
-                        "n": 4096, "bytes": 115.2e6,
+    "hla3_tc_kernels": {"src": ["hla3_sm103.cu", "sm103_prims.cuh"], "sha256": "dd16e8c0a54902eb", "workload": "hla3_f32",
+                        "n": 4096, "bytes": 115.0e6,
                         "how": "ncu capture of one forward's three launches (bench.py --only hla3_f32), caches "
-                               "flushed per launch: pre-pass 37.8 MB read, sweep 51.7 MB read + 0.1 MB written "
+                               "flushed per launch: pre-pass 37.8 MB read, sweep 51.6 MB read + 0.1 MB written "
                                "(outputs still dirty in L2 at its end), fix-up 25.6 MB read"},
     "bwd_tc_kernel": {"src": ["hla_backward_sm103.cu", "sm103_prims.cuh"], "sha256": "e1940b86e729b1d1",
                       "workload": "mid_bf16", "n": 2048, "bytes": 448.4e6,
