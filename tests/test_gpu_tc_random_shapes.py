@@ -67,3 +67,40 @@ def test_ahla_tensor_cores(hla, n, dims):
     torch.cuda.synchronize()
     ref = oracle.ahla_serial(q.reshape(B * H, n, d), k.reshape(B * H, n, d), v.reshape(B * H, n, dv), nthreads=3)
     assert rowerr(out.float().cpu().numpy().reshape(B * H, n, dv), ref) < TOL["bf16"]
+
+
+# ---------------------------------------------------------------------------------------------
+# the fused second-order forward (bf16, masked; plain and ratio-normalised; d, dv in {64, 128}),
+# at the same lengths and head counts, with segment lengths of 1..4 tiles or the planner's
+# ---------------------------------------------------------------------------------------------
+
+def _fused(hla, q, k, v, normalized):
+    tq, tk, tv = (hla_inputs.as_torch(x, "bf16", DEV) for x in (q, k, v))
+    ws = hla.alloc_workspace(hla.hla2_workspace_bytes(*q.shape, v.shape[-1], 128, torch.bfloat16), DEV)
+    out = hla.hla2_forward(tq, tk, tv, masked=True, normalized=normalized, eps=hla_inputs.EPS, chunk=128,
+                           workspace=ws)
+    torch.cuda.synchronize()
+    assert hla.hla_poll_error(ws) == 0
+    B, H, n, _ = q.shape
+    return out.float().cpu().numpy().reshape(B * H, n, -1)
+
+
+@pytest.mark.parametrize("n", LENGTHS)
+@pytest.mark.parametrize("bh", HEADS, ids=lambda x: "B%dH%d" % x)
+@pytest.mark.parametrize("dims", [(64, 64), (128, 128), (64, 128)], ids=lambda x: "d%ddv%d" % x)
+def test_fused_forward(hla, n, bh, dims, monkeypatch):
+    from parity import check_normalized
+    B, H = bh
+    d, dv = dims
+    seg = (n + 3 * H + d) % 5  # 0: the planner's segments, else segments of 1..4 tiles
+    if seg:
+        monkeypatch.setenv("HLA_FUSED_SEGMENT_TILES", str(seg))
+    assert hla.hla2_forward_path(B, H, n, d, dv, chunk=128)[0] == 1
+    q, k, v = hla_inputs.make_qkv(B, H, n, d, dv, seed=11000 + n + 17 * H + d + dv, dtype="bf16")
+    flat = lambda x: x.reshape(B * H, n, -1)
+    num_ref, den_ref = oracle.hla2_serial(flat(q), flat(k), flat(v), masked=True, normalized=False, return_den=True,
+                                          nthreads=8)
+    num = _fused(hla, q, k, v, False)
+    assert rowerr(num, num_ref) < TOL["bf16"], rowerr(num, num_ref)
+    o = _fused(hla, q, k, v, True)
+    check_normalized(o, num, num_ref, den_ref, hla_inputs.EPS, TOL["bf16"])
