@@ -12,10 +12,12 @@
 // G' = G + k (k^T C) at once.  The unmasked form skips G and h (and leaves them
 // untouched).
 //
-// Memory access: every matrix is read once by 16-byte asynchronous copies into
-// shared memory, issued a pass or more ahead of its use, and written once with
-// 16-byte stores; consecutive threads on consecutive columns.
+// Memory access: every matrix is read once into shared memory by a 1-D bulk copy
+// (one instruction per matrix, completing on an mbarrier), issued a pass or more
+// ahead of its use, and written once with 16-byte stores; consecutive threads on
+// consecutive columns.
 #include "hla_internal.h"
+#include "sm103_prims.cuh"
 
 namespace hla {
 namespace {
@@ -73,23 +75,22 @@ __device__ __forceinline__ float warp_dot(const float *a, const float *b, int n)
     return group_sum<32>(s);
 }
 
-// 16-byte asynchronous copy global -> shared (L1 bypassed), and its group bookkeeping: each thread
-// waits for its own copies, a barrier then makes every thread's copies visible
-__device__ __forceinline__ void cp16(void *dst, const void *src) {
-    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"((uint32_t)__cvta_generic_to_shared(dst)), "l"(src)
+// 1-D bulk copy global -> shared (16-byte aligned, a multiple of 16 bytes), completing on `bar`
+__device__ __forceinline__ void bulk_copy(void *dst, const void *src, uint32_t bytes, uint64_t *bar) {
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+                 ::"r"(sm103::smem_u32(dst)), "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes),
+                   "r"(sm103::smem_u32(bar))
                  : "memory");
 }
-__device__ __forceinline__ void cp_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-template <int N>
-__device__ __forceinline__ void cp_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
-
+constexpr unsigned long long kCopyWaitNs = 2000000000ull;
 __device__ __forceinline__ void store4(float4 *p, float4 v) { *p = v; }
 
 // One block per SM, heads hd = blockIdx.x, + gridDim.x, ...  The state of a head is staged in shared
 // memory in three buffers, one per pass (S; C with m; G with h), each refilled with the next head's
 // part as soon as its pass has read it, so that while one pass works the copies of the next two
-// parts (and of the next head's tokens) are in flight.  Updated values go to global memory straight
-// from registers.
+// parts (and of the next head's tokens) are in flight.  Thread 0 issues each refill as one bulk copy
+// on the buffer's mbarrier (phase = the block's head count); every thread waits on it, bounded: a
+// copy that never lands ends the block.  Updated values go to global memory straight from registers.
 //
 // kSDE: the state is (S, D, e) with D = S C - G and e = S m - h (masked operator only; rows of the
 // per-head record: S d*d | D d*dv | e d).  A token then updates
@@ -103,6 +104,7 @@ step2_kernel(const T *__restrict__ q, const T *__restrict__ k, const T *__restri
     __shared__ float qs[128], ks[128], vs[128], us[128];
     __shared__ float part[kStepThreads][12];
     __shared__ float kC[128], uC[128], qG[128];
+    __shared__ uint64_t bar[3];  // S and tokens; (C, m) or (D, e); (G, h)
 
     const int tid = threadIdx.x;
     if (kSDE) masked = 0;  // staging as for (S, C, m): no third buffer
@@ -113,29 +115,37 @@ step2_kernel(const T *__restrict__ q, const T *__restrict__ k, const T *__restri
     float4 *bT = bG + (masked ? nCm : 0);  // raw tokens q | k | v
     const T *tq = reinterpret_cast<const T *>(bT), *tk = tq + d, *tv = tk + d;
 
+    // thread 0 issues the copies: after a block barrier that ends the generic reads of the buffer
     auto load_S = [&](int hd) {  // S and the head's tokens
-        const float4 *src = reinterpret_cast<const float4 *>(state + hd * st_len);
-        for (int f = tid; f < nS; f += kStepThreads) cp16(bS + f, src + f);
-        if (tid < nt_q) {
-            cp16(bT + tid, reinterpret_cast<const float4 *>(q + (long long)hd * d) + tid);
-            cp16(bT + nt_q + tid, reinterpret_cast<const float4 *>(k + (long long)hd * d) + tid);
+        if (tid == 0) {
+            sm103::fence_async_smem();
+            sm103::mbar_arrive_expect_tx(&bar[0], (uint32_t)(16 * (nS + 2 * nt_q + nt_v)));
+            bulk_copy(bS, state + hd * st_len, 16u * nS, &bar[0]);
+            bulk_copy(bT, q + (long long)hd * d, 16u * nt_q, &bar[0]);
+            bulk_copy(bT + nt_q, k + (long long)hd * d, 16u * nt_q, &bar[0]);
+            bulk_copy(bT + 2 * nt_q, v + (long long)hd * dv, 16u * nt_v, &bar[0]);
         }
-        if (tid < nt_v) cp16(bT + 2 * nt_q + tid, reinterpret_cast<const float4 *>(v + (long long)hd * dv) + tid);
-        cp_commit();
     };
-    auto load_part = [&](float4 *dst, int hd, long long off) {  // (C, m) or (G, h)
-        const float4 *src = reinterpret_cast<const float4 *>(state + hd * st_len + off);
-        for (int f = tid; f < nCm; f += kStepThreads) cp16(dst + f, src + f);
-        cp_commit();
+    auto load_part = [&](float4 *dst, int hd, long long off, int b) {  // (C, m), (D, e) or (G, h)
+        if (tid == 0) {
+            sm103::fence_async_smem();
+            sm103::mbar_arrive_expect_tx(&bar[b], 16u * nCm);
+            bulk_copy(dst, state + hd * st_len + off, 16u * nCm, &bar[b]);
+        }
     };
     const long long offC = (long long)d * d, offG = offC + (long long)d * dv + d;
 
     int hd = blockIdx.x;
     if (hd >= BH) return;
+    if (tid == 0) {
+        for (int b = 0; b < 3; ++b) sm103::mbar_init(&bar[b], 1);
+        sm103::fence_mbar_init();
+    }
+    __syncthreads();
     load_S(hd);
-    load_part(bC, hd, offC);
-    if (masked) load_part(bG, hd, offG);
-    for (; hd < BH; hd += gridDim.x) {
+    load_part(bC, hd, offC, 1);
+    if (masked) load_part(bG, hd, offG, 2);
+    for (uint32_t par = 0; hd < BH; hd += gridDim.x, par ^= 1u) {
         const int nx = hd + gridDim.x;  // this block's next head (none: empty copy groups)
         float *S = state + hd * st_len;
         float *Cm = S + offC;
@@ -144,8 +154,7 @@ step2_kernel(const T *__restrict__ q, const T *__restrict__ k, const T *__restri
         float *h = G + (long long)d * dv;
 
         // ---- tokens, k.q ----
-        if (masked) cp_wait<2>(); else cp_wait<1>();  // S and tokens of this head
-        __syncthreads();
+        if (!sm103::mbar_wait(&bar[0], par, kCopyWaitNs)) return;  // S and tokens of this head
         if (tid < d) {
             qs[tid] = to_f32(tq[tid]);
             ks[tid] = to_f32(tk[tid]);
@@ -200,12 +209,11 @@ step2_kernel(const T *__restrict__ q, const T *__restrict__ k, const T *__restri
             }
         }
         __syncthreads();  // S buffer read, u' complete
-        if (nx < BH) load_S(nx); else cp_commit();
+        if (nx < BH) load_S(nx);
 
         if constexpr (kSDE) {
             // ---- pass over D: column sums q^T D (old D); D' = D + u' v^T; e' = e + u' ----
-            cp_wait<1>();  // (D, e) of this head
-            __syncthreads();
+            if (!sm103::mbar_wait(&bar[1], par, kCopyWaitNs)) return;  // (D, e) of this head
             const float *ev = reinterpret_cast<const float *>(bC + ((d * dv) >> 2));
             float *eg = Cm + (long long)d * dv;
             if (tid < d) eg[tid] = ev[tid] + us[tid];
@@ -229,7 +237,7 @@ step2_kernel(const T *__restrict__ q, const T *__restrict__ k, const T *__restri
                 part[tid][0] = acc.x; part[tid][1] = acc.y; part[tid][2] = acc.z; part[tid][3] = acc.w;
             }
             __syncthreads();  // (D, e) buffer read
-            if (nx < BH) load_part(bC, nx, offC); else cp_commit();
+            if (nx < BH) load_part(bC, nx, offC, 1);
             if (tid < dv) {
                 const int grp = tid >> 2, comp = tid & 3;
                 float a = 0.f;
@@ -242,8 +250,7 @@ step2_kernel(const T *__restrict__ q, const T *__restrict__ k, const T *__restri
         }
 
         // ---- pass over C: column sums k^T C, u'^T C; C' = C + q v^T; m' = m + q ----
-        if (masked) cp_wait<2>(); else cp_wait<1>();  // (C, m) of this head
-        __syncthreads();
+        if (!sm103::mbar_wait(&bar[1], par, kCopyWaitNs)) return;  // (C, m) of this head
         const float *mv = reinterpret_cast<const float *>(bC + ((d * dv) >> 2));
         if (tid < d) m[tid] = mv[tid] + qs[tid];
         const float uq = warp_dot(us, qs, d), km = warp_dot(ks, mv, d);
@@ -271,7 +278,7 @@ step2_kernel(const T *__restrict__ q, const T *__restrict__ k, const T *__restri
             part[tid][4] = acc_uC.x; part[tid][5] = acc_uC.y; part[tid][6] = acc_uC.z; part[tid][7] = acc_uC.w;
         }
         __syncthreads();  // (C, m) buffer read
-        if (nx < BH) load_part(bC, nx, offC); else cp_commit();
+        if (nx < BH) load_part(bC, nx, offC, 1);
         if (tid < dv) {
             const int grp = tid >> 2, comp = tid & 3;
             float a = 0.f, b = 0.f;
@@ -283,8 +290,7 @@ step2_kernel(const T *__restrict__ q, const T *__restrict__ k, const T *__restri
         // ---- pass over G: column sums q^T G (old G); G' = G + k (k^T C); h' = h + k (k.m) ----
         float qh = 0.f;
         if (masked) {
-            cp_wait<2>();  // (G, h) of this head
-            __syncthreads();
+            if (!sm103::mbar_wait(&bar[2], par, kCopyWaitNs)) return;  // (G, h) of this head
             const float *hv = reinterpret_cast<const float *>(bG + nC);
             if (tid < d) h[tid] = hv[tid] + ks[tid] * km;
             qh = warp_dot(qs, hv, d);
@@ -304,7 +310,7 @@ step2_kernel(const T *__restrict__ q, const T *__restrict__ k, const T *__restri
             }
             part[tid][8] = acc_qG.x; part[tid][9] = acc_qG.y; part[tid][10] = acc_qG.z; part[tid][11] = acc_qG.w;
             __syncthreads();  // part written, the (G, h) buffer read
-            if (nx < BH) load_part(bG, nx, offG); else cp_commit();
+            if (nx < BH) load_part(bG, nx, offG, 2);
             if (tid < dv) {
                 const int grp = tid >> 2, comp = tid & 3;
                 float c = 0.f;
@@ -326,7 +332,6 @@ step2_kernel(const T *__restrict__ q, const T *__restrict__ k, const T *__restri
         }
         __syncthreads();  // qs, ks, vs, us, kC, uC, qG read before the next head rewrites them
     }
-    cp_wait<0>();  // (only empty groups remain)
 }
 
 // dynamic shared memory of step2_kernel: S, (C, m), (G, h) if masked, tokens
