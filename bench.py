@@ -43,9 +43,9 @@ TRAFFIC = {
                           "n": 16384, "bytes": 526.6e6,
                           "how": "ncu capture at n=8192 (227.1 MB read + 36.2 MB written during the launch; outputs "
                                  "still dirty in L2 at its end are written later) scaled x2 to n=16384"},
-    "step2_kernel": {"src": ["hla_step.cu"], "sha256": "5542daa4b35fe2f4", "workload": "decode_bf16", "n": 0,
-                     "bytes": 750.6e6, "how": "ncu capture of one step at B64 H32 d128 (bench.py --profile-case "
-                                              "tuple_step): 406.4 MB read + 344.2 MB written"},
+    "step2_kernel": {"src": ["hla_step.cu"], "sha256": "7f4bfb053a9af874", "workload": "decode_bf16", "n": 0,
+                     "bytes": 750.3e6, "how": "ncu capture of one step at B64 H32 d128 (bench.py --profile-case "
+                                              "tuple_step): 406.4 MB read + 343.9 MB written"},
     "c3_kernels": {"src": ["hla3_chunked.cu"], "sha256": "17ac1acd5c9202d1", "workload": "hla3_f32", "n": 4096,
                    "bytes": 432.5e6, "how": "ncu capture of one forward's five launches (bench.py --only hla3_f32): "
                                             "373.0 MB read + 59.5 MB written, 6.4 x the token I/O (per-chunk records)"},
@@ -59,9 +59,9 @@ TRAFFIC = {
                       "how": "ncu capture of one backward (bench.py --only backward): 278.0 MB read + 170.4 MB "
                              "written; the per-tile records (X hi, lo; S_p, D_p: 96 MB) are written once and read "
                              "back once"},
-    "step2_kernel_sde": {"src": ["hla_step.cu"], "sha256": "5542daa4b35fe2f4", "workload": "decode_bf16", "n": 0,
-                         "bytes": 481.3e6, "how": "ncu capture of one step at B64 H32 d128 (bench.py --profile-case "
-                                                  "sde_step): 271.2 MB read + 210.1 MB written"},
+    "step2_kernel_sde": {"src": ["hla_step.cu"], "sha256": "7f4bfb053a9af874", "workload": "decode_bf16", "n": 0,
+                         "bytes": 480.2e6, "how": "ncu capture of one step at B64 H32 d128 (bench.py --profile-case "
+                                                  "sde_step): 271.1 MB read + 209.1 MB written"},
 }
 
 
