@@ -829,7 +829,7 @@ def bench_ahla(hla, dev, stream, hbm_peak, world, steps=20, warmup=3, decode_ste
                      "tokens_per_s": w.B * world / (us * 1e-6),
                      "roofline": {"bound": "hbm", "achieved": gbs, "peak": hbm_peak, "unit": "GB/s",
                                   "frac": gbs / hbm_peak, "traffic": None, "algorithmic_bytes": ahla_dec_bytes(w),
-                                  "kernel": "ahla_step_kernel"},
+                                  "kernel": "ahla_step_staged_kernel"},
                      "launches": decode_steps}
     return res
 

@@ -22,6 +22,7 @@
 
 #include "hla_internal.h"
 #include "simt_gemm.cuh"
+#include "sm103_prims.cuh"
 
 namespace hla {
 namespace {
@@ -323,6 +324,151 @@ __global__ void __launch_bounds__(kThreads) ahla_step_kernel(const T *__restrict
     }
 }
 
+// The same step, one 512-thread block per SM working through heads (hd = blockIdx.x, + gridDim.x,
+// ...), each head's [P | m] and [E | n] staged in shared memory by one 1-D bulk copy each, issued
+// a pass or more before use: while the P pass of a head runs, its [E | n] is in flight, and each
+// buffer takes the next head's part as soon as its pass has read it.  Updated values go to global
+// memory straight from registers.  Every thread waits on the buffer's mbarrier (phase = the block's
+// head count), bounded: a copy that never lands ends the block.
+constexpr int kStepPThreads = 512;
+constexpr unsigned long long kCopyWaitNs = 2000000000ull;
+
+__device__ __forceinline__ void bulk_copy(void *dst, const void *src, uint32_t bytes, uint64_t *bar) {
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+                 ::"r"(sm103::smem_u32(dst)), "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes),
+                   "r"(sm103::smem_u32(bar))
+                 : "memory");
+}
+
+template <typename T>
+__global__ void __launch_bounds__(kStepPThreads, 1)
+ahla_step_staged_kernel(const T *__restrict__ q, const T *__restrict__ k, const T *__restrict__ v, T *__restrict__ out,
+                        float *__restrict__ state, int BH, int d, int dv, int normalized, float eps) {
+    extern __shared__ float4 dyn[];
+    __shared__ float qs[128], ks[128], vs[128], rs[128], part[kStepPThreads][4], red[kStepPThreads / 32];
+    __shared__ float s_sc;
+    __shared__ uint64_t bar[2];  // [P | m] and tokens; [E | n]
+    const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+    const long long st = 2LL * d * dv + 2 * d;
+    const int nP = (d * dv + d) >> 2;  // float4 units of [P | m], of [E | n]
+    const int nt_q = d * (int)sizeof(T) / 16, nt_v = dv * (int)sizeof(T) / 16;
+    float4 *bP = dyn, *bE = bP + nP, *bT = bE + nP;
+    const T *tq = reinterpret_cast<const T *>(bT), *tk = tq + d, *tv = tk + d;
+    // thread 0 issues the copies, after a block barrier that ends the generic reads of the buffer
+    auto load_P = [&](int hd) {
+        if (tid == 0) {
+            sm103::fence_async_smem();
+            sm103::mbar_arrive_expect_tx(&bar[0], (uint32_t)(16 * (nP + 2 * nt_q + nt_v)));
+            bulk_copy(bP, state + hd * st, 16u * nP, &bar[0]);
+            bulk_copy(bT, q + (long long)hd * d, 16u * nt_q, &bar[0]);
+            bulk_copy(bT + nt_q, k + (long long)hd * d, 16u * nt_q, &bar[0]);
+            bulk_copy(bT + 2 * nt_q, v + (long long)hd * dv, 16u * nt_v, &bar[0]);
+        }
+    };
+    auto load_E = [&](int hd) {
+        if (tid == 0) {
+            sm103::fence_async_smem();
+            sm103::mbar_arrive_expect_tx(&bar[1], 16u * nP);
+            bulk_copy(bE, state + hd * st + (long long)d * dv + d, 16u * nP, &bar[1]);
+        }
+    };
+    // block sum of one value per thread (all threads call it; ends with a block barrier)
+    auto block_sum = [&](float x) {
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+        if (lane == 0) red[wid] = x;
+        __syncthreads();
+        float t = 0.f;
+        for (int w = 0; w < kStepPThreads / 32; ++w) t += red[w];
+        __syncthreads();
+        return t;
+    };
+    int hd = blockIdx.x;
+    if (hd >= BH) return;
+    if (tid == 0) {
+        sm103::mbar_init(&bar[0], 1);
+        sm103::mbar_init(&bar[1], 1);
+        sm103::fence_mbar_init();
+    }
+    __syncthreads();
+    load_P(hd);
+    load_E(hd);
+    const int wv = dv >> 2, n4 = (d * dv) >> 2, c4 = (tid % wv) * 4;  // kStepPThreads is a multiple of wv
+    for (uint32_t par = 0; hd < BH; hd += gridDim.x, par ^= 1u) {
+        const int nx = hd + gridDim.x;  // this block's next head
+        float *P = state + hd * st, *m = P + (long long)d * dv, *E = m + d, *nn = E + (long long)d * dv;
+        if (!sm103::mbar_wait(&bar[0], par, kCopyWaitNs)) return;  // [P | m] and tokens of this head
+        if (tid < d) {
+            qs[tid] = to_f32(tq[tid]);
+            ks[tid] = to_f32(tk[tid]);
+        }
+        if (tid < dv) vs[tid] = to_f32(tv[tid]);
+        __syncthreads();
+        // ---- [P | m]: P' = P + k v^T, m' = m + k, r = q^T P', s = q . m' ----
+        {
+            float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+            float4 *P4 = reinterpret_cast<float4 *>(P);
+            const float v0 = vs[c4], v1 = vs[c4 + 1], v2 = vs[c4 + 2], v3 = vs[c4 + 3];
+            for (int f = tid; f < n4; f += kStepPThreads) {
+                const int row = f / wv;
+                float4 pv = bP[f];
+                const float kr = ks[row], qr = qs[row];
+                pv.x += kr * v0; pv.y += kr * v1; pv.z += kr * v2; pv.w += kr * v3;
+                P4[f] = pv;
+                acc.x += qr * pv.x; acc.y += qr * pv.y; acc.z += qr * pv.z; acc.w += qr * pv.w;
+            }
+            part[tid][0] = acc.x; part[tid][1] = acc.y; part[tid][2] = acc.z; part[tid][3] = acc.w;
+            float sm = 0.f;
+            if (tid < d) {
+                const float mv = reinterpret_cast<const float *>(bP + n4)[tid] + ks[tid];
+                m[tid] = mv;
+                sm = qs[tid] * mv;
+            }
+            const float s_tot = block_sum(sm);  // s = q . m' (also: part written, the [P | m] buffer read)
+            if (nx < BH) load_P(nx);
+            if (tid < dv) {
+                const int grp = tid >> 2, comp = tid & 3;
+                float a = 0.f;
+                for (int g = grp; g < kStepPThreads; g += wv) a += part[g][comp];
+                rs[tid] = a;  // r = q^T P'
+            }
+            if (tid == 0) s_sc = s_tot;
+            __syncthreads();
+        }
+        // ---- [E | n]: E' = E + k r^T, n' = n + s k, o = q^T E', den = q . n' ----
+        if (!sm103::mbar_wait(&bar[1], par, kCopyWaitNs)) return;  // [E | n] of this head
+        {
+            float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+            float4 *E4 = reinterpret_cast<float4 *>(E);
+            const float r0 = rs[c4], r1 = rs[c4 + 1], r2 = rs[c4 + 2], r3 = rs[c4 + 3];
+            for (int f = tid; f < n4; f += kStepPThreads) {
+                const int row = f / wv;
+                float4 e = bE[f];
+                const float kr = ks[row], qr = qs[row];
+                e.x += kr * r0; e.y += kr * r1; e.z += kr * r2; e.w += kr * r3;
+                E4[f] = e;
+                acc.x += qr * e.x; acc.y += qr * e.y; acc.z += qr * e.z; acc.w += qr * e.w;
+            }
+            part[tid][0] = acc.x; part[tid][1] = acc.y; part[tid][2] = acc.z; part[tid][3] = acc.w;
+            float sn = 0.f;
+            if (tid < d) {
+                const float nv = reinterpret_cast<const float *>(bE + n4)[tid] + s_sc * ks[tid];
+                nn[tid] = nv;
+                sn = qs[tid] * nv;
+            }
+            const float den = block_sum(sn);  // den = q . n' (also: part written, the [E | n] buffer read)
+            if (nx < BH) load_E(nx);
+            if (tid < dv) {
+                const int grp = tid >> 2, comp = tid & 3;
+                float a = 0.f;
+                for (int g = grp; g < kStepPThreads; g += wv) a += part[g][comp];
+                from_f32(&out[(long long)hd * dv + tid], normalized ? a / (den + eps) : a);
+            }
+            __syncthreads();  // qs, ks, vs, rs, part, s_sc read before the next head rewrites them
+        }
+    }
+}
+
 template <typename T>
 cudaError_t forward_t(const Fwd2 &p, cudaStream_t stream) {
     const ALayout L = make_layout(p.BH, p.n, p.d, p.dv, p.chunk);
@@ -368,6 +514,35 @@ cudaError_t ahla_forward_launch(const Fwd2 &p, cudaStream_t stream) {
 cudaError_t ahla_step_launch(const void *q, const void *k, const void *v, void *out, hla_dtype dt, int BH, int d,
                              int dv, int normalized, float eps, float *state, cudaStream_t stream) {
     if (BH == 0) return cudaSuccess;
+    const auto al16 = [](const void *x) { return (reinterpret_cast<uintptr_t>(x) & 15u) == 0; };
+    const size_t tsz = dt == HLA_BF16 ? 2 : 4;
+    // the staged kernel copies whole 16-byte units: token rows, [P | m], [E | n] and the head stride
+    if (al16(q) && al16(k) && al16(v) && al16(state) && (d * tsz) % 16 == 0 && (dv * tsz) % 16 == 0 && d % 4 == 0 &&
+        dv % 4 == 0 && d <= 128 && dv <= 128) {
+        int dev = 0, sms = 0;
+        cudaGetDevice(&dev);
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+        const int grid = BH < sms ? BH : sms;
+        const size_t smem = 2 * 16 * (size_t)((d * dv + d) / 4) + tsz * (2 * (size_t)d + dv);
+        cudaError_t e;
+        if (dt == HLA_BF16) {
+            if ((e = cudaFuncSetAttribute(ahla_step_staged_kernel<__nv_bfloat16>,
+                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)))
+                return e;
+            ahla_step_staged_kernel<__nv_bfloat16><<<grid, kStepPThreads, smem, stream>>>(
+                static_cast<const __nv_bfloat16 *>(q), static_cast<const __nv_bfloat16 *>(k),
+                static_cast<const __nv_bfloat16 *>(v), static_cast<__nv_bfloat16 *>(out), state, BH, d, dv, normalized,
+                eps);
+        } else {
+            if ((e = cudaFuncSetAttribute(ahla_step_staged_kernel<float>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                          (int)smem)))
+                return e;
+            ahla_step_staged_kernel<float><<<grid, kStepPThreads, smem, stream>>>(
+                static_cast<const float *>(q), static_cast<const float *>(k), static_cast<const float *>(v),
+                static_cast<float *>(out), state, BH, d, dv, normalized, eps);
+        }
+        return cudaGetLastError();
+    }
     if (dt == HLA_BF16)
         ahla_step_kernel<__nv_bfloat16><<<BH, kThreads, 0, stream>>>(
             static_cast<const __nv_bfloat16 *>(q), static_cast<const __nv_bfloat16 *>(k),
