@@ -231,100 +231,12 @@ __global__ void __launch_bounds__(kThreads) ahla_out_kernel(const T *__restrict_
 
 // ---------------------------------------------------------------------------
 // decode step: P' = P + k v^T, m' = m + k, r = q^T P', s = q . m',
-// E' = E + k r^T, n' = n + s k, o = q^T E', den = q . n'.  One block per head;
-// P and E are read and written once with 16-byte accesses, consecutive threads
-// on consecutive column groups; every thread keeps one column group of the
-// column sums q^T P' (then q^T E'), combined across row groups in shared memory.
+// E' = E + k r^T, n' = n + s k, o = q^T E', den = q . n'.  P and E are read and
+// written once with 16-byte accesses, consecutive threads on consecutive column
+// groups; every thread keeps one column group of the column sums q^T P' (then
+// q^T E'), combined across row groups in shared memory.
 // ---------------------------------------------------------------------------
-template <typename T>
-__global__ void __launch_bounds__(kThreads) ahla_step_kernel(const T *__restrict__ q, const T *__restrict__ k,
-                                                             const T *__restrict__ v, T *__restrict__ out,
-                                                             float *__restrict__ state, int d, int dv, int normalized,
-                                                             float eps) {
-    __shared__ float qs[128], ks[128], vs[128], rs[128], part[kThreads][4], red[kThreads / 32];
-    __shared__ float s_sc;
-    const int hd = blockIdx.x, tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
-    float *P = state + (long long)hd * (2LL * d * dv + 2 * d), *m = P + (long long)d * dv, *E = m + d,
-          *nn = E + (long long)d * dv;
-    if (tid < d) {
-        qs[tid] = to_f32(q[(long long)hd * d + tid]);
-        ks[tid] = to_f32(k[(long long)hd * d + tid]);
-    }
-    if (tid < dv) vs[tid] = to_f32(v[(long long)hd * dv + tid]);
-    __syncthreads();
-    const int wv = dv >> 2, n4 = (d * dv) >> 2, c4 = (tid % wv) * 4;  // kThreads is a multiple of wv
-    // block sum of one value per thread (all threads call it)
-    auto block_sum = [&](float x) {
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
-        if (lane == 0) red[wid] = x;
-        __syncthreads();
-        float t = 0.f;
-        for (int w = 0; w < kThreads / 32; ++w) t += red[w];
-        __syncthreads();
-        return t;
-    };
-    // ---- [P | m] ----
-    {
-        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-        float4 *P4 = reinterpret_cast<float4 *>(P);
-        const float v0 = vs[c4], v1 = vs[c4 + 1], v2 = vs[c4 + 2], v3 = vs[c4 + 3];
-        for (int f = tid; f < n4; f += kThreads) {
-            const int row = f / wv;
-            float4 p = P4[f];
-            const float kr = ks[row], qr = qs[row];
-            p.x += kr * v0; p.y += kr * v1; p.z += kr * v2; p.w += kr * v3;
-            P4[f] = p;
-            acc.x += qr * p.x; acc.y += qr * p.y; acc.z += qr * p.z; acc.w += qr * p.w;
-        }
-        part[tid][0] = acc.x; part[tid][1] = acc.y; part[tid][2] = acc.z; part[tid][3] = acc.w;
-        float sm = 0.f;
-        if (tid < d) {
-            const float mv = m[tid] + ks[tid];
-            m[tid] = mv;
-            sm = qs[tid] * mv;
-        }
-        const float s_tot = block_sum(sm);  // s = q . m' (also orders part[] before the reads below)
-        if (tid < dv) {
-            const int grp = tid >> 2, comp = tid & 3;
-            float a = 0.f;
-            for (int g = grp; g < kThreads; g += wv) a += part[g][comp];
-            rs[tid] = a;  // r = q^T P'
-        }
-        if (tid == 0) s_sc = s_tot;
-        __syncthreads();
-    }
-    // ---- [E | n] ----
-    {
-        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-        float4 *E4 = reinterpret_cast<float4 *>(E);
-        const float r0 = rs[c4], r1 = rs[c4 + 1], r2 = rs[c4 + 2], r3 = rs[c4 + 3];
-        for (int f = tid; f < n4; f += kThreads) {
-            const int row = f / wv;
-            float4 e = E4[f];
-            const float kr = ks[row], qr = qs[row];
-            e.x += kr * r0; e.y += kr * r1; e.z += kr * r2; e.w += kr * r3;
-            E4[f] = e;
-            acc.x += qr * e.x; acc.y += qr * e.y; acc.z += qr * e.z; acc.w += qr * e.w;
-        }
-        part[tid][0] = acc.x; part[tid][1] = acc.y; part[tid][2] = acc.z; part[tid][3] = acc.w;
-        float sn = 0.f;
-        if (tid < d) {
-            const float nv = nn[tid] + s_sc * ks[tid];
-            nn[tid] = nv;
-            sn = qs[tid] * nv;
-        }
-        const float den = block_sum(sn);  // den = q . n'
-        if (tid < dv) {
-            const int grp = tid >> 2, comp = tid & 3;
-            float a = 0.f;
-            for (int g = grp; g < kThreads; g += wv) a += part[g][comp];
-            from_f32(&out[(long long)hd * dv + tid], normalized ? a / (den + eps) : a);
-        }
-    }
-}
-
-// The same step, one 512-thread block per SM working through heads (hd = blockIdx.x, + gridDim.x,
+// One 512-thread block per SM works through heads (hd = blockIdx.x, + gridDim.x,
 // ...), each head's [P | m] and [E | n] staged in shared memory by one 1-D bulk copy each, issued
 // a pass or more before use: while the P pass of a head runs, its [E | n] is in flight, and each
 // buffer takes the next head's part as soon as its pass has read it.  Updated values go to global
@@ -514,44 +426,33 @@ cudaError_t ahla_forward_launch(const Fwd2 &p, cudaStream_t stream) {
 cudaError_t ahla_step_launch(const void *q, const void *k, const void *v, void *out, hla_dtype dt, int BH, int d,
                              int dv, int normalized, float eps, float *state, cudaStream_t stream) {
     if (BH == 0) return cudaSuccess;
-    const auto al16 = [](const void *x) { return (reinterpret_cast<uintptr_t>(x) & 15u) == 0; };
+    // the staged kernel copies whole 16-byte units (token rows, [P | m], [E | n], the head stride):
+    // the entry point checks the 16-byte alignment of q, k, v and the state, and d, dv in
+    // {16, 32, 64, 128} make every row a multiple of 16 bytes
     const size_t tsz = dt == HLA_BF16 ? 2 : 4;
-    // the staged kernel copies whole 16-byte units: token rows, [P | m], [E | n] and the head stride
-    if (al16(q) && al16(k) && al16(v) && al16(state) && (d * tsz) % 16 == 0 && (dv * tsz) % 16 == 0 && d % 4 == 0 &&
-        dv % 4 == 0 && d <= 128 && dv <= 128) {
-        int dev = 0, sms = 0;
-        cudaGetDevice(&dev);
-        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-        const int grid = BH < sms ? BH : sms;
-        const size_t smem = 2 * 16 * (size_t)((d * dv + d) / 4) + tsz * (2 * (size_t)d + dv);
-        cudaError_t e;
-        if (dt == HLA_BF16) {
-            if ((e = cudaFuncSetAttribute(ahla_step_staged_kernel<__nv_bfloat16>,
-                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)))
-                return e;
-            ahla_step_staged_kernel<__nv_bfloat16><<<grid, kStepPThreads, smem, stream>>>(
-                static_cast<const __nv_bfloat16 *>(q), static_cast<const __nv_bfloat16 *>(k),
-                static_cast<const __nv_bfloat16 *>(v), static_cast<__nv_bfloat16 *>(out), state, BH, d, dv, normalized,
-                eps);
-        } else {
-            if ((e = cudaFuncSetAttribute(ahla_step_staged_kernel<float>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                          (int)smem)))
-                return e;
-            ahla_step_staged_kernel<float><<<grid, kStepPThreads, smem, stream>>>(
-                static_cast<const float *>(q), static_cast<const float *>(k), static_cast<const float *>(v),
-                static_cast<float *>(out), state, BH, d, dv, normalized, eps);
-        }
-        return cudaGetLastError();
-    }
-    if (dt == HLA_BF16)
-        ahla_step_kernel<__nv_bfloat16><<<BH, kThreads, 0, stream>>>(
+    if ((d * tsz) % 16 != 0 || (dv * tsz) % 16 != 0 || d % 4 != 0 || dv % 4 != 0 || d > 128 || dv > 128)
+        return cudaErrorInvalidValue;
+    int dev = 0, sms = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    const int grid = BH < sms ? BH : sms;
+    const size_t smem = 2 * 16 * (size_t)((d * dv + d) / 4) + tsz * (2 * (size_t)d + dv);
+    cudaError_t e;
+    if (dt == HLA_BF16) {
+        if ((e = cudaFuncSetAttribute(ahla_step_staged_kernel<__nv_bfloat16>,
+                                      cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)))
+            return e;
+        ahla_step_staged_kernel<__nv_bfloat16><<<grid, kStepPThreads, smem, stream>>>(
             static_cast<const __nv_bfloat16 *>(q), static_cast<const __nv_bfloat16 *>(k),
-            static_cast<const __nv_bfloat16 *>(v), static_cast<__nv_bfloat16 *>(out), state, d, dv, normalized, eps);
-    else
-        ahla_step_kernel<float><<<BH, kThreads, 0, stream>>>(static_cast<const float *>(q),
-                                                             static_cast<const float *>(k),
-                                                             static_cast<const float *>(v), static_cast<float *>(out),
-                                                             state, d, dv, normalized, eps);
+            static_cast<const __nv_bfloat16 *>(v), static_cast<__nv_bfloat16 *>(out), state, BH, d, dv, normalized, eps);
+    } else {
+        if ((e = cudaFuncSetAttribute(ahla_step_staged_kernel<float>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                      (int)smem)))
+            return e;
+        ahla_step_staged_kernel<float><<<grid, kStepPThreads, smem, stream>>>(
+            static_cast<const float *>(q), static_cast<const float *>(k), static_cast<const float *>(v),
+            static_cast<float *>(out), state, BH, d, dv, normalized, eps);
+    }
     return cudaGetLastError();
 }
 
