@@ -12,6 +12,14 @@
 // The carries compose across tiles as the semidirect product of Eq. semidirect
 // does (D_AB = D_A + D_B + S_A C_B is the D-form of G_AB = G_A + G_B + S_B C_A).
 //
+// The unmasked operator o_t = q_t^T S_t C_t (the online updates after Theorem 1
+// without G, h) is  o_t = sum_{j<=t} (x_t . q_j) v_j + x_t^T C_p: the same X, then
+//   T = L . (X Q^T),  O = T V + X C_p,  den_t = sum_{j<=t} T_tj + x_t . m_p
+//   C_p += Q^T V,  m_p += Q^T 1
+// in the same slots and TMEM regions (C and m where D and e sit).  It runs one
+// segment per head (the fix-up of later segments would need X, which is not kept)
+// and no state.
+//
 // Parallel structure: a work item is (head, segment of L consecutive tiles);
 // items are handed out by an atomic ticket in segment-major order, so the
 // segments of one head run on different SMs at staggered times.  Each item
@@ -132,6 +140,7 @@ struct Params {
     unsigned long long wait_ns;  // budget of a cross-SM chain wait
     int inject_skip_item;        // testing: this item does not publish its S prefix
     int out_blocks;              // 64-column blocks of an output row (dv / 64)
+    int unmasked;                // the unmasked operator (one segment per head, no state)
 };
 
 constexpr int kRingFloats = kD * kD + kD * kD + kD;
@@ -544,17 +553,28 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                     if (j + 1 < nt) load_tile(kK, &tm_k, head, (t0 + j + 1) * kTile, pol_first);
                     if (!bar_wait(ms, bEpX, tp, p)) break;  // X_hi, X_lo in SX, W; D_p read out of TMEM
                     tc_fence_after();
-                    mma128<false, false, 128, kFS>(tb + kTA, lk(qs), lk(kSX), 0u);      // T = Q X_hi^T
-                    mma128<false, false, 128, kFS>(tb + kTA, lk(qs), lk(kW), 1u);       // += Q X_lo^T
+                    if (!p.unmasked) {
+                        mma128<false, false, 128, kFS>(tb + kTA, lk(qs), lk(kSX), 0u);  // T = Q X_hi^T
+                        mma128<false, false, 128, kFS>(tb + kTA, lk(qs), lk(kW), 1u);   // += Q X_lo^T
+                    } else {
+                        mma128<false, false, 128, kFS>(tb + kTA, lk(kSX), lk(qs), 0u);  // T = X_hi Q^T
+                        mma128<false, false, 128, kFS>(tb + kTA, lk(kW), lk(qs), 1u);   // += X_lo Q^T
+                    }
                     umma_commit(&ms->bar[bEvT]);
                     if (!wait_ld(kV)) break;
                     tc_fence_after();
-                    mma128<true, true, kF>(tb + kTD, lm(kSX), lm(kV), 1u);        // D += X_hi^T V
-                    if (d_lo) mma128<true, true, kF>(tb + kTD, lm(kW), lm(kV), 1u);  // D += X_lo^T V
-                    umma_commit(&ms->bar[bEvD]);
-                    // O = Q D_p (D_p in SD since the X hand-off; TMEM X was read out then) runs while
-                    // the epilogue forms T
-                    mma128<false, true, kF, kFS>(tb + kTX, lk(qs), lm(kSD), 0u);
+                    if (!p.unmasked) {
+                        mma128<true, true, kF>(tb + kTD, lm(kSX), lm(kV), 1u);        // D += X_hi^T V
+                        if (d_lo) mma128<true, true, kF>(tb + kTD, lm(kW), lm(kV), 1u);  // D += X_lo^T V
+                        umma_commit(&ms->bar[bEvD]);
+                        // O = Q D_p (D_p in SD since the X hand-off; TMEM X was read out then) runs
+                        // while the epilogue forms T
+                        mma128<false, true, kF, kFS>(tb + kTX, lk(qs), lm(kSD), 0u);
+                    } else {
+                        mma128<true, true, kF>(tb + kTD, lm(qs), lm(kV), 1u);  // C += Q^T V
+                        mma128<false, true, kF, kFS>(tb + kTX, lk(kSX), lm(kSD), 0u);  // O = X_hi C_p
+                        umma_commit(&ms->bar[bEvD]);  // X (slot SX) read: the S split may overwrite it
+                    }
                     if (!bar_wait(ms, bEpT, tp, p)) break;  // T (bf16) in TMEM A
                     tc_fence_after();
                     mma128_ts<true, kF>(tb + kTX, tb + kTA, lm(kV), 1u);          // O += T V (T in TMEM)
@@ -774,7 +794,7 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                     for (int jj = 0; jj < 32; jj += 8) store_row8(slot(kSD), r, c0 + jj, f + jj);
                 }
                 float den_part = 0.f;
-                if (p.normalized && fcol) {
+                if (p.normalized && fcol && !p.unmasked) {
 #pragma unroll
                     for (int jj = 0; jj < 32; jj += 8) {
                         float q8[8];
@@ -805,8 +825,27 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 fence_async_smem();  // X_hi, X_lo and D_p (above) visible to the MMAs
                 epi_arrive(ms, bEpX);
 
-                // while T = Q X^T runs: column sums of X (e carry)
-                if (need_e) ecol = warp_colsum32(x);  // column c0 + lane over this warp's rows
+                // while T runs: column sums of X (e carry); unmasked: x_t . m_p (the carried part of the
+                // denominator) and column sums of Q (m carry)
+                if (need_e) {
+                    if (!p.unmasked) {
+                        ecol = warp_colsum32(x);  // column c0 + lane over this warp's rows
+                    } else {
+                        float qv[32];
+#pragma unroll
+                        for (int jj = 0; jj < 32; jj += 8) {
+                            float q8[8];
+                            tile_row8(qt, r, c0 + jj, q8);
+#pragma unroll
+                            for (int u = 0; u < 8; ++u) qv[jj + u] = fcol ? q8[u] : 0.f;
+                        }
+                        if (p.normalized && fcol) {
+#pragma unroll
+                            for (int jj = 0; jj < 32; ++jj) den_part += x[jj] * ms->eloc[c0 + jj];
+                        }
+                        ecol = warp_colsum32(qv);
+                    }
+                }
 
                 // T = L . (Q X^T) -> bf16 in TMEM; row sums
                 bar_wait(ms, bEvT, tp, p);
@@ -1334,7 +1373,8 @@ size_t fused2_workspace_bytes(int BH, int n, int d, int dv, int chunk, hla_dtype
 
 bool fused2_applicable(const Fwd2 &p) {
     if (getenv("HLA_DISABLE_FUSED")) return false;
-    if (p.dt != HLA_BF16 || !fused_dim(p.d) || !fused_dim(p.dv) || !p.masked) return false;
+    if (p.dt != HLA_BF16 || !fused_dim(p.d) || !fused_dim(p.dv)) return false;
+    if (!p.masked && (p.state_in || p.state_out)) return false;  // unmasked: no state
     if (p.n <= 0 || p.BH <= 0) return false;
     if (p.state_in && (p.d != kD || p.dv != kD)) return false;  // initial states in the 128 x 128 layout only
     const FusedLayout FL = fused_layout(p.BH, p.n);
@@ -1359,7 +1399,8 @@ cudaError_t fused2_forward(const Fwd2 &p, cudaStream_t stream) {
     kp.BH = p.BH;
     kp.n = p.n;
     kp.M = (p.n + kTile - 1) / kTile;
-    kp.L = segment_tiles(p.BH, kp.M, sms);
+    kp.unmasked = p.masked ? 0 : 1;
+    kp.L = kp.unmasked ? kp.M : segment_tiles(p.BH, kp.M, sms);  // unmasked: one segment per head
     kp.G = (kp.M + kp.L - 1) / kp.L;
     kp.n_items = kp.G * p.BH;
     kp.normalized = p.normalized;

@@ -22,11 +22,11 @@ def hla():
     return binding
 
 
-def run(hla, q, k, v, normalized, state_in=None, chunk=128):
+def run(hla, q, k, v, normalized, state_in=None, chunk=128, masked=True):
     tq, tk, tv = (hla_inputs.as_torch(x, "bf16", DEV) for x in (q, k, v))
     sin = None if state_in is None else torch.from_numpy(np.ascontiguousarray(state_in, np.float32)).to(DEV)
     ws = hla.alloc_workspace(hla.hla2_workspace_bytes(*q.shape, v.shape[-1], chunk, torch.bfloat16), DEV)
-    out = hla.hla2_forward(tq, tk, tv, masked=True, normalized=normalized, eps=hla_inputs.EPS, chunk=chunk,
+    out = hla.hla2_forward(tq, tk, tv, masked=masked, normalized=normalized, eps=hla_inputs.EPS, chunk=chunk,
                            state_in=sin, workspace=ws)
     torch.cuda.synchronize()
     assert hla.hla_poll_error(ws) == 0
@@ -55,7 +55,10 @@ def test_fused_path_selected(hla):
     assert hla.hla2_forward_path(2, 16, 16384, 128, 128, normalized=True) == (1, 1)
     assert hla.hla2_forward_path(2, 16, 16384, 128, 128, normalized=True, has_state_out=True) == (1, 3)
     assert hla.hla2_forward_path(2, 16, 16384, 128, 128, has_state_in=True, has_state_out=True) == (1, 4)
-    assert hla.hla2_forward_path(2, 16, 16384, 128, 128, masked=False)[0] == 0
+    # unmasked: one segment per head, no state
+    assert hla.hla2_forward_path(2, 16, 16384, 128, 128, masked=False) == (1, 1)
+    assert hla.hla2_forward_path(2, 16, 16384, 128, 128, masked=False, has_state_out=True)[0] == 0
+    assert hla.hla2_forward_path(2, 16, 16384, 128, 128, masked=False, has_state_in=True)[0] == 0
     # d, dv of 64 as zero-padded 128, any chunk; an initial state only in the 128 x 128 layout
     assert hla.hla2_forward_path(8, 16, 2048, 64, 64, chunk=64) == (1, 1)
     assert hla.hla2_forward_path(1, 1, 100, 64, 128, chunk=7)[0] == 1
@@ -208,3 +211,22 @@ def test_fused_state_in_out(hla, monkeypatch, alias):
     for name in ("S", "C", "m", "G", "h"):
         scale = max(np.abs(parts_r[name]).max(), np.abs(parts_r["S"]).max() * np.abs(parts_r["C"]).max())
         assert np.abs(parts_g[name] - parts_r[name]).max() <= 2e-5 * max(scale, 1.0), name
+
+
+@pytest.mark.parametrize("d,dv", [(64, 64), (128, 128), (64, 128), (128, 64)])
+@pytest.mark.parametrize("B,H,n", [(1, 1, 1), (1, 2, 129), (2, 3, 600), (1, 1, 1000)])
+@pytest.mark.parametrize("normalized", [False, True])
+def test_fused_unmasked(hla, d, dv, B, H, n, normalized):
+    """The unmasked operator (online updates after Theorem 1 without G, h) on the fused kernel:
+    T = L . (X Q^T), O = T V + X C_p, den = rowsum(T) + x . m_p, one segment per head."""
+    assert hla.hla2_forward_path(B, H, n, d, dv, masked=False, normalized=normalized, chunk=128) == (1, 1)
+    q, k, v = hla_inputs.make_qkv(B, H, n, d, dv, seed=7700 + n + d + 3 * dv, dtype="bf16")
+    flat = lambda x: x.reshape(B * H, n, -1)
+    num_ref, den_ref = oracle.hla2_serial(flat(q), flat(k), flat(v), masked=False, normalized=False,
+                                          return_den=True, nthreads=8)
+    num = run(hla, q, k, v, False, masked=False)
+    err = rowerr(num, num_ref)
+    assert err < 2e-2, err
+    if normalized:
+        o = run(hla, q, k, v, True, masked=False)
+        check_normalized(o, num, num_ref, den_ref, hla_inputs.EPS, 2e-2)
