@@ -16,9 +16,9 @@
 // without G, h) is  o_t = sum_{j<=t} (x_t . q_j) v_j + x_t^T C_p: the same X, then
 //   T = L . (X Q^T),  O = T V + X C_p,  den_t = sum_{j<=t} T_tj + x_t . m_p
 //   C_p += Q^T V,  m_p += Q^T 1
-// in the same slots and TMEM regions (C and m where D and e sit).  It runs one
-// segment per head (the fix-up of later segments would need X, which is not kept)
-// and no state.
+// in the same slots and TMEM regions (C and m where D and e sit): the kUnmasked
+// instantiation.  It runs one segment per head (the fix-up of later segments would
+// need X, which is not kept) and no state.
 //
 // Parallel structure: a work item is (head, segment of L consecutive tiles);
 // items are handed out by an atomic ticket in segment-major order, so the
@@ -140,7 +140,6 @@ struct Params {
     unsigned long long wait_ns;  // budget of a cross-SM chain wait
     int inject_skip_item;        // testing: this item does not publish its S prefix
     int out_blocks;              // 64-column blocks of an output row (dv / 64)
-    int unmasked;                // the unmasked operator (one segment per head, no state)
 };
 
 constexpr int kRingFloats = kD * kD + kD * kD + kD;
@@ -389,7 +388,7 @@ __device__ __forceinline__ void mma128_ts(uint32_t d_tmem, uint32_t a_tmem, uint
 // kState: the final state is wanted.  Then W and R are split hi + lo and the e carry kept
 // whatever the output (as for the normalised output), and D += X_hi^T V + X_lo^T V is issued
 // before O (X_lo is still in slot W), so that the prefixes in the ring are accurate to fp32 level.
-template <bool kState, bool kNarrow>
+template <bool kState, bool kNarrow, bool kUnmasked = false>
 __global__ void __launch_bounds__(kThreads, 1)
 hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                   const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_o, Params p) {
@@ -553,7 +552,7 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                     if (j + 1 < nt) load_tile(kK, &tm_k, head, (t0 + j + 1) * kTile, pol_first);
                     if (!bar_wait(ms, bEpX, tp, p)) break;  // X_hi, X_lo in SX, W; D_p read out of TMEM
                     tc_fence_after();
-                    if (!p.unmasked) {
+                    if constexpr (!kUnmasked) {
                         mma128<false, false, 128, kFS>(tb + kTA, lk(qs), lk(kSX), 0u);  // T = Q X_hi^T
                         mma128<false, false, 128, kFS>(tb + kTA, lk(qs), lk(kW), 1u);   // += Q X_lo^T
                     } else {
@@ -563,7 +562,7 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                     umma_commit(&ms->bar[bEvT]);
                     if (!wait_ld(kV)) break;
                     tc_fence_after();
-                    if (!p.unmasked) {
+                    if constexpr (!kUnmasked) {
                         mma128<true, true, kF>(tb + kTD, lm(kSX), lm(kV), 1u);        // D += X_hi^T V
                         if (d_lo) mma128<true, true, kF>(tb + kTD, lm(kW), lm(kV), 1u);  // D += X_lo^T V
                         umma_commit(&ms->bar[bEvD]);
@@ -794,7 +793,7 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                     for (int jj = 0; jj < 32; jj += 8) store_row8(slot(kSD), r, c0 + jj, f + jj);
                 }
                 float den_part = 0.f;
-                if (p.normalized && fcol && !p.unmasked) {
+                if (!kUnmasked && p.normalized && fcol) {
 #pragma unroll
                     for (int jj = 0; jj < 32; jj += 8) {
                         float q8[8];
@@ -828,7 +827,7 @@ hla2_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constan
                 // while T runs: column sums of X (e carry); unmasked: x_t . m_p (the carried part of the
                 // denominator) and column sums of Q (m carry)
                 if (need_e) {
-                    if (!p.unmasked) {
+                    if constexpr (!kUnmasked) {
                         ecol = warp_colsum32(x);  // column c0 + lane over this warp's rows
                     } else {
                         float qv[32];
@@ -1399,8 +1398,7 @@ cudaError_t fused2_forward(const Fwd2 &p, cudaStream_t stream) {
     kp.BH = p.BH;
     kp.n = p.n;
     kp.M = (p.n + kTile - 1) / kTile;
-    kp.unmasked = p.masked ? 0 : 1;
-    kp.L = kp.unmasked ? kp.M : segment_tiles(p.BH, kp.M, sms);  // unmasked: one segment per head
+    kp.L = p.masked ? segment_tiles(p.BH, kp.M, sms) : kp.M;  // unmasked: one segment per head
     kp.G = (kp.M + kp.L - 1) / kp.L;
     kp.n_items = kp.G * p.BH;
     kp.normalized = p.normalized;
@@ -1435,7 +1433,9 @@ cudaError_t fused2_forward(const Fwd2 &p, cudaStream_t stream) {
         return cudaGetLastError();
     };
     const bool narrow = p.d == 64 && p.dv == 64;
-    if (p.state_out)
+    if (!p.masked)  // no state (fused2_applicable)
+        e = narrow ? launch(hla2_fused_kernel<false, true, true>) : launch(hla2_fused_kernel<false, false, true>);
+    else if (p.state_out)
         e = narrow ? launch(hla2_fused_kernel<true, true>) : launch(hla2_fused_kernel<true, false>);
     else
         e = narrow ? launch(hla2_fused_kernel<false, true>) : launch(hla2_fused_kernel<false, false>);
