@@ -39,9 +39,9 @@ DEC = hla_inputs.WORKLOADS["decode_bf16"]
 # capture of the kernel sources (concatenated) whose SHA-256 starts with "sha256"
 # (summaries in profiles/); reported as null for any other source or workload.
 TRAFFIC = {
-    "hla2_fused_kernel": {"src": ["hla_fused_sm103.cu", "sm103_prims.cuh"], "sha256": "96ac4866ad9a6b85", "workload": "long_bf16_norm",
-                          "n": 16384, "bytes": 524.9e6,
-                          "how": "ncu capture at n=8192 (226.7 MB read + 35.8 MB written during the launch; outputs "
+    "hla2_fused_kernel": {"src": ["hla_fused_sm103.cu", "sm103_prims.cuh"], "sha256": "7ca8b7c6b836b2ff", "workload": "long_bf16_norm",
+                          "n": 16384, "bytes": 526.6e6,
+                          "how": "ncu capture at n=8192 (227.5 MB read + 35.8 MB written during the launch; outputs "
                                  "still dirty in L2 at its end are written later) scaled x2 to n=16384"},
     "step2_kernel": {"src": ["hla_step.cu"], "sha256": "7f4bfb053a9af874", "workload": "decode_bf16", "n": 0,
                      "bytes": 750.3e6, "how": "ncu capture of one step at B64 H32 d128 (bench.py --profile-case "

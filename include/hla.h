@@ -190,8 +190,8 @@ hla_status hla2_step_sde(const void *q, const void *k, const void *v, void *out,
  * on the current device, without launching anything:
  *   0  generic path: fp32 CUDA-core kernels (every supported shape);
  *   1  fused path: one persistent tcgen05/TMA kernel (bf16 tokens, d and dv
- *      in {64, 128}; masked: state_in only with d = dv = 128; unmasked: no
- *      states, one SM per head) on sm_103, plus two small kernels for
+ *      in {64, 128}; masked: state_in only with d = dv = 128; unmasked: the
+ *      plain output, no states, one SM per head) on sm_103, plus two small kernels for
  *      state_out (C = Q^T V and m = Q^T 1 on the tensor cores, then
  *      G = S C - D, h = S m - e from the forward's prefixes).  It works in
  *      128-token tiles whatever chunk is (chunk only changes the rounding,

@@ -147,6 +147,43 @@ def test_ahla_step(hla, d, dv, normalized):
     assert np.abs(st.cpu().numpy().reshape(B * H, -1) - rst).max() <= 2e-5 * np.abs(rst).max()
 
 
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+@pytest.mark.parametrize("normalized", [False, True])
+def test_ahla_step_more_heads_than_sms(hla, dtype, normalized):
+    """320 heads (more than the SMs): a block of the staged step works through two or three heads,
+    refilling its buffers a pass ahead; three steps after a random state, every head against the
+    oracle's single-token updates."""
+    B, H, d, dv, steps = 2, 160, 128, 64, 3
+    BH = B * H
+    L = hla.ahla_state_floats(d, dv)
+    # a state as ahla_forward leaves it: [P | m | E | n] of a 40-token prefix, from the oracle
+    w = hla_inputs.Workload("t", B, H, 0, d, dv, 64, dtype, True, normalized, 17, decode_prefix=40,
+                            decode_steps=steps)
+    (qp, kp, vp), (qs, ks, vs) = hla_inputs.make_decode(w)
+    flat = lambda x: x.reshape(BH, x.shape[-2], -1).astype(np.float64)
+    _, _, st0 = oracle.ahla_serial(flat(qp), flat(kp), flat(vp), return_den=True, return_state=True)
+    def steps_from(state0, norm):
+        st = torch.from_numpy(np.ascontiguousarray(state0.reshape(B, H, L), np.float32)).to(DEV)
+        outs = []
+        for s_ in range(steps):
+            o = hla.ahla_step(*(hla_inputs.as_torch(x[s_], dtype, DEV) for x in (qs, ks, vs)), st, normalized=norm,
+                              eps=hla_inputs.EPS)
+            outs.append(o.float().cpu().numpy().reshape(BH, dv))
+        torch.cuda.synchronize()
+        return np.stack(outs, axis=1), st.cpu().numpy().reshape(BH, -1)
+
+    got, st_got = steps_from(st0, normalized)
+    seq = lambda x: np.moveaxis(x.reshape(steps, BH, -1), 0, 1).astype(np.float64)
+    num, den, rst = oracle.ahla_serial(seq(qs), seq(ks), seq(vs), state_in=st0.astype(np.float64), return_den=True,
+                                       return_state=True)
+    if normalized:  # outputs in the token type (bf16 rounds them: its bar)
+        nums, _ = steps_from(st0, False)
+        check_normalized(got, nums, num, den, hla_inputs.EPS, TOL[dtype])
+    else:
+        assert rowerr(got, num) < TOL[dtype]
+    assert np.abs(st_got - rst).max() <= 2e-5 * np.abs(rst).max()
+
 # ----------------------------------------------------------------------------
 # the tensor-core path (bf16, d and dv in {64, 128}, plain output, no states)
 # ----------------------------------------------------------------------------

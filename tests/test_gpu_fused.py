@@ -55,8 +55,9 @@ def test_fused_path_selected(hla):
     assert hla.hla2_forward_path(2, 16, 16384, 128, 128, normalized=True) == (1, 1)
     assert hla.hla2_forward_path(2, 16, 16384, 128, 128, normalized=True, has_state_out=True) == (1, 3)
     assert hla.hla2_forward_path(2, 16, 16384, 128, 128, has_state_in=True, has_state_out=True) == (1, 4)
-    # unmasked: one segment per head, no state
+    # unmasked: plain output, one segment per head, no state
     assert hla.hla2_forward_path(2, 16, 16384, 128, 128, masked=False) == (1, 1)
+    assert hla.hla2_forward_path(2, 16, 16384, 128, 128, masked=False, normalized=True)[0] == 0
     assert hla.hla2_forward_path(2, 16, 16384, 128, 128, masked=False, has_state_out=True)[0] == 0
     assert hla.hla2_forward_path(2, 16, 16384, 128, 128, masked=False, has_state_in=True)[0] == 0
     # d, dv of 64 as zero-padded 128, any chunk; an initial state only in the 128 x 128 layout
@@ -217,9 +218,11 @@ def test_fused_state_in_out(hla, monkeypatch, alias):
 @pytest.mark.parametrize("B,H,n", [(1, 1, 1), (1, 2, 129), (2, 3, 600), (1, 1, 1000)])
 @pytest.mark.parametrize("normalized", [False, True])
 def test_fused_unmasked(hla, d, dv, B, H, n, normalized):
-    """The unmasked operator (online updates after Theorem 1 without G, h) on the fused kernel:
-    T = L . (X Q^T), O = T V + X C_p, den = rowsum(T) + x . m_p, one segment per head."""
-    assert hla.hla2_forward_path(B, H, n, d, dv, masked=False, normalized=normalized, chunk=128) == (1, 1)
+    """The unmasked operator (online updates after Theorem 1 without G, h): the plain output on the
+    fused kernel (T = L . (X Q^T), O = T V + X C_p, one segment per head), the ratio-normalised one
+    on the fp32 path."""
+    assert hla.hla2_forward_path(B, H, n, d, dv, masked=False, chunk=128) == (1, 1)
+    assert hla.hla2_forward_path(B, H, n, d, dv, masked=False, normalized=True, chunk=128)[0] == 0
     q, k, v = hla_inputs.make_qkv(B, H, n, d, dv, seed=7700 + n + d + 3 * dv, dtype="bf16")
     flat = lambda x: x.reshape(B * H, n, -1)
     num_ref, den_ref = oracle.hla2_serial(flat(q), flat(k), flat(v), masked=False, normalized=False,

@@ -104,3 +104,32 @@ def test_fused_forward(hla, n, bh, dims, monkeypatch):
     assert rowerr(num, num_ref) < TOL["bf16"], rowerr(num, num_ref)
     o = _fused(hla, q, k, v, True)
     check_normalized(o, num, num_ref, den_ref, hla_inputs.EPS, TOL["bf16"])
+
+
+@pytest.mark.parametrize("n", LENGTHS)
+@pytest.mark.parametrize("bh", HEADS, ids=lambda x: "B%dH%d" % x)
+@pytest.mark.parametrize("dims", [(64, 64), (128, 128)], ids=lambda x: "d%ddv%d" % x)
+def test_fused_forward_unmasked(hla, n, bh, dims):
+    """The unmasked operator: the plain output on the fused kernel (one segment per head), the
+    ratio-normalised one on the fp32 path."""
+    from parity import check_normalized
+    B, H = bh
+    d, dv = dims
+    assert hla.hla2_forward_path(B, H, n, d, dv, masked=False, chunk=128)[0] == 1
+    q, k, v = hla_inputs.make_qkv(B, H, n, d, dv, seed=12000 + n + 17 * H + d, dtype="bf16")
+    flat = lambda x: x.reshape(B * H, n, -1)
+    num_ref, den_ref = oracle.hla2_serial(flat(q), flat(k), flat(v), masked=False, normalized=False,
+                                          return_den=True, nthreads=8)
+
+    def fused(normalized):
+        tq, tk, tv = (hla_inputs.as_torch(x, "bf16", DEV) for x in (q, k, v))
+        ws = hla.alloc_workspace(hla.hla2_workspace_bytes(B, H, n, d, dv, 128, torch.bfloat16), DEV)
+        out = hla.hla2_forward(tq, tk, tv, masked=False, normalized=normalized, eps=hla_inputs.EPS, chunk=128,
+                               workspace=ws)
+        torch.cuda.synchronize()
+        assert hla.hla_poll_error(ws) == 0
+        return out.float().cpu().numpy().reshape(B * H, n, -1)
+
+    num = fused(False)
+    assert rowerr(num, num_ref) < TOL["bf16"], rowerr(num, num_ref)
+    check_normalized(fused(True), num, num_ref, den_ref, hla_inputs.EPS, TOL["bf16"])
