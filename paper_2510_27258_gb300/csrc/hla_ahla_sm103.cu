@@ -23,9 +23,12 @@
 // epilogue: warp w reads TMEM lanes 32 (w % 4) .. +31 (one row each) and columns
 // 32 (w / 4) .. +31.
 //
-// Scope: bf16 tokens, d and dv in {64, 128} (64 runs as a zero-padded 128: the
-// TMA box of columns 64..127 lies outside the tensor and is zero-filled), the
-// plain (unnormalised) output, no initial or final state.  Precision: W, R and
+// Scope: bf16 tokens, d and dv in {64, 128}, the plain (unnormalised) output, no
+// initial or final state.  d = dv = 64 has its own instantiation (kNarrow): the
+// products over the head size take 4 K steps and N = 64, and the epilogue reads
+// and writes 64 columns.  A mix of 64 and 128 runs as 128 with zero features
+// 64..127 (the TMA box of those columns lies outside the tensor and is
+// zero-filled).  Precision: W, R and
 // the bf16 copies of the carries are rounded to bf16 once; every product
 // accumulates in fp32.
 #include <vector>
@@ -117,12 +120,13 @@ __device__ __forceinline__ void store_row32(uint8_t *tile, int r, int c0, const 
 constexpr uint32_t kDescHi = (1024u >> 4) | (1u << 14) | (2u << 29);
 constexpr uint32_t kLboK = 1u << 16, kLboMN = (kBlockBytes >> 4) << 16;
 
-// D (+)= A B over K = 128 (8 steps of 16), A and B from shared memory (low descriptor words)
-template <bool A_MN, bool B_MN>
+// D (+)= A B over K = 16 KS (KS steps of 16), N columns, A and B from shared memory (low
+// descriptor words)
+template <bool A_MN, bool B_MN, int N = 128, int KS = 8>
 __device__ __forceinline__ void mma_ss(uint32_t d_tmem, uint32_t a_lo, uint32_t b_lo, uint32_t accumulate) {
-    constexpr uint32_t id = idesc_bf16(128, 128, A_MN, B_MN);
+    constexpr uint32_t id = idesc_bf16(128, N, A_MN, B_MN);
 #pragma unroll
-    for (int kk = 0; kk < 8; ++kk) {
+    for (int kk = 0; kk < KS; ++kk) {
         const uint32_t ka = A_MN ? kk * 128u : (kk >> 2) * (kBlockBytes >> 4) + (kk & 3) * 2u;
         const uint32_t kb = B_MN ? kk * 128u : (kk >> 2) * (kBlockBytes >> 4) + (kk & 3) * 2u;
         umma_bf16(d_tmem, (static_cast<uint64_t>(kDescHi) << 32) | (a_lo + ka),
@@ -131,15 +135,18 @@ __device__ __forceinline__ void mma_ss(uint32_t d_tmem, uint32_t a_lo, uint32_t 
 }
 
 // D (+)= A B with A (128 x 128 bf16) in TMEM: K elements 32g .. 32g + 31 of a row packed in
-// columns a_tmem + 32g .. +15, so K step kk starts at column 32 (kk / 2) + 8 (kk % 2); B MN-major
+// columns a_tmem + 32g .. +15, so K step kk starts at column 32 (kk / 2) + 8 (kk % 2); B MN-major,
+// N columns
+template <int N = 128>
 __device__ __forceinline__ void mma_ts(uint32_t d_tmem, uint32_t a_tmem, uint32_t b_lo, uint32_t accumulate) {
-    constexpr uint32_t id = idesc_bf16(128, 128, 0, 1);
+    constexpr uint32_t id = idesc_bf16(128, N, 0, 1);
 #pragma unroll
     for (int kk = 0; kk < 8; ++kk)
         umma_bf16_ts(d_tmem, a_tmem + 32u * (kk >> 1) + 8u * (kk & 1),
                      (static_cast<uint64_t>(kDescHi) << 32) | (b_lo + kk * 128u), id, kk > 0 ? 1u : accumulate);
 }
 
+template <bool kNarrow>
 __global__ void __launch_bounds__(kThreads, 1)
 ahla_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_o, Params p) {
@@ -170,6 +177,7 @@ ahla_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
     tc_fence_after();
     const uint32_t tb = ms->tmem_base;
     uint32_t n_tiles = 0;  // tiles swept by this CTA (barrier parities)
+    constexpr int kF = kNarrow ? 64 : 128, kFS = kF / 16;  // head size: N of the products, K steps over it
 
     if (issuer) {
         if (lane == 0) {
@@ -195,7 +203,7 @@ ahla_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
                 load_tile(kV, &tm_v, head, 0);
                 if (!wait_ld(kQ0) || !wait_ld(kK0)) break;
                 tc_fence_after();
-                mma_ss<false, false>(tb + kTA, lk(kQ0), lk(kK0), 0u);  // A = Q K^T
+                mma_ss<false, false, 128, kFS>(tb + kTA, lk(kQ0), lk(kK0), 0u);  // A = Q K^T
                 umma_commit(&ms->bar[bEvA]);
                 for (int j = 0; j < p.M; ++j) {
                     const uint32_t tp = n_tiles & 1;
@@ -211,24 +219,24 @@ ahla_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
                     }
                     if (!bar_wait(ms, bEpW, tp, p) || !wait_ld(kV)) break;  // W and P_p (bf16) ready
                     tc_fence_after();
-                    mma_ts(tb + kTR, tb + kTA, lm(kV), 0u);              // R = W V
-                    mma_ss<false, true>(tb + kTR, lk(qs), lm(kC), 1u);   //   + Q P_p
+                    mma_ts<kF>(tb + kTR, tb + kTA, lm(kV), 0u);                // R = W V
+                    mma_ss<false, true, kF, kFS>(tb + kTR, lk(qs), lm(kC), 1u);  //   + Q P_p
                     umma_commit(&ms->bar[bEvR]);
-                    mma_ss<true, true>(tb + kTP, lm(ks), lm(kV), 1u);    // P += K^T V (under the R epilogue)
+                    mma_ss<true, true, kF>(tb + kTP, lm(ks), lm(kV), 1u);  // P += K^T V (under the R epilogue)
                     umma_commit(&ms->bar[bEvV]);
                     if (!bar_wait(ms, bEvV, tp, p)) break;                // V read
                     if (more) load_tile(kV, &tm_v, head, (j + 1) * kTile);
                     if (!bar_wait(ms, bEpR, tp, p)) break;                // R and E_p (bf16) ready
                     tc_fence_after();
-                    mma_ts(tb + kTR, tb + kTA, lm(kR), 0u);              // O = W R
-                    mma_ss<false, true>(tb + kTR, lk(qs), lm(kC), 1u);   //   + Q E_p
+                    mma_ts<kF>(tb + kTR, tb + kTA, lm(kR), 0u);                // O = W R
+                    mma_ss<false, true, kF, kFS>(tb + kTR, lk(qs), lm(kC), 1u);  //   + Q E_p
                     umma_commit(&ms->bar[bEvO]);
-                    mma_ss<true, true>(tb + kTE, lm(ks), lm(kR), 1u);    // E += K^T R (under the O epilogue)
+                    mma_ss<true, true, kF>(tb + kTE, lm(ks), lm(kR), 1u);  // E += K^T R (under the O epilogue)
                     umma_commit(&ms->bar[bEvE]);
                     if (more) {  // the next A runs behind them (the products execute in issue order)
                         if (!wait_ld(qo) || !wait_ld(ko)) break;
                         tc_fence_after();
-                        mma_ss<false, false>(tb + kTA, lk(qo), lk(ko), 0u);  // next A = Q K^T
+                        mma_ss<false, false, 128, kFS>(tb + kTA, lk(qo), lk(ko), 0u);  // next A = Q K^T
                         umma_commit(&ms->bar[bEvA]);
                     } else if (!bar_wait(ms, bEvE, tp, p)) {  // every product of the head is done
                         break;
@@ -252,6 +260,9 @@ ahla_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
         const int r = 32 * qd + lane, c0 = 32 * cq;
         const uint32_t lane_base = (uint32_t)(32 * qd) << 16;
         const bool blk_zero = cq > qd;  // this 32-column block of W lies above the diagonal
+        // head size 64: the 64-column results (R, O) live in column quarters 0, 1 and the 64 x 64
+        // carries P, E also in lane quadrants 0, 1; the other warps skip them
+        const bool fcol = !kNarrow || cq < 2, frow = !kNarrow || qd < 2;
         for (int head = blockIdx.x; head < p.BH; head += gridDim.x) {
             if (n_tiles > 0) {  // the previous head's last E += K^T R is done before E is reset
                 bar_wait(ms, bEvE, (n_tiles - 1) & 1u, p);
@@ -295,7 +306,7 @@ ahla_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
                 }
                 if (et == 0) tma_store_wait_read();  // the previous output has left slot C
                 epi_sync();
-                {
+                if (fcol && frow) {
                     uint32_t a[32];
                     tmem_ld32(tb + lane_base + kTP + c0, a);
                     tmem_ld_wait();
@@ -307,21 +318,23 @@ ahla_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__
                 // (b) R -> bf16 (slot R); E_p -> bf16 (slot C, P_p read by now)
                 bar_wait(ms, bEvR, tp, p);
                 tc_fence_after();
-                {
+                if (fcol) {
                     uint32_t a[32];
                     tmem_ld32(tb + lane_base + kTR + c0, a);
                     tmem_ld_wait();
                     store_row32(slot(kR), r, c0, a);  // row = token
-                    tmem_ld32(tb + lane_base + kTE + c0, a);
-                    tmem_ld_wait();
-                    store_row32(slot(kC), r, c0, a);  // row = feature
+                    if (frow) {
+                        tmem_ld32(tb + lane_base + kTE + c0, a);
+                        tmem_ld_wait();
+                        store_row32(slot(kC), r, c0, a);  // row = feature
+                    }
                 }
                 fence_async_smem();
                 epi_arrive(ms, bEpR);
                 // (c) O -> bf16 (slot C, E_p read by now) -> TMA store
                 bar_wait(ms, bEvO, tp, p);
                 tc_fence_after();
-                {
+                if (fcol) {
                     uint32_t a[32];
                     tmem_ld32(tb + lane_base + kTR + c0, a);
                     tmem_ld_wait();
@@ -406,12 +419,14 @@ cudaError_t ahla_tc_forward(const Fwd2 &p, cudaStream_t stream) {
     kp.M = (p.n + kTile - 1) / kTile;
     kp.out_blocks = p.dv / 64;
     kp.err = reinterpret_cast<WsHeader *>(p.ws);
-    cudaError_t e = cudaFuncSetAttribute(ahla_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)kSmemBytes);
-    if (e) return e;
     const int grid = p.BH < sms ? p.BH : sms;
-    ahla_tc_kernel<<<grid, kThreads, kSmemBytes, stream>>>(mq, mk, mv, mo, kp);
-    return cudaGetLastError();
+    auto launch = [&](auto kern) -> cudaError_t {
+        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
+        if (e) return e;
+        kern<<<grid, kThreads, kSmemBytes, stream>>>(mq, mk, mv, mo, kp);
+        return cudaGetLastError();
+    };
+    return (p.d == 64 && p.dv == 64) ? launch(ahla_tc_kernel<true>) : launch(ahla_tc_kernel<false>);
 }
 
 }  // namespace hla
